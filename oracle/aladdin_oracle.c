@@ -1,0 +1,726 @@
+/*
+ * Aladdin scheduler oracle: a plain, slow CPU restatement of the scheduling
+ * rules of "Aladdin: Joint Placement and Scaling for SLO-Aware LLM Serving"
+ * (arxiv 2405.06856), in fp64, stepping every worker's future one decode
+ * iteration at a time.
+ *
+ * TEST INFRASTRUCTURE ONLY. Only the tests, __graft_entry__.smoke() and the
+ * CPU-baseline leg of bench.py may load or call this library. It shares no
+ * code, header, table or constant with the CUDA library, and the product
+ * path never reaches it.
+ *
+ * Models (Sec. 3), with the readings of the paper listed in the design doc:
+ *   KV usage      Eq. kv cache: a request with c context tokens holds h*c + j
+ *                 KV slots. In its s-th remaining decode iteration a request
+ *                 with l_in input and l_out generated tokens holds
+ *                 l_in + l_out + s tokens (footprint vector w of constraint (e),
+ *                 Sec. 4.2), and nothing after its last iteration.
+ *   Prefill       Eq. prefill iter time: t_pre = k1 * sum(l_in) + c1.
+ *   Decode        Eq. iter time: t_d = (k2 * l_ave + c2) * b + c3
+ *                 = k2 * (context tokens of the batch) + c2 * b + c3, used for
+ *                 every batch size b >= 1.
+ *   Worker scale  every latency coefficient of worker i is multiplied by
+ *                 scale[i] (1/sqrt(GPUs) in the mixed-config workload).
+ *
+ * Placement test of a candidate c (prompt l_in = a_c, predicted output r_c,
+ * waiting w_c ms) on worker i (Sec. 4.2, constraints (c), (d), (e); the exact
+ * per-request decode projection replaces the approximate constraint (b)):
+ *   tau      = t_pre(P_i + a_c): the prefill of every request placed on i in
+ *              this round (P_i input tokens) plus the candidate; it stalls the
+ *              requests that were decoding at round start.
+ *   KV       for every future iteration s: KV(s) <= M_i            (e)
+ *   TTFT     w + off_i + tau <= T_pre for the candidate and for every request
+ *              already placed on i in this round                  (c)
+ *   ongoing  tau + D_j <= theta * T_dec * r_j + bank_j              (d)
+ *   new      D_q <= theta * T_dec * r_q for the candidate and the requests
+ *              placed on i in this round (no stall: they decode after it)
+ *   where D_j is the projected time of request j's r_j remaining decode
+ *   iterations with the candidate added, off_i the time until worker i's next
+ *   iteration boundary, and bank_j = theta * T_dec * l_out_j - t_dec_j the
+ *   decode time request j saved so far (Table 1: t^dec_j; 0 when no history
+ *   is given).
+ *
+ * Every quantity above is affine in the candidate's prompt length l (KV
+ * tokens and tau grow by one token per unit of l; D_j by k2 for every
+ * iteration the candidate shares with j). The oracle carries each quantity
+ * as (value at l = 0, coefficient of l) while stepping, which gives for every
+ * constraint the largest admissible l. The pair's margin is the smallest of
+ * these bounds minus a_c: the number of extra prompt tokens the worker could
+ * still absorb for this candidate (negative: infeasible).
+ */
+#include <math.h>
+#include <stdint.h>
+#include <stdlib.h>
+#include <string.h>
+
+typedef struct {
+    double k1, c1;        /* prefill: ms per input token, ms */
+    double k2, c2, c3;    /* decode: ms per context token, ms per request, ms */
+    int64_t h, j;         /* KV slots per context token, per request */
+    double T_pre, T_dec;  /* TTFT SLO, per-token decode SLO (ms) */
+    double gamma, theta;  /* capacity_norm weight, SLO scaling knob */
+    int64_t K;            /* sequence limit (input + output tokens) */
+} orc_params;
+
+/* Cluster state in fixed-stride slots: worker w owns slots
+ * [w*cap, w*cap + n[w]). */
+typedef struct {
+    int32_t W, cap;
+    const int64_t* M;     /* [W] KV capacity (slots) */
+    const double* scale;  /* [W] latency coefficient multiplier */
+    double* off;          /* [W] ms from now to the worker's next iteration start */
+    double* clock;        /* [W] absolute ms at which the worker's next iteration
+                             starts (simulation only; may be NULL for scoring) */
+    int32_t* n;           /* [W] requests on the worker */
+    int32_t* in;          /* [W*cap] input length */
+    int32_t* gen;         /* [W*cap] output tokens generated so far */
+    int32_t* pred;        /* [W*cap] predicted output length */
+    double* tdec;         /* [W*cap] decode time so far (ms), or NULL */
+    uint8_t* pend;        /* [W*cap] 1: placed in the current round, prefill pending */
+    double* wait;         /* [W*cap] pending requests: wait since arrival (ms) */
+    int64_t* rid;         /* [W*cap] request id (simulation only), or NULL */
+} orc_cluster;
+
+typedef struct {
+    uint8_t flags;        /* bit0 KV, bit1 TTFT, bit2 ongoing ATGT, bit3 new ATGT */
+    double margin;        /* largest admissible prompt length minus a_c (tokens) */
+    double mscale;        /* token scale of the binding latency bound; 0 if KV binds */
+    int64_t kv_peak;      /* peak KV over all future iterations with the candidate */
+    double t_cand;        /* candidate's projected decode time, all iterations (ms) */
+    double near;          /* smallest |slack| / scale over latency constraints at a_c */
+} orc_pair;
+
+enum { ORC_OK = 0, ORC_ERR_ARG = -1, ORC_ERR_CAPACITY = -2, ORC_ERR_MEM = -3 };
+
+/* ---------------------------------------------------------------------- */
+/* A worker's own future, stepped one decode iteration at a time:
+ *   b[s] = number of its requests still decoding in iteration s,
+ *   Kt[s] = context tokens they hold in iteration s,   s = 1..S.         */
+typedef struct {
+    int32_t S;
+    int64_t* b;
+    int64_t* Kt;
+} orc_future;
+
+static int32_t remaining(const orc_cluster* cl, int64_t slot)
+{
+    return cl->pred[slot] - (cl->pend[slot] ? 0 : cl->gen[slot]);
+}
+
+static int64_t context(const orc_cluster* cl, int64_t slot)
+{
+    return (int64_t)cl->in[slot] + (cl->pend[slot] ? 0 : cl->gen[slot]);
+}
+
+static int future_build(const orc_cluster* cl, int w, orc_future* f)
+{
+    int64_t base = (int64_t)w * cl->cap;
+    int32_t S = 0;
+    for (int q = 0; q < cl->n[w]; ++q) {
+        int32_t r = remaining(cl, base + q);
+        if (r > S) S = r;
+    }
+    f->S = S;
+    f->b = (int64_t*)calloc((size_t)S + 2, sizeof(int64_t));
+    f->Kt = (int64_t*)calloc((size_t)S + 2, sizeof(int64_t));
+    if (!f->b || !f->Kt) return ORC_ERR_MEM;
+    for (int32_t s = 1; s <= S; ++s) {
+        int64_t b = 0, K = 0;
+        for (int q = 0; q < cl->n[w]; ++q) {
+            int64_t slot = base + q;
+            if (remaining(cl, slot) >= s) {
+                b += 1;
+                K += context(cl, slot) + s;
+            }
+        }
+        f->b[s] = b;
+        f->Kt[s] = K;
+    }
+    return ORC_OK;
+}
+
+static void future_free(orc_future* f)
+{
+    free(f->b);
+    free(f->Kt);
+    f->b = f->Kt = NULL;
+    f->S = 0;
+}
+
+static int64_t floor_div(int64_t x, int64_t d) /* d > 0 */
+{
+    int64_t q = x / d;
+    if ((x % d != 0) && (x < 0)) q -= 1;
+    return q;
+}
+
+/* Running minimum of the constraint bounds. */
+typedef struct {
+    double bound, bscale, near;
+    int ok[4];
+} orc_acc;
+
+/* A latency constraint slack(l) = slack0 - slope * l >= 0; scale_a is the sum
+ * of the magnitudes of its terms at l = a (the size rounding acts on). */
+static void lat_constraint(orc_acc* A, int group, double slack0, double slope,
+                           double scale_a, double a)
+{
+    double slack_a = slack0 - slope * a;
+    if (!(slack_a >= 0.0)) A->ok[group] = 0;
+    double b;
+    if (slope > 0.0) b = slack0 / slope;
+    else b = slack0 >= 0.0 ? INFINITY : -INFINITY;
+    if (b < A->bound) {
+        A->bound = b;
+        A->bscale = slope > 0.0 ? scale_a / slope : 0.0;
+    }
+    double rel = fabs(slack_a) / (scale_a > 0.0 ? scale_a : 1.0);
+    if (rel < A->near) A->near = rel;
+}
+
+/* Evaluate candidate (a_c, r_c, w_c) on worker w. T0, T1 are scratch arrays of
+ * at least max(S, r_c) + 1 doubles. */
+static void eval_pair(const orc_params* p, const orc_cluster* cl, int w, const orc_future* f,
+                      double* T0, double* T1, int32_t a_c, int32_t r_c, double w_c, orc_pair* out)
+{
+    const double sc = cl->scale[w];
+    const int64_t M = cl->M[w];
+    const int64_t base = (int64_t)w * cl->cap;
+    const int32_t S = f->S > r_c ? f->S : r_c;
+
+    /* Step every future iteration with the candidate added. The candidate holds
+     * l + s tokens in its s-th iteration (it has generated nothing yet). */
+    int64_t kv_hi0 = INT64_MIN; /* max KV at l = 0 over iterations shared with the candidate */
+    int64_t kv_lo = 0;          /* max KV over iterations after the candidate finished */
+    int64_t kv_peak = 0;
+    T0[0] = 0.0;
+    T1[0] = 0.0;
+    for (int32_t s = 1; s <= S; ++s) {
+        int64_t bw = s <= f->S ? f->b[s] : 0;
+        int64_t Kw = s <= f->S ? f->Kt[s] : 0;
+        int with_c = s <= r_c;
+        int64_t b = bw + (with_c ? 1 : 0);
+        int64_t K0 = Kw + (with_c ? s : 0); /* context tokens at l = 0 */
+        int64_t kv0 = p->h * K0 + p->j * b;
+        int64_t kv_a = kv0 + (with_c ? p->h * (int64_t)a_c : 0);
+        if (kv_a > kv_peak) kv_peak = kv_a;
+        if (with_c) {
+            if (kv0 > kv_hi0) kv_hi0 = kv0;
+        } else if (kv0 > kv_lo) {
+            kv_lo = kv0;
+        }
+        double t0 = sc * (p->c3 + p->c2 * (double)b + p->k2 * (double)K0);
+        double t1 = with_c ? sc * p->k2 : 0.0;
+        T0[s] = T0[s - 1] + t0;
+        T1[s] = T1[s - 1] + t1;
+    }
+
+    orc_acc A;
+    A.bound = INFINITY;
+    A.bscale = 0.0;
+    A.near = INFINITY;
+    for (int g = 0; g < 4; ++g) A.ok[g] = 1;
+    const double a = (double)a_c;
+
+    /* (e) KV capacity. */
+    double bkv;
+    if (kv_lo > M) {
+        bkv = -INFINITY;
+        A.ok[0] = 0;
+    } else {
+        bkv = (double)floor_div(M - kv_hi0, p->h);
+        if (kv_hi0 + p->h * (int64_t)a_c > M) A.ok[0] = 0;
+    }
+
+    /* Prefill of this round's placements plus the candidate (Eq. prefill). */
+    double P = 0.0;
+    for (int q = 0; q < cl->n[w]; ++q)
+        if (cl->pend[base + q]) P += (double)cl->in[base + q];
+    const double tau0 = sc * (p->k1 * P + p->c1);
+    const double tau1 = sc * p->k1;
+    const double tau_a = tau0 + tau1 * a;
+    const double off = cl->off ? cl->off[w] : 0.0;
+
+    /* (c) TTFT of the candidate and of this round's earlier placements. */
+    lat_constraint(&A, 1, p->T_pre - w_c - off - tau0, tau1, p->T_pre + w_c + off + tau_a, a);
+    for (int q = 0; q < cl->n[w]; ++q) {
+        int64_t slot = base + q;
+        if (!cl->pend[slot]) continue;
+        double wq = cl->wait[slot];
+        lat_constraint(&A, 1, p->T_pre - wq - off - tau0, tau1, p->T_pre + wq + off + tau_a, a);
+    }
+
+    /* (d) ongoing requests: stall plus remaining decode within their budget. */
+    for (int q = 0; q < cl->n[w]; ++q) {
+        int64_t slot = base + q;
+        int32_t r = remaining(cl, slot);
+        double D0 = T0[r], D1 = T1[r];
+        if (cl->pend[slot]) {
+            double budget = p->theta * p->T_dec * (double)r;
+            lat_constraint(&A, 3, budget - D0, D1, budget + D0 + D1 * a, a);
+        } else {
+            double bank = 0.0;
+            if (cl->tdec) bank = p->theta * p->T_dec * (double)cl->gen[slot] - cl->tdec[slot];
+            double budget = p->theta * p->T_dec * (double)r + bank;
+            lat_constraint(&A, 2, budget - tau0 - D0, tau1 + D1,
+                           p->theta * p->T_dec * (double)r + fabs(bank) + tau_a + D0 + D1 * a, a);
+        }
+    }
+    /* The candidate's own decode. */
+    {
+        double budget = p->theta * p->T_dec * (double)r_c;
+        double D0 = T0[r_c], D1 = T1[r_c];
+        lat_constraint(&A, 3, budget - D0, D1, budget + D0 + D1 * a, a);
+        out->t_cand = D0 + D1 * a;
+    }
+
+    double bound = A.bound, bscale = A.bscale;
+    if (bkv <= bound) {
+        bound = bkv;
+        bscale = 0.0;
+    }
+    out->flags = (uint8_t)((A.ok[0] ? 1 : 0) | (A.ok[1] ? 2 : 0) | (A.ok[2] ? 4 : 0) | (A.ok[3] ? 8 : 0));
+    out->margin = bound - a;
+    out->mscale = bscale;
+    out->kv_peak = kv_peak;
+    out->near = A.near;
+}
+
+/* ---------------------------------------------------------------------- */
+/* Algorithm 1 ordering: workers sorted on capacity_norm from large to small;
+ * capacity_norm = L2 norm of (batch size B, sum over requests of
+ * l_in + gamma * l_pred) (Sec. 4.2, Scheduling heuristic). Equal norms keep
+ * index order. */
+typedef struct {
+    double norm;
+    int32_t w;
+} orc_key;
+
+static int key_cmp(const void* x, const void* y)
+{
+    const orc_key* a = (const orc_key*)x;
+    const orc_key* b = (const orc_key*)y;
+    if (a->norm > b->norm) return -1;
+    if (a->norm < b->norm) return 1;
+    return a->w < b->w ? -1 : (a->w > b->w ? 1 : 0);
+}
+
+double orc_capacity_norm(const orc_params* p, const orc_cluster* cl, int w)
+{
+    int64_t base = (int64_t)w * cl->cap;
+    double B = (double)cl->n[w];
+    double L = 0.0;
+    for (int q = 0; q < cl->n[w]; ++q)
+        L += (double)cl->in[base + q] + p->gamma * (double)cl->pred[base + q];
+    return sqrt(B * B + L * L);
+}
+
+static int capacity_order(const orc_params* p, const orc_cluster* cl, int32_t* order)
+{
+    orc_key* keys = (orc_key*)malloc(sizeof(orc_key) * (size_t)cl->W);
+    if (!keys) return ORC_ERR_MEM;
+    for (int w = 0; w < cl->W; ++w) {
+        keys[w].norm = orc_capacity_norm(p, cl, w);
+        keys[w].w = w;
+    }
+    qsort(keys, (size_t)cl->W, sizeof(orc_key), key_cmp);
+    for (int i = 0; i < cl->W; ++i) order[i] = keys[i].w;
+    free(keys);
+    return ORC_OK;
+}
+
+int orc_order(const orc_params* p, const orc_cluster* cl, int32_t* order)
+{
+    return capacity_order(p, cl, order);
+}
+
+static int32_t max_remaining(const orc_cluster* cl)
+{
+    int32_t S = 0;
+    for (int w = 0; w < cl->W; ++w)
+        for (int q = 0; q < cl->n[w]; ++q) {
+            int32_t r = remaining(cl, (int64_t)w * cl->cap + q);
+            if (r > S) S = r;
+        }
+    return S;
+}
+
+static int32_t max_of(const int32_t* x, int64_t n)
+{
+    int32_t m = 0;
+    for (int64_t i = 0; i < n; ++i)
+        if (x[i] > m) m = x[i];
+    return m;
+}
+
+static void store_pair(const orc_pair* r, int64_t k, uint8_t* flags, double* margin, double* mscale,
+                       int64_t* kvpeak, double* tcand, double* near)
+{
+    if (flags) flags[k] = r->flags;
+    if (margin) margin[k] = r->margin;
+    if (mscale) mscale[k] = r->mscale;
+    if (kvpeak) kvpeak[k] = r->kv_peak;
+    if (tcand) tcand[k] = r->t_cand;
+    if (near) near[k] = r->near;
+}
+
+/* Score every (candidate, worker) pair; outputs are row-major [c][w]; every
+ * output pointer may be NULL. argbest[c] is the first feasible worker in
+ * capacity_norm order, -1 if none. */
+int orc_score(const orc_params* p, const orc_cluster* cl, int32_t C, const int32_t* cin,
+              const int32_t* cpred, const double* cwait, uint8_t* flags, double* margin,
+              double* mscale, int64_t* kvpeak, double* tcand, double* near, int32_t* argbest)
+{
+    const int W = cl->W;
+    int32_t S = max_remaining(cl);
+    int32_t Sc = max_of(cpred, C);
+    if (Sc > S) S = Sc;
+    double* T0 = (double*)malloc(sizeof(double) * ((size_t)S + 2));
+    double* T1 = (double*)malloc(sizeof(double) * ((size_t)S + 2));
+    uint8_t* feas = (uint8_t*)calloc((size_t)C * (size_t)W, 1);
+    int32_t* order = (int32_t*)malloc(sizeof(int32_t) * (size_t)W);
+    if (!T0 || !T1 || !feas || !order) return ORC_ERR_MEM;
+    for (int w = 0; w < W; ++w) {
+        orc_future f;
+        if (future_build(cl, w, &f) != ORC_OK) return ORC_ERR_MEM;
+        for (int32_t c = 0; c < C; ++c) {
+            orc_pair r;
+            eval_pair(p, cl, w, &f, T0, T1, cin[c], cpred[c], cwait ? cwait[c] : 0.0, &r);
+            int64_t k = (int64_t)c * W + w;
+            store_pair(&r, k, flags, margin, mscale, kvpeak, tcand, near);
+            feas[k] = r.flags == 15;
+        }
+        future_free(&f);
+    }
+    if (argbest) {
+        if (capacity_order(p, cl, order) != ORC_OK) return ORC_ERR_MEM;
+        for (int32_t c = 0; c < C; ++c) {
+            argbest[c] = -1;
+            for (int i = 0; i < W; ++i)
+                if (feas[(int64_t)c * W + order[i]]) {
+                    argbest[c] = order[i];
+                    break;
+                }
+        }
+    }
+    free(T0);
+    free(T1);
+    free(feas);
+    free(order);
+    return ORC_OK;
+}
+
+/* Score a list of (candidate, worker) pairs; outputs are per pair. */
+int orc_score_pairs(const orc_params* p, const orc_cluster* cl, int64_t npairs,
+                    const int32_t* pc, const int32_t* pw, const int32_t* cin,
+                    const int32_t* cpred, const double* cwait, uint8_t* flags, double* margin,
+                    double* mscale, int64_t* kvpeak, double* tcand, double* near)
+{
+    int32_t S = max_remaining(cl);
+    for (int64_t k = 0; k < npairs; ++k)
+        if (cpred[pc[k]] > S) S = cpred[pc[k]];
+    double* T0 = (double*)malloc(sizeof(double) * ((size_t)S + 2));
+    double* T1 = (double*)malloc(sizeof(double) * ((size_t)S + 2));
+    if (!T0 || !T1) return ORC_ERR_MEM;
+    for (int64_t k = 0; k < npairs; ++k) {
+        orc_future f;
+        if (future_build(cl, pw[k], &f) != ORC_OK) return ORC_ERR_MEM;
+        orc_pair r;
+        int32_t c = pc[k];
+        eval_pair(p, cl, pw[k], &f, T0, T1, cin[c], cpred[c], cwait ? cwait[c] : 0.0, &r);
+        store_pair(&r, k, flags, margin, mscale, kvpeak, tcand, near);
+        future_free(&f);
+    }
+    free(T0);
+    free(T1);
+    return ORC_OK;
+}
+
+/* KV curve of worker w with candidate (a_c, r_c): kv[s-1] = KV(s), s = 1..S,
+ * S = max(worker's longest remaining, r_c). Returns S (or < 0 on error); kv
+ * must hold at least K entries. */
+int32_t orc_kv_curve(const orc_params* p, const orc_cluster* cl, int w, int32_t a_c, int32_t r_c,
+                     int64_t* kv)
+{
+    orc_future f;
+    if (future_build(cl, w, &f) != ORC_OK) return ORC_ERR_MEM;
+    int32_t S = f.S > r_c ? f.S : r_c;
+    for (int32_t s = 1; s <= S; ++s) {
+        int64_t b = (s <= f.S ? f.b[s] : 0) + (s <= r_c ? 1 : 0);
+        int64_t K = (s <= f.S ? f.Kt[s] : 0) + (s <= r_c ? (int64_t)a_c + s : 0);
+        kv[s - 1] = p->h * K + p->j * b;
+    }
+    future_free(&f);
+    return S;
+}
+
+/* ---------------------------------------------------------------------- */
+/* One greedy placement round (Algorithm 1), candidates in index (arrival)
+ * order: each goes to the first feasible worker in capacity_norm order of the
+ * current state and becomes a pending request there (gen = 0, prefill at the
+ * worker's next iteration). placement[c] = worker, or -1 if no worker is
+ * feasible (the cluster is fixed; nothing is opened). */
+int orc_place_round(const orc_params* p, orc_cluster* cl, int32_t C, const int32_t* cin,
+                    const int32_t* cpred, const double* cwait, const int64_t* crid,
+                    int32_t* placement)
+{
+    const int W = cl->W;
+    int32_t S = (int32_t)p->K + 2;
+    double* T0 = (double*)malloc(sizeof(double) * ((size_t)S + 2));
+    double* T1 = (double*)malloc(sizeof(double) * ((size_t)S + 2));
+    int32_t* order = (int32_t*)malloc(sizeof(int32_t) * (size_t)W);
+    orc_future* fut = (orc_future*)calloc((size_t)W, sizeof(orc_future));
+    uint8_t* have = (uint8_t*)calloc((size_t)W, 1);
+    if (!T0 || !T1 || !order || !fut || !have) return ORC_ERR_MEM;
+    int rc = ORC_OK;
+    for (int32_t c = 0; c < C && rc == ORC_OK; ++c) {
+        placement[c] = -1;
+        if (capacity_order(p, cl, order) != ORC_OK) { rc = ORC_ERR_MEM; break; }
+        for (int i = 0; i < W; ++i) {
+            int w = order[i];
+            if (!have[w]) {
+                if (future_build(cl, w, &fut[w]) != ORC_OK) { rc = ORC_ERR_MEM; break; }
+                have[w] = 1;
+            }
+            orc_pair r;
+            eval_pair(p, cl, w, &fut[w], T0, T1, cin[c], cpred[c], cwait ? cwait[c] : 0.0, &r);
+            if (r.flags != 15) continue;
+            if (cl->n[w] >= cl->cap) { rc = ORC_ERR_CAPACITY; break; }
+            int64_t slot = (int64_t)w * cl->cap + cl->n[w];
+            cl->in[slot] = cin[c];
+            cl->gen[slot] = 0;
+            cl->pred[slot] = cpred[c];
+            if (cl->tdec) cl->tdec[slot] = 0.0;
+            cl->pend[slot] = 1;
+            cl->wait[slot] = cwait ? cwait[c] : 0.0;
+            if (cl->rid) cl->rid[slot] = crid ? crid[c] : c;
+            cl->n[w] += 1;
+            future_free(&fut[w]);
+            have[w] = 0;
+            placement[c] = w;
+            break;
+        }
+    }
+    for (int w = 0; w < W; ++w)
+        if (have[w]) future_free(&fut[w]);
+    free(T0);
+    free(T1);
+    free(order);
+    free(fut);
+    free(have);
+    return rc;
+}
+
+/* ---------------------------------------------------------------------- */
+/* Execute every worker from heartbeat time t_now for dt ms (continuous
+ * batching, Sec. 2.1): at its next iteration boundary (max(clock, t_now)) a
+ * worker first runs the prefill of this round's placements (stalling its
+ * decoding requests), then decode iterations back to back while they start
+ * before t_now + dt. Finished requests leave; their realized TTFT and ATGT
+ * (decode time / decode tokens, Sec. 2.2) are appended to the record arrays
+ * (rec_* may be NULL; *nrec counts). Afterwards off[w] is the time from
+ * t_now + dt to the worker's next iteration start. */
+int orc_advance(const orc_params* p, orc_cluster* cl, double t_now, double dt,
+                int64_t* rec_rid, double* rec_val, uint8_t* rec_kind, int64_t* nrec,
+                int64_t rec_cap)
+{
+    const double t_end = t_now + dt;
+    for (int w = 0; w < cl->W; ++w) {
+        const double sc = cl->scale[w];
+        const int64_t base = (int64_t)w * cl->cap;
+        double start = cl->clock[w] > t_now ? cl->clock[w] : t_now;
+        double P = 0.0;
+        int any = 0;
+        for (int q = 0; q < cl->n[w]; ++q)
+            if (cl->pend[base + q]) { P += (double)cl->in[base + q]; any = 1; }
+        if (any) {
+            double tau = sc * (p->k1 * P + p->c1);
+            for (int q = 0; q < cl->n[w]; ++q) {
+                int64_t slot = base + q;
+                if (cl->pend[slot]) {
+                    if (rec_rid && *nrec < rec_cap) {
+                        rec_rid[*nrec] = cl->rid ? cl->rid[slot] : slot;
+                        rec_val[*nrec] = cl->wait[slot] + (start - t_now) + tau;
+                        rec_kind[*nrec] = 0;
+                    }
+                    *nrec += 1;
+                    cl->pend[slot] = 0;
+                    cl->gen[slot] = 0;
+                    cl->tdec[slot] = 0.0;
+                } else {
+                    cl->tdec[slot] += tau;
+                }
+            }
+            start += tau;
+        }
+        while (cl->n[w] > 0 && start < t_end) {
+            int64_t b = cl->n[w], K = 0;
+            for (int q = 0; q < cl->n[w]; ++q) K += context(cl, base + q) + 1;
+            double t = sc * (p->c3 + p->c2 * (double)b + p->k2 * (double)K);
+            for (int q = 0; q < cl->n[w]; ++q) {
+                cl->gen[base + q] += 1;
+                cl->tdec[base + q] += t;
+            }
+            start += t;
+            /* Retire finished requests; the last slot moves into the hole. */
+            for (int q = 0; q < cl->n[w];) {
+                int64_t slot = base + q;
+                if (cl->gen[slot] >= cl->pred[slot]) {
+                    if (rec_rid && *nrec < rec_cap) {
+                        rec_rid[*nrec] = cl->rid ? cl->rid[slot] : slot;
+                        rec_val[*nrec] = cl->tdec[slot] / (double)cl->pred[slot];
+                        rec_kind[*nrec] = 1;
+                    }
+                    *nrec += 1;
+                    int64_t last = base + cl->n[w] - 1;
+                    cl->in[slot] = cl->in[last];
+                    cl->gen[slot] = cl->gen[last];
+                    cl->pred[slot] = cl->pred[last];
+                    cl->tdec[slot] = cl->tdec[last];
+                    cl->pend[slot] = cl->pend[last];
+                    cl->wait[slot] = cl->wait[last];
+                    if (cl->rid) cl->rid[slot] = cl->rid[last];
+                    cl->n[w] -= 1;
+                } else {
+                    ++q;
+                }
+            }
+        }
+        cl->clock[w] = start;
+        cl->off[w] = start > t_end ? start - t_end : 0.0;
+    }
+    return ORC_OK;
+}
+
+/* ---------------------------------------------------------------------- */
+/* Serve a request trace with N identical workers (large-scale simulation,
+ * Sec. 6.4): heartbeats every H ms; at each, the arrivals so far that are not
+ * yet placed form one placement round in arrival order, then every worker
+ * executes until the next heartbeat. A request still unplaced whose wait at
+ * the next heartbeat plus its prefill alone would exceed T_pre can no longer
+ * meet its TTFT: it is counted as failed and dropped. If drain is set the
+ * simulation continues without arrivals until every worker is empty, so that
+ * every admitted request's realized TTFT and ATGT are recorded.
+ * out[0] failed, out[1] placed, out[2] heartbeats, out[3] max realized TTFT,
+ * out[4] max realized ATGT, out[5] realized records. */
+int orc_simulate(const orc_params* p, int32_t N, int32_t cap, int64_t M, double scale,
+                 int64_t R, const double* t_arr, const int32_t* rin, const int32_t* rpred,
+                 double H, int32_t stop_at_fail, int32_t drain, double* out)
+{
+    orc_cluster cl;
+    memset(&cl, 0, sizeof(cl));
+    cl.W = N;
+    cl.cap = cap;
+    int64_t* Mv = (int64_t*)malloc(sizeof(int64_t) * (size_t)N);
+    double* sv = (double*)malloc(sizeof(double) * (size_t)N);
+    cl.off = (double*)calloc((size_t)N, sizeof(double));
+    cl.clock = (double*)calloc((size_t)N, sizeof(double));
+    cl.n = (int32_t*)calloc((size_t)N, sizeof(int32_t));
+    size_t slots = (size_t)N * (size_t)cap;
+    cl.in = (int32_t*)calloc(slots, sizeof(int32_t));
+    cl.gen = (int32_t*)calloc(slots, sizeof(int32_t));
+    cl.pred = (int32_t*)calloc(slots, sizeof(int32_t));
+    cl.tdec = (double*)calloc(slots, sizeof(double));
+    cl.pend = (uint8_t*)calloc(slots, 1);
+    cl.wait = (double*)calloc(slots, sizeof(double));
+    cl.rid = (int64_t*)calloc(slots, sizeof(int64_t));
+    int64_t* wl = (int64_t*)malloc(sizeof(int64_t) * (size_t)(R > 0 ? R : 1));
+    int32_t* cin = (int32_t*)malloc(sizeof(int32_t) * (size_t)(R > 0 ? R : 1));
+    int32_t* cpr = (int32_t*)malloc(sizeof(int32_t) * (size_t)(R > 0 ? R : 1));
+    double* cw = (double*)malloc(sizeof(double) * (size_t)(R > 0 ? R : 1));
+    int32_t* pl = (int32_t*)malloc(sizeof(int32_t) * (size_t)(R > 0 ? R : 1));
+    int64_t rec_cap = 4 * (R > 0 ? R : 1);
+    int64_t* rr = (int64_t*)malloc(sizeof(int64_t) * (size_t)rec_cap);
+    double* rv = (double*)malloc(sizeof(double) * (size_t)rec_cap);
+    uint8_t* rk = (uint8_t*)malloc((size_t)rec_cap);
+    if (!Mv || !sv || !cl.off || !cl.clock || !cl.n || !cl.in || !cl.gen || !cl.pred || !cl.tdec ||
+        !cl.pend || !cl.wait || !cl.rid || !wl || !cin || !cpr || !cw || !pl || !rr || !rv || !rk)
+        return ORC_ERR_MEM;
+    for (int w = 0; w < N; ++w) { Mv[w] = M; sv[w] = scale; }
+    cl.M = Mv;
+    cl.scale = sv;
+
+    int64_t next = 0, nwait = 0, failed = 0, placed = 0, hb = 0, nrec = 0;
+    double max_ttft = 0.0, max_atgt = 0.0;
+    int rc = ORC_OK;
+    for (;;) {
+        double t = (double)hb * H;
+        while (next < R && t_arr[next] <= t) wl[nwait++] = next++;
+        if (nwait > 0) {
+            for (int64_t i = 0; i < nwait; ++i) {
+                cin[i] = rin[wl[i]];
+                cpr[i] = rpred[wl[i]];
+                cw[i] = t - t_arr[wl[i]];
+            }
+            rc = orc_place_round(p, &cl, (int32_t)nwait, cin, cpr, cw, wl, pl);
+            if (rc != ORC_OK) break;
+            int64_t keep = 0;
+            for (int64_t i = 0; i < nwait; ++i) {
+                if (pl[i] >= 0) { placed++; continue; }
+                double tau_alone = scale * (p->k1 * (double)cin[i] + p->c1);
+                if (cw[i] + H + tau_alone > p->T_pre) failed++;
+                else wl[keep++] = wl[i];
+            }
+            nwait = keep;
+        }
+        if (failed > 0 && stop_at_fail) break;
+        int64_t nr0 = nrec;
+        orc_advance(p, &cl, t, H, rr, rv, rk, &nrec, rec_cap);
+        for (int64_t i = nr0; i < nrec && i < rec_cap; ++i) {
+            if (rk[i] == 0 && rv[i] > max_ttft) max_ttft = rv[i];
+            if (rk[i] == 1 && rv[i] > max_atgt) max_atgt = rv[i];
+        }
+        if (nrec > rec_cap / 2) nrec = 0; /* records are only used for the maxima */
+        hb++;
+        if (next >= R && nwait == 0) {
+            if (!drain) break;
+            int busy = 0;
+            for (int w = 0; w < N; ++w) busy |= cl.n[w] > 0;
+            if (!busy) break;
+        }
+    }
+    out[0] = (double)failed;
+    out[1] = (double)placed;
+    out[2] = (double)hb;
+    out[3] = max_ttft;
+    out[4] = max_atgt;
+    out[5] = (double)nrec;
+    free(Mv); free(sv); free(cl.off); free(cl.clock); free(cl.n); free(cl.in); free(cl.gen);
+    free(cl.pred); free(cl.tdec); free(cl.pend); free(cl.wait); free(cl.rid);
+    free(wl); free(cin); free(cpr); free(cw); free(pl); free(rr); free(rv); free(rk);
+    return rc;
+}
+
+/* Minimum-worker search (Sec. 4.1, Sec. 6.4): for each worker configuration
+ * (GPUs per worker, KV capacity, latency scale) the smallest worker count N in
+ * [1, n_max] that serves the whole trace with no failed request, found by
+ * doubling then bisection. n_out[o] = -1 if even n_max fails. */
+int orc_min_workers(const orc_params* p, int32_t n_opt, const int32_t* gpus, const int64_t* M,
+                    const double* scale, int32_t cap, int64_t R, const double* t_arr,
+                    const int32_t* rin, const int32_t* rpred, double H, int32_t n_max,
+                    int32_t* n_out)
+{
+    double out[6];
+    for (int o = 0; o < n_opt; ++o) {
+        int32_t lo = 0, hi = 1; /* lo fails (or is 0), hi to be tested */
+        int found = 0;
+        while (hi <= n_max) {
+            int rc = orc_simulate(p, hi, cap, M[o], scale[o], R, t_arr, rin, rpred, H, 1, 0, out);
+            if (rc != ORC_OK) return rc;
+            if (out[0] == 0.0) { found = 1; break; }
+            lo = hi;
+            hi = hi * 2 > n_max && hi < n_max ? n_max : hi * 2;
+        }
+        if (!found) { n_out[o] = -1; continue; }
+        while (hi - lo > 1) {
+            int32_t mid = lo + (hi - lo) / 2;
+            int rc = orc_simulate(p, mid, cap, M[o], scale[o], R, t_arr, rin, rpred, H, 1, 0, out);
+            if (rc != ORC_OK) return rc;
+            if (out[0] == 0.0) hi = mid;
+            else lo = mid;
+        }
+        n_out[o] = hi;
+        (void)gpus;
+    }
+    return ORC_OK;
+}
