@@ -1,0 +1,375 @@
+"""Benchmark of the Aladdin scheduler hot path on GB300.
+
+A step is one pass of the hot path over the 4,096-worker workload (128 ongoing
+requests per worker, 32,768 candidate queries, KV capacity 131,072, output
+lengths lognormal(256, 1.2) clipped at 4,096): the worker state, resident in
+HBM, is packed into the cluster and every worker's projection table is rebuilt
+(aladdin_cluster_load), then every candidate is scored against every worker
+with flags, margins and argbest written to HBM (aladdin_score).
+
+Prints one JSON line (rank 0). `value` is candidate x worker evaluations per
+second over all ranks with inputs resident in HBM; `e2e` is the same metric
+through the same C ABI with pinned host buffers (host-to-device copies of the
+state and candidates, device-to-host copies of all outputs inside the timed
+region). `--impl reference` times the CPU oracle instead (there is no upstream
+implementation to install: the paper ships no code).
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import math
+import os
+import statistics
+import subprocess
+import sys
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+METRIC = "candidate x worker placement evaluations/sec"
+UNIT = "evals/s"
+WORKLOAD = "w4096"
+WORKLOAD_DESC = ("4,096 workers x 128 ongoing requests (KV capacity 131,072 tokens), 32,768 candidate "
+                 "queries; input lognormal(512, 0.8) clip [16, 2048], output lognormal(256, 1.2) "
+                 "clip [8, 4096], generated ~ U[0, output); decode 8 ms + 0.05 ms/request + 2e-4 "
+                 "ms/KV token, prefill 10 ms + 0.1 ms/100 tokens, TTFT 1 s, ATGT 50 ms; seed 2")
+L2_FLUSH_BYTES = 256 << 20
+
+
+def algorithmic_bytes(W, B, C):
+    # state in (3 int32 per request) + candidates in (2 int32 + 1 fp32)
+    # + flags (u8) and margin (fp32) per pair + argbest (int32) per candidate
+    return W * B * 12 + C * 12 + C * W * 5 + C * 4
+
+
+def read_peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(path) as f:
+            d = json.load(f)
+        return float(d["hbm_gbs"]), "measured"
+    except Exception:
+        return 6800.0, "fallback"
+
+
+class ClockSampler:
+    """nvidia-smi samples of SM clock and throttle reasons during the timed region."""
+
+    def __init__(self, index):
+        self.index = index
+        self.proc = None
+        self.path = None
+
+    def start(self):
+        q = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+             "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+             "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+        self.path = "/tmp/aladdin_clocks_%d.csv" % os.getpid()
+        try:
+            self.f = open(self.path, "w")
+            self.proc = subprocess.Popen(["nvidia-smi", "-i", str(self.index), "--query-gpu=" + q,
+                                          "--format=csv,noheader,nounits", "-lms", "200"],
+                                         stdout=self.f, stderr=subprocess.DEVNULL)
+        except Exception:
+            self.proc = None
+
+    def stop(self):
+        if self.proc is None:
+            return None
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except Exception:
+            self.proc.kill()
+        self.f.close()
+        sm, mx, reasons = [], 0.0, set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for line in open(self.path):
+            parts = [x.strip() for x in line.split(",")]
+            if len(parts) < 9:
+                continue
+            try:
+                sm.append(float(parts[1]))
+                mx = max(mx, float(parts[2]))
+            except ValueError:
+                continue
+            for k, v in zip(names, parts[5:9]):
+                if v.lower() == "active":
+                    reasons.add(k)
+        os.unlink(self.path)
+        if not sm:
+            return None
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": mx, "reasons": sorted(reasons),
+                "samples": len(sm)}
+
+
+def dist_setup(args):
+    import torch
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    if world > 1:
+        import torch.distributed as dist
+        torch.cuda.set_device(local)
+        dist.init_process_group("nccl", device_id=torch.device("cuda", local))
+        return dist, rank, world, local
+    torch.cuda.set_device(0)
+    return None, 0, 1, 0
+
+
+def barrier_max(dist, value):
+    import torch
+    if dist is None:
+        return value
+    t = torch.tensor([value], dtype=torch.float64, device="cuda")
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def barrier(dist):
+    import torch
+    torch.cuda.synchronize()
+    if dist is not None:
+        dist.barrier()
+    torch.cuda.synchronize()
+
+
+# ---------------------------------------------------------------------------
+# CPU oracle baseline (bounded sample; spawn pool across host cores).
+
+def _oracle_slice(args):
+    wid, ncand = args
+    from oracle import oracle as O
+    from paper_2405_06856_gb300 import synth
+    wl = synth.config(WORKLOAD)
+    sub = O.Cluster(wl.params, wl.kv_capacity[wid], wl.lat_scale[wid], wl.b_cap,
+                    np.concatenate([[0], np.cumsum(np.diff(wl.roff)[wid])]).astype(np.int32),
+                    np.concatenate([wl.req_in[wl.roff[w]:wl.roff[w + 1]] for w in wid]),
+                    np.concatenate([wl.req_gen[wl.roff[w]:wl.roff[w + 1]] for w in wid]),
+                    np.concatenate([wl.req_pred[wl.roff[w]:wl.roff[w + 1]] for w in wid]))
+    t0 = time.perf_counter()
+    sub.score(wl.cand_in[:ncand], wl.cand_pred[:ncand], wl.cand_wait[:ncand],
+              want=("flags", "margin"))
+    return len(wid) * ncand, time.perf_counter() - t0
+
+
+def oracle_baseline(workers_per_core=4, ncand=32768, cores=None):
+    """Oracle evaluations/sec: each process scores all pairs of its own workers
+    against the first `ncand` candidates; throughput = pairs / wall time."""
+    import multiprocessing as mp
+    from oracle import oracle as O
+    O.build()
+    cores = cores or os.cpu_count() or 1
+    jobs = [(list(range(i * workers_per_core, (i + 1) * workers_per_core)), ncand)
+            for i in range(cores)]
+    ctx = mp.get_context("spawn")
+    t0 = time.perf_counter()
+    with ctx.Pool(cores) as pool:
+        res = pool.map(_oracle_slice, jobs)
+    wall = time.perf_counter() - t0
+    pairs = sum(r[0] for r in res)
+    busy = max(r[1] for r in res)
+    return {"value": pairs / busy, "unit": UNIT, "cores": cores, "kind": "oracle",
+            "sample": "%d workers x %d candidates of %s (%d pairs, %.1f s per process, %.1f s wall)"
+                      % (cores * workers_per_core, ncand, WORKLOAD, pairs, busy, wall)}
+
+
+# ---------------------------------------------------------------------------
+
+def run_reference(args):
+    dist, rank, world, local = (None, 0, 1, 0)
+    if int(os.environ.get("WORLD_SIZE", "1")) > 1 and int(os.environ.get("RANK", "0")) != 0:
+        return
+    steps, warm = args.steps, args.warmup
+    vals = []
+    base = None
+    for i in range(warm + steps):
+        b = oracle_baseline(workers_per_core=1, ncand=2048)
+        if i >= warm:
+            vals.append(b["value"])
+            base = b
+    v = float(statistics.median(vals)) if vals else 0.0
+    from paper_2405_06856_gb300 import synth
+    wl = synth.config(WORKLOAD, n_cand=16)
+    ms = wl.n_workers * 32768 / v * 1000.0 if v > 0 else None
+    base["value"] = v
+    line = {"impl": "reference", "metric": METRIC, "value": v, "unit": UNIT,
+            "n_gpus": args.gpus, "steps": steps, "warmup": warm, "ms_per_step": ms,
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+            "data": "synthetic", "config": {"workload": WORKLOAD_DESC},
+            "cpu_baseline": base,
+            "e2e": {"value": v, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(line))
+
+
+def run_ours(args):
+    import torch
+    from paper_2405_06856_gb300 import build as B
+    B.build()
+    from paper_2405_06856_gb300 import aladdin as A
+    from paper_2405_06856_gb300 import synth
+
+    # The oracle's process pool is started before the first CUDA call.
+    cpu = None
+    if args.cpu_baseline and int(os.environ.get("RANK", "0")) == 0 and args.gpus == 1:
+        cpu = oracle_baseline()
+
+    dist, rank, world, local = dist_setup(args)
+    dev = torch.device("cuda", local)
+    wl = synth.config(WORKLOAD)
+    W, C = wl.n_workers, wl.n_cand
+    Bq = int(np.diff(wl.roff).max())
+    stream = torch.cuda.current_stream().cuda_stream
+
+    d = lambda x: torch.from_numpy(np.ascontiguousarray(x)).to(dev)
+    roff, rin, rgen, rpred = d(wl.roff), d(wl.req_in), d(wl.req_gen), d(wl.req_pred)
+    cin, cpr, cw = d(wl.cand_in), d(wl.cand_pred), d(wl.cand_wait)
+    flags = torch.empty((C, W), dtype=torch.uint8, device=dev)
+    margin = torch.empty((C, W), dtype=torch.float32, device=dev)
+    arg = torch.empty(C, dtype=torch.int32, device=dev)
+    flush = torch.empty(L2_FLUSH_BYTES // 4, dtype=torch.float32, device=dev)
+    cl = A.Cluster.from_workload(wl, stream=stream)
+
+    def step():
+        A.aladdin_cluster_load(cl.handle, roff, rin, rgen, rpred)
+        A.aladdin_score(cl.handle, C, cin, cpr, cw, flags, margin, arg)
+
+    for _ in range(args.warmup):
+        step()
+    torch.cuda.synchronize()
+    assert cl.status() == A.OK
+    frac_feasible = float((flags == 15).float().mean().item())
+
+    # timed region: per-step CUDA events, L2 flushed (256 MiB write) between steps
+    starts = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
+    ends = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
+    A.aladdin_cluster_timing(cl.handle, 1)
+    sampler = ClockSampler(local)
+    barrier(dist)
+    sampler.start()
+    for i in range(args.steps):
+        flush.zero_()
+        starts[i].record()
+        step()
+        ends[i].record()
+    barrier(dist)
+    clocks = sampler.stop()
+    kern_ms, kern_n = A.aladdin_cluster_timing(cl.handle, 0)
+    step_ms = sum(s.elapsed_time(e) for s, e in zip(starts, ends)) / args.steps
+    step_ms = barrier_max(dist, step_ms)
+    value = world * C * W / (step_ms / 1000.0)
+
+    # end to end through the same API with pinned host buffers
+    pin = lambda x: torch.from_numpy(np.ascontiguousarray(x)).pin_memory()
+    h_roff, h_rin, h_rgen, h_rpred = pin(wl.roff), pin(wl.req_in), pin(wl.req_gen), pin(wl.req_pred)
+    h_cin, h_cpr, h_cw = pin(wl.cand_in), pin(wl.cand_pred), pin(wl.cand_wait)
+    h_flags = torch.empty((C, W), dtype=torch.uint8).pin_memory()
+    h_margin = torch.empty((C, W), dtype=torch.float32).pin_memory()
+    h_arg = torch.empty(C, dtype=torch.int32).pin_memory()
+
+    def step_host():
+        A.aladdin_cluster_load(cl.handle, h_roff, h_rin, h_rgen, h_rpred)
+        A.aladdin_score(cl.handle, C, h_cin, h_cpr, h_cw, h_flags, h_margin, h_arg)
+
+    for _ in range(2):
+        step_host()
+    torch.cuda.synchronize()
+    e2e_steps = max(3, min(args.steps, 10))
+    barrier(dist)
+    t0 = time.perf_counter()
+    for _ in range(e2e_steps):
+        step_host()
+    torch.cuda.synchronize()
+    e2e_ms = barrier_max(dist, (time.perf_counter() - t0) * 1000.0 / e2e_steps)
+    assert np.array_equal(h_arg.numpy(), arg.cpu().numpy())
+    h2d = wl.roff.nbytes + wl.req_in.nbytes + wl.req_gen.nbytes + wl.req_pred.nbytes + \
+        wl.cand_in.nbytes + wl.cand_pred.nbytes + wl.cand_wait.nbytes
+    d2h = C * W * 5 + C * 4
+
+    # round latency on the 256-worker workload (one greedy round of 2,048 candidates)
+    w2 = synth.config("w256", b_cap=128)
+    rounds = []
+    for _ in range(3):
+        with A.Cluster.from_workload(w2, stream=stream) as c2:
+            pl = torch.empty(w2.n_cand, dtype=torch.int32, device=dev)
+            t_in, t_pr, t_w = d(w2.cand_in), d(w2.cand_pred), d(w2.cand_wait)
+            torch.cuda.synchronize()
+            t0 = time.perf_counter()
+            A.aladdin_place_round(c2.handle, w2.n_cand, t_in, t_pr, t_w, pl)
+            rounds.append((time.perf_counter() - t0) * 1000.0)
+    round_ms = min(rounds)
+
+    peak, peak_kind = read_peaks()
+    kern_avg = kern_ms / max(kern_n, 1)
+    abytes = algorithmic_bytes(W, Bq, C)
+    achieved = abytes / (kern_avg / 1000.0) / 1e9
+    traffic = None
+    tp = os.path.join(ROOT, "profiles", "traffic_k_score_w4096.json")
+    if os.path.exists(tp):
+        try:
+            tj = json.load(open(tp))
+            if tj.get("source_hash") == kernel_source_hash():
+                traffic = tj["dram_bytes_per_launch"]
+        except Exception:
+            traffic = None
+
+    launches_per_step = 3 + 5  # load: pack, build, rank; score: count, scan, scatter, score, finalize
+    line = {"metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
+            "warmup": args.warmup, "ms_per_step": step_ms, "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "f32",
+            "data": "synthetic",
+            "config": {"workload": WORKLOAD_DESC, "n_workers": W, "requests_per_worker": Bq,
+                       "n_cand": C, "l2": "flushed between steps (256 MiB write)",
+                       "outputs": "flags u8 + margin f32 per pair, argbest per candidate",
+                       "parallelism": "replicas" if world > 1 else "single GPU",
+                       "feasible_fraction": round(frac_feasible, 4)},
+            "e2e": {"value": world * C * W / (e2e_ms / 1000.0), "unit": UNIT,
+                    "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h, "ms_per_step": e2e_ms},
+            "gpu_launches": launches_per_step * args.steps,
+            "roofline": {"bound": "hbm", "kernel": "k_score", "achieved": achieved, "peak": peak,
+                         "peak_kind": peak_kind, "unit": "GB/s", "frac": achieved / peak,
+                         "traffic": traffic, "algorithmic_bytes_per_launch": abytes,
+                         "kernel_ms": kern_avg, "launches": kern_n},
+            "round_latency_ms": {"workload": "256 workers x 64 requests, 2,048 candidates, one "
+                                             "greedy round", "value": round_ms},
+            "clocks": clocks}
+    if cpu is not None:
+        line["cpu_baseline"] = cpu
+    if rank == 0:
+        print(json.dumps(line))
+    cl.close()
+    if dist is not None:
+        dist.destroy_process_group()
+
+
+def kernel_source_hash():
+    import hashlib
+    h = hashlib.sha256()
+    for f in ("aladdin_dev.cuh", "score.cu"):
+        h.update(open(os.path.join(ROOT, "paper_2405_06856_gb300", "csrc", f), "rb").read())
+    return h.hexdigest()[:16]
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=20)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    ap.add_argument("--no-cpu-baseline", dest="cpu_baseline", action="store_false")
+    args = ap.parse_args()
+    if args.warmup < 3:
+        args.warmup = 3
+    if args.impl == "reference":
+        run_reference(args)
+    else:
+        run_ours(args)
+
+
+if __name__ == "__main__":
+    main()

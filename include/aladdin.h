@@ -1,0 +1,215 @@
+/*
+ * aladdin.h - C ABI of the GB300 scheduler hot path of Aladdin
+ * ("Aladdin: Joint Placement and Scaling for SLO-Aware LLM Serving",
+ * arxiv 2405.06856).
+ *
+ * The library scores candidate queries against serving workers (Sec. 4.2:
+ * constraints (c), (d), (e) with the paper's KV, prefill and decode models of
+ * Sec. 3), places them greedily with the best-fit heuristic (Algorithm 1) and
+ * searches the minimum number of workers per worker configuration (Sec. 4.1,
+ * Sec. 6.4). Every computation runs in CUDA kernels on the current GPU; there
+ * is no CPU fallback.
+ *
+ * Conventions
+ *  - Lengths are int32 token counts, times are milliseconds.
+ *  - Pointer arguments may point to host memory or to device memory of the
+ *    cluster's GPU; the library inspects each pointer. With device pointers a
+ *    call is asynchronous on the cluster's stream; when any output is in host
+ *    memory the call returns after the stream has completed.
+ *  - The caller owns every buffer it passes; the library never frees caller
+ *    memory and keeps no pointer to it after the call returns.
+ *  - Pair outputs are row-major [candidate][worker].
+ *  - Every function returns ALADDIN_OK (0) or a negative error code; nothing
+ *    else crosses the ABI. Results are deterministic: the same inputs give the
+ *    same bytes.
+ */
+#ifndef ALADDIN_H
+#define ALADDIN_H
+
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+#define ALADDIN_OK 0
+#define ALADDIN_ERR_ARG (-1)      /* null pointer, bad size, length or coefficient */
+#define ALADDIN_ERR_CAPACITY (-2) /* a worker would exceed its request slots b_cap */
+#define ALADDIN_ERR_CUDA (-3)     /* a CUDA runtime call failed */
+#define ALADDIN_ERR_TIMEOUT (-4)  /* a bounded device-side wait expired */
+#define ALADDIN_ERR_NOMEM (-5)    /* device or host allocation failed */
+#define ALADDIN_ERR_STATE (-6)    /* the cluster holds an invalid request (see
+                                     aladdin_cluster_load) */
+
+/* Pair flags (one byte per (candidate, worker)). */
+#define ALADDIN_FLAG_KV 1u        /* (e): KV usage stays within capacity every iteration */
+#define ALADDIN_FLAG_TTFT 2u      /* (c): candidate and this round's placements meet T_pre */
+#define ALADDIN_FLAG_ONGOING 4u   /* (d): requests decoding at round start absorb the stall */
+#define ALADDIN_FLAG_NEW 8u       /* candidate and this round's placements meet T_dec */
+#define ALADDIN_FEASIBLE 15u      /* all four */
+#define ALADDIN_FLAG_INVALID 128u /* the candidate itself is invalid (see aladdin_score) */
+
+#define ALADDIN_NONE (-1)         /* argbest / placement: no feasible worker */
+#define ALADDIN_INVALID (-2)      /* argbest / placement: the candidate is invalid */
+
+/* Performance models and SLOs (Sec. 3, Sec. 4.2).
+ *   prefill iteration (Eq. prefill iter time): t_pre = k1 * sum(l_in) + c1
+ *   decode iteration  (Eq. iter time):         t_d = k2 * sum(context) + c2 * b + c3
+ *   KV usage          (Eq. kv cache):          kv = h * (l_in + l_out) + j
+ * Requirements: k1, k2 > 0; c1, c2, c3 >= 0; h >= 1; j >= 0; T_pre > 0;
+ * T_dec > c3 (Eq. input limit); 0 < theta <= 1; gamma >= 0; 2 <= K <= 65536;
+ * b_cap a power of two in [32, 512]. */
+typedef struct aladdin_params {
+    double k1, c1;       /* prefill: ms per input token, ms */
+    double k2, c2, c3;   /* decode: ms per context token, ms per request, ms */
+    int32_t h, j;        /* KV slots per context token, per request */
+    double T_pre;        /* TTFT SLO (ms) */
+    double T_dec;        /* average token generation time SLO (ms per token) */
+    double gamma;        /* capacity_norm weight of predicted output (Sec. 4.2) */
+    double theta;        /* SLO scaling knob of (b), (d) */
+    int32_t K;           /* sequence limit: l_in + l_pred <= K for every request */
+    int32_t b_cap;       /* request slots per worker (ongoing + this round's) */
+} aladdin_params;
+
+/* One worker configuration (Sec. 4.1): GPUs per worker, KV capacity in KV
+ * slots (< 2^24), and a multiplier applied to every latency coefficient. */
+typedef struct aladdin_worker_cfg {
+    int32_t gpus;
+    int64_t kv_capacity;
+    double lat_scale;
+} aladdin_worker_cfg;
+
+typedef struct aladdin_cluster aladdin_cluster;
+
+/* Create a cluster of n_workers workers on the current CUDA device, bound to
+ * cuda_stream (a cudaStream_t; NULL = the legacy default stream).
+ * Worker w's ongoing requests (Table 1: l_in, l_out generated so far, l_pred)
+ * are [req_off[w], req_off[w+1]) of in / gen / pred; req_off has
+ * n_workers + 1 entries. tdec_ms (nullable) gives each request's decode time
+ * so far (Table 1: t^dec); when NULL every request is taken to have used
+ * exactly its theta-scaled budget so far. Each request needs in >= 0,
+ * 0 <= gen < pred and in + pred <= K; each worker at most b_cap requests.
+ * Errors: ALADDIN_ERR_ARG, ALADDIN_ERR_CAPACITY, ALADDIN_ERR_NOMEM,
+ * ALADDIN_ERR_CUDA. On error *out is NULL. */
+int aladdin_cluster_create(const aladdin_params* params, int32_t n_workers,
+                           const aladdin_worker_cfg* cfg, const int32_t* req_off,
+                           const int32_t* in, const int32_t* gen, const int32_t* pred,
+                           const float* tdec_ms, void* cuda_stream, aladdin_cluster** out);
+
+int aladdin_cluster_destroy(aladdin_cluster* cl);
+
+/* Replace every worker's requests (same layout as aladdin_cluster_create) and
+ * rebuild the per-worker projection tables: packing into device slots, sorting
+ * of remaining lengths, breakpoints, prefix sums, KV and latency curves at the
+ * breakpoints and the capacity_norm ranking (Sec. 4.2). Host inputs are
+ * validated before upload (ALADDIN_ERR_ARG / ALADDIN_ERR_CAPACITY). Device
+ * inputs are validated on the GPU: a worker holding an invalid request is made
+ * infeasible for every candidate and the cluster records ALADDIN_ERR_STATE,
+ * which aladdin_cluster_status returns. Any round in progress is discarded
+ * and the cluster clock is kept. */
+int aladdin_cluster_load(aladdin_cluster* cl, const int32_t* req_off, const int32_t* in,
+                         const int32_t* gen, const int32_t* pred, const float* tdec_ms);
+
+/* Score n_cand candidates (prompt length in[c], predicted output pred[c],
+ * wait_ms[c] since arrival, nullable = 0) against every worker.
+ *  flags  [n_cand*W] (nullable): ALADDIN_FLAG_* bits per pair.
+ *  margin [n_cand*W] (nullable): the largest prompt length the worker could
+ *         accept for this candidate (all constraints are monotone in it)
+ *         minus in[c]; >= 0 exactly when the pair is feasible, -inf when no
+ *         prompt length fits.
+ *  argbest[n_cand] (nullable): Algorithm 1's choice: the feasible worker with
+ *         the largest capacity_norm, lowest index on ties; ALADDIN_NONE if no
+ *         worker is feasible.
+ * A candidate with in < 0, pred < 1, in + pred > K or a negative or
+ * non-finite wait is invalid: its flags are ALADDIN_FLAG_INVALID, its margins
+ * NaN and its argbest ALADDIN_INVALID; the call still succeeds. Outputs of a
+ * pending round (placements so far) are included in the state scored. */
+int aladdin_score(aladdin_cluster* cl, int32_t n_cand, const int32_t* in, const int32_t* pred,
+                  const float* wait_ms, uint8_t* flags, float* margin, int32_t* argbest);
+
+/* As aladdin_score, plus two verification outputs per pair (each nullable):
+ * kv_peak [n_cand*W]: the worker's peak KV usage over all future iterations
+ * with the candidate added (exact integer), and t_cand_ms [n_cand*W]: the
+ * candidate's projected total decode time on the worker. */
+int aladdin_score_detail(aladdin_cluster* cl, int32_t n_cand, const int32_t* in,
+                         const int32_t* pred, const float* wait_ms, uint8_t* flags,
+                         float* margin, int32_t* argbest, int64_t* kv_peak, float* t_cand_ms);
+
+/* One greedy best-fit round (Algorithm 1): candidates in index order, each
+ * placed on the feasible worker of largest capacity_norm in the state left by
+ * the earlier placements, where it becomes a request of this round (prefill
+ * pending, gen = 0). placement[c] = worker, ALADDIN_NONE if none is feasible
+ * (the cluster is fixed: no worker is opened), ALADDIN_INVALID for an invalid
+ * candidate. Returns ALADDIN_ERR_CAPACITY if a chosen worker has no free slot
+ * (placements up to that candidate are kept). */
+int aladdin_place_round(aladdin_cluster* cl, int32_t n_cand, const int32_t* in,
+                        const int32_t* pred, const float* wait_ms, int32_t* placement);
+
+/* Execute every worker for dt_ms from the cluster clock (continuous batching,
+ * Sec. 2.1): at its next iteration boundary a worker runs the prefill of this
+ * round's placements (stalling its decoding requests), then decode iterations
+ * back to back while they start before clock + dt_ms; finished requests leave.
+ * The clock then advances by dt_ms and a new round begins.
+ * stats (nullable, host, 4 doubles) accumulates since creation:
+ * [0] requests whose prefill ran, [1] requests finished,
+ * [2] largest realized TTFT (ms), [3] largest realized ATGT (ms per token). */
+int aladdin_cluster_advance(aladdin_cluster* cl, double dt_ms, double* stats);
+
+/* Copy the cluster state to host arrays (each nullable): n[W] requests per
+ * worker, and per slot [W*b_cap] in, gen, pred, pending (1 = placed this
+ * round). Synchronous. */
+int aladdin_cluster_state(aladdin_cluster* cl, int32_t* n, int32_t* in, int32_t* gen,
+                          int32_t* pred, uint8_t* pending);
+
+/* Kernel timing (tracing): while enabled, CUDA events on the cluster's stream
+ * bracket every launch of the candidate x worker scoring kernel. Each call
+ * waits for the stream, returns in *kernel_ms (nullable) the summed event time
+ * of the launches bracketed since the previous call and in *launches
+ * (nullable) their number, forgets them, and turns the timing on (enable != 0)
+ * or off. */
+int aladdin_cluster_timing(aladdin_cluster* cl, int32_t enable, double* kernel_ms,
+                           int64_t* launches);
+
+/* ALADDIN_OK, or ALADDIN_ERR_STATE if an invalid request was loaded from device
+ * memory, or ALADDIN_ERR_CUDA. Synchronous. */
+int aladdin_cluster_status(aladdin_cluster* cl);
+
+/* A request trace: arrival times (ms, non-decreasing), prompt and predicted
+ * output lengths. */
+typedef struct aladdin_trace {
+    int64_t n;
+    const double* t_arr_ms;
+    const int32_t* in;
+    const int32_t* pred;
+} aladdin_trace;
+
+/* Minimum-worker search (Sec. 4.1, Sec. 6.4): for every worker configuration
+ * options[o], the smallest number of identical workers in [1, n_max] that
+ * serves the whole trace with every request placed within its TTFT (heartbeat
+ * every heartbeat_ms; at each, the waiting arrivals form one placement round,
+ * then the workers execute until the next heartbeat; a request that can no
+ * longer meet T_pre on an empty worker fails). Found by doubling then
+ * bisection; each simulation runs on the GPU. n_workers[o] = -1 if n_max
+ * workers fail. best_option (nullable) receives the option with the fewest
+ * total GPUs (gpus * n_workers; first on ties), total_gpus (nullable) that
+ * total. Trace arrays are host memory. */
+int aladdin_min_workers(const aladdin_params* params, int32_t n_options,
+                        const aladdin_worker_cfg* options, const aladdin_trace* trace,
+                        double heartbeat_ms, int32_t n_max, void* cuda_stream,
+                        int32_t* n_workers, int32_t* best_option, int64_t* total_gpus);
+
+/* Simulate the trace on n identical workers of configuration cfg (the check
+ * inside aladdin_min_workers). out (host, 5 doubles): [0] failed requests,
+ * [1] placed requests, [2] heartbeats run, [3] largest realized TTFT,
+ * [4] largest realized ATGT. With stop_at_fail the simulation ends at the
+ * first failure; with drain it continues after the last arrival until every
+ * worker is idle. */
+int aladdin_simulate(const aladdin_params* params, const aladdin_worker_cfg* cfg, int32_t n,
+                     const aladdin_trace* trace, double heartbeat_ms, int32_t stop_at_fail,
+                     int32_t drain, void* cuda_stream, double* out);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* ALADDIN_H */

@@ -1,0 +1,172 @@
+// Execution step of the fleet simulation (continuous batching, Sec. 2.1): one
+// warp per worker runs, from the worker's next iteration boundary, the prefill
+// of this round's placements (Eq. prefill iter time; it stalls the decoding
+// requests), then decode iterations back to back (Eq. iter time) while they
+// start before t_now + dt. Each iteration adds one token to every active
+// request; requests that reach their predicted length leave and their
+// realized ATGT (decode time over decode tokens, Sec. 2.2) is recorded.
+// Times accumulate in fp64 with explicitly rounded operations, in the same
+// order as the CPU reference, so both sides produce the same schedule.
+#include "aladdin_host.h"
+
+namespace aladdin {
+
+constexpr int ADV_WARPS = 4;
+
+__device__ __forceinline__ void atomic_max_nonneg(unsigned long long* addr, double v)
+{
+    atomicMax(addr, (unsigned long long)__double_as_longlong(v));
+}
+
+template <int E>
+__global__ void __launch_bounds__(ADV_WARPS * 32)
+k_advance(DevParams P, ClusterDev C, double t_now, double dt, unsigned long long* stats,
+          const int* halt)
+{
+    if (halt && *halt != 0) return;
+    const int lane = threadIdx.x & 31;
+    const int w = blockIdx.x * ADV_WARPS + (threadIdx.x >> 5);
+    if (w >= C.W) return;  // warp-uniform
+    const int n = C.n[w];
+    const long long base = (long long)w * C.cap;
+    const double s = C.scaled[w];
+    const double t_end = __dadd_rn(t_now, dt);
+
+    int in[E], gen[E], pred[E];
+    double tdec[E];
+    bool alive[E];
+    long long Pint = 0;
+    int npend = 0;
+    double maxttft = 0.0, maxatgt = 0.0;
+    unsigned long long nfin = 0;
+    double start = C.clock[w] > t_now ? C.clock[w] : t_now;
+#pragma unroll
+    for (int e = 0; e < E; ++e) {
+        const int x = e * 32 + lane;
+        alive[e] = x < n;
+        in[e] = gen[e] = 0;
+        pred[e] = 1;
+        tdec[e] = 0.0;
+        if (alive[e]) {
+            const long long slot = base + x;
+            in[e] = C.in[slot];
+            gen[e] = C.gen[slot];
+            pred[e] = C.pred[slot];
+            tdec[e] = C.tdec[slot];
+            if (C.pend[slot]) {
+                Pint += in[e];
+                npend += 1;
+            }
+        }
+    }
+    Pint = warp_reduce(Pint, OpAdd<long long>());
+    npend = warp_reduce(npend, OpAdd<int>());
+    if (npend > 0) {
+        const double tau = __dmul_rn(s, __dadd_rn(__dmul_rn(P.k1d, (double)Pint), P.c1d));
+        const double lead = __dsub_rn(start, t_now);
+#pragma unroll
+        for (int e = 0; e < E; ++e) {
+            if (!alive[e]) continue;
+            const long long slot = base + e * 32 + lane;
+            if (C.pend[slot]) {
+                const double ttft = __dadd_rn(__dadd_rn(C.wait[slot], lead), tau);
+                maxttft = fmax(maxttft, ttft);
+                gen[e] = 0;
+                tdec[e] = 0.0;
+            } else {
+                tdec[e] = __dadd_rn(tdec[e], tau);
+            }
+        }
+        start = __dadd_rn(start, tau);
+    }
+    // Decode iterations (bounded: every iteration finishes at least one token
+    // of every active request, so at most max(pred) iterations run).
+    for (;;) {
+        int b = 0;
+        long long K = 0;
+#pragma unroll
+        for (int e = 0; e < E; ++e)
+            if (alive[e]) {
+                b += 1;
+                K += (long long)in[e] + gen[e] + 1;
+            }
+        b = warp_reduce(b, OpAdd<int>());
+        K = warp_reduce(K, OpAdd<long long>());
+        if (b == 0 || !(start < t_end)) break;
+        const double t = __dmul_rn(
+            s, __dadd_rn(__dadd_rn(P.c3d, __dmul_rn(P.c2d, (double)b)), __dmul_rn(P.k2d, (double)K)));
+#pragma unroll
+        for (int e = 0; e < E; ++e)
+            if (alive[e]) {
+                gen[e] += 1;
+                tdec[e] = __dadd_rn(tdec[e], t);
+                if (gen[e] >= pred[e]) {
+                    maxatgt = fmax(maxatgt, __ddiv_rn(tdec[e], (double)pred[e]));
+                    nfin += 1;
+                    alive[e] = false;
+                }
+            }
+        start = __dadd_rn(start, t);
+    }
+    // Write the surviving requests back in their order, densely.
+    int pos = 0;
+#pragma unroll
+    for (int e = 0; e < E; ++e) {
+        const unsigned bal = __ballot_sync(FULL, alive[e]);
+        const int before = __popc(bal & ((1u << lane) - 1u));
+        const long long src = base + e * 32 + lane;
+        // read the fields that are not kept in registers before any write
+        double wt = 0.0;
+        if (alive[e]) wt = C.wait[src];
+        __syncwarp();
+        if (alive[e]) {
+            const long long dst = base + pos + before;
+            C.in[dst] = in[e];
+            C.gen[dst] = gen[e];
+            C.pred[dst] = pred[e];
+            C.tdec[dst] = tdec[e];
+            C.pend[dst] = 0;
+            C.wait[dst] = wt;
+        }
+        __syncwarp();
+        pos += __popc(bal);
+    }
+    maxttft = warp_reduce(maxttft, OpMax<double>());
+    maxatgt = warp_reduce(maxatgt, OpMax<double>());
+    nfin = warp_reduce(nfin, OpAdd<unsigned long long>());
+    if (lane == 0) {
+        C.n[w] = pos;
+        C.clock[w] = start;
+        C.off[w] = start > t_end ? (float)__dsub_rn(start, t_end) : 0.0f;
+        if (stats) {
+            if (npend) atomicAdd(&stats[0], (unsigned long long)npend);
+            if (nfin) atomicAdd(&stats[1], nfin);
+            if (npend) atomic_max_nonneg(&stats[2], maxttft);
+            if (nfin) atomic_max_nonneg(&stats[3], maxatgt);
+        }
+    }
+}
+
+template <int E>
+static cudaError_t advance_e(const DevParams& P, const ClusterDev& C, double t_now, double dt,
+                             unsigned long long* stats, const int* halt, cudaStream_t st)
+{
+    const int blocks = (C.W + ADV_WARPS - 1) / ADV_WARPS;
+    k_advance<E><<<blocks, ADV_WARPS * 32, 0, st>>>(P, C, t_now, dt, stats, halt);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_advance(const DevParams& P, const ClusterDev& C, double t_now, double dt,
+                           unsigned long long* stats, const int* halt, cudaStream_t st)
+{
+    switch (lanes_per_worker(C.cap)) {
+    case 1: return advance_e<1>(P, C, t_now, dt, stats, halt, st);
+    case 2: return advance_e<2>(P, C, t_now, dt, stats, halt, st);
+    case 4: return advance_e<4>(P, C, t_now, dt, stats, halt, st);
+    case 8: return advance_e<8>(P, C, t_now, dt, stats, halt, st);
+    case 16: return advance_e<16>(P, C, t_now, dt, stats, halt, st);
+    default: return cudaErrorInvalidValue;
+    }
+}
+
+}  // namespace aladdin

@@ -1,0 +1,546 @@
+// Device-side data layout and the two primitives every kernel of the library
+// shares: building one worker's projection table (one warp per worker) and
+// evaluating one (candidate, worker) pair against a table row in O(1).
+//
+// Method (Sec. 3 and Sec. 4.2 of arxiv 2405.06856). For worker i with requests
+// j (context a_j = l_in + l_out, remaining decode iterations r_j) the future
+// iteration s has b(s) = #{r_j >= s} active requests holding
+// K(s) = sum_{r_j >= s} (a_j + s) context tokens; its KV usage is
+// h K(s) + j b(s) (Eq. kv cache) and it lasts t(s) = c3 + c2 b(s) + k2 K(s)
+// (Eq. iter time). Sorting the distinct remaining lengths rho_1 < ... < rho_R
+// turns both curves into segments on which b is constant: with
+// n_p = #{r_j > rho_p}, A_p = sum_{r_j > rho_p} a_j,
+//   K(s) = A_p + s n_p                      for rho_p < s <= rho_{p+1},
+//   T(x) = sum_{s<=x} t(s) = c2 PR_p + k2 PRA_p + x (c3 + c2 n_p + k2 A_p)
+//          + k2 n_p x (x + 1) / 2           for rho_p <= x <= rho_{p+1},
+// where PR_p = sum_{r_j <= rho_p} r_j and
+// PRA_p = sum_{r_j <= rho_p} (r_j a_j + r_j (r_j + 1) / 2) are exact integer
+// prefix sums. KV grows inside a segment, so its maximum sits at a breakpoint
+// (the paper's observation that a request's KV peaks just before it finishes).
+//
+// A candidate (prompt a, predicted output r, wait w) inserts one breakpoint.
+// Every constraint of the placement test is monotone and affine in a, so each
+// becomes "a <= bound" with a bound that is O(1) to evaluate from the row p of
+// the segment containing r (rho_p <= r < rho_{p+1}):
+//   KV (e):  a <= floor((M - j - PM_p)/h) and
+//            a <= floor((M - j(n_p+1))/h) - A_p - r (n_p + 1), and no KV peak
+//            after the candidate exceeds M (SM_p <= M);
+//   TTFT (c): a <= (T_pre - w - off)/(s k1) - c1/k1 - P, and the same for the
+//            largest wait among this round's placements;
+//   ongoing (d), requests finishing with or before the candidate:
+//            a <= min_{r_j <= r} (u_j - s(k1 P + c1)) / (s (k2 r_j + k1)),
+//            u_j = sigma_j - s (c2 r_j + k2 r_j (r_j + 1)/2), a prefix minimum;
+//            requests finishing after it:
+//            a <= (min_{r_j > r} sigma_j / s - s(k1 P + c1)/s - X(r)) / (k2 r + k1),
+//            X(r) = c2 r + k2 r (r + 1) / 2, a suffix minimum;
+//   new requests (no stall): the same with k1 = 0 and P = 0;
+//   candidate: a <= theta T_dec/(s k2) - X(r)/(k2 r) - T_u(r)/(k2 r).
+// Here sigma_j = theta T_dec r_j + bank_j - T(r_j) is request j's slack before
+// the candidate, s the worker's latency scale and P its pending prefill tokens.
+// The pair's margin is the smallest bound minus a.
+#pragma once
+
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+namespace aladdin {
+
+constexpr unsigned FULL = 0xffffffffu;
+constexpr int ROW_F4 = 3;               // float4 per table row
+constexpr long long LL_NONE = (-0x7fffffffffffffffLL - 1);
+
+struct DevParams {
+    float k1, c1, k2, c2, c3;
+    int32_t h, j;
+    float T_pre, T_dec, gamma, theta;
+    int32_t K, cap;
+    // derived in double on the host, rounded once
+    float c2_over_k2, c3_over_k2, c1_over_k1, inv_k1, theta_Tdec, thTdec_over_k2;
+    // double copies for execution (advance) and exact capacity_norm keys
+    double k1d, c1d, k2d, c2d, c3d, T_pred, T_decd, gammad, thetad;
+};
+
+// Exact integer aggregates of one table row (verification outputs only).
+struct __align__(16) AuxRow {
+    long long PM;   // max_{m <= p} KV(rho_m) + h rho_m, LL_NONE for p = 0
+    long long SM;   // max_{m > p} KV(rho_m), 0 if none
+    long long A;    // sum_{r_j > rho_p} a_j
+    long long PR;   // sum_{r_j <= rho_p} r_j
+    long long PRA;  // sum_{r_j <= rho_p} (r_j a_j + r_j (r_j + 1) / 2)
+    int32_t n;      // #{r_j > rho_p}
+    int32_t rho;    // rho_p
+};
+
+struct ClusterDev {
+    int32_t W, cap, rows;      // rows per worker = cap + 1
+    const float* scale;        // [W] latency coefficient multiplier
+    const double* scaled;      // [W] the same in double (execution)
+    const int32_t* M;          // [W] KV capacity (slots)
+    float* off;                // [W] ms from the round's time to the next iteration start
+    double* clock;             // [W] absolute ms of the next iteration start
+    int32_t* n;                // [W] requests
+    int32_t* in;               // [W*cap]
+    int32_t* gen;              // [W*cap]
+    int32_t* pred;             // [W*cap]
+    double* tdec;              // [W*cap] decode time so far (ms)
+    uint8_t* pend;             // [W*cap] 1: placed this round, prefill pending
+    double* wait;              // [W*cap] pending: wait since arrival at placement
+    float4* tab;               // [W*rows*ROW_F4] scoring rows
+    AuxRow* aux;               // [W*rows]
+    int32_t* R;                // [W] breakpoints
+    float4* wrec;              // [W] {1/s, ZO, ZW, rank bits}
+    double* key;               // [W] capacity_norm^2
+    int32_t* rank;             // [W]
+    int32_t* order;            // [W] worker at rank
+    unsigned int* err;         // sticky error bits (1: invalid request)
+};
+
+// Table row p of a worker (3 x float4):
+//  v0 = {rho_{p+1} (int bits; INT_MAX for the last row), kvB1, kvE, -(n_p + 1)}
+//  v1 = {beta0n, beta1s, nh, pmA}
+//  v2 = {pmAp, Gt, Gpt, rho_p (int bits)}
+// kvB1 = floor((M - j - PM_p)/h) (+inf for p = 0, -inf if SM_p > M)
+// kvE  = floor((M - j (n_p + 1))/h) - A_p
+// beta0n = -(c2/k2 PR_p + PRA_p); beta1s = (c3 + c2 n_p)/k2 + A_p + n_p/2 - theta T_dec/(s k2)
+// nh = -n_p/2; pmA / pmAp prefix-minimum bounds of ongoing / new requests with
+// r_j <= rho_p; Gt / Gpt = suffix-minimum slack of ongoing / new requests with
+// r_j > rho_p, over s, ongoing ones less the stall's constant part.
+
+// Derived per-candidate values (3 x float4), identical for every worker.
+struct __align__(16) CandRec {
+    float a, r, inv_r, U;          // U = -c2/k2 - (r + 1)/2
+    float inv_d1, nXd1, inv_d2, Zc;  // 1/(k2 r + k1), -X(r)/(k2 r + k1), 1/(k2 r), (T_pre - w)/k1
+    int32_t ri, orig, valid, pad;
+};
+
+__device__ __forceinline__ float f_inf() { return __int_as_float(0x7f800000); }
+
+__device__ __forceinline__ long long floor_div_ll(long long x, long long d)
+{
+    long long q = x / d;
+    if ((x % d != 0) && (x < 0)) q -= 1;
+    return q;
+}
+
+__device__ __forceinline__ CandRec make_cand(const DevParams& P, int32_t in, int32_t pred, float w,
+                                             int32_t orig)
+{
+    CandRec c;
+    const bool ok = in >= 0 && pred >= 1 && (long long)in + pred <= (long long)P.K &&
+                    w >= 0.0f && w <= 3.0e38f;
+    const int32_t r = ok ? pred : 1;
+    const float rf = (float)r;
+    c.a = ok ? (float)in : 0.0f;
+    c.r = rf;
+    c.inv_r = 1.0f / rf;
+    c.U = -P.c2_over_k2 - 0.5f * (rf + 1.0f);
+    const float d1 = P.k2 * rf + P.k1;
+    c.inv_d1 = 1.0f / d1;
+    const float X = P.c2 * rf + P.k2 * (0.5f * rf * (rf + 1.0f));
+    c.nXd1 = -X * c.inv_d1;
+    c.inv_d2 = 1.0f / (P.k2 * rf);
+    c.Zc = (P.T_pre - (ok ? w : 0.0f)) * P.inv_k1;
+    c.ri = ok ? r : 0;
+    c.orig = orig;
+    c.valid = ok ? 1 : 0;
+    c.pad = 0;
+    return c;
+}
+
+// Bounds of one pair; returns the four flag bits, writes the margin.
+__device__ __forceinline__ unsigned eval_pair(const float4 v0, const float4 v1, const float4 v2,
+                                              const float4 wr, const CandRec& c, float& margin)
+{
+    const float kv2 = fmaf(c.r, v0.w, v0.z);
+    const float kvm = fminf(v0.y, kv2);
+    const float tt = fminf(fmaf(c.Zc, wr.x, -wr.y), wr.z);
+    const float ca = fmaf(v1.x, c.inv_r, fmaf(v1.z, c.r, c.U - v1.y));
+    const float s1 = fmaf(v2.y, c.inv_d1, c.nXd1);
+    const float s2 = fmaf(v2.z, c.inv_d2, c.U);
+    const float gon = fminf(v1.w, s1);
+    const float gnew = fminf(fminf(v2.x, s2), ca);
+    margin = fminf(fminf(kvm, tt), fminf(gon, gnew)) - c.a;
+    return (kvm >= c.a ? 1u : 0u) | (tt >= c.a ? 2u : 0u) | (gon >= c.a ? 4u : 0u) |
+           (gnew >= c.a ? 8u : 0u);
+}
+
+// Row index p of worker w containing remaining length r: the first row whose
+// rho_{p+1} exceeds r (row R has rho_{R+1} = INT_MAX).
+// NC: read through the read-only path (only for tables not written by the
+// running kernel).
+template <bool NC = true>
+__device__ __forceinline__ int find_row(const float4* tab, long long rowbase, int R, int r)
+{
+    int lo = 0, hi = R;
+    while (lo < hi) {
+        const int mid = (lo + hi) >> 1;
+        const float* px = &tab[(rowbase + mid) * ROW_F4].x;
+        const int nxt = __float_as_int(NC ? __ldg(px) : *px);
+        if (nxt > r) hi = mid;
+        else lo = mid + 1;
+    }
+    return lo;
+}
+
+// ---------------------------------------------------------------------------
+// Warp-level scans over the E x 32 element layout (element x = e * 32 + lane).
+
+template <typename T>
+struct OpMin {
+    __device__ __forceinline__ T operator()(T a, T b) const { return a < b ? a : b; }
+};
+template <typename T>
+struct OpMax {
+    __device__ __forceinline__ T operator()(T a, T b) const { return a > b ? a : b; }
+};
+template <typename T>
+struct OpAdd {
+    __device__ __forceinline__ T operator()(T a, T b) const { return a + b; }
+};
+
+// Inclusive prefix over x; returns the total.
+template <int E, typename T, typename Op>
+__device__ __forceinline__ T scan_prefix(T (&v)[E], Op op, T ident)
+{
+    const int lane = threadIdx.x & 31;
+    T carry = ident;
+#pragma unroll
+    for (int e = 0; e < E; ++e) {
+        T s = v[e];
+#pragma unroll
+        for (int d = 1; d < 32; d <<= 1) {
+            const T u = __shfl_up_sync(FULL, s, d);
+            if (lane >= d) s = op(s, u);
+        }
+        s = op(carry, s);
+        v[e] = s;
+        carry = __shfl_sync(FULL, s, 31);
+    }
+    return carry;
+}
+
+// Exclusive suffix over x (elements y > x); returns the total.
+template <int E, typename T, typename Op>
+__device__ __forceinline__ T scan_suffix_excl(T (&v)[E], Op op, T ident)
+{
+    const int lane = threadIdx.x & 31;
+    T carry = ident;
+#pragma unroll
+    for (int e = E - 1; e >= 0; --e) {
+        T s = v[e];
+#pragma unroll
+        for (int d = 1; d < 32; d <<= 1) {
+            const T u = __shfl_down_sync(FULL, s, d);
+            if (lane + d < 32) s = op(s, u);
+        }
+        T nxt = __shfl_down_sync(FULL, s, 1);
+        if (lane == 31) nxt = ident;
+        const T row_total = __shfl_sync(FULL, s, 0);
+        v[e] = op(nxt, carry);
+        carry = op(carry, row_total);
+    }
+    return carry;
+}
+
+template <typename T, typename Op>
+__device__ __forceinline__ T warp_reduce(T v, Op op)
+{
+#pragma unroll
+    for (int d = 16; d > 0; d >>= 1) v = op(v, __shfl_xor_sync(FULL, v, d));
+    return v;
+}
+
+template <int E>
+struct BuildSmem {
+    long long kvrho[32 * E + 1];
+    int32_t a[32 * E];
+    float bank[32 * E];
+    float Tp[32 * E + 1];
+    uint8_t pend[32 * E];
+};
+
+__device__ __forceinline__ void write_row(const DevParams& P, const ClusterDev& C, long long rowid,
+                                          float s, float inv_s, int M, long long P_pend,
+                                          int rho, int rho_next, int n_p, long long A, long long PR,
+                                          long long PRA, long long PM, long long SM, float pmA,
+                                          float pmAp, float smS, float smSp)
+{
+    float kvB1;
+    if (SM > (long long)M) kvB1 = -f_inf();
+    else if (PM == LL_NONE) kvB1 = f_inf();
+    else kvB1 = (float)floor_div_ll((long long)M - P.j - PM, P.h);
+    const float kvE = (float)(floor_div_ll((long long)M - (long long)P.j * (n_p + 1), P.h) - A);
+    const float nf = (float)n_p;
+    float4 v0, v1, v2;
+    v0.x = __int_as_float(rho_next);
+    v0.y = kvB1;
+    v0.z = kvE;
+    v0.w = -(nf + 1.0f);
+    v1.x = -(P.c2_over_k2 * (float)PR + (float)PRA);
+    v1.y = P.c3_over_k2 + P.c2_over_k2 * nf + (float)A + 0.5f * nf - P.thTdec_over_k2 * inv_s;
+    v1.z = -0.5f * nf;
+    v1.w = pmA;
+    v2.x = pmAp;
+    v2.y = smS * inv_s - (P.k1 * (float)P_pend + P.c1);
+    v2.z = smSp * inv_s;
+    v2.w = __int_as_float(rho);
+    float4* t = C.tab + rowid * ROW_F4;
+    t[0] = v0;
+    t[1] = v1;
+    t[2] = v2;
+    AuxRow ar;
+    ar.PM = PM;
+    ar.SM = SM;
+    ar.A = A;
+    ar.PR = PR;
+    ar.PRA = PRA;
+    ar.n = n_p;
+    ar.rho = rho;
+    C.aux[rowid] = ar;
+    (void)s;
+}
+
+// Build worker w's table (rows 0..R), its record and its capacity_norm key.
+// Called by all 32 lanes of one warp. Requests are loaded from the slot
+// arrays; an invalid request (in < 0, gen outside [0, pred), in + pred > K)
+// makes the worker infeasible for every candidate and sets err bit 1.
+template <int E>
+__device__ void build_table(const DevParams& P, const ClusterDev& C, int w, BuildSmem<E>& sm)
+{
+    const int lane = threadIdx.x & 31;
+    const int n = C.n[w];
+    const long long base = (long long)w * C.cap;
+    const long long rowbase = (long long)w * C.rows;
+    const float s = C.scale[w];
+    const float inv_s = 1.0f / s;
+    const int M = C.M[w];
+
+    unsigned key[E];
+    long long sumP = 0, sumIn = 0, sumPred = 0;
+    float wpmax = -f_inf();
+    int npend = 0;
+    int bad = 0;
+#pragma unroll
+    for (int e = 0; e < E; ++e) {
+        const int i = e * 32 + lane;
+        if (i < n) {
+            const long long slot = base + i;
+            const int pd = C.pend[slot];
+            const int g = pd ? 0 : C.gen[slot];
+            const int pr = C.pred[slot];
+            const int in = C.in[slot];
+            if (in < 0 || g < 0 || g >= pr || (long long)in + pr > (long long)P.K) bad = 1;
+            int r = pr - g;
+            r = r < 1 ? 1 : (r > P.K ? P.K : r);
+            int a = in + g;
+            a = a < 0 ? 0 : (a > P.K ? P.K : a);
+            key[e] = ((unsigned)r << 9) | (unsigned)i;
+            sm.a[i] = a;
+            sm.pend[i] = (uint8_t)pd;
+            sm.bank[i] = pd ? 0.0f : (float)(P.thetad * P.T_decd * (double)g - C.tdec[slot]);
+            sumIn += in;
+            sumPred += pr;
+            if (pd) {
+                sumP += in;
+                wpmax = fmaxf(wpmax, (float)C.wait[slot]);
+                npend += 1;
+            }
+        } else {
+            key[e] = 0xffffffffu;
+        }
+    }
+    sumP = warp_reduce(sumP, OpAdd<long long>());
+    sumIn = warp_reduce(sumIn, OpAdd<long long>());
+    sumPred = warp_reduce(sumPred, OpAdd<long long>());
+    wpmax = warp_reduce(wpmax, OpMax<float>());
+    npend = warp_reduce(npend, OpAdd<int>());
+    bad = __any_sync(FULL, bad);
+    __syncwarp();
+
+    // Bitonic sort of (r, slot) keys, ascending.
+#pragma unroll
+    for (int k = 2; k <= 32 * E; k <<= 1) {
+#pragma unroll
+        for (int jj = k >> 1; jj > 0; jj >>= 1) {
+            if (jj >= 32) {
+                const int je = jj >> 5;
+#pragma unroll
+                for (int e = 0; e < E; ++e) {
+                    if ((e & je) == 0) {
+                        const int e2 = e | je;
+                        const bool asc = ((e * 32 + lane) & k) == 0;
+                        const unsigned lo = min(key[e], key[e2]);
+                        const unsigned hi = max(key[e], key[e2]);
+                        key[e] = asc ? lo : hi;
+                        key[e2] = asc ? hi : lo;
+                    }
+                }
+            } else {
+#pragma unroll
+                for (int e = 0; e < E; ++e) {
+                    const bool asc = ((e * 32 + lane) & k) == 0;
+                    const unsigned v = __shfl_xor_sync(FULL, key[e], jj);
+                    const bool lower = (lane & jj) == 0;
+                    key[e] = (asc == lower) ? min(key[e], v) : max(key[e], v);
+                }
+            }
+        }
+    }
+
+    int r[E], a[E], pd[E];
+    float bank[E];
+#pragma unroll
+    for (int e = 0; e < E; ++e) {
+        const int x = e * 32 + lane;
+        if (x < n) {
+            r[e] = (int)(key[e] >> 9);
+            const int i = (int)(key[e] & 511u);
+            a[e] = sm.a[i];
+            pd[e] = sm.pend[i];
+            bank[e] = sm.bank[i];
+        } else {
+            r[e] = 0x7fffffff;
+            a[e] = 0;
+            pd[e] = 0;
+            bank[e] = 0.0f;
+        }
+    }
+    // Neighbours in sorted order.
+    int rnext[E], first[E], last[E];
+#pragma unroll
+    for (int e = 0; e < E; ++e) {
+        const int dn = __shfl_down_sync(FULL, r[e], 1);
+        const int up = __shfl_up_sync(FULL, r[e], 1);
+        int wrap_n = -1, wrap_p = -1;
+        if (e + 1 < E) wrap_n = __shfl_sync(FULL, r[e + 1 < E ? e + 1 : e], 0);
+        if (e > 0) wrap_p = __shfl_sync(FULL, r[e > 0 ? e - 1 : e], 31);
+        const int nx = lane < 31 ? dn : wrap_n;
+        const int pv = lane > 0 ? up : wrap_p;
+        const int x = e * 32 + lane;
+        const bool valid = x < n;
+        rnext[e] = nx;
+        first[e] = valid && (x == 0 || pv != r[e]);
+        last[e] = valid && (x == n - 1 || nx != r[e]);
+    }
+    // Prefix sums over the sorted order.
+    int rowid[E];
+    long long pre_r[E], pre_ra[E], pre_a[E];
+#pragma unroll
+    for (int e = 0; e < E; ++e) {
+        const bool valid = e * 32 + lane < n;
+        rowid[e] = first[e];
+        const long long rr = valid ? (long long)r[e] : 0;
+        const long long aa = valid ? (long long)a[e] : 0;
+        pre_r[e] = rr;
+        pre_ra[e] = rr * aa + rr * (rr + 1) / 2;
+        pre_a[e] = aa;
+    }
+    const int R = scan_prefix<E>(rowid, OpAdd<int>(), 0);
+    scan_prefix<E>(pre_r, OpAdd<long long>(), 0LL);
+    scan_prefix<E>(pre_ra, OpAdd<long long>(), 0LL);
+    const long long tot_a = scan_prefix<E>(pre_a, OpAdd<long long>(), 0LL);
+
+    // Per-breakpoint KV and cumulative decode time.
+#pragma unroll
+    for (int e = 0; e < E; ++e) {
+        const int x = e * 32 + lane;
+        if (first[e]) {
+            const long long b_at = n - x;
+            const long long Kat = tot_a - (pre_a[e] - a[e]) + (long long)r[e] * b_at;
+            sm.kvrho[rowid[e]] = (long long)P.h * Kat + (long long)P.j * b_at;
+        }
+        if (last[e]) {
+            const long long np = n - (x + 1);
+            const long long A = tot_a - pre_a[e];
+            const long long rr = r[e];
+            const long long Sb = pre_r[e] + rr * np;
+            const long long SK = pre_ra[e] + np * (rr * (rr + 1) / 2) + rr * A;
+            sm.Tp[rowid[e]] = s * (P.c3 * (float)rr + P.c2 * (float)Sb + P.k2 * (float)SK);
+        }
+    }
+    __syncwarp();
+
+    // Per-request bounds and slacks.
+    const float stall0 = s * (P.k1 * (float)sumP + P.c1);
+    float pmA[E], pmAp[E], smS[E], smSp[E];
+    long long PMx[E], SMx[E];
+#pragma unroll
+    for (int e = 0; e < E; ++e) {
+        const int x = e * 32 + lane;
+        const bool valid = x < n;
+        pmA[e] = f_inf();
+        pmAp[e] = f_inf();
+        smS[e] = f_inf();
+        smSp[e] = f_inf();
+        PMx[e] = LL_NONE;
+        SMx[e] = LL_NONE;
+        if (valid) {
+            const float rf = (float)r[e];
+            const float Tj = sm.Tp[rowid[e]];
+            const float sigma = P.theta_Tdec * rf + bank[e] - Tj;
+            const float u = sigma - s * (P.c2 * rf + P.k2 * (0.5f * rf * (rf + 1.0f)));
+            if (pd[e]) {
+                pmAp[e] = u / (s * P.k2 * rf);
+                smSp[e] = sigma;
+            } else {
+                pmA[e] = (u - stall0) / (s * (P.k2 * rf + P.k1));
+                smS[e] = sigma;
+            }
+        }
+        if (last[e]) {
+            const long long kv = sm.kvrho[rowid[e]];
+            PMx[e] = kv + (long long)P.h * r[e];
+            SMx[e] = kv;
+        }
+    }
+    scan_prefix<E>(pmA, OpMin<float>(), f_inf());
+    scan_prefix<E>(pmAp, OpMin<float>(), f_inf());
+    const float smS0 = scan_suffix_excl<E>(smS, OpMin<float>(), f_inf());
+    const float smSp0 = scan_suffix_excl<E>(smSp, OpMin<float>(), f_inf());
+    scan_prefix<E>(PMx, OpMax<long long>(), LL_NONE);
+    const long long SM0 = scan_suffix_excl<E>(SMx, OpMax<long long>(), LL_NONE);
+
+    if (!bad) {
+#pragma unroll
+        for (int e = 0; e < E; ++e) {
+            if (last[e]) {
+                const int x = e * 32 + lane;
+                const int np = n - (x + 1);
+                const long long A = tot_a - pre_a[e];
+                const int nxt = (x == n - 1) ? 0x7fffffff : rnext[e];
+                const long long SM = SMx[e] == LL_NONE ? 0 : SMx[e];
+                write_row(P, C, rowbase + rowid[e], s, inv_s, M, sumP, r[e], nxt, np, A,
+                          pre_r[e], pre_ra[e], PMx[e], SM, pmA[e], pmAp[e], smS[e], smSp[e]);
+            }
+        }
+    }
+    if (lane == 0) {
+        if (!bad) {
+            write_row(P, C, rowbase, s, inv_s, M, sumP, 0, n > 0 ? r[0] : 0x7fffffff, n, tot_a, 0,
+                      0, LL_NONE, SM0 == LL_NONE ? 0 : SM0, f_inf(), f_inf(), smS0, smSp0);
+            C.R[w] = R;
+        } else {
+            // An invalid request: no candidate fits this worker.
+            write_row(P, C, rowbase, s, inv_s, M, 0, 0, 0x7fffffff, 0, 0, 0, 0, LL_NONE,
+                      (long long)M + 1, f_inf(), f_inf(), f_inf(), f_inf());
+            C.R[w] = 0;
+            atomicOr(C.err, 1u);
+        }
+        const float off = C.off[w];
+        const float ZO = off * inv_s * P.inv_k1 + P.c1_over_k1 + (float)sumP;
+        const float ZW = npend > 0 ? (P.T_pre - wpmax - off) * inv_s * P.inv_k1 - P.c1_over_k1 -
+                                         (float)sumP
+                                   : f_inf();
+        float4 wr = C.wrec[w];
+        wr.x = inv_s;
+        wr.y = ZO;
+        wr.z = ZW;
+        C.wrec[w] = wr;
+        const double B = (double)n;
+        const double L = __dadd_rn((double)sumIn, __dmul_rn(P.gammad, (double)sumPred));
+        C.key[w] = bad ? -1.0 : __dadd_rn(__dmul_rn(B, B), __dmul_rn(L, L));
+    }
+    __syncwarp();
+}
+
+}  // namespace aladdin

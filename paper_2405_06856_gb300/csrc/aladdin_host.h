@@ -1,0 +1,64 @@
+// Host-side internals shared by the library's translation units.
+#pragma once
+
+#include <cuda_runtime.h>
+
+#include "aladdin_dev.cuh"
+
+namespace aladdin {
+
+// Elements per lane of the per-warp table builder for a slot capacity.
+inline int lanes_per_worker(int cap) { return cap / 32; }
+
+// K2: rebuild the tables of `count` workers (all workers when list == nullptr).
+cudaError_t launch_build(const DevParams& P, const ClusterDev& C, const int32_t* list, int count,
+                         cudaStream_t st);
+// capacity_norm ranks (descending key, lowest index on ties) and rank -> worker.
+cudaError_t launch_rank(const ClusterDev& C, cudaStream_t st);
+
+struct ScoreBuffers {
+    CandRec* sorted;       // [n_cand]
+    int32_t* hist;         // [K + 2]
+    unsigned int* best;    // [n_cand]
+};
+
+// K3 pipeline: validate + derive + counting-sort candidates by predicted
+// output, score every pair, finalize argbest. Device pointers only.
+cudaError_t launch_score(const DevParams& P, const ClusterDev& C, int n_cand, const int32_t* in,
+                         const int32_t* pred, const float* wait, uint8_t* flags, float* margin,
+                         int32_t* argbest, int64_t* kv_peak, float* t_cand, const ScoreBuffers& B,
+                         cudaStream_t st, cudaEvent_t ev0 = nullptr, cudaEvent_t ev1 = nullptr);
+
+// K4: one greedy round over candidates in index order.
+struct RoundIO {
+    // direct mode
+    const int32_t* in;
+    const int32_t* pred;
+    const float* wait;
+    int n_cand;
+    int32_t* placement;
+    // trace mode (fleet simulation): candidates = waiting list then arrivals
+    int sim;
+    const double* t_arr;
+    const int32_t* tin;
+    const int32_t* tpred;
+    long long* wl;           // waiting list (trace indices), rewritten in place
+    int* n_wait;             // device
+    long long arr_begin, arr_end;
+    double t_now, H;
+    unsigned long long* counters;  // [0] failed, [1] placed, [2] heartbeat of the halt
+    int* status;             // device: 0 ok, 1 halted at the first failure, -2 capacity
+    int stop_at_fail;
+    long long hb;
+};
+cudaError_t launch_round(const DevParams& P, const ClusterDev& C, const RoundIO& io,
+                         cudaStream_t st);
+
+// Execution of every worker for dt ms from t_now.
+// stats: device [0] prefills run, [1] finished, [2] max TTFT bits, [3] max
+// ATGT bits (non-negative doubles compare like their bit patterns). halt
+// (device, nullable): nothing runs when *halt != 0.
+cudaError_t launch_advance(const DevParams& P, const ClusterDev& C, double t_now, double dt,
+                           unsigned long long* stats, const int* halt, cudaStream_t st);
+
+}  // namespace aladdin

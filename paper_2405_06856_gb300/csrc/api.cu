@@ -1,0 +1,854 @@
+// C ABI of the library (include/aladdin.h): cluster object, pointer
+// classification and staging, host-side validation, and the heartbeat loop of
+// the fleet simulation and minimum-worker search.
+#include <cmath>
+#include <cstring>
+#include <new>
+#include <vector>
+
+#include "../../include/aladdin.h"
+#include "aladdin_host.h"
+
+using namespace aladdin;
+
+namespace {
+
+struct DevBuf {
+    void* p = nullptr;
+    size_t bytes = 0;
+    cudaError_t ensure(size_t need)
+    {
+        if (need <= bytes) return cudaSuccess;
+        if (p) cudaFree(p);
+        p = nullptr;
+        bytes = 0;
+        size_t cap = need < 4096 ? 4096 : need + need / 4;
+        cudaError_t e = cudaMalloc(&p, cap);
+        if (e == cudaSuccess) bytes = cap;
+        return e;
+    }
+    void release()
+    {
+        if (p) cudaFree(p);
+        p = nullptr;
+        bytes = 0;
+    }
+    template <typename T>
+    T* as() const { return reinterpret_cast<T*>(p); }
+};
+
+enum PtrKind { PK_NULL = 0, PK_HOST = 1, PK_DEV = 2 };
+
+PtrKind ptr_kind(const void* p)
+{
+    if (!p) return PK_NULL;
+    cudaPointerAttributes a;
+    cudaError_t e = cudaPointerGetAttributes(&a, p);
+    if (e != cudaSuccess) {
+        cudaGetLastError();
+        return PK_HOST;
+    }
+    if (a.type == cudaMemoryTypeDevice || a.type == cudaMemoryTypeManaged) return PK_DEV;
+    return PK_HOST;
+}
+
+bool finite_nonneg(double x) { return std::isfinite(x) && x >= 0.0; }
+
+int check_params(const aladdin_params* p)
+{
+    if (!p) return ALADDIN_ERR_ARG;
+    if (!(std::isfinite(p->k1) && p->k1 > 0 && std::isfinite(p->k2) && p->k2 > 0)) return ALADDIN_ERR_ARG;
+    if (!(finite_nonneg(p->c1) && finite_nonneg(p->c2) && finite_nonneg(p->c3))) return ALADDIN_ERR_ARG;
+    if (p->h < 1 || p->j < 0) return ALADDIN_ERR_ARG;
+    if (!(std::isfinite(p->T_pre) && p->T_pre > 0)) return ALADDIN_ERR_ARG;
+    if (!(std::isfinite(p->T_dec) && p->T_dec > p->c3)) return ALADDIN_ERR_ARG;
+    if (!(std::isfinite(p->theta) && p->theta > 0 && p->theta <= 1)) return ALADDIN_ERR_ARG;
+    if (!finite_nonneg(p->gamma)) return ALADDIN_ERR_ARG;
+    if (p->K < 2 || p->K > 65536) return ALADDIN_ERR_ARG;
+    const int b = p->b_cap;
+    if (!(b == 32 || b == 64 || b == 128 || b == 256 || b == 512)) return ALADDIN_ERR_ARG;
+    return ALADDIN_OK;
+}
+
+int check_cfg(const aladdin_worker_cfg& c)
+{
+    if (c.gpus < 1) return ALADDIN_ERR_ARG;
+    if (c.kv_capacity < 0 || c.kv_capacity >= (1LL << 24)) return ALADDIN_ERR_ARG;
+    if (!(std::isfinite(c.lat_scale) && c.lat_scale > 0)) return ALADDIN_ERR_ARG;
+    return ALADDIN_OK;
+}
+
+DevParams make_devparams(const aladdin_params& p)
+{
+    DevParams d;
+    d.k1 = (float)p.k1;
+    d.c1 = (float)p.c1;
+    d.k2 = (float)p.k2;
+    d.c2 = (float)p.c2;
+    d.c3 = (float)p.c3;
+    d.h = p.h;
+    d.j = p.j;
+    d.T_pre = (float)p.T_pre;
+    d.T_dec = (float)p.T_dec;
+    d.gamma = (float)p.gamma;
+    d.theta = (float)p.theta;
+    d.K = p.K;
+    d.cap = p.b_cap;
+    d.c2_over_k2 = (float)(p.c2 / p.k2);
+    d.c3_over_k2 = (float)(p.c3 / p.k2);
+    d.c1_over_k1 = (float)(p.c1 / p.k1);
+    d.inv_k1 = (float)(1.0 / p.k1);
+    d.theta_Tdec = (float)(p.theta * p.T_dec);
+    d.thTdec_over_k2 = (float)(p.theta * p.T_dec / p.k2);
+    d.k1d = p.k1;
+    d.c1d = p.c1;
+    d.k2d = p.k2;
+    d.c2d = p.c2;
+    d.c3d = p.c3;
+    d.T_pred = p.T_pre;
+    d.T_decd = p.T_dec;
+    d.gammad = p.gamma;
+    d.thetad = p.theta;
+    return d;
+}
+
+}  // namespace
+
+struct aladdin_cluster {
+    int device = 0;
+    cudaStream_t st = nullptr;
+    aladdin_params hp;
+    DevParams dp;
+    ClusterDev dev;
+    int W = 0, cap = 0, rows = 0;
+    double t_now = 0.0;
+    std::vector<void*> owned;
+    // scratch and staging (grow-only)
+    DevBuf sorted, hist, best;
+    DevBuf s_in, s_pred, s_wait, s_flags, s_margin, s_arg, s_kv, s_tc, s_place;
+    DevBuf s_off, s_rin, s_rgen, s_rpred, s_rtdec;
+    unsigned long long* d_stats = nullptr;
+    int* d_status = nullptr;
+    // optional CUDA-event timing of the scoring kernel
+    bool timing = false;
+    std::vector<cudaEvent_t> ev;   // pairs (start, stop)
+    std::vector<cudaEvent_t> ev_free;
+
+    cudaError_t alloc(void** p, size_t bytes)
+    {
+        cudaError_t e = cudaMalloc(p, bytes);
+        if (e == cudaSuccess) owned.push_back(*p);
+        return e;
+    }
+    void clear_events()
+    {
+        for (cudaEvent_t e : ev) ev_free.push_back(e);
+        ev.clear();
+    }
+    cudaEvent_t take_event()
+    {
+        if (!ev_free.empty()) {
+            cudaEvent_t e = ev_free.back();
+            ev_free.pop_back();
+            return e;
+        }
+        cudaEvent_t e = nullptr;
+        if (cudaEventCreate(&e) != cudaSuccess) return nullptr;
+        return e;
+    }
+    ~aladdin_cluster()
+    {
+        clear_events();
+        for (cudaEvent_t e : ev_free) cudaEventDestroy(e);
+        for (void* p : owned) cudaFree(p);
+        DevBuf* bufs[] = {&sorted, &hist, &best, &s_in, &s_pred, &s_wait, &s_flags, &s_margin,
+                          &s_arg, &s_kv, &s_tc, &s_place, &s_off, &s_rin, &s_rgen, &s_rpred,
+                          &s_rtdec};
+        for (DevBuf* b : bufs) b->release();
+    }
+};
+
+namespace {
+
+#define CK(x)                                  \
+    do {                                       \
+        cudaError_t e_ = (x);                  \
+        if (e_ != cudaSuccess) {               \
+            cudaGetLastError();                \
+            return ALADDIN_ERR_CUDA;           \
+        }                                      \
+    } while (0)
+
+// Allocate the device state of a cluster with W empty workers.
+int cluster_alloc(aladdin_cluster* cl, const aladdin_params& p, int W,
+                  const aladdin_worker_cfg* cfg, cudaStream_t st)
+{
+    cl->hp = p;
+    cl->dp = make_devparams(p);
+    cl->W = W;
+    cl->cap = p.b_cap;
+    cl->rows = p.b_cap + 1;
+    cl->st = st;
+    CK(cudaGetDevice(&cl->device));
+    ClusterDev& d = cl->dev;
+    d.W = W;
+    d.cap = cl->cap;
+    d.rows = cl->rows;
+    const size_t slots = (size_t)W * cl->cap, rows = (size_t)W * cl->rows;
+    void* p0;
+#define AL(field, type, count)                                           \
+    CK(cl->alloc(&p0, sizeof(type) * (count)));                          \
+    d.field = reinterpret_cast<type*>(p0);
+    float* scale;
+    double* scaled;
+    int32_t* M;
+    CK(cl->alloc(&p0, sizeof(float) * W)); scale = (float*)p0;
+    CK(cl->alloc(&p0, sizeof(double) * W)); scaled = (double*)p0;
+    CK(cl->alloc(&p0, sizeof(int32_t) * W)); M = (int32_t*)p0;
+    d.scale = scale;
+    d.scaled = scaled;
+    d.M = M;
+    AL(off, float, W);
+    AL(clock, double, W);
+    AL(n, int32_t, W);
+    AL(in, int32_t, slots);
+    AL(gen, int32_t, slots);
+    AL(pred, int32_t, slots);
+    AL(tdec, double, slots);
+    AL(pend, uint8_t, slots);
+    AL(wait, double, slots);
+    AL(tab, float4, rows * ROW_F4);
+    AL(aux, AuxRow, rows);
+    AL(R, int32_t, W);
+    AL(wrec, float4, W);
+    AL(key, double, W);
+    AL(rank, int32_t, W);
+    AL(order, int32_t, W);
+    AL(err, unsigned int, 1);
+#undef AL
+    CK(cl->alloc(&p0, sizeof(unsigned long long) * 4)); cl->d_stats = (unsigned long long*)p0;
+    CK(cl->alloc(&p0, sizeof(int) * 4)); cl->d_status = (int*)p0;
+
+    std::vector<float> hs(W);
+    std::vector<double> hsd(W);
+    std::vector<int32_t> hM(W);
+    for (int w = 0; w < W; ++w) {
+        hs[w] = (float)cfg[w].lat_scale;
+        hsd[w] = cfg[w].lat_scale;
+        hM[w] = (int32_t)cfg[w].kv_capacity;
+    }
+    CK(cudaMemcpyAsync(scale, hs.data(), sizeof(float) * W, cudaMemcpyHostToDevice, st));
+    CK(cudaMemcpyAsync(scaled, hsd.data(), sizeof(double) * W, cudaMemcpyHostToDevice, st));
+    CK(cudaMemcpyAsync(M, hM.data(), sizeof(int32_t) * W, cudaMemcpyHostToDevice, st));
+    CK(cudaMemsetAsync(d.off, 0, sizeof(float) * W, st));
+    CK(cudaMemsetAsync(d.clock, 0, sizeof(double) * W, st));
+    CK(cudaMemsetAsync(d.n, 0, sizeof(int32_t) * W, st));
+    CK(cudaMemsetAsync(d.pend, 0, slots, st));
+    CK(cudaMemsetAsync(d.wrec, 0, sizeof(float4) * W, st));
+    CK(cudaMemsetAsync(d.err, 0, sizeof(unsigned int), st));
+    CK(cudaMemsetAsync(cl->d_stats, 0, sizeof(unsigned long long) * 4, st));
+    CK(cudaMemsetAsync(cl->d_status, 0, sizeof(int) * 4, st));
+    // host vectors above must outlive the async copies
+    CK(cudaStreamSynchronize(st));
+    return ALADDIN_OK;
+}
+
+int refresh_tables(aladdin_cluster* cl)
+{
+    CK(launch_build(cl->dp, cl->dev, nullptr, cl->W, cl->st));
+    CK(launch_rank(cl->dev, cl->st));
+    return ALADDIN_OK;
+}
+
+// Copy count elements of a caller array to host memory.
+template <typename T>
+int fetch_host(const T* src, size_t count, std::vector<T>& dst)
+{
+    dst.resize(count);
+    if (count == 0) return ALADDIN_OK;
+    if (ptr_kind(src) == PK_DEV) {
+        CK(cudaMemcpy(dst.data(), src, sizeof(T) * count, cudaMemcpyDeviceToHost));
+    } else {
+        std::memcpy(dst.data(), src, sizeof(T) * count);
+    }
+    return ALADDIN_OK;
+}
+
+// Load requests given in CSR form (host path: validate + pack on the host).
+int load_requests_host(aladdin_cluster* cl, const int32_t* req_off, const int32_t* in,
+                       const int32_t* gen, const int32_t* pred, const float* tdec)
+{
+    const int W = cl->W, cap = cl->cap;
+    std::vector<int32_t> off;
+    int rc = fetch_host(req_off, (size_t)W + 1, off);
+    if (rc) return rc;
+    if (off[0] != 0) return ALADDIN_ERR_ARG;
+    for (int w = 0; w < W; ++w) {
+        if (off[w + 1] < off[w]) return ALADDIN_ERR_ARG;
+        if (off[w + 1] - off[w] > cap) return ALADDIN_ERR_CAPACITY;
+    }
+    const size_t N = (size_t)off[W];
+    if (N > 0 && (!in || !gen || !pred)) return ALADDIN_ERR_ARG;
+    std::vector<int32_t> vin, vgen, vpred;
+    std::vector<float> vt;
+    if ((rc = fetch_host(in, N, vin)) || (rc = fetch_host(gen, N, vgen)) ||
+        (rc = fetch_host(pred, N, vpred)))
+        return rc;
+    if (tdec && (rc = fetch_host(tdec, N, vt))) return rc;
+    const aladdin_params& p = cl->hp;
+    for (size_t i = 0; i < N; ++i) {
+        if (vin[i] < 0 || vgen[i] < 0 || vgen[i] >= vpred[i] ||
+            (long long)vin[i] + vpred[i] > (long long)p.K)
+            return ALADDIN_ERR_ARG;
+        if (tdec && !(std::isfinite(vt[i]) && vt[i] >= 0)) return ALADDIN_ERR_ARG;
+    }
+    const size_t slots = (size_t)W * cap;
+    std::vector<int32_t> si(slots, 0), sg(slots, 0), sp(slots, 1), sn(W);
+    std::vector<double> stdec(slots, 0.0);
+    for (int w = 0; w < W; ++w) {
+        sn[w] = off[w + 1] - off[w];
+        for (int q = 0; q < sn[w]; ++q) {
+            const size_t src = (size_t)off[w] + q, dst = (size_t)w * cap + q;
+            si[dst] = vin[src];
+            sg[dst] = vgen[src];
+            sp[dst] = vpred[src];
+            stdec[dst] = tdec ? (double)vt[src] : p.theta * p.T_dec * (double)vgen[src];
+        }
+    }
+    ClusterDev& d = cl->dev;
+    CK(cudaMemcpyAsync(d.n, sn.data(), sizeof(int32_t) * W, cudaMemcpyHostToDevice, cl->st));
+    CK(cudaMemcpyAsync(d.in, si.data(), sizeof(int32_t) * slots, cudaMemcpyHostToDevice, cl->st));
+    CK(cudaMemcpyAsync(d.gen, sg.data(), sizeof(int32_t) * slots, cudaMemcpyHostToDevice, cl->st));
+    CK(cudaMemcpyAsync(d.pred, sp.data(), sizeof(int32_t) * slots, cudaMemcpyHostToDevice, cl->st));
+    CK(cudaMemcpyAsync(d.tdec, stdec.data(), sizeof(double) * slots, cudaMemcpyHostToDevice, cl->st));
+    CK(cudaMemsetAsync(d.pend, 0, slots, cl->st));
+    CK(cudaStreamSynchronize(cl->st));
+    return ALADDIN_OK;
+}
+
+// Device path: pack CSR requests into slots on the GPU (one warp per worker);
+// a worker whose request count exceeds the slots or that holds an invalid
+// request is replaced by a single invalid request so that the table builder
+// marks it infeasible and records the error.
+__global__ void k_pack(DevParams P, ClusterDev C, const int32_t* __restrict__ off,
+                       const int32_t* __restrict__ in, const int32_t* __restrict__ gen,
+                       const int32_t* __restrict__ pred, const float* __restrict__ tdec)
+{
+    const int lane = threadIdx.x & 31;
+    const int w = blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
+    if (w >= C.W) return;
+    const int a = off[w], b = off[w + 1];
+    const long long base = (long long)w * C.cap;
+    int n = b - a;
+    const bool over = n < 0 || n > C.cap;
+    if (over) n = 0;
+    for (int q = lane; q < n; q += 32) {
+        const long long dst = base + q;
+        const int g = gen[a + q];
+        C.in[dst] = in[a + q];
+        C.gen[dst] = g;
+        C.pred[dst] = pred[a + q];
+        C.tdec[dst] = tdec ? (double)tdec[a + q] : P.thetad * P.T_decd * (double)g;
+        C.pend[dst] = 0;
+    }
+    if (lane == 0) {
+        if (over) {
+            C.in[base] = -1;
+            C.gen[base] = 0;
+            C.pred[base] = 1;
+            C.tdec[base] = 0.0;
+            C.pend[base] = 0;
+            atomicOr(C.err, 2u);
+        }
+        C.n[w] = over ? 1 : n;
+    }
+}
+
+int load_requests(aladdin_cluster* cl, const int32_t* req_off, const int32_t* in,
+                  const int32_t* gen, const int32_t* pred, const float* tdec)
+{
+    if (!req_off) return ALADDIN_ERR_ARG;
+    const bool dev = ptr_kind(req_off) == PK_DEV && (!in || ptr_kind(in) == PK_DEV) &&
+                     (!gen || ptr_kind(gen) == PK_DEV) && (!pred || ptr_kind(pred) == PK_DEV) &&
+                     (!tdec || ptr_kind(tdec) == PK_DEV);
+    if (!dev) return load_requests_host(cl, req_off, in, gen, pred, tdec);
+    if (!in || !gen || !pred) return ALADDIN_ERR_ARG;
+    const int wpb = 4;
+    k_pack<<<(cl->W + wpb - 1) / wpb, 32 * wpb, 0, cl->st>>>(cl->dp, cl->dev, req_off, in, gen,
+                                                             pred, tdec);
+    CK(cudaGetLastError());
+    return ALADDIN_OK;
+}
+
+// Stage an input array on the device: returns a device pointer.
+template <typename T>
+int stage_in(aladdin_cluster* cl, DevBuf& buf, const T* src, size_t count, const T** out)
+{
+    if (!src) {
+        *out = nullptr;
+        return ALADDIN_OK;
+    }
+    if (ptr_kind(src) == PK_DEV) {
+        *out = src;
+        return ALADDIN_OK;
+    }
+    CK(buf.ensure(sizeof(T) * count));
+    CK(cudaMemcpyAsync(buf.p, src, sizeof(T) * count, cudaMemcpyHostToDevice, cl->st));
+    *out = buf.as<T>();
+    return ALADDIN_OK;
+}
+
+template <typename T>
+int stage_out(DevBuf& buf, T* dst, size_t count, T** out, bool* host)
+{
+    *host = false;
+    if (!dst) {
+        *out = nullptr;
+        return ALADDIN_OK;
+    }
+    if (ptr_kind(dst) == PK_DEV) {
+        *out = dst;
+        return ALADDIN_OK;
+    }
+    CK(buf.ensure(sizeof(T) * count));
+    *out = buf.as<T>();
+    *host = true;
+    return ALADDIN_OK;
+}
+
+int score_impl(aladdin_cluster* cl, int32_t n, const int32_t* in, const int32_t* pred,
+               const float* wait, uint8_t* flags, float* margin, int32_t* argbest,
+               int64_t* kv_peak, float* t_cand)
+{
+    if (!cl || n < 0) return ALADDIN_ERR_ARG;
+    if (n == 0) return ALADDIN_OK;
+    if (!in || !pred) return ALADDIN_ERR_ARG;
+    CK(cudaSetDevice(cl->device));
+    const size_t C = (size_t)n, pairs = C * (size_t)cl->W;
+    const int32_t *din, *dpred;
+    const float* dwait;
+    int rc;
+    if ((rc = stage_in(cl, cl->s_in, in, C, &din)) || (rc = stage_in(cl, cl->s_pred, pred, C, &dpred)) ||
+        (rc = stage_in(cl, cl->s_wait, wait, C, &dwait)))
+        return rc;
+    uint8_t* dflags;
+    float *dmargin, *dtc;
+    int32_t* darg;
+    int64_t* dkv;
+    bool hf, hm, ha, hk, ht;
+    if ((rc = stage_out(cl->s_flags, flags, pairs, &dflags, &hf)) ||
+        (rc = stage_out(cl->s_margin, margin, pairs, &dmargin, &hm)) ||
+        (rc = stage_out(cl->s_arg, argbest, C, &darg, &ha)) ||
+        (rc = stage_out(cl->s_kv, kv_peak, pairs, &dkv, &hk)) ||
+        (rc = stage_out(cl->s_tc, t_cand, pairs, &dtc, &ht)))
+        return rc;
+    CK(cl->sorted.ensure(sizeof(CandRec) * C));
+    CK(cl->hist.ensure(sizeof(int32_t) * ((size_t)cl->hp.K + 2)));
+    CK(cl->best.ensure(sizeof(unsigned int) * C));
+    ScoreBuffers B{cl->sorted.as<CandRec>(), cl->hist.as<int32_t>(), cl->best.as<unsigned int>()};
+    cudaEvent_t e0 = nullptr, e1 = nullptr;
+    if (cl->timing && (dflags || dmargin || darg)) {
+        e0 = cl->take_event();
+        e1 = cl->take_event();
+        if (e0 && e1) {
+            cl->ev.push_back(e0);
+            cl->ev.push_back(e1);
+        } else {
+            e0 = e1 = nullptr;
+        }
+    }
+    CK(launch_score(cl->dp, cl->dev, n, din, dpred, dwait, dflags, dmargin, darg, dkv, dtc, B, cl->st,
+                    e0, e1));
+    if (hf) CK(cudaMemcpyAsync(flags, dflags, pairs, cudaMemcpyDeviceToHost, cl->st));
+    if (hm) CK(cudaMemcpyAsync(margin, dmargin, sizeof(float) * pairs, cudaMemcpyDeviceToHost, cl->st));
+    if (ha) CK(cudaMemcpyAsync(argbest, darg, sizeof(int32_t) * C, cudaMemcpyDeviceToHost, cl->st));
+    if (hk) CK(cudaMemcpyAsync(kv_peak, dkv, sizeof(int64_t) * pairs, cudaMemcpyDeviceToHost, cl->st));
+    if (ht) CK(cudaMemcpyAsync(t_cand, dtc, sizeof(float) * pairs, cudaMemcpyDeviceToHost, cl->st));
+    // host inputs were staged asynchronously from caller memory: complete
+    // before returning whenever host memory is involved
+    const bool any_host = hf || hm || ha || hk || ht || ptr_kind(in) == PK_HOST ||
+                          ptr_kind(pred) == PK_HOST || (wait && ptr_kind(wait) == PK_HOST);
+    if (any_host) CK(cudaStreamSynchronize(cl->st));
+    return ALADDIN_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+int aladdin_cluster_create(const aladdin_params* params, int32_t n_workers,
+                           const aladdin_worker_cfg* cfg, const int32_t* req_off,
+                           const int32_t* in, const int32_t* gen, const int32_t* pred,
+                           const float* tdec_ms, void* cuda_stream, aladdin_cluster** out)
+{
+    if (!out) return ALADDIN_ERR_ARG;
+    *out = nullptr;
+    int rc = check_params(params);
+    if (rc) return rc;
+    if (n_workers < 1 || !cfg || !req_off) return ALADDIN_ERR_ARG;
+    std::vector<aladdin_worker_cfg> hc;
+    if ((rc = fetch_host(cfg, (size_t)n_workers, hc))) return rc;
+    for (int w = 0; w < n_workers; ++w)
+        if ((rc = check_cfg(hc[w]))) return rc;
+    aladdin_cluster* cl = new (std::nothrow) aladdin_cluster();
+    if (!cl) return ALADDIN_ERR_NOMEM;
+    rc = cluster_alloc(cl, *params, n_workers, hc.data(), (cudaStream_t)cuda_stream);
+    if (!rc) rc = load_requests_host(cl, req_off, in, gen, pred, tdec_ms);
+    if (!rc) rc = refresh_tables(cl);
+    if (!rc && cudaStreamSynchronize(cl->st) != cudaSuccess) rc = ALADDIN_ERR_CUDA;
+    if (rc) {
+        delete cl;
+        return rc == ALADDIN_ERR_CUDA && cudaGetLastError() == cudaErrorMemoryAllocation
+                   ? ALADDIN_ERR_NOMEM
+                   : rc;
+    }
+    *out = cl;
+    return ALADDIN_OK;
+}
+
+int aladdin_cluster_destroy(aladdin_cluster* cl)
+{
+    if (!cl) return ALADDIN_ERR_ARG;
+    cudaSetDevice(cl->device);
+    cudaStreamSynchronize(cl->st);
+    delete cl;
+    return ALADDIN_OK;
+}
+
+int aladdin_cluster_load(aladdin_cluster* cl, const int32_t* req_off, const int32_t* in,
+                         const int32_t* gen, const int32_t* pred, const float* tdec_ms)
+{
+    if (!cl) return ALADDIN_ERR_ARG;
+    CK(cudaSetDevice(cl->device));
+    int rc = load_requests(cl, req_off, in, gen, pred, tdec_ms);
+    if (rc) return rc;
+    return refresh_tables(cl);
+}
+
+int aladdin_score(aladdin_cluster* cl, int32_t n_cand, const int32_t* in, const int32_t* pred,
+                  const float* wait_ms, uint8_t* flags, float* margin, int32_t* argbest)
+{
+    return score_impl(cl, n_cand, in, pred, wait_ms, flags, margin, argbest, nullptr, nullptr);
+}
+
+int aladdin_score_detail(aladdin_cluster* cl, int32_t n_cand, const int32_t* in,
+                         const int32_t* pred, const float* wait_ms, uint8_t* flags,
+                         float* margin, int32_t* argbest, int64_t* kv_peak, float* t_cand_ms)
+{
+    return score_impl(cl, n_cand, in, pred, wait_ms, flags, margin, argbest, kv_peak, t_cand_ms);
+}
+
+int aladdin_place_round(aladdin_cluster* cl, int32_t n_cand, const int32_t* in,
+                        const int32_t* pred, const float* wait_ms, int32_t* placement)
+{
+    if (!cl || n_cand < 0) return ALADDIN_ERR_ARG;
+    if (n_cand == 0) return ALADDIN_OK;
+    if (!in || !pred || !placement) return ALADDIN_ERR_ARG;
+    CK(cudaSetDevice(cl->device));
+    const size_t C = (size_t)n_cand;
+    const int32_t *din, *dpred;
+    const float* dwait;
+    int rc;
+    if ((rc = stage_in(cl, cl->s_in, in, C, &din)) || (rc = stage_in(cl, cl->s_pred, pred, C, &dpred)) ||
+        (rc = stage_in(cl, cl->s_wait, wait_ms, C, &dwait)))
+        return rc;
+    int32_t* dpl;
+    bool hp;
+    if ((rc = stage_out(cl->s_place, placement, C, &dpl, &hp))) return rc;
+    CK(cudaMemsetAsync(cl->d_status, 0, sizeof(int), cl->st));
+    RoundIO io;
+    std::memset(&io, 0, sizeof(io));
+    io.in = din;
+    io.pred = dpred;
+    io.wait = dwait;
+    io.n_cand = n_cand;
+    io.placement = dpl;
+    io.sim = 0;
+    io.status = cl->d_status;
+    CK(launch_round(cl->dp, cl->dev, io, cl->st));
+    CK(launch_rank(cl->dev, cl->st));
+    if (hp) CK(cudaMemcpyAsync(placement, dpl, sizeof(int32_t) * C, cudaMemcpyDeviceToHost, cl->st));
+    int status = 0;
+    CK(cudaMemcpyAsync(&status, cl->d_status, sizeof(int), cudaMemcpyDeviceToHost, cl->st));
+    CK(cudaStreamSynchronize(cl->st));
+    return status == -2 ? ALADDIN_ERR_CAPACITY : ALADDIN_OK;
+}
+
+int aladdin_cluster_advance(aladdin_cluster* cl, double dt_ms, double* stats)
+{
+    if (!cl || !(std::isfinite(dt_ms) && dt_ms >= 0)) return ALADDIN_ERR_ARG;
+    CK(cudaSetDevice(cl->device));
+    CK(launch_advance(cl->dp, cl->dev, cl->t_now, dt_ms, cl->d_stats, nullptr, cl->st));
+    cl->t_now += dt_ms;
+    int rc = refresh_tables(cl);
+    if (rc) return rc;
+    if (stats) {
+        unsigned long long s[4];
+        CK(cudaMemcpyAsync(s, cl->d_stats, sizeof(s), cudaMemcpyDeviceToHost, cl->st));
+        CK(cudaStreamSynchronize(cl->st));
+        stats[0] = (double)s[0];
+        stats[1] = (double)s[1];
+        double a, b;
+        std::memcpy(&a, &s[2], 8);
+        std::memcpy(&b, &s[3], 8);
+        stats[2] = a;
+        stats[3] = b;
+    }
+    return ALADDIN_OK;
+}
+
+int aladdin_cluster_state(aladdin_cluster* cl, int32_t* n, int32_t* in, int32_t* gen,
+                          int32_t* pred, uint8_t* pending)
+{
+    if (!cl) return ALADDIN_ERR_ARG;
+    CK(cudaSetDevice(cl->device));
+    const size_t slots = (size_t)cl->W * cl->cap;
+    const ClusterDev& d = cl->dev;
+    if (n) CK(cudaMemcpyAsync(n, d.n, sizeof(int32_t) * cl->W, cudaMemcpyDeviceToHost, cl->st));
+    if (in) CK(cudaMemcpyAsync(in, d.in, sizeof(int32_t) * slots, cudaMemcpyDeviceToHost, cl->st));
+    if (gen) CK(cudaMemcpyAsync(gen, d.gen, sizeof(int32_t) * slots, cudaMemcpyDeviceToHost, cl->st));
+    if (pred) CK(cudaMemcpyAsync(pred, d.pred, sizeof(int32_t) * slots, cudaMemcpyDeviceToHost, cl->st));
+    if (pending) CK(cudaMemcpyAsync(pending, d.pend, slots, cudaMemcpyDeviceToHost, cl->st));
+    CK(cudaStreamSynchronize(cl->st));
+    return ALADDIN_OK;
+}
+
+int aladdin_cluster_timing(aladdin_cluster* cl, int32_t enable, double* kernel_ms,
+                           int64_t* launches)
+{
+    if (!cl) return ALADDIN_ERR_ARG;
+    CK(cudaSetDevice(cl->device));
+    CK(cudaStreamSynchronize(cl->st));
+    double total = 0.0;
+    for (size_t i = 0; i + 1 < cl->ev.size(); i += 2) {
+        float ms = 0.0f;
+        CK(cudaEventElapsedTime(&ms, cl->ev[i], cl->ev[i + 1]));
+        total += ms;
+    }
+    if (kernel_ms) *kernel_ms = total;
+    if (launches) *launches = (int64_t)(cl->ev.size() / 2);
+    cl->clear_events();
+    cl->timing = enable != 0;
+    return ALADDIN_OK;
+}
+
+int aladdin_cluster_status(aladdin_cluster* cl)
+{
+    if (!cl) return ALADDIN_ERR_ARG;
+    CK(cudaSetDevice(cl->device));
+    unsigned int err = 0;
+    CK(cudaMemcpyAsync(&err, cl->dev.err, sizeof(err), cudaMemcpyDeviceToHost, cl->st));
+    CK(cudaStreamSynchronize(cl->st));
+    return err ? ALADDIN_ERR_STATE : ALADDIN_OK;
+}
+
+}  // extern "C"
+
+// ---------------------------------------------------------------------------
+// Fleet simulation.
+
+namespace {
+
+struct DevTrace {
+    int64_t n = 0;
+    double* t = nullptr;
+    int32_t* in = nullptr;
+    int32_t* pred = nullptr;
+    std::vector<double> host_t;
+    ~DevTrace()
+    {
+        if (t) cudaFree(t);
+        if (in) cudaFree(in);
+        if (pred) cudaFree(pred);
+    }
+};
+
+int upload_trace(const aladdin_params& p, const aladdin_trace* tr, DevTrace& d, cudaStream_t st)
+{
+    if (!tr || tr->n < 0 || (tr->n > 0 && (!tr->t_arr_ms || !tr->in || !tr->pred)))
+        return ALADDIN_ERR_ARG;
+    d.n = tr->n;
+    d.host_t.assign(tr->t_arr_ms, tr->t_arr_ms + tr->n);
+    for (int64_t i = 0; i < tr->n; ++i) {
+        if (!std::isfinite(tr->t_arr_ms[i]) || (i > 0 && tr->t_arr_ms[i] < tr->t_arr_ms[i - 1]))
+            return ALADDIN_ERR_ARG;
+        if (tr->in[i] < 0 || tr->pred[i] < 1 || (long long)tr->in[i] + tr->pred[i] > p.K)
+            return ALADDIN_ERR_ARG;
+    }
+    const size_t n = (size_t)(tr->n > 0 ? tr->n : 1);
+    CK(cudaMalloc(&d.t, sizeof(double) * n));
+    CK(cudaMalloc(&d.in, sizeof(int32_t) * n));
+    CK(cudaMalloc(&d.pred, sizeof(int32_t) * n));
+    if (tr->n > 0) {
+        CK(cudaMemcpyAsync(d.t, tr->t_arr_ms, sizeof(double) * tr->n, cudaMemcpyHostToDevice, st));
+        CK(cudaMemcpyAsync(d.in, tr->in, sizeof(int32_t) * tr->n, cudaMemcpyHostToDevice, st));
+        CK(cudaMemcpyAsync(d.pred, tr->pred, sizeof(int32_t) * tr->n, cudaMemcpyHostToDevice, st));
+    }
+    CK(cudaStreamSynchronize(st));
+    return ALADDIN_OK;
+}
+
+__global__ void k_busy(const int32_t* __restrict__ n, int W, int* out)
+{
+    int any = 0;
+    for (int w = threadIdx.x; w < W; w += blockDim.x) any |= n[w] > 0;
+    any = __syncthreads_or(any);
+    if (threadIdx.x == 0) *out = any;
+}
+
+// One simulation; out[0..4] as aladdin_simulate.
+int simulate_impl(const aladdin_params& p, const aladdin_worker_cfg& cfg, int32_t N,
+                  const DevTrace& tr, double H, bool stop_at_fail, bool drain, cudaStream_t st,
+                  double* out)
+{
+    aladdin_cluster cl;
+    std::vector<aladdin_worker_cfg> cfgs((size_t)N, cfg);
+    int rc = cluster_alloc(&cl, p, N, cfgs.data(), st);
+    if (rc) return rc;
+    rc = refresh_tables(&cl);
+    if (rc) return rc;
+    DevBuf wl, cnt;
+    CK(wl.ensure(sizeof(long long) * (size_t)(tr.n > 0 ? tr.n : 1)));
+    CK(cnt.ensure(sizeof(unsigned long long) * 4 + sizeof(int) * 4));
+    unsigned long long* counters = cnt.as<unsigned long long>();
+    int* nwait = reinterpret_cast<int*>(counters + 4);
+    int* busy = nwait + 1;
+    CK(cudaMemsetAsync(cnt.p, 0, sizeof(unsigned long long) * 4 + sizeof(int) * 4, st));
+
+    int64_t next = 0;
+    long long hb = 0;
+    bool halted = false;
+    unsigned long long hc[4] = {0, 0, 0, 0};
+    for (;;) {
+        const double t = (double)hb * H;
+        int64_t end = next;
+        while (end < tr.n && tr.host_t[(size_t)end] <= t) ++end;
+        RoundIO io;
+        std::memset(&io, 0, sizeof(io));
+        io.sim = 1;
+        io.t_arr = tr.t;
+        io.tin = tr.in;
+        io.tpred = tr.pred;
+        io.wl = wl.as<long long>();
+        io.n_wait = nwait;
+        io.arr_begin = next;
+        io.arr_end = end;
+        io.t_now = t;
+        io.H = H;
+        io.counters = counters;
+        io.status = cl.d_status;
+        io.stop_at_fail = stop_at_fail ? 1 : 0;
+        io.hb = hb;
+        CK(launch_round(cl.dp, cl.dev, io, st));
+        next = end;
+        CK(launch_advance(cl.dp, cl.dev, t, H, cl.d_stats, cl.d_status, st));
+        CK(launch_build(cl.dp, cl.dev, nullptr, cl.W, st));
+        hb++;
+        const bool tail = next >= tr.n;
+        if (tail || (hb & 31) == 0) {
+            int hs[2] = {0, 0};
+            if (drain && tail) k_busy<<<1, 1024, 0, st>>>(cl.dev.n, cl.W, busy);
+            CK(cudaMemcpyAsync(hc, counters, sizeof(hc), cudaMemcpyDeviceToHost, st));
+            CK(cudaMemcpyAsync(hs, nwait, sizeof(hs), cudaMemcpyDeviceToHost, st));
+            int status = 0;
+            CK(cudaMemcpyAsync(&status, cl.d_status, sizeof(int), cudaMemcpyDeviceToHost, st));
+            CK(cudaStreamSynchronize(st));
+            if (status == -2) return ALADDIN_ERR_CAPACITY;
+            if (status == 1) {
+                halted = true;
+                break;
+            }
+            if (tail && hs[0] == 0 && (!drain || hs[1] == 0)) break;
+        }
+    }
+    unsigned long long s[4];
+    CK(cudaMemcpyAsync(s, cl.d_stats, sizeof(s), cudaMemcpyDeviceToHost, st));
+    CK(cudaMemcpyAsync(hc, counters, sizeof(hc), cudaMemcpyDeviceToHost, st));
+    CK(cudaStreamSynchronize(st));
+    out[0] = (double)hc[0];
+    out[1] = (double)hc[1];
+    out[2] = halted ? (double)hc[2] : (double)hb;
+    std::memcpy(&out[3], &s[2], 8);
+    std::memcpy(&out[4], &s[3], 8);
+    wl.release();
+    cnt.release();
+    return ALADDIN_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+int aladdin_simulate(const aladdin_params* params, const aladdin_worker_cfg* cfg, int32_t n,
+                     const aladdin_trace* trace, double heartbeat_ms, int32_t stop_at_fail,
+                     int32_t drain, void* cuda_stream, double* out)
+{
+    int rc = check_params(params);
+    if (rc) return rc;
+    if (!cfg || n < 1 || !out || !(std::isfinite(heartbeat_ms) && heartbeat_ms > 0))
+        return ALADDIN_ERR_ARG;
+    if ((rc = check_cfg(*cfg))) return rc;
+    cudaStream_t st = (cudaStream_t)cuda_stream;
+    DevTrace tr;
+    if ((rc = upload_trace(*params, trace, tr, st))) return rc;
+    return simulate_impl(*params, *cfg, n, tr, heartbeat_ms, stop_at_fail != 0, drain != 0, st, out);
+}
+
+int aladdin_min_workers(const aladdin_params* params, int32_t n_options,
+                        const aladdin_worker_cfg* options, const aladdin_trace* trace,
+                        double heartbeat_ms, int32_t n_max, void* cuda_stream,
+                        int32_t* n_workers, int32_t* best_option, int64_t* total_gpus)
+{
+    int rc = check_params(params);
+    if (rc) return rc;
+    if (n_options < 1 || !options || !n_workers || n_max < 1 ||
+        !(std::isfinite(heartbeat_ms) && heartbeat_ms > 0))
+        return ALADDIN_ERR_ARG;
+    for (int o = 0; o < n_options; ++o)
+        if ((rc = check_cfg(options[o]))) return rc;
+    cudaStream_t st = (cudaStream_t)cuda_stream;
+    DevTrace tr;
+    if ((rc = upload_trace(*params, trace, tr, st))) return rc;
+    double out[5];
+    for (int o = 0; o < n_options; ++o) {
+        int32_t lo = 0, hi = 1;
+        bool found = false;
+        while (hi <= n_max) {
+            if ((rc = simulate_impl(*params, options[o], hi, tr, heartbeat_ms, true, false, st, out)))
+                return rc;
+            if (out[0] == 0.0) {
+                found = true;
+                break;
+            }
+            lo = hi;
+            hi = (hi * 2 > n_max && hi < n_max) ? n_max : hi * 2;
+        }
+        if (!found) {
+            n_workers[o] = -1;
+            continue;
+        }
+        while (hi - lo > 1) {
+            const int32_t mid = lo + (hi - lo) / 2;
+            if ((rc = simulate_impl(*params, options[o], mid, tr, heartbeat_ms, true, false, st, out)))
+                return rc;
+            if (out[0] == 0.0) hi = mid;
+            else lo = mid;
+        }
+        n_workers[o] = hi;
+    }
+    int best = -1;
+    int64_t bestg = 0;
+    for (int o = 0; o < n_options; ++o) {
+        if (n_workers[o] < 0) continue;
+        const int64_t g = (int64_t)options[o].gpus * n_workers[o];
+        if (best < 0 || g < bestg) {
+            best = o;
+            bestg = g;
+        }
+    }
+    if (best_option) *best_option = best;
+    if (total_gpus) *total_gpus = best < 0 ? -1 : bestg;
+    return ALADDIN_OK;
+}
+
+}  // extern "C"

@@ -1,0 +1,214 @@
+"""Parity of the CUDA scoring path (aladdin_score / aladdin_score_detail)
+with the oracle, element by element, through the C ABI."""
+import numpy as np
+import pytest
+
+from parity import check_argbest, compare_pairs
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module")
+def A():
+    import torch
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    torch.cuda.init()
+    from paper_2405_06856_gb300 import build
+    build.build()
+    from paper_2405_06856_gb300 import aladdin
+    return aladdin
+
+
+def run_full(A, orc, wl, detail=True, label=""):
+    with A.Cluster.from_workload(wl) as cl:
+        g = cl.score(wl.cand_in, wl.cand_pred, wl.cand_wait, detail=detail)
+    oc = orc.Cluster.from_workload(wl)
+    ref = oc.score(wl.cand_in, wl.cand_pred, wl.cand_wait)
+    near = compare_pairs(ref, g["flags"], g["margin"], wl.cand_in, g.get("kvpeak"), g.get("tcand"),
+                         label)
+    check_argbest(oc.order(), g["flags"], g["argbest"], label)
+    if near == 0:
+        assert np.array_equal(g["argbest"], ref["argbest"])
+    return g, ref, near
+
+
+def test_tiny_literal(A, orc, synth):
+    wl = synth.config("tiny")
+    g, ref, near = run_full(A, orc, wl, label="tiny")
+
+
+@pytest.mark.parametrize("seed,tpre,tdec", [(101, 40.0, 30.0), (102, 1000.0, 50.0),
+                                            (103, 25.0, 20.0), (104, 80.0, 14.0)])
+def test_tiny_mixed_load(A, orc, synth, seed, tpre, tdec):
+    wl = synth.config("tiny", per_worker_random=True, seed=seed, n_cand=300,
+                      params=dict(T_pre=tpre, T_dec=tdec))
+    g, ref, near = run_full(A, orc, wl, label="tiny-mixed-%d" % seed)
+    frac = (g["flags"] == 15).mean()
+    assert 0.0 < frac < 1.0
+
+
+def test_every_constraint_group_binds(A, orc, synth):
+    """Across seeds every flag bit is seen cleared on some pair."""
+    seen = 0
+    for seed in range(110, 114):
+        wl = synth.config("tiny", per_worker_random=True, seed=seed, n_cand=200,
+                          params=dict(T_pre=22.0, T_dec=16.0))
+        g, ref, near = run_full(A, orc, wl, label="groups-%d" % seed)
+        for b in range(4):
+            if ((g["flags"] >> b) & 1 == 0).any():
+                seen |= 1 << b
+    assert seen == 15
+
+
+def test_scale_h_j_and_history(A, orc, synth):
+    """Non-unit KV coefficients, mixed latency scales and a decode history."""
+    wl = synth.config("tiny", per_worker_random=True, seed=120, n_cand=256, gpus_cycle=(1, 2, 4, 8),
+                      kv_per_gpu=40000, params=dict(h=2, j=3, T_pre=70.0, T_dec=24.0, theta=0.9))
+    rng = np.random.default_rng(5)
+    tdec = (wl.req_gen * rng.uniform(8.0, 30.0, len(wl.req_gen))).astype(np.float32)
+    with A.Cluster.from_workload(wl, tdec_ms=tdec) as cl:
+        g = cl.score(wl.cand_in, wl.cand_pred, wl.cand_wait, detail=True)
+    oc = orc.Cluster.from_workload(wl, tdec=tdec.astype(np.float64))
+    ref = oc.score(wl.cand_in, wl.cand_pred, wl.cand_wait)
+    compare_pairs(ref, g["flags"], g["margin"], wl.cand_in, g["kvpeak"], g["tcand"], "hist")
+    check_argbest(oc.order(), g["flags"], g["argbest"], "hist")
+
+
+def test_w256(A, orc, synth):
+    wl = synth.config("w256")
+    g, ref, near = run_full(A, orc, wl, label="w256")
+    print("w256: near pairs %d of %d, feasible %.3f" % (near, g["flags"].size,
+                                                         (g["flags"] == 15).mean()))
+
+
+def test_ragged_and_edge_shapes(A, orc, synth):
+    """W not a multiple of 4 (scalar store path), one worker, one candidate,
+    empty workers, candidates at the sequence limit, and chunk tails."""
+    for W, C, seed in ((7, 257, 130), (1, 1, 131), (33, 513, 132), (130, 1000, 133)):
+        wl = synth.make_cluster("edge", seed, W, 20, 30000, C, per_worker_random=True,
+                                params=dict(T_pre=50.0, T_dec=25.0, K=4096))
+        wl.cand_pred[: min(3, C)] = 4096 - wl.cand_in[: min(3, C)]
+        run_full(A, orc, wl, label="edge-W%d-C%d" % (W, C))
+
+
+def test_invalid_candidates(A, orc, synth):
+    wl = synth.config("tiny", per_worker_random=True, seed=140, n_cand=40)
+    cin, cpr, cw = wl.cand_in.copy(), wl.cand_pred.copy(), wl.cand_wait.copy()
+    cin[3] = -1
+    cpr[5] = 0
+    cpr[7] = wl.params["K"]          # in + pred > K
+    cw[9] = np.nan
+    cw[11] = -1.0
+    bad = [3, 5, 7, 9, 11]
+    with A.Cluster.from_workload(wl) as cl:
+        g = cl.score(cin, cpr, cw, detail=True)
+    assert np.all(g["flags"][bad] == A.FLAG_INVALID)
+    assert np.all(np.isnan(g["margin"][bad]))
+    assert np.all(g["argbest"][bad] == A.INVALID)
+    good = np.setdiff1d(np.arange(40), bad)
+    oc = orc.Cluster.from_workload(wl)
+    ref = oc.score(cin[good], cpr[good], cw[good])
+    compare_pairs(ref, g["flags"][good], g["margin"][good], cin[good], g["kvpeak"][good],
+                  g["tcand"][good], "valid-rows")
+
+
+def test_device_and_host_pointers_agree(A, synth):
+    import torch
+    wl = synth.config("w256", n_cand=700)
+    dev = torch.device("cuda")
+    with A.Cluster.from_workload(wl) as cl:
+        h = cl.score(wl.cand_in, wl.cand_pred, wl.cand_wait)
+        C, W = wl.n_cand, wl.n_workers
+        f = torch.zeros((C, W), dtype=torch.uint8, device=dev)
+        m = torch.zeros((C, W), dtype=torch.float32, device=dev)
+        a = torch.zeros(C, dtype=torch.int32, device=dev)
+        A.aladdin_score(cl.handle, C, torch.from_numpy(wl.cand_in).to(dev),
+                        torch.from_numpy(wl.cand_pred).to(dev), torch.from_numpy(wl.cand_wait).to(dev),
+                        f, m, a)
+        torch.cuda.synchronize()
+        assert np.array_equal(f.cpu().numpy(), h["flags"])
+        assert np.array_equal(m.cpu().numpy().view(np.uint32), h["margin"].view(np.uint32))
+        assert np.array_equal(a.cpu().numpy(), h["argbest"])
+        # argbest only (no pair outputs) gives the same choice
+        a2 = torch.zeros(C, dtype=torch.int32, device=dev)
+        A.aladdin_score(cl.handle, C, torch.from_numpy(wl.cand_in).to(dev),
+                        torch.from_numpy(wl.cand_pred).to(dev), torch.from_numpy(wl.cand_wait).to(dev),
+                        None, None, a2)
+        torch.cuda.synchronize()
+        assert np.array_equal(a2.cpu().numpy(), h["argbest"])
+
+
+def test_deterministic(A, synth):
+    wl = synth.config("w256", n_cand=1500)
+    with A.Cluster.from_workload(wl) as cl:
+        a = cl.score(wl.cand_in, wl.cand_pred, wl.cand_wait)
+        b = cl.score(wl.cand_in, wl.cand_pred, wl.cand_wait)
+    for k in a:
+        assert a[k].tobytes() == b[k].tobytes(), k
+
+
+def test_load_device_state(A, orc, synth):
+    """aladdin_cluster_load from device memory equals creation from host memory;
+    an invalid request loaded from device memory poisons only its worker."""
+    import torch
+    wl = synth.config("tiny", per_worker_random=True, seed=150, n_cand=64)
+    wl2 = synth.config("tiny", per_worker_random=True, seed=151, n_cand=64)
+    dev = torch.device("cuda")
+    with A.Cluster.from_workload(wl) as cl:
+        t = lambda x: torch.from_numpy(np.ascontiguousarray(x)).to(dev)
+        cl.load(t(wl2.roff), t(wl2.req_in), t(wl2.req_gen), t(wl2.req_pred))
+        torch.cuda.synchronize()
+        g = cl.score(wl2.cand_in, wl2.cand_pred, wl2.cand_wait)
+        assert cl.status() == A.OK
+        ref = orc.Cluster.from_workload(wl2).score(wl2.cand_in, wl2.cand_pred, wl2.cand_wait)
+        compare_pairs(ref, g["flags"], g["margin"], wl2.cand_in, label="load")
+        gen = wl2.req_gen.copy()
+        w_bad = int(np.argmax(np.diff(wl2.roff) > 0))
+        gen[wl2.roff[w_bad]] = wl2.req_pred[wl2.roff[w_bad]]  # gen == pred: invalid
+        cl.load(t(wl2.roff), t(wl2.req_in), t(gen), t(wl2.req_pred))
+        torch.cuda.synchronize()
+        assert cl.status() == A.ERR_STATE
+        g2 = cl.score(wl2.cand_in, wl2.cand_pred, wl2.cand_wait)
+        assert np.all(g2["flags"][:, w_bad] & 1 == 0)
+        keep = np.arange(wl2.n_workers) != w_bad
+        assert np.array_equal(g2["flags"][:, keep], g["flags"][:, keep])
+    # host path rejects the same state up front
+    with pytest.raises(A.AladdinError):
+        A.Cluster(wl2.params, wl2.gpus, wl2.kv_capacity, wl2.lat_scale, wl2.b_cap, wl2.roff,
+                  wl2.req_in, gen, wl2.req_pred)
+
+
+def test_w4096_sampled(A, orc, synth):
+    """The 4,096-worker workload at full size: sampled pairs and sampled
+    argbest rows against the oracle."""
+    import torch
+    wl = synth.config("w4096")
+    C, W = wl.n_cand, wl.n_workers
+    dev = torch.device("cuda")
+    with A.Cluster.from_workload(wl) as cl:
+        f = torch.zeros((C, W), dtype=torch.uint8, device=dev)
+        m = torch.zeros((C, W), dtype=torch.float32, device=dev)
+        a = torch.zeros(C, dtype=torch.int32, device=dev)
+        A.aladdin_score(cl.handle, C, torch.from_numpy(wl.cand_in).to(dev),
+                        torch.from_numpy(wl.cand_pred).to(dev), torch.from_numpy(wl.cand_wait).to(dev),
+                        f, m, a)
+        torch.cuda.synchronize()
+        rng = np.random.default_rng(9)
+        pc = rng.integers(0, C, 3000).astype(np.int32)
+        pw = rng.integers(0, W, 3000).astype(np.int32)
+        oc = orc.Cluster.from_workload(wl)
+        ref = oc.score_pairs(pc, pw, wl.cand_in, wl.cand_pred, wl.cand_wait)
+        fi = f[torch.from_numpy(pc).long().to(dev), torch.from_numpy(pw).long().to(dev)].cpu().numpy()
+        mi = m[torch.from_numpy(pc).long().to(dev), torch.from_numpy(pw).long().to(dev)].cpu().numpy()
+        compare_pairs(ref, fi, mi, wl.cand_in[pc], label="w4096-sampled")
+        fr = (f == 15).float().mean().item()
+        assert 0.05 < fr < 0.999
+        rows = rng.integers(0, C, 6)
+        order = oc.order()
+        sub = oc.score(wl.cand_in[rows], wl.cand_pred[rows], wl.cand_wait[rows],
+                       want=("flags", "margin", "mscale", "near", "argbest"))
+        fr_rows = f[torch.from_numpy(rows).long().to(dev)].cpu().numpy()
+        mr_rows = m[torch.from_numpy(rows).long().to(dev)].cpu().numpy()
+        compare_pairs(sub, fr_rows, mr_rows, wl.cand_in[rows], label="w4096-rows")
+        check_argbest(order, fr_rows, a.cpu().numpy()[rows], "w4096-rows")
