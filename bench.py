@@ -347,6 +347,34 @@ def run_ours(args):
         dist.destroy_process_group()
 
 
+def run_kernel_only(args):
+    """The device-resident step only (warm-up + steps), nothing else: the
+    command profiled by ncu."""
+    import torch
+    from paper_2405_06856_gb300 import build as B
+    B.build()
+    from paper_2405_06856_gb300 import aladdin as A
+    from paper_2405_06856_gb300 import synth
+    torch.cuda.set_device(0)
+    dev = torch.device("cuda", 0)
+    wl = synth.config(WORKLOAD)
+    W, C = wl.n_workers, wl.n_cand
+    d = lambda x: torch.from_numpy(np.ascontiguousarray(x)).to(dev)
+    roff, rin, rgen, rpred = d(wl.roff), d(wl.req_in), d(wl.req_gen), d(wl.req_pred)
+    cin, cpr, cw = d(wl.cand_in), d(wl.cand_pred), d(wl.cand_wait)
+    flags = torch.empty((C, W), dtype=torch.uint8, device=dev)
+    margin = torch.empty((C, W), dtype=torch.float32, device=dev)
+    arg = torch.empty(C, dtype=torch.int32, device=dev)
+    cl = A.Cluster.from_workload(wl, stream=torch.cuda.current_stream().cuda_stream)
+    for _ in range(args.warmup + args.steps):
+        A.aladdin_cluster_load(cl.handle, roff, rin, rgen, rpred)
+        A.aladdin_score(cl.handle, C, cin, cpr, cw, flags, margin, arg)
+    torch.cuda.synchronize()
+    assert cl.status() == A.OK
+    cl.close()
+    print("kernel mode ok: %d steps" % (args.warmup + args.steps))
+
+
 def kernel_source_hash():
     import hashlib
     h = hashlib.sha256()
@@ -362,11 +390,15 @@ def main():
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--no-cpu-baseline", dest="cpu_baseline", action="store_false")
+    ap.add_argument("--mode", default="full", choices=["full", "kernel"],
+                    help="kernel: only warm-up + steps of the device-resident step (for profilers)")
     args = ap.parse_args()
     if args.warmup < 3:
         args.warmup = 3
     if args.impl == "reference":
         run_reference(args)
+    elif args.mode == "kernel":
+        run_kernel_only(args)
     else:
         run_ours(args)
 

@@ -29,7 +29,7 @@ def compare_pairs(ref, flags, margin, cand_in, kvpeak=None, tcand=None, label=""
     fin = np.isfinite(ref["margin"])
     assert np.all(np.isneginf(m[~fin])), "%s: -inf margins differ" % label
     tol = margin_tol(ref["margin"], ref["mscale"], cand_in)
-    err = np.abs(m - ref["margin"])
+    err = np.where(fin, np.abs(np.where(fin, m, 0.0) - np.where(fin, ref["margin"], 0.0)), 0.0)
     badm = fin & (err > tol)
     assert not badm.any(), "%s: %d margin mismatches, worst %s vs %s" % (
         label, int(badm.sum()), m[badm][:3], ref["margin"][badm][:3])
