@@ -170,8 +170,10 @@ int aladdin_cluster_state(aladdin_cluster* cl, int32_t* n, int32_t* in, int32_t*
 int aladdin_cluster_timing(aladdin_cluster* cl, int32_t enable, double* kernel_ms,
                            int64_t* launches);
 
-/* ALADDIN_OK, or ALADDIN_ERR_STATE if an invalid request was loaded from device
- * memory, or ALADDIN_ERR_CUDA. Synchronous. */
+/* ALADDIN_OK; ALADDIN_ERR_TIMEOUT if a kernel gave up a bounded wait for its
+ * own shared-memory copies (its outputs for that call are incomplete);
+ * ALADDIN_ERR_STATE if an invalid request was loaded from device memory; or
+ * ALADDIN_ERR_CUDA. Errors are sticky. Synchronous. */
 int aladdin_cluster_status(aladdin_cluster* cl);
 
 /* A request trace: arrival times (ms, non-decreasing), prompt and predicted

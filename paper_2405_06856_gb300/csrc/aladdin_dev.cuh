@@ -89,7 +89,7 @@ struct ClusterDev {
     AuxRow* aux;               // [W*rows]
     int32_t* R;                // [W] breakpoints
     float4* wrec;              // [W] {1/s, ZO, ZW, rank bits}
-    double* key;               // [W] capacity_norm^2
+    unsigned long long* key;   // [W] order-preserving code of capacity_norm^2 (0: unusable)
     int32_t* rank;             // [W]
     int32_t* order;            // [W] worker at rank
     unsigned int* err;         // sticky error bits (1: invalid request)
@@ -538,7 +538,11 @@ __device__ void build_table(const DevParams& P, const ClusterDev& C, int w, Buil
         C.wrec[w] = wr;
         const double B = (double)n;
         const double L = __dadd_rn((double)sumIn, __dmul_rn(P.gammad, (double)sumPred));
-        C.key[w] = bad ? -1.0 : __dadd_rn(__dmul_rn(B, B), __dmul_rn(L, L));
+        // capacity_norm^2 is exact here (integer and half-integer terms below
+        // 2^53); non-negative doubles order like their bit patterns, and code 0
+        // is kept for a worker holding an invalid request.
+        const double q = __dadd_rn(__dmul_rn(B, B), __dmul_rn(L, L));
+        C.key[w] = bad ? 0ull : (unsigned long long)__double_as_longlong(q) + 1ull;
     }
     __syncwarp();
 }

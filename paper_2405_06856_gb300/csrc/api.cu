@@ -221,7 +221,7 @@ int cluster_alloc(aladdin_cluster* cl, const aladdin_params& p, int W,
     AL(aux, AuxRow, rows);
     AL(R, int32_t, W);
     AL(wrec, float4, W);
-    AL(key, double, W);
+    AL(key, unsigned long long, W);
     AL(rank, int32_t, W);
     AL(order, int32_t, W);
     AL(err, unsigned int, 1);
@@ -639,6 +639,7 @@ int aladdin_cluster_status(aladdin_cluster* cl)
     unsigned int err = 0;
     CK(cudaMemcpyAsync(&err, cl->dev.err, sizeof(err), cudaMemcpyDeviceToHost, cl->st));
     CK(cudaStreamSynchronize(cl->st));
+    if (err & 4u) return ALADDIN_ERR_TIMEOUT;
     return err ? ALADDIN_ERR_STATE : ALADDIN_OK;
 }
 

@@ -19,13 +19,13 @@ constexpr int ROUND_WARPS = ROUND_THREADS / 32;
 template <int E>
 struct RoundSmem {
     BuildSmem<E> build;
-    double bk[ROUND_WARPS];
+    unsigned long long bk[ROUND_WARPS];
     int bw[ROUND_WARPS];
     int winner;
     int stop;
 };
 
-__device__ __forceinline__ void better(double& bk, int& bw, double ok, int ow)
+__device__ __forceinline__ void better(unsigned long long& bk, int& bw, unsigned long long ok, int ow)
 {
     if (ow != 0x7fffffff && (bw == 0x7fffffff || ok > bk || (ok == bk && ow < bw))) {
         bk = ok;
@@ -63,7 +63,7 @@ __global__ void __launch_bounds__(ROUND_THREADS) k_round(DevParams P, ClusterDev
         const CandRec cr = make_cand(P, a, r, (float)wd, c);
         int winner = -2;
         if (cr.valid) {
-            double bk = 0.0;
+            unsigned long long bk = 0ull;
             int bw = 0x7fffffff;
             for (int w = tid; w < C.W; w += ROUND_THREADS) {
                 const long long rb = (long long)w * C.rows;
@@ -75,7 +75,7 @@ __global__ void __launch_bounds__(ROUND_THREADS) k_round(DevParams P, ClusterDev
             }
 #pragma unroll
             for (int d = 16; d > 0; d >>= 1) {
-                const double ok = __shfl_xor_sync(FULL, bk, d);
+                const unsigned long long ok = __shfl_xor_sync(FULL, bk, d);
                 const int ow = __shfl_xor_sync(FULL, bw, d);
                 better(bk, bw, ok, ow);
             }
@@ -85,11 +85,11 @@ __global__ void __launch_bounds__(ROUND_THREADS) k_round(DevParams P, ClusterDev
             }
             __syncthreads();
             if (warp == 0) {
-                bk = lane < ROUND_WARPS ? sm.bk[lane] : 0.0;
+                bk = lane < ROUND_WARPS ? sm.bk[lane] : 0ull;
                 bw = lane < ROUND_WARPS ? sm.bw[lane] : 0x7fffffff;
 #pragma unroll
                 for (int d = 16; d > 0; d >>= 1) {
-                    const double ok = __shfl_xor_sync(FULL, bk, d);
+                    const unsigned long long ok = __shfl_xor_sync(FULL, bk, d);
                     const int ow = __shfl_xor_sync(FULL, bw, d);
                     better(bk, bw, ok, ow);
                 }

@@ -1,15 +1,18 @@
 // K3: batched candidate x worker scoring.
 //
 // Candidates are validated, turned into per-candidate constants and
-// counting-sorted by predicted output length. A warp owns a tile of
-// 32 x SLOTS consecutive workers (SLOTS per lane) and sweeps a chunk of the
-// sorted candidates: each lane keeps the table row of each of its workers in
-// registers and only steps to the next row when the candidate's length
-// crosses that worker's next breakpoint, so a pair costs one row compare and
-// the O(1) bound arithmetic of eval_pair. Flags and margins of one candidate
-// are written as one coalesced row segment per warp (streaming stores); the
-// per-candidate argbest is the smallest capacity_norm rank among feasible
-// workers (warp min-reduction, one atomic per warp and candidate).
+// counting-sorted by predicted output length. A CTA owns a tile of
+// SCORE_WARPS x 32 x SLOTS consecutive workers and a contiguous range of the
+// sorted candidates; the grid is one wave of CTAs with equal shares. Candidate
+// records are staged into shared memory in chunks by TMA bulk copies (double
+// buffered, mbarrier completion). Each lane keeps, per worker, the table row of
+// the segment containing the current candidate length and the next row, so a
+// breakpoint crossing is a register move while the row after it is fetched in
+// the background; a pair costs the O(1) bound arithmetic only. Flags and
+// margins of one candidate are one coalesced row segment per warp (streaming
+// stores); argbest is the smallest capacity_norm rank among feasible workers,
+// reduced per warp, merged across the CTA's warps in shared memory and
+// committed with one atomic per CTA and candidate.
 #include "aladdin_host.h"
 
 namespace aladdin {
@@ -70,14 +73,21 @@ __global__ void __launch_bounds__(SCAN_THREADS) k_scan_hist(int32_t* hist, int l
     }
 }
 
-__global__ void k_cand_scatter(DevParams P, int n, const int32_t* __restrict__ in,
+// Sorted record: the CandRec constants, with the third float4 holding
+// {valid ? predicted output : 0, original index, low and high words of
+// index * W} (the start of the candidate's output row).
+__global__ void k_cand_scatter(DevParams P, int n, int W, const int32_t* __restrict__ in,
                                const int32_t* __restrict__ pred, const float* __restrict__ wait,
                                int32_t* cursor, CandRec* sorted)
 {
     const int c = blockIdx.x * blockDim.x + threadIdx.x;
     if (c >= n) return;
-    const CandRec rec = make_cand(P, in[c], pred[c], wait ? wait[c] : 0.0f, c);
+    CandRec rec = make_cand(P, in[c], pred[c], wait ? wait[c] : 0.0f, c);
     const int pos = atomicAdd(&cursor[rec.valid ? rec.ri : 0], 1);
+    const unsigned long long rowoff = (unsigned long long)c * (unsigned long long)W;
+    rec.ri = rec.valid ? rec.ri : 0;
+    rec.valid = (int32_t)(unsigned)(rowoff & 0xffffffffull);
+    rec.pad = (int32_t)(unsigned)(rowoff >> 32);
     sorted[pos] = rec;
 }
 
@@ -91,48 +101,306 @@ struct ScoreArgs {
     int tiles, chunks;
 };
 
-__device__ __forceinline__ void load_row(const float4* __restrict__ tab, long long row, float4& v0,
-                                         float4& v1, float4& v2)
+struct Row {
+    float4 v0, v1, v2;
+};
+
+__device__ __forceinline__ Row load_row(const float4* __restrict__ tab, long long row)
 {
     const float4* t = tab + row * ROW_F4;
-    v0 = __ldg(t);
-    v1 = __ldg(t + 1);
-    v2 = __ldg(t + 2);
+    Row r;
+    r.v0 = __ldg(t);
+    r.v1 = __ldg(t + 1);
+    r.v2 = __ldg(t + 2);
+    return r;
 }
 
-template <int SLOTS, bool STORE, bool VEC>
-__global__ void __launch_bounds__(SCORE_WARPS * 32) k_score(ScoreArgs A)
+__device__ __forceinline__ unsigned prmt(unsigned a, unsigned b, unsigned sel)
+{
+    unsigned d;
+    asm("prmt.b32 %0, %1, %2, %3;" : "=r"(d) : "r"(a), "r"(b), "r"(sel));
+    return d;
+}
+
+// Flag bytes of SLOTS pairs from the sign bits of their group headrooms
+// d[g][k] = bound_g - a (bit g of byte k set iff d[g][k] >= 0). prmt with the
+// sign-replicate selector (bit 3 of a selector nibble) turns the top byte of
+// each headroom into 0x00 / 0xff, one byte per slot.
+template <int SLOTS>
+__device__ __forceinline__ unsigned pack_flags(const float (&d)[4][SLOTS])
+{
+    unsigned acc = 0;
+#pragma unroll
+    for (int g = 0; g < 4; ++g) {
+        unsigned S;
+        if (SLOTS == 4) {
+            const unsigned t1 = prmt(__float_as_uint(d[g][0]), __float_as_uint(d[g][1 % SLOTS]), 0x00fbu);
+            const unsigned t2 = prmt(__float_as_uint(d[g][2 % SLOTS]), __float_as_uint(d[g][3 % SLOTS]), 0x00fbu);
+            S = prmt(t1, t2, 0x5410u);
+        } else if (SLOTS == 2) {
+            S = prmt(__float_as_uint(d[g][0]), __float_as_uint(d[g][1 % SLOTS]), 0x00fbu);
+        } else {
+            S = prmt(__float_as_uint(d[g][0]), 0u, 0x000bu);
+        }
+        acc |= ~S & (0x01010101u << g);
+    }
+    return SLOTS == 4 ? acc : (SLOTS == 2 ? (acc & 0xffffu) : (acc & 0xffu));
+}
+
+#ifndef ALADDIN_SCORE_SLOTS
+#define ALADDIN_SCORE_SLOTS 2
+#endif
+constexpr int CHUNK = 256;               // candidates per staged chunk
+constexpr long long WAIT_LIMIT = 1ll << 26;  // mbarrier polls before giving up
+constexpr unsigned ERR_TIMEOUT_BIT = 4u;
+
+__device__ __forceinline__ unsigned smem_addr(const void* p)
+{
+    return (unsigned)__cvta_generic_to_shared(p);
+}
+
+__device__ __forceinline__ void mbar_init(unsigned long long* bar, unsigned count)
+{
+    asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(smem_addr(bar)), "r"(count) : "memory");
+}
+
+// One elected thread: expect `bytes` and start the bulk copy of `bytes`
+// (multiple of 16, both addresses 16-byte aligned) from global to shared.
+__device__ __forceinline__ void tma_load(void* dst, const void* src, unsigned bytes,
+                                         unsigned long long* bar)
+{
+    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+    asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(smem_addr(bar)),
+                 "r"(bytes)
+                 : "memory");
+    asm volatile(
+        "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(
+            smem_addr(dst)),
+        "l"(src), "r"(bytes), "r"(smem_addr(bar))
+        : "memory");
+}
+
+// Bounded wait for the phase with the given parity; false if the limit ran out.
+__device__ __forceinline__ bool mbar_wait(unsigned long long* bar, unsigned parity)
+{
+    for (long long it = 0; it < WAIT_LIMIT; ++it) {
+        unsigned done;
+        asm volatile(
+            "{\n .reg .pred p;\n mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n selp.u32 %0, 1, 0, p;\n}"
+            : "=r"(done)
+            : "r"(smem_addr(bar)), "r"(parity)
+            : "memory");
+        if (done) return true;
+    }
+    return false;
+}
+
+struct VecArgs {
+    ClusterDev C;
+    const float4* __restrict__ cand;   // sorted records, 3 float4 each
+    int n_cand;
+    uint8_t* flags;
+    float* margin;
+    unsigned int* best;
+    int tiles;       // worker tiles of SCORE_WARPS * 32 * SLOTS
+    int per_tile;    // CTAs per tile
+};
+
+template <int SLOTS>
+struct __align__(16) ScoreSmem {
+    float4 cs[2][CHUNK * 3];
+    unsigned kmin[SCORE_WARPS][CHUNK];
+    unsigned long long bar[2];
+    int stop;
+};
+
+template <int SLOTS, bool SF, bool SMG, bool ARG>
+__global__ void __launch_bounds__(SCORE_WARPS * 32) k_score(VecArgs A)
+{
+    extern __shared__ __align__(16) unsigned char smraw[];
+    ScoreSmem<SLOTS>& sm = *reinterpret_cast<ScoreSmem<SLOTS>*>(smraw);
+    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    const int W = A.C.W;
+    const int tile = blockIdx.x % A.tiles;
+    const int part = blockIdx.x / A.tiles;
+    // this CTA's candidate range [cb, ce)
+    const int cb = (int)(((long long)A.n_cand * part) / A.per_tile);
+    const int ce = (int)(((long long)A.n_cand * (part + 1)) / A.per_tile);
+    if (cb >= ce) return;  // CTA-uniform
+    const int nchunks = (ce - cb + CHUNK - 1) / CHUNK;
+
+    if (tid == 0) {
+        mbar_init(&sm.bar[0], 1);
+        mbar_init(&sm.bar[1], 1);
+        asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+        sm.stop = 0;
+    }
+    __syncthreads();
+    if (tid == 0) {
+        const int n0 = min(CHUNK, ce - cb);
+        tma_load(sm.cs[0], A.cand + (size_t)cb * 3, (unsigned)n0 * 48u, &sm.bar[0]);
+    }
+
+    const int wbase = (tile * SCORE_WARPS + warp) * 32 * SLOTS;
+    const int w0 = wbase + lane * SLOTS;
+    const bool live = w0 < W;
+    const bool warp_live = wbase < W;
+    const bool all_live = wbase + 32 * SLOTS <= W;
+    uint8_t* const fbase = SF ? A.flags + (live ? w0 : 0) : nullptr;
+    float* const mbase = SMG ? A.margin + (live ? w0 : 0) : nullptr;
+
+    Row cur[SLOTS], nxt[SLOTS];
+    float inv_s[SLOTS], nZO[SLOTS], ZW[SLOTS];
+    unsigned rank[SLOTS];
+    int p[SLOTS], R[SLOTS];
+    long long rb[SLOTS];
+    bool have_rows = false;
+
+    for (int k = 0; k < nchunks; ++k) {
+        const int buf = k & 1;
+        const int c0 = cb + k * CHUNK;
+        const int nc = min(CHUNK, ce - c0);
+        if (tid == 0 && k + 1 < nchunks) {
+            const int c1 = c0 + CHUNK;
+            const int n1 = min(CHUNK, ce - c1);
+            tma_load(sm.cs[buf ^ 1], A.cand + (size_t)c1 * 3, (unsigned)n1 * 48u, &sm.bar[buf ^ 1]);
+        }
+        if (!mbar_wait(&sm.bar[buf], (unsigned)((k >> 1) & 1))) {
+            if (lane == 0) atomicOr(A.C.err, ERR_TIMEOUT_BIT);
+            sm.stop = 1;
+        }
+        __syncthreads();
+        if (sm.stop) {
+            // let the other buffer's copy (if any) land before the CTA exits
+            if (tid == 0 && k + 1 < nchunks) mbar_wait(&sm.bar[buf ^ 1], (unsigned)(((k + 1) >> 1) & 1));
+            return;
+        }
+        const float4* cs = sm.cs[buf];
+        if (warp_live) {
+            if (!have_rows) {
+                const int r_first = __float_as_int(cs[2].x);
+#pragma unroll
+                for (int s = 0; s < SLOTS; ++s) {
+                    const int wc = live ? w0 + s : W - 1;
+                    rb[s] = (long long)wc * A.C.rows;
+                    R[s] = __ldg(&A.C.R[wc]);
+                    p[s] = find_row(A.C.tab, rb[s], R[s], r_first);
+                    cur[s] = load_row(A.C.tab, rb[s] + p[s]);
+                    nxt[s] = load_row(A.C.tab, rb[s] + min(p[s] + 1, R[s]));
+                    const float4 wr = __ldg(&A.C.wrec[wc]);
+                    inv_s[s] = wr.x;
+                    nZO[s] = -wr.y;
+                    ZW[s] = wr.z;
+                    rank[s] = live ? (unsigned)__float_as_int(wr.w) : 0xffffffffu;
+                }
+                have_rows = true;
+            }
+            for (int i = 0; i < nc; ++i) {
+                const float4 q0 = cs[3 * i], q1 = cs[3 * i + 1], q2 = cs[3 * i + 2];
+                const int ri = __float_as_int(q2.x);
+                const size_t off = ((size_t)(unsigned)__float_as_int(q2.w) << 32) |
+                                   (size_t)(unsigned)__float_as_int(q2.z);
+                if (ri == 0) {  // invalid candidate (warp-uniform)
+                    if (live) {
+#pragma unroll
+                        for (int s = 0; s < SLOTS; ++s) {
+                            if (SF) fbase[off + s] = 0x80;
+                            if (SMG) mbase[off + s] = __int_as_float(0x7fc00000);
+                        }
+                    }
+                    if (ARG && lane == 0) sm.kmin[warp][i] = 0xffffffffu;
+                    continue;
+                }
+                bool need = false;
+#pragma unroll
+                for (int s = 0; s < SLOTS; ++s) need |= ri >= __float_as_int(cur[s].v0.x);
+                if (__any_sync(FULL, need)) {
+#pragma unroll
+                    for (int s = 0; s < SLOTS; ++s) {
+                        while (ri >= __float_as_int(cur[s].v0.x) && p[s] < R[s]) {
+                            p[s] += 1;
+                            cur[s] = nxt[s];
+                            nxt[s] = load_row(A.C.tab, rb[s] + min(p[s] + 1, R[s]));
+                        }
+                    }
+                }
+                const float a = q0.x, r = q0.y, inv_r = q0.z, U = q0.w;
+                const float inv_d1 = q1.x, nXd1 = q1.y, inv_d2 = q1.z, Zc = q1.w;
+                float d[4][SLOTS], m[SLOTS];
+                unsigned kmin = 0xffffffffu;
+#pragma unroll
+                for (int s = 0; s < SLOTS; ++s) {
+                    const Row& c = cur[s];
+                    const float kvm = fminf(c.v0.y, fmaf(r, c.v0.w, c.v0.z));
+                    const float tt = fminf(fmaf(Zc, inv_s[s], nZO[s]), ZW[s]);
+                    const float ca = fmaf(c.v1.x, inv_r, fmaf(c.v1.z, r, U - c.v1.y));
+                    const float gon = fminf(c.v1.w, fmaf(c.v2.y, inv_d1, nXd1));
+                    const float gnew = fminf(fminf(c.v2.x, fmaf(c.v2.z, inv_d2, U)), ca);
+                    d[0][s] = kvm - a;
+                    d[1][s] = tt - a;
+                    d[2][s] = gon - a;
+                    d[3][s] = gnew - a;
+                    m[s] = fminf(fminf(d[0][s], d[1][s]), fminf(d[2][s], d[3][s]));
+                    if (ARG) kmin = min(kmin, (__float_as_uint(m[s]) & 0x80000000u) | rank[s]);
+                }
+                if (all_live || live) {
+                    if (SF) {
+                        const unsigned f = pack_flags<SLOTS>(d);
+                        if (SLOTS == 4) __stcs(reinterpret_cast<unsigned int*>(fbase + off), f);
+                        else if (SLOTS == 2) __stcs(reinterpret_cast<unsigned short*>(fbase + off), (unsigned short)f);
+                        else fbase[off] = (uint8_t)f;
+                    }
+                    if (SMG) {
+                        if (SLOTS == 4)
+                            __stcs(reinterpret_cast<float4*>(mbase + off),
+                                   make_float4(m[0], m[1 % SLOTS], m[2 % SLOTS], m[3 % SLOTS]));
+                        else if (SLOTS == 2)
+                            __stcs(reinterpret_cast<float2*>(mbase + off), make_float2(m[0], m[1 % SLOTS]));
+                        else __stcs(mbase + off, m[0]);
+                    }
+                }
+                if (ARG) {
+                    kmin = __reduce_min_sync(FULL, kmin);
+                    sm.kmin[warp][i] = kmin;  // same value from every lane
+                }
+            }
+        } else if (ARG) {
+            for (int i = tid & 31; i < nc; i += 32) sm.kmin[warp][i] = 0xffffffffu;
+        }
+        __syncthreads();
+        if (ARG) {
+            for (int i = tid; i < nc; i += SCORE_WARPS * 32) {
+                unsigned v = sm.kmin[0][i];
+#pragma unroll
+                for (int q = 1; q < SCORE_WARPS; ++q) v = min(v, sm.kmin[q][i]);
+                if (v < 0x80000000u) atomicMin(A.best + __float_as_int(cs[3 * i + 2].y), v);
+            }
+        }
+        __syncthreads();  // buffer `buf` and kmin are reused two chunks later
+    }
+}
+
+// Fallback for W % 4 != 0 or unaligned outputs: one worker per lane, scalar
+// stores.
+template <bool SF, bool SMG, bool ARG>
+__global__ void __launch_bounds__(SCORE_WARPS * 32) k_score_scalar(ScoreArgs A)
 {
     const int lane = threadIdx.x & 31;
     const int unit = blockIdx.x * SCORE_WARPS + (threadIdx.x >> 5);
-    if (unit >= A.tiles * A.chunks) return;  // warp-uniform
-    const int tile = unit % A.tiles;
-    const int chunk = unit / A.tiles;
+    if (unit >= A.tiles * A.chunks) return;
+    const int tile = unit % A.tiles, chunk = unit / A.tiles;
     const int W = A.C.W;
-    const int w0 = tile * 32 * SLOTS + lane * SLOTS;
+    const int w = tile * 32 + lane;
+    const bool live = w < W;
+    const int wc = live ? w : W - 1;
     const int c0 = chunk * SCORE_CHUNK;
     const int c1 = min(c0 + SCORE_CHUNK, A.n_cand);
-
-    float4 v0[SLOTS], v1[SLOTS], v2[SLOTS], wr[SLOTS];
-    int p[SLOTS], Rk[SLOTS];
-    long long rb[SLOTS];
-    unsigned rk[SLOTS];
-    bool live[SLOTS];
-    const int r_first = __ldg(&A.cand[c0].ri);
-#pragma unroll
-    for (int k = 0; k < SLOTS; ++k) {
-        const int w = w0 + k;
-        live[k] = w < W;
-        const int wc = live[k] ? w : 0;
-        rb[k] = (long long)wc * A.C.rows;
-        const int R = live[k] ? A.C.R[wc] : 0;
-        Rk[k] = R;
-        p[k] = live[k] ? find_row(A.C.tab, rb[k], R, r_first) : 0;
-        load_row(A.C.tab, rb[k] + p[k], v0[k], v1[k], v2[k]);
-        wr[k] = __ldg(&A.C.wrec[wc]);
-        rk[k] = (unsigned)__float_as_int(wr[k].w);
-    }
-
+    const long long rb = (long long)wc * A.C.rows;
+    const int R = A.C.R[wc];
+    int p = find_row(A.C.tab, rb, R, __ldg(&A.cand[c0].ri));
+    Row cur = load_row(A.C.tab, rb + p);
+    const float4 wr = __ldg(&A.C.wrec[wc]);
+    const unsigned rank = live ? (unsigned)__float_as_int(wr.w) : 0xffffffffu;
     for (int c = c0; c < c1; ++c) {
         const float4* cp = reinterpret_cast<const float4*>(A.cand + c);
         const float4 q0 = __ldg(cp), q1 = __ldg(cp + 1), q2 = __ldg(cp + 2);
@@ -141,61 +409,75 @@ __global__ void __launch_bounds__(SCORE_WARPS * 32) k_score(ScoreArgs A)
         cr.inv_d1 = q1.x; cr.nXd1 = q1.y; cr.inv_d2 = q1.z; cr.Zc = q1.w;
         cr.ri = __float_as_int(q2.x);
         cr.orig = __float_as_int(q2.y);
-        cr.valid = __float_as_int(q2.z);
-        const size_t rowoff = (size_t)cr.orig * (size_t)W;
+        cr.valid = cr.ri != 0;
+        const size_t off = (size_t)cr.orig * (size_t)W + (size_t)w;
         if (!cr.valid) {
-            if (STORE) {
-#pragma unroll
-                for (int k = 0; k < SLOTS; ++k)
-                    if (live[k]) {
-                        if (A.flags) A.flags[rowoff + w0 + k] = 0x80;
-                        if (A.margin) A.margin[rowoff + w0 + k] = __int_as_float(0x7fc00000);
-                    }
+            if (live) {
+                if (SF) A.flags[off] = 0x80;
+                if (SMG) A.margin[off] = __int_as_float(0x7fc00000);
             }
             continue;
         }
-        unsigned bestv = 0xffffffffu;
-        unsigned fpack = 0;
-        float mg[SLOTS];
-#pragma unroll
-        for (int k = 0; k < SLOTS; ++k) {
-            mg[k] = 0.0f;
-            if (live[k]) {
-                while (cr.ri >= __float_as_int(v0[k].x) && p[k] < Rk[k]) {
-                    p[k] += 1;
-                    load_row(A.C.tab, rb[k] + p[k], v0[k], v1[k], v2[k]);
-                }
-                float m;
-                const unsigned f = eval_pair(v0[k], v1[k], v2[k], wr[k], cr, m);
-                mg[k] = m;
-                fpack |= f << (8 * k);
-                if (f == 15u) bestv = min(bestv, rk[k]);
-            }
+        while (cr.ri >= __float_as_int(cur.v0.x) && p < R) {
+            p += 1;
+            cur = load_row(A.C.tab, rb + p);
         }
-        if (STORE) {
-            if (VEC) {
-                if (live[0]) {
-                    if (A.flags)
-                        __stcs(reinterpret_cast<unsigned int*>(A.flags + rowoff + w0), fpack);
-                    if (A.margin)
-                        __stcs(reinterpret_cast<float4*>(A.margin + rowoff + w0),
-                               make_float4(mg[0], mg[SLOTS > 1 ? 1 : 0], mg[SLOTS > 2 ? 2 : 0],
-                                           mg[SLOTS > 3 ? 3 : 0]));
-                }
-            } else {
-#pragma unroll
-                for (int k = 0; k < SLOTS; ++k)
-                    if (live[k]) {
-                        if (A.flags) A.flags[rowoff + w0 + k] = (uint8_t)((fpack >> (8 * k)) & 0xffu);
-                        if (A.margin) __stcs(A.margin + rowoff + w0 + k, mg[k]);
-                    }
-            }
+        float m;
+        const unsigned f = eval_pair(cur.v0, cur.v1, cur.v2, wr, cr, m);
+        if (live) {
+            if (SF) A.flags[off] = (uint8_t)f;
+            if (SMG) __stcs(A.margin + off, m);
         }
-        if (A.best) {
-            bestv = __reduce_min_sync(FULL, bestv);
-            if (lane == 0 && bestv != 0xffffffffu) atomicMin(A.best + cr.orig, bestv);
+        if (ARG) {
+            unsigned kmin = (f == 15u) ? rank : 0xffffffffu;
+            kmin = __reduce_min_sync(FULL, kmin);
+            if (lane == 0 && kmin != 0xffffffffu) atomicMin(A.best + cr.orig, kmin);
         }
     }
+}
+
+template <int SLOTS, bool SF, bool SMG, bool ARG>
+static cudaError_t launch_vec(const ScoreArgs& A0, cudaStream_t st)
+{
+    VecArgs A;
+    A.C = A0.C;
+    A.cand = reinterpret_cast<const float4*>(A0.cand);
+    A.n_cand = A0.n_cand;
+    A.flags = A0.flags;
+    A.margin = A0.margin;
+    A.best = A0.best;
+    A.tiles = (A.C.W + SCORE_WARPS * 32 * SLOTS - 1) / (SCORE_WARPS * 32 * SLOTS);
+    const size_t smem = sizeof(ScoreSmem<SLOTS>);
+    static int per_sm = 0, sms = 0;  // occupancy of this instantiation (per process)
+    if (per_sm == 0) {
+        cudaError_t e = cudaFuncSetAttribute(k_score<SLOTS, SF, SMG, ARG>,
+                                             cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+        if (e != cudaSuccess) return e;
+        int dev = 0;
+        cudaGetDevice(&dev);
+        cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+        e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, k_score<SLOTS, SF, SMG, ARG>,
+                                                          SCORE_WARPS * 32, smem);
+        if (e != cudaSuccess || per_sm < 1) per_sm = 1;
+    }
+    // one wave: per_tile CTAs share each worker tile's candidates equally
+    const int wave = per_sm * sms;
+    int per_tile = wave / A.tiles;
+    if (per_tile < 1) per_tile = 1;
+    const int max_parts = (A.n_cand + 63) / 64;  // at least 64 candidates per CTA
+    if (per_tile > max_parts) per_tile = max_parts;
+    A.per_tile = per_tile;
+    k_score<SLOTS, SF, SMG, ARG><<<A.tiles * per_tile, SCORE_WARPS * 32, smem, st>>>(A);
+    return cudaGetLastError();
+}
+
+template <bool SF, bool SMG, bool ARG>
+static void launch_scalar(const ScoreArgs& A0, cudaStream_t st)
+{
+    ScoreArgs A = A0;
+    A.tiles = (A.C.W + 31) / 32;
+    const int units = A.tiles * A.chunks;
+    k_score_scalar<SF, SMG, ARG><<<(units + SCORE_WARPS - 1) / SCORE_WARPS, SCORE_WARPS * 32, 0, st>>>(A);
 }
 
 __global__ void k_finalize(DevParams P, int n, const int32_t* __restrict__ in,
@@ -264,7 +546,7 @@ cudaError_t launch_score(const DevParams& P, const ClusterDev& C, int n, const i
         if (e != cudaSuccess) return e;
         k_cand_count<<<nb, tb, 0, st>>>(P, n, in, pred, wait, B.hist, B.best);
         k_scan_hist<<<1, SCAN_THREADS, 0, st>>>(B.hist, P.K + 1);
-        k_cand_scatter<<<nb, tb, 0, st>>>(P, n, in, pred, wait, B.hist, B.sorted);
+        k_cand_scatter<<<nb, tb, 0, st>>>(P, n, C.W, in, pred, wait, B.hist, B.sorted);
         e = cudaGetLastError();
         if (e != cudaSuccess) return e;
 
@@ -276,22 +558,28 @@ cudaError_t launch_score(const DevParams& P, const ClusterDev& C, int n, const i
         A.margin = margin;
         A.best = argbest ? B.best : nullptr;
         A.chunks = (n + SCORE_CHUNK - 1) / SCORE_CHUNK;
-        const bool store = flags || margin;
         if (ev0) cudaEventRecord(ev0, st);
         const bool vec = (C.W % 4 == 0) && (((uintptr_t)flags & 3) == 0) &&
                          (((uintptr_t)margin & 15) == 0);
-        if (store && vec) {
-            A.tiles = (C.W + 127) / 128;
-            const int units = A.tiles * A.chunks;
-            k_score<4, true, true><<<(units + SCORE_WARPS - 1) / SCORE_WARPS, SCORE_WARPS * 32, 0, st>>>(A);
-        } else if (store) {
-            A.tiles = (C.W + 31) / 32;
-            const int units = A.tiles * A.chunks;
-            k_score<1, true, false><<<(units + SCORE_WARPS - 1) / SCORE_WARPS, SCORE_WARPS * 32, 0, st>>>(A);
+        constexpr int S = ALADDIN_SCORE_SLOTS;
+        const bool sf = flags != nullptr, smg = margin != nullptr, arg = argbest != nullptr;
+        if (vec) {
+            if (sf && smg && arg) e = launch_vec<S, true, true, true>(A, st);
+            else if (sf && smg) e = launch_vec<S, true, true, false>(A, st);
+            else if (sf && arg) e = launch_vec<S, true, false, true>(A, st);
+            else if (smg && arg) e = launch_vec<S, false, true, true>(A, st);
+            else if (sf) e = launch_vec<S, true, false, false>(A, st);
+            else if (smg) e = launch_vec<S, false, true, false>(A, st);
+            else e = launch_vec<S, false, false, true>(A, st);
+            if (e != cudaSuccess) return e;
         } else {
-            A.tiles = (C.W + 127) / 128;
-            const int units = A.tiles * A.chunks;
-            k_score<4, false, false><<<(units + SCORE_WARPS - 1) / SCORE_WARPS, SCORE_WARPS * 32, 0, st>>>(A);
+            if (sf && smg && arg) launch_scalar<true, true, true>(A, st);
+            else if (sf && smg) launch_scalar<true, true, false>(A, st);
+            else if (sf && arg) launch_scalar<true, false, true>(A, st);
+            else if (smg && arg) launch_scalar<false, true, true>(A, st);
+            else if (sf) launch_scalar<true, false, false>(A, st);
+            else if (smg) launch_scalar<false, true, false>(A, st);
+            else launch_scalar<false, false, true>(A, st);
         }
         if (ev1) cudaEventRecord(ev1, st);
         e = cudaGetLastError();

@@ -49,39 +49,47 @@ cudaError_t launch_build(const DevParams& P, const ClusterDev& C, const int32_t*
 }
 
 // rank[w] = number of workers ordered before w: larger key, or equal key and
-// smaller index (a stable descending sort). Keys are tiled through shared
-// memory; O(W^2) comparisons, each thread one worker.
+// smaller index (a stable descending sort by capacity_norm). A 2-D grid of
+// CTAs counts, for a tile of 256 workers, the workers of one 1024-key chunk
+// that precede each of them (integer compares on keys staged in shared
+// memory) and adds the count to rank[w]; k_order then inverts the ranks.
 constexpr int RANK_TILE = 256;
+constexpr int RANK_CHUNK = 1024;
 
-__global__ void __launch_bounds__(RANK_TILE) k_rank(ClusterDev C)
+__global__ void __launch_bounds__(RANK_TILE) k_rank_count(ClusterDev C)
 {
-    __shared__ double ks[RANK_TILE];
+    __shared__ unsigned long long ks[RANK_CHUNK];
     const int w = blockIdx.x * RANK_TILE + threadIdx.x;
-    const double kw = w < C.W ? C.key[w] : 0.0;
+    const int v0 = blockIdx.y * RANK_CHUNK;
+    const int lim = min(RANK_CHUNK, C.W - v0);
+    for (int i = threadIdx.x; i < lim; i += RANK_TILE) ks[i] = C.key[v0 + i];
+    __syncthreads();
+    if (w >= C.W) return;
+    const unsigned long long kw = C.key[w];
     int cnt = 0;
-    for (int t0 = 0; t0 < C.W; t0 += RANK_TILE) {
-        const int v = t0 + threadIdx.x;
-        ks[threadIdx.x] = v < C.W ? C.key[v] : -2.0;
-        __syncthreads();
-        const int lim = min(RANK_TILE, C.W - t0);
-        for (int i = 0; i < lim; ++i) {
-            const double kv = ks[i];
-            const int vi = t0 + i;
-            cnt += (kv > kw) || (kv == kw && vi < w);
-        }
-        __syncthreads();
+    for (int i = 0; i < lim; ++i) {
+        const unsigned long long kv = ks[i];
+        cnt += (kv > kw) || (kv == kw && v0 + i < w);
     }
-    if (w < C.W) {
-        C.rank[w] = cnt;
-        C.order[cnt] = w;
-        C.wrec[w].w = __int_as_float(cnt);
-    }
+    if (cnt) atomicAdd(&C.rank[w], cnt);
+}
+
+__global__ void k_order(ClusterDev C)
+{
+    const int w = blockIdx.x * blockDim.x + threadIdx.x;
+    if (w >= C.W) return;
+    const int r = C.rank[w];
+    C.order[r] = w;
+    C.wrec[w].w = __int_as_float(r);
 }
 
 cudaError_t launch_rank(const ClusterDev& C, cudaStream_t st)
 {
-    const int blocks = (C.W + RANK_TILE - 1) / RANK_TILE;
-    k_rank<<<blocks, RANK_TILE, 0, st>>>(C);
+    cudaError_t e = cudaMemsetAsync(C.rank, 0, sizeof(int32_t) * (size_t)C.W, st);
+    if (e != cudaSuccess) return e;
+    dim3 grid((C.W + RANK_TILE - 1) / RANK_TILE, (C.W + RANK_CHUNK - 1) / RANK_CHUNK);
+    k_rank_count<<<grid, RANK_TILE, 0, st>>>(C);
+    k_order<<<(C.W + 255) / 256, 256, 0, st>>>(C);
     return cudaGetLastError();
 }
 
