@@ -115,6 +115,14 @@ __device__ __forceinline__ Row load_row(const float4* __restrict__ tab, long lon
     return r;
 }
 
+// Ask L1 to hold the row (48 bytes: up to two 128-byte lines).
+__device__ __forceinline__ void prefetch_row(const float4* tab, long long row)
+{
+    const char* b = reinterpret_cast<const char*>(tab + row * ROW_F4);
+    asm volatile("prefetch.global.L1 [%0];" ::"l"(b));
+    asm volatile("prefetch.global.L1 [%0];" ::"l"(b + 47));
+}
+
 __device__ __forceinline__ unsigned prmt(unsigned a, unsigned b, unsigned sel)
 {
     unsigned d;
@@ -142,13 +150,20 @@ __device__ __forceinline__ unsigned pack_flags(const float (&d)[4][SLOTS])
         } else {
             S = prmt(__float_as_uint(d[g][0]), 0u, 0x000bu);
         }
-        acc |= ~S & (0x01010101u << g);
+        const unsigned mask = SLOTS == 4 ? 0x01010101u : (SLOTS == 2 ? 0x0101u : 0x01u);
+        acc |= ~S & (mask << g);
     }
-    return SLOTS == 4 ? acc : (SLOTS == 2 ? (acc & 0xffffu) : (acc & 0xffu));
+    return acc;
 }
 
 #ifndef ALADDIN_SCORE_SLOTS
-#define ALADDIN_SCORE_SLOTS 2
+#define ALADDIN_SCORE_SLOTS 4
+#endif
+#ifndef ALADDIN_SCORE_PF
+#define ALADDIN_SCORE_PF 1
+#endif
+#ifndef ALADDIN_SCORE_MINB
+#define ALADDIN_SCORE_MINB 4
 #endif
 constexpr int CHUNK = 256;               // candidates per staged chunk
 constexpr long long WAIT_LIMIT = 1ll << 26;  // mbarrier polls before giving up
@@ -215,7 +230,7 @@ struct __align__(16) ScoreSmem {
 };
 
 template <int SLOTS, bool SF, bool SMG, bool ARG>
-__global__ void __launch_bounds__(SCORE_WARPS * 32) k_score(VecArgs A)
+__global__ void __launch_bounds__(SCORE_WARPS * 32, ALADDIN_SCORE_MINB) k_score(VecArgs A)
 {
     extern __shared__ __align__(16) unsigned char smraw[];
     ScoreSmem<SLOTS>& sm = *reinterpret_cast<ScoreSmem<SLOTS>*>(smraw);
@@ -245,15 +260,18 @@ __global__ void __launch_bounds__(SCORE_WARPS * 32) k_score(VecArgs A)
     const int w0 = wbase + lane * SLOTS;
     const bool live = w0 < W;
     const bool warp_live = wbase < W;
-    const bool all_live = wbase + 32 * SLOTS <= W;
     uint8_t* const fbase = SF ? A.flags + (live ? w0 : 0) : nullptr;
     float* const mbase = SMG ? A.margin + (live ? w0 : 0) : nullptr;
 
-    Row cur[SLOTS], nxt[SLOTS];
+    Row cur[SLOTS];
+#if !ALADDIN_SCORE_PF
+    Row nxt[SLOTS];
+#endif
     float inv_s[SLOTS], nZO[SLOTS], ZW[SLOTS];
     unsigned rank[SLOTS];
     int p[SLOTS], R[SLOTS];
     long long rb[SLOTS];
+    int nb = 0;  // smallest next breakpoint over this lane's workers
     bool have_rows = false;
 
     for (int k = 0; k < nchunks; ++k) {
@@ -286,7 +304,11 @@ __global__ void __launch_bounds__(SCORE_WARPS * 32) k_score(VecArgs A)
                     R[s] = __ldg(&A.C.R[wc]);
                     p[s] = find_row(A.C.tab, rb[s], R[s], r_first);
                     cur[s] = load_row(A.C.tab, rb[s] + p[s]);
+#if ALADDIN_SCORE_PF
+                    prefetch_row(A.C.tab, rb[s] + min(p[s] + 1, R[s]));
+#else
                     nxt[s] = load_row(A.C.tab, rb[s] + min(p[s] + 1, R[s]));
+#endif
                     const float4 wr = __ldg(&A.C.wrec[wc]);
                     inv_s[s] = wr.x;
                     nZO[s] = -wr.y;
@@ -294,12 +316,17 @@ __global__ void __launch_bounds__(SCORE_WARPS * 32) k_score(VecArgs A)
                     rank[s] = live ? (unsigned)__float_as_int(wr.w) : 0xffffffffu;
                 }
                 have_rows = true;
+                nb = __float_as_int(cur[0].v0.x);
+#pragma unroll
+                for (int s = 1; s < SLOTS; ++s) nb = min(nb, __float_as_int(cur[s].v0.x));
             }
-            for (int i = 0; i < nc; ++i) {
-                const float4 q0 = cs[3 * i], q1 = cs[3 * i + 1], q2 = cs[3 * i + 2];
+            const float4* q = cs;
+            unsigned* kslot = &sm.kmin[warp][0];
+            for (int i = 0; i < nc; ++i, q += 3, ++kslot) {
+                const float4 q0 = q[0], q1 = q[1], q2 = q[2];
                 const int ri = __float_as_int(q2.x);
-                const size_t off = ((size_t)(unsigned)__float_as_int(q2.w) << 32) |
-                                   (size_t)(unsigned)__float_as_int(q2.z);
+                const unsigned long long off =
+                    ((unsigned long long)__float_as_uint(q2.w) << 32) | __float_as_uint(q2.z);
                 if (ri == 0) {  // invalid candidate (warp-uniform)
                     if (live) {
 #pragma unroll
@@ -308,21 +335,26 @@ __global__ void __launch_bounds__(SCORE_WARPS * 32) k_score(VecArgs A)
                             if (SMG) mbase[off + s] = __int_as_float(0x7fc00000);
                         }
                     }
-                    if (ARG && lane == 0) sm.kmin[warp][i] = 0xffffffffu;
+                    if (ARG) *kslot = 0xffffffffu;
                     continue;
                 }
-                bool need = false;
-#pragma unroll
-                for (int s = 0; s < SLOTS; ++s) need |= ri >= __float_as_int(cur[s].v0.x);
-                if (__any_sync(FULL, need)) {
+                if (__any_sync(FULL, ri >= nb)) {
 #pragma unroll
                     for (int s = 0; s < SLOTS; ++s) {
                         while (ri >= __float_as_int(cur[s].v0.x) && p[s] < R[s]) {
                             p[s] += 1;
+#if ALADDIN_SCORE_PF
+                            cur[s] = load_row(A.C.tab, rb[s] + p[s]);
+                            prefetch_row(A.C.tab, rb[s] + min(p[s] + 1, R[s]));
+#else
                             cur[s] = nxt[s];
                             nxt[s] = load_row(A.C.tab, rb[s] + min(p[s] + 1, R[s]));
+#endif
                         }
                     }
+                    nb = __float_as_int(cur[0].v0.x);
+#pragma unroll
+                    for (int s = 1; s < SLOTS; ++s) nb = min(nb, __float_as_int(cur[s].v0.x));
                 }
                 const float a = q0.x, r = q0.y, inv_r = q0.z, U = q0.w;
                 const float inv_d1 = q1.x, nXd1 = q1.y, inv_d2 = q1.z, Zc = q1.w;
@@ -343,7 +375,7 @@ __global__ void __launch_bounds__(SCORE_WARPS * 32) k_score(VecArgs A)
                     m[s] = fminf(fminf(d[0][s], d[1][s]), fminf(d[2][s], d[3][s]));
                     if (ARG) kmin = min(kmin, (__float_as_uint(m[s]) & 0x80000000u) | rank[s]);
                 }
-                if (all_live || live) {
+                if (live) {
                     if (SF) {
                         const unsigned f = pack_flags<SLOTS>(d);
                         if (SLOTS == 4) __stcs(reinterpret_cast<unsigned int*>(fbase + off), f);
@@ -359,10 +391,7 @@ __global__ void __launch_bounds__(SCORE_WARPS * 32) k_score(VecArgs A)
                         else __stcs(mbase + off, m[0]);
                     }
                 }
-                if (ARG) {
-                    kmin = __reduce_min_sync(FULL, kmin);
-                    sm.kmin[warp][i] = kmin;  // same value from every lane
-                }
+                if (ARG) *kslot = __reduce_min_sync(FULL, kmin);  // same value from every lane
             }
         } else if (ARG) {
             for (int i = tid & 31; i < nc; i += 32) sm.kmin[warp][i] = 0xffffffffu;
