@@ -107,9 +107,12 @@ struct ClusterDev {
 // r_j > rho_p, over s, ongoing ones less the stall's constant part.
 
 // Derived per-candidate values (3 x float4), identical for every worker.
+// Bounds are compared with the prompt length a by subtracting a first, so the
+// a-dependent constants of the candidate carry it: Ua = U - a with
+// U = -c2/k2 - (r + 1)/2, and nXd1a = -X(r)/(k2 r + k1) - a.
 struct __align__(16) CandRec {
-    float a, r, inv_r, U;          // U = -c2/k2 - (r + 1)/2
-    float inv_d1, nXd1, inv_d2, Zc;  // 1/(k2 r + k1), -X(r)/(k2 r + k1), 1/(k2 r), (T_pre - w)/k1
+    float a, r, inv_r, Ua;             // prompt, output, 1/r, U - a
+    float inv_d1, nXd1a, inv_d2, Zc;   // 1/(k2 r + k1), -X(r)/(k2 r + k1) - a, 1/(k2 r), (T_pre - w)/k1
     int32_t ri, orig, valid, pad;
 };
 
@@ -130,14 +133,15 @@ __device__ __forceinline__ CandRec make_cand(const DevParams& P, int32_t in, int
                     w >= 0.0f && w <= 3.0e38f;
     const int32_t r = ok ? pred : 1;
     const float rf = (float)r;
-    c.a = ok ? (float)in : 0.0f;
+    const float a = ok ? (float)in : 0.0f;
+    c.a = a;
     c.r = rf;
     c.inv_r = 1.0f / rf;
-    c.U = -P.c2_over_k2 - 0.5f * (rf + 1.0f);
+    c.Ua = (-P.c2_over_k2 - 0.5f * (rf + 1.0f)) - a;
     const float d1 = P.k2 * rf + P.k1;
     c.inv_d1 = 1.0f / d1;
     const float X = P.c2 * rf + P.k2 * (0.5f * rf * (rf + 1.0f));
-    c.nXd1 = -X * c.inv_d1;
+    c.nXd1a = -X * c.inv_d1 - a;
     c.inv_d2 = 1.0f / (P.k2 * rf);
     c.Zc = (P.T_pre - (ok ? w : 0.0f)) * P.inv_k1;
     c.ri = ok ? r : 0;
@@ -147,21 +151,28 @@ __device__ __forceinline__ CandRec make_cand(const DevParams& P, int32_t in, int
     return c;
 }
 
+// Headroom of one pair per constraint group (bound - a): d[0] KV, d[1] TTFT,
+// d[2] ongoing ATGT, d[3] new ATGT. The flags are the groups with d >= 0 and
+// the margin is min(d).
+__device__ __forceinline__ void pair_headroom(const float4 v0, const float4 v1, const float4 v2,
+                                              const float4 wr, const CandRec& c, float (&d)[4])
+{
+    d[0] = fminf(v0.y - c.a, fmaf(c.r, v0.w, v0.z - c.a));
+    d[1] = fminf(fmaf(c.Zc, wr.x, -wr.y - c.a), wr.z - c.a);
+    d[2] = fminf(v1.w - c.a, fmaf(v2.y, c.inv_d1, c.nXd1a));
+    d[3] = fminf(fminf(v2.x - c.a, fmaf(v2.z, c.inv_d2, c.Ua)),
+                 fmaf(v1.x, c.inv_r, fmaf(v1.z, c.r, c.Ua - v1.y)));
+}
+
 // Bounds of one pair; returns the four flag bits, writes the margin.
 __device__ __forceinline__ unsigned eval_pair(const float4 v0, const float4 v1, const float4 v2,
                                               const float4 wr, const CandRec& c, float& margin)
 {
-    const float kv2 = fmaf(c.r, v0.w, v0.z);
-    const float kvm = fminf(v0.y, kv2);
-    const float tt = fminf(fmaf(c.Zc, wr.x, -wr.y), wr.z);
-    const float ca = fmaf(v1.x, c.inv_r, fmaf(v1.z, c.r, c.U - v1.y));
-    const float s1 = fmaf(v2.y, c.inv_d1, c.nXd1);
-    const float s2 = fmaf(v2.z, c.inv_d2, c.U);
-    const float gon = fminf(v1.w, s1);
-    const float gnew = fminf(fminf(v2.x, s2), ca);
-    margin = fminf(fminf(kvm, tt), fminf(gon, gnew)) - c.a;
-    return (kvm >= c.a ? 1u : 0u) | (tt >= c.a ? 2u : 0u) | (gon >= c.a ? 4u : 0u) |
-           (gnew >= c.a ? 8u : 0u);
+    float d[4];
+    pair_headroom(v0, v1, v2, wr, c, d);
+    margin = fminf(fminf(d[0], d[1]), fminf(d[2], d[3]));
+    return (d[0] >= 0.0f ? 1u : 0u) | (d[1] >= 0.0f ? 2u : 0u) | (d[2] >= 0.0f ? 4u : 0u) |
+           (d[3] >= 0.0f ? 8u : 0u);
 }
 
 // Row index p of worker w containing remaining length r: the first row whose

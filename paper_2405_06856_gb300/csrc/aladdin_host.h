@@ -17,7 +17,7 @@ cudaError_t launch_build(const DevParams& P, const ClusterDev& C, const int32_t*
 cudaError_t launch_rank(const ClusterDev& C, cudaStream_t st);
 
 struct ScoreBuffers {
-    CandRec* sorted;       // [n_cand]
+    float4* sorted;        // [n_cand * 5] sorted candidate records
     int32_t* hist;         // [K + 2]
     unsigned int* best;    // [n_cand]
 };
@@ -27,7 +27,8 @@ struct ScoreBuffers {
 cudaError_t launch_score(const DevParams& P, const ClusterDev& C, int n_cand, const int32_t* in,
                          const int32_t* pred, const float* wait, uint8_t* flags, float* margin,
                          int32_t* argbest, int64_t* kv_peak, float* t_cand, const ScoreBuffers& B,
-                         cudaStream_t st, cudaEvent_t ev0 = nullptr, cudaEvent_t ev1 = nullptr);
+                         bool pend, cudaStream_t st, cudaEvent_t ev0 = nullptr,
+                         cudaEvent_t ev1 = nullptr);
 
 // K4: one greedy round over candidates in index order.
 struct RoundIO {

@@ -122,6 +122,7 @@ struct aladdin_cluster {
     ClusterDev dev;
     int W = 0, cap = 0, rows = 0;
     double t_now = 0.0;
+    bool round_open = false;  // some worker holds requests placed in the open round
     std::vector<void*> owned;
     // scratch and staging (grow-only)
     DevBuf sorted, hist, best;
@@ -442,10 +443,10 @@ int score_impl(aladdin_cluster* cl, int32_t n, const int32_t* in, const int32_t*
         (rc = stage_out(cl->s_kv, kv_peak, pairs, &dkv, &hk)) ||
         (rc = stage_out(cl->s_tc, t_cand, pairs, &dtc, &ht)))
         return rc;
-    CK(cl->sorted.ensure(sizeof(CandRec) * C));
+    CK(cl->sorted.ensure(sizeof(float4) * 5 * C));
     CK(cl->hist.ensure(sizeof(int32_t) * ((size_t)cl->hp.K + 2)));
     CK(cl->best.ensure(sizeof(unsigned int) * C));
-    ScoreBuffers B{cl->sorted.as<CandRec>(), cl->hist.as<int32_t>(), cl->best.as<unsigned int>()};
+    ScoreBuffers B{cl->sorted.as<float4>(), cl->hist.as<int32_t>(), cl->best.as<unsigned int>()};
     cudaEvent_t e0 = nullptr, e1 = nullptr;
     if (cl->timing && (dflags || dmargin || darg)) {
         e0 = cl->take_event();
@@ -457,8 +458,8 @@ int score_impl(aladdin_cluster* cl, int32_t n, const int32_t* in, const int32_t*
             e0 = e1 = nullptr;
         }
     }
-    CK(launch_score(cl->dp, cl->dev, n, din, dpred, dwait, dflags, dmargin, darg, dkv, dtc, B, cl->st,
-                    e0, e1));
+    CK(launch_score(cl->dp, cl->dev, n, din, dpred, dwait, dflags, dmargin, darg, dkv, dtc, B,
+                    cl->round_open, cl->st, e0, e1));
     if (hf) CK(cudaMemcpyAsync(flags, dflags, pairs, cudaMemcpyDeviceToHost, cl->st));
     if (hm) CK(cudaMemcpyAsync(margin, dmargin, sizeof(float) * pairs, cudaMemcpyDeviceToHost, cl->st));
     if (ha) CK(cudaMemcpyAsync(argbest, darg, sizeof(int32_t) * C, cudaMemcpyDeviceToHost, cl->st));
@@ -522,6 +523,7 @@ int aladdin_cluster_load(aladdin_cluster* cl, const int32_t* req_off, const int3
     CK(cudaSetDevice(cl->device));
     int rc = load_requests(cl, req_off, in, gen, pred, tdec_ms);
     if (rc) return rc;
+    cl->round_open = false;
     return refresh_tables(cl);
 }
 
@@ -567,6 +569,7 @@ int aladdin_place_round(aladdin_cluster* cl, int32_t n_cand, const int32_t* in,
     io.status = cl->d_status;
     CK(launch_round(cl->dp, cl->dev, io, cl->st));
     CK(launch_rank(cl->dev, cl->st));
+    cl->round_open = true;
     if (hp) CK(cudaMemcpyAsync(placement, dpl, sizeof(int32_t) * C, cudaMemcpyDeviceToHost, cl->st));
     int status = 0;
     CK(cudaMemcpyAsync(&status, cl->d_status, sizeof(int), cudaMemcpyDeviceToHost, cl->st));
@@ -580,6 +583,7 @@ int aladdin_cluster_advance(aladdin_cluster* cl, double dt_ms, double* stats)
     CK(cudaSetDevice(cl->device));
     CK(launch_advance(cl->dp, cl->dev, cl->t_now, dt_ms, cl->d_stats, nullptr, cl->st));
     cl->t_now += dt_ms;
+    cl->round_open = false;
     int rc = refresh_tables(cl);
     if (rc) return rc;
     if (stats) {

@@ -73,33 +73,41 @@ __global__ void __launch_bounds__(SCAN_THREADS) k_scan_hist(int32_t* hist, int l
     }
 }
 
-// Sorted record: the CandRec constants, with the third float4 holding
-// {valid ? predicted output : 0, original index, low and high words of
-// index * W} (the start of the candidate's output row).
-__global__ void k_cand_scatter(DevParams P, int n, int W, const int32_t* __restrict__ in,
-                               const int32_t* __restrict__ pred, const float* __restrict__ wait,
-                               int32_t* cursor, CandRec* sorted)
-{
-    const int c = blockIdx.x * blockDim.x + threadIdx.x;
-    if (c >= n) return;
-    CandRec rec = make_cand(P, in[c], pred[c], wait ? wait[c] : 0.0f, c);
-    const int pos = atomicAdd(&cursor[rec.valid ? rec.ri : 0], 1);
-    const unsigned long long rowoff = (unsigned long long)c * (unsigned long long)W;
-    rec.ri = rec.valid ? rec.ri : 0;
-    rec.valid = (int32_t)(unsigned)(rowoff & 0xffffffffull);
-    rec.pad = (int32_t)(unsigned)(rowoff >> 32);
-    sorted[pos] = rec;
-}
+// Sorted record (5 x float4), the per-candidate constants stored twice so that
+// a 16-byte shared-memory load yields ready-made operand pairs for the packed
+// f32x2 arithmetic: {a, a, r, r}, {1/r, 1/r, Ua, Ua}, {inv_d1, inv_d1, nXd1a,
+// nXd1a}, {inv_d2, inv_d2, Zc, Zc}, {valid ? r : 0, original index, low and
+// high words of index * W (the start of the candidate's output row)}.
+constexpr int REC_F4 = 5;
 
 struct ScoreArgs {
     ClusterDev C;
-    const CandRec* __restrict__ cand;
+    const float4* __restrict__ cand;
     int n_cand;
     uint8_t* flags;
     float* margin;
     unsigned int* best;
     int tiles, chunks;
 };
+
+__global__ void k_cand_scatter(DevParams P, int n, int W, const int32_t* __restrict__ in,
+                               const int32_t* __restrict__ pred, const float* __restrict__ wait,
+                               int32_t* cursor, float4* sorted)
+{
+    const int c = blockIdx.x * blockDim.x + threadIdx.x;
+    if (c >= n) return;
+    const CandRec rec = make_cand(P, in[c], pred[c], wait ? wait[c] : 0.0f, c);
+    const int pos = atomicAdd(&cursor[rec.valid ? rec.ri : 0], 1);
+    const unsigned long long rowoff = (unsigned long long)c * (unsigned long long)W;
+    float4* o = sorted + (size_t)pos * REC_F4;
+    o[0] = make_float4(rec.a, rec.a, rec.r, rec.r);
+    o[1] = make_float4(rec.inv_r, rec.inv_r, rec.Ua, rec.Ua);
+    o[2] = make_float4(rec.inv_d1, rec.inv_d1, rec.nXd1a, rec.nXd1a);
+    o[3] = make_float4(rec.inv_d2, rec.inv_d2, rec.Zc, rec.Zc);
+    o[4] = make_float4(__int_as_float(rec.valid ? rec.ri : 0), __int_as_float(c),
+                       __uint_as_float((unsigned)(rowoff & 0xffffffffull)),
+                       __uint_as_float((unsigned)(rowoff >> 32)));
+}
 
 struct Row {
     float4 v0, v1, v2;
@@ -130,8 +138,33 @@ __device__ __forceinline__ unsigned prmt(unsigned a, unsigned b, unsigned sel)
     return d;
 }
 
+// Packed pairs of fp32 held in one 64-bit register (Blackwell f32x2
+// arithmetic: two independent round-to-nearest operations, bit-identical to
+// the scalar ones). Low word = slot 2j, high word = slot 2j + 1.
+typedef unsigned long long f2x;
+
+__device__ __forceinline__ f2x fma2(f2x a, f2x b, f2x c)
+{
+    f2x d;
+    asm("fma.rn.f32x2 %0, %1, %2, %3;" : "=l"(d) : "l"(a), "l"(b), "l"(c));
+    return d;
+}
+__device__ __forceinline__ f2x sub2(f2x a, f2x b)
+{
+    f2x d;
+    asm("sub.rn.f32x2 %0, %1, %2;" : "=l"(d) : "l"(a), "l"(b));
+    return d;
+}
+__device__ __forceinline__ float lo(f2x v) { return __uint_as_float((unsigned)v); }
+__device__ __forceinline__ float hi(f2x v) { return __uint_as_float((unsigned)(v >> 32)); }
+__device__ __forceinline__ f2x set_half(f2x v, int h, float x)
+{
+    const f2x b = (f2x)__float_as_uint(x);
+    return h ? ((v & 0xffffffffull) | (b << 32)) : ((v & 0xffffffff00000000ull) | b);
+}
+
 // Flag bytes of SLOTS pairs from the sign bits of their group headrooms
-// d[g][k] = bound_g - a (bit g of byte k set iff d[g][k] >= 0). prmt with the
+// d[g][k] (bit g of byte k set iff d[g][k] >= 0). prmt with the
 // sign-replicate selector (bit 3 of a selector nibble) turns the top byte of
 // each headroom into 0x00 / 0xff, one byte per slot.
 template <int SLOTS>
@@ -145,12 +178,10 @@ __device__ __forceinline__ unsigned pack_flags(const float (&d)[4][SLOTS])
             const unsigned t1 = prmt(__float_as_uint(d[g][0]), __float_as_uint(d[g][1 % SLOTS]), 0x00fbu);
             const unsigned t2 = prmt(__float_as_uint(d[g][2 % SLOTS]), __float_as_uint(d[g][3 % SLOTS]), 0x00fbu);
             S = prmt(t1, t2, 0x5410u);
-        } else if (SLOTS == 2) {
-            S = prmt(__float_as_uint(d[g][0]), __float_as_uint(d[g][1 % SLOTS]), 0x00fbu);
         } else {
-            S = prmt(__float_as_uint(d[g][0]), 0u, 0x000bu);
+            S = prmt(__float_as_uint(d[g][0]), __float_as_uint(d[g][1 % SLOTS]), 0x00fbu);
         }
-        const unsigned mask = SLOTS == 4 ? 0x01010101u : (SLOTS == 2 ? 0x0101u : 0x01u);
+        const unsigned mask = SLOTS == 4 ? 0x01010101u : 0x0101u;
         acc |= ~S & (mask << g);
     }
     return acc;
@@ -159,13 +190,10 @@ __device__ __forceinline__ unsigned pack_flags(const float (&d)[4][SLOTS])
 #ifndef ALADDIN_SCORE_SLOTS
 #define ALADDIN_SCORE_SLOTS 4
 #endif
-#ifndef ALADDIN_SCORE_PF
-#define ALADDIN_SCORE_PF 1
-#endif
 #ifndef ALADDIN_SCORE_MINB
 #define ALADDIN_SCORE_MINB 4
 #endif
-constexpr int CHUNK = 256;               // candidates per staged chunk
+constexpr int CHUNK = 256;                   // candidates per staged chunk
 constexpr long long WAIT_LIMIT = 1ll << 26;  // mbarrier polls before giving up
 constexpr unsigned ERR_TIMEOUT_BIT = 4u;
 
@@ -212,7 +240,7 @@ __device__ __forceinline__ bool mbar_wait(unsigned long long* bar, unsigned pari
 
 struct VecArgs {
     ClusterDev C;
-    const float4* __restrict__ cand;   // sorted records, 3 float4 each
+    const float4* __restrict__ cand;   // sorted records, REC_F4 float4 each
     int n_cand;
     uint8_t* flags;
     float* margin;
@@ -221,24 +249,81 @@ struct VecArgs {
     int per_tile;    // CTAs per tile
 };
 
-template <int SLOTS>
 struct __align__(16) ScoreSmem {
-    float4 cs[2][CHUNK * 3];
+    float4 cs[2][CHUNK * REC_F4];
     unsigned kmin[SCORE_WARPS][CHUNK];
     unsigned long long bar[2];
     int stop;
 };
 
-template <int SLOTS, bool SF, bool SMG, bool ARG>
+// Worker state of one lane for a pair of slots (low word: slot 2j, high
+// word: slot 2j + 1).
+template <bool PEND>
+struct SlotPair {
+    f2x kvB1, kvE, np1n, b0n, b1, nh, pmA, Gt, inv_s, nZO;
+    f2x pmAp, Gpt, ZW;  // used only with requests of an open round (PEND)
+};
+
+template <bool PEND>
+__device__ __forceinline__ void set_row_slot(SlotPair<PEND>& q, int h, const Row& r)
+{
+    q.kvB1 = set_half(q.kvB1, h, r.v0.y);
+    q.kvE = set_half(q.kvE, h, r.v0.z);
+    q.np1n = set_half(q.np1n, h, r.v0.w);
+    q.b0n = set_half(q.b0n, h, r.v1.x);
+    q.b1 = set_half(q.b1, h, r.v1.y);
+    q.nh = set_half(q.nh, h, r.v1.z);
+    q.pmA = set_half(q.pmA, h, r.v1.w);
+    q.Gt = set_half(q.Gt, h, r.v2.y);
+    if (PEND) {
+        q.pmAp = set_half(q.pmAp, h, r.v2.x);
+        q.Gpt = set_half(q.Gpt, h, r.v2.z);
+    }
+}
+
+// Scalar worker state of one lane slot.
+template <bool PEND>
+struct SlotS {
+    float kvB1, kvE, np1n, b0n, b1, nh, pmA, Gt, inv_s, nZO;
+    float pmAp, Gpt, ZW;  // used only with requests of an open round (PEND)
+};
+
+template <bool PEND>
+__device__ __forceinline__ void set_row_s(SlotS<PEND>& q, const Row& r)
+{
+    q.kvB1 = r.v0.y;
+    q.kvE = r.v0.z;
+    q.np1n = r.v0.w;
+    q.b0n = r.v1.x;
+    q.b1 = r.v1.y;
+    q.nh = r.v1.z;
+    q.pmA = r.v1.w;
+    q.Gt = r.v2.y;
+    if (PEND) {
+        q.pmAp = r.v2.x;
+        q.Gpt = r.v2.z;
+    }
+}
+
+#ifndef ALADDIN_SCORE_F32X2
+#define ALADDIN_SCORE_F32X2 0
+#endif
+
+// One CTA = SCORE_WARPS warps x 32 lanes x SLOTS consecutive workers and one
+// contiguous range of sorted candidates (one wave of CTAs, equal shares).
+// Requires W % 4 == 0 and 16-byte aligned outputs. PEND: some worker holds
+// requests placed in an open round (pending prefill and its TTFT/ATGT bounds).
+template <int SLOTS, bool SF, bool SMG, bool ARG, bool PEND>
 __global__ void __launch_bounds__(SCORE_WARPS * 32, ALADDIN_SCORE_MINB) k_score(VecArgs A)
 {
+    static_assert(SLOTS == 2 || SLOTS == 4, "slots come in pairs");
+    constexpr int NP = SLOTS / 2;
     extern __shared__ __align__(16) unsigned char smraw[];
-    ScoreSmem<SLOTS>& sm = *reinterpret_cast<ScoreSmem<SLOTS>*>(smraw);
+    ScoreSmem& sm = *reinterpret_cast<ScoreSmem*>(smraw);
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
     const int W = A.C.W;
     const int tile = blockIdx.x % A.tiles;
     const int part = blockIdx.x / A.tiles;
-    // this CTA's candidate range [cb, ce)
     const int cb = (int)(((long long)A.n_cand * part) / A.per_tile);
     const int ce = (int)(((long long)A.n_cand * (part + 1)) / A.per_tile);
     if (cb >= ce) return;  // CTA-uniform
@@ -253,7 +338,7 @@ __global__ void __launch_bounds__(SCORE_WARPS * 32, ALADDIN_SCORE_MINB) k_score(
     __syncthreads();
     if (tid == 0) {
         const int n0 = min(CHUNK, ce - cb);
-        tma_load(sm.cs[0], A.cand + (size_t)cb * 3, (unsigned)n0 * 48u, &sm.bar[0]);
+        tma_load(sm.cs[0], A.cand + (size_t)cb * REC_F4, (unsigned)n0 * (REC_F4 * 16u), &sm.bar[0]);
     }
 
     const int wbase = (tile * SCORE_WARPS + warp) * 32 * SLOTS;
@@ -262,15 +347,15 @@ __global__ void __launch_bounds__(SCORE_WARPS * 32, ALADDIN_SCORE_MINB) k_score(
     const bool warp_live = wbase < W;
     uint8_t* const fbase = SF ? A.flags + (live ? w0 : 0) : nullptr;
     float* const mbase = SMG ? A.margin + (live ? w0 : 0) : nullptr;
+    const int last_row = A.C.rows - 1;
 
-    Row cur[SLOTS];
-#if !ALADDIN_SCORE_PF
-    Row nxt[SLOTS];
+#if ALADDIN_SCORE_F32X2
+    SlotPair<PEND> st[NP];
+#else
+    SlotS<PEND> ss[SLOTS];
 #endif
-    float inv_s[SLOTS], nZO[SLOTS], ZW[SLOTS];
+    int rnext[SLOTS], p[SLOTS], wk[SLOTS];
     unsigned rank[SLOTS];
-    int p[SLOTS], R[SLOTS];
-    long long rb[SLOTS];
     int nb = 0;  // smallest next breakpoint over this lane's workers
     bool have_rows = false;
 
@@ -281,7 +366,8 @@ __global__ void __launch_bounds__(SCORE_WARPS * 32, ALADDIN_SCORE_MINB) k_score(
         if (tid == 0 && k + 1 < nchunks) {
             const int c1 = c0 + CHUNK;
             const int n1 = min(CHUNK, ce - c1);
-            tma_load(sm.cs[buf ^ 1], A.cand + (size_t)c1 * 3, (unsigned)n1 * 48u, &sm.bar[buf ^ 1]);
+            tma_load(sm.cs[buf ^ 1], A.cand + (size_t)c1 * REC_F4, (unsigned)n1 * (REC_F4 * 16u),
+                     &sm.bar[buf ^ 1]);
         }
         if (!mbar_wait(&sm.bar[buf], (unsigned)((k >> 1) & 1))) {
             if (lane == 0) atomicOr(A.C.err, ERR_TIMEOUT_BIT);
@@ -289,44 +375,47 @@ __global__ void __launch_bounds__(SCORE_WARPS * 32, ALADDIN_SCORE_MINB) k_score(
         }
         __syncthreads();
         if (sm.stop) {
-            // let the other buffer's copy (if any) land before the CTA exits
             if (tid == 0 && k + 1 < nchunks) mbar_wait(&sm.bar[buf ^ 1], (unsigned)(((k + 1) >> 1) & 1));
             return;
         }
         const float4* cs = sm.cs[buf];
         if (warp_live) {
             if (!have_rows) {
-                const int r_first = __float_as_int(cs[2].x);
+                const int r_first = __float_as_int(cs[4].x);
 #pragma unroll
                 for (int s = 0; s < SLOTS; ++s) {
-                    const int wc = live ? w0 + s : W - 1;
-                    rb[s] = (long long)wc * A.C.rows;
-                    R[s] = __ldg(&A.C.R[wc]);
-                    p[s] = find_row(A.C.tab, rb[s], R[s], r_first);
-                    cur[s] = load_row(A.C.tab, rb[s] + p[s]);
-#if ALADDIN_SCORE_PF
-                    prefetch_row(A.C.tab, rb[s] + min(p[s] + 1, R[s]));
+                    wk[s] = live ? w0 + s : W - 1;
+                    const long long rb = (long long)wk[s] * A.C.rows;
+                    p[s] = find_row(A.C.tab, rb, __ldg(&A.C.R[wk[s]]), r_first);
+                    const Row r = load_row(A.C.tab, rb + p[s]);
+                    prefetch_row(A.C.tab, rb + min(p[s] + 1, last_row));
+                    rnext[s] = __float_as_int(r.v0.x);
+                    const float4 wr = __ldg(&A.C.wrec[wk[s]]);
+#if ALADDIN_SCORE_F32X2
+                    set_row_slot<PEND>(st[s >> 1], s & 1, r);
+                    st[s >> 1].inv_s = set_half(st[s >> 1].inv_s, s & 1, wr.x);
+                    st[s >> 1].nZO = set_half(st[s >> 1].nZO, s & 1, -wr.y);
+                    st[s >> 1].ZW = set_half(st[s >> 1].ZW, s & 1, wr.z);
 #else
-                    nxt[s] = load_row(A.C.tab, rb[s] + min(p[s] + 1, R[s]));
+                    set_row_s<PEND>(ss[s], r);
+                    ss[s].inv_s = wr.x;
+                    ss[s].nZO = -wr.y;
+                    ss[s].ZW = wr.z;
 #endif
-                    const float4 wr = __ldg(&A.C.wrec[wc]);
-                    inv_s[s] = wr.x;
-                    nZO[s] = -wr.y;
-                    ZW[s] = wr.z;
                     rank[s] = live ? (unsigned)__float_as_int(wr.w) : 0xffffffffu;
                 }
-                have_rows = true;
-                nb = __float_as_int(cur[0].v0.x);
+                nb = rnext[0];
 #pragma unroll
-                for (int s = 1; s < SLOTS; ++s) nb = min(nb, __float_as_int(cur[s].v0.x));
+                for (int s = 1; s < SLOTS; ++s) nb = min(nb, rnext[s]);
+                have_rows = true;
             }
             const float4* q = cs;
             unsigned* kslot = &sm.kmin[warp][0];
-            for (int i = 0; i < nc; ++i, q += 3, ++kslot) {
-                const float4 q0 = q[0], q1 = q[1], q2 = q[2];
-                const int ri = __float_as_int(q2.x);
+            for (int i = 0; i < nc; ++i, q += REC_F4, ++kslot) {
+                const float4 q4 = q[4];
+                const int ri = __float_as_int(q4.x);
                 const unsigned long long off =
-                    ((unsigned long long)__float_as_uint(q2.w) << 32) | __float_as_uint(q2.z);
+                    ((unsigned long long)__float_as_uint(q4.w) << 32) | __float_as_uint(q4.z);
                 if (ri == 0) {  // invalid candidate (warp-uniform)
                     if (live) {
 #pragma unroll
@@ -341,68 +430,115 @@ __global__ void __launch_bounds__(SCORE_WARPS * 32, ALADDIN_SCORE_MINB) k_score(
                 if (__any_sync(FULL, ri >= nb)) {
 #pragma unroll
                     for (int s = 0; s < SLOTS; ++s) {
-                        while (ri >= __float_as_int(cur[s].v0.x) && p[s] < R[s]) {
+                        while (ri >= rnext[s] && p[s] < last_row) {
                             p[s] += 1;
-#if ALADDIN_SCORE_PF
-                            cur[s] = load_row(A.C.tab, rb[s] + p[s]);
-                            prefetch_row(A.C.tab, rb[s] + min(p[s] + 1, R[s]));
+                            const long long rb = (long long)wk[s] * A.C.rows;
+                            const Row r = load_row(A.C.tab, rb + p[s]);
+                            prefetch_row(A.C.tab, rb + min(p[s] + 1, last_row));
+                            rnext[s] = __float_as_int(r.v0.x);
+#if ALADDIN_SCORE_F32X2
+                            set_row_slot<PEND>(st[s >> 1], s & 1, r);
 #else
-                            cur[s] = nxt[s];
-                            nxt[s] = load_row(A.C.tab, rb[s] + min(p[s] + 1, R[s]));
+                            set_row_s<PEND>(ss[s], r);
 #endif
                         }
                     }
-                    nb = __float_as_int(cur[0].v0.x);
+                    nb = rnext[0];
 #pragma unroll
-                    for (int s = 1; s < SLOTS; ++s) nb = min(nb, __float_as_int(cur[s].v0.x));
+                    for (int s = 1; s < SLOTS; ++s) nb = min(nb, rnext[s]);
                 }
-                const float a = q0.x, r = q0.y, inv_r = q0.z, U = q0.w;
-                const float inv_d1 = q1.x, nXd1 = q1.y, inv_d2 = q1.z, Zc = q1.w;
+#if ALADDIN_SCORE_F32X2
+                const ulonglong2* qq = reinterpret_cast<const ulonglong2*>(q);
+                const ulonglong2 q0 = qq[0], q1 = qq[1], q2 = qq[2], q3 = qq[3];
+                const f2x a2 = q0.x, r2 = q0.y, ir2 = q1.x, Ua2 = q1.y;
+                const f2x id1 = q2.x, nX2 = q2.y, id2 = q3.x, Zc2 = q3.y;
+                float d[4][SLOTS], m[SLOTS];
+                unsigned kmin = 0xffffffffu;
+#pragma unroll
+                for (int j = 0; j < NP; ++j) {
+                    const SlotPair<PEND>& t = st[j];
+                    const f2x kv1 = sub2(t.kvB1, a2);
+                    const f2x kv2 = fma2(r2, t.np1n, sub2(t.kvE, a2));
+                    const f2x tt = fma2(Zc2, t.inv_s, sub2(t.nZO, a2));
+                    const f2x on1 = sub2(t.pmA, a2);
+                    const f2x on2 = fma2(t.Gt, id1, nX2);
+                    const f2x ca = fma2(t.b0n, ir2, fma2(t.nh, r2, sub2(Ua2, t.b1)));
+                    f2x ttw = 0, nw1 = 0, nw2 = 0;
+                    if (PEND) {
+                        ttw = sub2(t.ZW, a2);
+                        nw1 = sub2(t.pmAp, a2);
+                        nw2 = fma2(t.Gpt, id2, Ua2);
+                    }
+#pragma unroll
+                    for (int h = 0; h < 2; ++h) {
+                        const int s = 2 * j + h;
+                        const float e_kv1 = h ? hi(kv1) : lo(kv1), e_kv2 = h ? hi(kv2) : lo(kv2);
+                        const float e_tt = h ? hi(tt) : lo(tt);
+                        const float e_on1 = h ? hi(on1) : lo(on1), e_on2 = h ? hi(on2) : lo(on2);
+                        const float e_ca = h ? hi(ca) : lo(ca);
+                        d[0][s] = fminf(e_kv1, e_kv2);
+                        d[2][s] = fminf(e_on1, e_on2);
+                        if (PEND) {
+                            d[1][s] = fminf(e_tt, h ? hi(ttw) : lo(ttw));
+                            d[3][s] = fminf(fminf(h ? hi(nw1) : lo(nw1), h ? hi(nw2) : lo(nw2)), e_ca);
+                        } else {
+                            d[1][s] = e_tt;
+                            d[3][s] = e_ca;
+                        }
+                        m[s] = fminf(fminf(d[0][s], d[1][s]), fminf(d[2][s], d[3][s]));
+                        if (ARG) kmin = min(kmin, (__float_as_uint(m[s]) & 0x80000000u) | rank[s]);
+                    }
+                }
+#else
+                const float4 q0 = q[0], q1 = q[1], q2 = q[2], q3 = q[3];
+                const float a = q0.x, r = q0.z, ir = q1.x, Ua = q1.z;
+                const float id1 = q2.x, nX = q2.z, id2 = q3.x, Zc = q3.z;
                 float d[4][SLOTS], m[SLOTS];
                 unsigned kmin = 0xffffffffu;
 #pragma unroll
                 for (int s = 0; s < SLOTS; ++s) {
-                    const Row& c = cur[s];
-                    const float kvm = fminf(c.v0.y, fmaf(r, c.v0.w, c.v0.z));
-                    const float tt = fminf(fmaf(Zc, inv_s[s], nZO[s]), ZW[s]);
-                    const float ca = fmaf(c.v1.x, inv_r, fmaf(c.v1.z, r, U - c.v1.y));
-                    const float gon = fminf(c.v1.w, fmaf(c.v2.y, inv_d1, nXd1));
-                    const float gnew = fminf(fminf(c.v2.x, fmaf(c.v2.z, inv_d2, U)), ca);
-                    d[0][s] = kvm - a;
-                    d[1][s] = tt - a;
-                    d[2][s] = gon - a;
-                    d[3][s] = gnew - a;
+                    const SlotS<PEND>& t = ss[s];
+                    d[0][s] = fminf(t.kvB1 - a, fmaf(r, t.np1n, t.kvE - a));
+                    const float tt = fmaf(Zc, t.inv_s, t.nZO - a);
+                    d[2][s] = fminf(t.pmA - a, fmaf(t.Gt, id1, nX));
+                    const float ca = fmaf(t.b0n, ir, fmaf(t.nh, r, Ua - t.b1));
+                    if (PEND) {
+                        d[1][s] = fminf(tt, t.ZW - a);
+                        d[3][s] = fminf(fminf(t.pmAp - a, fmaf(t.Gpt, id2, Ua)), ca);
+                    } else {
+                        d[1][s] = tt;
+                        d[3][s] = ca;
+                    }
                     m[s] = fminf(fminf(d[0][s], d[1][s]), fminf(d[2][s], d[3][s]));
                     if (ARG) kmin = min(kmin, (__float_as_uint(m[s]) & 0x80000000u) | rank[s]);
                 }
+#endif
                 if (live) {
                     if (SF) {
                         const unsigned f = pack_flags<SLOTS>(d);
                         if (SLOTS == 4) __stcs(reinterpret_cast<unsigned int*>(fbase + off), f);
-                        else if (SLOTS == 2) __stcs(reinterpret_cast<unsigned short*>(fbase + off), (unsigned short)f);
-                        else fbase[off] = (uint8_t)f;
+                        else __stcs(reinterpret_cast<unsigned short*>(fbase + off), (unsigned short)f);
                     }
                     if (SMG) {
                         if (SLOTS == 4)
                             __stcs(reinterpret_cast<float4*>(mbase + off),
-                                   make_float4(m[0], m[1 % SLOTS], m[2 % SLOTS], m[3 % SLOTS]));
-                        else if (SLOTS == 2)
-                            __stcs(reinterpret_cast<float2*>(mbase + off), make_float2(m[0], m[1 % SLOTS]));
-                        else __stcs(mbase + off, m[0]);
+                                   make_float4(m[0], m[1], m[2 % SLOTS], m[3 % SLOTS]));
+                        else
+                            __stcs(reinterpret_cast<float2*>(mbase + off), make_float2(m[0], m[1]));
                     }
                 }
                 if (ARG) *kslot = __reduce_min_sync(FULL, kmin);  // same value from every lane
             }
         } else if (ARG) {
-            for (int i = tid & 31; i < nc; i += 32) sm.kmin[warp][i] = 0xffffffffu;
+            for (int i = lane; i < nc; i += 32) sm.kmin[warp][i] = 0xffffffffu;
         }
         __syncthreads();
         if (ARG) {
             for (int i = tid; i < nc; i += SCORE_WARPS * 32) {
                 unsigned v = sm.kmin[0][i];
 #pragma unroll
-                for (int q = 1; q < SCORE_WARPS; ++q) v = min(v, sm.kmin[q][i]);
-                if (v < 0x80000000u) atomicMin(A.best + __float_as_int(cs[3 * i + 2].y), v);
+                for (int w = 1; w < SCORE_WARPS; ++w) v = min(v, sm.kmin[w][i]);
+                if (v < 0x80000000u) atomicMin(A.best + __float_as_int(cs[REC_F4 * i + 4].y), v);
             }
         }
         __syncthreads();  // buffer `buf` and kmin are reused two chunks later
@@ -410,7 +546,7 @@ __global__ void __launch_bounds__(SCORE_WARPS * 32, ALADDIN_SCORE_MINB) k_score(
 }
 
 // Fallback for W % 4 != 0 or unaligned outputs: one worker per lane, scalar
-// stores.
+// arithmetic and stores, candidate records read from global memory.
 template <bool SF, bool SMG, bool ARG>
 __global__ void __launch_bounds__(SCORE_WARPS * 32) k_score_scalar(ScoreArgs A)
 {
@@ -425,29 +561,30 @@ __global__ void __launch_bounds__(SCORE_WARPS * 32) k_score_scalar(ScoreArgs A)
     const int c0 = chunk * SCORE_CHUNK;
     const int c1 = min(c0 + SCORE_CHUNK, A.n_cand);
     const long long rb = (long long)wc * A.C.rows;
-    const int R = A.C.R[wc];
-    int p = find_row(A.C.tab, rb, R, __ldg(&A.cand[c0].ri));
+    const int last_row = A.C.rows - 1;
+    const float4* recs = reinterpret_cast<const float4*>(A.cand);
+    int p = find_row(A.C.tab, rb, A.C.R[wc], __float_as_int(__ldg(&recs[(size_t)c0 * REC_F4 + 4].x)));
     Row cur = load_row(A.C.tab, rb + p);
     const float4 wr = __ldg(&A.C.wrec[wc]);
     const unsigned rank = live ? (unsigned)__float_as_int(wr.w) : 0xffffffffu;
     for (int c = c0; c < c1; ++c) {
-        const float4* cp = reinterpret_cast<const float4*>(A.cand + c);
-        const float4 q0 = __ldg(cp), q1 = __ldg(cp + 1), q2 = __ldg(cp + 2);
+        const float4* cp = recs + (size_t)c * REC_F4;
+        const float4 q0 = __ldg(cp), q1 = __ldg(cp + 1), q2 = __ldg(cp + 2), q3 = __ldg(cp + 3),
+                     q4 = __ldg(cp + 4);
         CandRec cr;
-        cr.a = q0.x; cr.r = q0.y; cr.inv_r = q0.z; cr.U = q0.w;
-        cr.inv_d1 = q1.x; cr.nXd1 = q1.y; cr.inv_d2 = q1.z; cr.Zc = q1.w;
-        cr.ri = __float_as_int(q2.x);
-        cr.orig = __float_as_int(q2.y);
-        cr.valid = cr.ri != 0;
+        cr.a = q0.x; cr.r = q0.z; cr.inv_r = q1.x; cr.Ua = q1.z;
+        cr.inv_d1 = q2.x; cr.nXd1a = q2.z; cr.inv_d2 = q3.x; cr.Zc = q3.z;
+        cr.ri = __float_as_int(q4.x);
+        cr.orig = __float_as_int(q4.y);
         const size_t off = (size_t)cr.orig * (size_t)W + (size_t)w;
-        if (!cr.valid) {
+        if (cr.ri == 0) {
             if (live) {
                 if (SF) A.flags[off] = 0x80;
                 if (SMG) A.margin[off] = __int_as_float(0x7fc00000);
             }
             continue;
         }
-        while (cr.ri >= __float_as_int(cur.v0.x) && p < R) {
+        while (cr.ri >= __float_as_int(cur.v0.x) && p < last_row) {
             p += 1;
             cur = load_row(A.C.tab, rb + p);
         }
@@ -465,7 +602,7 @@ __global__ void __launch_bounds__(SCORE_WARPS * 32) k_score_scalar(ScoreArgs A)
     }
 }
 
-template <int SLOTS, bool SF, bool SMG, bool ARG>
+template <int SLOTS, bool SF, bool SMG, bool ARG, bool PEND>
 static cudaError_t launch_vec(const ScoreArgs& A0, cudaStream_t st)
 {
     VecArgs A;
@@ -476,18 +613,19 @@ static cudaError_t launch_vec(const ScoreArgs& A0, cudaStream_t st)
     A.margin = A0.margin;
     A.best = A0.best;
     A.tiles = (A.C.W + SCORE_WARPS * 32 * SLOTS - 1) / (SCORE_WARPS * 32 * SLOTS);
-    const size_t smem = sizeof(ScoreSmem<SLOTS>);
+    const size_t smem = sizeof(ScoreSmem);
     static int per_sm = 0, sms = 0;  // occupancy of this instantiation (per process)
     if (per_sm == 0) {
-        cudaError_t e = cudaFuncSetAttribute(k_score<SLOTS, SF, SMG, ARG>,
+        cudaError_t e = cudaFuncSetAttribute(k_score<SLOTS, SF, SMG, ARG, PEND>,
                                              cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
         if (e != cudaSuccess) return e;
         int dev = 0;
         cudaGetDevice(&dev);
         cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
-        e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, k_score<SLOTS, SF, SMG, ARG>,
+        int ps = 0;
+        e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&ps, k_score<SLOTS, SF, SMG, ARG, PEND>,
                                                           SCORE_WARPS * 32, smem);
-        if (e != cudaSuccess || per_sm < 1) per_sm = 1;
+        per_sm = (e != cudaSuccess || ps < 1) ? 1 : ps;
     }
     // one wave: per_tile CTAs share each worker tile's candidates equally
     const int wave = per_sm * sms;
@@ -496,8 +634,21 @@ static cudaError_t launch_vec(const ScoreArgs& A0, cudaStream_t st)
     const int max_parts = (A.n_cand + 63) / 64;  // at least 64 candidates per CTA
     if (per_tile > max_parts) per_tile = max_parts;
     A.per_tile = per_tile;
-    k_score<SLOTS, SF, SMG, ARG><<<A.tiles * per_tile, SCORE_WARPS * 32, smem, st>>>(A);
+    k_score<SLOTS, SF, SMG, ARG, PEND><<<A.tiles * per_tile, SCORE_WARPS * 32, smem, st>>>(A);
     return cudaGetLastError();
+}
+
+template <bool PEND>
+static cudaError_t dispatch_vec(bool sf, bool smg, bool arg, const ScoreArgs& A, cudaStream_t st)
+{
+    constexpr int S = ALADDIN_SCORE_SLOTS;
+    if (sf && smg && arg) return launch_vec<S, true, true, true, PEND>(A, st);
+    if (sf && smg) return launch_vec<S, true, true, false, PEND>(A, st);
+    if (sf && arg) return launch_vec<S, true, false, true, PEND>(A, st);
+    if (smg && arg) return launch_vec<S, false, true, true, PEND>(A, st);
+    if (sf) return launch_vec<S, true, false, false, PEND>(A, st);
+    if (smg) return launch_vec<S, false, true, false, PEND>(A, st);
+    return launch_vec<S, false, false, true, PEND>(A, st);
 }
 
 template <bool SF, bool SMG, bool ARG>
@@ -564,7 +715,7 @@ __global__ void k_detail(DevParams P, ClusterDev C, int n, const int32_t* __rest
 cudaError_t launch_score(const DevParams& P, const ClusterDev& C, int n, const int32_t* in,
                          const int32_t* pred, const float* wait, uint8_t* flags, float* margin,
                          int32_t* argbest, int64_t* kv_peak, float* t_cand, const ScoreBuffers& B,
-                         cudaStream_t st, cudaEvent_t ev0, cudaEvent_t ev1)
+                         bool pend, cudaStream_t st, cudaEvent_t ev0, cudaEvent_t ev1)
 {
     if (n <= 0) return cudaSuccess;
     cudaError_t e;
@@ -587,19 +738,13 @@ cudaError_t launch_score(const DevParams& P, const ClusterDev& C, int n, const i
         A.margin = margin;
         A.best = argbest ? B.best : nullptr;
         A.chunks = (n + SCORE_CHUNK - 1) / SCORE_CHUNK;
+        A.tiles = 0;
         if (ev0) cudaEventRecord(ev0, st);
         const bool vec = (C.W % 4 == 0) && (((uintptr_t)flags & 3) == 0) &&
                          (((uintptr_t)margin & 15) == 0);
-        constexpr int S = ALADDIN_SCORE_SLOTS;
         const bool sf = flags != nullptr, smg = margin != nullptr, arg = argbest != nullptr;
         if (vec) {
-            if (sf && smg && arg) e = launch_vec<S, true, true, true>(A, st);
-            else if (sf && smg) e = launch_vec<S, true, true, false>(A, st);
-            else if (sf && arg) e = launch_vec<S, true, false, true>(A, st);
-            else if (smg && arg) e = launch_vec<S, false, true, true>(A, st);
-            else if (sf) e = launch_vec<S, true, false, false>(A, st);
-            else if (smg) e = launch_vec<S, false, true, false>(A, st);
-            else e = launch_vec<S, false, false, true>(A, st);
+            e = pend ? dispatch_vec<true>(sf, smg, arg, A, st) : dispatch_vec<false>(sf, smg, arg, A, st);
             if (e != cudaSuccess) return e;
         } else {
             if (sf && smg && arg) launch_scalar<true, true, true>(A, st);
