@@ -46,7 +46,7 @@
 namespace aladdin {
 
 constexpr unsigned FULL = 0xffffffffu;
-constexpr int ROW_F4 = 3;               // float4 per table row
+constexpr int ROW_F4 = 2;               // float4 per table row
 constexpr long long LL_NONE = (-0x7fffffffffffffffLL - 1);
 
 struct DevParams {
@@ -86,6 +86,7 @@ struct ClusterDev {
     uint8_t* pend;             // [W*cap] 1: placed this round, prefill pending
     double* wait;              // [W*cap] pending: wait since arrival at placement
     float4* tab;               // [W*rows*ROW_F4] scoring rows
+    float2* tab2;              // [W*rows] bounds of requests placed in an open round
     AuxRow* aux;               // [W*rows]
     int32_t* R;                // [W] breakpoints
     float4* wrec;              // [W] {1/s, ZO, ZW, rank bits}
@@ -95,24 +96,24 @@ struct ClusterDev {
     unsigned int* err;         // sticky error bits (1: invalid request)
 };
 
-// Table row p of a worker (3 x float4):
-//  v0 = {rho_{p+1} (int bits; INT_MAX for the last row), kvB1, kvE, -(n_p + 1)}
-//  v1 = {beta0n, beta1s, nh, pmA}
-//  v2 = {pmAp, Gt, Gpt, rho_p (int bits)}
+// Table row p of a worker (2 x float4, 32 bytes) and its side entry:
+//  v0 = {rho_{p+1} (int bits; INT_MAX for the last row), kvB1, kvE, beta0n}
+//  v1 = {beta1s, nh, pmA, Gt}
+//  tab2 = {pmAp, Gpt}: only requests placed in an open round use these
 // kvB1 = floor((M - j - PM_p)/h) (+inf for p = 0, -inf if SM_p > M)
 // kvE  = floor((M - j (n_p + 1))/h) - A_p
 // beta0n = -(c2/k2 PR_p + PRA_p); beta1s = (c3 + c2 n_p)/k2 + A_p + n_p/2 - theta T_dec/(s k2)
-// nh = -n_p/2; pmA / pmAp prefix-minimum bounds of ongoing / new requests with
-// r_j <= rho_p; Gt / Gpt = suffix-minimum slack of ongoing / new requests with
-// r_j > rho_p, over s, ongoing ones less the stall's constant part.
+// nh = -n_p/2 (so -(n_p + 1) = 2 nh - 1); pmA / pmAp prefix-minimum bounds of
+// ongoing / new requests with r_j <= rho_p; Gt / Gpt = suffix-minimum slack of
+// ongoing / new requests with r_j > rho_p, over s, ongoing ones less the
+// stall's constant part.
 
 // Derived per-candidate values (3 x float4), identical for every worker.
-// Bounds are compared with the prompt length a by subtracting a first, so the
-// a-dependent constants of the candidate carry it: Ua = U - a with
-// U = -c2/k2 - (r + 1)/2, and nXd1a = -X(r)/(k2 r + k1) - a.
+// Bounds are compared with the prompt length a as headrooms bound - a; the
+// candidate's decode bound carries a in Ua = U - a with U = -c2/k2 - (r + 1)/2.
 struct __align__(16) CandRec {
     float a, r, inv_r, Ua;             // prompt, output, 1/r, U - a
-    float inv_d1, nXd1a, inv_d2, Zc;   // 1/(k2 r + k1), -X(r)/(k2 r + k1) - a, 1/(k2 r), (T_pre - w)/k1
+    float inv_d1, nXd1, inv_d2, Zc;    // 1/(k2 r + k1), -X(r)/(k2 r + k1), 1/(k2 r), (T_pre - w)/k1
     int32_t ri, orig, valid, pad;
 };
 
@@ -141,7 +142,7 @@ __device__ __forceinline__ CandRec make_cand(const DevParams& P, int32_t in, int
     const float d1 = P.k2 * rf + P.k1;
     c.inv_d1 = 1.0f / d1;
     const float X = P.c2 * rf + P.k2 * (0.5f * rf * (rf + 1.0f));
-    c.nXd1a = -X * c.inv_d1 - a;
+    c.nXd1 = -X * c.inv_d1;
     c.inv_d2 = 1.0f / (P.k2 * rf);
     c.Zc = (P.T_pre - (ok ? w : 0.0f)) * P.inv_k1;
     c.ri = ok ? r : 0;
@@ -154,22 +155,23 @@ __device__ __forceinline__ CandRec make_cand(const DevParams& P, int32_t in, int
 // Headroom of one pair per constraint group (bound - a): d[0] KV, d[1] TTFT,
 // d[2] ongoing ATGT, d[3] new ATGT. The flags are the groups with d >= 0 and
 // the margin is min(d).
-__device__ __forceinline__ void pair_headroom(const float4 v0, const float4 v1, const float4 v2,
+__device__ __forceinline__ void pair_headroom(const float4 v0, const float4 v1, const float2 ext,
                                               const float4 wr, const CandRec& c, float (&d)[4])
 {
-    d[0] = fminf(v0.y - c.a, fmaf(c.r, v0.w, v0.z - c.a));
-    d[1] = fminf(fmaf(c.Zc, wr.x, -wr.y - c.a), wr.z - c.a);
-    d[2] = fminf(v1.w - c.a, fmaf(v2.y, c.inv_d1, c.nXd1a));
-    d[3] = fminf(fminf(v2.x - c.a, fmaf(v2.z, c.inv_d2, c.Ua)),
-                 fmaf(v1.x, c.inv_r, fmaf(v1.z, c.r, c.Ua - v1.y)));
+    const float np1n = fmaf(2.0f, v1.y, -1.0f);
+    d[0] = fminf(v0.y, fmaf(c.r, np1n, v0.z)) - c.a;
+    d[1] = fminf(fmaf(c.Zc, wr.x, -wr.y), wr.z) - c.a;
+    d[2] = fminf(v1.z, fmaf(v1.w, c.inv_d1, c.nXd1)) - c.a;
+    d[3] = fminf(fminf(ext.x - c.a, fmaf(ext.y, c.inv_d2, c.Ua)),
+                 fmaf(v0.w, c.inv_r, fmaf(v1.y, c.r, c.Ua - v1.x)));
 }
 
 // Bounds of one pair; returns the four flag bits, writes the margin.
-__device__ __forceinline__ unsigned eval_pair(const float4 v0, const float4 v1, const float4 v2,
+__device__ __forceinline__ unsigned eval_pair(const float4 v0, const float4 v1, const float2 ext,
                                               const float4 wr, const CandRec& c, float& margin)
 {
     float d[4];
-    pair_headroom(v0, v1, v2, wr, c, d);
+    pair_headroom(v0, v1, ext, wr, c, d);
     margin = fminf(fminf(d[0], d[1]), fminf(d[2], d[3]));
     return (d[0] >= 0.0f ? 1u : 0u) | (d[1] >= 0.0f ? 2u : 0u) | (d[2] >= 0.0f ? 4u : 0u) |
            (d[3] >= 0.0f ? 8u : 0u);
@@ -282,23 +284,19 @@ __device__ __forceinline__ void write_row(const DevParams& P, const ClusterDev& 
     else kvB1 = (float)floor_div_ll((long long)M - P.j - PM, P.h);
     const float kvE = (float)(floor_div_ll((long long)M - (long long)P.j * (n_p + 1), P.h) - A);
     const float nf = (float)n_p;
-    float4 v0, v1, v2;
+    float4 v0, v1;
     v0.x = __int_as_float(rho_next);
     v0.y = kvB1;
     v0.z = kvE;
-    v0.w = -(nf + 1.0f);
-    v1.x = -(P.c2_over_k2 * (float)PR + (float)PRA);
-    v1.y = P.c3_over_k2 + P.c2_over_k2 * nf + (float)A + 0.5f * nf - P.thTdec_over_k2 * inv_s;
-    v1.z = -0.5f * nf;
-    v1.w = pmA;
-    v2.x = pmAp;
-    v2.y = smS * inv_s - (P.k1 * (float)P_pend + P.c1);
-    v2.z = smSp * inv_s;
-    v2.w = __int_as_float(rho);
+    v0.w = -(P.c2_over_k2 * (float)PR + (float)PRA);
+    v1.x = P.c3_over_k2 + P.c2_over_k2 * nf + (float)A + 0.5f * nf - P.thTdec_over_k2 * inv_s;
+    v1.y = -0.5f * nf;
+    v1.z = pmA;
+    v1.w = smS * inv_s - (P.k1 * (float)P_pend + P.c1);
     float4* t = C.tab + rowid * ROW_F4;
     t[0] = v0;
     t[1] = v1;
-    t[2] = v2;
+    C.tab2[rowid] = make_float2(pmAp, smSp * inv_s);
     AuxRow ar;
     ar.PM = PM;
     ar.SM = SM;

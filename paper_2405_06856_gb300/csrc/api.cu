@@ -219,6 +219,7 @@ int cluster_alloc(aladdin_cluster* cl, const aladdin_params& p, int W,
     AL(pend, uint8_t, slots);
     AL(wait, double, slots);
     AL(tab, float4, rows * ROW_F4);
+    AL(tab2, float2, rows);
     AL(aux, AuxRow, rows);
     AL(R, int32_t, W);
     AL(wrec, float4, W);

@@ -70,7 +70,7 @@ __global__ void __launch_bounds__(ROUND_THREADS) k_round(DevParams P, ClusterDev
                 const int p = find_row<false>(C.tab, rb, C.R[w], cr.ri);
                 const float4* t = C.tab + (rb + p) * ROW_F4;
                 float m;
-                const unsigned f = eval_pair(t[0], t[1], t[2], C.wrec[w], cr, m);
+                const unsigned f = eval_pair(t[0], t[1], C.tab2[rb + p], C.wrec[w], cr, m);
                 if (f == 15u) better(bk, bw, C.key[w], w);
             }
 #pragma unroll

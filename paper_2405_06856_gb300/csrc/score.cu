@@ -73,12 +73,10 @@ __global__ void __launch_bounds__(SCAN_THREADS) k_scan_hist(int32_t* hist, int l
     }
 }
 
-// Sorted record (5 x float4), the per-candidate constants stored twice so that
-// a 16-byte shared-memory load yields ready-made operand pairs for the packed
-// f32x2 arithmetic: {a, a, r, r}, {1/r, 1/r, Ua, Ua}, {inv_d1, inv_d1, nXd1a,
-// nXd1a}, {inv_d2, inv_d2, Zc, Zc}, {valid ? r : 0, original index, low and
-// high words of index * W (the start of the candidate's output row)}.
-constexpr int REC_F4 = 5;
+// Sorted record (3 x float4): {a, r, 1/r, Ua}, {inv_d1, nXd1, inv_d2, Zc},
+// {valid ? r : 0, original index, low and high words of index * W (the start
+// of the candidate's output row)}.
+constexpr int REC_F4 = 3;
 
 struct ScoreArgs {
     ClusterDev C;
@@ -100,17 +98,15 @@ __global__ void k_cand_scatter(DevParams P, int n, int W, const int32_t* __restr
     const int pos = atomicAdd(&cursor[rec.valid ? rec.ri : 0], 1);
     const unsigned long long rowoff = (unsigned long long)c * (unsigned long long)W;
     float4* o = sorted + (size_t)pos * REC_F4;
-    o[0] = make_float4(rec.a, rec.a, rec.r, rec.r);
-    o[1] = make_float4(rec.inv_r, rec.inv_r, rec.Ua, rec.Ua);
-    o[2] = make_float4(rec.inv_d1, rec.inv_d1, rec.nXd1a, rec.nXd1a);
-    o[3] = make_float4(rec.inv_d2, rec.inv_d2, rec.Zc, rec.Zc);
-    o[4] = make_float4(__int_as_float(rec.valid ? rec.ri : 0), __int_as_float(c),
+    o[0] = make_float4(rec.a, rec.r, rec.inv_r, rec.Ua);
+    o[1] = make_float4(rec.inv_d1, rec.nXd1, rec.inv_d2, rec.Zc);
+    o[2] = make_float4(__int_as_float(rec.valid ? rec.ri : 0), __int_as_float(c),
                        __uint_as_float((unsigned)(rowoff & 0xffffffffull)),
                        __uint_as_float((unsigned)(rowoff >> 32)));
 }
 
 struct Row {
-    float4 v0, v1, v2;
+    float4 v0, v1;
 };
 
 __device__ __forceinline__ Row load_row(const float4* __restrict__ tab, long long row)
@@ -119,16 +115,7 @@ __device__ __forceinline__ Row load_row(const float4* __restrict__ tab, long lon
     Row r;
     r.v0 = __ldg(t);
     r.v1 = __ldg(t + 1);
-    r.v2 = __ldg(t + 2);
     return r;
-}
-
-// Ask L1 to hold the row (48 bytes: up to two 128-byte lines).
-__device__ __forceinline__ void prefetch_row(const float4* tab, long long row)
-{
-    const char* b = reinterpret_cast<const char*>(tab + row * ROW_F4);
-    asm volatile("prefetch.global.L1 [%0];" ::"l"(b));
-    asm volatile("prefetch.global.L1 [%0];" ::"l"(b + 47));
 }
 
 __device__ __forceinline__ unsigned prmt(unsigned a, unsigned b, unsigned sel)
@@ -136,31 +123,6 @@ __device__ __forceinline__ unsigned prmt(unsigned a, unsigned b, unsigned sel)
     unsigned d;
     asm("prmt.b32 %0, %1, %2, %3;" : "=r"(d) : "r"(a), "r"(b), "r"(sel));
     return d;
-}
-
-// Packed pairs of fp32 held in one 64-bit register (Blackwell f32x2
-// arithmetic: two independent round-to-nearest operations, bit-identical to
-// the scalar ones). Low word = slot 2j, high word = slot 2j + 1.
-typedef unsigned long long f2x;
-
-__device__ __forceinline__ f2x fma2(f2x a, f2x b, f2x c)
-{
-    f2x d;
-    asm("fma.rn.f32x2 %0, %1, %2, %3;" : "=l"(d) : "l"(a), "l"(b), "l"(c));
-    return d;
-}
-__device__ __forceinline__ f2x sub2(f2x a, f2x b)
-{
-    f2x d;
-    asm("sub.rn.f32x2 %0, %1, %2;" : "=l"(d) : "l"(a), "l"(b));
-    return d;
-}
-__device__ __forceinline__ float lo(f2x v) { return __uint_as_float((unsigned)v); }
-__device__ __forceinline__ float hi(f2x v) { return __uint_as_float((unsigned)(v >> 32)); }
-__device__ __forceinline__ f2x set_half(f2x v, int h, float x)
-{
-    const f2x b = (f2x)__float_as_uint(x);
-    return h ? ((v & 0xffffffffull) | (b << 32)) : ((v & 0xffffffff00000000ull) | b);
 }
 
 // Flag bytes of SLOTS pairs from the sign bits of their group headrooms
@@ -191,7 +153,7 @@ __device__ __forceinline__ unsigned pack_flags(const float (&d)[4][SLOTS])
 #define ALADDIN_SCORE_SLOTS 4
 #endif
 #ifndef ALADDIN_SCORE_MINB
-#define ALADDIN_SCORE_MINB 4
+#define ALADDIN_SCORE_MINB 5
 #endif
 constexpr int CHUNK = 256;                   // candidates per staged chunk
 constexpr long long WAIT_LIMIT = 1ll << 26;  // mbarrier polls before giving up
@@ -256,68 +218,67 @@ struct __align__(16) ScoreSmem {
     int stop;
 };
 
-// Worker state of one lane for a pair of slots (low word: slot 2j, high
-// word: slot 2j + 1).
-template <bool PEND>
-struct SlotPair {
-    f2x kvB1, kvE, np1n, b0n, b1, nh, pmA, Gt, inv_s, nZO;
-    f2x pmAp, Gpt, ZW;  // used only with requests of an open round (PEND)
-};
+// Worker state of one lane slot: the fields of the current table row that a
+// pair reads, the next row (raw), and the worker's record.
+#ifndef ALADDIN_SCORE_PF
+#define ALADDIN_SCORE_PF 1
+#endif
 
-template <bool PEND>
-__device__ __forceinline__ void set_row_slot(SlotPair<PEND>& q, int h, const Row& r)
+// Ask L1 to hold a row (32 bytes).
+__device__ __forceinline__ void prefetch_row(const float4* tab, long long row)
 {
-    q.kvB1 = set_half(q.kvB1, h, r.v0.y);
-    q.kvE = set_half(q.kvE, h, r.v0.z);
-    q.np1n = set_half(q.np1n, h, r.v0.w);
-    q.b0n = set_half(q.b0n, h, r.v1.x);
-    q.b1 = set_half(q.b1, h, r.v1.y);
-    q.nh = set_half(q.nh, h, r.v1.z);
-    q.pmA = set_half(q.pmA, h, r.v1.w);
-    q.Gt = set_half(q.Gt, h, r.v2.y);
-    if (PEND) {
-        q.pmAp = set_half(q.pmAp, h, r.v2.x);
-        q.Gpt = set_half(q.Gpt, h, r.v2.z);
-    }
+    asm volatile("prefetch.global.L1 [%0];" ::"l"(tab + row * ROW_F4));
 }
 
-// Scalar worker state of one lane slot.
 template <bool PEND>
-struct SlotS {
-    float kvB1, kvE, np1n, b0n, b1, nh, pmA, Gt, inv_s, nZO;
-    float pmAp, Gpt, ZW;  // used only with requests of an open round (PEND)
+struct Slot {
+    float kvB1, kvE, np1n, b0n, b1, nh, pmA, Gt;
+    float pmAp, Gpt;           // PEND only
+    int rnext;                 // rho_{p+1} of the current row
+#if !ALADDIN_SCORE_PF
+    Row nxt;                   // row p + 1
+    float2 nxt2;               // its side entry (PEND only)
+#endif
 };
 
 template <bool PEND>
-__device__ __forceinline__ void set_row_s(SlotS<PEND>& q, const Row& r)
+__device__ __forceinline__ void take_row(Slot<PEND>& q, const Row& r, const float2 e)
 {
+    q.rnext = __float_as_int(r.v0.x);
     q.kvB1 = r.v0.y;
     q.kvE = r.v0.z;
-    q.np1n = r.v0.w;
-    q.b0n = r.v1.x;
-    q.b1 = r.v1.y;
-    q.nh = r.v1.z;
-    q.pmA = r.v1.w;
-    q.Gt = r.v2.y;
+    q.b0n = r.v0.w;
+    q.b1 = r.v1.x;
+    q.nh = r.v1.y;
+    q.np1n = fmaf(2.0f, r.v1.y, -1.0f);
+    q.pmA = r.v1.z;
+    q.Gt = r.v1.w;
     if (PEND) {
-        q.pmAp = r.v2.x;
-        q.Gpt = r.v2.z;
+        q.pmAp = e.x;
+        q.Gpt = e.y;
     }
 }
-
-#ifndef ALADDIN_SCORE_F32X2
-#define ALADDIN_SCORE_F32X2 0
-#endif
 
 // One CTA = SCORE_WARPS warps x 32 lanes x SLOTS consecutive workers and one
 // contiguous range of sorted candidates (one wave of CTAs, equal shares).
 // Requires W % 4 == 0 and 16-byte aligned outputs. PEND: some worker holds
 // requests placed in an open round (pending prefill and its TTFT/ATGT bounds).
-template <int SLOTS, bool SF, bool SMG, bool ARG, bool PEND>
-__global__ void __launch_bounds__(SCORE_WARPS * 32, ALADDIN_SCORE_MINB) k_score(VecArgs A)
+#ifndef ALADDIN_STORE_HINT
+#define ALADDIN_STORE_HINT 1
+#endif
+template <typename T>
+__device__ __forceinline__ void st_out(T* p, T v)
 {
-    static_assert(SLOTS == 2 || SLOTS == 4, "slots come in pairs");
-    constexpr int NP = SLOTS / 2;
+#if ALADDIN_STORE_HINT
+    __stcs(p, v);
+#else
+    *p = v;
+#endif
+}
+
+template <int SLOTS, bool SF, bool SMG, bool ARG, bool PEND, bool FULLT>
+__global__ void __launch_bounds__(SCORE_WARPS * 32, PEND ? 3 : ALADDIN_SCORE_MINB) k_score(VecArgs A)
+{
     extern __shared__ __align__(16) unsigned char smraw[];
     ScoreSmem& sm = *reinterpret_cast<ScoreSmem*>(smraw);
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
@@ -343,18 +304,15 @@ __global__ void __launch_bounds__(SCORE_WARPS * 32, ALADDIN_SCORE_MINB) k_score(
 
     const int wbase = (tile * SCORE_WARPS + warp) * 32 * SLOTS;
     const int w0 = wbase + lane * SLOTS;
-    const bool live = w0 < W;
-    const bool warp_live = wbase < W;
+    const bool live = FULLT || w0 < W;
+    const bool warp_live = FULLT || wbase < W;
     uint8_t* const fbase = SF ? A.flags + (live ? w0 : 0) : nullptr;
     float* const mbase = SMG ? A.margin + (live ? w0 : 0) : nullptr;
     const int last_row = A.C.rows - 1;
 
-#if ALADDIN_SCORE_F32X2
-    SlotPair<PEND> st[NP];
-#else
-    SlotS<PEND> ss[SLOTS];
-#endif
-    int rnext[SLOTS], p[SLOTS], wk[SLOTS];
+    Slot<PEND> ss[SLOTS];
+    int p[SLOTS], wk[SLOTS];
+    float inv_s[SLOTS], nZO[SLOTS], ZW[SLOTS];
     unsigned rank[SLOTS];
     int nb = 0;  // smallest next breakpoint over this lane's workers
     bool have_rows = false;
@@ -381,38 +339,36 @@ __global__ void __launch_bounds__(SCORE_WARPS * 32, ALADDIN_SCORE_MINB) k_score(
         const float4* cs = sm.cs[buf];
         if (warp_live) {
             if (!have_rows) {
-                const int r_first = __float_as_int(cs[4].x);
+                const int r_first = __float_as_int(cs[2].x);
 #pragma unroll
                 for (int s = 0; s < SLOTS; ++s) {
                     wk[s] = live ? w0 + s : W - 1;
                     const long long rb = (long long)wk[s] * A.C.rows;
                     p[s] = find_row(A.C.tab, rb, __ldg(&A.C.R[wk[s]]), r_first);
-                    const Row r = load_row(A.C.tab, rb + p[s]);
-                    prefetch_row(A.C.tab, rb + min(p[s] + 1, last_row));
-                    rnext[s] = __float_as_int(r.v0.x);
-                    const float4 wr = __ldg(&A.C.wrec[wk[s]]);
-#if ALADDIN_SCORE_F32X2
-                    set_row_slot<PEND>(st[s >> 1], s & 1, r);
-                    st[s >> 1].inv_s = set_half(st[s >> 1].inv_s, s & 1, wr.x);
-                    st[s >> 1].nZO = set_half(st[s >> 1].nZO, s & 1, -wr.y);
-                    st[s >> 1].ZW = set_half(st[s >> 1].ZW, s & 1, wr.z);
+                    const long long pn = rb + min(p[s] + 1, last_row);
+                    take_row<PEND>(ss[s], load_row(A.C.tab, rb + p[s]),
+                                   PEND ? __ldg(&A.C.tab2[rb + p[s]]) : make_float2(0.f, 0.f));
+#if ALADDIN_SCORE_PF
+                    prefetch_row(A.C.tab, pn);
 #else
-                    set_row_s<PEND>(ss[s], r);
-                    ss[s].inv_s = wr.x;
-                    ss[s].nZO = -wr.y;
-                    ss[s].ZW = wr.z;
+                    ss[s].nxt = load_row(A.C.tab, pn);
+                    if (PEND) ss[s].nxt2 = __ldg(&A.C.tab2[pn]);
 #endif
+                    const float4 wr = __ldg(&A.C.wrec[wk[s]]);
+                    inv_s[s] = wr.x;
+                    nZO[s] = -wr.y;
+                    ZW[s] = wr.z;
                     rank[s] = live ? (unsigned)__float_as_int(wr.w) : 0xffffffffu;
                 }
-                nb = rnext[0];
+                nb = ss[0].rnext;
 #pragma unroll
-                for (int s = 1; s < SLOTS; ++s) nb = min(nb, rnext[s]);
+                for (int s = 1; s < SLOTS; ++s) nb = min(nb, ss[s].rnext);
                 have_rows = true;
             }
             const float4* q = cs;
             unsigned* kslot = &sm.kmin[warp][0];
             for (int i = 0; i < nc; ++i, q += REC_F4, ++kslot) {
-                const float4 q4 = q[4];
+                const float4 q4 = q[2];
                 const int ri = __float_as_int(q4.x);
                 const unsigned long long off =
                     ((unsigned long long)__float_as_uint(q4.w) << 32) | __float_as_uint(q4.z);
@@ -430,101 +386,62 @@ __global__ void __launch_bounds__(SCORE_WARPS * 32, ALADDIN_SCORE_MINB) k_score(
                 if (__any_sync(FULL, ri >= nb)) {
 #pragma unroll
                     for (int s = 0; s < SLOTS; ++s) {
-                        while (ri >= rnext[s] && p[s] < last_row) {
+                        // step to the row whose segment holds ri; the next row
+                        // is already in registers, the one after is fetched
+                        // now and needed only at the next crossing
+                        while (ri >= ss[s].rnext && p[s] < last_row) {
                             p[s] += 1;
                             const long long rb = (long long)wk[s] * A.C.rows;
-                            const Row r = load_row(A.C.tab, rb + p[s]);
-                            prefetch_row(A.C.tab, rb + min(p[s] + 1, last_row));
-                            rnext[s] = __float_as_int(r.v0.x);
-#if ALADDIN_SCORE_F32X2
-                            set_row_slot<PEND>(st[s >> 1], s & 1, r);
+                            const long long pn = rb + min(p[s] + 1, last_row);
+#if ALADDIN_SCORE_PF
+                            take_row<PEND>(ss[s], load_row(A.C.tab, rb + p[s]),
+                                           PEND ? __ldg(&A.C.tab2[rb + p[s]]) : make_float2(0.f, 0.f));
+                            prefetch_row(A.C.tab, pn);
 #else
-                            set_row_s<PEND>(ss[s], r);
+                            take_row<PEND>(ss[s], ss[s].nxt, ss[s].nxt2);
+                            ss[s].nxt = load_row(A.C.tab, pn);
+                            if (PEND) ss[s].nxt2 = __ldg(&A.C.tab2[pn]);
 #endif
                         }
                     }
-                    nb = rnext[0];
+                    nb = ss[0].rnext;
 #pragma unroll
-                    for (int s = 1; s < SLOTS; ++s) nb = min(nb, rnext[s]);
+                    for (int s = 1; s < SLOTS; ++s) nb = min(nb, ss[s].rnext);
                 }
-#if ALADDIN_SCORE_F32X2
-                const ulonglong2* qq = reinterpret_cast<const ulonglong2*>(q);
-                const ulonglong2 q0 = qq[0], q1 = qq[1], q2 = qq[2], q3 = qq[3];
-                const f2x a2 = q0.x, r2 = q0.y, ir2 = q1.x, Ua2 = q1.y;
-                const f2x id1 = q2.x, nX2 = q2.y, id2 = q3.x, Zc2 = q3.y;
-                float d[4][SLOTS], m[SLOTS];
-                unsigned kmin = 0xffffffffu;
-#pragma unroll
-                for (int j = 0; j < NP; ++j) {
-                    const SlotPair<PEND>& t = st[j];
-                    const f2x kv1 = sub2(t.kvB1, a2);
-                    const f2x kv2 = fma2(r2, t.np1n, sub2(t.kvE, a2));
-                    const f2x tt = fma2(Zc2, t.inv_s, sub2(t.nZO, a2));
-                    const f2x on1 = sub2(t.pmA, a2);
-                    const f2x on2 = fma2(t.Gt, id1, nX2);
-                    const f2x ca = fma2(t.b0n, ir2, fma2(t.nh, r2, sub2(Ua2, t.b1)));
-                    f2x ttw = 0, nw1 = 0, nw2 = 0;
-                    if (PEND) {
-                        ttw = sub2(t.ZW, a2);
-                        nw1 = sub2(t.pmAp, a2);
-                        nw2 = fma2(t.Gpt, id2, Ua2);
-                    }
-#pragma unroll
-                    for (int h = 0; h < 2; ++h) {
-                        const int s = 2 * j + h;
-                        const float e_kv1 = h ? hi(kv1) : lo(kv1), e_kv2 = h ? hi(kv2) : lo(kv2);
-                        const float e_tt = h ? hi(tt) : lo(tt);
-                        const float e_on1 = h ? hi(on1) : lo(on1), e_on2 = h ? hi(on2) : lo(on2);
-                        const float e_ca = h ? hi(ca) : lo(ca);
-                        d[0][s] = fminf(e_kv1, e_kv2);
-                        d[2][s] = fminf(e_on1, e_on2);
-                        if (PEND) {
-                            d[1][s] = fminf(e_tt, h ? hi(ttw) : lo(ttw));
-                            d[3][s] = fminf(fminf(h ? hi(nw1) : lo(nw1), h ? hi(nw2) : lo(nw2)), e_ca);
-                        } else {
-                            d[1][s] = e_tt;
-                            d[3][s] = e_ca;
-                        }
-                        m[s] = fminf(fminf(d[0][s], d[1][s]), fminf(d[2][s], d[3][s]));
-                        if (ARG) kmin = min(kmin, (__float_as_uint(m[s]) & 0x80000000u) | rank[s]);
-                    }
-                }
-#else
-                const float4 q0 = q[0], q1 = q[1], q2 = q[2], q3 = q[3];
-                const float a = q0.x, r = q0.z, ir = q1.x, Ua = q1.z;
-                const float id1 = q2.x, nX = q2.z, id2 = q3.x, Zc = q3.z;
+                const float4 q0 = q[0], q1 = q[1];
+                const float a = q0.x, r = q0.y, ir = q0.z, Ua = q0.w;
+                const float id1 = q1.x, nX = q1.y, id2 = q1.z, Zc = q1.w;
                 float d[4][SLOTS], m[SLOTS];
                 unsigned kmin = 0xffffffffu;
 #pragma unroll
                 for (int s = 0; s < SLOTS; ++s) {
-                    const SlotS<PEND>& t = ss[s];
-                    d[0][s] = fminf(t.kvB1 - a, fmaf(r, t.np1n, t.kvE - a));
-                    const float tt = fmaf(Zc, t.inv_s, t.nZO - a);
-                    d[2][s] = fminf(t.pmA - a, fmaf(t.Gt, id1, nX));
+                    const Slot<PEND>& t = ss[s];
+                    d[0][s] = fminf(t.kvB1, fmaf(r, t.np1n, t.kvE)) - a;
+                    const float tt = fmaf(Zc, inv_s[s], nZO[s]);
+                    d[2][s] = fminf(t.pmA, fmaf(t.Gt, id1, nX)) - a;
                     const float ca = fmaf(t.b0n, ir, fmaf(t.nh, r, Ua - t.b1));
                     if (PEND) {
-                        d[1][s] = fminf(tt, t.ZW - a);
+                        d[1][s] = fminf(tt, ZW[s]) - a;
                         d[3][s] = fminf(fminf(t.pmAp - a, fmaf(t.Gpt, id2, Ua)), ca);
                     } else {
-                        d[1][s] = tt;
+                        d[1][s] = tt - a;
                         d[3][s] = ca;
                     }
                     m[s] = fminf(fminf(d[0][s], d[1][s]), fminf(d[2][s], d[3][s]));
                     if (ARG) kmin = min(kmin, (__float_as_uint(m[s]) & 0x80000000u) | rank[s]);
                 }
-#endif
                 if (live) {
                     if (SF) {
                         const unsigned f = pack_flags<SLOTS>(d);
-                        if (SLOTS == 4) __stcs(reinterpret_cast<unsigned int*>(fbase + off), f);
-                        else __stcs(reinterpret_cast<unsigned short*>(fbase + off), (unsigned short)f);
+                        if (SLOTS == 4) st_out(reinterpret_cast<unsigned int*>(fbase + off), f);
+                        else st_out(reinterpret_cast<unsigned short*>(fbase + off), (unsigned short)f);
                     }
                     if (SMG) {
                         if (SLOTS == 4)
-                            __stcs(reinterpret_cast<float4*>(mbase + off),
+                            st_out(reinterpret_cast<float4*>(mbase + off),
                                    make_float4(m[0], m[1], m[2 % SLOTS], m[3 % SLOTS]));
                         else
-                            __stcs(reinterpret_cast<float2*>(mbase + off), make_float2(m[0], m[1]));
+                            st_out(reinterpret_cast<float2*>(mbase + off), make_float2(m[0], m[1]));
                     }
                 }
                 if (ARG) *kslot = __reduce_min_sync(FULL, kmin);  // same value from every lane
@@ -538,7 +455,7 @@ __global__ void __launch_bounds__(SCORE_WARPS * 32, ALADDIN_SCORE_MINB) k_score(
                 unsigned v = sm.kmin[0][i];
 #pragma unroll
                 for (int w = 1; w < SCORE_WARPS; ++w) v = min(v, sm.kmin[w][i]);
-                if (v < 0x80000000u) atomicMin(A.best + __float_as_int(cs[REC_F4 * i + 4].y), v);
+                if (v < 0x80000000u) atomicMin(A.best + __float_as_int(cs[REC_F4 * i + 2].y), v);
             }
         }
         __syncthreads();  // buffer `buf` and kmin are reused two chunks later
@@ -546,7 +463,7 @@ __global__ void __launch_bounds__(SCORE_WARPS * 32, ALADDIN_SCORE_MINB) k_score(
 }
 
 // Fallback for W % 4 != 0 or unaligned outputs: one worker per lane, scalar
-// arithmetic and stores, candidate records read from global memory.
+// stores, candidate records read from global memory.
 template <bool SF, bool SMG, bool ARG>
 __global__ void __launch_bounds__(SCORE_WARPS * 32) k_score_scalar(ScoreArgs A)
 {
@@ -563,19 +480,19 @@ __global__ void __launch_bounds__(SCORE_WARPS * 32) k_score_scalar(ScoreArgs A)
     const long long rb = (long long)wc * A.C.rows;
     const int last_row = A.C.rows - 1;
     const float4* recs = reinterpret_cast<const float4*>(A.cand);
-    int p = find_row(A.C.tab, rb, A.C.R[wc], __float_as_int(__ldg(&recs[(size_t)c0 * REC_F4 + 4].x)));
+    int p = find_row(A.C.tab, rb, A.C.R[wc], __float_as_int(__ldg(&recs[(size_t)c0 * REC_F4 + 2].x)));
     Row cur = load_row(A.C.tab, rb + p);
+    float2 ext = __ldg(&A.C.tab2[rb + p]);
     const float4 wr = __ldg(&A.C.wrec[wc]);
     const unsigned rank = live ? (unsigned)__float_as_int(wr.w) : 0xffffffffu;
     for (int c = c0; c < c1; ++c) {
         const float4* cp = recs + (size_t)c * REC_F4;
-        const float4 q0 = __ldg(cp), q1 = __ldg(cp + 1), q2 = __ldg(cp + 2), q3 = __ldg(cp + 3),
-                     q4 = __ldg(cp + 4);
+        const float4 q0 = __ldg(cp), q1 = __ldg(cp + 1), q2 = __ldg(cp + 2);
         CandRec cr;
-        cr.a = q0.x; cr.r = q0.z; cr.inv_r = q1.x; cr.Ua = q1.z;
-        cr.inv_d1 = q2.x; cr.nXd1a = q2.z; cr.inv_d2 = q3.x; cr.Zc = q3.z;
-        cr.ri = __float_as_int(q4.x);
-        cr.orig = __float_as_int(q4.y);
+        cr.a = q0.x; cr.r = q0.y; cr.inv_r = q0.z; cr.Ua = q0.w;
+        cr.inv_d1 = q1.x; cr.nXd1 = q1.y; cr.inv_d2 = q1.z; cr.Zc = q1.w;
+        cr.ri = __float_as_int(q2.x);
+        cr.orig = __float_as_int(q2.y);
         const size_t off = (size_t)cr.orig * (size_t)W + (size_t)w;
         if (cr.ri == 0) {
             if (live) {
@@ -587,9 +504,10 @@ __global__ void __launch_bounds__(SCORE_WARPS * 32) k_score_scalar(ScoreArgs A)
         while (cr.ri >= __float_as_int(cur.v0.x) && p < last_row) {
             p += 1;
             cur = load_row(A.C.tab, rb + p);
+            ext = __ldg(&A.C.tab2[rb + p]);
         }
         float m;
-        const unsigned f = eval_pair(cur.v0, cur.v1, cur.v2, wr, cr, m);
+        const unsigned f = eval_pair(cur.v0, cur.v1, ext, wr, cr, m);
         if (live) {
             if (SF) A.flags[off] = (uint8_t)f;
             if (SMG) __stcs(A.margin + off, m);
@@ -602,7 +520,7 @@ __global__ void __launch_bounds__(SCORE_WARPS * 32) k_score_scalar(ScoreArgs A)
     }
 }
 
-template <int SLOTS, bool SF, bool SMG, bool ARG, bool PEND>
+template <int SLOTS, bool SF, bool SMG, bool ARG, bool PEND, bool FULLT>
 static cudaError_t launch_vec(const ScoreArgs& A0, cudaStream_t st)
 {
     VecArgs A;
@@ -616,14 +534,14 @@ static cudaError_t launch_vec(const ScoreArgs& A0, cudaStream_t st)
     const size_t smem = sizeof(ScoreSmem);
     static int per_sm = 0, sms = 0;  // occupancy of this instantiation (per process)
     if (per_sm == 0) {
-        cudaError_t e = cudaFuncSetAttribute(k_score<SLOTS, SF, SMG, ARG, PEND>,
+        cudaError_t e = cudaFuncSetAttribute(k_score<SLOTS, SF, SMG, ARG, PEND, FULLT>,
                                              cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
         if (e != cudaSuccess) return e;
         int dev = 0;
         cudaGetDevice(&dev);
         cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
         int ps = 0;
-        e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&ps, k_score<SLOTS, SF, SMG, ARG, PEND>,
+        e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&ps, k_score<SLOTS, SF, SMG, ARG, PEND, FULLT>,
                                                           SCORE_WARPS * 32, smem);
         per_sm = (e != cudaSuccess || ps < 1) ? 1 : ps;
     }
@@ -634,21 +552,30 @@ static cudaError_t launch_vec(const ScoreArgs& A0, cudaStream_t st)
     const int max_parts = (A.n_cand + 63) / 64;  // at least 64 candidates per CTA
     if (per_tile > max_parts) per_tile = max_parts;
     A.per_tile = per_tile;
-    k_score<SLOTS, SF, SMG, ARG, PEND><<<A.tiles * per_tile, SCORE_WARPS * 32, smem, st>>>(A);
+    k_score<SLOTS, SF, SMG, ARG, PEND, FULLT><<<A.tiles * per_tile, SCORE_WARPS * 32, smem, st>>>(A);
     return cudaGetLastError();
+}
+
+template <bool PEND, bool FULLT>
+static cudaError_t dispatch_vec2(bool sf, bool smg, bool arg, const ScoreArgs& A, cudaStream_t st)
+{
+    constexpr int S = ALADDIN_SCORE_SLOTS;
+    if (sf && smg && arg) return launch_vec<S, true, true, true, PEND, FULLT>(A, st);
+    if (sf && smg) return launch_vec<S, true, true, false, PEND, FULLT>(A, st);
+    if (sf && arg) return launch_vec<S, true, false, true, PEND, FULLT>(A, st);
+    if (smg && arg) return launch_vec<S, false, true, true, PEND, FULLT>(A, st);
+    if (sf) return launch_vec<S, true, false, false, PEND, FULLT>(A, st);
+    if (smg) return launch_vec<S, false, true, false, PEND, FULLT>(A, st);
+    return launch_vec<S, false, false, true, PEND, FULLT>(A, st);
 }
 
 template <bool PEND>
 static cudaError_t dispatch_vec(bool sf, bool smg, bool arg, const ScoreArgs& A, cudaStream_t st)
 {
-    constexpr int S = ALADDIN_SCORE_SLOTS;
-    if (sf && smg && arg) return launch_vec<S, true, true, true, PEND>(A, st);
-    if (sf && smg) return launch_vec<S, true, true, false, PEND>(A, st);
-    if (sf && arg) return launch_vec<S, true, false, true, PEND>(A, st);
-    if (smg && arg) return launch_vec<S, false, true, true, PEND>(A, st);
-    if (sf) return launch_vec<S, true, false, false, PEND>(A, st);
-    if (smg) return launch_vec<S, false, true, false, PEND>(A, st);
-    return launch_vec<S, false, false, true, PEND>(A, st);
+    // every lane of every CTA tile holds a worker: no per-lane predicate
+    const bool full = A.C.W % (SCORE_WARPS * 32 * ALADDIN_SCORE_SLOTS) == 0;
+    return full ? dispatch_vec2<PEND, true>(sf, smg, arg, A, st)
+                : dispatch_vec2<PEND, false>(sf, smg, arg, A, st);
 }
 
 template <bool SF, bool SMG, bool ARG>
