@@ -40,6 +40,8 @@ extern "C" {
 #define ALADDIN_ERR_NOMEM (-5)    /* device or host allocation failed */
 #define ALADDIN_ERR_STATE (-6)    /* the cluster holds an invalid request (see
                                      aladdin_cluster_load) */
+#define ALADDIN_ERR_SCRATCH (-7)  /* more candidates than aladdin_score_noalloc's
+                                     fixed scratch holds */
 
 /* Pair flags (one byte per (candidate, worker)). */
 #define ALADDIN_FLAG_KV 1u        /* (e): KV usage stays within capacity every iteration */
@@ -134,6 +136,28 @@ int aladdin_score(aladdin_cluster* cl, int32_t n_cand, const int32_t* in, const 
 int aladdin_score_detail(aladdin_cluster* cl, int32_t n_cand, const int32_t* in,
                          const int32_t* pred, const float* wait_ms, uint8_t* flags,
                          float* margin, int32_t* argbest, int64_t* kv_peak, float* t_cand_ms);
+
+/* Maximum candidates per call of aladdin_score_noalloc. */
+#define ALADDIN_NOALLOC_MAX_CAND 32768
+
+/* aladdin_score for callers that cannot allocate device memory during the
+ * call: code recording a CUDA stream capture, processes whose device memory
+ * is reserved up front by another allocator (a serving engine owning the
+ * KV-cache pool), real-time scheduling loops. The paper has no counterpart;
+ * this is a property of the library.
+ * Same inputs, outputs and results as aladdin_score, but every pointer must be
+ * device (or managed) memory of the cluster's GPU (ALADDIN_ERR_ARG otherwise),
+ * the call is asynchronous on the cluster's stream, and it calls no
+ * allocator: its scratch is a fixed device array (about 2 MB) built into the
+ * library, held by every GPU that loads it until the process exits.
+ * n_cand may be at most ALADDIN_NOALLOC_MAX_CAND (ALADDIN_ERR_SCRATCH
+ * otherwise). The first call on a device looks up the array's device address;
+ * make that first call before any stream capture. All calls share the array:
+ * calls that overlap on the GPU (several streams, or several clusters on one
+ * device) race on it, and the caller must serialize them. */
+int aladdin_score_noalloc(aladdin_cluster* cl, int32_t n_cand, const int32_t* in,
+                          const int32_t* pred, const float* wait_ms, uint8_t* flags,
+                          float* margin, int32_t* argbest);
 
 /* One greedy best-fit round (Algorithm 1): candidates in index order, each
  * placed on the feasible worker of largest capacity_norm in the state left by

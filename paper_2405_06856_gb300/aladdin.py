@@ -18,12 +18,15 @@ LIB_PATH = os.path.join(_HERE, "_build", "libaladdin.so")
 
 OK = 0
 ERR_ARG, ERR_CAPACITY, ERR_CUDA, ERR_TIMEOUT, ERR_NOMEM, ERR_STATE = -1, -2, -3, -4, -5, -6
+ERR_SCRATCH = -7
+NOALLOC_MAX_CAND = 32768
 FLAG_KV, FLAG_TTFT, FLAG_ONGOING, FLAG_NEW, FEASIBLE, FLAG_INVALID = 1, 2, 4, 8, 15, 128
 NONE, INVALID = -1, -2
 
 _NAMES = {ERR_ARG: "ALADDIN_ERR_ARG", ERR_CAPACITY: "ALADDIN_ERR_CAPACITY",
           ERR_CUDA: "ALADDIN_ERR_CUDA", ERR_TIMEOUT: "ALADDIN_ERR_TIMEOUT",
-          ERR_NOMEM: "ALADDIN_ERR_NOMEM", ERR_STATE: "ALADDIN_ERR_STATE"}
+          ERR_NOMEM: "ALADDIN_ERR_NOMEM", ERR_STATE: "ALADDIN_ERR_STATE",
+          ERR_SCRATCH: "ALADDIN_ERR_SCRATCH"}
 
 
 class AladdinError(RuntimeError):
@@ -61,6 +64,7 @@ _sig = {
     "aladdin_cluster_load": [_P, _P, _P, _P, _P, _P],
     "aladdin_score": [_P, C.c_int32, _P, _P, _P, _P, _P, _P],
     "aladdin_score_detail": [_P, C.c_int32, _P, _P, _P, _P, _P, _P, _P, _P],
+    "aladdin_score_noalloc": [_P, C.c_int32, _P, _P, _P, _P, _P, _P],
     "aladdin_place_round": [_P, C.c_int32, _P, _P, _P, _P],
     "aladdin_cluster_advance": [_P, C.c_double, _P],
     "aladdin_cluster_state": [_P, _P, _P, _P, _P, _P],
@@ -161,6 +165,13 @@ def aladdin_cluster_load(cl, req_off, req_in, req_gen, req_pred, tdec_ms=None):
 def aladdin_score(cl, n_cand, cand_in, cand_pred, wait_ms, flags, margin, argbest):
     _check(_lib.aladdin_score(cl, int(n_cand), _ptr(cand_in), _ptr(cand_pred), _ptr(wait_ms),
                               _ptr(flags), _ptr(margin), _ptr(argbest)), "aladdin_score")
+
+
+def aladdin_score_noalloc(cl, n_cand, cand_in, cand_pred, wait_ms, flags, margin, argbest):
+    """aladdin_score without any allocation (device tensors only)."""
+    _check(_lib.aladdin_score_noalloc(cl, int(n_cand), _ptr(cand_in), _ptr(cand_pred),
+                                      _ptr(wait_ms), _ptr(flags), _ptr(margin), _ptr(argbest)),
+           "aladdin_score_noalloc")
 
 
 def aladdin_score_detail(cl, n_cand, cand_in, cand_pred, wait_ms, flags, margin, argbest,

@@ -62,4 +62,18 @@ cudaError_t launch_round(const DevParams& P, const ClusterDev& C, const RoundIO&
 cudaError_t launch_advance(const DevParams& P, const ClusterDev& C, double t_now, double dt,
                            unsigned long long* stats, const int* halt, cudaStream_t st);
 
+// What another translation unit may read of a cluster (see cluster_view).
+struct ClusterView {
+    int device;
+    cudaStream_t stream;
+    DevParams dp;
+    ClusterDev dev;
+    bool round_open;
+};
+
+}  // namespace aladdin
+
+struct aladdin_cluster;
+namespace aladdin {
+int cluster_view(aladdin_cluster* cl, ClusterView* v);
 }  // namespace aladdin

@@ -651,6 +651,22 @@ int aladdin_cluster_status(aladdin_cluster* cl)
 }  // extern "C"
 
 // ---------------------------------------------------------------------------
+// Read-only view of a cluster for other translation units of the library.
+
+namespace aladdin {
+int cluster_view(aladdin_cluster* cl, ClusterView* v)
+{
+    if (!cl || !v) return ALADDIN_ERR_ARG;
+    v->device = cl->device;
+    v->stream = cl->st;
+    v->dp = cl->dp;
+    v->dev = cl->dev;
+    v->round_open = cl->round_open;
+    return ALADDIN_OK;
+}
+}  // namespace aladdin
+
+// ---------------------------------------------------------------------------
 // Fleet simulation.
 
 namespace {
