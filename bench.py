@@ -308,15 +308,7 @@ def run_ours(args):
     kern_avg = kern_ms / max(kern_n, 1)
     abytes = algorithmic_bytes(W, Bq, C)
     achieved = abytes / (kern_avg / 1000.0) / 1e9
-    traffic = None
-    tp = os.path.join(ROOT, "profiles", "traffic_k_score_w4096.json")
-    if os.path.exists(tp):
-        try:
-            tj = json.load(open(tp))
-            if tj.get("source_hash") == kernel_source_hash():
-                traffic = tj["dram_bytes_per_launch"]
-        except Exception:
-            traffic = None
+    traffic = profiled_traffic()
 
     launches_per_step = 3 + 5  # load: pack, build, rank; score: count, scan, scatter, score, finalize
     line = {"metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
@@ -373,6 +365,22 @@ def run_kernel_only(args):
     assert cl.status() == A.OK
     cl.close()
     print("kernel mode ok: %d steps" % (args.warmup + args.steps))
+
+
+def profiled_traffic():
+    """DRAM bytes per launch of the scoring kernel from the committed ncu
+    summary, or None if the kernel source changed since it was taken."""
+    import re
+    path = os.path.join(ROOT, "profiles", "k_score_w4096.md")
+    try:
+        txt = open(path).read()
+        t = re.search(r"traffic_bytes_per_launch:\s*(\d+)", txt)
+        h = re.search(r"source_hash:\s*(\w+)", txt)
+        if t and h and h.group(1) == kernel_source_hash():
+            return int(t.group(1))
+    except OSError:
+        pass
+    return None
 
 
 def kernel_source_hash():
