@@ -94,6 +94,8 @@ struct ClusterDev {
     int32_t* rank;             // [W]
     int32_t* order;            // [W] worker at rank
     unsigned int* err;         // sticky error bits (1: invalid request)
+    int32_t* ovf;              // [W] workers left to the full-capacity table build
+    int* novf;                 // their count
 };
 
 // Table row p of a worker (2 x float4, 32 bytes) and its side entry:

@@ -227,6 +227,8 @@ int cluster_alloc(aladdin_cluster* cl, const aladdin_params& p, int W,
     AL(rank, int32_t, W);
     AL(order, int32_t, W);
     AL(err, unsigned int, 1);
+    AL(ovf, int32_t, W);
+    AL(novf, int, 1);
 #undef AL
     CK(cl->alloc(&p0, sizeof(unsigned long long) * 4)); cl->d_stats = (unsigned long long*)p0;
     CK(cl->alloc(&p0, sizeof(int) * 4)); cl->d_status = (int*)p0;

@@ -19,18 +19,69 @@ k_build(DevParams P, ClusterDev C, const int32_t* __restrict__ list, int count)
     build_table<E>(P, C, w, sm[warp]);
 }
 
+// Workers of a cluster with b_cap > 128 slots usually hold far fewer
+// requests than slots. The build runs as a cascade: a 128-element warp build
+// for every worker that fits (fewer registers, a quarter of the sorting work
+// of a 512-slot build), the full-capacity build only for the workers that do
+// not, listed on the device by the first pass.
+constexpr int E_LO = 4;
+
+template <int E>
+__global__ void __launch_bounds__(BUILD_WARPS * 32)
+k_build_lo(DevParams P, ClusterDev C, int count, int32_t* __restrict__ ovf, int* __restrict__ novf)
+{
+    extern __shared__ __align__(16) unsigned char smraw[];
+    BuildSmem<E>* sm = reinterpret_cast<BuildSmem<E>*>(smraw);
+    const int warp = threadIdx.x >> 5;
+    const int w = blockIdx.x * BUILD_WARPS + warp;
+    if (w >= count) return;
+    if (C.n[w] > 32 * E) {  // warp-uniform
+        if ((threadIdx.x & 31) == 0) ovf[atomicAdd(novf, 1)] = w;
+        return;
+    }
+    build_table<E>(P, C, w, sm[warp]);
+}
+
+template <int E>
+__global__ void __launch_bounds__(BUILD_WARPS * 32)
+k_build_ovf(DevParams P, ClusterDev C, const int32_t* __restrict__ ovf, const int* __restrict__ novf)
+{
+    extern __shared__ __align__(16) unsigned char smraw[];
+    BuildSmem<E>* sm = reinterpret_cast<BuildSmem<E>*>(smraw);
+    const int warp = threadIdx.x >> 5;
+    const int idx = blockIdx.x * BUILD_WARPS + warp;
+    if (idx >= *novf) return;
+    build_table<E>(P, C, ovf[idx], sm[warp]);
+}
+
+template <typename K>
+static cudaError_t allow_smem(K kern, size_t smem)
+{
+    if (smem > 48 * 1024)
+        return cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    return cudaSuccess;
+}
+
 template <int E>
 static cudaError_t build_e(const DevParams& P, const ClusterDev& C, const int32_t* list, int count,
                            cudaStream_t st)
 {
     if (count <= 0) return cudaSuccess;
-    const size_t smem = sizeof(BuildSmem<E>) * BUILD_WARPS;
-    if (smem > 48 * 1024) {
-        cudaError_t e = cudaFuncSetAttribute(k_build<E>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                             (int)smem);
-        if (e != cudaSuccess) return e;
-    }
     const int blocks = (count + BUILD_WARPS - 1) / BUILD_WARPS;
+    cudaError_t e;
+    if (E > E_LO && !list) {
+        constexpr int EL = E > E_LO ? E_LO : E;
+        const size_t slo = sizeof(BuildSmem<EL>) * BUILD_WARPS;
+        const size_t shi = sizeof(BuildSmem<E>) * BUILD_WARPS;
+        if ((e = allow_smem(k_build_lo<EL>, slo)) != cudaSuccess) return e;
+        if ((e = allow_smem(k_build_ovf<E>, shi)) != cudaSuccess) return e;
+        if ((e = cudaMemsetAsync(C.novf, 0, sizeof(int), st)) != cudaSuccess) return e;
+        k_build_lo<EL><<<blocks, BUILD_WARPS * 32, slo, st>>>(P, C, count, C.ovf, C.novf);
+        k_build_ovf<E><<<blocks, BUILD_WARPS * 32, shi, st>>>(P, C, C.ovf, C.novf);
+        return cudaGetLastError();
+    }
+    const size_t smem = sizeof(BuildSmem<E>) * BUILD_WARPS;
+    if ((e = allow_smem(k_build<E>, smem)) != cudaSuccess) return e;
     k_build<E><<<blocks, BUILD_WARPS * 32, smem, st>>>(P, C, list, count);
     return cudaGetLastError();
 }
@@ -50,11 +101,11 @@ cudaError_t launch_build(const DevParams& P, const ClusterDev& C, const int32_t*
 
 // rank[w] = number of workers ordered before w: larger key, or equal key and
 // smaller index (a stable descending sort by capacity_norm). A 2-D grid of
-// CTAs counts, for a tile of 256 workers, the workers of one 1024-key chunk
+// CTAs counts, for a tile of 256 workers, the workers of one 256-key chunk
 // that precede each of them (integer compares on keys staged in shared
 // memory) and adds the count to rank[w]; k_order then inverts the ranks.
 constexpr int RANK_TILE = 256;
-constexpr int RANK_CHUNK = 1024;
+constexpr int RANK_CHUNK = 256;
 
 __global__ void __launch_bounds__(RANK_TILE) k_rank_count(ClusterDev C)
 {
