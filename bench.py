@@ -369,6 +369,30 @@ def run_kernel_only(args):
     print("kernel mode ok: %d steps" % (args.warmup + args.steps))
 
 
+def run_round_only(args):
+    """Greedy rounds on the 256-worker workload only (warm-up + steps rounds,
+    each on a fresh cluster): the command profiled for the round kernel."""
+    import torch
+    from paper_2405_06856_gb300 import build as B
+    B.build()
+    from paper_2405_06856_gb300 import aladdin as A
+    from paper_2405_06856_gb300 import synth
+    torch.cuda.set_device(0)
+    dev = torch.device("cuda", 0)
+    w2 = synth.config("w256", b_cap=128)
+    d = lambda x: torch.from_numpy(np.ascontiguousarray(x)).to(dev)
+    t_in, t_pr, t_w = d(w2.cand_in), d(w2.cand_pred), d(w2.cand_wait)
+    times = []
+    for _ in range(args.warmup + args.steps):
+        with A.Cluster.from_workload(w2, stream=torch.cuda.current_stream().cuda_stream) as c2:
+            pl = torch.empty(w2.n_cand, dtype=torch.int32, device=dev)
+            torch.cuda.synchronize()
+            t0 = time.perf_counter()
+            A.aladdin_place_round(c2.handle, w2.n_cand, t_in, t_pr, t_w, pl)
+            times.append((time.perf_counter() - t0) * 1000.0)
+    print("round mode ok: %d rounds, best %.2f ms" % (len(times), min(times)))
+
+
 def profiled_traffic():
     """DRAM bytes per launch of the scoring kernel from the committed ncu
     summary, or None if the kernel source changed since it was taken."""
@@ -400,7 +424,7 @@ def main():
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--no-cpu-baseline", dest="cpu_baseline", action="store_false")
-    ap.add_argument("--mode", default="full", choices=["full", "kernel"],
+    ap.add_argument("--mode", default="full", choices=["full", "kernel", "round"],
                     help="kernel: only warm-up + steps of the device-resident step (for profilers)")
     args = ap.parse_args()
     if args.warmup < 3:
@@ -409,6 +433,8 @@ def main():
         run_reference(args)
     elif args.mode == "kernel":
         run_kernel_only(args)
+    elif args.mode == "round":
+        run_round_only(args)
     else:
         run_ours(args)
 

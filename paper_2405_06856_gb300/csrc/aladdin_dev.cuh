@@ -213,23 +213,28 @@ struct OpAdd {
     __device__ __forceinline__ T operator()(T a, T b) const { return a + b; }
 };
 
-// Inclusive prefix over x; returns the total.
+// Inclusive prefix over x; returns the total. All E rows are scanned at once
+// (independent shuffle chains); only the E row totals chain through a carry.
 template <int E, typename T, typename Op>
 __device__ __forceinline__ T scan_prefix(T (&v)[E], Op op, T ident)
 {
     const int lane = threadIdx.x & 31;
+#pragma unroll
+    for (int d = 1; d < 32; d <<= 1) {
+#pragma unroll
+        for (int e = 0; e < E; ++e) {
+            const T u = __shfl_up_sync(FULL, v[e], d);
+            if (lane >= d) v[e] = op(v[e], u);
+        }
+    }
+    T tot[E];
+#pragma unroll
+    for (int e = 0; e < E; ++e) tot[e] = __shfl_sync(FULL, v[e], 31);
     T carry = ident;
 #pragma unroll
     for (int e = 0; e < E; ++e) {
-        T s = v[e];
-#pragma unroll
-        for (int d = 1; d < 32; d <<= 1) {
-            const T u = __shfl_up_sync(FULL, s, d);
-            if (lane >= d) s = op(s, u);
-        }
-        s = op(carry, s);
-        v[e] = s;
-        carry = __shfl_sync(FULL, s, 31);
+        v[e] = op(carry, v[e]);
+        carry = op(carry, tot[e]);
     }
     return carry;
 }
@@ -239,20 +244,26 @@ template <int E, typename T, typename Op>
 __device__ __forceinline__ T scan_suffix_excl(T (&v)[E], Op op, T ident)
 {
     const int lane = threadIdx.x & 31;
+#pragma unroll
+    for (int d = 1; d < 32; d <<= 1) {
+#pragma unroll
+        for (int e = 0; e < E; ++e) {
+            const T u = __shfl_down_sync(FULL, v[e], d);
+            if (lane + d < 32) v[e] = op(v[e], u);
+        }
+    }
+    T tot[E], nxt[E];
+#pragma unroll
+    for (int e = 0; e < E; ++e) {
+        tot[e] = __shfl_sync(FULL, v[e], 0);
+        nxt[e] = __shfl_down_sync(FULL, v[e], 1);
+        if (lane == 31) nxt[e] = ident;
+    }
     T carry = ident;
 #pragma unroll
     for (int e = E - 1; e >= 0; --e) {
-        T s = v[e];
-#pragma unroll
-        for (int d = 1; d < 32; d <<= 1) {
-            const T u = __shfl_down_sync(FULL, s, d);
-            if (lane + d < 32) s = op(s, u);
-        }
-        T nxt = __shfl_down_sync(FULL, s, 1);
-        if (lane == 31) nxt = ident;
-        const T row_total = __shfl_sync(FULL, s, 0);
-        v[e] = op(nxt, carry);
-        carry = op(carry, row_total);
+        v[e] = op(nxt[e], carry);
+        carry = op(carry, tot[e]);
     }
     return carry;
 }
