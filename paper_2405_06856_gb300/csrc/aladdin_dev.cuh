@@ -123,6 +123,7 @@ __device__ __forceinline__ float f_inf() { return __int_as_float(0x7f800000); }
 
 __device__ __forceinline__ long long floor_div_ll(long long x, long long d)
 {
+    if (d == 1) return x;
     long long q = x / d;
     if ((x % d != 0) && (x < 0)) q -= 1;
     return q;
@@ -213,59 +214,135 @@ struct OpAdd {
     __device__ __forceinline__ T operator()(T a, T b) const { return a + b; }
 };
 
-// Inclusive prefix over x; returns the total. All E rows are scanned at once
-// (independent shuffle chains); only the E row totals chain through a carry.
+// One value set of a fused scan: v[E] scanned over x with operator op.
+// Several independent sets advance level by level together (scan_*_fused),
+// so that their shuffles issue back to back instead of one latency chain per
+// set; only the E row totals chain through a carry.
 template <int E, typename T, typename Op>
-__device__ __forceinline__ T scan_prefix(T (&v)[E], Op op, T ident)
-{
-    const int lane = threadIdx.x & 31;
+struct ScanSet {
+    static constexpr int kE = E;
+    T (&v)[E];
+    Op op;
+    T ident;
+    T u[E], tot[E];
+    T total;
+    __device__ __forceinline__ ScanSet(T (&x)[E], Op o, T id) : v(x), op(o), ident(id) {}
+    __device__ __forceinline__ void fetch_up(int d)
+    {
 #pragma unroll
-    for (int d = 1; d < 32; d <<= 1) {
+        for (int e = 0; e < E; ++e) u[e] = __shfl_up_sync(FULL, v[e], d);
+    }
+    __device__ __forceinline__ void apply_up(int d, int lane)
+    {
+#pragma unroll
+        for (int e = 0; e < E; ++e)
+            if (lane >= d) v[e] = op(v[e], u[e]);
+    }
+    __device__ __forceinline__ void fetch_down(int d)
+    {
+#pragma unroll
+        for (int e = 0; e < E; ++e) u[e] = __shfl_down_sync(FULL, v[e], d);
+    }
+    __device__ __forceinline__ void apply_down(int d, int lane)
+    {
+#pragma unroll
+        for (int e = 0; e < E; ++e)
+            if (lane + d < 32) v[e] = op(v[e], u[e]);
+    }
+    __device__ __forceinline__ void fetch_tot_prefix()
+    {
+#pragma unroll
+        for (int e = 0; e < E; ++e) tot[e] = __shfl_sync(FULL, v[e], 31);
+    }
+    __device__ __forceinline__ void carry_prefix()
+    {
+        T carry = ident;
 #pragma unroll
         for (int e = 0; e < E; ++e) {
-            const T u = __shfl_up_sync(FULL, v[e], d);
-            if (lane >= d) v[e] = op(v[e], u);
+            v[e] = op(carry, v[e]);
+            carry = op(carry, tot[e]);
+        }
+        total = carry;
+    }
+    __device__ __forceinline__ void fetch_tot_suffix()
+    {
+#pragma unroll
+        for (int e = 0; e < E; ++e) {
+            tot[e] = __shfl_sync(FULL, v[e], 0);
+            u[e] = __shfl_down_sync(FULL, v[e], 1);
         }
     }
-    T tot[E];
+    __device__ __forceinline__ void carry_suffix(int lane)
+    {
+        T carry = ident;
 #pragma unroll
-    for (int e = 0; e < E; ++e) tot[e] = __shfl_sync(FULL, v[e], 31);
-    T carry = ident;
-#pragma unroll
-    for (int e = 0; e < E; ++e) {
-        v[e] = op(carry, v[e]);
-        carry = op(carry, tot[e]);
+        for (int e = E - 1; e >= 0; --e) {
+            const T nx = lane == 31 ? ident : u[e];
+            v[e] = op(nx, carry);
+            carry = op(carry, tot[e]);
+        }
+        total = carry;
     }
-    return carry;
+};
+
+template <int E, typename T, typename Op>
+__device__ __forceinline__ ScanSet<E, T, Op> scan_set(T (&v)[E], Op op, T ident)
+{
+    return ScanSet<E, T, Op>(v, op, ident);
 }
 
-// Exclusive suffix over x (elements y > x); returns the total.
-template <int E, typename T, typename Op>
-__device__ __forceinline__ T scan_suffix_excl(T (&v)[E], Op op, T ident)
+// Sets are fused while the values in flight fit in registers (E <= 4);
+// with more elements per lane the E chains of each set already overlap.
+constexpr int FUSE_MAX_E = 4;
+
+template <typename... S>
+__device__ __forceinline__ void scan_prefix_sets(S&... s)
 {
     const int lane = threadIdx.x & 31;
 #pragma unroll
     for (int d = 1; d < 32; d <<= 1) {
-#pragma unroll
-        for (int e = 0; e < E; ++e) {
-            const T u = __shfl_down_sync(FULL, v[e], d);
-            if (lane + d < 32) v[e] = op(v[e], u);
-        }
+        (s.fetch_up(d), ...);
+        (s.apply_up(d, lane), ...);
     }
-    T tot[E], nxt[E];
+    (s.fetch_tot_prefix(), ...);
+    (s.carry_prefix(), ...);
+}
+
+template <typename... S>
+__device__ __forceinline__ void scan_suffix_excl_sets(S&... s)
+{
+    const int lane = threadIdx.x & 31;
 #pragma unroll
-    for (int e = 0; e < E; ++e) {
-        tot[e] = __shfl_sync(FULL, v[e], 0);
-        nxt[e] = __shfl_down_sync(FULL, v[e], 1);
-        if (lane == 31) nxt[e] = ident;
+    for (int d = 1; d < 32; d <<= 1) {
+        (s.fetch_down(d), ...);
+        (s.apply_down(d, lane), ...);
     }
-    T carry = ident;
-#pragma unroll
-    for (int e = E - 1; e >= 0; --e) {
-        v[e] = op(nxt[e], carry);
-        carry = op(carry, tot[e]);
+    (s.fetch_tot_suffix(), ...);
+    (s.carry_suffix(lane), ...);
+}
+
+// Inclusive prefix scans over x of every set; each set's total in .total.
+template <typename S0, typename... S>
+__device__ __forceinline__ void scan_prefix_fused(S0& s0, S&... s)
+{
+    if constexpr (S0::kE <= FUSE_MAX_E) {
+        scan_prefix_sets(s0, s...);
+    } else {
+        scan_prefix_sets(s0);
+        (scan_prefix_sets(s), ...);
     }
-    return carry;
+}
+
+// Exclusive suffix scans over x (elements y > x) of every set; totals in .total.
+template <typename S0, typename... S>
+__device__ __forceinline__ void scan_suffix_excl_fused(S0& s0, S&... s)
+{
+    if constexpr (S0::kE <= FUSE_MAX_E) {
+        scan_suffix_excl_sets(s0, s...);
+    } else {
+        scan_suffix_excl_sets(s0);
+        (scan_suffix_excl_sets(s), ...);
+    }
 }
 
 template <typename T, typename Op>
@@ -285,11 +362,18 @@ struct BuildSmem {
     uint8_t pend[32 * E];
 };
 
-__device__ __forceinline__ void write_row(const DevParams& P, const ClusterDev& C, long long rowid,
-                                          float s, float inv_s, int M, long long P_pend,
-                                          int rho, int rho_next, int n_p, long long A, long long PR,
-                                          long long PRA, long long PM, long long SM, float pmA,
-                                          float pmAp, float smS, float smSp)
+// One table row in its stored form (see the layout above) and its exact
+// integer aggregates.
+struct RowVals {
+    float4 v0, v1;
+    float2 ext;
+    AuxRow aux;
+};
+
+__device__ __forceinline__ RowVals make_row(const DevParams& P, float inv_s, int M, long long P_pend,
+                                            int rho, int rho_next, int n_p, long long A,
+                                            long long PR, long long PRA, long long PM, long long SM,
+                                            float pmA, float pmAp, float smS, float smSp)
 {
     float kvB1;
     if (SM > (long long)M) kvB1 = -f_inf();
@@ -297,45 +381,82 @@ __device__ __forceinline__ void write_row(const DevParams& P, const ClusterDev& 
     else kvB1 = (float)floor_div_ll((long long)M - P.j - PM, P.h);
     const float kvE = (float)(floor_div_ll((long long)M - (long long)P.j * (n_p + 1), P.h) - A);
     const float nf = (float)n_p;
-    float4 v0, v1;
-    v0.x = __int_as_float(rho_next);
-    v0.y = kvB1;
-    v0.z = kvE;
-    v0.w = -(P.c2_over_k2 * (float)PR + (float)PRA);
-    v1.x = P.c3_over_k2 + P.c2_over_k2 * nf + (float)A + 0.5f * nf - P.thTdec_over_k2 * inv_s;
-    v1.y = -0.5f * nf;
-    v1.z = pmA;
-    v1.w = smS * inv_s - (P.k1 * (float)P_pend + P.c1);
-    float4* t = C.tab + rowid * ROW_F4;
-    t[0] = v0;
-    t[1] = v1;
-    C.tab2[rowid] = make_float2(pmAp, smSp * inv_s);
-    AuxRow ar;
-    ar.PM = PM;
-    ar.SM = SM;
-    ar.A = A;
-    ar.PR = PR;
-    ar.PRA = PRA;
-    ar.n = n_p;
-    ar.rho = rho;
-    C.aux[rowid] = ar;
-    (void)s;
+    RowVals o;
+    o.v0.x = __int_as_float(rho_next);
+    o.v0.y = kvB1;
+    o.v0.z = kvE;
+    o.v0.w = -(P.c2_over_k2 * (float)PR + (float)PRA);
+    o.v1.x = P.c3_over_k2 + P.c2_over_k2 * nf + (float)A + 0.5f * nf - P.thTdec_over_k2 * inv_s;
+    o.v1.y = -0.5f * nf;
+    o.v1.z = pmA;
+    o.v1.w = smS * inv_s - (P.k1 * (float)P_pend + P.c1);
+    o.ext = make_float2(pmAp, smSp * inv_s);
+    o.aux.PM = PM;
+    o.aux.SM = SM;
+    o.aux.A = A;
+    o.aux.PR = PR;
+    o.aux.PRA = PRA;
+    o.aux.n = n_p;
+    o.aux.rho = rho;
+    return o;
 }
+
+__device__ __forceinline__ void store_row(const ClusterDev& C, long long rowid, const RowVals& o)
+{
+    float4* t = C.tab + rowid * ROW_F4;
+    t[0] = o.v0;
+    t[1] = o.v1;
+    C.tab2[rowid] = o.ext;
+    C.aux[rowid] = o.aux;
+}
+
+// Shared-memory copies of one worker's breakpoints, record and key, kept by
+// the sliced placement round (pointers to this worker's entries).
+struct SliceCache {
+    unsigned short* rho;  // rho_{q+1} of rows q = 0..R-1
+    int* R;
+    float4* wrec;
+    unsigned long long* key;
+};
 
 // Build worker w's table (rows 0..R), its record and its capacity_norm key.
 // Called by all 32 lanes of one warp. Requests are loaded from the slot
 // arrays; an invalid request (in < 0, gen outside [0, pred), in + pred > K)
 // makes the worker infeasible for every candidate and sets err bit 1.
+// With `cache`, the worker's shared-memory copies are refreshed as well.
+// With a valid `cand`, the candidate is evaluated against the new table by
+// the lane that holds its row, and every lane returns its flags (else 0).
 template <int E>
-__device__ void build_table(const DevParams& P, const ClusterDev& C, int w, BuildSmem<E>& sm)
+__device__ unsigned build_table(const DevParams& P, const ClusterDev& C, int w, BuildSmem<E>& sm,
+                                const SliceCache* cache = nullptr, const CandRec* cand = nullptr)
 {
     const int lane = threadIdx.x & 31;
-    const int n = C.n[w];
     const long long base = (long long)w * C.cap;
     const long long rowbase = (long long)w * C.rows;
+    // Independent loads first: the slot loads do not wait for n (every slot
+    // below 32 E lies inside the worker's slot range; those past n are masked).
+    const int n = C.n[w];
     const float s = C.scale[w];
-    const float inv_s = 1.0f / s;
     const int M = C.M[w];
+    const float off = C.off[w];
+    const float rank_bits = C.wrec[w].w;
+    constexpr bool PRELOAD = E <= FUSE_MAX_E;  // registers allow it
+    constexpr int EL = PRELOAD ? E : 1;
+    int l_pd[EL], l_g[EL], l_pr[EL], l_in[EL];
+    double l_td[EL], l_wt[EL];
+    if constexpr (PRELOAD) {
+#pragma unroll
+        for (int e = 0; e < EL; ++e) {
+            const long long slot = base + e * 32 + lane;
+            l_pd[e] = C.pend[slot];
+            l_g[e] = C.gen[slot];
+            l_pr[e] = C.pred[slot];
+            l_in[e] = C.in[slot];
+            l_td[e] = C.tdec[slot];
+            l_wt[e] = C.wait[slot];
+        }
+    }
+    const float inv_s = 1.0f / s;
 
     unsigned key[E];
     long long sumP = 0, sumIn = 0, sumPred = 0;
@@ -347,10 +468,10 @@ __device__ void build_table(const DevParams& P, const ClusterDev& C, int w, Buil
         const int i = e * 32 + lane;
         if (i < n) {
             const long long slot = base + i;
-            const int pd = C.pend[slot];
-            const int g = pd ? 0 : C.gen[slot];
-            const int pr = C.pred[slot];
-            const int in = C.in[slot];
+            const int pd = PRELOAD ? l_pd[e % EL] : C.pend[slot];
+            const int g = pd ? 0 : (PRELOAD ? l_g[e % EL] : C.gen[slot]);
+            const int pr = PRELOAD ? l_pr[e % EL] : C.pred[slot];
+            const int in = PRELOAD ? l_in[e % EL] : C.in[slot];
             if (in < 0 || g < 0 || g >= pr || (long long)in + pr > (long long)P.K) bad = 1;
             int r = pr - g;
             r = r < 1 ? 1 : (r > P.K ? P.K : r);
@@ -359,23 +480,34 @@ __device__ void build_table(const DevParams& P, const ClusterDev& C, int w, Buil
             key[e] = ((unsigned)r << 9) | (unsigned)i;
             sm.a[i] = a;
             sm.pend[i] = (uint8_t)pd;
-            sm.bank[i] = pd ? 0.0f : (float)(P.thetad * P.T_decd * (double)g - C.tdec[slot]);
+            sm.bank[i] = pd ? 0.0f
+                            : (float)(P.thetad * P.T_decd * (double)g -
+                                      (PRELOAD ? l_td[e % EL] : C.tdec[slot]));
             sumIn += in;
             sumPred += pr;
             if (pd) {
                 sumP += in;
-                wpmax = fmaxf(wpmax, (float)C.wait[slot]);
+                wpmax = fmaxf(wpmax, (float)(PRELOAD ? l_wt[e % EL] : C.wait[slot]));
                 npend += 1;
             }
         } else {
             key[e] = 0xffffffffu;
         }
     }
-    sumP = warp_reduce(sumP, OpAdd<long long>());
-    sumIn = warp_reduce(sumIn, OpAdd<long long>());
-    sumPred = warp_reduce(sumPred, OpAdd<long long>());
-    wpmax = warp_reduce(wpmax, OpMax<float>());
-    npend = warp_reduce(npend, OpAdd<int>());
+    // Warp sums, interleaved.
+#pragma unroll
+    for (int d = 16; d > 0; d >>= 1) {
+        const long long o0 = __shfl_xor_sync(FULL, sumP, d);
+        const long long o1 = __shfl_xor_sync(FULL, sumIn, d);
+        const long long o2 = __shfl_xor_sync(FULL, sumPred, d);
+        const float o3 = __shfl_xor_sync(FULL, wpmax, d);
+        const int o4 = __shfl_xor_sync(FULL, npend, d);
+        sumP += o0;
+        sumIn += o1;
+        sumPred += o2;
+        wpmax = wpmax > o3 ? wpmax : o3;
+        npend += o4;
+    }
     bad = __any_sync(FULL, bad);
     __syncwarp();
 
@@ -444,6 +576,7 @@ __device__ void build_table(const DevParams& P, const ClusterDev& C, int w, Buil
         first[e] = valid && (x == 0 || pv != r[e]);
         last[e] = valid && (x == n - 1 || nx != r[e]);
     }
+    const int r0 = __shfl_sync(FULL, r[0], 0);
     // Prefix sums over the sorted order.
     int rowid[E];
     long long pre_r[E], pre_ra[E], pre_a[E];
@@ -457,10 +590,13 @@ __device__ void build_table(const DevParams& P, const ClusterDev& C, int w, Buil
         pre_ra[e] = rr * aa + rr * (rr + 1) / 2;
         pre_a[e] = aa;
     }
-    const int R = scan_prefix<E>(rowid, OpAdd<int>(), 0);
-    scan_prefix<E>(pre_r, OpAdd<long long>(), 0LL);
-    scan_prefix<E>(pre_ra, OpAdd<long long>(), 0LL);
-    const long long tot_a = scan_prefix<E>(pre_a, OpAdd<long long>(), 0LL);
+    auto s_row = scan_set(rowid, OpAdd<int>(), 0);
+    auto s_r = scan_set(pre_r, OpAdd<long long>(), 0LL);
+    auto s_ra = scan_set(pre_ra, OpAdd<long long>(), 0LL);
+    auto s_a = scan_set(pre_a, OpAdd<long long>(), 0LL);
+    scan_prefix_fused(s_row, s_r, s_ra, s_a);
+    const int R = s_row.total;
+    const long long tot_a = s_a.total;
 
     // Per-breakpoint KV and cumulative decode time.
 #pragma unroll
@@ -473,8 +609,8 @@ __device__ void build_table(const DevParams& P, const ClusterDev& C, int w, Buil
         }
         if (last[e]) {
             const long long np = n - (x + 1);
-            const long long A = tot_a - pre_a[e];
             const long long rr = r[e];
+            const long long A = tot_a - pre_a[e];
             const long long Sb = pre_r[e] + rr * np;
             const long long SK = pre_ra[e] + np * (rr * (rr + 1) / 2) + rr * A;
             sm.Tp[rowid[e]] = s * (P.c3 * (float)rr + P.c2 * (float)Sb + P.k2 * (float)SK);
@@ -515,12 +651,29 @@ __device__ void build_table(const DevParams& P, const ClusterDev& C, int w, Buil
             SMx[e] = kv;
         }
     }
-    scan_prefix<E>(pmA, OpMin<float>(), f_inf());
-    scan_prefix<E>(pmAp, OpMin<float>(), f_inf());
-    const float smS0 = scan_suffix_excl<E>(smS, OpMin<float>(), f_inf());
-    const float smSp0 = scan_suffix_excl<E>(smSp, OpMin<float>(), f_inf());
-    scan_prefix<E>(PMx, OpMax<long long>(), LL_NONE);
-    const long long SM0 = scan_suffix_excl<E>(SMx, OpMax<long long>(), LL_NONE);
+    auto s_pmA = scan_set(pmA, OpMin<float>(), f_inf());
+    auto s_pmAp = scan_set(pmAp, OpMin<float>(), f_inf());
+    auto s_PM = scan_set(PMx, OpMax<long long>(), LL_NONE);
+    auto s_smS = scan_set(smS, OpMin<float>(), f_inf());
+    auto s_smSp = scan_set(smSp, OpMin<float>(), f_inf());
+    auto s_SM = scan_set(SMx, OpMax<long long>(), LL_NONE);
+    scan_prefix_fused(s_pmA, s_pmAp, s_PM);
+    scan_suffix_excl_fused(s_smS, s_smSp, s_SM);
+    const float smS0 = s_smS.total;
+    const float smSp0 = s_smSp.total;
+    const long long SM0 = s_SM.total;
+
+    // Worker record (every lane; lane 0 stores it).
+    float4 wr;
+    wr.x = inv_s;
+    wr.y = off * inv_s * P.inv_k1 + P.c1_over_k1 + (float)sumP;
+    wr.z = npend > 0 ? (P.T_pre - wpmax - off) * inv_s * P.inv_k1 - P.c1_over_k1 - (float)sumP
+                     : f_inf();
+    wr.w = rank_bits;
+    const bool want = cand != nullptr && cand->valid;
+    const int rc = want ? cand->ri : 0;
+    unsigned cf = 0;
+    bool mine = false;
 
     if (!bad) {
 #pragma unroll
@@ -531,32 +684,37 @@ __device__ void build_table(const DevParams& P, const ClusterDev& C, int w, Buil
                 const long long A = tot_a - pre_a[e];
                 const int nxt = (x == n - 1) ? 0x7fffffff : rnext[e];
                 const long long SM = SMx[e] == LL_NONE ? 0 : SMx[e];
-                write_row(P, C, rowbase + rowid[e], s, inv_s, M, sumP, r[e], nxt, np, A,
-                          pre_r[e], pre_ra[e], PMx[e], SM, pmA[e], pmAp[e], smS[e], smSp[e]);
+                const RowVals o = make_row(P, inv_s, M, sumP, r[e], nxt, np, A, pre_r[e], pre_ra[e],
+                                           PMx[e], SM, pmA[e], pmAp[e], smS[e], smSp[e]);
+                store_row(C, rowbase + rowid[e], o);
+                if (cache && rowid[e] < R) cache->rho[rowid[e]] = (unsigned short)nxt;
+                if (want && r[e] <= rc && rc < nxt) {
+                    float m;
+                    cf = eval_pair(o.v0, o.v1, o.ext, wr, *cand, m);
+                    mine = true;
+                }
             }
         }
     }
     if (lane == 0) {
+        RowVals o;
         if (!bad) {
-            write_row(P, C, rowbase, s, inv_s, M, sumP, 0, n > 0 ? r[0] : 0x7fffffff, n, tot_a, 0,
-                      0, LL_NONE, SM0 == LL_NONE ? 0 : SM0, f_inf(), f_inf(), smS0, smSp0);
+            o = make_row(P, inv_s, M, sumP, 0, n > 0 ? r0 : 0x7fffffff, n, tot_a, 0, 0, LL_NONE,
+                         SM0 == LL_NONE ? 0 : SM0, f_inf(), f_inf(), smS0, smSp0);
             C.R[w] = R;
         } else {
             // An invalid request: no candidate fits this worker.
-            write_row(P, C, rowbase, s, inv_s, M, 0, 0, 0x7fffffff, 0, 0, 0, 0, LL_NONE,
-                      (long long)M + 1, f_inf(), f_inf(), f_inf(), f_inf());
+            o = make_row(P, inv_s, M, 0, 0, 0x7fffffff, 0, 0, 0, 0, LL_NONE, (long long)M + 1,
+                         f_inf(), f_inf(), f_inf(), f_inf());
             C.R[w] = 0;
             atomicOr(C.err, 1u);
         }
-        const float off = C.off[w];
-        const float ZO = off * inv_s * P.inv_k1 + P.c1_over_k1 + (float)sumP;
-        const float ZW = npend > 0 ? (P.T_pre - wpmax - off) * inv_s * P.inv_k1 - P.c1_over_k1 -
-                                         (float)sumP
-                                   : f_inf();
-        float4 wr = C.wrec[w];
-        wr.x = inv_s;
-        wr.y = ZO;
-        wr.z = ZW;
+        store_row(C, rowbase, o);
+        if (want && (bad || n == 0 || rc < r0)) {
+            float m;
+            cf = eval_pair(o.v0, o.v1, o.ext, wr, *cand, m);
+            mine = true;
+        }
         C.wrec[w] = wr;
         const double B = (double)n;
         const double L = __dadd_rn((double)sumIn, __dmul_rn(P.gammad, (double)sumPred));
@@ -564,9 +722,19 @@ __device__ void build_table(const DevParams& P, const ClusterDev& C, int w, Buil
         // 2^53); non-negative doubles order like their bit patterns, and code 0
         // is kept for a worker holding an invalid request.
         const double q = __dadd_rn(__dmul_rn(B, B), __dmul_rn(L, L));
-        C.key[w] = bad ? 0ull : (unsigned long long)__double_as_longlong(q) + 1ull;
+        const unsigned long long kq = bad ? 0ull : (unsigned long long)__double_as_longlong(q) + 1ull;
+        C.key[w] = kq;
+        if (cache) {
+            if (!bad && n > 0 && R > 0) cache->rho[0] = (unsigned short)r0;
+            *cache->R = bad ? 0 : R;
+            *cache->wrec = wr;
+            *cache->key = kq;
+        }
     }
     __syncwarp();
+    if (!want) return 0u;
+    const unsigned who = __ballot_sync(FULL, mine);
+    return __shfl_sync(FULL, cf, who ? __ffs(who) - 1 : 0);
 }
 
 }  // namespace aladdin

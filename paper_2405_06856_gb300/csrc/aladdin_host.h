@@ -51,7 +51,12 @@ struct RoundIO {
     int* status;             // device: 0 ok, 1 halted at the first failure, -2 capacity
     int stop_at_fail;
     long long hb;
+    // exchange buffer of the sliced round (ROUND_XBUF_BYTES), or nullptr to
+    // use the single-CTA round
+    void* xbuf;
 };
+constexpr int ROUND_XBUF_SMS = 1024;  // largest SM count the exchange buffer serves
+constexpr size_t ROUND_XBUF_BYTES = 24 * (size_t)ROUND_XBUF_SMS + 16;
 cudaError_t launch_round(const DevParams& P, const ClusterDev& C, const RoundIO& io,
                          cudaStream_t st);
 

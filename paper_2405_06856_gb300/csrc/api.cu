@@ -130,6 +130,7 @@ struct aladdin_cluster {
     DevBuf s_off, s_rin, s_rgen, s_rpred, s_rtdec;
     unsigned long long* d_stats = nullptr;
     int* d_status = nullptr;
+    void* d_xround = nullptr;  // exchange buffer of the sliced placement round
     // optional CUDA-event timing of the scoring kernel
     bool timing = false;
     std::vector<cudaEvent_t> ev;   // pairs (start, stop)
@@ -232,6 +233,7 @@ int cluster_alloc(aladdin_cluster* cl, const aladdin_params& p, int W,
 #undef AL
     CK(cl->alloc(&p0, sizeof(unsigned long long) * 4)); cl->d_stats = (unsigned long long*)p0;
     CK(cl->alloc(&p0, sizeof(int) * 4)); cl->d_status = (int*)p0;
+    CK(cl->alloc(&p0, ROUND_XBUF_BYTES)); cl->d_xround = p0;
 
     std::vector<float> hs(W);
     std::vector<double> hsd(W);
@@ -570,6 +572,7 @@ int aladdin_place_round(aladdin_cluster* cl, int32_t n_cand, const int32_t* in,
     io.placement = dpl;
     io.sim = 0;
     io.status = cl->d_status;
+    io.xbuf = cl->d_xround;
     CK(launch_round(cl->dp, cl->dev, io, cl->st));
     CK(launch_rank(cl->dev, cl->st));
     cl->round_open = true;
@@ -577,6 +580,7 @@ int aladdin_place_round(aladdin_cluster* cl, int32_t n_cand, const int32_t* in,
     int status = 0;
     CK(cudaMemcpyAsync(&status, cl->d_status, sizeof(int), cudaMemcpyDeviceToHost, cl->st));
     CK(cudaStreamSynchronize(cl->st));
+    if (status == -4) return ALADDIN_ERR_TIMEOUT;
     return status == -2 ? ALADDIN_ERR_CAPACITY : ALADDIN_OK;
 }
 
@@ -763,6 +767,7 @@ int simulate_impl(const aladdin_params& p, const aladdin_worker_cfg& cfg, int32_
         io.status = cl.d_status;
         io.stop_at_fail = stop_at_fail ? 1 : 0;
         io.hb = hb;
+        io.xbuf = cl.d_xround;
         CK(launch_round(cl.dp, cl.dev, io, st));
         next = end;
         CK(launch_advance(cl.dp, cl.dev, t, H, cl.d_stats, cl.d_status, st));
@@ -778,6 +783,7 @@ int simulate_impl(const aladdin_params& p, const aladdin_worker_cfg& cfg, int32_
             CK(cudaMemcpyAsync(&status, cl.d_status, sizeof(int), cudaMemcpyDeviceToHost, st));
             CK(cudaStreamSynchronize(st));
             if (status == -2) return ALADDIN_ERR_CAPACITY;
+            if (status == -4) return ALADDIN_ERR_TIMEOUT;
             if (status == 1) {
                 halted = true;
                 break;

@@ -148,6 +148,351 @@ __global__ void __launch_bounds__(ROUND_THREADS) k_round(DevParams P, ClusterDev
     }
 }
 
+// ---------------------------------------------------------------------------
+// Sliced round: the workers are split into contiguous slices, one per CTA of a
+// cooperative grid (one CTA when they fit). Each CTA keeps its slice's
+// breakpoints (16-bit rho_{p+1} of rows 0..R-1), request counts, worker
+// records and keys in shared memory, so locating a candidate's row is a
+// shared-memory search and one global load of the row.
+//
+// Candidate c is committed lazily: its winner's request is appended, and the
+// winner's table rebuilt, by warp 0 of the owning CTA at the start of step
+// c + 1, which evaluates candidate c + 1 against that worker inside the
+// rebuild while the other warps evaluate it against the rest of the slice.
+// A step ends with one CTA barrier after which every warp reduces the warp
+// bests itself; with several CTAs the CTA bests are exchanged through global
+// memory behind one grid barrier (an arrival counter polled with a bounded
+// wait) and a second CTA barrier.
+constexpr int R2_MAX_WARPS = 16;
+// 512 threads (128 registers each) for up to 128 slots per worker; 256
+// threads (255 registers) for larger tables, whose rebuild needs them.
+template <int E>
+__host__ __device__ constexpr int r2_threads()
+{
+    return E >= 8 ? 256 : 512;
+}
+constexpr long long GRID_WAIT_LIMIT = 1ll << 22;  // polls of the arrival counter (seconds)
+constexpr int NONE = 0x7fffffff;
+
+struct R2Args {
+    DevParams P;
+    ClusterDev C;
+    RoundIO io;
+    int G;                          // CTAs
+    int slice;                      // workers per CTA
+    unsigned long long* xkey;       // [2 * G] best key per CTA (two parities)
+    int* xidx;                      // [2 * G] its worker (NONE: none; bit 30: full)
+    unsigned int* arrive;           // grid arrival counter, zero at launch
+};
+
+template <int E>
+struct R2Smem {
+    BuildSmem<E> build;
+    unsigned long long bk[2][R2_MAX_WARPS];
+    int bw[2][R2_MAX_WARPS];
+    int bf[2][R2_MAX_WARPS];
+    int gwin[2];
+    int stop;
+};
+
+__device__ __forceinline__ unsigned ld_acquire(const unsigned* p)
+{
+    unsigned v;
+    asm volatile("ld.acquire.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
+    return v;
+}
+
+__device__ __forceinline__ int r2_find(const unsigned short* rho, int R, int r)
+{
+    int lo = 0, hi = R;  // first row whose rho_{p+1} exceeds r; row R is unbounded
+    while (lo < hi) {
+        const int mid = (lo + hi) >> 1;
+        if ((int)rho[mid] > r) hi = mid;
+        else lo = mid + 1;
+    }
+    return lo;
+}
+
+// better() carrying the winner's "worker full" flag along.
+__device__ __forceinline__ void better_f(unsigned long long& bk, int& bw, int& bf,
+                                         unsigned long long ok, int ow, int of)
+{
+    if (ow != NONE && (bw == NONE || ok > bk || (ok == bk && ow < bw))) {
+        bk = ok;
+        bw = ow;
+        bf = of;
+    }
+}
+
+__device__ __forceinline__ void reduce_f(unsigned long long& bk, int& bw, int& bf, int width)
+{
+#pragma unroll
+    for (int d = 16; d > 0; d >>= 1) {
+        if (d >= width) continue;
+        const unsigned long long ok = __shfl_xor_sync(FULL, bk, d);
+        const int ow = __shfl_xor_sync(FULL, bw, d);
+        const int of = __shfl_xor_sync(FULL, bf, d);
+        better_f(bk, bw, bf, ok, ow, of);
+    }
+}
+
+template <int E>
+__global__ void __launch_bounds__(r2_threads<E>(), 1) k_round2(R2Args A)
+{
+    constexpr int R2_THREADS = r2_threads<E>();
+    constexpr int R2_WARPS = R2_THREADS / 32;
+    extern __shared__ __align__(16) unsigned char smraw[];
+    R2Smem<E>& sm = *reinterpret_cast<R2Smem<E>*>(smraw);
+    const int cap = A.C.cap;
+    unsigned char* tail = smraw + ((sizeof(R2Smem<E>) + 15) / 16) * 16;
+    float4* wrec_s = reinterpret_cast<float4*>(tail);
+    unsigned long long* key_s = reinterpret_cast<unsigned long long*>(wrec_s + A.slice);
+    int* R_s = reinterpret_cast<int*>(key_s + A.slice);
+    int* n_s = R_s + A.slice;
+    unsigned short* rho = reinterpret_cast<unsigned short*>(n_s + A.slice);
+
+    const DevParams& P = A.P;
+    const ClusterDev& C = A.C;
+    const RoundIO& io = A.io;
+    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    const int g = blockIdx.x;
+    const int w_lo = g * A.slice;
+    const int nloc = max(0, min(C.W, w_lo + A.slice) - w_lo);
+
+    // slice state into shared memory
+    for (int lw = tid; lw < nloc; lw += R2_THREADS) {
+        const int w = w_lo + lw;
+        R_s[lw] = C.R[w];
+        n_s[lw] = C.n[w];
+        wrec_s[lw] = C.wrec[w];
+        key_s[lw] = C.key[w];
+    }
+    __syncthreads();
+    for (int k = tid; k < nloc * cap; k += R2_THREADS) {
+        const int lw = k / cap, q = k - lw * cap;
+        if (q < R_s[lw])
+            rho[k] = (unsigned short)__float_as_int(C.tab[((long long)(w_lo + lw) * C.rows + q) * ROW_F4].x);
+    }
+    if (tid == 0) sm.stop = (io.sim && *io.status != 0) ? 1 : 0;
+    __syncthreads();
+    if (sm.stop) return;
+
+    const int n_wait0 = io.sim ? *io.n_wait : 0;
+    const int n_cand = io.sim ? n_wait0 + (int)(io.arr_end - io.arr_begin) : io.n_cand;
+    int keep = 0;        // CTA 0 thread 0: new waiting-list length
+    int pend_w = -1;     // this slice's winner of the previous step, not yet appended
+    int32_t pa = 0, pr = 0;
+    double pwd = 0.0;    // its request
+
+    auto append = [&](int w) {  // warp 0: commit the owed request to w
+        if (lane == 0) {
+            const int lw = w - w_lo;
+            const int nw = n_s[lw];
+            const long long slot = (long long)w * C.cap + nw;
+            C.in[slot] = pa;
+            C.gen[slot] = 0;
+            C.pred[slot] = pr;
+            C.tdec[slot] = 0.0;
+            C.pend[slot] = 1;
+            C.wait[slot] = pwd;
+            C.n[w] = nw + 1;
+            n_s[lw] = nw + 1;
+        }
+        __syncwarp();
+    };
+
+    for (int c = 0; c < n_cand; ++c) {
+        const int par = c & 1;
+        long long tix = 0;
+        int32_t a, r;
+        double wd;
+        if (io.sim) {
+            tix = c < n_wait0 ? io.wl[c] : io.arr_begin + (c - n_wait0);
+            a = io.tin[tix];
+            r = io.tpred[tix];
+            wd = io.t_now - io.t_arr[tix];
+        } else {
+            a = io.in[c];
+            r = io.pred[c];
+            wd = io.wait ? (double)io.wait[c] : 0.0;
+        }
+        const CandRec cr = make_cand(P, a, r, (float)wd, c);
+        unsigned long long bk = 0ull;
+        int bw = NONE, bf = 0;
+        const bool rebuilding = pend_w >= 0;
+        if (rebuilding && warp == 0) {
+            append(pend_w);
+            const int lw = pend_w - w_lo;
+            SliceCache sc{rho + (long long)lw * cap, &R_s[lw], &wrec_s[lw], &key_s[lw]};
+            const unsigned f = build_table<E>(P, C, pend_w, sm.build, &sc, cr.valid ? &cr : nullptr);
+            if (lane == 0 && cr.valid && f == 15u) bk = key_s[lw], bw = pend_w, bf = n_s[lw] >= cap;
+        } else if (cr.valid) {
+            const int first = rebuilding ? tid - 32 : tid;
+            const int stride = rebuilding ? R2_THREADS - 32 : R2_THREADS;
+            for (int lw = first; lw < nloc; lw += stride) {
+                const int w = w_lo + lw;
+                if (w == pend_w) continue;
+                const int p = r2_find(rho + (long long)lw * cap, R_s[lw], cr.ri);
+                const long long row = (long long)w * C.rows + p;
+                const float4* t = C.tab + row * ROW_F4;
+                float m;
+                const unsigned f = eval_pair(t[0], t[1], C.tab2[row], wrec_s[lw], cr, m);
+                if (f == 15u) better_f(bk, bw, bf, key_s[lw], w, n_s[lw] >= cap);
+            }
+        }
+        reduce_f(bk, bw, bf, 32);
+        if (lane == 0) {
+            sm.bk[par][warp] = bk;
+            sm.bw[par][warp] = bw;
+            sm.bf[par][warp] = bf;
+        }
+        __syncthreads();
+        // every warp reduces the warp bests itself
+        bk = lane < R2_WARPS ? sm.bk[par][lane] : 0ull;
+        bw = lane < R2_WARPS ? sm.bw[par][lane] : NONE;
+        bf = lane < R2_WARPS ? sm.bf[par][lane] : 0;
+        reduce_f(bk, bw, bf, 32);  // every lane ends with the CTA best
+        if (A.G > 1) {
+            if (warp == 0) {
+                if (lane == 0) {
+                    A.xkey[par * A.G + g] = bk;
+                    A.xidx[par * A.G + g] = bw == NONE ? NONE : (bw | (bf ? 0x40000000 : 0));
+                    __threadfence();
+                    atomicAdd(A.arrive, 1u);
+                    const unsigned target = (unsigned)(c + 1) * (unsigned)A.G;
+                    bool ok = false;
+                    for (long long it = 0; it < GRID_WAIT_LIMIT; ++it) {
+                        if (ld_acquire(A.arrive) >= target) {
+                            ok = true;
+                            break;
+                        }
+                        __nanosleep(32);
+                    }
+                    __threadfence();
+                    if (!ok) {
+                        atomicOr(C.err, 4u);
+                        *io.status = -4;  // ALADDIN_ERR_TIMEOUT
+                        sm.stop = 2;
+                    }
+                }
+                __syncwarp();
+                bk = 0ull;
+                bw = NONE;
+                bf = 0;
+                for (int q = lane; q < A.G; q += 32) {
+                    const int iq = __ldcg(&A.xidx[par * A.G + q]);
+                    const int wq = iq == NONE ? NONE : (iq & 0x3fffffff);
+                    better_f(bk, bw, bf, __ldcg(&A.xkey[par * A.G + q]), wq,
+                             iq != NONE && (iq & 0x40000000));
+                }
+                reduce_f(bk, bw, bf, 32);
+                if (lane == 0) sm.gwin[par] = bw == NONE ? NONE : (bw | (bf ? 0x40000000 : 0));
+            }
+            __syncthreads();
+            if (sm.stop) break;
+            const int gw = sm.gwin[par];
+            bw = gw == NONE ? NONE : (gw & 0x3fffffff);
+            bf = gw != NONE && (gw & 0x40000000);
+        }
+        const int winner = !cr.valid ? -2 : (bw == NONE ? -1 : bw);
+        if (winner >= 0 && bf) {
+            if (tid == 0 && g == 0) {
+                *io.status = -2;  // ALADDIN_ERR_CAPACITY
+                if (!io.sim)
+                    for (int k = c; k < n_cand; ++k) io.placement[k] = -1;
+            }
+            pend_w = -1;
+            break;
+        }
+        pend_w = (winner >= w_lo && winner < w_lo + nloc) ? winner : -1;
+        pa = a;
+        pr = r;
+        pwd = wd;
+        if (g == 0 && tid == 0) {
+            if (!io.sim) {
+                io.placement[c] = winner;
+            } else if (winner >= 0) {
+                io.counters[1] += 1;
+            } else {
+                const double tau_alone = C.scaled[0] * (P.k1d * (double)a + P.c1d);
+                if (winner == -2 || wd + io.H + tau_alone > P.T_pred) io.counters[0] += 1;
+                else io.wl[keep++] = tix;
+            }
+        }
+    }
+    if (pend_w >= 0 && warp == 0) {
+        append(pend_w);
+        const int lw = pend_w - w_lo;
+        SliceCache sc{rho + (long long)lw * cap, &R_s[lw], &wrec_s[lw], &key_s[lw]};
+        build_table<E>(P, C, pend_w, sm.build, &sc, nullptr);
+    }
+    if (g == 0 && tid == 0 && io.sim && !sm.stop && *io.status == 0) {
+        *io.n_wait = keep;
+        if (io.stop_at_fail && io.counters[0] > 0) {
+            *io.status = 1;
+            io.counters[2] = (unsigned long long)io.hb;
+        }
+    }
+}
+
+// Shared memory of k_round2 for a slice of `slice` workers.
+template <int E>
+static size_t r2_smem(int slice, int cap)
+{
+    return ((sizeof(R2Smem<E>) + 15) / 16) * 16 + (size_t)slice * (16 + 8 + 4 + 4) +
+           (size_t)slice * cap * 2;
+}
+
+template <int E>
+static cudaError_t round2_e(const DevParams& P, const ClusterDev& C, const RoundIO& io,
+                            cudaStream_t st, bool* used)
+{
+    *used = false;
+    if (P.K > 65535) return cudaSuccess;  // 16-bit breakpoints
+    int dev = 0, sms = 0, smem_max = 0, coop = 0;
+    cudaError_t e;
+    if ((e = cudaGetDevice(&dev)) != cudaSuccess) return e;
+    if ((e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev)) != cudaSuccess ||
+        (e = cudaDeviceGetAttribute(&smem_max, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev)) !=
+            cudaSuccess ||
+        (e = cudaDeviceGetAttribute(&coop, cudaDevAttrCooperativeLaunch, dev)) != cudaSuccess)
+        return e;
+    if (sms > ROUND_XBUF_SMS) return cudaSuccess;
+    const size_t budget = (size_t)smem_max - 1024;
+    const size_t per_w = 32 + (size_t)C.cap * 2;
+    const size_t base = r2_smem<E>(0, C.cap);
+    if (budget <= base + per_w) return cudaSuccess;
+    const int slice_max = (int)((budget - base) / per_w);
+    int G = (C.W + slice_max - 1) / slice_max;
+    if (G > sms || (G > 1 && !coop)) return cudaSuccess;  // use the single-CTA round
+    const int slice = (C.W + G - 1) / G;
+    const size_t smem = r2_smem<E>(slice, C.cap);
+    e = cudaFuncSetAttribute(k_round2<E>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         (int)smem);
+    if (e != cudaSuccess) return e;
+    R2Args A;
+    A.P = P;
+    A.C = C;
+    A.io = io;
+    A.G = G;
+    A.slice = slice;
+    A.xkey = reinterpret_cast<unsigned long long*>(io.xbuf);
+    A.xidx = reinterpret_cast<int*>(A.xkey + 2 * ROUND_XBUF_SMS);
+    A.arrive = reinterpret_cast<unsigned int*>(A.xidx + 2 * ROUND_XBUF_SMS);
+    if (G > 1) {
+        e = cudaMemsetAsync(A.arrive, 0, sizeof(unsigned int), st);
+        if (e != cudaSuccess) return e;
+        void* args[] = {&A};
+        e = cudaLaunchCooperativeKernel((const void*)k_round2<E>, dim3(G), dim3(r2_threads<E>()), args,
+                                        smem, st);
+    } else {
+        k_round2<E><<<1, r2_threads<E>(), smem, st>>>(A);
+        e = cudaGetLastError();
+    }
+    if (e == cudaSuccess) *used = true;
+    return e;
+}
+
 template <int E>
 static cudaError_t round_e(const DevParams& P, const ClusterDev& C, const RoundIO& io,
                            cudaStream_t st)
@@ -165,6 +510,19 @@ static cudaError_t round_e(const DevParams& P, const ClusterDev& C, const RoundI
 cudaError_t launch_round(const DevParams& P, const ClusterDev& C, const RoundIO& io,
                          cudaStream_t st)
 {
+    if (io.xbuf) {
+        bool used = false;
+        cudaError_t e = cudaSuccess;
+        switch (lanes_per_worker(C.cap)) {
+        case 1: e = round2_e<1>(P, C, io, st, &used); break;
+        case 2: e = round2_e<2>(P, C, io, st, &used); break;
+        case 4: e = round2_e<4>(P, C, io, st, &used); break;
+        case 8: e = round2_e<8>(P, C, io, st, &used); break;
+        case 16: e = round2_e<16>(P, C, io, st, &used); break;
+        default: return cudaErrorInvalidValue;
+        }
+        if (e != cudaSuccess || used) return e;
+    }
     switch (lanes_per_worker(C.cap)) {
     case 1: return round_e<1>(P, C, io, st);
     case 2: return round_e<2>(P, C, io, st);

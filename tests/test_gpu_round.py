@@ -151,3 +151,38 @@ def test_min_workers_matches_oracle(A, orc, synth):
     assert np.array_equal(got, ref), (got, ref)
     tot = [g * n if n > 0 else 10**9 for g, n in zip(gpus, ref)]
     assert total == min(tot) and best == int(np.argmin(tot))
+
+
+@pytest.mark.parametrize("W,b_cap,seed,per_worker,tpre,tdec", [
+    (1500, 512, 230, 12, 60.0, 12.0), (4096, 128, 231, 12, 60.0, 12.0),
+    (1500, 512, 232, 40, 40.0, 11.0)])
+def test_round_many_slices(A, orc, synth, W, b_cap, seed, per_worker, tpre, tdec):
+    """Clusters whose worker state does not fit one CTA's shared memory: the
+    round runs as a cooperative grid of worker slices exchanging per-slice
+    bests each candidate."""
+    wl = synth.make_cluster("slices", seed, W, per_worker, 60000, 1000, per_worker_random=True,
+                            b_cap=b_cap, params=dict(T_pre=tpre, T_dec=tdec))
+    with A.Cluster.from_workload(wl) as cl:
+        pl = cl.place_round(wl.cand_in, wl.cand_pred, wl.cand_wait)
+        oc = orc.Cluster.from_workload(wl)
+        ref = oc.place_round(wl.cand_in, wl.cand_pred, wl.cand_wait)
+        assert np.array_equal(pl, ref), np.argwhere(pl != ref)[:5]
+        assert 0 < (pl >= 0).mean() < 1
+        assert_same_state(cl, oc, "slices-%d" % W)
+        assert cl.status() == A.OK
+
+
+def test_simulate_many_slices(A, orc, synth):
+    """Fleet simulation on 450 workers of 512 slots (several worker slices):
+    waiting list, failures and realized latencies match the oracle."""
+    tr = synth.diurnal_trace(11, 6000, 3000.0, 500.0)
+    p = dict(synth.BASE_PARAMS, T_pre=100.0, T_dec=14.0)
+    ref = orc.simulate(p, 450, 512, 12000, 1.0, tr, 100.0, stop_at_fail=False, drain=True)
+    out = np.zeros(5)
+    A.aladdin_simulate(A.make_params(p, 512), A.make_cfgs([1], [12000], [1.0])[0], 450,
+                       A.make_trace(tr.t_arr, tr.req_in, tr.req_pred), 100.0, 0, 1, out)
+    assert ref["failed"] > 0
+    assert int(out[0]) == ref["failed"] and int(out[1]) == ref["placed"], (out, ref)
+    assert int(out[2]) == ref["heartbeats"]
+    assert out[3] == pytest.approx(ref["max_ttft"], rel=1e-12)
+    assert out[4] == pytest.approx(ref["max_atgt"], rel=1e-12)
