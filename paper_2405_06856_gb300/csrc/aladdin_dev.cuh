@@ -221,6 +221,7 @@ struct OpAdd {
 template <int E, typename T, typename Op>
 struct ScanSet {
     static constexpr int kE = E;
+    using value_type = T;
     T (&v)[E];
     Op op;
     T ident;
@@ -353,14 +354,74 @@ __device__ __forceinline__ T warp_reduce(T v, Op op)
     return v;
 }
 
-template <int E>
+// Scratch of one table build: EW element rows per lane, NW warps per worker.
+template <int EW, int NW = 1>
 struct BuildSmem {
-    long long kvrho[32 * E + 1];
-    int32_t a[32 * E];
-    float bank[32 * E];
-    float Tp[32 * E + 1];
-    uint8_t pend[32 * E];
+    static constexpr int N = 32 * EW * NW;
+    long long kvrho[N + 1];
+    int32_t a[N];
+    float bank[N];
+    float Tp[N + 1];
+    unsigned sorted[NW > 1 ? N : 1];  // cooperative builds: merged keys
+    alignas(16) unsigned runs[NW > 1 ? N : 1];  // each warp's keys (read as uint4)
+    long long pll[6][NW];             // per-warp partials
+    float pf[7][NW];
+    int pi[3][NW];
+    unsigned cflag;
+    uint8_t pend[N];
 };
+
+// Barrier of the NW warps building one table (warps 0..NW-1 of the CTA when
+// NW > 1; named barrier 1, so that the other warps may run on).
+template <int NW>
+__device__ __forceinline__ void group_sync()
+{
+    if constexpr (NW == 1) {
+        __syncwarp();
+    } else {
+        asm volatile("bar.sync 1, %0;" ::"r"(NW * 32) : "memory");
+    }
+}
+
+// Cross-warp combination of per-warp scan totals: the carry into warp q
+// (op over warps before q for a prefix, after q for a suffix) and the total.
+template <int NW, typename T, typename Op>
+__device__ __forceinline__ T carry_in(const T* part, int q, bool suffix, Op op, T ident, T& all)
+{
+    T c = ident;
+    all = ident;
+#pragma unroll
+    for (int k = 0; k < NW; ++k) {
+        const T t = part[k];
+        if (suffix ? k > q : k < q) c = op(c, t);
+        all = op(all, t);
+    }
+    return c;
+}
+
+template <int NW, typename Set>
+__device__ __forceinline__ void add_carry_prefix(Set& st, typename Set::value_type* part, int q)
+{
+    if constexpr (NW > 1) {
+        typename Set::value_type all;
+        const auto c = carry_in<NW>(part, q, false, st.op, st.ident, all);
+#pragma unroll
+        for (int e = 0; e < Set::kE; ++e) st.v[e] = st.op(c, st.v[e]);
+        st.total = all;
+    }
+}
+
+template <int NW, typename Set>
+__device__ __forceinline__ void add_carry_suffix(Set& st, typename Set::value_type* part, int q)
+{
+    if constexpr (NW > 1) {
+        typename Set::value_type all;
+        const auto c = carry_in<NW>(part, q, true, st.op, st.ident, all);
+#pragma unroll
+        for (int e = 0; e < Set::kE; ++e) st.v[e] = st.op(st.v[e], c);
+        st.total = all;
+    }
+}
 
 // One table row in its stored form (see the layout above) and its exact
 // integer aggregates.
@@ -420,21 +481,29 @@ struct SliceCache {
 };
 
 // Build worker w's table (rows 0..R), its record and its capacity_norm key.
-// Called by all 32 lanes of one warp. Requests are loaded from the slot
-// arrays; an invalid request (in < 0, gen outside [0, pred), in + pred > K)
-// makes the worker infeasible for every candidate and sets err bit 1.
-// With `cache`, the worker's shared-memory copies are refreshed as well.
-// With a valid `cand`, the candidate is evaluated against the new table by
-// the lane that holds its row, and every lane returns its flags (else 0).
-template <int E>
-__device__ unsigned build_table(const DevParams& P, const ClusterDev& C, int w, BuildSmem<E>& sm,
-                                const SliceCache* cache = nullptr, const CandRec* cand = nullptr)
+// Called by all lanes of NW warps (warps 0..NW-1 of the CTA when NW > 1);
+// element x = (q EW + e) 32 + lane of warp q, so 32 EW NW slots are covered.
+// Requests are loaded from the slot arrays; an invalid request (in < 0, gen
+// outside [0, pred), in + pred > K) makes the worker infeasible for every
+// candidate and sets err bit 1. With `cache`, the worker's shared-memory
+// copies are refreshed as well. With a valid `cand`, the candidate is
+// evaluated against the new table by the lane that holds its row, and every
+// lane returns its flags (else 0).
+template <int EW, int NW = 1>
+__device__ unsigned build_table(const DevParams& P, const ClusterDev& C, int w,
+                                BuildSmem<EW, NW>& sm, const SliceCache* cache = nullptr,
+                                const CandRec* cand = nullptr)
 {
+    constexpr int E = EW;
+    constexpr int RUN = 32 * EW;  // elements per warp
     const int lane = threadIdx.x & 31;
+    const int q = NW > 1 ? (int)(threadIdx.x >> 5) : 0;
+    const int x0 = q * RUN;
     const long long base = (long long)w * C.cap;
     const long long rowbase = (long long)w * C.rows;
     // Independent loads first: the slot loads do not wait for n (every slot
-    // below 32 E lies inside the worker's slot range; those past n are masked).
+    // below 32 E NW lies inside the worker's slot range; those past n are
+    // masked).
     const int n = C.n[w];
     const float s = C.scale[w];
     const int M = C.M[w];
@@ -447,7 +516,7 @@ __device__ unsigned build_table(const DevParams& P, const ClusterDev& C, int w, 
     if constexpr (PRELOAD) {
 #pragma unroll
         for (int e = 0; e < EL; ++e) {
-            const long long slot = base + e * 32 + lane;
+            const long long slot = base + x0 + e * 32 + lane;
             l_pd[e] = C.pend[slot];
             l_g[e] = C.gen[slot];
             l_pr[e] = C.pred[slot];
@@ -465,7 +534,7 @@ __device__ unsigned build_table(const DevParams& P, const ClusterDev& C, int w, 
     int bad = 0;
 #pragma unroll
     for (int e = 0; e < E; ++e) {
-        const int i = e * 32 + lane;
+        const int i = x0 + e * 32 + lane;
         if (i < n) {
             const long long slot = base + i;
             const int pd = PRELOAD ? l_pd[e % EL] : C.pend[slot];
@@ -494,7 +563,8 @@ __device__ unsigned build_table(const DevParams& P, const ClusterDev& C, int w, 
             key[e] = 0xffffffffu;
         }
     }
-    // Warp sums, interleaved.
+    // Sums over the worker's requests (warp shuffles interleaved, then the
+    // NW warp partials in warp order).
 #pragma unroll
     for (int d = 16; d > 0; d >>= 1) {
         const long long o0 = __shfl_xor_sync(FULL, sumP, d);
@@ -509,11 +579,77 @@ __device__ unsigned build_table(const DevParams& P, const ClusterDev& C, int w, 
         npend += o4;
     }
     bad = __any_sync(FULL, bad);
-    __syncwarp();
-
-    // Bitonic sort of (r, slot) keys, ascending.
+    if constexpr (NW > 1) {
+        if (lane == 0) {
+            sm.pll[0][q] = sumP;
+            sm.pll[1][q] = sumIn;
+            sm.pll[2][q] = sumPred;
+            sm.pf[0][q] = wpmax;
+            sm.pi[0][q] = npend;
+            sm.pi[1][q] = bad;
+        }
+    }
+    group_sync<NW>();
+    if constexpr (NW > 1) {
+        sumP = 0;
+        sumIn = 0;
+        sumPred = 0;
+        wpmax = -f_inf();
+        npend = 0;
+        bad = 0;
 #pragma unroll
-    for (int k = 2; k <= 32 * E; k <<= 1) {
+        for (int k = 0; k < NW; ++k) {
+            sumP += sm.pll[0][k];
+            sumIn += sm.pll[1][k];
+            sumPred += sm.pll[2][k];
+            const float o3 = sm.pf[0][k];
+            wpmax = wpmax > o3 ? wpmax : o3;
+            npend += sm.pi[0][k];
+            bad |= sm.pi[1][k];
+        }
+    }
+
+    // capacity_norm key: capacity_norm^2 is exact here (integer and
+    // half-integer terms below 2^53); non-negative doubles order like their
+    // bit patterns, and code 0 is kept for a worker holding an invalid request.
+    const double kB = (double)n;
+    const double kL = __dadd_rn((double)sumIn, __dmul_rn(P.gammad, (double)sumPred));
+    const double kQ = __dadd_rn(__dmul_rn(kB, kB), __dmul_rn(kL, kL));
+    const unsigned long long kq = bad ? 0ull : (unsigned long long)__double_as_longlong(kQ) + 1ull;
+
+    constexpr int N = BuildSmem<EW, NW>::N;
+    // Cooperative builds of up to 256 slots rank every key by counting the
+    // keys below it (keys of valid requests are distinct); larger ones sort
+    // each warp's run and merge the runs.
+    constexpr bool COUNT_RANK = NW > 1 && N <= 256;
+    if constexpr (COUNT_RANK) {
+#pragma unroll
+        for (int e = 0; e < E; ++e) sm.runs[x0 + e * 32 + lane] = key[e];
+        group_sync<NW>();
+        int rank[E];
+#pragma unroll
+        for (int e = 0; e < E; ++e) rank[e] = 0;
+        const uint4* run4 = reinterpret_cast<const uint4*>(sm.runs);
+#pragma unroll 8
+        for (int k = 0; k < N / 4; ++k) {
+            const uint4 v = run4[k];
+#pragma unroll
+            for (int e = 0; e < E; ++e)
+                rank[e] += (v.x < key[e]) + (v.y < key[e]) + (v.z < key[e]) + (v.w < key[e]);
+        }
+#pragma unroll
+        for (int e = 0; e < E; ++e)
+            if (x0 + e * 32 + lane < n) sm.sorted[rank[e]] = key[e];
+        group_sync<NW>();
+#pragma unroll
+        for (int e = 0; e < E; ++e) {
+            const int x = x0 + e * 32 + lane;
+            key[e] = x < n ? sm.sorted[x] : 0xffffffffu;
+        }
+    }
+    // Bitonic sort of (r, slot) keys, ascending, within each warp's run.
+#pragma unroll
+    for (int k = 2; k <= (COUNT_RANK ? 1 : RUN); k <<= 1) {
 #pragma unroll
         for (int jj = k >> 1; jj > 0; jj >>= 1) {
             if (jj >= 32) {
@@ -540,12 +676,41 @@ __device__ unsigned build_table(const DevParams& P, const ClusterDev& C, int w, 
             }
         }
     }
+    if constexpr (NW > 1 && !COUNT_RANK) {
+        // Merge the NW sorted runs: a key's rank is its position in its run
+        // plus the keys of the other runs before it (equal padding keys of
+        // earlier runs first).
+#pragma unroll
+        for (int e = 0; e < E; ++e) sm.runs[x0 + e * 32 + lane] = key[e];
+        group_sync<NW>();
+#pragma unroll
+        for (int e = 0; e < E; ++e) {
+            int rank = e * 32 + lane;
+#pragma unroll
+            for (int q2 = 0; q2 < NW; ++q2) {
+                if (q2 == q) continue;
+                const unsigned* run = sm.runs + q2 * RUN;
+                int lo = 0, hi = RUN;
+                while (lo < hi) {
+                    const int mid = (lo + hi) >> 1;
+                    const unsigned v = run[mid];
+                    if (q2 < q ? v <= key[e] : v < key[e]) lo = mid + 1;
+                    else hi = mid;
+                }
+                rank += lo;
+            }
+            sm.sorted[rank] = key[e];
+        }
+        group_sync<NW>();
+#pragma unroll
+        for (int e = 0; e < E; ++e) key[e] = sm.sorted[x0 + e * 32 + lane];
+    }
 
     int r[E], a[E], pd[E];
     float bank[E];
 #pragma unroll
     for (int e = 0; e < E; ++e) {
-        const int x = e * 32 + lane;
+        const int x = x0 + e * 32 + lane;
         if (x < n) {
             r[e] = (int)(key[e] >> 9);
             const int i = (int)(key[e] & 511u);
@@ -563,26 +728,34 @@ __device__ unsigned build_table(const DevParams& P, const ClusterDev& C, int w, 
     int rnext[E], first[E], last[E];
 #pragma unroll
     for (int e = 0; e < E; ++e) {
-        const int dn = __shfl_down_sync(FULL, r[e], 1);
-        const int up = __shfl_up_sync(FULL, r[e], 1);
-        int wrap_n = -1, wrap_p = -1;
-        if (e + 1 < E) wrap_n = __shfl_sync(FULL, r[e + 1 < E ? e + 1 : e], 0);
-        if (e > 0) wrap_p = __shfl_sync(FULL, r[e > 0 ? e - 1 : e], 31);
-        const int nx = lane < 31 ? dn : wrap_n;
-        const int pv = lane > 0 ? up : wrap_p;
-        const int x = e * 32 + lane;
+        const int x = x0 + e * 32 + lane;
+        int nx, pv;
+        if constexpr (NW > 1) {
+            nx = x + 1 < n ? (int)(sm.sorted[x + 1] >> 9) : -1;
+            pv = x > 0 && x - 1 < n ? (int)(sm.sorted[x - 1] >> 9) : -1;
+        } else {
+            const int dn = __shfl_down_sync(FULL, r[e], 1);
+            const int up = __shfl_up_sync(FULL, r[e], 1);
+            int wrap_n = -1, wrap_p = -1;
+            if (e + 1 < E) wrap_n = __shfl_sync(FULL, r[e + 1 < E ? e + 1 : e], 0);
+            if (e > 0) wrap_p = __shfl_sync(FULL, r[e > 0 ? e - 1 : e], 31);
+            nx = lane < 31 ? dn : wrap_n;
+            pv = lane > 0 ? up : wrap_p;
+        }
         const bool valid = x < n;
         rnext[e] = nx;
         first[e] = valid && (x == 0 || pv != r[e]);
         last[e] = valid && (x == n - 1 || nx != r[e]);
     }
-    const int r0 = __shfl_sync(FULL, r[0], 0);
+    int r0;
+    if constexpr (NW > 1) r0 = n > 0 ? (int)(sm.sorted[0] >> 9) : 0x7fffffff;
+    else r0 = __shfl_sync(FULL, r[0], 0);
     // Prefix sums over the sorted order.
     int rowid[E];
     long long pre_r[E], pre_ra[E], pre_a[E];
 #pragma unroll
     for (int e = 0; e < E; ++e) {
-        const bool valid = e * 32 + lane < n;
+        const bool valid = x0 + e * 32 + lane < n;
         rowid[e] = first[e];
         const long long rr = valid ? (long long)r[e] : 0;
         const long long aa = valid ? (long long)a[e] : 0;
@@ -595,13 +768,26 @@ __device__ unsigned build_table(const DevParams& P, const ClusterDev& C, int w, 
     auto s_ra = scan_set(pre_ra, OpAdd<long long>(), 0LL);
     auto s_a = scan_set(pre_a, OpAdd<long long>(), 0LL);
     scan_prefix_fused(s_row, s_r, s_ra, s_a);
+    if constexpr (NW > 1) {
+        if (lane == 0) {
+            sm.pi[2][q] = s_row.total;
+            sm.pll[3][q] = s_r.total;
+            sm.pll[4][q] = s_ra.total;
+            sm.pll[5][q] = s_a.total;
+        }
+        group_sync<NW>();
+        add_carry_prefix<NW>(s_row, sm.pi[2], q);
+        add_carry_prefix<NW>(s_r, sm.pll[3], q);
+        add_carry_prefix<NW>(s_ra, sm.pll[4], q);
+        add_carry_prefix<NW>(s_a, sm.pll[5], q);
+    }
     const int R = s_row.total;
     const long long tot_a = s_a.total;
 
     // Per-breakpoint KV and cumulative decode time.
 #pragma unroll
     for (int e = 0; e < E; ++e) {
-        const int x = e * 32 + lane;
+        const int x = x0 + e * 32 + lane;
         if (first[e]) {
             const long long b_at = n - x;
             const long long Kat = tot_a - (pre_a[e] - a[e]) + (long long)r[e] * b_at;
@@ -616,7 +802,7 @@ __device__ unsigned build_table(const DevParams& P, const ClusterDev& C, int w, 
             sm.Tp[rowid[e]] = s * (P.c3 * (float)rr + P.c2 * (float)Sb + P.k2 * (float)SK);
         }
     }
-    __syncwarp();
+    group_sync<NW>();
 
     // Per-request bounds and slacks.
     const float stall0 = s * (P.k1 * (float)sumP + P.c1);
@@ -624,7 +810,7 @@ __device__ unsigned build_table(const DevParams& P, const ClusterDev& C, int w, 
     long long PMx[E], SMx[E];
 #pragma unroll
     for (int e = 0; e < E; ++e) {
-        const int x = e * 32 + lane;
+        const int x = x0 + e * 32 + lane;
         const bool valid = x < n;
         pmA[e] = f_inf();
         pmAp[e] = f_inf();
@@ -659,11 +845,28 @@ __device__ unsigned build_table(const DevParams& P, const ClusterDev& C, int w, 
     auto s_SM = scan_set(SMx, OpMax<long long>(), LL_NONE);
     scan_prefix_fused(s_pmA, s_pmAp, s_PM);
     scan_suffix_excl_fused(s_smS, s_smSp, s_SM);
+    if constexpr (NW > 1) {
+        if (lane == 0) {
+            sm.pf[1][q] = s_pmA.total;
+            sm.pf[2][q] = s_pmAp.total;
+            sm.pll[0][q] = s_PM.total;  // the request sums were consumed above
+            sm.pf[3][q] = s_smS.total;
+            sm.pf[4][q] = s_smSp.total;
+            sm.pll[1][q] = s_SM.total;
+        }
+        group_sync<NW>();
+        add_carry_prefix<NW>(s_pmA, sm.pf[1], q);
+        add_carry_prefix<NW>(s_pmAp, sm.pf[2], q);
+        add_carry_prefix<NW>(s_PM, sm.pll[0], q);
+        add_carry_suffix<NW>(s_smS, sm.pf[3], q);
+        add_carry_suffix<NW>(s_smSp, sm.pf[4], q);
+        add_carry_suffix<NW>(s_SM, sm.pll[1], q);
+    }
     const float smS0 = s_smS.total;
     const float smSp0 = s_smSp.total;
     const long long SM0 = s_SM.total;
 
-    // Worker record (every lane; lane 0 stores it).
+    // Worker record (every lane; the first lane stores it).
     float4 wr;
     wr.x = inv_s;
     wr.y = off * inv_s * P.inv_k1 + P.c1_over_k1 + (float)sumP;
@@ -679,7 +882,7 @@ __device__ unsigned build_table(const DevParams& P, const ClusterDev& C, int w, 
 #pragma unroll
         for (int e = 0; e < E; ++e) {
             if (last[e]) {
-                const int x = e * 32 + lane;
+                const int x = x0 + e * 32 + lane;
                 const int np = n - (x + 1);
                 const long long A = tot_a - pre_a[e];
                 const int nxt = (x == n - 1) ? 0x7fffffff : rnext[e];
@@ -696,7 +899,7 @@ __device__ unsigned build_table(const DevParams& P, const ClusterDev& C, int w, 
             }
         }
     }
-    if (lane == 0) {
+    if (q == 0 && lane == 0) {
         RowVals o;
         if (!bad) {
             o = make_row(P, inv_s, M, sumP, 0, n > 0 ? r0 : 0x7fffffff, n, tot_a, 0, 0, LL_NONE,
@@ -716,13 +919,6 @@ __device__ unsigned build_table(const DevParams& P, const ClusterDev& C, int w, 
             mine = true;
         }
         C.wrec[w] = wr;
-        const double B = (double)n;
-        const double L = __dadd_rn((double)sumIn, __dmul_rn(P.gammad, (double)sumPred));
-        // capacity_norm^2 is exact here (integer and half-integer terms below
-        // 2^53); non-negative doubles order like their bit patterns, and code 0
-        // is kept for a worker holding an invalid request.
-        const double q = __dadd_rn(__dmul_rn(B, B), __dmul_rn(L, L));
-        const unsigned long long kq = bad ? 0ull : (unsigned long long)__double_as_longlong(q) + 1ull;
         C.key[w] = kq;
         if (cache) {
             if (!bad && n > 0 && R > 0) cache->rho[0] = (unsigned short)r0;
@@ -731,10 +927,16 @@ __device__ unsigned build_table(const DevParams& P, const ClusterDev& C, int w, 
             *cache->key = kq;
         }
     }
-    __syncwarp();
-    if (!want) return 0u;
-    const unsigned who = __ballot_sync(FULL, mine);
-    return __shfl_sync(FULL, cf, who ? __ffs(who) - 1 : 0);
+    if constexpr (NW > 1) {
+        if (mine) sm.cflag = cf;  // exactly one lane of the group holds the row
+        group_sync<NW>();
+        return want ? sm.cflag : 0u;
+    } else {
+        __syncwarp();
+        if (!want) return 0u;
+        const unsigned who = __ballot_sync(FULL, mine);
+        return __shfl_sync(FULL, cf, who ? __ffs(who) - 1 : 0);
+    }
 }
 
 }  // namespace aladdin

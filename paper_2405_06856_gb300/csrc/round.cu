@@ -163,14 +163,16 @@ __global__ void __launch_bounds__(ROUND_THREADS) k_round(DevParams P, ClusterDev
 // bests itself; with several CTAs the CTA bests are exchanged through global
 // memory behind one grid barrier (an arrival counter polled with a bounded
 // wait) and a second CTA barrier.
-constexpr int R2_MAX_WARPS = 16;
-// 512 threads (128 registers each) for up to 128 slots per worker; 256
-// threads (255 registers) for larger tables, whose rebuild needs them.
+// The winner's table is rebuilt by NW cooperating warps (EW element rows per
+// lane, E = EW NW), chosen so that the rebuild's latency stays low and its
+// registers within the 128 a thread of a 512-thread CTA has.
+constexpr int R2_THREADS = 512;
+constexpr int R2_WARPS = R2_THREADS / 32;
 template <int E>
-__host__ __device__ constexpr int r2_threads()
-{
-    return E >= 8 ? 256 : 512;
-}
+struct R2Split {
+    static constexpr int NW = E <= 4 ? E : 8;
+    static constexpr int EW = E / NW;
+};
 constexpr long long GRID_WAIT_LIMIT = 1ll << 22;  // polls of the arrival counter (seconds)
 constexpr int NONE = 0x7fffffff;
 
@@ -187,10 +189,10 @@ struct R2Args {
 
 template <int E>
 struct R2Smem {
-    BuildSmem<E> build;
-    unsigned long long bk[2][R2_MAX_WARPS];
-    int bw[2][R2_MAX_WARPS];
-    int bf[2][R2_MAX_WARPS];
+    BuildSmem<R2Split<E>::EW, R2Split<E>::NW> build;
+    unsigned long long bk[2][R2_WARPS];
+    int bw[2][R2_WARPS];
+    int bf[2][R2_WARPS];
     int gwin[2];
     int stop;
 };
@@ -224,23 +226,34 @@ __device__ __forceinline__ void better_f(unsigned long long& bk, int& bw, int& b
     }
 }
 
-__device__ __forceinline__ void reduce_f(unsigned long long& bk, int& bw, int& bf, int width)
+// Warp-wide best_f: the largest key, then the lowest worker index among equal
+// keys (warp max/min reductions on the key's halves); every lane ends with it.
+__device__ __forceinline__ void reduce_f(unsigned long long& bk, int& bw, int& bf)
 {
-#pragma unroll
-    for (int d = 16; d > 0; d >>= 1) {
-        if (d >= width) continue;
-        const unsigned long long ok = __shfl_xor_sync(FULL, bk, d);
-        const int ow = __shfl_xor_sync(FULL, bw, d);
-        const int of = __shfl_xor_sync(FULL, bf, d);
-        better_f(bk, bw, bf, ok, ow, of);
+    const bool has = bw != NONE;
+    const unsigned hi = has ? (unsigned)(bk >> 32) : 0u;
+    const unsigned lo = has ? (unsigned)bk : 0u;
+    const unsigned mhi = __reduce_max_sync(FULL, hi);
+    const unsigned mlo = __reduce_max_sync(FULL, hi == mhi ? lo : 0u);
+    const bool top = has && hi == mhi && lo == mlo;
+    const unsigned widx = __reduce_min_sync(FULL, top ? (unsigned)bw : 0xffffffffu);
+    const unsigned who = __ballot_sync(FULL, top && (unsigned)bw == widx);
+    const int of = __shfl_sync(FULL, bf, who ? __ffs(who) - 1 : 0);
+    if (who) {
+        bk = ((unsigned long long)mhi << 32) | mlo;
+        bw = (int)widx;
+        bf = of;
+    } else {
+        bk = 0ull;
+        bw = NONE;
+        bf = 0;
     }
 }
 
 template <int E>
-__global__ void __launch_bounds__(r2_threads<E>(), 1) k_round2(R2Args A)
+__global__ void __launch_bounds__(R2_THREADS, 1) k_round2(R2Args A)
 {
-    constexpr int R2_THREADS = r2_threads<E>();
-    constexpr int R2_WARPS = R2_THREADS / 32;
+    constexpr int NW = R2Split<E>::NW, EW = R2Split<E>::EW;
     extern __shared__ __align__(16) unsigned char smraw[];
     R2Smem<E>& sm = *reinterpret_cast<R2Smem<E>*>(smraw);
     const int cap = A.C.cap;
@@ -284,8 +297,8 @@ __global__ void __launch_bounds__(r2_threads<E>(), 1) k_round2(R2Args A)
     int32_t pa = 0, pr = 0;
     double pwd = 0.0;    // its request
 
-    auto append = [&](int w) {  // warp 0: commit the owed request to w
-        if (lane == 0) {
+    auto append = [&](int w) {  // rebuild group: commit the owed request to w
+        if (tid == 0) {
             const int lw = w - w_lo;
             const int nw = n_s[lw];
             const long long slot = (long long)w * C.cap + nw;
@@ -298,7 +311,7 @@ __global__ void __launch_bounds__(r2_threads<E>(), 1) k_round2(R2Args A)
             C.n[w] = nw + 1;
             n_s[lw] = nw + 1;
         }
-        __syncwarp();
+        group_sync<NW>();
     };
 
     for (int c = 0; c < n_cand; ++c) {
@@ -320,15 +333,16 @@ __global__ void __launch_bounds__(r2_threads<E>(), 1) k_round2(R2Args A)
         unsigned long long bk = 0ull;
         int bw = NONE, bf = 0;
         const bool rebuilding = pend_w >= 0;
-        if (rebuilding && warp == 0) {
+        if (rebuilding && warp < NW) {
             append(pend_w);
             const int lw = pend_w - w_lo;
             SliceCache sc{rho + (long long)lw * cap, &R_s[lw], &wrec_s[lw], &key_s[lw]};
-            const unsigned f = build_table<E>(P, C, pend_w, sm.build, &sc, cr.valid ? &cr : nullptr);
-            if (lane == 0 && cr.valid && f == 15u) bk = key_s[lw], bw = pend_w, bf = n_s[lw] >= cap;
+            const unsigned f =
+                build_table<EW, NW>(P, C, pend_w, sm.build, &sc, cr.valid ? &cr : nullptr);
+            if (tid == 0 && cr.valid && f == 15u) bk = key_s[lw], bw = pend_w, bf = n_s[lw] >= cap;
         } else if (cr.valid) {
-            const int first = rebuilding ? tid - 32 : tid;
-            const int stride = rebuilding ? R2_THREADS - 32 : R2_THREADS;
+            const int first = rebuilding ? tid - 32 * NW : tid;
+            const int stride = rebuilding ? R2_THREADS - 32 * NW : R2_THREADS;
             for (int lw = first; lw < nloc; lw += stride) {
                 const int w = w_lo + lw;
                 if (w == pend_w) continue;
@@ -340,7 +354,7 @@ __global__ void __launch_bounds__(r2_threads<E>(), 1) k_round2(R2Args A)
                 if (f == 15u) better_f(bk, bw, bf, key_s[lw], w, n_s[lw] >= cap);
             }
         }
-        reduce_f(bk, bw, bf, 32);
+        reduce_f(bk, bw, bf);
         if (lane == 0) {
             sm.bk[par][warp] = bk;
             sm.bw[par][warp] = bw;
@@ -351,7 +365,7 @@ __global__ void __launch_bounds__(r2_threads<E>(), 1) k_round2(R2Args A)
         bk = lane < R2_WARPS ? sm.bk[par][lane] : 0ull;
         bw = lane < R2_WARPS ? sm.bw[par][lane] : NONE;
         bf = lane < R2_WARPS ? sm.bf[par][lane] : 0;
-        reduce_f(bk, bw, bf, 32);  // every lane ends with the CTA best
+        reduce_f(bk, bw, bf);  // every lane ends with the CTA best
         if (A.G > 1) {
             if (warp == 0) {
                 if (lane == 0) {
@@ -385,7 +399,7 @@ __global__ void __launch_bounds__(r2_threads<E>(), 1) k_round2(R2Args A)
                     better_f(bk, bw, bf, __ldcg(&A.xkey[par * A.G + q]), wq,
                              iq != NONE && (iq & 0x40000000));
                 }
-                reduce_f(bk, bw, bf, 32);
+                reduce_f(bk, bw, bf);
                 if (lane == 0) sm.gwin[par] = bw == NONE ? NONE : (bw | (bf ? 0x40000000 : 0));
             }
             __syncthreads();
@@ -420,11 +434,11 @@ __global__ void __launch_bounds__(r2_threads<E>(), 1) k_round2(R2Args A)
             }
         }
     }
-    if (pend_w >= 0 && warp == 0) {
+    if (pend_w >= 0 && warp < NW) {
         append(pend_w);
         const int lw = pend_w - w_lo;
         SliceCache sc{rho + (long long)lw * cap, &R_s[lw], &wrec_s[lw], &key_s[lw]};
-        build_table<E>(P, C, pend_w, sm.build, &sc, nullptr);
+        build_table<EW, NW>(P, C, pend_w, sm.build, &sc, nullptr);
     }
     if (g == 0 && tid == 0 && io.sim && !sm.stop && *io.status == 0) {
         *io.n_wait = keep;
@@ -483,10 +497,10 @@ static cudaError_t round2_e(const DevParams& P, const ClusterDev& C, const Round
         e = cudaMemsetAsync(A.arrive, 0, sizeof(unsigned int), st);
         if (e != cudaSuccess) return e;
         void* args[] = {&A};
-        e = cudaLaunchCooperativeKernel((const void*)k_round2<E>, dim3(G), dim3(r2_threads<E>()), args,
+        e = cudaLaunchCooperativeKernel((const void*)k_round2<E>, dim3(G), dim3(R2_THREADS), args,
                                         smem, st);
     } else {
-        k_round2<E><<<1, r2_threads<E>(), smem, st>>>(A);
+        k_round2<E><<<1, R2_THREADS, smem, st>>>(A);
         e = cudaGetLastError();
     }
     if (e == cudaSuccess) *used = true;
