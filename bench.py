@@ -39,6 +39,9 @@ WORKLOAD_DESC = ("4,096 workers x 128 ongoing requests (KV capacity 131,072 toke
                  "clip [8, 4096], generated ~ U[0, output); decode 8 ms + 0.05 ms/request + 2e-4 "
                  "ms/KV token, prefill 10 ms + 0.1 ms/100 tokens, TTFT 1 s, ATGT 50 ms; seed 2")
 L2_FLUSH_BYTES = 256 << 20
+# minimum-worker search: KV tokens per GPU and per-worker request slots
+MW_KV_PER_GPU = 32768
+MW_B_CAP = 1024
 
 
 def algorithmic_bytes(W, B, C):
@@ -303,6 +306,7 @@ def run_ours(args):
             A.aladdin_place_round(c2.handle, w2.n_cand, t_in, t_pr, t_w, pl)
             rounds.append((time.perf_counter() - t0) * 1000.0)
     round_ms = min(rounds)
+    r16k = rounds_w16384(A, synth, stream)
 
     peak, peak_kind = read_peaks()
     kern_avg = kern_ms / max(kern_n, 1)
@@ -331,6 +335,7 @@ def run_ours(args):
                          "kernel_ms": kern_avg, "launches": kern_n},
             "round_latency_ms": {"workload": "256 workers x 64 requests, 2,048 candidates, one "
                                              "greedy round", "value": round_ms},
+            "rounds_w16384": r16k,
             "clocks": clocks}
     if cpu is not None:
         line["cpu_baseline"] = cpu
@@ -339,6 +344,71 @@ def run_ours(args):
     cl.close()
     if dist is not None:
         dist.destroy_process_group()
+
+
+def rounds_w16384(A, synth, stream, n_rounds=10, dt_ms=100.0):
+    """Ten consecutive greedy rounds on the 16,384-worker workload (1/2/4/8-GPU
+    workers, 256 requests each): the 131,072 candidates arrive over ten
+    heartbeats, each round placing its share, then every worker executes
+    100 ms. Round time is the synchronous aladdin_place_round call with host
+    arrays (upload, the round, the capacity_norm ranking and the download)."""
+    wl = synth.config("w16384")
+    bounds = np.linspace(0, wl.n_cand, n_rounds + 1).astype(int)
+    rounds, advances, placed = [], [], 0
+    with A.Cluster.from_workload(wl, stream=stream) as cl:
+        for k in range(n_rounds):
+            a, b = int(bounds[k]), int(bounds[k + 1])
+            t0 = time.perf_counter()
+            pl = cl.place_round(wl.cand_in[a:b], wl.cand_pred[a:b], wl.cand_wait[a:b])
+            rounds.append((time.perf_counter() - t0) * 1000.0)
+            placed += int((pl >= 0).sum())
+            t0 = time.perf_counter()
+            cl.advance(dt_ms)
+            advances.append((time.perf_counter() - t0) * 1000.0)
+        assert cl.status() == A.OK
+    return {"workload": "16,384 workers of 1/2/4/8 GPUs (KV 131,072 per GPU, latency x 1/sqrt(GPUs)), "
+                        "256 requests each; 131,072 candidates over 10 greedy rounds of 13,107, "
+                        "100 ms of execution between rounds; seed 3",
+            "rounds": n_rounds, "candidates_per_round": int(bounds[1] - bounds[0]),
+            "ms_per_round": statistics.mean(rounds), "ms_max_round": max(rounds),
+            "ms_per_advance": statistics.mean(advances),
+            "placed_fraction": placed / float(wl.n_cand)}
+
+
+def min_workers_config(synth):
+    """The minimum-worker search workload: a 1,000,000-request diurnal trace
+    (peak 2,000 req/s, peak:trough 4:1) and 1/2/4/8-GPU worker options."""
+    tr = synth.diurnal_trace(4, 1_000_000, 2000.0, 500.0)
+    gpus = [1, 2, 4, 8]
+    kv = [MW_KV_PER_GPU * g for g in gpus]
+    scale = [1.0 / math.sqrt(g) for g in gpus]
+    return tr, gpus, kv, scale
+
+
+def run_min_workers(args):
+    """Minimum-worker search (binary search over the worker count for each
+    worker option, every probe a fleet simulation on the device)."""
+    import torch
+    from paper_2405_06856_gb300 import build as B
+    B.build()
+    from paper_2405_06856_gb300 import aladdin as A
+    from paper_2405_06856_gb300 import synth
+    torch.cuda.set_device(0)
+    tr, gpus, kv, scale = min_workers_config(synth)
+    p = dict(synth.BASE_PARAMS)
+    got = np.zeros(len(gpus), np.int32)
+    stream = torch.cuda.current_stream().cuda_stream
+    torch.cuda.synchronize()
+    t0 = time.perf_counter()
+    best, total = A.aladdin_min_workers(A.make_params(p, MW_B_CAP), A.make_cfgs(gpus, kv, scale),
+                                        A.make_trace(tr.t_arr, tr.req_in, tr.req_pred), 100.0,
+                                        4096, got, stream=stream)
+    wall = time.perf_counter() - t0
+    print(json.dumps({"mode": "min_workers", "requests": len(tr.t_arr),
+                      "trace_span_s": float(tr.t_arr[-1] / 1000.0),
+                      "gpus_per_worker": gpus, "kv_per_worker": kv,
+                      "min_workers": got.tolist(), "best_gpus_per_worker": gpus[best],
+                      "total_gpus": int(total), "wall_s": wall}))
 
 
 def run_kernel_only(args):
@@ -424,7 +494,7 @@ def main():
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--no-cpu-baseline", dest="cpu_baseline", action="store_false")
-    ap.add_argument("--mode", default="full", choices=["full", "kernel", "round"],
+    ap.add_argument("--mode", default="full", choices=["full", "kernel", "round", "minworkers"],
                     help="kernel: only warm-up + steps of the device-resident step (for profilers)")
     args = ap.parse_args()
     if args.warmup < 3:
@@ -435,6 +505,8 @@ def main():
         run_kernel_only(args)
     elif args.mode == "round":
         run_round_only(args)
+    elif args.mode == "minworkers":
+        run_min_workers(args)
     else:
         run_ours(args)
 

@@ -60,7 +60,7 @@ extern "C" {
  *   KV usage          (Eq. kv cache):          kv = h * (l_in + l_out) + j
  * Requirements: k1, k2 > 0; c1, c2, c3 >= 0; h >= 1; j >= 0; T_pre > 0;
  * T_dec > c3 (Eq. input limit); 0 < theta <= 1; gamma >= 0; 2 <= K <= 65536;
- * b_cap a power of two in [32, 512]. */
+ * b_cap a power of two in [32, 1024]. */
 typedef struct aladdin_params {
     double k1, c1;       /* prefill: ms per input token, ms */
     double k2, c2, c3;   /* decode: ms per context token, ms per request, ms */

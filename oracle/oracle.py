@@ -206,6 +206,23 @@ class Cluster:
             raise RuntimeError("orc_place_round failed: %d" % rc)
         return pl
 
+    def commit(self, w, a, r, wait=0.0, rid=0):
+        """Append request (prompt a, predicted output r) to worker w as a
+        placement of the open round (Algorithm 1's commit step, in a pending
+        state: gen 0, no decode history)."""
+        w = int(w)
+        if self.n[w] >= self.cap:
+            raise OverflowError("worker request capacity exceeded")
+        slot = w * self.cap + int(self.n[w])
+        self.inp[slot] = a
+        self.gen[slot] = 0
+        self.pred[slot] = r
+        self.tdec[slot] = 0.0
+        self.pend[slot] = 1
+        self.wait[slot] = wait
+        self.rid[slot] = rid
+        self.n[w] += 1
+
     def advance(self, t_now, dt, rec_cap=1 << 16):
         rr = np.zeros(rec_cap, np.int64)
         rv = np.zeros(rec_cap)

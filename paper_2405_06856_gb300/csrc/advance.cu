@@ -165,6 +165,7 @@ cudaError_t launch_advance(const DevParams& P, const ClusterDev& C, double t_now
     case 4: return advance_e<4>(P, C, t_now, dt, stats, halt, st);
     case 8: return advance_e<8>(P, C, t_now, dt, stats, halt, st);
     case 16: return advance_e<16>(P, C, t_now, dt, stats, halt, st);
+    case 32: return advance_e<32>(P, C, t_now, dt, stats, halt, st);
     default: return cudaErrorInvalidValue;
     }
 }

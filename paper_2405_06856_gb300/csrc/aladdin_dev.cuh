@@ -96,6 +96,8 @@ struct ClusterDev {
     unsigned int* err;         // sticky error bits (1: invalid request)
     int32_t* ovf;              // [W] workers left to the full-capacity table build
     int* novf;                 // their count
+    uint32_t* skey;            // [W*cap] (r << 10 | slot) of the requests in sorted order,
+                               // written by every table build
 };
 
 // Table row p of a worker (2 x float4, 32 bytes) and its side entry:
@@ -474,7 +476,8 @@ __device__ __forceinline__ void store_row(const ClusterDev& C, long long rowid, 
 // Shared-memory copies of one worker's breakpoints, record and key, kept by
 // the sliced placement round (pointers to this worker's entries).
 struct SliceCache {
-    unsigned short* rho;  // rho_{q+1} of rows q = 0..R-1
+    unsigned short* rho;  // rho_{q+1} - 1 of rows q = 0..min(R, rc)-1
+    int rc;               // rows held
     int* R;
     float4* wrec;
     unsigned long long* key;
@@ -489,11 +492,12 @@ struct SliceCache {
 // copies are refreshed as well. With a valid `cand`, the candidate is
 // evaluated against the new table by the lane that holds its row, and every
 // lane returns its flags (else 0).
-template <int EW, int NW = 1>
+template <int EW, int NW = 1, bool INSERT = false>
 __device__ unsigned build_table(const DevParams& P, const ClusterDev& C, int w,
                                 BuildSmem<EW, NW>& sm, const SliceCache* cache = nullptr,
                                 const CandRec* cand = nullptr)
 {
+    static_assert(!INSERT || NW > 1, "the insertion path is for cooperative builds");
     constexpr int E = EW;
     constexpr int RUN = 32 * EW;  // elements per warp
     const int lane = threadIdx.x & 31;
@@ -501,9 +505,9 @@ __device__ unsigned build_table(const DevParams& P, const ClusterDev& C, int w,
     const int x0 = q * RUN;
     const long long base = (long long)w * C.cap;
     const long long rowbase = (long long)w * C.rows;
-    // Independent loads first: the slot loads do not wait for n (every slot
-    // below 32 E NW lies inside the worker's slot range; those past n are
-    // masked).
+    // Independent loads first: the slot loads do not wait for n (slots below
+    // the capacity lie inside the worker's slot range; those past n are
+    // masked). A build may cover more elements than the capacity (padding).
     const int n = C.n[w];
     const float s = C.scale[w];
     const int M = C.M[w];
@@ -513,16 +517,32 @@ __device__ unsigned build_table(const DevParams& P, const ClusterDev& C, int w,
     constexpr int EL = PRELOAD ? E : 1;
     int l_pd[EL], l_g[EL], l_pr[EL], l_in[EL];
     double l_td[EL], l_wt[EL];
+    unsigned l_sk[INSERT ? E : 1];
+    if constexpr (INSERT) {
+        // The previous build's sorted keys (all requests but the last, which
+        // was just appended).
+#pragma unroll
+        for (int e = 0; e < E; ++e) {
+            const int x = x0 + e * 32 + lane;
+            l_sk[e] = x < C.cap ? C.skey[base + x] : 0xffffffffu;
+        }
+    }
     if constexpr (PRELOAD) {
 #pragma unroll
         for (int e = 0; e < EL; ++e) {
-            const long long slot = base + x0 + e * 32 + lane;
-            l_pd[e] = C.pend[slot];
-            l_g[e] = C.gen[slot];
-            l_pr[e] = C.pred[slot];
-            l_in[e] = C.in[slot];
-            l_td[e] = C.tdec[slot];
-            l_wt[e] = C.wait[slot];
+            const int x = x0 + e * 32 + lane;
+            const long long slot = base + x;
+            l_pd[e] = 0;
+            l_g[e] = l_pr[e] = l_in[e] = 0;
+            l_td[e] = l_wt[e] = 0.0;
+            if (x < C.cap) {
+                l_pd[e] = C.pend[slot];
+                l_g[e] = C.gen[slot];
+                l_pr[e] = C.pred[slot];
+                l_in[e] = C.in[slot];
+                l_td[e] = C.tdec[slot];
+                l_wt[e] = C.wait[slot];
+            }
         }
     }
     const float inv_s = 1.0f / s;
@@ -546,7 +566,7 @@ __device__ unsigned build_table(const DevParams& P, const ClusterDev& C, int w,
             r = r < 1 ? 1 : (r > P.K ? P.K : r);
             int a = in + g;
             a = a < 0 ? 0 : (a > P.K ? P.K : a);
-            key[e] = ((unsigned)r << 9) | (unsigned)i;
+            key[e] = ((unsigned)r << 10) | (unsigned)i;
             sm.a[i] = a;
             sm.pend[i] = (uint8_t)pd;
             sm.bank[i] = pd ? 0.0f
@@ -612,16 +632,43 @@ __device__ unsigned build_table(const DevParams& P, const ClusterDev& C, int w,
     // capacity_norm key: capacity_norm^2 is exact here (integer and
     // half-integer terms below 2^53); non-negative doubles order like their
     // bit patterns, and code 0 is kept for a worker holding an invalid request.
-    const double kB = (double)n;
-    const double kL = __dadd_rn((double)sumIn, __dmul_rn(P.gammad, (double)sumPred));
-    const double kQ = __dadd_rn(__dmul_rn(kB, kB), __dmul_rn(kL, kL));
-    const unsigned long long kq = bad ? 0ull : (unsigned long long)__double_as_longlong(kQ) + 1ull;
+    unsigned long long kq = 0ull;
+    if (q == 0 && lane == 0) {  // fp64 is slow on this part: one lane
+        const double kB = (double)n;
+        const double kL = __dadd_rn((double)sumIn, __dmul_rn(P.gammad, (double)sumPred));
+        const double kQ = __dadd_rn(__dmul_rn(kB, kB), __dmul_rn(kL, kL));
+        kq = bad ? 0ull : (unsigned long long)__double_as_longlong(kQ) + 1ull;
+    }
 
     constexpr int N = BuildSmem<EW, NW>::N;
     // Cooperative builds of up to 256 slots rank every key by counting the
     // keys below it (keys of valid requests are distinct); larger ones sort
     // each warp's run and merge the runs.
-    constexpr bool COUNT_RANK = NW > 1 && N <= 256;
+    constexpr bool COUNT_RANK = NW > 1 && N <= 256 && !INSERT;
+    if constexpr (INSERT) {
+        // Insert the appended request's key into the previous sorted order.
+#pragma unroll
+        for (int e = 0; e < E; ++e) {
+            const int x = x0 + e * 32 + lane;
+            if (x < n - 1) sm.runs[x] = l_sk[e];
+            if (x == n - 1) sm.cflag = key[e];
+        }
+        group_sync<NW>();
+        const unsigned knew = sm.cflag;
+        int lo = 0, hi = n - 1;  // old keys below knew (keys are distinct)
+        while (lo < hi) {
+            const int mid = (lo + hi) >> 1;
+            if (sm.runs[mid] < knew) lo = mid + 1;
+            else hi = mid;
+        }
+#pragma unroll
+        for (int e = 0; e < E; ++e) {
+            const int x = x0 + e * 32 + lane;
+            key[e] = x < n ? (x < lo ? sm.runs[x] : (x == lo ? knew : sm.runs[x - 1])) : 0xffffffffu;
+            if (x < n) sm.sorted[x] = key[e];
+        }
+        group_sync<NW>();
+    }
     if constexpr (COUNT_RANK) {
 #pragma unroll
         for (int e = 0; e < E; ++e) sm.runs[x0 + e * 32 + lane] = key[e];
@@ -649,7 +696,7 @@ __device__ unsigned build_table(const DevParams& P, const ClusterDev& C, int w,
     }
     // Bitonic sort of (r, slot) keys, ascending, within each warp's run.
 #pragma unroll
-    for (int k = 2; k <= (COUNT_RANK ? 1 : RUN); k <<= 1) {
+    for (int k = 2; k <= (COUNT_RANK || INSERT ? 1 : RUN); k <<= 1) {
 #pragma unroll
         for (int jj = k >> 1; jj > 0; jj >>= 1) {
             if (jj >= 32) {
@@ -676,7 +723,7 @@ __device__ unsigned build_table(const DevParams& P, const ClusterDev& C, int w,
             }
         }
     }
-    if constexpr (NW > 1 && !COUNT_RANK) {
+    if constexpr (NW > 1 && !COUNT_RANK && !INSERT) {
         // Merge the NW sorted runs: a key's rank is its position in its run
         // plus the keys of the other runs before it (equal padding keys of
         // earlier runs first).
@@ -685,20 +732,26 @@ __device__ unsigned build_table(const DevParams& P, const ClusterDev& C, int w,
         group_sync<NW>();
 #pragma unroll
         for (int e = 0; e < E; ++e) {
+            // In every other run, the count of keys before this one: a
+            // fixed-step search, the NW searches advancing together.
+            int cnt[NW];
+#pragma unroll
+            for (int q2 = 0; q2 < NW; ++q2) cnt[q2] = 0;
+#pragma unroll
+            for (int st = RUN; st >= 1; st >>= 1) {
+#pragma unroll
+                for (int q2 = 0; q2 < NW; ++q2) {
+                    const int probe = cnt[q2] + st;
+                    if (probe <= RUN) {
+                        const unsigned v = sm.runs[q2 * RUN + probe - 1];
+                        if (q2 < q ? v <= key[e] : v < key[e]) cnt[q2] = probe;
+                    }
+                }
+            }
             int rank = e * 32 + lane;
 #pragma unroll
-            for (int q2 = 0; q2 < NW; ++q2) {
-                if (q2 == q) continue;
-                const unsigned* run = sm.runs + q2 * RUN;
-                int lo = 0, hi = RUN;
-                while (lo < hi) {
-                    const int mid = (lo + hi) >> 1;
-                    const unsigned v = run[mid];
-                    if (q2 < q ? v <= key[e] : v < key[e]) lo = mid + 1;
-                    else hi = mid;
-                }
-                rank += lo;
-            }
+            for (int q2 = 0; q2 < NW; ++q2)
+                if (q2 != q) rank += cnt[q2];
             sm.sorted[rank] = key[e];
         }
         group_sync<NW>();
@@ -712,8 +765,8 @@ __device__ unsigned build_table(const DevParams& P, const ClusterDev& C, int w,
     for (int e = 0; e < E; ++e) {
         const int x = x0 + e * 32 + lane;
         if (x < n) {
-            r[e] = (int)(key[e] >> 9);
-            const int i = (int)(key[e] & 511u);
+            r[e] = (int)(key[e] >> 10);
+            const int i = (int)(key[e] & 1023u);
             a[e] = sm.a[i];
             pd[e] = sm.pend[i];
             bank[e] = sm.bank[i];
@@ -724,6 +777,12 @@ __device__ unsigned build_table(const DevParams& P, const ClusterDev& C, int w,
             bank[e] = 0.0f;
         }
     }
+    // The sorted order, kept for the next build's insertion.
+#pragma unroll
+    for (int e = 0; e < E; ++e) {
+        const int x = x0 + e * 32 + lane;
+        if (x < n) C.skey[base + x] = key[e];
+    }
     // Neighbours in sorted order.
     int rnext[E], first[E], last[E];
 #pragma unroll
@@ -731,8 +790,8 @@ __device__ unsigned build_table(const DevParams& P, const ClusterDev& C, int w,
         const int x = x0 + e * 32 + lane;
         int nx, pv;
         if constexpr (NW > 1) {
-            nx = x + 1 < n ? (int)(sm.sorted[x + 1] >> 9) : -1;
-            pv = x > 0 && x - 1 < n ? (int)(sm.sorted[x - 1] >> 9) : -1;
+            nx = x + 1 < n ? (int)(sm.sorted[x + 1] >> 10) : -1;
+            pv = x > 0 && x - 1 < n ? (int)(sm.sorted[x - 1] >> 10) : -1;
         } else {
             const int dn = __shfl_down_sync(FULL, r[e], 1);
             const int up = __shfl_up_sync(FULL, r[e], 1);
@@ -748,7 +807,7 @@ __device__ unsigned build_table(const DevParams& P, const ClusterDev& C, int w,
         last[e] = valid && (x == n - 1 || nx != r[e]);
     }
     int r0;
-    if constexpr (NW > 1) r0 = n > 0 ? (int)(sm.sorted[0] >> 9) : 0x7fffffff;
+    if constexpr (NW > 1) r0 = n > 0 ? (int)(sm.sorted[0] >> 10) : 0x7fffffff;
     else r0 = __shfl_sync(FULL, r[0], 0);
     // Prefix sums over the sorted order.
     int rowid[E];
@@ -890,7 +949,8 @@ __device__ unsigned build_table(const DevParams& P, const ClusterDev& C, int w,
                 const RowVals o = make_row(P, inv_s, M, sumP, r[e], nxt, np, A, pre_r[e], pre_ra[e],
                                            PMx[e], SM, pmA[e], pmAp[e], smS[e], smSp[e]);
                 store_row(C, rowbase + rowid[e], o);
-                if (cache && rowid[e] < R) cache->rho[rowid[e]] = (unsigned short)nxt;
+                if (cache && rowid[e] < R && rowid[e] < cache->rc)
+                    cache->rho[rowid[e]] = (unsigned short)(nxt - 1);
                 if (want && r[e] <= rc && rc < nxt) {
                     float m;
                     cf = eval_pair(o.v0, o.v1, o.ext, wr, *cand, m);
@@ -921,7 +981,7 @@ __device__ unsigned build_table(const DevParams& P, const ClusterDev& C, int w,
         C.wrec[w] = wr;
         C.key[w] = kq;
         if (cache) {
-            if (!bad && n > 0 && R > 0) cache->rho[0] = (unsigned short)r0;
+            if (!bad && n > 0 && R > 0) cache->rho[0] = (unsigned short)(r0 - 1);
             *cache->R = bad ? 0 : R;
             *cache->wrec = wr;
             *cache->key = kq;
@@ -937,6 +997,31 @@ __device__ unsigned build_table(const DevParams& P, const ClusterDev& C, int w,
         const unsigned who = __ballot_sync(FULL, mine);
         return __shfl_sync(FULL, cf, who ? __ffs(who) - 1 : 0);
     }
+}
+
+// build_table with the fewest elements per lane that cover the worker's n
+// requests (a table of 1,024 slots holding 300 requests sorts and scans 512
+// elements, not 1,024). smem holds a BuildSmem<EWMAX, NW>; the smaller
+// variants use a prefix of it. n is the worker's current count (uniform over
+// the NW warps).
+template <int EWMAX, int NW, bool INSERT = false>
+__device__ __forceinline__ unsigned build_table_fit(const DevParams& P, const ClusterDev& C, int w,
+                                                    int n, unsigned char* smem,
+                                                    const SliceCache* cache = nullptr,
+                                                    const CandRec* cand = nullptr)
+{
+    if constexpr (EWMAX >= 4) {
+        if (n > 64 * NW)  // more than the EW = 2 variant covers
+            return build_table<4, NW, INSERT>(P, C, w, *reinterpret_cast<BuildSmem<4, NW>*>(smem),
+                                              cache, cand);
+    }
+    if constexpr (EWMAX >= 2) {
+        if (n > 32 * NW)
+            return build_table<2, NW, INSERT>(P, C, w, *reinterpret_cast<BuildSmem<2, NW>*>(smem),
+                                              cache, cand);
+    }
+    return build_table<1, NW, INSERT>(P, C, w, *reinterpret_cast<BuildSmem<1, NW>*>(smem), cache,
+                                      cand);
 }
 
 }  // namespace aladdin

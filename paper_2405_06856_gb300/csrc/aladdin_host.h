@@ -56,7 +56,7 @@ struct RoundIO {
     void* xbuf;
 };
 constexpr int ROUND_XBUF_SMS = 1024;  // largest SM count the exchange buffer serves
-constexpr size_t ROUND_XBUF_BYTES = 24 * (size_t)ROUND_XBUF_SMS + 16;
+constexpr size_t ROUND_XBUF_BYTES = 32 * (size_t)ROUND_XBUF_SMS + 16;
 cudaError_t launch_round(const DevParams& P, const ClusterDev& C, const RoundIO& io,
                          cudaStream_t st);
 

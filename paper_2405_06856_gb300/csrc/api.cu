@@ -66,7 +66,7 @@ int check_params(const aladdin_params* p)
     if (!finite_nonneg(p->gamma)) return ALADDIN_ERR_ARG;
     if (p->K < 2 || p->K > 65536) return ALADDIN_ERR_ARG;
     const int b = p->b_cap;
-    if (!(b == 32 || b == 64 || b == 128 || b == 256 || b == 512)) return ALADDIN_ERR_ARG;
+    if (!(b == 32 || b == 64 || b == 128 || b == 256 || b == 512 || b == 1024)) return ALADDIN_ERR_ARG;
     return ALADDIN_OK;
 }
 
@@ -230,6 +230,7 @@ int cluster_alloc(aladdin_cluster* cl, const aladdin_params& p, int W,
     AL(err, unsigned int, 1);
     AL(ovf, int32_t, W);
     AL(novf, int, 1);
+    AL(skey, uint32_t, slots);
 #undef AL
     CK(cl->alloc(&p0, sizeof(unsigned long long) * 4)); cl->d_stats = (unsigned long long*)p0;
     CK(cl->alloc(&p0, sizeof(int) * 4)); cl->d_status = (int*)p0;

@@ -170,8 +170,11 @@ constexpr int R2_THREADS = 512;
 constexpr int R2_WARPS = R2_THREADS / 32;
 template <int E>
 struct R2Split {
-    static constexpr int NW = E <= 4 ? E : 8;
-    static constexpr int EW = E / NW;
+    // up to 256 slots: NW warps cover the capacity with one element a lane;
+    // larger tables: 12 warps (4 left for evaluation) with up to E/8
+    // elements a lane, the build sized to the worker's count
+    static constexpr int NW = E <= 8 ? E : 12;
+    static constexpr int EW = E <= 8 ? 1 : E / 8;
 };
 constexpr long long GRID_WAIT_LIMIT = 1ll << 22;  // polls of the arrival counter (seconds)
 constexpr int NONE = 0x7fffffff;
@@ -182,8 +185,9 @@ struct R2Args {
     RoundIO io;
     int G;                          // CTAs
     int slice;                      // workers per CTA
-    unsigned long long* xkey;       // [2 * G] best key per CTA (two parities)
-    int* xidx;                      // [2 * G] its worker (NONE: none; bit 30: full)
+    int rc;                         // breakpoint rows per worker held in shared memory
+    ulonglong2* xrec;               // [2][G] per CTA (two parities): best key, its
+                                    // worker (NONE: none; bit 30: full)
     unsigned int* arrive;           // grid arrival counter, zero at launch
 };
 
@@ -197,6 +201,11 @@ struct R2Smem {
     int stop;
 };
 
+__device__ __forceinline__ void red_release_add(unsigned* p, unsigned v)
+{
+    asm volatile("red.release.gpu.global.add.u32 [%0], %1;" ::"l"(p), "r"(v) : "memory");
+}
+
 __device__ __forceinline__ unsigned ld_acquire(const unsigned* p)
 {
     unsigned v;
@@ -204,13 +213,26 @@ __device__ __forceinline__ unsigned ld_acquire(const unsigned* p)
     return v;
 }
 
-__device__ __forceinline__ int r2_find(const unsigned short* rho, int R, int r)
+// Row of remaining length r: the first row q whose rho_{q+1} exceeds r (row R
+// is unbounded). Shared memory holds rho_{q+1} - 1 for the first rc rows; a
+// worker with more rows continues in the table's global rows.
+__device__ __forceinline__ int r2_find(const unsigned short* rho, int R, int rc, int r,
+                                       const float4* tab, long long rowbase)
 {
-    int lo = 0, hi = R;  // first row whose rho_{p+1} exceeds r; row R is unbounded
+    const int Rs = R < rc ? R : rc;
+    int lo = 0, hi = Rs;
     while (lo < hi) {
         const int mid = (lo + hi) >> 1;
-        if ((int)rho[mid] > r) hi = mid;
+        if ((int)rho[mid] >= r) hi = mid;
         else lo = mid + 1;
+    }
+    if (lo == Rs && R > Rs) {
+        hi = R;
+        while (lo < hi) {
+            const int mid = (lo + hi) >> 1;
+            if (__float_as_int(tab[(rowbase + mid) * ROW_F4].x) > r) hi = mid;
+            else lo = mid + 1;
+        }
     }
     return lo;
 }
@@ -254,6 +276,8 @@ template <int E>
 __global__ void __launch_bounds__(R2_THREADS, 1) k_round2(R2Args A)
 {
     constexpr int NW = R2Split<E>::NW, EW = R2Split<E>::EW;
+    // the winner's previous sorted order is current: insert its new key
+    constexpr bool NW_INSERT = NW > 1;
     extern __shared__ __align__(16) unsigned char smraw[];
     R2Smem<E>& sm = *reinterpret_cast<R2Smem<E>*>(smraw);
     const int cap = A.C.cap;
@@ -281,10 +305,12 @@ __global__ void __launch_bounds__(R2_THREADS, 1) k_round2(R2Args A)
         key_s[lw] = C.key[w];
     }
     __syncthreads();
-    for (int k = tid; k < nloc * cap; k += R2_THREADS) {
-        const int lw = k / cap, q = k - lw * cap;
+    const int rc = A.rc;
+    for (int k = tid; k < nloc * rc; k += R2_THREADS) {
+        const int lw = k / rc, q = k - lw * rc;
         if (q < R_s[lw])
-            rho[k] = (unsigned short)__float_as_int(C.tab[((long long)(w_lo + lw) * C.rows + q) * ROW_F4].x);
+            rho[k] = (unsigned short)(
+                __float_as_int(C.tab[((long long)(w_lo + lw) * C.rows + q) * ROW_F4].x) - 1);
     }
     if (tid == 0) sm.stop = (io.sim && *io.status != 0) ? 1 : 0;
     __syncthreads();
@@ -336,9 +362,10 @@ __global__ void __launch_bounds__(R2_THREADS, 1) k_round2(R2Args A)
         if (rebuilding && warp < NW) {
             append(pend_w);
             const int lw = pend_w - w_lo;
-            SliceCache sc{rho + (long long)lw * cap, &R_s[lw], &wrec_s[lw], &key_s[lw]};
-            const unsigned f =
-                build_table<EW, NW>(P, C, pend_w, sm.build, &sc, cr.valid ? &cr : nullptr);
+            SliceCache sc{rho + (long long)lw * rc, rc, &R_s[lw], &wrec_s[lw], &key_s[lw]};
+            const unsigned f = build_table_fit<EW, NW, NW_INSERT>(P, C, pend_w, n_s[lw],
+                                                       reinterpret_cast<unsigned char*>(&sm.build),
+                                                       &sc, cr.valid ? &cr : nullptr);
             if (tid == 0 && cr.valid && f == 15u) bk = key_s[lw], bw = pend_w, bf = n_s[lw] >= cap;
         } else if (cr.valid) {
             const int first = rebuilding ? tid - 32 * NW : tid;
@@ -346,8 +373,9 @@ __global__ void __launch_bounds__(R2_THREADS, 1) k_round2(R2Args A)
             for (int lw = first; lw < nloc; lw += stride) {
                 const int w = w_lo + lw;
                 if (w == pend_w) continue;
-                const int p = r2_find(rho + (long long)lw * cap, R_s[lw], cr.ri);
-                const long long row = (long long)w * C.rows + p;
+                const long long rb = (long long)w * C.rows;
+                const int p = r2_find(rho + (long long)lw * rc, R_s[lw], rc, cr.ri, C.tab, rb);
+                const long long row = rb + p;
                 const float4* t = C.tab + row * ROW_F4;
                 float m;
                 const unsigned f = eval_pair(t[0], t[1], C.tab2[row], wrec_s[lw], cr, m);
@@ -369,34 +397,46 @@ __global__ void __launch_bounds__(R2_THREADS, 1) k_round2(R2Args A)
         if (A.G > 1) {
             if (warp == 0) {
                 if (lane == 0) {
-                    A.xkey[par * A.G + g] = bk;
-                    A.xidx[par * A.G + g] = bw == NONE ? NONE : (bw | (bf ? 0x40000000 : 0));
-                    __threadfence();
-                    atomicAdd(A.arrive, 1u);
-                    const unsigned target = (unsigned)(c + 1) * (unsigned)A.G;
-                    bool ok = false;
-                    for (long long it = 0; it < GRID_WAIT_LIMIT; ++it) {
-                        if (ld_acquire(A.arrive) >= target) {
-                            ok = true;
-                            break;
-                        }
-                        __nanosleep(32);
-                    }
-                    __threadfence();
-                    if (!ok) {
-                        atomicOr(C.err, 4u);
-                        *io.status = -4;  // ALADDIN_ERR_TIMEOUT
-                        sm.stop = 2;
-                    }
+                    const int xi = bw == NONE ? NONE : (bw | (bf ? 0x40000000 : 0));
+                    A.xrec[par * A.G + g] = make_ulonglong2(bk, (unsigned long long)(unsigned)xi);
+                    red_release_add(A.arrive, 1u);  // orders the store before it
                 }
-                __syncwarp();
+                // every lane acquires the counter, so its loads below see the
+                // other CTAs' entries
+                const unsigned target = (unsigned)(c + 1) * (unsigned)A.G;
+                bool ok = false;
+                for (long long it = 0; it < GRID_WAIT_LIMIT; ++it) {
+                    if (ld_acquire(A.arrive) >= target) {
+                        ok = true;
+                        break;
+                    }
+                    __nanosleep(32);
+                }
+                if (!ok && lane == 0) {
+                    atomicOr(C.err, 4u);
+                    *io.status = -4;  // ALADDIN_ERR_TIMEOUT
+                    sm.stop = 2;
+                }
                 bk = 0ull;
                 bw = NONE;
                 bf = 0;
-                for (int q = lane; q < A.G; q += 32) {
-                    const int iq = __ldcg(&A.xidx[par * A.G + q]);
-                    const int wq = iq == NONE ? NONE : (iq & 0x3fffffff);
-                    better_f(bk, bw, bf, __ldcg(&A.xkey[par * A.G + q]), wq,
+                // up to 8 entries a lane loaded together, then any beyond 256 CTAs
+                ulonglong2 xv[8];
+#pragma unroll
+                for (int k = 0; k < 8; ++k) {
+                    const int q = lane + 32 * k;
+                    xv[k] = q < A.G ? __ldcg(&A.xrec[par * A.G + q]) : make_ulonglong2(0ull, NONE);
+                }
+                for (int q = lane + 256; q < A.G; q += 32) {
+                    const ulonglong2 v = __ldcg(&A.xrec[par * A.G + q]);
+                    const int iq = (int)v.y;
+                    better_f(bk, bw, bf, v.x, iq == NONE ? NONE : (iq & 0x3fffffff),
+                             iq != NONE && (iq & 0x40000000));
+                }
+#pragma unroll
+                for (int k = 0; k < 8; ++k) {
+                    const int iq = (int)xv[k].y;
+                    better_f(bk, bw, bf, xv[k].x, iq == NONE ? NONE : (iq & 0x3fffffff),
                              iq != NONE && (iq & 0x40000000));
                 }
                 reduce_f(bk, bw, bf);
@@ -437,8 +477,10 @@ __global__ void __launch_bounds__(R2_THREADS, 1) k_round2(R2Args A)
     if (pend_w >= 0 && warp < NW) {
         append(pend_w);
         const int lw = pend_w - w_lo;
-        SliceCache sc{rho + (long long)lw * cap, &R_s[lw], &wrec_s[lw], &key_s[lw]};
-        build_table<EW, NW>(P, C, pend_w, sm.build, &sc, nullptr);
+        SliceCache sc{rho + (long long)lw * rc, rc, &R_s[lw], &wrec_s[lw], &key_s[lw]};
+        build_table_fit<EW, NW, NW_INSERT>(P, C, pend_w, n_s[lw],
+                                           reinterpret_cast<unsigned char*>(&sm.build),
+                                &sc, nullptr);
     }
     if (g == 0 && tid == 0 && io.sim && !sm.stop && *io.status == 0) {
         *io.n_wait = keep;
@@ -449,20 +491,21 @@ __global__ void __launch_bounds__(R2_THREADS, 1) k_round2(R2Args A)
     }
 }
 
-// Shared memory of k_round2 for a slice of `slice` workers.
+// Shared memory of k_round2 for a slice of `slice` workers holding rc rows.
 template <int E>
-static size_t r2_smem(int slice, int cap)
+static size_t r2_smem(int slice, int rc)
 {
     return ((sizeof(R2Smem<E>) + 15) / 16) * 16 + (size_t)slice * (16 + 8 + 4 + 4) +
-           (size_t)slice * cap * 2;
+           (size_t)slice * rc * 2;
 }
+constexpr int R2_MIN_RC = 64;  // fewer rows per worker in shared memory: use the plain round
 
 template <int E>
 static cudaError_t round2_e(const DevParams& P, const ClusterDev& C, const RoundIO& io,
                             cudaStream_t st, bool* used)
 {
     *used = false;
-    if (P.K > 65535) return cudaSuccess;  // 16-bit breakpoints
+    if (P.K > 65536) return cudaSuccess;  // breakpoints held as 16-bit rho - 1
     int dev = 0, sms = 0, smem_max = 0, coop = 0;
     cudaError_t e;
     if ((e = cudaGetDevice(&dev)) != cudaSuccess) return e;
@@ -473,14 +516,22 @@ static cudaError_t round2_e(const DevParams& P, const ClusterDev& C, const Round
         return e;
     if (sms > ROUND_XBUF_SMS) return cudaSuccess;
     const size_t budget = (size_t)smem_max - 1024;
-    const size_t per_w = 32 + (size_t)C.cap * 2;
-    const size_t base = r2_smem<E>(0, C.cap);
-    if (budget <= base + per_w) return cudaSuccess;
-    const int slice_max = (int)((budget - base) / per_w);
-    int G = (C.W + slice_max - 1) / slice_max;
-    if (G > sms || (G > 1 && !coop)) return cudaSuccess;  // use the single-CTA round
+    const size_t base = r2_smem<E>(0, 0);
+    if (budget <= base + 32 + 2 * R2_MIN_RC) return cudaSuccess;
+    // As few CTAs as hold every worker's rows; beyond one CTA per SM, the
+    // slices hold only the first rc rows of each worker.
+    int rc = C.cap;
+    const long long slice_max = (long long)((budget - base) / (32 + 2 * (size_t)rc));
+    int G = (int)((C.W + slice_max - 1) / slice_max);
+    if (G > sms) {
+        G = sms;
+        const long long sl = (C.W + G - 1) / G;
+        rc = (int)((((budget - base) / (size_t)sl) - 32) / 2) & ~7;
+        if (rc < R2_MIN_RC) return cudaSuccess;
+    }
+    if (G > 1 && !coop) return cudaSuccess;  // use the single-CTA round
     const int slice = (C.W + G - 1) / G;
-    const size_t smem = r2_smem<E>(slice, C.cap);
+    const size_t smem = r2_smem<E>(slice, rc);
     e = cudaFuncSetAttribute(k_round2<E>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          (int)smem);
     if (e != cudaSuccess) return e;
@@ -490,9 +541,9 @@ static cudaError_t round2_e(const DevParams& P, const ClusterDev& C, const Round
     A.io = io;
     A.G = G;
     A.slice = slice;
-    A.xkey = reinterpret_cast<unsigned long long*>(io.xbuf);
-    A.xidx = reinterpret_cast<int*>(A.xkey + 2 * ROUND_XBUF_SMS);
-    A.arrive = reinterpret_cast<unsigned int*>(A.xidx + 2 * ROUND_XBUF_SMS);
+    A.rc = rc;
+    A.xrec = reinterpret_cast<ulonglong2*>(io.xbuf);
+    A.arrive = reinterpret_cast<unsigned int*>(A.xrec + 2 * ROUND_XBUF_SMS);
     if (G > 1) {
         e = cudaMemsetAsync(A.arrive, 0, sizeof(unsigned int), st);
         if (e != cudaSuccess) return e;
@@ -533,6 +584,7 @@ cudaError_t launch_round(const DevParams& P, const ClusterDev& C, const RoundIO&
         case 4: e = round2_e<4>(P, C, io, st, &used); break;
         case 8: e = round2_e<8>(P, C, io, st, &used); break;
         case 16: e = round2_e<16>(P, C, io, st, &used); break;
+        case 32: e = round2_e<32>(P, C, io, st, &used); break;
         default: return cudaErrorInvalidValue;
         }
         if (e != cudaSuccess || used) return e;
@@ -543,7 +595,7 @@ cudaError_t launch_round(const DevParams& P, const ClusterDev& C, const RoundIO&
     case 4: return round_e<4>(P, C, io, st);
     case 8: return round_e<8>(P, C, io, st);
     case 16: return round_e<16>(P, C, io, st);
-    default: return cudaErrorInvalidValue;
+    default: return cudaErrorNotSupported;  // 1,024 slots need the sliced round
     }
 }
 

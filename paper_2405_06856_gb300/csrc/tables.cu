@@ -54,6 +54,22 @@ k_build_ovf(DevParams P, ClusterDev C, const int32_t* __restrict__ ovf, const in
     build_table<E>(P, C, ovf[idx], sm[warp]);
 }
 
+// Tables of 1,024 slots: one CTA of NW cooperating warps per worker (a
+// single warp cannot hold 32 elements per lane in registers). The workers are
+// `list[0..count)` with count read on the device (count_dev) or given.
+template <int EW, int NW>
+__global__ void __launch_bounds__(NW * 32)
+k_build_coop(DevParams P, ClusterDev C, const int32_t* __restrict__ list, int count,
+             const int* __restrict__ count_dev)
+{
+    extern __shared__ __align__(16) unsigned char smraw[];
+    BuildSmem<EW, NW>& sm = *reinterpret_cast<BuildSmem<EW, NW>*>(smraw);
+    const int n = count_dev ? *count_dev : count;
+    if ((int)blockIdx.x >= n) return;  // CTA-uniform
+    const int w = list ? list[blockIdx.x] : (int)blockIdx.x;
+    build_table_fit<EW, NW>(P, C, w, C.n[w], reinterpret_cast<unsigned char*>(&sm));
+}
+
 template <typename K>
 static cudaError_t allow_smem(K kern, size_t smem)
 {
@@ -62,6 +78,8 @@ static cudaError_t allow_smem(K kern, size_t smem)
     return cudaSuccess;
 }
 
+constexpr int COOP_NW = 8;
+
 template <int E>
 static cudaError_t build_e(const DevParams& P, const ClusterDev& C, const int32_t* list, int count,
                            cudaStream_t st)
@@ -69,21 +87,37 @@ static cudaError_t build_e(const DevParams& P, const ClusterDev& C, const int32_
     if (count <= 0) return cudaSuccess;
     const int blocks = (count + BUILD_WARPS - 1) / BUILD_WARPS;
     cudaError_t e;
-    if (E > E_LO && !list) {
-        constexpr int EL = E > E_LO ? E_LO : E;
-        const size_t slo = sizeof(BuildSmem<EL>) * BUILD_WARPS;
-        const size_t shi = sizeof(BuildSmem<E>) * BUILD_WARPS;
-        if ((e = allow_smem(k_build_lo<EL>, slo)) != cudaSuccess) return e;
-        if ((e = allow_smem(k_build_ovf<E>, shi)) != cudaSuccess) return e;
+    if constexpr (E > 16) {
+        constexpr int EW = E / COOP_NW;
+        const size_t sc = sizeof(BuildSmem<EW, COOP_NW>);
+        if ((e = allow_smem(k_build_coop<EW, COOP_NW>, sc)) != cudaSuccess) return e;
+        if (list) {
+            k_build_coop<EW, COOP_NW><<<count, COOP_NW * 32, sc, st>>>(P, C, list, count, nullptr);
+            return cudaGetLastError();
+        }
+        const size_t slo = sizeof(BuildSmem<E_LO>) * BUILD_WARPS;
+        if ((e = allow_smem(k_build_lo<E_LO>, slo)) != cudaSuccess) return e;
         if ((e = cudaMemsetAsync(C.novf, 0, sizeof(int), st)) != cudaSuccess) return e;
-        k_build_lo<EL><<<blocks, BUILD_WARPS * 32, slo, st>>>(P, C, count, C.ovf, C.novf);
-        k_build_ovf<E><<<blocks, BUILD_WARPS * 32, shi, st>>>(P, C, C.ovf, C.novf);
+        k_build_lo<E_LO><<<blocks, BUILD_WARPS * 32, slo, st>>>(P, C, count, C.ovf, C.novf);
+        k_build_coop<EW, COOP_NW><<<count, COOP_NW * 32, sc, st>>>(P, C, C.ovf, 0, C.novf);
+        return cudaGetLastError();
+    } else {
+        if (E > E_LO && !list) {
+            constexpr int EL = E > E_LO ? E_LO : E;
+            const size_t slo = sizeof(BuildSmem<EL>) * BUILD_WARPS;
+            const size_t shi = sizeof(BuildSmem<E>) * BUILD_WARPS;
+            if ((e = allow_smem(k_build_lo<EL>, slo)) != cudaSuccess) return e;
+            if ((e = allow_smem(k_build_ovf<E>, shi)) != cudaSuccess) return e;
+            if ((e = cudaMemsetAsync(C.novf, 0, sizeof(int), st)) != cudaSuccess) return e;
+            k_build_lo<EL><<<blocks, BUILD_WARPS * 32, slo, st>>>(P, C, count, C.ovf, C.novf);
+            k_build_ovf<E><<<blocks, BUILD_WARPS * 32, shi, st>>>(P, C, C.ovf, C.novf);
+            return cudaGetLastError();
+        }
+        const size_t smem = sizeof(BuildSmem<E>) * BUILD_WARPS;
+        if ((e = allow_smem(k_build<E>, smem)) != cudaSuccess) return e;
+        k_build<E><<<blocks, BUILD_WARPS * 32, smem, st>>>(P, C, list, count);
         return cudaGetLastError();
     }
-    const size_t smem = sizeof(BuildSmem<E>) * BUILD_WARPS;
-    if ((e = allow_smem(k_build<E>, smem)) != cudaSuccess) return e;
-    k_build<E><<<blocks, BUILD_WARPS * 32, smem, st>>>(P, C, list, count);
-    return cudaGetLastError();
 }
 
 cudaError_t launch_build(const DevParams& P, const ClusterDev& C, const int32_t* list, int count,
@@ -95,6 +129,7 @@ cudaError_t launch_build(const DevParams& P, const ClusterDev& C, const int32_t*
     case 4: return build_e<4>(P, C, list, count, st);
     case 8: return build_e<8>(P, C, list, count, st);
     case 16: return build_e<16>(P, C, list, count, st);
+    case 32: return build_e<32>(P, C, list, count, st);
     default: return cudaErrorInvalidValue;
     }
 }

@@ -123,8 +123,9 @@ def config(name, **over):
     w4096    4,096 workers, KV 131,072, 128 requests each, 32,768 candidates,
              output sigma 1.2 clipped at 4,096, seed 2.
     w16384   16,384 workers of 1/2/4/8 GPUs (KV 131,072 per GPU, latency
-             coefficients x 1/sqrt(GPUs)), 256 requests each, 131,072
-             candidates, output law as w4096, seed 3.
+             coefficients x 1/sqrt(GPUs)), 256 requests each (1,024 request
+             slots: an 8-GPU worker meets its SLOs with several hundred),
+             131,072 candidates, output law as w4096, seed 3.
     """
     if name == "tiny":
         kw = dict(seed=0, n_workers=16, per_worker=32, kv_per_gpu=16384, n_cand=64)
@@ -136,7 +137,7 @@ def config(name, **over):
     elif name == "w16384":
         kw = dict(seed=3, n_workers=16384, per_worker=256, kv_per_gpu=131072,
                   n_cand=131072, out_law=HEAVY_OUT, gpus_cycle=(1, 2, 4, 8),
-                  b_cap=512)
+                  b_cap=1024)
     else:
         raise KeyError(name)
     kw.update(over)

@@ -61,7 +61,7 @@ def test_create_rejects_bad_params(lib, bad):
     assert rc == lib.ERR_ARG and not h.value
 
 
-@pytest.mark.parametrize("b_cap", [16, 48, 1024])
+@pytest.mark.parametrize("b_cap", [16, 48, 2048])
 def test_create_rejects_bad_capacity(lib, b_cap):
     from paper_2405_06856_gb300 import synth
     p = lib.make_params(synth.BASE_PARAMS, b_cap)

@@ -186,3 +186,130 @@ def test_simulate_many_slices(A, orc, synth):
     assert int(out[2]) == ref["heartbeats"]
     assert out[3] == pytest.approx(ref["max_ttft"], rel=1e-12)
     assert out[4] == pytest.approx(ref["max_atgt"], rel=1e-12)
+
+
+def sorted_state(n, inp, gen, pred, pend, cap):
+    """Per-worker request multisets as one array sorted by (worker, in, gen,
+    pred, pend)."""
+    W = len(n)
+    slot = np.arange(W * cap) % cap
+    w = np.arange(W * cap) // cap
+    live = slot < np.repeat(n, cap)
+    cols = (w[live], inp[live], gen[live], pred[live], pend[live].astype(np.int32))
+    o = np.lexsort(cols[::-1])
+    return np.stack([c[o] for c in cols])
+
+
+def test_w16384_rounds_sampled(A, orc, synth):
+    """The 16,384-worker workload (1/2/4/8-GPU workers) at full size: three of
+    its consecutive greedy rounds with 100 ms of execution between them.
+    Sampled candidates are placed by the oracle on the same state (the others
+    take the GPU's placement); after each execution step the whole cluster
+    state must equal the oracle's."""
+    wl = synth.config("w16384")
+    C = wl.n_cand
+    bounds = np.linspace(0, C, 11).astype(int)
+    oc = orc.Cluster.from_workload(wl)
+    for w in range(oc.W):  # explicit "no history" decode time, as the library assumes
+        s = w * oc.cap
+        k = int(oc.n[w])
+        oc.tdec[s:s + k] = wl.params["theta"] * wl.params["T_dec"] * oc.gen[s:s + k]
+    oc.has_tdec = True
+    rng = np.random.default_rng(17)
+    t = 0.0
+    with A.Cluster.from_workload(wl) as cl:
+        for k in range(3):
+            a, b = int(bounds[k]), int(bounds[k + 1])
+            pl = cl.place_round(wl.cand_in[a:b], wl.cand_pred[a:b], wl.cand_wait[a:b])
+            assert cl.status() == A.OK
+            sample = set(rng.choice(b - a, 6, replace=False).tolist()) | {0, b - a - 1}
+            for i in range(b - a):
+                c = a + i
+                if i in sample:
+                    ref = oc.place_round(wl.cand_in[c:c + 1], wl.cand_pred[c:c + 1],
+                                         wl.cand_wait[c:c + 1].astype(np.float64))
+                    assert ref[0] == pl[i], (k, i, ref[0], pl[i])
+                elif pl[i] >= 0:
+                    oc.commit(pl[i], wl.cand_in[c], wl.cand_pred[c], float(wl.cand_wait[c]), c)
+            cl.advance(100.0)
+            oc.advance(t, 100.0)
+            t += 100.0
+            n, i_, g_, p_, pe = cl.state()
+            assert np.array_equal(n, oc.n), k
+            got = sorted_state(n, i_, g_, p_, pe, cl.b_cap)
+            ref = sorted_state(oc.n, oc.inp, oc.gen, oc.pred, oc.pend, oc.cap)
+            assert np.array_equal(got, ref), k
+
+
+def test_capacity_1024(A, orc, synth):
+    """Workers of 1,024 request slots (tables built by cooperating warps):
+    scoring, a greedy round and an execution step against the oracle."""
+    wl = synth.make_cluster("c1024", 250, 40, 700, 400000, 300, per_worker_random=True,
+                            b_cap=1024, gpus_cycle=(1, 2, 4, 8),
+                            params=dict(T_pre=3000.0, T_dec=120.0))
+    assert np.diff(wl.roff).max() > 512
+    with A.Cluster.from_workload(wl) as cl:
+        g = cl.score(wl.cand_in, wl.cand_pred, wl.cand_wait, detail=True)
+        oc = orc.Cluster.from_workload(wl)
+        ref = oc.score(wl.cand_in, wl.cand_pred, wl.cand_wait)
+        compare_pairs(ref, g["flags"], g["margin"], wl.cand_in, g["kvpeak"], g["tcand"], "c1024")
+        assert 0 < (g["flags"] == 15).mean() < 1
+        pl = cl.place_round(wl.cand_in, wl.cand_pred, wl.cand_wait)
+        rp = oc.place_round(wl.cand_in, wl.cand_pred, wl.cand_wait)
+        assert np.array_equal(pl, rp), np.argwhere(pl != rp)[:5]
+        assert (pl >= 0).any()
+        assert_same_state(cl, oc, "c1024-round")
+        for w in range(oc.W):
+            s = w * oc.cap
+            k = int(oc.n[w])
+            oc.tdec[s:s + k] = np.where(oc.pend[s:s + k] == 1, 0.0,
+                                        wl.params["theta"] * wl.params["T_dec"] * oc.gen[s:s + k])
+        oc.has_tdec = True
+        cl.advance(100.0)
+        oc.advance(0.0, 100.0)
+        assert_same_state(cl, oc, "c1024-advance")
+
+
+def test_round_rows_beyond_shared_memory(A, orc, synth):
+    """20,000 workers of 1,024 slots: each CTA of the round holds about 740
+    breakpoint rows per worker (one CTA per SM), fewer than the three heavy
+    workers have (about 900 distinct remaining lengths each); their row search
+    continues in the table in global memory."""
+    import dataclasses
+    W = 20000
+    wl = synth.make_cluster("rows", 240, W, 3, 65536, 300, per_worker_random=True, b_cap=1024,
+                            params=dict(T_pre=2000.0, T_dec=85.0))
+    heavy = {7: 900, 9000: 880, 19999: 910}
+    counts = np.diff(wl.roff).astype(np.int64)
+    ins, gens, preds = [], [], []
+    for w in range(W):
+        a, b = int(wl.roff[w]), int(wl.roff[w + 1])
+        if w in heavy:
+            r = np.arange(1, heavy[w] + 1, dtype=np.int32)  # distinct remaining lengths
+            ins.append(np.full(len(r), 16, np.int32))
+            gens.append(np.ones(len(r), np.int32))
+            preds.append(r + 1)
+            counts[w] = len(r)
+        else:
+            ins.append(wl.req_in[a:b])
+            gens.append(wl.req_gen[a:b])
+            preds.append(wl.req_pred[a:b])
+    roff = np.zeros(W + 1, np.int32)
+    np.cumsum(counts, out=roff[1:])
+    kv = wl.kv_capacity.copy()
+    for w in heavy:
+        kv[w] = 240000  # the KV constraint binds after some placements
+    rng = np.random.default_rng(241)
+    wl = dataclasses.replace(wl, roff=roff, req_in=np.concatenate(ins),
+                             req_gen=np.concatenate(gens), req_pred=np.concatenate(preds),
+                             kv_capacity=kv,
+                             cand_pred=rng.integers(1, 2500, wl.n_cand).astype(np.int32))
+    with A.Cluster.from_workload(wl) as cl:
+        pl = cl.place_round(wl.cand_in, wl.cand_pred, wl.cand_wait)
+        oc = orc.Cluster.from_workload(wl)
+        rp = oc.place_round(wl.cand_in, wl.cand_pred, wl.cand_wait)
+        assert np.array_equal(pl, rp), np.argwhere(pl != rp)[:5]
+        on_heavy = np.isin(pl, list(heavy))
+        assert on_heavy.any() and (~on_heavy).any()
+        assert (wl.cand_pred[on_heavy] > 750).any()
+        assert_same_state(cl, oc, "rows")
