@@ -629,15 +629,24 @@ __device__ unsigned build_table(const DevParams& P, const ClusterDev& C, int w,
         }
     }
 
-    // capacity_norm key: capacity_norm^2 is exact here (integer and
-    // half-integer terms below 2^53); non-negative doubles order like their
-    // bit patterns, and code 0 is kept for a worker holding an invalid request.
+    // capacity_norm key (one lane; code 0 is kept for a worker holding an
+    // invalid request): capacity_norm^2 is exact (integer and half-integer
+    // terms below 2^53) and non-negative doubles order like their bit
+    // patterns; with gamma = 1/2 the same order comes from integers.
     unsigned long long kq = 0ull;
-    if (q == 0 && lane == 0) {  // fp64 is slow on this part: one lane
-        const double kB = (double)n;
-        const double kL = __dadd_rn((double)sumIn, __dmul_rn(P.gammad, (double)sumPred));
-        const double kQ = __dadd_rn(__dmul_rn(kB, kB), __dmul_rn(kL, kL));
-        kq = bad ? 0ull : (unsigned long long)__double_as_longlong(kQ) + 1ull;
+    if (q == 0 && lane == 0 && !bad) {
+        if (P.gammad == 0.5) {
+            // 4 capacity_norm^2 = (2B)^2 + (2 sum in + sum pred)^2 in integers
+            // (the same order and ties as the exact double value)
+            const unsigned long long b2 = 2ull * (unsigned long long)n;
+            const unsigned long long s2 = 2ull * (unsigned long long)sumIn + (unsigned long long)sumPred;
+            kq = b2 * b2 + s2 * s2 + 1ull;
+        } else {
+            const double kB = (double)n;
+            const double kL = __dadd_rn((double)sumIn, __dmul_rn(P.gammad, (double)sumPred));
+            const double kQ = __dadd_rn(__dmul_rn(kB, kB), __dmul_rn(kL, kL));
+            kq = (unsigned long long)__double_as_longlong(kQ) + 1ull;
+        }
     }
 
     constexpr int N = BuildSmem<EW, NW>::N;
