@@ -176,6 +176,10 @@ struct R2Split {
     static constexpr int NW = E <= 8 ? E : 12;
     static constexpr int EW = E <= 8 ? 1 : E / 8;
 };
+// Breakpoint rows of a worker in shared memory are 16-bit; rc (a multiple of
+// 8) plus this pad makes the per-worker stride an odd number of 32-bit words,
+// so that lanes searching neighbouring workers start on different banks.
+constexpr int R2_RHO_PAD = 2;
 constexpr long long GRID_WAIT_LIMIT = 1ll << 22;  // polls of the arrival counter (seconds)
 constexpr int NONE = 0x7fffffff;
 
@@ -306,10 +310,11 @@ __global__ void __launch_bounds__(R2_THREADS, 1) k_round2(R2Args A)
     }
     __syncthreads();
     const int rc = A.rc;
+    const int rs = rc + R2_RHO_PAD;  // per-worker stride: an odd number of words
     for (int k = tid; k < nloc * rc; k += R2_THREADS) {
         const int lw = k / rc, q = k - lw * rc;
         if (q < R_s[lw])
-            rho[k] = (unsigned short)(
+            rho[lw * rs + q] = (unsigned short)(
                 __float_as_int(C.tab[((long long)(w_lo + lw) * C.rows + q) * ROW_F4].x) - 1);
     }
     if (tid == 0) sm.stop = (io.sim && *io.status != 0) ? 1 : 0;
@@ -362,7 +367,7 @@ __global__ void __launch_bounds__(R2_THREADS, 1) k_round2(R2Args A)
         if (rebuilding && warp < NW) {
             append(pend_w);
             const int lw = pend_w - w_lo;
-            SliceCache sc{rho + (long long)lw * rc, rc, &R_s[lw], &wrec_s[lw], &key_s[lw]};
+            SliceCache sc{rho + (long long)lw * rs, rc, &R_s[lw], &wrec_s[lw], &key_s[lw]};
             const unsigned f = build_table_fit<EW, NW, NW_INSERT>(P, C, pend_w, n_s[lw],
                                                        reinterpret_cast<unsigned char*>(&sm.build),
                                                        &sc, cr.valid ? &cr : nullptr);
@@ -374,7 +379,7 @@ __global__ void __launch_bounds__(R2_THREADS, 1) k_round2(R2Args A)
                 const int w = w_lo + lw;
                 if (w == pend_w) continue;
                 const long long rb = (long long)w * C.rows;
-                const int p = r2_find(rho + (long long)lw * rc, R_s[lw], rc, cr.ri, C.tab, rb);
+                const int p = r2_find(rho + (long long)lw * rs, R_s[lw], rc, cr.ri, C.tab, rb);
                 const long long row = rb + p;
                 const float4* t = C.tab + row * ROW_F4;
                 float m;
@@ -477,7 +482,7 @@ __global__ void __launch_bounds__(R2_THREADS, 1) k_round2(R2Args A)
     if (pend_w >= 0 && warp < NW) {
         append(pend_w);
         const int lw = pend_w - w_lo;
-        SliceCache sc{rho + (long long)lw * rc, rc, &R_s[lw], &wrec_s[lw], &key_s[lw]};
+        SliceCache sc{rho + (long long)lw * rs, rc, &R_s[lw], &wrec_s[lw], &key_s[lw]};
         build_table_fit<EW, NW, NW_INSERT>(P, C, pend_w, n_s[lw],
                                            reinterpret_cast<unsigned char*>(&sm.build),
                                 &sc, nullptr);
@@ -496,7 +501,7 @@ template <int E>
 static size_t r2_smem(int slice, int rc)
 {
     return ((sizeof(R2Smem<E>) + 15) / 16) * 16 + (size_t)slice * (16 + 8 + 4 + 4) +
-           (size_t)slice * rc * 2;
+           (size_t)slice * (rc + R2_RHO_PAD) * 2;
 }
 constexpr int R2_MIN_RC = 64;  // fewer rows per worker in shared memory: use the plain round
 
@@ -517,16 +522,17 @@ static cudaError_t round2_e(const DevParams& P, const ClusterDev& C, const Round
     if (sms > ROUND_XBUF_SMS) return cudaSuccess;
     const size_t budget = (size_t)smem_max - 1024;
     const size_t base = r2_smem<E>(0, 0);
-    if (budget <= base + 32 + 2 * R2_MIN_RC) return cudaSuccess;
+    if (budget <= base + 32 + 2 * (R2_MIN_RC + R2_RHO_PAD)) return cudaSuccess;
     // As few CTAs as hold every worker's rows; beyond one CTA per SM, the
     // slices hold only the first rc rows of each worker.
     int rc = C.cap;
-    const long long slice_max = (long long)((budget - base) / (32 + 2 * (size_t)rc));
+    const long long slice_max =
+        (long long)((budget - base) / (32 + 2 * (size_t)(rc + R2_RHO_PAD)));
     int G = (int)((C.W + slice_max - 1) / slice_max);
     if (G > sms) {
         G = sms;
         const long long sl = (C.W + G - 1) / G;
-        rc = (int)((((budget - base) / (size_t)sl) - 32) / 2) & ~7;
+        rc = ((int)((((budget - base) / (size_t)sl) - 32) / 2) - R2_RHO_PAD) & ~7;
         if (rc < R2_MIN_RC) return cudaSuccess;
     }
     if (G > 1 && !coop) return cudaSuccess;  // use the single-CTA round

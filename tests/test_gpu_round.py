@@ -313,3 +313,22 @@ def test_round_rows_beyond_shared_memory(A, orc, synth):
         assert on_heavy.any() and (~on_heavy).any()
         assert (wl.cand_pred[on_heavy] > 750).any()
         assert_same_state(cl, oc, "rows")
+
+
+def test_min_workers_four_options(A, orc, synth):
+    """The minimum-worker search of the 1/2/4/8-GPU options (KV 32,768 tokens
+    per GPU, latency x 1/sqrt(GPUs), 1,024 request slots) on the diurnal
+    trace scaled down to 10,000 requests at a peak of 200 req/s."""
+    tr = synth.diurnal_trace(14, 10000, 200.0, 50.0)
+    p = dict(synth.BASE_PARAMS)
+    gpus = [1, 2, 4, 8]
+    M = [32768 * g for g in gpus]
+    sc = [1.0 / np.sqrt(g) for g in gpus]
+    ref = orc.min_workers(p, gpus, M, sc, 1024, tr, 100.0, 256)
+    got = np.zeros(4, np.int32)
+    best, total = A.aladdin_min_workers(A.make_params(p, 1024), A.make_cfgs(gpus, M, sc),
+                                        A.make_trace(tr.t_arr, tr.req_in, tr.req_pred), 100.0, 256,
+                                        got)
+    assert np.array_equal(got, ref), (got, ref)
+    tot = [g * n for g, n in zip(gpus, ref)]
+    assert total == min(tot) and best == int(np.argmin(tot))
