@@ -40,7 +40,7 @@ WORKLOAD_DESC = ("4,096 workers x 128 ongoing requests (KV capacity 131,072 toke
                  "ms/KV token, prefill 10 ms + 0.1 ms/100 tokens, TTFT 1 s, ATGT 50 ms; seed 2")
 L2_FLUSH_BYTES = 256 << 20
 # minimum-worker search: KV tokens per GPU and per-worker request slots
-MW_KV_PER_GPU = 32768
+MW_KV_PER_GPU = 65536
 MW_B_CAP = 1024
 
 

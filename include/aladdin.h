@@ -13,9 +13,13 @@
  * Conventions
  *  - Lengths are int32 token counts, times are milliseconds.
  *  - Pointer arguments may point to host memory or to device memory of the
- *    cluster's GPU; the library inspects each pointer. With device pointers a
- *    call is asynchronous on the cluster's stream; when any output is in host
- *    memory the call returns after the stream has completed.
+ *    cluster's GPU; the library inspects each pointer. Page-locked host memory
+ *    that the GPU can address (cudaHostAlloc, cudaHostRegister, torch
+ *    pin_memory) is read and written in place by the kernels, like device
+ *    memory; pageable host memory is staged through device buffers. With
+ *    device pointers only, a call is asynchronous on the cluster's stream;
+ *    when any argument is in host memory the call returns after the stream
+ *    has completed.
  *  - The caller owns every buffer it passes; the library never frees caller
  *    memory and keeps no pointer to it after the call returns.
  *  - Pair outputs are row-major [candidate][worker].
@@ -103,11 +107,12 @@ int aladdin_cluster_destroy(aladdin_cluster* cl);
 /* Replace every worker's requests (same layout as aladdin_cluster_create) and
  * rebuild the per-worker projection tables: packing into device slots, sorting
  * of remaining lengths, breakpoints, prefix sums, KV and latency curves at the
- * breakpoints and the capacity_norm ranking (Sec. 4.2). Host inputs are
- * validated before upload (ALADDIN_ERR_ARG / ALADDIN_ERR_CAPACITY). Device
- * inputs are validated on the GPU: a worker holding an invalid request is made
- * infeasible for every candidate and the cluster records ALADDIN_ERR_STATE,
- * which aladdin_cluster_status returns. Any round in progress is discarded
+ * breakpoints and the capacity_norm ranking (Sec. 4.2). Pageable host inputs
+ * are validated on the host before upload (ALADDIN_ERR_ARG /
+ * ALADDIN_ERR_CAPACITY). Device and page-locked host inputs are packed and
+ * validated on the GPU: a worker holding an invalid request is made infeasible
+ * for every candidate and the cluster records ALADDIN_ERR_STATE, which
+ * aladdin_cluster_status returns. Any round in progress is discarded
  * and the cluster clock is kept. */
 int aladdin_cluster_load(aladdin_cluster* cl, const int32_t* req_off, const int32_t* in,
                          const int32_t* gen, const int32_t* pred, const float* tdec_ms);
@@ -194,9 +199,9 @@ int aladdin_cluster_state(aladdin_cluster* cl, int32_t* n, int32_t* in, int32_t*
 int aladdin_cluster_timing(aladdin_cluster* cl, int32_t enable, double* kernel_ms,
                            int64_t* launches);
 
-/* ALADDIN_OK; ALADDIN_ERR_TIMEOUT if a kernel gave up a bounded wait for its
- * own shared-memory copies (its outputs for that call are incomplete);
- * ALADDIN_ERR_STATE if an invalid request was loaded from device memory; or
+/* ALADDIN_OK; ALADDIN_ERR_TIMEOUT if a kernel gave up a bounded wait (its
+ * outputs for that call are incomplete); ALADDIN_ERR_STATE if an invalid
+ * request was loaded from device or page-locked host memory; or
  * ALADDIN_ERR_CUDA. Errors are sticky. Synchronous. */
 int aladdin_cluster_status(aladdin_cluster* cl);
 

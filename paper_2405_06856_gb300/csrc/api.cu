@@ -37,10 +37,14 @@ struct DevBuf {
     T* as() const { return reinterpret_cast<T*>(p); }
 };
 
-enum PtrKind { PK_NULL = 0, PK_HOST = 1, PK_DEV = 2 };
+// Pointer kinds: device memory; page-locked host memory mapped into the
+// device's address space (kernels read and write it in place, over the
+// CPU-GPU link, without a staging copy); pageable host memory (staged).
+enum PtrKind { PK_NULL = 0, PK_HOST = 1, PK_DEV = 2, PK_MAPPED = 3 };
 
-PtrKind ptr_kind(const void* p)
+PtrKind ptr_kind(const void* p, void** devp = nullptr)
 {
+    if (devp) *devp = nullptr;
     if (!p) return PK_NULL;
     cudaPointerAttributes a;
     cudaError_t e = cudaPointerGetAttributes(&a, p);
@@ -48,8 +52,25 @@ PtrKind ptr_kind(const void* p)
         cudaGetLastError();
         return PK_HOST;
     }
-    if (a.type == cudaMemoryTypeDevice || a.type == cudaMemoryTypeManaged) return PK_DEV;
+    if (a.type == cudaMemoryTypeDevice || a.type == cudaMemoryTypeManaged) {
+        if (devp) *devp = const_cast<void*>(p);
+        return PK_DEV;
+    }
+    if (a.type == cudaMemoryTypeHost && a.devicePointer) {
+        if (devp) *devp = a.devicePointer;
+        return PK_MAPPED;
+    }
     return PK_HOST;
+}
+
+// The device-accessible address of p (device or mapped page-locked memory).
+template <typename T>
+bool device_view(const T* p, T** out)
+{
+    void* d = nullptr;
+    const PtrKind k = ptr_kind(p, &d);
+    *out = reinterpret_cast<T*>(d);
+    return k == PK_DEV || k == PK_MAPPED;
 }
 
 bool finite_nonneg(double x) { return std::isfinite(x) && x >= 0.0; }
@@ -375,14 +396,17 @@ int load_requests(aladdin_cluster* cl, const int32_t* req_off, const int32_t* in
                   const int32_t* gen, const int32_t* pred, const float* tdec)
 {
     if (!req_off) return ALADDIN_ERR_ARG;
-    const bool dev = ptr_kind(req_off) == PK_DEV && (!in || ptr_kind(in) == PK_DEV) &&
-                     (!gen || ptr_kind(gen) == PK_DEV) && (!pred || ptr_kind(pred) == PK_DEV) &&
-                     (!tdec || ptr_kind(tdec) == PK_DEV);
+    // device or page-locked host arrays: packed on the device, read in place
+    int32_t *d_off = nullptr, *d_in = nullptr, *d_gen = nullptr, *d_pred = nullptr;
+    float* d_tdec = nullptr;
+    const bool dev = device_view(req_off, &d_off) && (!in || device_view(in, &d_in)) &&
+                     (!gen || device_view(gen, &d_gen)) && (!pred || device_view(pred, &d_pred)) &&
+                     (!tdec || device_view(tdec, &d_tdec));
     if (!dev) return load_requests_host(cl, req_off, in, gen, pred, tdec);
     if (!in || !gen || !pred) return ALADDIN_ERR_ARG;
     const int wpb = 4;
-    k_pack<<<(cl->W + wpb - 1) / wpb, 32 * wpb, 0, cl->st>>>(cl->dp, cl->dev, req_off, in, gen,
-                                                             pred, tdec);
+    k_pack<<<(cl->W + wpb - 1) / wpb, 32 * wpb, 0, cl->st>>>(cl->dp, cl->dev, d_off, d_in, d_gen,
+                                                             d_pred, d_tdec);
     CK(cudaGetLastError());
     return ALADDIN_OK;
 }
@@ -395,8 +419,9 @@ int stage_in(aladdin_cluster* cl, DevBuf& buf, const T* src, size_t count, const
         *out = nullptr;
         return ALADDIN_OK;
     }
-    if (ptr_kind(src) == PK_DEV) {
-        *out = src;
+    T* d = nullptr;
+    if (device_view(src, &d)) {
+        *out = d;
         return ALADDIN_OK;
     }
     CK(buf.ensure(sizeof(T) * count));
@@ -413,8 +438,9 @@ int stage_out(DevBuf& buf, T* dst, size_t count, T** out, bool* host)
         *out = nullptr;
         return ALADDIN_OK;
     }
-    if (ptr_kind(dst) == PK_DEV) {
-        *out = dst;
+    T* d = nullptr;
+    if (device_view(dst, &d)) {  // device memory, or page-locked host memory written in place
+        *out = d;
         return ALADDIN_OK;
     }
     CK(buf.ensure(sizeof(T) * count));
@@ -471,10 +497,11 @@ int score_impl(aladdin_cluster* cl, int32_t n, const int32_t* in, const int32_t*
     if (ha) CK(cudaMemcpyAsync(argbest, darg, sizeof(int32_t) * C, cudaMemcpyDeviceToHost, cl->st));
     if (hk) CK(cudaMemcpyAsync(kv_peak, dkv, sizeof(int64_t) * pairs, cudaMemcpyDeviceToHost, cl->st));
     if (ht) CK(cudaMemcpyAsync(t_cand, dtc, sizeof(float) * pairs, cudaMemcpyDeviceToHost, cl->st));
-    // host inputs were staged asynchronously from caller memory: complete
-    // before returning whenever host memory is involved
-    const bool any_host = hf || hm || ha || hk || ht || ptr_kind(in) == PK_HOST ||
-                          ptr_kind(pred) == PK_HOST || (wait && ptr_kind(wait) == PK_HOST);
+    // complete before returning whenever host memory is involved (staged or
+    // read and written in place)
+    auto on_host = [](const void* p) { return p && ptr_kind(p) != PK_DEV; };
+    const bool any_host = on_host(in) || on_host(pred) || on_host(wait) || on_host(flags) ||
+                          on_host(margin) || on_host(argbest) || on_host(kv_peak) || on_host(t_cand);
     if (any_host) CK(cudaStreamSynchronize(cl->st));
     return ALADDIN_OK;
 }

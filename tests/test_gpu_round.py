@@ -316,13 +316,13 @@ def test_round_rows_beyond_shared_memory(A, orc, synth):
 
 
 def test_min_workers_four_options(A, orc, synth):
-    """The minimum-worker search of the 1/2/4/8-GPU options (KV 32,768 tokens
+    """The minimum-worker search of the 1/2/4/8-GPU options (KV 65,536 tokens
     per GPU, latency x 1/sqrt(GPUs), 1,024 request slots) on the diurnal
     trace scaled down to 10,000 requests at a peak of 200 req/s."""
     tr = synth.diurnal_trace(14, 10000, 200.0, 50.0)
     p = dict(synth.BASE_PARAMS)
     gpus = [1, 2, 4, 8]
-    M = [32768 * g for g in gpus]
+    M = [65536 * g for g in gpus]
     sc = [1.0 / np.sqrt(g) for g in gpus]
     ref = orc.min_workers(p, gpus, M, sc, 1024, tr, 100.0, 256)
     got = np.zeros(4, np.int32)

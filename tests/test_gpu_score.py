@@ -213,3 +213,39 @@ def test_w4096_sampled(A, orc, synth):
         mr_rows = m[torch.from_numpy(rows).long().to(dev)].cpu().numpy()
         compare_pairs(sub, fr_rows, mr_rows, wl.cand_in[rows], label="w4096-rows")
         check_argbest(order, fr_rows, a.cpu().numpy()[rows], "w4096-rows")
+
+
+def test_page_locked_host_buffers(A, orc, synth):
+    """Page-locked host arrays are read and written in place by the kernels
+    (state packed on the device, outputs written over the CPU-GPU link): the
+    results equal the device-buffer results byte for byte, and the state
+    packed from them scores like the oracle."""
+    import torch
+    wl = synth.config("w256", n_cand=600)
+    dev = torch.device("cuda")
+    pin = lambda x: torch.from_numpy(np.ascontiguousarray(x)).pin_memory()
+    C, W = wl.n_cand, wl.n_workers
+    with A.Cluster.from_workload(wl) as cl:
+        cl.load(pin(wl.roff), pin(wl.req_in), pin(wl.req_gen), pin(wl.req_pred))
+        assert cl.status() == A.OK
+        hf = torch.zeros((C, W), dtype=torch.uint8).pin_memory()
+        hm = torch.zeros((C, W), dtype=torch.float32).pin_memory()
+        ha = torch.zeros(C, dtype=torch.int32).pin_memory()
+        A.aladdin_score(cl.handle, C, pin(wl.cand_in), pin(wl.cand_pred), pin(wl.cand_wait), hf, hm,
+                        ha)
+        df = torch.zeros((C, W), dtype=torch.uint8, device=dev)
+        dm = torch.zeros((C, W), dtype=torch.float32, device=dev)
+        da = torch.zeros(C, dtype=torch.int32, device=dev)
+        A.aladdin_score(cl.handle, C, torch.from_numpy(wl.cand_in).to(dev),
+                        torch.from_numpy(wl.cand_pred).to(dev), torch.from_numpy(wl.cand_wait).to(dev),
+                        df, dm, da)
+        torch.cuda.synchronize()
+        assert np.array_equal(hf.numpy(), df.cpu().numpy())
+        assert np.array_equal(hm.numpy().view(np.uint32), dm.cpu().numpy().view(np.uint32))
+        assert np.array_equal(ha.numpy(), da.cpu().numpy())
+        ref = orc.Cluster.from_workload(wl).score(wl.cand_in, wl.cand_pred, wl.cand_wait)
+        compare_pairs(ref, hf.numpy(), hm.numpy(), wl.cand_in, label="pinned")
+        hp = torch.zeros(C, dtype=torch.int32).pin_memory()
+        A.aladdin_place_round(cl.handle, C, pin(wl.cand_in), pin(wl.cand_pred), pin(wl.cand_wait), hp)
+        rp = orc.Cluster.from_workload(wl).place_round(wl.cand_in, wl.cand_pred, wl.cand_wait)
+        assert np.array_equal(hp.numpy(), rp)
