@@ -47,6 +47,17 @@
  * constraint the largest admissible l. The pair's margin is the smallest of
  * these bounds minus a_c: the number of extra prompt tokens the worker could
  * still absorb for this candidate (negative: infeasible).
+ *
+ * Approximate mode (mode 1): the MIP's own decode constraints replace the
+ * projection of groups 2 and 3, as the paper states them (Sec. 4.2):
+ *   (d) ongoing  tau <= theta * min_j (T_dec * l_out_j - t_dec_j) over the
+ *                requests decoding at round start (t_dec_j = theta * T_dec *
+ *                l_out_j when no history is given)
+ *   (b) new      sum over the worker's requests and the candidate of
+ *                (l_in + gamma * l_pred) <= theta * l_d(B), B = requests with
+ *                the candidate, l_d(b) = (T_dec / scale_i - c3 - c2 b) / k2
+ *                (Eq. input limit).
+ * KV (e) and TTFT (c) are as in the exact mode.
  */
 #include <math.h>
 #include <stdint.h>
@@ -60,6 +71,8 @@ typedef struct {
     double T_pre, T_dec;  /* TTFT SLO, per-token decode SLO (ms) */
     double gamma, theta;  /* capacity_norm weight, SLO scaling knob */
     int64_t K;            /* sequence limit (input + output tokens) */
+    int64_t mode;         /* 0: exact decode projection; 1: approximate
+                             constraints (b) and (d) of the MIP (Sec. 4.2) */
 } orc_params;
 
 /* Cluster state in fixed-stride slots: worker w owns slots
@@ -250,6 +263,31 @@ static void eval_pair(const orc_params* p, const orc_cluster* cl, int w, const o
         lat_constraint(&A, 1, p->T_pre - wq - off - tau0, tau1, p->T_pre + wq + off + tau_a, a);
     }
 
+    if (p->mode == 1) {
+        /* (d) as stated: the stall within theta times the smallest decode time
+         * an ongoing request has saved so far. */
+        for (int q = 0; q < cl->n[w]; ++q) {
+            int64_t slot = base + q;
+            if (cl->pend[slot]) continue;
+            double g = (double)cl->gen[slot];
+            double td = cl->tdec ? cl->tdec[slot] : p->theta * p->T_dec * g;
+            double saved = p->theta * (p->T_dec * g - td);
+            lat_constraint(&A, 2, saved - tau0, tau1, fabs(saved) + tau_a, a);
+        }
+        /* (b) with Eq. input limit: weighted context of the batch with the
+         * candidate within theta * l_d(B). */
+        double L = 0.0;
+        for (int q = 0; q < cl->n[w]; ++q)
+            L += (double)cl->in[base + q] + p->gamma * (double)cl->pred[base + q];
+        double B = (double)cl->n[w] + 1.0;
+        double ld = (p->T_dec / sc - p->c3 - p->c2 * B) / p->k2;
+        double cap_b = p->theta * ld - L - p->gamma * (double)r_c;
+        lat_constraint(&A, 3, cap_b, 1.0, fabs(p->theta * ld) + L + p->gamma * (double)r_c + a, a);
+        {
+            double D0 = T0[r_c], D1 = T1[r_c];
+            out->t_cand = D0 + D1 * a;
+        }
+    } else {
     /* (d) ongoing requests: stall plus remaining decode within their budget. */
     for (int q = 0; q < cl->n[w]; ++q) {
         int64_t slot = base + q;
@@ -272,6 +310,7 @@ static void eval_pair(const orc_params* p, const orc_cluster* cl, int w, const o
         double D0 = T0[r_c], D1 = T1[r_c];
         lat_constraint(&A, 3, budget - D0, D1, budget + D0 + D1 * a, a);
         out->t_cand = D0 + D1 * a;
+    }
     }
 
     double bound = A.bound, bscale = A.bscale;

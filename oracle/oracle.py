@@ -36,7 +36,8 @@ class Params(C.Structure):
     _fields_ = [("k1", C.c_double), ("c1", C.c_double), ("k2", C.c_double),
                 ("c2", C.c_double), ("c3", C.c_double), ("h", C.c_int64),
                 ("j", C.c_int64), ("T_pre", C.c_double), ("T_dec", C.c_double),
-                ("gamma", C.c_double), ("theta", C.c_double), ("K", C.c_int64)]
+                ("gamma", C.c_double), ("theta", C.c_double), ("K", C.c_int64),
+                ("mode", C.c_int64)]
 
 
 class ClusterStruct(C.Structure):
@@ -74,7 +75,8 @@ def lib():
 def make_params(d):
     return Params(float(d["k1"]), float(d["c1"]), float(d["k2"]), float(d["c2"]),
                   float(d["c3"]), int(d["h"]), int(d["j"]), float(d["T_pre"]),
-                  float(d["T_dec"]), float(d["gamma"]), float(d["theta"]), int(d["K"]))
+                  float(d["T_dec"]), float(d["gamma"]), float(d["theta"]), int(d["K"]),
+                  int(d.get("mode", 0)))
 
 
 def _ptr(a):

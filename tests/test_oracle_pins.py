@@ -377,3 +377,68 @@ def test_min_workers_linear_scan(orc, synth):
     assert all(oks[first - 1:]), oks   # monotone on this trace
     got = orc.min_workers(p, [1], [32768], [1.0], 256, tr, 100.0, 16)
     assert got[0] == first
+
+
+# --------------------------------------------------------------------------
+# Approximate mode: the MIP's constraints (b) (with Eq. input limit) and (d)
+# as stated in Sec. 4.2, worked by hand.
+
+APPROX = dict(k1=0.01, c1=5.0, k2=0.001, c2=1.0, c3=10.0, h=1, j=0, T_pre=1000.0, T_dec=50.0,
+              gamma=0.5, theta=0.8, K=8192, mode=1)
+
+
+@pytest.mark.parametrize("T_dec,tdec,flags,margin", [
+    # (b): L = (100 + 0.5*60) + (300 + 0.5*40) = 450; l_d(3) = (50 - 10 - 3)/0.001
+    # = 37,000; bound 0.8*37,000 - 450 - 0.5*30 = 29,135. (d): saved time
+    # 0.8*(50*20 - 700) = 240 and 0.8*(50*5 - 200) = 40; stall 0.01*a + 5 <= 40
+    # gives a <= 3,500 (binding). TTFT: a <= (1000 - 5)/0.01 = 99,500.
+    (50.0, [700.0, 200.0], 15, 3500.0 - 150.0),
+    # request 2 saved only 0.8*(250 - 249) = 0.8 ms < the 6.5 ms stall: (d) fails,
+    # bound (0.8 - 5)/0.01 = -420
+    (50.0, [700.0, 249.0], 11, -420.0 - 150.0),
+    # T_dec 10.5: l_d(3) = (10.5 - 10 - 3)/0.001 = -2,500, bound 0.8*(-2,500) - 465
+    # = -2,465: (b) fails; saved 0.8*(210 - 150) = 48 and 0.8*(52.5 - 40) = 10
+    # keep (d) (a <= 500)
+    (10.5, [150.0, 40.0], 7, -2465.0 - 150.0),
+])
+def test_approx_hand_example(orc, T_dec, tdec, flags, margin):
+    p = dict(APPROX, T_dec=T_dec)
+    cl = one_worker(orc, p, 10**6, [(100, 20, 60), (300, 5, 40)], tdec=tdec)
+    r = cl.score([150], [30], [0.0])
+    assert int(r["flags"][0, 0]) == flags
+    assert r["margin"][0, 0] == pytest.approx(margin, rel=1e-12)
+
+
+def test_approx_input_limit_per_request(orc, synth):
+    """Each request added to a worker lowers the (b) bound by theta * c2 / k2
+    (Eq. input limit's slope in the batch size) plus its own l_in + gamma
+    l_pred, whatever the rest of the worker holds."""
+    rng = np.random.default_rng(31)
+    p = dict(APPROX, T_dec=100.0, T_pre=1e9)
+    # every request has generated 10 tokens in no time: (d) allows a stall of
+    # 0.8 * 100 * 10 = 800 ms (a <= 79,500), looser than (b) (a <= ~60,000)
+    for _ in range(20):
+        n = int(rng.integers(1, 12))
+        reqs = [(int(rng.integers(16, 500)), 10, int(rng.integers(11, 300))) for _ in range(n)]
+        cand_in, cand_pred = int(rng.integers(16, 200)), int(rng.integers(8, 200))
+        margins = []
+        for k in (n - 1, n):
+            cl = one_worker(orc, p, 10**9, reqs[:k], tdec=[0.0] * k)
+            margins.append(cl.score([cand_in], [cand_pred], [0.0])["margin"][0, 0])
+        added = reqs[n - 1][0] + p["gamma"] * reqs[n - 1][2]
+        assert margins[0] - margins[1] == pytest.approx(p["theta"] * p["c2"] / p["k2"] + added,
+                                                        rel=1e-12)
+
+
+def test_approx_and_exact_share_kv_and_ttft(orc, synth):
+    """Switching the mode changes only the two decode-SLO groups: the KV and
+    TTFT flags and the KV peaks of every pair are the same."""
+    wl = synth.config("tiny", per_worker_random=True, seed=32, n_cand=80,
+                      params=dict(T_pre=60.0, T_dec=30.0, theta=0.9))
+    ex = orc.Cluster.from_workload(wl).score(wl.cand_in, wl.cand_pred, wl.cand_wait)
+    ap = orc.Cluster(dict(wl.params, mode=1), wl.kv_capacity, wl.lat_scale, wl.b_cap, wl.roff,
+                     wl.req_in, wl.req_gen, wl.req_pred).score(wl.cand_in, wl.cand_pred,
+                                                               wl.cand_wait)
+    assert np.array_equal(ex["flags"] & 3, ap["flags"] & 3)
+    assert np.array_equal(ex["kvpeak"], ap["kvpeak"])
+    assert (ex["flags"] != ap["flags"]).any()
