@@ -307,6 +307,7 @@ def run_ours(args):
             rounds.append((time.perf_counter() - t0) * 1000.0)
     round_ms = min(rounds)
     r16k = rounds_w16384(A, synth, stream)
+    apx = approx_mode(A, synth, dev, stream, flush)
 
     peak, peak_kind = read_peaks()
     kern_avg = kern_ms / max(kern_n, 1)
@@ -336,6 +337,7 @@ def run_ours(args):
             "round_latency_ms": {"workload": "256 workers x 64 requests, 2,048 candidates, one "
                                              "greedy round", "value": round_ms},
             "rounds_w16384": r16k,
+            "approx_mode": apx,
             "clocks": clocks}
     if cpu is not None:
         line["cpu_baseline"] = cpu
@@ -373,6 +375,50 @@ def rounds_w16384(A, synth, stream, n_rounds=10, dt_ms=100.0):
             "ms_per_round": statistics.mean(rounds), "ms_max_round": max(rounds),
             "ms_per_advance": statistics.mean(advances),
             "placed_fraction": placed / float(wl.n_cand)}
+
+
+def approx_mode(A, synth, dev, stream, flush, launches=10):
+    """The approximate mode (the placement MIP's constraints (b), with Eq.
+    input limit, and (d)): scoring-kernel time on the 4,096-worker workload
+    (theta 0.9), and on the 256-worker workload with a decode history how its
+    flags differ from the exact projection's."""
+    import torch
+    wl = synth.config(WORKLOAD, params=dict(theta=0.9, mode=1))
+    W, C = wl.n_workers, wl.n_cand
+    d = lambda x: torch.from_numpy(np.ascontiguousarray(x)).to(dev)
+    cin, cpr, cw = d(wl.cand_in), d(wl.cand_pred), d(wl.cand_wait)
+    f = torch.empty((C, W), dtype=torch.uint8, device=dev)
+    m = torch.empty((C, W), dtype=torch.float32, device=dev)
+    a = torch.empty(C, dtype=torch.int32, device=dev)
+    with A.Cluster.from_workload(wl, stream=stream) as cl:
+        for _ in range(3):
+            A.aladdin_score(cl.handle, C, cin, cpr, cw, f, m, a)
+        torch.cuda.synchronize()
+        A.aladdin_cluster_timing(cl.handle, 1)
+        for _ in range(launches):
+            flush.zero_()
+            A.aladdin_score(cl.handle, C, cin, cpr, cw, f, m, a)
+        kern_ms, kern_n = A.aladdin_cluster_timing(cl.handle, 0)
+        feas4096 = float((f == 15).float().mean().item())
+    kern = kern_ms / max(kern_n, 1)
+    # flags of both modes on the 256-worker workload with a decode history
+    gen = synth.config("w256").req_gen
+    tdec = (gen * np.random.default_rng(7).uniform(10.0, 50.0, len(gen))).astype(np.float32)
+    out = {}
+    for mode in (0, 1):
+        w2 = synth.config("w256", params=dict(theta=0.9, mode=mode))
+        with A.Cluster.from_workload(w2, tdec_ms=tdec, stream=stream) as c2:
+            out[mode] = c2.score(w2.cand_in, w2.cand_pred, w2.cand_wait)["flags"]
+    ex, ap = out[0] == 15, out[1] == 15
+    return {"workload": "4,096-worker workload with theta 0.9 (scoring time); 256-worker workload "
+                        "with theta 0.9 and decode histories of 10-50 ms a token (flag gap)",
+            "k_score_us": kern * 1000.0,
+            "evals_per_s_kernel": C * W / (kern / 1000.0),
+            "feasible_fraction_w4096": round(feas4096, 4),
+            "w256_feasible_exact": round(float(ex.mean()), 4),
+            "w256_feasible_approx": round(float(ap.mean()), 4),
+            "w256_approx_feasible_exact_infeasible": round(float((ap & ~ex).mean()), 4),
+            "w256_exact_feasible_approx_infeasible": round(float((ex & ~ap).mean()), 4)}
 
 
 def min_workers_config(synth):

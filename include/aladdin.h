@@ -58,13 +58,27 @@ extern "C" {
 #define ALADDIN_NONE (-1)         /* argbest / placement: no feasible worker */
 #define ALADDIN_INVALID (-2)      /* argbest / placement: the candidate is invalid */
 
+/* Decode-SLO constraints of a placement (the flag bits 4 and 8):
+ *   EXACT   every request's remaining decode projected iteration by iteration
+ *           with the candidate added (the stall of this round's prefill
+ *           charged to the requests decoding at round start);
+ *   APPROX  the placement MIP's own constraints (Sec. 4.2): bit 4 is (d), the
+ *           stall within theta * min_j (T_dec * l_out_j - t_dec_j) over the
+ *           requests decoding at round start; bit 8 is (b), sum over the
+ *           worker's requests and the candidate of (l_in + gamma * l_pred)
+ *           within theta * l_d(B) with Eq. input limit l_d(b) = (T_dec /
+ *           lat_scale - c3 - c2 b) / k2 and B the requests with the candidate.
+ * KV (bit 1) and TTFT (bit 2) are the same in both modes. */
+#define ALADDIN_MODE_EXACT 0
+#define ALADDIN_MODE_APPROX 1
+
 /* Performance models and SLOs (Sec. 3, Sec. 4.2).
  *   prefill iteration (Eq. prefill iter time): t_pre = k1 * sum(l_in) + c1
  *   decode iteration  (Eq. iter time):         t_d = k2 * sum(context) + c2 * b + c3
  *   KV usage          (Eq. kv cache):          kv = h * (l_in + l_out) + j
  * Requirements: k1, k2 > 0; c1, c2, c3 >= 0; h >= 1; j >= 0; T_pre > 0;
  * T_dec > c3 (Eq. input limit); 0 < theta <= 1; gamma >= 0; 2 <= K <= 65536;
- * b_cap a power of two in [32, 1024]. */
+ * b_cap a power of two in [32, 1024]; mode one of the two above. */
 typedef struct aladdin_params {
     double k1, c1;       /* prefill: ms per input token, ms */
     double k2, c2, c3;   /* decode: ms per context token, ms per request, ms */
@@ -75,6 +89,7 @@ typedef struct aladdin_params {
     double theta;        /* SLO scaling knob of (b), (d) */
     int32_t K;           /* sequence limit: l_in + l_pred <= K for every request */
     int32_t b_cap;       /* request slots per worker (ongoing + this round's) */
+    int32_t mode;        /* ALADDIN_MODE_EXACT or ALADDIN_MODE_APPROX */
 } aladdin_params;
 
 /* One worker configuration (Sec. 4.1): GPUs per worker, KV capacity in KV

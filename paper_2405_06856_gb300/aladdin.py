@@ -19,6 +19,7 @@ LIB_PATH = os.path.join(_HERE, "_build", "libaladdin.so")
 OK = 0
 ERR_ARG, ERR_CAPACITY, ERR_CUDA, ERR_TIMEOUT, ERR_NOMEM, ERR_STATE = -1, -2, -3, -4, -5, -6
 ERR_SCRATCH = -7
+MODE_EXACT, MODE_APPROX = 0, 1
 NOALLOC_MAX_CAND = 32768
 FLAG_KV, FLAG_TTFT, FLAG_ONGOING, FLAG_NEW, FEASIBLE, FLAG_INVALID = 1, 2, 4, 8, 15, 128
 NONE, INVALID = -1, -2
@@ -45,7 +46,7 @@ class aladdin_params(C.Structure):
     _fields_ = [("k1", C.c_double), ("c1", C.c_double), ("k2", C.c_double), ("c2", C.c_double),
                 ("c3", C.c_double), ("h", C.c_int32), ("j", C.c_int32), ("T_pre", C.c_double),
                 ("T_dec", C.c_double), ("gamma", C.c_double), ("theta", C.c_double),
-                ("K", C.c_int32), ("b_cap", C.c_int32)]
+                ("K", C.c_int32), ("b_cap", C.c_int32), ("mode", C.c_int32)]
 
 
 class aladdin_worker_cfg(C.Structure):
@@ -118,7 +119,7 @@ def make_params(d, b_cap):
     return aladdin_params(float(d["k1"]), float(d["c1"]), float(d["k2"]), float(d["c2"]),
                           float(d["c3"]), int(d["h"]), int(d["j"]), float(d["T_pre"]),
                           float(d["T_dec"]), float(d["gamma"]), float(d["theta"]), int(d["K"]),
-                          int(b_cap))
+                          int(b_cap), int(d.get("mode", MODE_EXACT)))
 
 
 def make_cfgs(gpus, kv_capacity, lat_scale):

@@ -54,6 +54,7 @@ struct DevParams {
     int32_t h, j;
     float T_pre, T_dec, gamma, theta;
     int32_t K, cap;
+    int32_t approx;  // 1: the MIP's constraints (b) and (d) replace the projection
     // derived in double on the host, rounded once
     float c2_over_k2, c3_over_k2, c1_over_k1, inv_k1, theta_Tdec, thTdec_over_k2;
     // double copies for execution (advance) and exact capacity_norm keys
@@ -98,6 +99,8 @@ struct ClusterDev {
     int* novf;                 // their count
     uint32_t* skey;            // [W*cap] (r << 10 | slot) of the requests in sorted order,
                                // written by every table build
+    float2* wapx;              // [W] approximate mode: prompt bounds of (d) and of (b)
+                               // before the candidate's gamma * l_pred
 };
 
 // Table row p of a worker (2 x float4, 32 bytes) and its side entry:
@@ -143,7 +146,8 @@ __device__ __forceinline__ CandRec make_cand(const DevParams& P, int32_t in, int
     c.a = a;
     c.r = rf;
     c.inv_r = 1.0f / rf;
-    c.Ua = (-P.c2_over_k2 - 0.5f * (rf + 1.0f)) - a;
+    // approximate mode: a + gamma * l_pred, the candidate's share of (b)
+    c.Ua = P.approx ? fmaf(P.gamma, rf, a) : (-P.c2_over_k2 - 0.5f * (rf + 1.0f)) - a;
     const float d1 = P.k2 * rf + P.k1;
     c.inv_d1 = 1.0f / d1;
     const float X = P.c2 * rf + P.k2 * (0.5f * rf * (rf + 1.0f));
@@ -177,6 +181,24 @@ __device__ __forceinline__ unsigned eval_pair(const float4 v0, const float4 v1, 
 {
     float d[4];
     pair_headroom(v0, v1, ext, wr, c, d);
+    margin = fminf(fminf(d[0], d[1]), fminf(d[2], d[3]));
+    return (d[0] >= 0.0f ? 1u : 0u) | (d[1] >= 0.0f ? 2u : 0u) | (d[2] >= 0.0f ? 4u : 0u) |
+           (d[3] >= 0.0f ? 8u : 0u);
+}
+
+// eval_pair in either mode; wa = the worker's approximate-mode bounds.
+__device__ __forceinline__ unsigned eval_pair_mode(bool approx, const float4 v0, const float4 v1,
+                                                   const float2 ext, const float4 wr,
+                                                   const float2 wa, const CandRec& c,
+                                                   float& margin)
+{
+    if (!approx) return eval_pair(v0, v1, ext, wr, c, margin);
+    float d[4];
+    const float np1n = fmaf(2.0f, v1.y, -1.0f);
+    d[0] = fminf(v0.y, fmaf(c.r, np1n, v0.z)) - c.a;
+    d[1] = fminf(fmaf(c.Zc, wr.x, -wr.y), wr.z) - c.a;
+    d[2] = wa.x - c.a;
+    d[3] = wa.y - c.Ua;
     margin = fminf(fminf(d[0], d[1]), fminf(d[2], d[3]));
     return (d[0] >= 0.0f ? 1u : 0u) | (d[1] >= 0.0f ? 2u : 0u) | (d[2] >= 0.0f ? 4u : 0u) |
            (d[3] >= 0.0f ? 8u : 0u);
@@ -367,6 +389,7 @@ struct BuildSmem {
     unsigned sorted[NW > 1 ? N : 1];  // cooperative builds: merged keys
     alignas(16) unsigned runs[NW > 1 ? N : 1];  // each warp's keys (read as uint4)
     long long pll[6][NW];             // per-warp partials
+    double pdm[NW];
     float pf[7][NW];
     int pi[3][NW];
     unsigned cflag;
@@ -569,9 +592,8 @@ __device__ unsigned build_table(const DevParams& P, const ClusterDev& C, int w,
             key[e] = ((unsigned)r << 10) | (unsigned)i;
             sm.a[i] = a;
             sm.pend[i] = (uint8_t)pd;
-            sm.bank[i] = pd ? 0.0f
-                            : (float)(P.thetad * P.T_decd * (double)g -
-                                      (PRELOAD ? l_td[e % EL] : C.tdec[slot]));
+            const double td = PRELOAD ? l_td[e % EL] : C.tdec[slot];
+            sm.bank[i] = pd ? 0.0f : (float)(P.thetad * P.T_decd * (double)g - td);
             sumIn += in;
             sumPred += pr;
             if (pd) {
@@ -627,6 +649,35 @@ __device__ unsigned build_table(const DevParams& P, const ClusterDev& C, int w,
             npend += sm.pi[0][k];
             bad |= sm.pi[1][k];
         }
+    }
+    // Approximate mode: prompt bounds of (d) (stall within the smallest
+    // theta-scaled saved decode time) and of (b) (weighted context within
+    // theta * l_d(n + 1), Eq. input limit), in fp64, rounded once.
+    float2 wa = make_float2(0.0f, 0.0f);
+    if (P.approx) {
+        double dmin = __longlong_as_double(0x7ff0000000000000ll);  // +inf: nothing decoding
+#pragma unroll
+        for (int e = 0; e < E; ++e) {
+            const int i = x0 + e * 32 + lane;
+            if (i < n) {  // reloaded: the preloaded registers stay short-lived
+                const long long slot = base + i;
+                if (!C.pend[slot])  // decode time saved so far, theta-scaled
+                    dmin = fmin(dmin, P.thetad * (P.T_decd * (double)C.gen[slot] - C.tdec[slot]));
+            }
+        }
+#pragma unroll
+        for (int d = 16; d > 0; d >>= 1) dmin = fmin(dmin, __shfl_xor_sync(FULL, dmin, d));
+        if constexpr (NW > 1) {
+            if (lane == 0) sm.pdm[q] = dmin;
+            group_sync<NW>();
+#pragma unroll
+            for (int k = 0; k < NW; ++k) dmin = fmin(dmin, sm.pdm[k]);
+        }
+        const double s_d = C.scaled[w];
+        const double tau0 = s_d * (P.k1d * (double)sumP + P.c1d);
+        wa.x = (float)((dmin - tau0) / (s_d * P.k1d));
+        const double ld = (P.T_decd / s_d - P.c3d - P.c2d * (double)(n + 1)) / P.k2d;
+        wa.y = (float)(P.thetad * ld - ((double)sumIn + P.gammad * (double)sumPred));
     }
 
     // capacity_norm key (one lane; code 0 is kept for a worker holding an
@@ -962,7 +1013,7 @@ __device__ unsigned build_table(const DevParams& P, const ClusterDev& C, int w,
                     cache->rho[rowid[e]] = (unsigned short)(nxt - 1);
                 if (want && r[e] <= rc && rc < nxt) {
                     float m;
-                    cf = eval_pair(o.v0, o.v1, o.ext, wr, *cand, m);
+                    cf = eval_pair_mode(P.approx, o.v0, o.v1, o.ext, wr, wa, *cand, m);
                     mine = true;
                 }
             }
@@ -984,10 +1035,11 @@ __device__ unsigned build_table(const DevParams& P, const ClusterDev& C, int w,
         store_row(C, rowbase, o);
         if (want && (bad || n == 0 || rc < r0)) {
             float m;
-            cf = eval_pair(o.v0, o.v1, o.ext, wr, *cand, m);
+            cf = eval_pair_mode(P.approx, o.v0, o.v1, o.ext, wr, wa, *cand, m);
             mine = true;
         }
         C.wrec[w] = wr;
+        if (P.approx) C.wapx[w] = wa;
         C.key[w] = kq;
         if (cache) {
             if (!bad && n > 0 && R > 0) cache->rho[0] = (unsigned short)(r0 - 1);

@@ -88,6 +88,7 @@ int check_params(const aladdin_params* p)
     if (p->K < 2 || p->K > 65536) return ALADDIN_ERR_ARG;
     const int b = p->b_cap;
     if (!(b == 32 || b == 64 || b == 128 || b == 256 || b == 512 || b == 1024)) return ALADDIN_ERR_ARG;
+    if (p->mode != ALADDIN_MODE_EXACT && p->mode != ALADDIN_MODE_APPROX) return ALADDIN_ERR_ARG;
     return ALADDIN_OK;
 }
 
@@ -114,6 +115,7 @@ DevParams make_devparams(const aladdin_params& p)
     d.gamma = (float)p.gamma;
     d.theta = (float)p.theta;
     d.K = p.K;
+    d.approx = p.mode == ALADDIN_MODE_APPROX ? 1 : 0;
     d.cap = p.b_cap;
     d.c2_over_k2 = (float)(p.c2 / p.k2);
     d.c3_over_k2 = (float)(p.c3 / p.k2);
@@ -252,6 +254,7 @@ int cluster_alloc(aladdin_cluster* cl, const aladdin_params& p, int W,
     AL(ovf, int32_t, W);
     AL(novf, int, 1);
     AL(skey, uint32_t, slots);
+    AL(wapx, float2, W);
 #undef AL
     CK(cl->alloc(&p0, sizeof(unsigned long long) * 4)); cl->d_stats = (unsigned long long*)p0;
     CK(cl->alloc(&p0, sizeof(int) * 4)); cl->d_status = (int*)p0;

@@ -70,7 +70,9 @@ __global__ void __launch_bounds__(ROUND_THREADS) k_round(DevParams P, ClusterDev
                 const int p = find_row<false>(C.tab, rb, C.R[w], cr.ri);
                 const float4* t = C.tab + (rb + p) * ROW_F4;
                 float m;
-                const unsigned f = eval_pair(t[0], t[1], C.tab2[rb + p], C.wrec[w], cr, m);
+                const unsigned f =
+                    eval_pair_mode(P.approx != 0, t[0], t[1], C.tab2[rb + p], C.wrec[w],
+                                   P.approx ? C.wapx[w] : make_float2(0.0f, 0.0f), cr, m);
                 if (f == 15u) better(bk, bw, C.key[w], w);
             }
 #pragma unroll
@@ -383,7 +385,9 @@ __global__ void __launch_bounds__(R2_THREADS, 1) k_round2(R2Args A)
                 const long long row = rb + p;
                 const float4* t = C.tab + row * ROW_F4;
                 float m;
-                const unsigned f = eval_pair(t[0], t[1], C.tab2[row], wrec_s[lw], cr, m);
+                const unsigned f =
+                    eval_pair_mode(P.approx != 0, t[0], t[1], C.tab2[row], wrec_s[lw],
+                                   P.approx ? C.wapx[w] : make_float2(0.0f, 0.0f), cr, m);
                 if (f == 15u) better_f(bk, bw, bf, key_s[lw], w, n_s[lw] >= cap);
             }
         }

@@ -86,6 +86,7 @@ struct ScoreArgs {
     float* margin;
     unsigned int* best;
     int tiles, chunks;
+    int approx;  // approximate-mode constraints (b) and (d)
 };
 
 __global__ void k_cand_scatter(DevParams P, int n, int W, const int32_t* __restrict__ in,
@@ -276,7 +277,7 @@ __device__ __forceinline__ void st_out(T* p, T v)
 #endif
 }
 
-template <int SLOTS, bool SF, bool SMG, bool ARG, bool PEND, bool FULLT>
+template <int SLOTS, bool SF, bool SMG, bool ARG, bool PEND, bool FULLT, bool APPROX>
 __global__ void __launch_bounds__(SCORE_WARPS * 32, PEND ? 3 : ALADDIN_SCORE_MINB) k_score(VecArgs A)
 {
     extern __shared__ __align__(16) unsigned char smraw[];
@@ -313,6 +314,7 @@ __global__ void __launch_bounds__(SCORE_WARPS * 32, PEND ? 3 : ALADDIN_SCORE_MIN
     Slot<PEND> ss[SLOTS];
     int p[SLOTS], wk[SLOTS];
     float inv_s[SLOTS], nZO[SLOTS], ZW[SLOTS];
+    float bd[APPROX ? SLOTS : 1], bq[APPROX ? SLOTS : 1];  // approximate-mode bounds
     unsigned rank[SLOTS];
     int nb = 0;  // smallest next breakpoint over this lane's workers
     bool have_rows = false;
@@ -359,6 +361,11 @@ __global__ void __launch_bounds__(SCORE_WARPS * 32, PEND ? 3 : ALADDIN_SCORE_MIN
                     nZO[s] = -wr.y;
                     ZW[s] = wr.z;
                     rank[s] = live ? (unsigned)__float_as_int(wr.w) : 0xffffffffu;
+                    if constexpr (APPROX) {
+                        const float2 wa = __ldg(&A.C.wapx[wk[s]]);
+                        bd[s] = wa.x;
+                        bq[s] = wa.y;
+                    }
                 }
                 nb = ss[0].rnext;
 #pragma unroll
@@ -418,14 +425,21 @@ __global__ void __launch_bounds__(SCORE_WARPS * 32, PEND ? 3 : ALADDIN_SCORE_MIN
                     const Slot<PEND>& t = ss[s];
                     d[0][s] = fminf(t.kvB1, fmaf(r, t.np1n, t.kvE)) - a;
                     const float tt = fmaf(Zc, inv_s[s], nZO[s]);
-                    d[2][s] = fminf(t.pmA, fmaf(t.Gt, id1, nX)) - a;
-                    const float ca = fmaf(t.b0n, ir, fmaf(t.nh, r, Ua - t.b1));
-                    if (PEND) {
-                        d[1][s] = fminf(tt, ZW[s]) - a;
-                        d[3][s] = fminf(fminf(t.pmAp - a, fmaf(t.Gpt, id2, Ua)), ca);
+                    if constexpr (APPROX) {
+                        // (d) and (b) of the placement MIP; Ua holds a + gamma r
+                        d[2][s] = bd[s % (APPROX ? SLOTS : 1)] - a;
+                        d[3][s] = bq[s % (APPROX ? SLOTS : 1)] - Ua;
+                        d[1][s] = (PEND ? fminf(tt, ZW[s]) : tt) - a;
                     } else {
-                        d[1][s] = tt - a;
-                        d[3][s] = ca;
+                        d[2][s] = fminf(t.pmA, fmaf(t.Gt, id1, nX)) - a;
+                        const float ca = fmaf(t.b0n, ir, fmaf(t.nh, r, Ua - t.b1));
+                        if (PEND) {
+                            d[1][s] = fminf(tt, ZW[s]) - a;
+                            d[3][s] = fminf(fminf(t.pmAp - a, fmaf(t.Gpt, id2, Ua)), ca);
+                        } else {
+                            d[1][s] = tt - a;
+                            d[3][s] = ca;
+                        }
                     }
                     m[s] = fminf(fminf(d[0][s], d[1][s]), fminf(d[2][s], d[3][s]));
                     if (ARG) kmin = min(kmin, (__float_as_uint(m[s]) & 0x80000000u) | rank[s]);
@@ -484,6 +498,7 @@ __global__ void __launch_bounds__(SCORE_WARPS * 32) k_score_scalar(ScoreArgs A)
     Row cur = load_row(A.C.tab, rb + p);
     float2 ext = __ldg(&A.C.tab2[rb + p]);
     const float4 wr = __ldg(&A.C.wrec[wc]);
+    const float2 wa = A.approx ? __ldg(&A.C.wapx[wc]) : make_float2(0.0f, 0.0f);
     const unsigned rank = live ? (unsigned)__float_as_int(wr.w) : 0xffffffffu;
     for (int c = c0; c < c1; ++c) {
         const float4* cp = recs + (size_t)c * REC_F4;
@@ -507,7 +522,7 @@ __global__ void __launch_bounds__(SCORE_WARPS * 32) k_score_scalar(ScoreArgs A)
             ext = __ldg(&A.C.tab2[rb + p]);
         }
         float m;
-        const unsigned f = eval_pair(cur.v0, cur.v1, ext, wr, cr, m);
+        const unsigned f = eval_pair_mode(A.approx != 0, cur.v0, cur.v1, ext, wr, wa, cr, m);
         if (live) {
             if (SF) A.flags[off] = (uint8_t)f;
             if (SMG) __stcs(A.margin + off, m);
@@ -520,7 +535,7 @@ __global__ void __launch_bounds__(SCORE_WARPS * 32) k_score_scalar(ScoreArgs A)
     }
 }
 
-template <int SLOTS, bool SF, bool SMG, bool ARG, bool PEND, bool FULLT>
+template <int SLOTS, bool SF, bool SMG, bool ARG, bool PEND, bool FULLT, bool APPROX>
 static cudaError_t launch_vec(const ScoreArgs& A0, cudaStream_t st)
 {
     VecArgs A;
@@ -534,14 +549,14 @@ static cudaError_t launch_vec(const ScoreArgs& A0, cudaStream_t st)
     const size_t smem = sizeof(ScoreSmem);
     static int per_sm = 0, sms = 0;  // occupancy of this instantiation (per process)
     if (per_sm == 0) {
-        cudaError_t e = cudaFuncSetAttribute(k_score<SLOTS, SF, SMG, ARG, PEND, FULLT>,
+        cudaError_t e = cudaFuncSetAttribute(k_score<SLOTS, SF, SMG, ARG, PEND, FULLT, APPROX>,
                                              cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
         if (e != cudaSuccess) return e;
         int dev = 0;
         cudaGetDevice(&dev);
         cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
         int ps = 0;
-        e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&ps, k_score<SLOTS, SF, SMG, ARG, PEND, FULLT>,
+        e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&ps, k_score<SLOTS, SF, SMG, ARG, PEND, FULLT, APPROX>,
                                                           SCORE_WARPS * 32, smem);
         per_sm = (e != cudaSuccess || ps < 1) ? 1 : ps;
     }
@@ -552,30 +567,39 @@ static cudaError_t launch_vec(const ScoreArgs& A0, cudaStream_t st)
     const int max_parts = (A.n_cand + 63) / 64;  // at least 64 candidates per CTA
     if (per_tile > max_parts) per_tile = max_parts;
     A.per_tile = per_tile;
-    k_score<SLOTS, SF, SMG, ARG, PEND, FULLT><<<A.tiles * per_tile, SCORE_WARPS * 32, smem, st>>>(A);
+    k_score<SLOTS, SF, SMG, ARG, PEND, FULLT, APPROX><<<A.tiles * per_tile, SCORE_WARPS * 32, smem, st>>>(A);
     return cudaGetLastError();
 }
 
-template <bool PEND, bool FULLT>
-static cudaError_t dispatch_vec2(bool sf, bool smg, bool arg, const ScoreArgs& A, cudaStream_t st)
+template <bool PEND, bool FULLT, bool APPROX>
+static cudaError_t dispatch_vec3(bool sf, bool smg, bool arg, const ScoreArgs& A, cudaStream_t st)
 {
     constexpr int S = ALADDIN_SCORE_SLOTS;
-    if (sf && smg && arg) return launch_vec<S, true, true, true, PEND, FULLT>(A, st);
-    if (sf && smg) return launch_vec<S, true, true, false, PEND, FULLT>(A, st);
-    if (sf && arg) return launch_vec<S, true, false, true, PEND, FULLT>(A, st);
-    if (smg && arg) return launch_vec<S, false, true, true, PEND, FULLT>(A, st);
-    if (sf) return launch_vec<S, true, false, false, PEND, FULLT>(A, st);
-    if (smg) return launch_vec<S, false, true, false, PEND, FULLT>(A, st);
-    return launch_vec<S, false, false, true, PEND, FULLT>(A, st);
+    if (sf && smg && arg) return launch_vec<S, true, true, true, PEND, FULLT, APPROX>(A, st);
+    if (sf && smg) return launch_vec<S, true, true, false, PEND, FULLT, APPROX>(A, st);
+    if (sf && arg) return launch_vec<S, true, false, true, PEND, FULLT, APPROX>(A, st);
+    if (smg && arg) return launch_vec<S, false, true, true, PEND, FULLT, APPROX>(A, st);
+    if (sf) return launch_vec<S, true, false, false, PEND, FULLT, APPROX>(A, st);
+    if (smg) return launch_vec<S, false, true, false, PEND, FULLT, APPROX>(A, st);
+    return launch_vec<S, false, false, true, PEND, FULLT, APPROX>(A, st);
+}
+
+template <bool PEND, bool FULLT>
+static cudaError_t dispatch_vec2(bool approx, bool sf, bool smg, bool arg, const ScoreArgs& A,
+                                 cudaStream_t st)
+{
+    return approx ? dispatch_vec3<PEND, FULLT, true>(sf, smg, arg, A, st)
+                  : dispatch_vec3<PEND, FULLT, false>(sf, smg, arg, A, st);
 }
 
 template <bool PEND>
-static cudaError_t dispatch_vec(bool sf, bool smg, bool arg, const ScoreArgs& A, cudaStream_t st)
+static cudaError_t dispatch_vec(bool approx, bool sf, bool smg, bool arg, const ScoreArgs& A,
+                                cudaStream_t st)
 {
     // every lane of every CTA tile holds a worker: no per-lane predicate
     const bool full = A.C.W % (SCORE_WARPS * 32 * ALADDIN_SCORE_SLOTS) == 0;
-    return full ? dispatch_vec2<PEND, true>(sf, smg, arg, A, st)
-                : dispatch_vec2<PEND, false>(sf, smg, arg, A, st);
+    return full ? dispatch_vec2<PEND, true>(approx, sf, smg, arg, A, st)
+                : dispatch_vec2<PEND, false>(approx, sf, smg, arg, A, st);
 }
 
 template <bool SF, bool SMG, bool ARG>
@@ -666,12 +690,15 @@ cudaError_t launch_score(const DevParams& P, const ClusterDev& C, int n, const i
         A.best = argbest ? B.best : nullptr;
         A.chunks = (n + SCORE_CHUNK - 1) / SCORE_CHUNK;
         A.tiles = 0;
+        A.approx = P.approx;
         if (ev0) cudaEventRecord(ev0, st);
         const bool vec = (C.W % 4 == 0) && (((uintptr_t)flags & 3) == 0) &&
                          (((uintptr_t)margin & 15) == 0);
         const bool sf = flags != nullptr, smg = margin != nullptr, arg = argbest != nullptr;
         if (vec) {
-            e = pend ? dispatch_vec<true>(sf, smg, arg, A, st) : dispatch_vec<false>(sf, smg, arg, A, st);
+            const bool ap = P.approx != 0;
+            e = pend ? dispatch_vec<true>(ap, sf, smg, arg, A, st)
+                     : dispatch_vec<false>(ap, sf, smg, arg, A, st);
             if (e != cudaSuccess) return e;
         } else {
             if (sf && smg && arg) launch_scalar<true, true, true>(A, st);

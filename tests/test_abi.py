@@ -39,7 +39,7 @@ def test_library_exports_every_declared_symbol(lib):
 
 
 def test_struct_layout(lib):
-    assert ctypes.sizeof(lib.aladdin_params) == 5 * 8 + 2 * 4 + 4 * 8 + 2 * 4
+    assert ctypes.sizeof(lib.aladdin_params) == 5 * 8 + 2 * 4 + 4 * 8 + 3 * 4 + 4  # padded
     assert ctypes.sizeof(lib.aladdin_worker_cfg) == 24
     assert ctypes.sizeof(lib.aladdin_trace) == 32
 
