@@ -58,6 +58,28 @@
  *                the candidate, l_d(b) = (T_dec / scale_i - c3 - c2 b) / k2
  *                (Eq. input limit).
  * KV (e) and TTFT (c) are as in the exact mode.
+ *
+ * Serving setting (phase):
+ *   0 mixed     continuous batching with prefill and decode on the same
+ *               worker (Sec. 5.1, default continuous batching).
+ *   1 decode    split-phase inference (Sec. 5.1): the worker is a decode
+ *               instance; requests arrive with their prompt processed
+ *               elsewhere, so no prefill runs on it. Nothing stalls its
+ *               decoding requests (tau = 0), TTFT (c) is the prefill
+ *               instance's concern and is not tested, and in the approximate
+ *               mode (d) is vacuous. A request arrives holding its prompt's
+ *               KV, as in the mixed setting.
+ * Placement policy (Sec. 6.1 baselines, Sec. 6.4):
+ *   0 best-fit  Algorithm 1 (the feasibility test above, capacity_norm order).
+ *   1 JSQ       join the shortest queue: the worker holding the fewest
+ *               requests, lowest index on ties; no feasibility test.
+ *   2 Po2       power of two choices: two workers drawn uniformly at random
+ *               (SplitMix64, below), the one holding fewer requests, the
+ *               first drawn on ties; no feasibility test.
+ * In the simulation a placement that breaks an SLO shows up when the
+ * workers execute: a realized TTFT above T_pre, a realized ATGT above T_dec
+ * (each beyond a relative 1e-5) or an iteration whose KV exceeds M counts as
+ * a violation and fails the run like an unplaced request.
  */
 #include <math.h>
 #include <stdint.h>
@@ -73,7 +95,14 @@ typedef struct {
     int64_t K;            /* sequence limit (input + output tokens) */
     int64_t mode;         /* 0: exact decode projection; 1: approximate
                              constraints (b) and (d) of the MIP (Sec. 4.2) */
+    int64_t phase;        /* 0: mixed prefill + decode; 1: decode instance */
+    int64_t policy;       /* 0: best-fit; 1: JSQ; 2: power of two choices */
+    uint64_t seed;        /* SplitMix64 seed of the power-of-two draws */
 } orc_params;
+
+/* Relative slack of a realized latency over its SLO before it counts as a
+ * violation (the rounding of the fp32 placement test). */
+#define ORC_SLO_TOL 1e-5
 
 /* Cluster state in fixed-stride slots: worker w owns slots
  * [w*cap, w*cap + n[w]). */
@@ -249,24 +278,29 @@ static void eval_pair(const orc_params* p, const orc_cluster* cl, int w, const o
     double P = 0.0;
     for (int q = 0; q < cl->n[w]; ++q)
         if (cl->pend[base + q]) P += (double)cl->in[base + q];
-    const double tau0 = sc * (p->k1 * P + p->c1);
-    const double tau1 = sc * p->k1;
+    /* A decode instance runs no prefill: no stall and no TTFT test. */
+    const int decode = p->phase == 1;
+    const double tau0 = decode ? 0.0 : sc * (p->k1 * P + p->c1);
+    const double tau1 = decode ? 0.0 : sc * p->k1;
     const double tau_a = tau0 + tau1 * a;
     const double off = cl->off ? cl->off[w] : 0.0;
 
     /* (c) TTFT of the candidate and of this round's earlier placements. */
-    lat_constraint(&A, 1, p->T_pre - w_c - off - tau0, tau1, p->T_pre + w_c + off + tau_a, a);
-    for (int q = 0; q < cl->n[w]; ++q) {
-        int64_t slot = base + q;
-        if (!cl->pend[slot]) continue;
-        double wq = cl->wait[slot];
-        lat_constraint(&A, 1, p->T_pre - wq - off - tau0, tau1, p->T_pre + wq + off + tau_a, a);
+    if (!decode) {
+        lat_constraint(&A, 1, p->T_pre - w_c - off - tau0, tau1, p->T_pre + w_c + off + tau_a, a);
+        for (int q = 0; q < cl->n[w]; ++q) {
+            int64_t slot = base + q;
+            if (!cl->pend[slot]) continue;
+            double wq = cl->wait[slot];
+            lat_constraint(&A, 1, p->T_pre - wq - off - tau0, tau1, p->T_pre + wq + off + tau_a,
+                           a);
+        }
     }
 
     if (p->mode == 1) {
         /* (d) as stated: the stall within theta times the smallest decode time
-         * an ongoing request has saved so far. */
-        for (int q = 0; q < cl->n[w]; ++q) {
+         * an ongoing request has saved so far (vacuous without a prefill). */
+        for (int q = 0; q < cl->n[w] && !decode; ++q) {
             int64_t slot = base + q;
             if (cl->pend[slot]) continue;
             double g = (double)cl->gen[slot];
@@ -494,16 +528,96 @@ int32_t orc_kv_curve(const orc_params* p, const orc_cluster* cl, int w, int32_t 
 }
 
 /* ---------------------------------------------------------------------- */
-/* One greedy placement round (Algorithm 1), candidates in index (arrival)
- * order: each goes to the first feasible worker in capacity_norm order of the
- * current state and becomes a pending request there (gen = 0, prefill at the
- * worker's next iteration). placement[c] = worker, or -1 if no worker is
- * feasible (the cluster is fixed; nothing is opened). */
+/* SplitMix64 (G. Steele, D. Lea, C. Flood, "Fast splittable pseudorandom
+ * number generators", OOPSLA 2014): the n-th output (n = 1, 2, ...) of the
+ * stream seeded with s is mix(s + n * 0x9E3779B97F4A7C15), all mod 2^64. */
+uint64_t orc_splitmix64(uint64_t s, uint64_t n)
+{
+    uint64_t z = s + n * 0x9E3779B97F4A7C15ull;
+    z = (z ^ (z >> 30)) * 0xBF58476D1CE4E5B9ull;
+    z = (z ^ (z >> 27)) * 0x94D049BB133111EBull;
+    return z ^ (z >> 31);
+}
+
+/* Draw k (0 or 1) of the power-of-two choice for request id rid: output
+ * 2 rid + k + 1 of the seeded stream, mapped to [0, W) by its upper 32 bits
+ * times W over 2^32. */
+int32_t orc_po2_draw(uint64_t seed, int64_t rid, int k, int32_t W)
+{
+    uint64_t x = orc_splitmix64(seed, 2ull * (uint64_t)rid + (uint64_t)k + 1ull);
+    return (int32_t)(((x >> 32) * (uint64_t)W) >> 32);
+}
+
+/* The worker a load-balancing policy picks (JSQ or power of two choices). */
+static int pick_by_queue(const orc_params* p, const orc_cluster* cl, int64_t rid)
+{
+    if (p->policy == 1) {
+        int best = 0;
+        for (int w = 1; w < cl->W; ++w)
+            if (cl->n[w] < cl->n[best]) best = w;
+        return best;
+    }
+    int w1 = orc_po2_draw(p->seed, rid, 0, cl->W);
+    int w2 = orc_po2_draw(p->seed, rid, 1, cl->W);
+    return cl->n[w2] < cl->n[w1] ? w2 : w1;
+}
+
+/* ---------------------------------------------------------------------- */
+/* One placement round, candidates in index (arrival) order. Best-fit
+ * (Algorithm 1): each goes to the first feasible worker in capacity_norm
+ * order of the current state. JSQ / power of two: each goes to the worker the
+ * policy picks, feasible or not. The request becomes a pending request there
+ * (gen = 0, prefill at the worker's next iteration). placement[c] = worker,
+ * or -1 if no worker is feasible (best-fit; the cluster is fixed, nothing is
+ * opened). A chosen worker without a free slot is ORC_ERR_CAPACITY, or, with
+ * refuse_full (simulation of JSQ / power of two), placement -3 and the round
+ * goes on. The power-of-two draws use crid[c] (c if crid is NULL). */
+static int place_round_impl(const orc_params* p, orc_cluster* cl, int32_t C, const int32_t* cin,
+                            const int32_t* cpred, const double* cwait, const int64_t* crid,
+                            int32_t* placement, int refuse_full);
+
 int orc_place_round(const orc_params* p, orc_cluster* cl, int32_t C, const int32_t* cin,
                     const int32_t* cpred, const double* cwait, const int64_t* crid,
                     int32_t* placement)
 {
+    return place_round_impl(p, cl, C, cin, cpred, cwait, crid, placement, 0);
+}
+
+static void append_request(orc_cluster* cl, int w, int32_t a, int32_t r, double wait, int64_t rid)
+{
+    int64_t slot = (int64_t)w * cl->cap + cl->n[w];
+    cl->in[slot] = a;
+    cl->gen[slot] = 0;
+    cl->pred[slot] = r;
+    if (cl->tdec) cl->tdec[slot] = 0.0;
+    cl->pend[slot] = 1;
+    cl->wait[slot] = wait;
+    if (cl->rid) cl->rid[slot] = rid;
+    cl->n[w] += 1;
+}
+
+static int place_round_impl(const orc_params* p, orc_cluster* cl, int32_t C, const int32_t* cin,
+                            const int32_t* cpred, const double* cwait, const int64_t* crid,
+                            int32_t* placement, int refuse_full)
+{
     const int W = cl->W;
+    if (p->policy != 0) {
+        for (int32_t c = 0; c < C; ++c) {
+            int64_t rid = crid ? crid[c] : c;
+            int w = pick_by_queue(p, cl, rid);
+            if (cl->n[w] >= cl->cap) {
+                if (!refuse_full) {
+                    for (int32_t k = c; k < C; ++k) placement[k] = -1;
+                    return ORC_ERR_CAPACITY;
+                }
+                placement[c] = -3;
+                continue;
+            }
+            append_request(cl, w, cin[c], cpred[c], cwait ? cwait[c] : 0.0, rid);
+            placement[c] = w;
+        }
+        return ORC_OK;
+    }
     int32_t S = (int32_t)p->K + 2;
     double* T0 = (double*)malloc(sizeof(double) * ((size_t)S + 2));
     double* T1 = (double*)malloc(sizeof(double) * ((size_t)S + 2));
@@ -525,15 +639,7 @@ int orc_place_round(const orc_params* p, orc_cluster* cl, int32_t C, const int32
             eval_pair(p, cl, w, &fut[w], T0, T1, cin[c], cpred[c], cwait ? cwait[c] : 0.0, &r);
             if (r.flags != 15) continue;
             if (cl->n[w] >= cl->cap) { rc = ORC_ERR_CAPACITY; break; }
-            int64_t slot = (int64_t)w * cl->cap + cl->n[w];
-            cl->in[slot] = cin[c];
-            cl->gen[slot] = 0;
-            cl->pred[slot] = cpred[c];
-            if (cl->tdec) cl->tdec[slot] = 0.0;
-            cl->pend[slot] = 1;
-            cl->wait[slot] = cwait ? cwait[c] : 0.0;
-            if (cl->rid) cl->rid[slot] = crid ? crid[c] : c;
-            cl->n[w] += 1;
+            append_request(cl, w, cin[c], cpred[c], cwait ? cwait[c] : 0.0, crid ? crid[c] : c);
             future_free(&fut[w]);
             have[w] = 0;
             placement[c] = w;
@@ -557,13 +663,19 @@ int orc_place_round(const orc_params* p, orc_cluster* cl, int32_t C, const int32
  * decoding requests), then decode iterations back to back while they start
  * before t_now + dt. Finished requests leave; their realized TTFT and ATGT
  * (decode time / decode tokens, Sec. 2.2) are appended to the record arrays
- * (rec_* may be NULL; *nrec counts). Afterwards off[w] is the time from
+ * (rec_* may be NULL; *nrec counts). On a decode instance (phase 1) the
+ * round's placements join the batch at the boundary without a prefill and
+ * record no TTFT. viol (nullable, 3 counters) accumulates the realized
+ * violations: [0] TTFT above T_pre, [1] ATGT above T_dec (each beyond the
+ * relative ORC_SLO_TOL), [2] decode iterations whose KV usage
+ * h * context + j * batch exceeds M. Afterwards off[w] is the time from
  * t_now + dt to the worker's next iteration start. */
 int orc_advance(const orc_params* p, orc_cluster* cl, double t_now, double dt,
                 int64_t* rec_rid, double* rec_val, uint8_t* rec_kind, int64_t* nrec,
-                int64_t rec_cap)
+                int64_t rec_cap, int64_t* viol)
 {
     const double t_end = t_now + dt;
+    const int decode = p->phase == 1;
     for (int w = 0; w < cl->W; ++w) {
         const double sc = cl->scale[w];
         const int64_t base = (int64_t)w * cl->cap;
@@ -572,17 +684,27 @@ int orc_advance(const orc_params* p, orc_cluster* cl, double t_now, double dt,
         int any = 0;
         for (int q = 0; q < cl->n[w]; ++q)
             if (cl->pend[base + q]) { P += (double)cl->in[base + q]; any = 1; }
-        if (any) {
+        if (any && decode) {
+            for (int q = 0; q < cl->n[w]; ++q) {
+                int64_t slot = base + q;
+                if (!cl->pend[slot]) continue;
+                cl->pend[slot] = 0;
+                cl->gen[slot] = 0;
+                cl->tdec[slot] = 0.0;
+            }
+        } else if (any) {
             double tau = sc * (p->k1 * P + p->c1);
             for (int q = 0; q < cl->n[w]; ++q) {
                 int64_t slot = base + q;
                 if (cl->pend[slot]) {
+                    double ttft = cl->wait[slot] + (start - t_now) + tau;
                     if (rec_rid && *nrec < rec_cap) {
                         rec_rid[*nrec] = cl->rid ? cl->rid[slot] : slot;
-                        rec_val[*nrec] = cl->wait[slot] + (start - t_now) + tau;
+                        rec_val[*nrec] = ttft;
                         rec_kind[*nrec] = 0;
                     }
                     *nrec += 1;
+                    if (viol && ttft > p->T_pre * (1.0 + ORC_SLO_TOL)) viol[0] += 1;
                     cl->pend[slot] = 0;
                     cl->gen[slot] = 0;
                     cl->tdec[slot] = 0.0;
@@ -595,6 +717,7 @@ int orc_advance(const orc_params* p, orc_cluster* cl, double t_now, double dt,
         while (cl->n[w] > 0 && start < t_end) {
             int64_t b = cl->n[w], K = 0;
             for (int q = 0; q < cl->n[w]; ++q) K += context(cl, base + q) + 1;
+            if (viol && p->h * K + p->j * b > cl->M[w]) viol[2] += 1;
             double t = sc * (p->c3 + p->c2 * (double)b + p->k2 * (double)K);
             for (int q = 0; q < cl->n[w]; ++q) {
                 cl->gen[base + q] += 1;
@@ -605,12 +728,14 @@ int orc_advance(const orc_params* p, orc_cluster* cl, double t_now, double dt,
             for (int q = 0; q < cl->n[w];) {
                 int64_t slot = base + q;
                 if (cl->gen[slot] >= cl->pred[slot]) {
+                    double atgt = cl->tdec[slot] / (double)cl->pred[slot];
                     if (rec_rid && *nrec < rec_cap) {
                         rec_rid[*nrec] = cl->rid ? cl->rid[slot] : slot;
-                        rec_val[*nrec] = cl->tdec[slot] / (double)cl->pred[slot];
+                        rec_val[*nrec] = atgt;
                         rec_kind[*nrec] = 1;
                     }
                     *nrec += 1;
+                    if (viol && atgt > p->T_dec * (1.0 + ORC_SLO_TOL)) viol[1] += 1;
                     int64_t last = base + cl->n[w] - 1;
                     cl->in[slot] = cl->in[last];
                     cl->gen[slot] = cl->gen[last];
@@ -637,11 +762,17 @@ int orc_advance(const orc_params* p, orc_cluster* cl, double t_now, double dt,
  * yet placed form one placement round in arrival order, then every worker
  * executes until the next heartbeat. A request still unplaced whose wait at
  * the next heartbeat plus its prefill alone would exceed T_pre can no longer
- * meet its TTFT: it is counted as failed and dropped. If drain is set the
- * simulation continues without arrivals until every worker is empty, so that
- * every admitted request's realized TTFT and ATGT are recorded.
+ * meet its TTFT: it is counted as failed and dropped. On a decode instance
+ * (phase 1) nothing absorbs a wait, so a request not placed at the first
+ * heartbeat after its arrival fails (Algorithm 1 would have opened a worker
+ * for it). JSQ and power of two place every request at once; one whose
+ * worker has no free slot fails. Every realized violation (see orc_advance)
+ * also counts as a failure. If drain is set the simulation continues without
+ * arrivals until every worker is empty, so that every admitted request's
+ * realized TTFT and ATGT are recorded.
  * out[0] failed, out[1] placed, out[2] heartbeats, out[3] max realized TTFT,
- * out[4] max realized ATGT, out[5] realized records. */
+ * out[4] max realized ATGT, out[5] realized records, out[6] realized
+ * violations (included in out[0]). */
 int orc_simulate(const orc_params* p, int32_t N, int32_t cap, int64_t M, double scale,
                  int64_t R, const double* t_arr, const int32_t* rin, const int32_t* rpred,
                  double H, int32_t stop_at_fail, int32_t drain, double* out)
@@ -679,7 +810,7 @@ int orc_simulate(const orc_params* p, int32_t N, int32_t cap, int64_t M, double 
     cl.M = Mv;
     cl.scale = sv;
 
-    int64_t next = 0, nwait = 0, failed = 0, placed = 0, hb = 0, nrec = 0;
+    int64_t next = 0, nwait = 0, failed = 0, placed = 0, hb = 0, nrec = 0, violations = 0;
     double max_ttft = 0.0, max_atgt = 0.0;
     int rc = ORC_OK;
     for (;;) {
@@ -691,20 +822,23 @@ int orc_simulate(const orc_params* p, int32_t N, int32_t cap, int64_t M, double 
                 cpr[i] = rpred[wl[i]];
                 cw[i] = t - t_arr[wl[i]];
             }
-            rc = orc_place_round(p, &cl, (int32_t)nwait, cin, cpr, cw, wl, pl);
+            rc = place_round_impl(p, &cl, (int32_t)nwait, cin, cpr, cw, wl, pl, 1);
             if (rc != ORC_OK) break;
             int64_t keep = 0;
             for (int64_t i = 0; i < nwait; ++i) {
                 if (pl[i] >= 0) { placed++; continue; }
                 double tau_alone = scale * (p->k1 * (double)cin[i] + p->c1);
-                if (cw[i] + H + tau_alone > p->T_pre) failed++;
+                if (pl[i] == -3 || p->phase == 1 || cw[i] + H + tau_alone > p->T_pre) failed++;
                 else wl[keep++] = wl[i];
             }
             nwait = keep;
         }
         if (failed > 0 && stop_at_fail) break;
         int64_t nr0 = nrec;
-        orc_advance(p, &cl, t, H, rr, rv, rk, &nrec, rec_cap);
+        int64_t vv[3] = {0, 0, 0};
+        orc_advance(p, &cl, t, H, rr, rv, rk, &nrec, rec_cap, vv);
+        violations += vv[0] + vv[1] + vv[2];
+        failed += vv[0] + vv[1] + vv[2];
         for (int64_t i = nr0; i < nrec && i < rec_cap; ++i) {
             if (rk[i] == 0 && rv[i] > max_ttft) max_ttft = rv[i];
             if (rk[i] == 1 && rv[i] > max_atgt) max_atgt = rv[i];
@@ -724,6 +858,7 @@ int orc_simulate(const orc_params* p, int32_t N, int32_t cap, int64_t M, double 
     out[3] = max_ttft;
     out[4] = max_atgt;
     out[5] = (double)nrec;
+    out[6] = (double)violations;
     free(Mv); free(sv); free(cl.off); free(cl.clock); free(cl.n); free(cl.in); free(cl.gen);
     free(cl.pred); free(cl.tdec); free(cl.pend); free(cl.wait); free(cl.rid);
     free(wl); free(cin); free(cpr); free(cw); free(pl); free(rr); free(rv); free(rk);
@@ -733,18 +868,22 @@ int orc_simulate(const orc_params* p, int32_t N, int32_t cap, int64_t M, double 
 /* Minimum-worker search (Sec. 4.1, Sec. 6.4): for each worker configuration
  * (GPUs per worker, KV capacity, latency scale) the smallest worker count N in
  * [1, n_max] that serves the whole trace with no failed request, found by
- * doubling then bisection. n_out[o] = -1 if even n_max fails. */
+ * doubling then bisection. n_out[o] = -1 if even n_max fails. JSQ and power
+ * of two admit without a test, so their runs drain the workers to see every
+ * request's realized latencies; best-fit's admitted requests meet them by
+ * construction. */
 int orc_min_workers(const orc_params* p, int32_t n_opt, const int32_t* gpus, const int64_t* M,
                     const double* scale, int32_t cap, int64_t R, const double* t_arr,
                     const int32_t* rin, const int32_t* rpred, double H, int32_t n_max,
                     int32_t* n_out)
 {
-    double out[6];
+    double out[7];
+    const int32_t drain = p->policy != 0;
     for (int o = 0; o < n_opt; ++o) {
         int32_t lo = 0, hi = 1; /* lo fails (or is 0), hi to be tested */
         int found = 0;
         while (hi <= n_max) {
-            int rc = orc_simulate(p, hi, cap, M[o], scale[o], R, t_arr, rin, rpred, H, 1, 0, out);
+            int rc = orc_simulate(p, hi, cap, M[o], scale[o], R, t_arr, rin, rpred, H, 1, drain, out);
             if (rc != ORC_OK) return rc;
             if (out[0] == 0.0) { found = 1; break; }
             lo = hi;
@@ -753,7 +892,8 @@ int orc_min_workers(const orc_params* p, int32_t n_opt, const int32_t* gpus, con
         if (!found) { n_out[o] = -1; continue; }
         while (hi - lo > 1) {
             int32_t mid = lo + (hi - lo) / 2;
-            int rc = orc_simulate(p, mid, cap, M[o], scale[o], R, t_arr, rin, rpred, H, 1, 0, out);
+            int rc = orc_simulate(p, mid, cap, M[o], scale[o], R, t_arr, rin, rpred, H, 1, drain,
+                                  out);
             if (rc != ORC_OK) return rc;
             if (out[0] == 0.0) hi = mid;
             else lo = mid;

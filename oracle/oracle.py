@@ -17,6 +17,8 @@ LIB = os.path.join(HERE, "_build", "liboracle.so")
 
 FLAG_KV, FLAG_TTFT, FLAG_ONGOING, FLAG_NEW = 1, 2, 4, 8
 FEASIBLE = 15
+PHASE_MIXED, PHASE_DECODE = 0, 1
+POLICY_BESTFIT, POLICY_JSQ, POLICY_PO2 = 0, 1, 2
 
 
 def build(force=False):
@@ -37,7 +39,8 @@ class Params(C.Structure):
                 ("c2", C.c_double), ("c3", C.c_double), ("h", C.c_int64),
                 ("j", C.c_int64), ("T_pre", C.c_double), ("T_dec", C.c_double),
                 ("gamma", C.c_double), ("theta", C.c_double), ("K", C.c_int64),
-                ("mode", C.c_int64)]
+                ("mode", C.c_int64), ("phase", C.c_int64), ("policy", C.c_int64),
+                ("seed", C.c_uint64)]
 
 
 class ClusterStruct(C.Structure):
@@ -61,7 +64,11 @@ def lib():
         _lib.orc_kv_curve.argtypes = [P, P, C.c_int, C.c_int32, C.c_int32, P]
         _lib.orc_kv_curve.restype = C.c_int32
         _lib.orc_place_round.argtypes = [P, P, C.c_int32, P, P, P, P, P]
-        _lib.orc_advance.argtypes = [P, P, C.c_double, C.c_double, P, P, P, P, C.c_int64]
+        _lib.orc_advance.argtypes = [P, P, C.c_double, C.c_double, P, P, P, P, C.c_int64, P]
+        _lib.orc_splitmix64.argtypes = [C.c_uint64, C.c_uint64]
+        _lib.orc_splitmix64.restype = C.c_uint64
+        _lib.orc_po2_draw.argtypes = [C.c_uint64, C.c_int64, C.c_int, C.c_int32]
+        _lib.orc_po2_draw.restype = C.c_int32
         _lib.orc_simulate.argtypes = [P, C.c_int32, C.c_int32, C.c_int64, C.c_double, C.c_int64,
                                       P, P, P, C.c_double, C.c_int32, C.c_int32, P]
         _lib.orc_min_workers.argtypes = [P, C.c_int32, P, P, P, C.c_int32, C.c_int64, P, P, P,
@@ -76,7 +83,8 @@ def make_params(d):
     return Params(float(d["k1"]), float(d["c1"]), float(d["k2"]), float(d["c2"]),
                   float(d["c3"]), int(d["h"]), int(d["j"]), float(d["T_pre"]),
                   float(d["T_dec"]), float(d["gamma"]), float(d["theta"]), int(d["K"]),
-                  int(d.get("mode", 0)))
+                  int(d.get("mode", 0)), int(d.get("phase", 0)), int(d.get("policy", 0)),
+                  int(d.get("seed", 0)) & 0xFFFFFFFFFFFFFFFF)
 
 
 def _ptr(a):
@@ -225,7 +233,10 @@ class Cluster:
         self.rid[slot] = rid
         self.n[w] += 1
 
-    def advance(self, t_now, dt, rec_cap=1 << 16):
+    def advance(self, t_now, dt, rec_cap=1 << 16, violations=None):
+        """Execute every worker for dt ms; returns the realized records (request
+        id, value, kind 0 TTFT / 1 ATGT). ``violations`` (int64[3], optional)
+        accumulates realized TTFT, ATGT and KV-overflow violations."""
         rr = np.zeros(rec_cap, np.int64)
         rv = np.zeros(rec_cap)
         rk = np.zeros(rec_cap, np.uint8)
@@ -233,7 +244,8 @@ class Cluster:
         st = self.struct(with_tdec=True)
         self.has_tdec = True
         rc = lib().orc_advance(C.byref(self._p), C.byref(st), float(t_now), float(dt),
-                               _ptr(rr), _ptr(rv), _ptr(rk), C.byref(nrec), rec_cap)
+                               _ptr(rr), _ptr(rv), _ptr(rk), C.byref(nrec), rec_cap,
+                               _ptr(violations))
         if rc != 0:
             raise RuntimeError("orc_advance failed")
         k = min(nrec.value, rec_cap)
@@ -246,8 +258,18 @@ class Cluster:
                 self.pend[s:s + k].copy())
 
 
+def splitmix64(seed, n):
+    """Output n (n >= 1) of the SplitMix64 stream seeded with ``seed``."""
+    return int(lib().orc_splitmix64(int(seed) & 0xFFFFFFFFFFFFFFFF, int(n)))
+
+
+def po2_draw(seed, rid, k, W):
+    """Worker of draw k (0 or 1) of the power-of-two choice for request rid."""
+    return int(lib().orc_po2_draw(int(seed) & 0xFFFFFFFFFFFFFFFF, int(rid), int(k), int(W)))
+
+
 def simulate(params, N, cap, M, scale, trace, H, stop_at_fail=True, drain=False):
-    out = np.zeros(6)
+    out = np.zeros(7)
     p = make_params(params)
     t = np.ascontiguousarray(trace.t_arr, np.float64)
     ri = np.ascontiguousarray(trace.req_in, np.int32)
@@ -260,7 +282,7 @@ def simulate(params, N, cap, M, scale, trace, H, stop_at_fail=True, drain=False)
     if rc != 0:
         raise RuntimeError("orc_simulate failed: %d" % rc)
     return dict(failed=int(out[0]), placed=int(out[1]), heartbeats=int(out[2]),
-                max_ttft=out[3], max_atgt=out[4])
+                max_ttft=out[3], max_atgt=out[4], violations=int(out[6]))
 
 
 def min_workers(params, gpus, M, scale, cap, trace, H, n_max):
