@@ -72,13 +72,47 @@ extern "C" {
 #define ALADDIN_MODE_EXACT 0
 #define ALADDIN_MODE_APPROX 1
 
+/* Serving setting of the workers (Sec. 5.1):
+ *   MIXED   default continuous batching: prefill and decode on the same
+ *           worker; a round's prefill stalls the worker's decoding requests.
+ *   DECODE  split-phase inference: the workers are decode instances and a
+ *           request arrives with its prompt processed by a prefill instance
+ *           (its prompt's KV cache comes with it). No prefill runs on the
+ *           worker, so nothing is stalled (tau = 0 in (d) and in the exact
+ *           projection) and TTFT (c) is not tested: flag bit 2 is always set
+ *           and (d) of the approximate mode is vacuous (bit 4 set). In the
+ *           simulation a request that no worker takes at the first heartbeat
+ *           after its arrival fails (nothing absorbs a wait). */
+#define ALADDIN_PHASE_MIXED 0
+#define ALADDIN_PHASE_DECODE 1
+
+/* Placement policy of aladdin_place_round, aladdin_simulate and
+ * aladdin_min_workers (Sec. 6.1 baselines, Sec. 6.4); scoring is the same
+ * under every policy.
+ *   BESTFIT  Algorithm 1: the feasible worker of largest capacity_norm.
+ *   JSQ      join the shortest queue: the worker holding the fewest requests,
+ *            lowest index on ties, without a feasibility test.
+ *   PO2      power of two choices: two workers drawn uniformly at random, the
+ *            one holding fewer requests (the first drawn on ties), without a
+ *            feasibility test. Draw k (0, 1) of request id q is output
+ *            2 q + k + 1 of the SplitMix64 stream seeded with params.seed
+ *            (Steele, Lea, Flood, OOPSLA 2014), mapped to a worker as
+ *            (upper 32 bits x W) >> 32. Request ids are trace indices in the
+ *            simulation and, in aladdin_place_round, the count of candidates
+ *            the cluster was given in earlier rounds plus the index in the
+ *            call. */
+#define ALADDIN_POLICY_BESTFIT 0
+#define ALADDIN_POLICY_JSQ 1
+#define ALADDIN_POLICY_PO2 2
+
 /* Performance models and SLOs (Sec. 3, Sec. 4.2).
  *   prefill iteration (Eq. prefill iter time): t_pre = k1 * sum(l_in) + c1
  *   decode iteration  (Eq. iter time):         t_d = k2 * sum(context) + c2 * b + c3
  *   KV usage          (Eq. kv cache):          kv = h * (l_in + l_out) + j
  * Requirements: k1, k2 > 0; c1, c2, c3 >= 0; h >= 1; j >= 0; T_pre > 0;
  * T_dec > c3 (Eq. input limit); 0 < theta <= 1; gamma >= 0; 2 <= K <= 65536;
- * b_cap a power of two in [32, 1024]; mode one of the two above. */
+ * b_cap a power of two in [32, 1024]; mode, phase and policy one of the
+ * values above. */
 typedef struct aladdin_params {
     double k1, c1;       /* prefill: ms per input token, ms */
     double k2, c2, c3;   /* decode: ms per context token, ms per request, ms */
@@ -90,6 +124,9 @@ typedef struct aladdin_params {
     int32_t K;           /* sequence limit: l_in + l_pred <= K for every request */
     int32_t b_cap;       /* request slots per worker (ongoing + this round's) */
     int32_t mode;        /* ALADDIN_MODE_EXACT or ALADDIN_MODE_APPROX */
+    int32_t phase;       /* ALADDIN_PHASE_MIXED or ALADDIN_PHASE_DECODE */
+    int32_t policy;      /* ALADDIN_POLICY_BESTFIT, _JSQ or _PO2 */
+    uint64_t seed;       /* SplitMix64 seed of the power-of-two draws */
 } aladdin_params;
 
 /* One worker configuration (Sec. 4.1): GPUs per worker, KV capacity in KV
@@ -179,24 +216,31 @@ int aladdin_score_noalloc(aladdin_cluster* cl, int32_t n_cand, const int32_t* in
                           const int32_t* pred, const float* wait_ms, uint8_t* flags,
                           float* margin, int32_t* argbest);
 
-/* One greedy best-fit round (Algorithm 1): candidates in index order, each
- * placed on the feasible worker of largest capacity_norm in the state left by
- * the earlier placements, where it becomes a request of this round (prefill
- * pending, gen = 0). placement[c] = worker, ALADDIN_NONE if none is feasible
- * (the cluster is fixed: no worker is opened), ALADDIN_INVALID for an invalid
- * candidate. Returns ALADDIN_ERR_CAPACITY if a chosen worker has no free slot
- * (placements up to that candidate are kept). */
+/* One placement round: candidates in index order, each placed in the state
+ * left by the earlier placements, where it becomes a request of this round
+ * (prefill pending, gen = 0). With ALADDIN_POLICY_BESTFIT (Algorithm 1) the
+ * worker is the feasible one of largest capacity_norm; with JSQ or PO2 it is
+ * the policy's choice, feasible or not. placement[c] = worker, ALADDIN_NONE
+ * if no worker is feasible (best-fit; the cluster is fixed: no worker is
+ * opened), ALADDIN_INVALID for an invalid candidate. Returns
+ * ALADDIN_ERR_CAPACITY if a chosen worker has no free slot (placements up to
+ * that candidate are kept, the later ones are ALADDIN_NONE). */
 int aladdin_place_round(aladdin_cluster* cl, int32_t n_cand, const int32_t* in,
                         const int32_t* pred, const float* wait_ms, int32_t* placement);
 
 /* Execute every worker for dt_ms from the cluster clock (continuous batching,
  * Sec. 2.1): at its next iteration boundary a worker runs the prefill of this
- * round's placements (stalling its decoding requests), then decode iterations
- * back to back while they start before clock + dt_ms; finished requests leave.
- * The clock then advances by dt_ms and a new round begins.
- * stats (nullable, host, 4 doubles) accumulates since creation:
- * [0] requests whose prefill ran, [1] requests finished,
- * [2] largest realized TTFT (ms), [3] largest realized ATGT (ms per token). */
+ * round's placements (stalling its decoding requests; on a decode instance
+ * they join the batch without one), then decode iterations back to back
+ * while they start before clock + dt_ms; finished requests leave. The clock
+ * then advances by dt_ms and a new round begins.
+ * stats (nullable, host, 7 doubles) accumulates since creation:
+ * [0] requests whose prefill ran (joined the batch, on a decode instance),
+ * [1] requests finished, [2] largest realized TTFT (ms; mixed setting only),
+ * [3] largest realized ATGT (ms per token), and the realized violations:
+ * [4] TTFTs above T_pre, [5] ATGTs above T_dec (each beyond a relative 1e-5,
+ * the rounding of the fp32 placement test), [6] decode iterations whose KV
+ * usage h * context + j * batch exceeded the worker's capacity. */
 int aladdin_cluster_advance(aladdin_cluster* cl, double dt_ms, double* stats);
 
 /* Copy the cluster state to host arrays (each nullable): n[W] requests per
@@ -231,25 +275,34 @@ typedef struct aladdin_trace {
 
 /* Minimum-worker search (Sec. 4.1, Sec. 6.4): for every worker configuration
  * options[o], the smallest number of identical workers in [1, n_max] that
- * serves the whole trace with every request placed within its TTFT (heartbeat
- * every heartbeat_ms; at each, the waiting arrivals form one placement round,
- * then the workers execute until the next heartbeat; a request that can no
- * longer meet T_pre on an empty worker fails). Found by doubling then
- * bisection; each simulation runs on the GPU. n_workers[o] = -1 if n_max
- * workers fail. best_option (nullable) receives the option with the fewest
- * total GPUs (gpus * n_workers; first on ties), total_gpus (nullable) that
- * total. Trace arrays are host memory. */
+ * serves the whole trace with no failed request under params.policy and
+ * params.phase (see aladdin_simulate; heartbeat every heartbeat_ms). Found by
+ * doubling then bisection; each simulation runs on the GPU. JSQ and PO2
+ * admit without a test, so their simulations drain the workers after the
+ * last arrival to realize every request's latencies; best-fit's admissions
+ * meet them by construction. n_workers[o] = -1 if n_max workers fail.
+ * best_option (nullable) receives the option with the fewest total GPUs
+ * (gpus * n_workers; first on ties), total_gpus (nullable) that total. Trace
+ * arrays are host memory. */
 int aladdin_min_workers(const aladdin_params* params, int32_t n_options,
                         const aladdin_worker_cfg* options, const aladdin_trace* trace,
                         double heartbeat_ms, int32_t n_max, void* cuda_stream,
                         int32_t* n_workers, int32_t* best_option, int64_t* total_gpus);
 
 /* Simulate the trace on n identical workers of configuration cfg (the check
- * inside aladdin_min_workers). out (host, 5 doubles): [0] failed requests,
- * [1] placed requests, [2] heartbeats run, [3] largest realized TTFT,
- * [4] largest realized ATGT. With stop_at_fail the simulation ends at the
- * first failure; with drain it continues after the last arrival until every
- * worker is idle. */
+ * inside aladdin_min_workers). At every heartbeat the arrivals so far that
+ * are not placed form one placement round (params.policy), then the workers
+ * execute until the next heartbeat. A request fails when it can no longer be
+ * placed in time: best-fit in the mixed setting keeps an unplaced request
+ * waiting while its wait at the next heartbeat plus its prefill alone stay
+ * within T_pre; on a decode instance it fails at its first heartbeat; JSQ and
+ * PO2 place every request at once and one whose worker has no free slot
+ * fails. Every realized violation (aladdin_cluster_advance stats [4]-[6])
+ * counts as a failure too. out (host, 6 doubles): [0] failures, [1] placed
+ * requests, [2] heartbeats run, [3] largest realized TTFT, [4] largest
+ * realized ATGT, [5] realized violations (included in [0]). With
+ * stop_at_fail the simulation ends at the heartbeat after the first failure;
+ * with drain it continues after the last arrival until every worker is idle. */
 int aladdin_simulate(const aladdin_params* params, const aladdin_worker_cfg* cfg, int32_t n,
                      const aladdin_trace* trace, double heartbeat_ms, int32_t stop_at_fail,
                      int32_t drain, void* cuda_stream, double* out);

@@ -20,6 +20,10 @@ OK = 0
 ERR_ARG, ERR_CAPACITY, ERR_CUDA, ERR_TIMEOUT, ERR_NOMEM, ERR_STATE = -1, -2, -3, -4, -5, -6
 ERR_SCRATCH = -7
 MODE_EXACT, MODE_APPROX = 0, 1
+PHASE_MIXED, PHASE_DECODE = 0, 1
+POLICY_BESTFIT, POLICY_JSQ, POLICY_PO2 = 0, 1, 2
+ADVANCE_STATS = 7     # doubles written by aladdin_cluster_advance
+SIMULATE_OUT = 6      # doubles written by aladdin_simulate
 NOALLOC_MAX_CAND = 32768
 FLAG_KV, FLAG_TTFT, FLAG_ONGOING, FLAG_NEW, FEASIBLE, FLAG_INVALID = 1, 2, 4, 8, 15, 128
 NONE, INVALID = -1, -2
@@ -46,7 +50,8 @@ class aladdin_params(C.Structure):
     _fields_ = [("k1", C.c_double), ("c1", C.c_double), ("k2", C.c_double), ("c2", C.c_double),
                 ("c3", C.c_double), ("h", C.c_int32), ("j", C.c_int32), ("T_pre", C.c_double),
                 ("T_dec", C.c_double), ("gamma", C.c_double), ("theta", C.c_double),
-                ("K", C.c_int32), ("b_cap", C.c_int32), ("mode", C.c_int32)]
+                ("K", C.c_int32), ("b_cap", C.c_int32), ("mode", C.c_int32),
+                ("phase", C.c_int32), ("policy", C.c_int32), ("seed", C.c_uint64)]
 
 
 class aladdin_worker_cfg(C.Structure):
@@ -119,7 +124,9 @@ def make_params(d, b_cap):
     return aladdin_params(float(d["k1"]), float(d["c1"]), float(d["k2"]), float(d["c2"]),
                           float(d["c3"]), int(d["h"]), int(d["j"]), float(d["T_pre"]),
                           float(d["T_dec"]), float(d["gamma"]), float(d["theta"]), int(d["K"]),
-                          int(b_cap), int(d.get("mode", MODE_EXACT)))
+                          int(b_cap), int(d.get("mode", MODE_EXACT)),
+                          int(d.get("phase", PHASE_MIXED)), int(d.get("policy", POLICY_BESTFIT)),
+                          int(d.get("seed", 0)) & 0xFFFFFFFFFFFFFFFF)
 
 
 def make_cfgs(gpus, kv_capacity, lat_scale):
@@ -292,7 +299,7 @@ class Cluster:
         return pl
 
     def advance(self, dt_ms):
-        st = np.zeros(4)
+        st = np.zeros(ADVANCE_STATS)
         aladdin_cluster_advance(self.handle, dt_ms, st)
         return st
 

@@ -4,7 +4,13 @@
 // requests), then decode iterations back to back (Eq. iter time) while they
 // start before t_now + dt. Each iteration adds one token to every active
 // request; requests that reach their predicted length leave and their
-// realized ATGT (decode time over decode tokens, Sec. 2.2) is recorded.
+// realized ATGT (decode time over decode tokens, Sec. 2.2) is recorded. On a
+// decode instance (split-phase inference) the round's placements join the
+// batch at the boundary with no prefill and no TTFT. Realized violations are
+// counted: TTFT above T_pre, ATGT above T_dec (each beyond SLO_TOL) and
+// decode iterations whose KV usage h * context + j * batch exceeds the
+// worker's capacity M (what a placement without a feasibility test, JSQ or
+// power of two, can cause).
 // Times accumulate in fp64 with explicitly rounded operations, in the same
 // order as the CPU reference, so both sides produce the same schedule.
 #include "aladdin_host.h"
@@ -21,7 +27,7 @@ __device__ __forceinline__ void atomic_max_nonneg(unsigned long long* addr, doub
 template <int E>
 __global__ void __launch_bounds__(ADV_WARPS * 32)
 k_advance(DevParams P, ClusterDev C, double t_now, double dt, unsigned long long* stats,
-          const int* halt)
+          const int* halt, unsigned long long* fail)
 {
     if (halt && *halt != 0) return;
     const int lane = threadIdx.x & 31;
@@ -38,7 +44,8 @@ k_advance(DevParams P, ClusterDev C, double t_now, double dt, unsigned long long
     long long Pint = 0;
     int npend = 0;
     double maxttft = 0.0, maxatgt = 0.0;
-    unsigned long long nfin = 0;
+    unsigned long long nfin = 0, vttft = 0, vatgt = 0, vkv = 0;
+    const long long Mw = C.M[w];
     double start = C.clock[w] > t_now ? C.clock[w] : t_now;
 #pragma unroll
     for (int e = 0; e < E; ++e) {
@@ -61,7 +68,17 @@ k_advance(DevParams P, ClusterDev C, double t_now, double dt, unsigned long long
     }
     Pint = warp_reduce(Pint, OpAdd<long long>());
     npend = warp_reduce(npend, OpAdd<int>());
-    if (npend > 0) {
+    if (npend > 0 && P.decode) {
+        // decode instance: the placements join the batch, nothing is stalled
+#pragma unroll
+        for (int e = 0; e < E; ++e) {
+            if (!alive[e]) continue;
+            if (C.pend[base + e * 32 + lane]) {
+                gen[e] = 0;
+                tdec[e] = 0.0;
+            }
+        }
+    } else if (npend > 0) {
         const double tau = __dmul_rn(s, __dadd_rn(__dmul_rn(P.k1d, (double)Pint), P.c1d));
         const double lead = __dsub_rn(start, t_now);
 #pragma unroll
@@ -71,6 +88,7 @@ k_advance(DevParams P, ClusterDev C, double t_now, double dt, unsigned long long
             if (C.pend[slot]) {
                 const double ttft = __dadd_rn(__dadd_rn(C.wait[slot], lead), tau);
                 maxttft = fmax(maxttft, ttft);
+                vttft += ttft > P.T_pre_viol ? 1 : 0;
                 gen[e] = 0;
                 tdec[e] = 0.0;
             } else {
@@ -93,6 +111,7 @@ k_advance(DevParams P, ClusterDev C, double t_now, double dt, unsigned long long
         b = warp_reduce(b, OpAdd<int>());
         K = warp_reduce(K, OpAdd<long long>());
         if (b == 0 || !(start < t_end)) break;
+        vkv += (long long)P.h * K + (long long)P.j * b > Mw ? 1 : 0;
         const double t = __dmul_rn(
             s, __dadd_rn(__dadd_rn(P.c3d, __dmul_rn(P.c2d, (double)b)), __dmul_rn(P.k2d, (double)K)));
 #pragma unroll
@@ -101,7 +120,9 @@ k_advance(DevParams P, ClusterDev C, double t_now, double dt, unsigned long long
                 gen[e] += 1;
                 tdec[e] = __dadd_rn(tdec[e], t);
                 if (gen[e] >= pred[e]) {
-                    maxatgt = fmax(maxatgt, __ddiv_rn(tdec[e], (double)pred[e]));
+                    const double atgt = __ddiv_rn(tdec[e], (double)pred[e]);
+                    maxatgt = fmax(maxatgt, atgt);
+                    vatgt += atgt > P.T_dec_viol ? 1 : 0;
                     nfin += 1;
                     alive[e] = false;
                 }
@@ -134,6 +155,8 @@ k_advance(DevParams P, ClusterDev C, double t_now, double dt, unsigned long long
     maxttft = warp_reduce(maxttft, OpMax<double>());
     maxatgt = warp_reduce(maxatgt, OpMax<double>());
     nfin = warp_reduce(nfin, OpAdd<unsigned long long>());
+    vttft = warp_reduce(vttft, OpAdd<unsigned long long>());
+    vatgt = warp_reduce(vatgt, OpAdd<unsigned long long>());
     if (lane == 0) {
         C.n[w] = pos;
         C.clock[w] = start;
@@ -141,31 +164,38 @@ k_advance(DevParams P, ClusterDev C, double t_now, double dt, unsigned long long
         if (stats) {
             if (npend) atomicAdd(&stats[0], (unsigned long long)npend);
             if (nfin) atomicAdd(&stats[1], nfin);
-            if (npend) atomic_max_nonneg(&stats[2], maxttft);
+            if (npend && !P.decode) atomic_max_nonneg(&stats[2], maxttft);
             if (nfin) atomic_max_nonneg(&stats[3], maxatgt);
+            if (vttft) atomicAdd(&stats[4], vttft);
+            if (vatgt) atomicAdd(&stats[5], vatgt);
+            if (vkv) atomicAdd(&stats[6], vkv);
         }
+        const unsigned long long v = vttft + vatgt + vkv;
+        if (fail && v) atomicAdd(fail, v);
     }
 }
 
 template <int E>
 static cudaError_t advance_e(const DevParams& P, const ClusterDev& C, double t_now, double dt,
-                             unsigned long long* stats, const int* halt, cudaStream_t st)
+                             unsigned long long* stats, const int* halt, unsigned long long* fail,
+                             cudaStream_t st)
 {
     const int blocks = (C.W + ADV_WARPS - 1) / ADV_WARPS;
-    k_advance<E><<<blocks, ADV_WARPS * 32, 0, st>>>(P, C, t_now, dt, stats, halt);
+    k_advance<E><<<blocks, ADV_WARPS * 32, 0, st>>>(P, C, t_now, dt, stats, halt, fail);
     return cudaGetLastError();
 }
 
 cudaError_t launch_advance(const DevParams& P, const ClusterDev& C, double t_now, double dt,
-                           unsigned long long* stats, const int* halt, cudaStream_t st)
+                           unsigned long long* stats, const int* halt, cudaStream_t st,
+                           unsigned long long* fail)
 {
     switch (lanes_per_worker(C.cap)) {
-    case 1: return advance_e<1>(P, C, t_now, dt, stats, halt, st);
-    case 2: return advance_e<2>(P, C, t_now, dt, stats, halt, st);
-    case 4: return advance_e<4>(P, C, t_now, dt, stats, halt, st);
-    case 8: return advance_e<8>(P, C, t_now, dt, stats, halt, st);
-    case 16: return advance_e<16>(P, C, t_now, dt, stats, halt, st);
-    case 32: return advance_e<32>(P, C, t_now, dt, stats, halt, st);
+    case 1: return advance_e<1>(P, C, t_now, dt, stats, halt, fail, st);
+    case 2: return advance_e<2>(P, C, t_now, dt, stats, halt, fail, st);
+    case 4: return advance_e<4>(P, C, t_now, dt, stats, halt, fail, st);
+    case 8: return advance_e<8>(P, C, t_now, dt, stats, halt, fail, st);
+    case 16: return advance_e<16>(P, C, t_now, dt, stats, halt, fail, st);
+    case 32: return advance_e<32>(P, C, t_now, dt, stats, halt, fail, st);
     default: return cudaErrorInvalidValue;
     }
 }

@@ -59,7 +59,16 @@ struct DevParams {
     float c2_over_k2, c3_over_k2, c1_over_k1, inv_k1, theta_Tdec, thTdec_over_k2;
     // double copies for execution (advance) and exact capacity_norm keys
     double k1d, c1d, k2d, c2d, c3d, T_pred, T_decd, gammad, thetad;
+    // realized latencies above these count as SLO violations (execution)
+    double T_pre_viol, T_dec_viol;
+    int32_t decode;          // 1: decode instance of split-phase inference (no prefill)
+    int32_t policy;          // ALADDIN_POLICY_* of placement rounds
+    unsigned long long seed; // SplitMix64 seed of the power-of-two draws
 };
+
+// Relative slack of a realized latency over its SLO before the execution step
+// counts it as a violation: the rounding of the fp32 placement test.
+constexpr double SLO_TOL = 1e-5;
 
 // Exact integer aggregates of one table row (verification outputs only).
 struct __align__(16) AuxRow {
@@ -153,7 +162,8 @@ __device__ __forceinline__ CandRec make_cand(const DevParams& P, int32_t in, int
     const float X = P.c2 * rf + P.k2 * (0.5f * rf * (rf + 1.0f));
     c.nXd1 = -X * c.inv_d1;
     c.inv_d2 = 1.0f / (P.k2 * rf);
-    c.Zc = (P.T_pre - (ok ? w : 0.0f)) * P.inv_k1;
+    // decode instance: no TTFT test (the bound is +inf for every worker)
+    c.Zc = P.decode ? f_inf() : (P.T_pre - (ok ? w : 0.0f)) * P.inv_k1;
     c.ri = ok ? r : 0;
     c.orig = orig;
     c.valid = ok ? 1 : 0;
@@ -674,8 +684,12 @@ __device__ unsigned build_table(const DevParams& P, const ClusterDev& C, int w,
             for (int k = 0; k < NW; ++k) dmin = fmin(dmin, sm.pdm[k]);
         }
         const double s_d = C.scaled[w];
-        const double tau0 = s_d * (P.k1d * (double)sumP + P.c1d);
-        wa.x = (float)((dmin - tau0) / (s_d * P.k1d));
+        if (P.decode) {
+            wa.x = f_inf();  // no prefill, no stall: (d) is vacuous
+        } else {
+            const double tau0 = s_d * (P.k1d * (double)sumP + P.c1d);
+            wa.x = (float)((dmin - tau0) / (s_d * P.k1d));
+        }
         const double ld = (P.T_decd / s_d - P.c3d - P.c2d * (double)(n + 1)) / P.k2d;
         wa.y = (float)(P.thetad * ld - ((double)sumIn + P.gammad * (double)sumPred));
     }
@@ -988,9 +1002,12 @@ __device__ unsigned build_table(const DevParams& P, const ClusterDev& C, int w,
     // Worker record (every lane; the first lane stores it).
     float4 wr;
     wr.x = inv_s;
-    wr.y = off * inv_s * P.inv_k1 + P.c1_over_k1 + (float)sumP;
-    wr.z = npend > 0 ? (P.T_pre - wpmax - off) * inv_s * P.inv_k1 - P.c1_over_k1 - (float)sumP
-                     : f_inf();
+    // TTFT bounds (the candidate's Zc is +inf on a decode instance, and so is
+    // its bound Zc / s - wr.y)
+    wr.y = P.decode ? 0.0f : off * inv_s * P.inv_k1 + P.c1_over_k1 + (float)sumP;
+    wr.z = (npend > 0 && !P.decode)
+               ? (P.T_pre - wpmax - off) * inv_s * P.inv_k1 - P.c1_over_k1 - (float)sumP
+               : f_inf();
     wr.w = rank_bits;
     const bool want = cand != nullptr && cand->valid;
     const int rc = want ? cand->ri : 0;

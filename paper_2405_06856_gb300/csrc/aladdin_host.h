@@ -54,6 +54,8 @@ struct RoundIO {
     // exchange buffer of the sliced round (ROUND_XBUF_BYTES), or nullptr to
     // use the single-CTA round
     void* xbuf;
+    // power-of-two draws: request id of direct-mode candidate c is rid0 + c
+    long long rid0;
 };
 constexpr int ROUND_XBUF_SMS = 1024;  // largest SM count the exchange buffer serves
 constexpr size_t ROUND_XBUF_BYTES = 32 * (size_t)ROUND_XBUF_SMS + 16;
@@ -62,10 +64,20 @@ cudaError_t launch_round(const DevParams& P, const ClusterDev& C, const RoundIO&
 
 // Execution of every worker for dt ms from t_now.
 // stats: device [0] prefills run, [1] finished, [2] max TTFT bits, [3] max
-// ATGT bits (non-negative doubles compare like their bit patterns). halt
-// (device, nullable): nothing runs when *halt != 0.
+// ATGT bits (non-negative doubles compare like their bit patterns), realized
+// violations [4] TTFT, [5] ATGT, [6] KV-overflow iterations. halt (device,
+// nullable): nothing runs when *halt != 0. fail (device, nullable): every
+// violation is also added to it (the simulation's failure counter).
+constexpr int STATS_N = 7;
 cudaError_t launch_advance(const DevParams& P, const ClusterDev& C, double t_now, double dt,
-                           unsigned long long* stats, const int* halt, cudaStream_t st);
+                           unsigned long long* stats, const int* halt, cudaStream_t st,
+                           unsigned long long* fail = nullptr);
+
+// One round of a load-balancing policy (JSQ or power of two choices; the
+// RoundIO of launch_round): each candidate goes to the policy's worker
+// without a feasibility test. Tables are not rebuilt.
+cudaError_t launch_round_queue(const DevParams& P, const ClusterDev& C, const RoundIO& io,
+                               cudaStream_t st);
 
 // What another translation unit may read of a cluster (see cluster_view).
 struct ClusterView {

@@ -89,6 +89,10 @@ int check_params(const aladdin_params* p)
     const int b = p->b_cap;
     if (!(b == 32 || b == 64 || b == 128 || b == 256 || b == 512 || b == 1024)) return ALADDIN_ERR_ARG;
     if (p->mode != ALADDIN_MODE_EXACT && p->mode != ALADDIN_MODE_APPROX) return ALADDIN_ERR_ARG;
+    if (p->phase != ALADDIN_PHASE_MIXED && p->phase != ALADDIN_PHASE_DECODE) return ALADDIN_ERR_ARG;
+    if (p->policy != ALADDIN_POLICY_BESTFIT && p->policy != ALADDIN_POLICY_JSQ &&
+        p->policy != ALADDIN_POLICY_PO2)
+        return ALADDIN_ERR_ARG;
     return ALADDIN_OK;
 }
 
@@ -103,8 +107,14 @@ int check_cfg(const aladdin_worker_cfg& c)
 DevParams make_devparams(const aladdin_params& p)
 {
     DevParams d;
-    d.k1 = (float)p.k1;
-    d.c1 = (float)p.c1;
+    // A decode instance runs no prefill: its cost, and so every stall term,
+    // is zero (the TTFT terms are switched off by d.decode).
+    const bool dec = p.phase == ALADDIN_PHASE_DECODE;
+    d.decode = dec ? 1 : 0;
+    d.policy = p.policy;
+    d.seed = (unsigned long long)p.seed;
+    d.k1 = dec ? 0.0f : (float)p.k1;
+    d.c1 = dec ? 0.0f : (float)p.c1;
     d.k2 = (float)p.k2;
     d.c2 = (float)p.c2;
     d.c3 = (float)p.c3;
@@ -119,12 +129,12 @@ DevParams make_devparams(const aladdin_params& p)
     d.cap = p.b_cap;
     d.c2_over_k2 = (float)(p.c2 / p.k2);
     d.c3_over_k2 = (float)(p.c3 / p.k2);
-    d.c1_over_k1 = (float)(p.c1 / p.k1);
-    d.inv_k1 = (float)(1.0 / p.k1);
+    d.c1_over_k1 = dec ? 0.0f : (float)(p.c1 / p.k1);
+    d.inv_k1 = dec ? 0.0f : (float)(1.0 / p.k1);
     d.theta_Tdec = (float)(p.theta * p.T_dec);
     d.thTdec_over_k2 = (float)(p.theta * p.T_dec / p.k2);
-    d.k1d = p.k1;
-    d.c1d = p.c1;
+    d.k1d = dec ? 0.0 : p.k1;
+    d.c1d = dec ? 0.0 : p.c1;
     d.k2d = p.k2;
     d.c2d = p.c2;
     d.c3d = p.c3;
@@ -132,6 +142,8 @@ DevParams make_devparams(const aladdin_params& p)
     d.T_decd = p.T_dec;
     d.gammad = p.gamma;
     d.thetad = p.theta;
+    d.T_pre_viol = p.T_pre * (1.0 + SLO_TOL);
+    d.T_dec_viol = p.T_dec * (1.0 + SLO_TOL);
     return d;
 }
 
@@ -146,6 +158,7 @@ struct aladdin_cluster {
     int W = 0, cap = 0, rows = 0;
     double t_now = 0.0;
     bool round_open = false;  // some worker holds requests placed in the open round
+    long long rid_next = 0;   // request id of the next power-of-two draw (place_round)
     std::vector<void*> owned;
     // scratch and staging (grow-only)
     DevBuf sorted, hist, best;
@@ -256,7 +269,8 @@ int cluster_alloc(aladdin_cluster* cl, const aladdin_params& p, int W,
     AL(skey, uint32_t, slots);
     AL(wapx, float2, W);
 #undef AL
-    CK(cl->alloc(&p0, sizeof(unsigned long long) * 4)); cl->d_stats = (unsigned long long*)p0;
+    CK(cl->alloc(&p0, sizeof(unsigned long long) * STATS_N));
+    cl->d_stats = (unsigned long long*)p0;
     CK(cl->alloc(&p0, sizeof(int) * 4)); cl->d_status = (int*)p0;
     CK(cl->alloc(&p0, ROUND_XBUF_BYTES)); cl->d_xround = p0;
 
@@ -277,7 +291,7 @@ int cluster_alloc(aladdin_cluster* cl, const aladdin_params& p, int W,
     CK(cudaMemsetAsync(d.pend, 0, slots, st));
     CK(cudaMemsetAsync(d.wrec, 0, sizeof(float4) * W, st));
     CK(cudaMemsetAsync(d.err, 0, sizeof(unsigned int), st));
-    CK(cudaMemsetAsync(cl->d_stats, 0, sizeof(unsigned long long) * 4, st));
+    CK(cudaMemsetAsync(cl->d_stats, 0, sizeof(unsigned long long) * STATS_N, st));
     CK(cudaMemsetAsync(cl->d_status, 0, sizeof(int) * 4, st));
     // host vectors above must outlive the async copies
     CK(cudaStreamSynchronize(st));
@@ -604,8 +618,18 @@ int aladdin_place_round(aladdin_cluster* cl, int32_t n_cand, const int32_t* in,
     io.sim = 0;
     io.status = cl->d_status;
     io.xbuf = cl->d_xround;
-    CK(launch_round(cl->dp, cl->dev, io, cl->st));
-    CK(launch_rank(cl->dev, cl->st));
+    io.rid0 = cl->rid_next;
+    if (cl->hp.policy == ALADDIN_POLICY_BESTFIT) {
+        CK(launch_round(cl->dp, cl->dev, io, cl->st));
+        CK(launch_rank(cl->dev, cl->st));
+    } else {
+        // JSQ / power of two: no table is read while placing; every worker's
+        // table is rebuilt afterwards for the scoring calls that follow
+        CK(launch_round_queue(cl->dp, cl->dev, io, cl->st));
+        int trc = refresh_tables(cl);
+        if (trc) return trc;
+    }
+    cl->rid_next += n_cand;
     cl->round_open = true;
     if (hp) CK(cudaMemcpyAsync(placement, dpl, sizeof(int32_t) * C, cudaMemcpyDeviceToHost, cl->st));
     int status = 0;
@@ -625,7 +649,7 @@ int aladdin_cluster_advance(aladdin_cluster* cl, double dt_ms, double* stats)
     int rc = refresh_tables(cl);
     if (rc) return rc;
     if (stats) {
-        unsigned long long s[4];
+        unsigned long long s[STATS_N];
         CK(cudaMemcpyAsync(s, cl->d_stats, sizeof(s), cudaMemcpyDeviceToHost, cl->st));
         CK(cudaStreamSynchronize(cl->st));
         stats[0] = (double)s[0];
@@ -635,6 +659,7 @@ int aladdin_cluster_advance(aladdin_cluster* cl, double dt_ms, double* stats)
         std::memcpy(&b, &s[3], 8);
         stats[2] = a;
         stats[3] = b;
+        for (int k = 4; k < STATS_N; ++k) stats[k] = (double)s[k];
     }
     return ALADDIN_OK;
 }
@@ -755,7 +780,7 @@ __global__ void k_busy(const int32_t* __restrict__ n, int W, int* out)
     if (threadIdx.x == 0) *out = any;
 }
 
-// One simulation; out[0..4] as aladdin_simulate.
+// One simulation; out[0..5] as aladdin_simulate.
 int simulate_impl(const aladdin_params& p, const aladdin_worker_cfg& cfg, int32_t N,
                   const DevTrace& tr, double H, bool stop_at_fail, bool drain, cudaStream_t st,
                   double* out)
@@ -799,10 +824,14 @@ int simulate_impl(const aladdin_params& p, const aladdin_worker_cfg& cfg, int32_
         io.stop_at_fail = stop_at_fail ? 1 : 0;
         io.hb = hb;
         io.xbuf = cl.d_xround;
-        CK(launch_round(cl.dp, cl.dev, io, st));
+        const bool bestfit = p.policy == ALADDIN_POLICY_BESTFIT;
+        if (bestfit) CK(launch_round(cl.dp, cl.dev, io, st));
+        else CK(launch_round_queue(cl.dp, cl.dev, io, st));
         next = end;
-        CK(launch_advance(cl.dp, cl.dev, t, H, cl.d_stats, cl.d_status, st));
-        CK(launch_build(cl.dp, cl.dev, nullptr, cl.W, st));
+        // realized violations count as failures (counters[0])
+        CK(launch_advance(cl.dp, cl.dev, t, H, cl.d_stats, cl.d_status, st, counters));
+        // JSQ and power of two read no table
+        if (bestfit) CK(launch_build(cl.dp, cl.dev, nullptr, cl.W, st));
         hb++;
         const bool tail = next >= tr.n;
         if (tail || (hb & 31) == 0) {
@@ -822,7 +851,7 @@ int simulate_impl(const aladdin_params& p, const aladdin_worker_cfg& cfg, int32_
             if (tail && hs[0] == 0 && (!drain || hs[1] == 0)) break;
         }
     }
-    unsigned long long s[4];
+    unsigned long long s[STATS_N];
     CK(cudaMemcpyAsync(s, cl.d_stats, sizeof(s), cudaMemcpyDeviceToHost, st));
     CK(cudaMemcpyAsync(hc, counters, sizeof(hc), cudaMemcpyDeviceToHost, st));
     CK(cudaStreamSynchronize(st));
@@ -831,6 +860,7 @@ int simulate_impl(const aladdin_params& p, const aladdin_worker_cfg& cfg, int32_
     out[2] = halted ? (double)hc[2] : (double)hb;
     std::memcpy(&out[3], &s[2], 8);
     std::memcpy(&out[4], &s[3], 8);
+    out[5] = (double)(s[4] + s[5] + s[6]);
     wl.release();
     cnt.release();
     return ALADDIN_OK;
@@ -870,12 +900,15 @@ int aladdin_min_workers(const aladdin_params* params, int32_t n_options,
     cudaStream_t st = (cudaStream_t)cuda_stream;
     DevTrace tr;
     if ((rc = upload_trace(*params, trace, tr, st))) return rc;
-    double out[5];
+    double out[6];
+    // JSQ and power of two admit without a test: drain to realize every
+    // request's latencies
+    const bool drain = params->policy != ALADDIN_POLICY_BESTFIT;
     for (int o = 0; o < n_options; ++o) {
         int32_t lo = 0, hi = 1;
         bool found = false;
         while (hi <= n_max) {
-            if ((rc = simulate_impl(*params, options[o], hi, tr, heartbeat_ms, true, false, st, out)))
+            if ((rc = simulate_impl(*params, options[o], hi, tr, heartbeat_ms, true, drain, st, out)))
                 return rc;
             if (out[0] == 0.0) {
                 found = true;
@@ -890,7 +923,8 @@ int aladdin_min_workers(const aladdin_params* params, int32_t n_options,
         }
         while (hi - lo > 1) {
             const int32_t mid = lo + (hi - lo) / 2;
-            if ((rc = simulate_impl(*params, options[o], mid, tr, heartbeat_ms, true, false, st, out)))
+            if ((rc = simulate_impl(*params, options[o], mid, tr, heartbeat_ms, true, drain, st,
+                                    out)))
                 return rc;
             if (out[0] == 0.0) hi = mid;
             else lo = mid;

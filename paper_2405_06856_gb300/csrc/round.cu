@@ -8,7 +8,8 @@
 // worker and rebuilds only that worker's table and key before the next
 // candidate. In trace mode (fleet simulation) the candidates are the waiting
 // requests followed by the heartbeat's arrivals; unplaced requests that can
-// still meet their TTFT stay in the waiting list, the others fail.
+// still meet their TTFT stay in the waiting list, the others fail (on a
+// decode instance every unplaced request fails).
 #include "aladdin_host.h"
 
 namespace aladdin {
@@ -130,7 +131,9 @@ __global__ void __launch_bounds__(ROUND_THREADS) k_round(DevParams P, ClusterDev
                 io.counters[1] += 1;
             } else {
                 const double tau_alone = C.scaled[0] * (P.k1d * (double)a + P.c1d);
-                if (winner == -2 || wd + io.H + tau_alone > P.T_pred) io.counters[0] += 1;
+                // a decode instance has no TTFT budget to absorb a wait
+                if (winner == -2 || P.decode || wd + io.H + tau_alone > P.T_pred)
+                    io.counters[0] += 1;
                 else io.wl[keep++] = tix;
             }
         }
@@ -478,7 +481,9 @@ __global__ void __launch_bounds__(R2_THREADS, 1) k_round2(R2Args A)
                 io.counters[1] += 1;
             } else {
                 const double tau_alone = C.scaled[0] * (P.k1d * (double)a + P.c1d);
-                if (winner == -2 || wd + io.H + tau_alone > P.T_pred) io.counters[0] += 1;
+                // a decode instance has no TTFT budget to absorb a wait
+                if (winner == -2 || P.decode || wd + io.H + tau_alone > P.T_pred)
+                    io.counters[0] += 1;
                 else io.wl[keep++] = tix;
             }
         }

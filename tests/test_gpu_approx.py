@@ -108,7 +108,7 @@ def test_approx_round_and_simulation(A, orc, synth):
     p = dict(synth.BASE_PARAMS, T_dec=30.0, theta=0.9, mode=1)
     for N in (3, 6):
         ref = orc.simulate(p, N, 256, 65536, 1.0, tr, 100.0, stop_at_fail=False, drain=True)
-        out = np.zeros(5)
+        out = np.zeros(A.SIMULATE_OUT)
         A.aladdin_simulate(A.make_params(p, 256), A.make_cfgs([1], [65536], [1.0])[0], N,
                            A.make_trace(tr.t_arr, tr.req_in, tr.req_pred), 100.0, 0, 1, out)
         assert int(out[0]) == ref["failed"] and int(out[1]) == ref["placed"], (N, out, ref)

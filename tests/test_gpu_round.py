@@ -117,7 +117,7 @@ def test_simulate_matches_oracle(A, orc, synth):
     p = dict(synth.BASE_PARAMS)
     for N in (2, 4, 6):
         ref = orc.simulate(p, N, 256, 65536, 1.0, tr, 100.0, stop_at_fail=False, drain=True)
-        out = np.zeros(5)
+        out = np.zeros(A.SIMULATE_OUT)
         A.aladdin_simulate(A.make_params(p, 256), A.make_cfgs([1], [65536], [1.0])[0], N,
                            A.make_trace(tr.t_arr, tr.req_in, tr.req_pred), 100.0, 0, 1, out)
         assert int(out[0]) == ref["failed"] and int(out[1]) == ref["placed"], (N, out, ref)
@@ -130,7 +130,7 @@ def test_simulate_stop_at_fail(A, orc, synth):
     tr = synth.diurnal_trace(8, 500, 60.0, 15.0)
     p = dict(synth.BASE_PARAMS, T_dec=30.0)
     ref = orc.simulate(p, 1, 256, 32768, 1.0, tr, 100.0, stop_at_fail=True)
-    out = np.zeros(5)
+    out = np.zeros(A.SIMULATE_OUT)
     A.aladdin_simulate(A.make_params(p, 256), A.make_cfgs([1], [32768], [1.0])[0], 1,
                        A.make_trace(tr.t_arr, tr.req_in, tr.req_pred), 100.0, 1, 0, out)
     assert ref["failed"] > 0
@@ -178,7 +178,7 @@ def test_simulate_many_slices(A, orc, synth):
     tr = synth.diurnal_trace(11, 6000, 3000.0, 500.0)
     p = dict(synth.BASE_PARAMS, T_pre=100.0, T_dec=14.0)
     ref = orc.simulate(p, 450, 512, 12000, 1.0, tr, 100.0, stop_at_fail=False, drain=True)
-    out = np.zeros(5)
+    out = np.zeros(A.SIMULATE_OUT)
     A.aladdin_simulate(A.make_params(p, 512), A.make_cfgs([1], [12000], [1.0])[0], 450,
                        A.make_trace(tr.t_arr, tr.req_in, tr.req_pred), 100.0, 0, 1, out)
     assert ref["failed"] > 0
