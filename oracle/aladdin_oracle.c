@@ -903,3 +903,105 @@ int orc_min_workers(const orc_params* p, int32_t n_opt, const int32_t* gpus, con
     }
     return ORC_OK;
 }
+
+/* ---------------------------------------------------------------------- */
+/* Worker configuration (Sec. 4.1) and the worker-count model (Sec. 5.2).  */
+
+/* Worker configurations from the tensor-parallel model of Sec. 4.1 for
+ * N_g GPUs per worker: KV capacity M = N_g m_gpu - m_model, and the latency
+ * multiplier of the decode model, the iteration time t_compute + t_comm with
+ * t_compute = k4 / N_g + c4 (Eq. TP compute) and t_comm = kc (N_g - 1) / N_g
+ * (the all-reduce overhead), relative to one GPU (k4 + c4). */
+void orc_tp_config(double k4, double c4, double kc, double m_gpu, double m_model, int32_t g,
+                   double* M, double* scale)
+{
+    double ng = (double)g;
+    *M = ng * m_gpu - m_model;
+    *scale = (k4 / ng + c4 + kc * (ng - 1.0) / ng) / (k4 + c4);
+}
+
+/* Mean KV demand of a running request, "learned from the historical data"
+ * (Sec. 4.1, Eq. max throughput): over every decode iteration s = 1..l_pred
+ * of every request of a trace, the KV the request holds, h (l_in + s) + j
+ * (the footprint vector w of (e)), averaged; l_ave likewise for its context
+ * l_in + s. A request counts once per iteration it runs (a time average). */
+void orc_trace_demand(const orc_params* p, int64_t R, const int32_t* rin, const int32_t* rpred,
+                      double* m_r, double* l_ave)
+{
+    double kv = 0.0, ctx = 0.0, it = 0.0;
+    for (int64_t q = 0; q < R; ++q)
+        for (int32_t s = 1; s <= rpred[q]; ++s) {
+            kv += (double)(p->h * ((int64_t)rin[q] + s) + p->j);
+            ctx += (double)((int64_t)rin[q] + s);
+            it += 1.0;
+        }
+    *m_r = it > 0.0 ? kv / it : 0.0;
+    *l_ave = it > 0.0 ? ctx / it : 0.0;
+}
+
+/* Eq. max throughput: decode tokens per ms per GPU of a worker of g GPUs,
+ * KV capacity M and latency multiplier scale. The batch is bounded by the KV
+ * cache, b_kv = M / m_r, and by the ATGT SLO: B, the batch whose iteration
+ * scale (c3 + c2 B + k2 B l_ave) equals T_dec (Eq. iter time with the batch's
+ * context B l_ave; Eq. input limit). T_max = min(b_kv / (g t(b_kv)),
+ * B / (g T_dec)); both batches are kept fractional, as in the equation. */
+double orc_max_throughput(const orc_params* p, int32_t g, double M, double scale, double m_r,
+                          double l_ave)
+{
+    double b_kv = M / m_r;
+    double t_kv = scale * (p->c3 + p->c2 * b_kv + p->k2 * (b_kv * l_ave));
+    double B = (p->T_dec / scale - p->c3) / (p->c2 + p->k2 * l_ave);
+    double by_kv = b_kv / ((double)g * t_kv);
+    double by_slo = B / ((double)g * p->T_dec);
+    return by_kv < by_slo ? by_kv : by_slo;
+}
+
+/* The worker configuration of largest T_max (first on ties); T_max of each
+ * into tmax (nullable). */
+int32_t orc_pick_config(const orc_params* p, int32_t n, const int32_t* gpus, const double* M,
+                        const double* scale, double m_r, double l_ave, double* tmax)
+{
+    int32_t best = -1;
+    double bv = 0.0;
+    for (int32_t o = 0; o < n; ++o) {
+        double v = orc_max_throughput(p, gpus[o], M[o], scale[o], m_r, l_ave);
+        if (tmax) tmax[o] = v;
+        if (best < 0 || v > bv) {
+            best = o;
+            bv = v;
+        }
+    }
+    return best;
+}
+
+/* Eq. total_worker_pre: N_w = ceil(k5 r_a + c5) for arrival rates above R.
+ * k5, c5 by ordinary least squares over the (rate, minimum workers) points
+ * whose rate exceeds R. Returns the number of points used (< 2, or all rates
+ * equal: no fit, k5 = c5 = 0). */
+int32_t orc_fit_workers(int32_t n, const double* rate, const int32_t* nw, double R, double* k5,
+                        double* c5)
+{
+    double m = 0.0, sx = 0.0, sy = 0.0, sxx = 0.0, sxy = 0.0;
+    for (int32_t k = 0; k < n; ++k) {
+        if (!(rate[k] > R)) continue;
+        m += 1.0;
+        sx += rate[k];
+        sy += (double)nw[k];
+        sxx += rate[k] * rate[k];
+        sxy += rate[k] * (double)nw[k];
+    }
+    double den = m * sxx - sx * sx;
+    if (m < 2.0 || !(den > 0.0)) {
+        *k5 = 0.0;
+        *c5 = 0.0;
+        return (int32_t)m;
+    }
+    *k5 = (m * sxy - sx * sy) / den;
+    *c5 = (sy - *k5 * sx) / m;
+    return (int32_t)m;
+}
+
+int64_t orc_predict_workers(double k5, double c5, double rate)
+{
+    return (int64_t)ceil(k5 * rate + c5);
+}

@@ -73,6 +73,17 @@ def lib():
                                       P, P, P, C.c_double, C.c_int32, C.c_int32, P]
         _lib.orc_min_workers.argtypes = [P, C.c_int32, P, P, P, C.c_int32, C.c_int64, P, P, P,
                                          C.c_double, C.c_int32, P]
+        D = C.c_double
+        _lib.orc_tp_config.argtypes = [D, D, D, D, D, C.c_int32, P, P]
+        _lib.orc_trace_demand.argtypes = [P, C.c_int64, P, P, P, P]
+        _lib.orc_max_throughput.argtypes = [P, C.c_int32, D, D, D, D]
+        _lib.orc_max_throughput.restype = D
+        _lib.orc_pick_config.argtypes = [P, C.c_int32, P, P, P, D, D, P]
+        _lib.orc_pick_config.restype = C.c_int32
+        _lib.orc_fit_workers.argtypes = [C.c_int32, P, P, D, P, P]
+        _lib.orc_fit_workers.restype = C.c_int32
+        _lib.orc_predict_workers.argtypes = [D, D, D]
+        _lib.orc_predict_workers.restype = C.c_int64
         _lib.orc_capacity_norm.argtypes = [P, P, C.c_int]
         _lib.orc_capacity_norm.restype = C.c_double
         _lib.orc_order.argtypes = [P, P, P]
@@ -299,3 +310,58 @@ def min_workers(params, gpus, M, scale, cap, trace, H, n_max):
     if rc != 0:
         raise RuntimeError("orc_min_workers failed: %d" % rc)
     return n_out
+
+
+# ---------------------------------------------------------------------------
+# Worker configuration (Sec. 4.1) and the worker-count model (Sec. 5.2).
+
+def tp_config(k4, c4, kc, m_gpu, m_model, g):
+    """(KV capacity, latency multiplier) of a worker of g GPUs."""
+    M = C.c_double()
+    sc = C.c_double()
+    lib().orc_tp_config(float(k4), float(c4), float(kc), float(m_gpu), float(m_model), int(g),
+                        C.byref(M), C.byref(sc))
+    return M.value, sc.value
+
+
+def trace_demand(params, req_in, req_pred):
+    """(m_r, l_ave): iteration-averaged KV demand and context of a request."""
+    p = make_params(params)
+    ri = np.ascontiguousarray(req_in, np.int32)
+    rp = np.ascontiguousarray(req_pred, np.int32)
+    m = C.c_double()
+    l = C.c_double()
+    lib().orc_trace_demand(C.byref(p), len(ri), _ptr(ri), _ptr(rp), C.byref(m), C.byref(l))
+    return m.value, l.value
+
+
+def max_throughput(params, g, M, scale, m_r, l_ave):
+    p = make_params(params)
+    return lib().orc_max_throughput(C.byref(p), int(g), float(M), float(scale), float(m_r),
+                                    float(l_ave))
+
+
+def pick_config(params, gpus, M, scale, m_r, l_ave):
+    """(best option, T_max per option)."""
+    p = make_params(params)
+    g = np.ascontiguousarray(gpus, np.int32)
+    Mv = np.ascontiguousarray(M, np.float64)
+    sv = np.ascontiguousarray(scale, np.float64)
+    t = np.zeros(len(g))
+    best = lib().orc_pick_config(C.byref(p), len(g), _ptr(g), _ptr(Mv), _ptr(sv), float(m_r),
+                                 float(l_ave), _ptr(t))
+    return int(best), t
+
+
+def fit_workers(rates, nw, R=0.0):
+    """(k5, c5, points used) of Eq. total_worker_pre."""
+    r = np.ascontiguousarray(rates, np.float64)
+    n = np.ascontiguousarray(nw, np.int32)
+    k5 = C.c_double()
+    c5 = C.c_double()
+    used = lib().orc_fit_workers(len(r), _ptr(r), _ptr(n), float(R), C.byref(k5), C.byref(c5))
+    return k5.value, c5.value, int(used)
+
+
+def predict_workers(k5, c5, rate):
+    return int(lib().orc_predict_workers(float(k5), float(c5), float(rate)))
