@@ -308,6 +308,8 @@ def run_ours(args):
     round_ms = min(rounds)
     r16k = rounds_w16384(A, synth, stream)
     apx = approx_mode(A, synth, dev, stream, flush)
+    pol = policy_compare(A, synth, stream, 20_000, [1, 2])
+    wmod = worker_model(A, synth, stream, fit_n=0)
 
     peak, peak_kind = read_peaks()
     kern_avg = kern_ms / max(kern_n, 1)
@@ -338,6 +340,8 @@ def run_ours(args):
                                              "greedy round", "value": round_ms},
             "rounds_w16384": r16k,
             "approx_mode": apx,
+            "policies": pol,
+            "worker_config": wmod,
             "clocks": clocks}
     if cpu is not None:
         line["cpu_baseline"] = cpu
@@ -429,6 +433,100 @@ def min_workers_config(synth):
     kv = [MW_KV_PER_GPU * g for g in gpus]
     scale = [1.0 / math.sqrt(g) for g in gpus]
     return tr, gpus, kv, scale
+
+
+POLICIES = (("best_fit", 0), ("jsq", 1), ("power_of_two", 2))
+PHASES = (("mixed", 0), ("decode", 1))
+
+
+def policy_compare(A, synth, stream, n_requests, gpus, seed=4):
+    """GPUs each placement policy needs to serve a diurnal trace with every
+    SLO met (P100), in the mixed setting and on the decode instances of
+    split-phase inference (the comparison of Sec. 6.4): the minimum-worker
+    search per worker option, on the device, for best-fit (Algorithm 1), JSQ
+    and the power of two choices."""
+    tr = synth.diurnal_trace(seed, n_requests, 2000.0, 500.0)
+    kv = [MW_KV_PER_GPU * g for g in gpus]
+    scale = [1.0 / math.sqrt(g) for g in gpus]
+    trace = A.make_trace(tr.t_arr, tr.req_in, tr.req_pred)
+    out = {"workload": "diurnal trace of %d requests (peak 2,000 req/s, peak:trough 4:1, %.0f s), "
+                       "%s-GPU workers of %d KV tokens per GPU, latency x 1/sqrt(GPUs); "
+                       "P100: no failed request and no realized TTFT, ATGT or KV violation"
+                       % (n_requests, tr.t_arr[-1] / 1000.0, "/".join(map(str, gpus)),
+                          MW_KV_PER_GPU)}
+    for pname, phase in PHASES:
+        res = {}
+        for name, policy in POLICIES:
+            p = dict(synth.BASE_PARAMS, phase=phase, policy=policy, seed=12345)
+            got = np.zeros(len(gpus), np.int32)
+            t0 = time.perf_counter()
+            best, total = A.aladdin_min_workers(A.make_params(p, MW_B_CAP),
+                                                A.make_cfgs(gpus, kv, scale), trace, 100.0, 4096,
+                                                got, stream=stream)
+            res[name] = {"min_workers": got.tolist(), "total_gpus": int(total),
+                         "best_gpus_per_worker": gpus[best] if best >= 0 else None,
+                         "search_s": round(time.perf_counter() - t0, 2)}
+        bf = res["best_fit"]["total_gpus"]
+        for name in ("jsq", "power_of_two"):
+            o = res[name]["total_gpus"]
+            res["gpus_saved_vs_" + name] = round(1.0 - bf / o, 4) if bf > 0 and o > 0 else None
+        out[pname] = res
+    return out
+
+
+def worker_model(A, synth, stream, trace_n=100_000, fit_n=20_000,
+                 fit_rates=(250.0, 500.0, 1000.0, 1500.0, 2000.0)):
+    """The worker-configuration model of Sec. 4.1 (Eq. max throughput of each
+    1/2/4/8-GPU option from the diurnal trace's demand, the optimal option)
+    and Eq. total_worker_pre fitted to best-fit minimum-worker searches of
+    that option at constant arrival rates (Sec. 5.2)."""
+    tr = synth.diurnal_trace(4, trace_n, 2000.0, 500.0)
+    gpus = [1, 2, 4, 8]
+    kv = [MW_KV_PER_GPU * g for g in gpus]
+    scale = [1.0 / math.sqrt(g) for g in gpus]
+    p = dict(synth.BASE_PARAMS)
+    prm = A.make_params(p, MW_B_CAP)
+    trace = A.make_trace(tr.t_arr, tr.req_in, tr.req_pred)
+    m_r, l_ave = A.aladdin_trace_demand(prm, trace, stream=stream)
+    tmax = np.zeros(len(gpus))
+    best = A.aladdin_pick_config(prm, A.make_cfgs(gpus, kv, scale), trace, tmax, stream=stream)
+    out = {"demand": {"m_r": round(m_r, 3), "l_ave": round(l_ave, 3)},
+           "t_max_tokens_per_ms_per_gpu": [round(float(v), 4) for v in tmax],
+           "picked_gpus_per_worker": gpus[best]}
+    if fit_n:
+        trs = [synth.diurnal_trace(40 + k, fit_n, r, r) for k, r in enumerate(fit_rates)]
+        nw = np.zeros(len(trs), np.int32)
+        t0 = time.perf_counter()
+        k5, c5 = A.aladdin_fit_workers(prm, A.make_cfgs([gpus[best]], [kv[best]],
+                                                        [scale[best]])[0],
+                                       [A.make_trace(t.t_arr, t.req_in, t.req_pred) for t in trs],
+                                       list(fit_rates), 0.0, 100.0, 4096, nw, stream=stream)
+        pred = [A.aladdin_predict_workers(k5, c5, r) for r in fit_rates]
+        out["n_w_model"] = {"workload": "constant-rate Poisson traces of %d requests, %d-GPU "
+                                        "workers, best-fit" % (fit_n, gpus[best]),
+                            "rates_req_s": list(fit_rates), "min_workers": nw.tolist(),
+                            "k5": k5, "c5": c5, "predicted": pred,
+                            "fit_s": round(time.perf_counter() - t0, 2)}
+    return out
+
+
+def run_policies(args):
+    """Best-fit against JSQ and the power of two choices (Sec. 6.4): GPUs each
+    needs, mixed setting and decode instances, on a 100,000-request trace; the
+    worker-configuration picker and the fitted worker-count model."""
+    import torch
+    from paper_2405_06856_gb300 import build as B
+    B.build()
+    from paper_2405_06856_gb300 import aladdin as A
+    from paper_2405_06856_gb300 import synth
+    torch.cuda.set_device(0)
+    stream = torch.cuda.current_stream().cuda_stream
+    t0 = time.perf_counter()
+    res = policy_compare(A, synth, stream, 100_000, [1, 2, 4, 8])
+    res["worker_model"] = worker_model(A, synth, stream)
+    res["mode"] = "policies"
+    res["wall_s"] = round(time.perf_counter() - t0, 1)
+    print(json.dumps(res))
 
 
 def run_min_workers(args):
@@ -540,7 +638,8 @@ def main():
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--no-cpu-baseline", dest="cpu_baseline", action="store_false")
-    ap.add_argument("--mode", default="full", choices=["full", "kernel", "round", "minworkers"],
+    ap.add_argument("--mode", default="full",
+                    choices=["full", "kernel", "round", "minworkers", "policies"],
                     help="kernel: only warm-up + steps of the device-resident step (for profilers)")
     args = ap.parse_args()
     if args.warmup < 3:
@@ -553,6 +652,8 @@ def main():
         run_round_only(args)
     elif args.mode == "minworkers":
         run_min_workers(args)
+    elif args.mode == "policies":
+        run_policies(args)
     else:
         run_ours(args)
 

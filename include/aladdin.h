@@ -307,6 +307,70 @@ int aladdin_simulate(const aladdin_params* params, const aladdin_worker_cfg* cfg
                      const aladdin_trace* trace, double heartbeat_ms, int32_t stop_at_fail,
                      int32_t drain, void* cuda_stream, double* out);
 
+/* ------------------------------------------------------------------------
+ * Worker configuration (Sec. 4.1) and the worker-count model (Sec. 5.2).
+ */
+
+/* Tensor-parallel model of a worker of N_g GPUs (Sec. 4.1): compute time
+ * k4 / N_g + c4 (Eq. TP compute), all-reduce time kc (N_g - 1) / N_g, KV
+ * capacity N_g m_gpu - m_model (KV slots). */
+typedef struct aladdin_tp_model {
+    double k4, c4;     /* compute: ms, split across GPUs / not split */
+    double kc;         /* all-reduce overhead scale (ms) */
+    double m_gpu;      /* KV slots one GPU's memory holds */
+    double m_model;    /* KV slots the model's weights take from a worker */
+} aladdin_tp_model;
+
+/* Worker configurations for gpus[o] GPUs per worker (o < n): kv_capacity =
+ * floor(N_g m_gpu - m_model) and lat_scale = (k4 / N_g + c4 + kc (N_g - 1) /
+ * N_g) / (k4 + c4), the iteration time relative to one GPU, which multiplies
+ * every latency coefficient of aladdin_params (written to out[o]).
+ * ALADDIN_ERR_ARG if a coefficient is negative or not finite, k4 + c4 <= 0, a
+ * GPU count is below 1, or a capacity falls outside [1, 2^24). Host arrays;
+ * no GPU work. */
+int aladdin_tp_configs(const aladdin_tp_model* tp, int32_t n, const int32_t* gpus,
+                       aladdin_worker_cfg* out);
+
+/* Demand of a trace (Sec. 4.1, "learned from the historical data"): over
+ * every decode iteration s = 1..l_pred of every request, the KV the request
+ * holds, h (l_in + s) + j (the footprint vector w of (e)), averaged into
+ * *m_r, and its context l_in + s averaged into *l_ave (each nullable). The
+ * sums are exact integers reduced on the GPU; each average is one division.
+ * Trace arrays are host memory; synchronous on cuda_stream. */
+int aladdin_trace_demand(const aladdin_params* params, const aladdin_trace* trace,
+                         void* cuda_stream, double* m_r, double* l_ave);
+
+/* Eq. max throughput of each worker configuration options[o]: decode tokens
+ * per ms per GPU, T_max = min(b_kv / (g t(b_kv)), B / (g T_dec)), with the KV
+ * batch b_kv = kv_capacity / m_r, its iteration time t(b) = lat_scale (c3 +
+ * c2 b + k2 b l_ave) (Eq. iter time) and the SLO batch B = (T_dec /
+ * lat_scale - c3) / (c2 + k2 l_ave) (Eq. input limit); m_r and l_ave are the
+ * trace's demand (aladdin_trace_demand). Both batches stay fractional, as in
+ * the equation. t_max[o] (nullable) receives T_max, *best_option the option
+ * of largest T_max (the optimal worker configuration; first on ties).
+ * Trace arrays are host memory; synchronous. */
+int aladdin_pick_config(const aladdin_params* params, int32_t n_options,
+                        const aladdin_worker_cfg* options, const aladdin_trace* trace,
+                        void* cuda_stream, double* t_max, int32_t* best_option);
+
+/* Eq. total_worker_pre, N_w = ceil(k5 r_a + c5) for arrival rates r_a > R:
+ * for each trace k (requests arriving at rate rates[k], requests per second)
+ * the minimum number of workers of configuration cfg that serves it
+ * (aladdin_min_workers: params.policy and params.phase, heartbeat_ms, at
+ * most n_max workers) into n_workers[k], then k5 and c5 by ordinary least
+ * squares over the traces whose rate exceeds R and whose search succeeded.
+ * Returns ALADDIN_ERR_ARG (after filling n_workers, with k5 = c5 = 0) when
+ * fewer than two such traces, or only one distinct rate, remain. Trace arrays
+ * are host memory; every simulation runs on the GPU. */
+int aladdin_fit_workers(const aladdin_params* params, const aladdin_worker_cfg* cfg,
+                        int32_t n_traces, const aladdin_trace* traces, const double* rates,
+                        double R, double heartbeat_ms, int32_t n_max, void* cuda_stream,
+                        int32_t* n_workers, double* k5, double* c5);
+
+/* Eq. total_worker_pre: *n_workers = ceil(k5 rate + c5). ALADDIN_ERR_ARG if
+ * the value is not finite or outside the int64 range. */
+int aladdin_predict_workers(double k5, double c5, double rate, int64_t* n_workers);
+
 #ifdef __cplusplus
 }
 #endif

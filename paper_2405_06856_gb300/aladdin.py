@@ -58,6 +58,11 @@ class aladdin_worker_cfg(C.Structure):
     _fields_ = [("gpus", C.c_int32), ("kv_capacity", C.c_int64), ("lat_scale", C.c_double)]
 
 
+class aladdin_tp_model(C.Structure):
+    _fields_ = [("k4", C.c_double), ("c4", C.c_double), ("kc", C.c_double),
+                ("m_gpu", C.c_double), ("m_model", C.c_double)]
+
+
 class aladdin_trace(C.Structure):
     _fields_ = [("n", C.c_int64), ("t_arr_ms", C.c_void_p), ("in_", C.c_void_p),
                 ("pred", C.c_void_p)]
@@ -78,6 +83,12 @@ _sig = {
     "aladdin_cluster_timing": [_P, C.c_int32, _P, _P],
     "aladdin_min_workers": [_P, C.c_int32, _P, _P, C.c_double, C.c_int32, _P, _P, _P, _P],
     "aladdin_simulate": [_P, _P, C.c_int32, _P, C.c_double, C.c_int32, C.c_int32, _P, _P],
+    "aladdin_tp_configs": [_P, C.c_int32, _P, _P],
+    "aladdin_trace_demand": [_P, _P, _P, _P, _P],
+    "aladdin_pick_config": [_P, C.c_int32, _P, _P, _P, _P, _P],
+    "aladdin_fit_workers": [_P, _P, C.c_int32, _P, _P, C.c_double, C.c_double, C.c_int32, _P, _P,
+                            _P, _P],
+    "aladdin_predict_workers": [C.c_double, C.c_double, C.c_double, _P],
 }
 for _n, _a in _sig.items():
     f = getattr(_lib, _n)
@@ -230,6 +241,55 @@ def aladdin_simulate(params, cfg, n, trace, heartbeat_ms, stop_at_fail, drain, o
     _check(_lib.aladdin_simulate(C.byref(params), C.byref(cfg), int(n), C.byref(trace),
                                  float(heartbeat_ms), int(stop_at_fail), int(drain), stream,
                                  _ptr(out)), "aladdin_simulate")
+
+
+def aladdin_tp_configs(tp, gpus):
+    """Worker configurations (an aladdin_worker_cfg array) for the GPU counts."""
+    g = np.ascontiguousarray(gpus, np.int32)
+    out = (aladdin_worker_cfg * len(g))()
+    _check(_lib.aladdin_tp_configs(C.byref(tp), len(g), _ptr(g), C.cast(out, C.c_void_p)),
+           "aladdin_tp_configs")
+    return out
+
+
+def aladdin_trace_demand(params, trace, stream=None):
+    """(m_r, l_ave) of the trace."""
+    m = C.c_double()
+    l = C.c_double()
+    _check(_lib.aladdin_trace_demand(C.byref(params), C.byref(trace), stream, C.byref(m),
+                                     C.byref(l)), "aladdin_trace_demand")
+    return m.value, l.value
+
+
+def aladdin_pick_config(params, options, trace, t_max=None, stream=None):
+    """Best option (index into options); t_max (float64[n], optional) receives
+    each option's Eq. max throughput."""
+    best = C.c_int32(-1)
+    _check(_lib.aladdin_pick_config(C.byref(params), len(options), C.cast(options, C.c_void_p),
+                                    C.byref(trace), stream, _ptr(t_max), C.byref(best)),
+           "aladdin_pick_config")
+    return best.value
+
+
+def aladdin_fit_workers(params, cfg, traces, rates, R, heartbeat_ms, n_max, n_workers,
+                        stream=None):
+    """(k5, c5); n_workers (int32[len(traces)]) receives each search's count."""
+    arr = (aladdin_trace * len(traces))(*traces)
+    r = np.ascontiguousarray(rates, np.float64)
+    k5 = C.c_double()
+    c5 = C.c_double()
+    _check(_lib.aladdin_fit_workers(C.byref(params), C.byref(cfg), len(traces),
+                                    C.cast(arr, C.c_void_p), _ptr(r), float(R),
+                                    float(heartbeat_ms), int(n_max), stream, _ptr(n_workers),
+                                    C.byref(k5), C.byref(c5)), "aladdin_fit_workers")
+    return k5.value, c5.value
+
+
+def aladdin_predict_workers(k5, c5, rate):
+    n = C.c_int64()
+    _check(_lib.aladdin_predict_workers(float(k5), float(c5), float(rate), C.byref(n)),
+           "aladdin_predict_workers")
+    return n.value
 
 
 # ---------------------------------------------------------------------------

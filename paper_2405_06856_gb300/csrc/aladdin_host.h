@@ -79,6 +79,12 @@ cudaError_t launch_advance(const DevParams& P, const ClusterDev& C, double t_now
 cudaError_t launch_round_queue(const DevParams& P, const ClusterDev& C, const RoundIO& io,
                                cudaStream_t st);
 
+// Exact integer sums over a trace for the worker-configuration model:
+// sums[0] = sum of predicted outputs (decode iterations), sums[1] = sum over
+// requests and their iterations of the context l_in + s. Device pointers.
+cudaError_t launch_trace_demand(const int32_t* in, const int32_t* pred, long long n,
+                                unsigned long long* sums, cudaStream_t st);
+
 // What another translation unit may read of a cluster (see cluster_view).
 struct ClusterView {
     int device;

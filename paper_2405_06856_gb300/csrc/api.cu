@@ -866,6 +866,73 @@ int simulate_impl(const aladdin_params& p, const aladdin_worker_cfg& cfg, int32_
     return ALADDIN_OK;
 }
 
+// Smallest worker count in [1, n_max] of configuration cfg that serves the
+// trace with no failure (doubling then bisection), -1 if n_max fails.
+int search_min_workers(const aladdin_params& p, const aladdin_worker_cfg& cfg, const DevTrace& tr,
+                       double H, int32_t n_max, cudaStream_t st, int32_t* n_out)
+{
+    // JSQ and power of two admit without a test: drain to realize every
+    // request's latencies
+    const bool drain = p.policy != ALADDIN_POLICY_BESTFIT;
+    double out[6];
+    int rc;
+    int32_t lo = 0, hi = 1;
+    bool found = false;
+    while (hi <= n_max) {
+        if ((rc = simulate_impl(p, cfg, hi, tr, H, true, drain, st, out))) return rc;
+        if (out[0] == 0.0) {
+            found = true;
+            break;
+        }
+        lo = hi;
+        hi = (hi * 2 > n_max && hi < n_max) ? n_max : hi * 2;
+    }
+    if (!found) {
+        *n_out = -1;
+        return ALADDIN_OK;
+    }
+    while (hi - lo > 1) {
+        const int32_t mid = lo + (hi - lo) / 2;
+        if ((rc = simulate_impl(p, cfg, mid, tr, H, true, drain, st, out))) return rc;
+        if (out[0] == 0.0) hi = mid;
+        else lo = mid;
+    }
+    *n_out = hi;
+    return ALADDIN_OK;
+}
+
+bool finite_pos(double x) { return std::isfinite(x) && x > 0.0; }
+
+// Eq. max throughput of one configuration (tokens per ms per GPU).
+double max_throughput(const aladdin_params& p, const aladdin_worker_cfg& c, double m_r,
+                      double l_ave)
+{
+    const double b_kv = (double)c.kv_capacity / m_r;
+    const double t_kv = c.lat_scale * (p.c3 + p.c2 * b_kv + p.k2 * (b_kv * l_ave));
+    const double B = (p.T_dec / c.lat_scale - p.c3) / (p.c2 + p.k2 * l_ave);
+    const double by_kv = b_kv / ((double)c.gpus * t_kv);
+    const double by_slo = B / ((double)c.gpus * p.T_dec);
+    return by_kv < by_slo ? by_kv : by_slo;
+}
+
+int trace_demand_impl(const aladdin_params& p, const DevTrace& tr, cudaStream_t st, double* m_r,
+                      double* l_ave)
+{
+    DevBuf sums;
+    CK(sums.ensure(2 * sizeof(unsigned long long)));
+    CK(launch_trace_demand(tr.in, tr.pred, tr.n, sums.as<unsigned long long>(), st));
+    unsigned long long h[2] = {0, 0};
+    CK(cudaMemcpyAsync(h, sums.p, sizeof(h), cudaMemcpyDeviceToHost, st));
+    CK(cudaStreamSynchronize(st));
+    sums.release();
+    if (h[0] == 0) return ALADDIN_ERR_ARG;  // an empty trace has no demand
+    // KV slots summed over all iterations: h * context + j per iteration
+    const unsigned long long kv = (unsigned long long)p.h * h[1] + (unsigned long long)p.j * h[0];
+    if (m_r) *m_r = (double)kv / (double)h[0];
+    if (l_ave) *l_ave = (double)h[1] / (double)h[0];
+    return ALADDIN_OK;
+}
+
 }  // namespace
 
 extern "C" {
@@ -900,37 +967,10 @@ int aladdin_min_workers(const aladdin_params* params, int32_t n_options,
     cudaStream_t st = (cudaStream_t)cuda_stream;
     DevTrace tr;
     if ((rc = upload_trace(*params, trace, tr, st))) return rc;
-    double out[6];
-    // JSQ and power of two admit without a test: drain to realize every
-    // request's latencies
-    const bool drain = params->policy != ALADDIN_POLICY_BESTFIT;
-    for (int o = 0; o < n_options; ++o) {
-        int32_t lo = 0, hi = 1;
-        bool found = false;
-        while (hi <= n_max) {
-            if ((rc = simulate_impl(*params, options[o], hi, tr, heartbeat_ms, true, drain, st, out)))
-                return rc;
-            if (out[0] == 0.0) {
-                found = true;
-                break;
-            }
-            lo = hi;
-            hi = (hi * 2 > n_max && hi < n_max) ? n_max : hi * 2;
-        }
-        if (!found) {
-            n_workers[o] = -1;
-            continue;
-        }
-        while (hi - lo > 1) {
-            const int32_t mid = lo + (hi - lo) / 2;
-            if ((rc = simulate_impl(*params, options[o], mid, tr, heartbeat_ms, true, drain, st,
-                                    out)))
-                return rc;
-            if (out[0] == 0.0) hi = mid;
-            else lo = mid;
-        }
-        n_workers[o] = hi;
-    }
+    for (int o = 0; o < n_options; ++o)
+        if ((rc = search_min_workers(*params, options[o], tr, heartbeat_ms, n_max, st,
+                                     &n_workers[o])))
+            return rc;
     int best = -1;
     int64_t bestg = 0;
     for (int o = 0; o < n_options; ++o) {
@@ -943,6 +983,113 @@ int aladdin_min_workers(const aladdin_params* params, int32_t n_options,
     }
     if (best_option) *best_option = best;
     if (total_gpus) *total_gpus = best < 0 ? -1 : bestg;
+    return ALADDIN_OK;
+}
+
+int aladdin_tp_configs(const aladdin_tp_model* tp, int32_t n, const int32_t* gpus,
+                       aladdin_worker_cfg* out)
+{
+    if (!tp || n < 1 || !gpus || !out) return ALADDIN_ERR_ARG;
+    if (!(finite_nonneg(tp->k4) && finite_nonneg(tp->c4) && finite_nonneg(tp->kc) &&
+          finite_nonneg(tp->m_gpu) && finite_nonneg(tp->m_model) && tp->k4 + tp->c4 > 0.0))
+        return ALADDIN_ERR_ARG;
+    for (int32_t o = 0; o < n; ++o) {
+        if (gpus[o] < 1) return ALADDIN_ERR_ARG;
+        const double ng = (double)gpus[o];
+        const double M = std::floor(ng * tp->m_gpu - tp->m_model);
+        if (!(M >= 1.0 && M < (double)(1LL << 24))) return ALADDIN_ERR_ARG;
+        out[o].gpus = gpus[o];
+        out[o].kv_capacity = (int64_t)M;
+        out[o].lat_scale = (tp->k4 / ng + tp->c4 + tp->kc * (ng - 1.0) / ng) / (tp->k4 + tp->c4);
+    }
+    return ALADDIN_OK;
+}
+
+int aladdin_trace_demand(const aladdin_params* params, const aladdin_trace* trace,
+                         void* cuda_stream, double* m_r, double* l_ave)
+{
+    int rc = check_params(params);
+    if (rc) return rc;
+    cudaStream_t st = (cudaStream_t)cuda_stream;
+    DevTrace tr;
+    if ((rc = upload_trace(*params, trace, tr, st))) return rc;
+    return trace_demand_impl(*params, tr, st, m_r, l_ave);
+}
+
+int aladdin_pick_config(const aladdin_params* params, int32_t n_options,
+                        const aladdin_worker_cfg* options, const aladdin_trace* trace,
+                        void* cuda_stream, double* t_max, int32_t* best_option)
+{
+    int rc = check_params(params);
+    if (rc) return rc;
+    if (n_options < 1 || !options || !best_option) return ALADDIN_ERR_ARG;
+    for (int o = 0; o < n_options; ++o)
+        if ((rc = check_cfg(options[o])) || options[o].kv_capacity < 1) return ALADDIN_ERR_ARG;
+    cudaStream_t st = (cudaStream_t)cuda_stream;
+    DevTrace tr;
+    if ((rc = upload_trace(*params, trace, tr, st))) return rc;
+    double m_r = 0.0, l_ave = 0.0;
+    if ((rc = trace_demand_impl(*params, tr, st, &m_r, &l_ave))) return rc;
+    int32_t best = -1;
+    double bv = 0.0;
+    for (int o = 0; o < n_options; ++o) {
+        const double v = max_throughput(*params, options[o], m_r, l_ave);
+        if (t_max) t_max[o] = v;
+        if (best < 0 || v > bv) {
+            best = o;
+            bv = v;
+        }
+    }
+    *best_option = best;
+    return ALADDIN_OK;
+}
+
+int aladdin_fit_workers(const aladdin_params* params, const aladdin_worker_cfg* cfg,
+                        int32_t n_traces, const aladdin_trace* traces, const double* rates,
+                        double R, double heartbeat_ms, int32_t n_max, void* cuda_stream,
+                        int32_t* n_workers, double* k5, double* c5)
+{
+    int rc = check_params(params);
+    if (rc) return rc;
+    if (!cfg || n_traces < 1 || !traces || !rates || !n_workers || !k5 || !c5 || n_max < 1 ||
+        !finite_pos(heartbeat_ms) || std::isnan(R))
+        return ALADDIN_ERR_ARG;
+    if ((rc = check_cfg(*cfg))) return rc;
+    for (int k = 0; k < n_traces; ++k)
+        if (!std::isfinite(rates[k])) return ALADDIN_ERR_ARG;
+    *k5 = 0.0;
+    *c5 = 0.0;
+    cudaStream_t st = (cudaStream_t)cuda_stream;
+    for (int k = 0; k < n_traces; ++k) {
+        DevTrace tr;
+        if ((rc = upload_trace(*params, &traces[k], tr, st))) return rc;
+        if ((rc = search_min_workers(*params, *cfg, tr, heartbeat_ms, n_max, st, &n_workers[k])))
+            return rc;
+    }
+    // ordinary least squares over the usable points above R
+    double m = 0.0, sx = 0.0, sy = 0.0, sxx = 0.0, sxy = 0.0;
+    for (int k = 0; k < n_traces; ++k) {
+        if (!(rates[k] > R) || n_workers[k] < 1) continue;
+        const double x = rates[k], y = (double)n_workers[k];
+        m += 1.0;
+        sx += x;
+        sy += y;
+        sxx += x * x;
+        sxy += x * y;
+    }
+    const double den = m * sxx - sx * sx;
+    if (m < 2.0 || !(den > 0.0)) return ALADDIN_ERR_ARG;
+    *k5 = (m * sxy - sx * sy) / den;
+    *c5 = (sy - *k5 * sx) / m;
+    return ALADDIN_OK;
+}
+
+int aladdin_predict_workers(double k5, double c5, double rate, int64_t* n_workers)
+{
+    if (!n_workers) return ALADDIN_ERR_ARG;
+    const double v = std::ceil(k5 * rate + c5);
+    if (!(std::isfinite(v) && v >= -9.2e18 && v <= 9.2e18)) return ALADDIN_ERR_ARG;
+    *n_workers = (int64_t)v;
     return ALADDIN_OK;
 }
 

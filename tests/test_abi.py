@@ -86,3 +86,33 @@ def test_null_arguments(lib):
     cfg = lib.make_cfgs([1], [1 << 24], [1.0])  # capacity must be < 2^24
     assert lib._lib.aladdin_simulate(ctypes.byref(p), ctypes.cast(cfg, ctypes.c_void_p), 1, None,
                                      100.0, 1, 0, None, None) == lib.ERR_ARG
+
+
+# --------------------------------------------------------------------------
+# Host-only entry points of the worker-configuration model, against the oracle.
+
+def test_tp_configs_match_oracle(lib, orc):
+    tp = lib.aladdin_tp_model(30.0, 10.0, 4.0, 80_000.0, 30_000.0)
+    gpus = [1, 2, 4, 8]
+    cfgs = lib.aladdin_tp_configs(tp, gpus)
+    for o, g in enumerate(gpus):
+        M, s = orc.tp_config(30.0, 10.0, 4.0, 80_000.0, 30_000.0, g)
+        assert cfgs[o].gpus == g and cfgs[o].kv_capacity == int(np.floor(M))
+        assert cfgs[o].lat_scale == pytest.approx(s, rel=1e-15)
+
+
+@pytest.mark.parametrize("tp,gpus", [((30.0, 10.0, 4.0, 10.0, 30.0), [1]),     # capacity < 1
+                                     ((0.0, 0.0, 1.0, 1e5, 0.0), [1]),        # k4 + c4 = 0
+                                     ((30.0, -1.0, 4.0, 1e5, 0.0), [1]),
+                                     ((30.0, 10.0, 4.0, 1e5, 0.0), [0]),
+                                     ((30.0, 10.0, 4.0, 1e7, 0.0), [2])])    # >= 2^24
+def test_tp_configs_reject(lib, tp, gpus):
+    with pytest.raises(lib.AladdinError):
+        lib.aladdin_tp_configs(lib.aladdin_tp_model(*tp), gpus)
+
+
+def test_predict_workers_matches_oracle(lib, orc):
+    for k5, c5, r in ((0.06, 4.0, 1234.0), (0.013, -2.5, 977.0), (1e-3, 0.0, 250.0)):
+        assert lib.aladdin_predict_workers(k5, c5, r) == orc.predict_workers(k5, c5, r)
+    with pytest.raises(lib.AladdinError):
+        lib.aladdin_predict_workers(float("inf"), 0.0, 1.0)
