@@ -182,6 +182,140 @@ def oracle_baseline(workers_per_core=4, ncand=32768, cores=None):
                       % (cores * workers_per_core, ncand, WORKLOAD, pairs, busy, wall)}
 
 
+def _oracle_config_job(job):
+    """One oracle measurement of --mode configs (runs in a spawned process)."""
+    kind, name = job[0], job[1]
+    from oracle import oracle as O
+    from paper_2405_06856_gb300 import synth
+    if kind == "search":
+        g, n = job[2], job[3]
+        tr = synth.diurnal_trace(4, n, 2000.0, 500.0)
+        t0 = time.perf_counter()
+        got = O.min_workers(dict(synth.BASE_PARAMS), [g], [MW_KV_PER_GPU * g],
+                            [1.0 / math.sqrt(g)], MW_B_CAP, tr, 100.0, 4096)
+        return (kind, name, g, int(got[0]), time.perf_counter() - t0)
+    wl = synth.config(name)
+    if kind == "score":
+        oc = O.Cluster.from_workload(wl)
+        t0 = time.perf_counter()
+        oc.score(wl.cand_in, wl.cand_pred, wl.cand_wait, want=("flags", "margin", "argbest"))
+        return (kind, name, wl.n_cand * wl.n_workers, time.perf_counter() - t0)
+    if kind == "sample":
+        # every pair of a few random workers with the first ncand candidates
+        nw, ncand = job[2], job[3]
+        wid = np.sort(np.random.default_rng(17).choice(wl.n_workers, nw, replace=False))
+        sub = O.Cluster(wl.params, wl.kv_capacity[wid], wl.lat_scale[wid], wl.b_cap,
+                        np.concatenate([[0], np.cumsum(np.diff(wl.roff)[wid])]).astype(np.int32),
+                        np.concatenate([wl.req_in[wl.roff[w]:wl.roff[w + 1]] for w in wid]),
+                        np.concatenate([wl.req_gen[wl.roff[w]:wl.roff[w + 1]] for w in wid]),
+                        np.concatenate([wl.req_pred[wl.roff[w]:wl.roff[w + 1]] for w in wid]))
+        t0 = time.perf_counter()
+        sub.score(wl.cand_in[:ncand], wl.cand_pred[:ncand], wl.cand_wait[:ncand],
+                  want=("flags", "margin"))
+        return (kind, name, nw * ncand, time.perf_counter() - t0)
+    oc = O.Cluster.from_workload(wl)  # round
+    t0 = time.perf_counter()
+    oc.place_round(wl.cand_in, wl.cand_pred, wl.cand_wait)
+    return (kind, name, wl.n_cand, time.perf_counter() - t0)
+
+
+def run_configs(args):
+    """Every workload of the scope table, on the GPU and with the oracle (one
+    host core per oracle job, jobs in parallel on a spawn pool started before
+    the first CUDA call): scoring evaluations/s and fraction of the HBM
+    roofline (tiny, w256, w4096, w16384), one greedy round (tiny, w256; the
+    16,384-worker rounds run as in the default line), and the minimum-worker
+    search on a 10,000-request scale-down of the 1,000,000-request trace."""
+    import multiprocessing as mp
+    from oracle import oracle as O
+    O.build()
+    jobs = [("score", "tiny"), ("round", "tiny"), ("score", "w256"), ("round", "w256"),
+            ("sample", "w4096", 8, 8192), ("sample", "w16384", 8, 8192)]
+    jobs += [("search", "trace10k", g, 10_000) for g in (1, 2, 4, 8)]
+    ctx = mp.get_context("spawn")
+    pool = ctx.Pool(min(len(jobs), os.cpu_count() or 1))
+    pending = pool.map_async(_oracle_config_job, jobs)
+
+    import torch
+    from paper_2405_06856_gb300 import build as B
+    B.build()
+    from paper_2405_06856_gb300 import aladdin as A
+    from paper_2405_06856_gb300 import synth
+    torch.cuda.set_device(0)
+    dev = torch.device("cuda", 0)
+    stream = torch.cuda.current_stream().cuda_stream
+    peak, peak_kind = read_peaks()
+    flush = torch.empty(L2_FLUSH_BYTES // 4, dtype=torch.float32, device=dev)
+    d = lambda x: torch.from_numpy(np.ascontiguousarray(x)).to(dev)
+    gpu = {}
+    for name in ("tiny", "w256", "w4096", "w16384"):
+        wl = synth.config(name)
+        W, C = wl.n_workers, wl.n_cand
+        cin, cpr, cw = d(wl.cand_in), d(wl.cand_pred), d(wl.cand_wait)
+        f = torch.empty((C, W), dtype=torch.uint8, device=dev)
+        m = torch.empty((C, W), dtype=torch.float32, device=dev)
+        a = torch.empty(C, dtype=torch.int32, device=dev)
+        with A.Cluster.from_workload(wl, stream=stream) as cl:
+            for _ in range(3):
+                A.aladdin_score(cl.handle, C, cin, cpr, cw, f, m, a)
+            torch.cuda.synchronize()
+            A.aladdin_cluster_timing(cl.handle, 1)
+            for _ in range(10):
+                flush.zero_()
+                A.aladdin_score(cl.handle, C, cin, cpr, cw, f, m, a)
+            kern_ms, kern_n = A.aladdin_cluster_timing(cl.handle, 0)
+            feas = float((f == 15).float().mean().item())
+        kern = kern_ms / max(kern_n, 1)
+        nbytes = len(wl.req_in) * 12 + C * 12 + C * W * 5 + C * 4
+        row = {"workers": W, "candidates": C, "k_score_ms": round(kern, 4),
+               "evals_per_s": C * W / (kern / 1000.0),
+               "hbm_frac": round(nbytes / (kern / 1000.0) / 1e9 / peak, 4),
+               "feasible_fraction": round(feas, 4)}
+        if name in ("tiny", "w256"):
+            rms = []
+            for _ in range(3):
+                with A.Cluster.from_workload(wl, stream=stream) as c2:
+                    pl = torch.empty(C, dtype=torch.int32, device=dev)
+                    torch.cuda.synchronize()
+                    t0 = time.perf_counter()
+                    A.aladdin_place_round(c2.handle, C, cin, cpr, cw, pl)
+                    rms.append((time.perf_counter() - t0) * 1000.0)
+            row["round_ms"] = round(min(rms), 3)
+        gpu[name] = row
+        del f, m
+        torch.cuda.empty_cache()
+    gpu["w16384"]["rounds"] = rounds_w16384(A, synth, stream)
+    tr = synth.diurnal_trace(4, 10_000, 2000.0, 500.0)
+    gpus = [1, 2, 4, 8]
+    got = np.zeros(4, np.int32)
+    torch.cuda.synchronize()
+    t0 = time.perf_counter()
+    A.aladdin_min_workers(A.make_params(dict(synth.BASE_PARAMS), MW_B_CAP),
+                          A.make_cfgs(gpus, [MW_KV_PER_GPU * g for g in gpus],
+                                      [1.0 / math.sqrt(g) for g in gpus]),
+                          A.make_trace(tr.t_arr, tr.req_in, tr.req_pred), 100.0, 4096, got,
+                          stream=stream)
+    gpu["search_10k"] = {"min_workers": got.tolist(), "wall_s": round(time.perf_counter() - t0, 2)}
+
+    res = pending.get()
+    pool.close()
+    orc = {}
+    for r in res:
+        if r[0] == "search":
+            orc.setdefault("search_10k", {"min_workers": [], "s_per_option": []})
+            orc["search_10k"]["min_workers"].append(r[3])
+            orc["search_10k"]["s_per_option"].append(round(r[4], 2))
+        elif r[0] == "round":
+            orc.setdefault(r[1], {})["round_ms"] = round(r[3] * 1000.0, 2)
+        else:
+            orc.setdefault(r[1], {})["evals_per_s_1core"] = r[2] / r[3]
+            if r[0] == "sample":
+                orc[r[1]]["sample"] = ("%d pairs (8 random workers x 8,192 candidates), "
+                                       "extrapolated" % r[2])
+    print(json.dumps({"mode": "configs", "peak_gbs": peak, "peak_kind": peak_kind,
+                      "host_cores": os.cpu_count(), "gpu": gpu, "oracle": orc}))
+
+
 # ---------------------------------------------------------------------------
 
 def run_reference(args):
@@ -639,7 +773,7 @@ def main():
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--no-cpu-baseline", dest="cpu_baseline", action="store_false")
     ap.add_argument("--mode", default="full",
-                    choices=["full", "kernel", "round", "minworkers", "policies"],
+                    choices=["full", "kernel", "round", "minworkers", "policies", "configs"],
                     help="kernel: only warm-up + steps of the device-resident step (for profilers)")
     args = ap.parse_args()
     if args.warmup < 3:
@@ -654,6 +788,8 @@ def main():
         run_min_workers(args)
     elif args.mode == "policies":
         run_policies(args)
+    elif args.mode == "configs":
+        run_configs(args)
     else:
         run_ours(args)
 
