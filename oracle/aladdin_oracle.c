@@ -98,6 +98,7 @@ typedef struct {
     int64_t phase;        /* 0: mixed prefill + decode; 1: decode instance */
     int64_t policy;       /* 0: best-fit; 1: JSQ; 2: power of two choices */
     uint64_t seed;        /* SplitMix64 seed of the power-of-two draws */
+    int64_t rebalance;    /* 1: Algorithm 2 after every placement round (simulation) */
 } orc_params;
 
 /* Relative slack of a realized latency over its SLO before it counts as a
@@ -121,6 +122,13 @@ typedef struct {
     uint8_t* pend;        /* [W*cap] 1: placed in the current round, prefill pending */
     double* wait;         /* [W*cap] pending requests: wait since arrival (ms) */
     int64_t* rid;         /* [W*cap] request id (simulation only), or NULL */
+    int32_t* real;        /* [W*cap] real output length (unknown to the scheduler), or
+                             NULL: every prediction is exact */
+    int64_t* le;          /* [W] Algorithm 2's output-length error l^e, or NULL */
+    int32_t* be;          /* [W] Algorithm 2's batch-size error b^e, or NULL */
+    const int32_t* repred;/* [K+1] re-prediction: the output length predicted for a
+                             request that has generated x tokens without finishing,
+                             or NULL (x + 1) */
 } orc_cluster;
 
 typedef struct {
@@ -573,17 +581,19 @@ static int pick_by_queue(const orc_params* p, const orc_cluster* cl, int64_t rid
  * refuse_full (simulation of JSQ / power of two), placement -3 and the round
  * goes on. The power-of-two draws use crid[c] (c if crid is NULL). */
 static int place_round_impl(const orc_params* p, orc_cluster* cl, int32_t C, const int32_t* cin,
-                            const int32_t* cpred, const double* cwait, const int64_t* crid,
-                            int32_t* placement, int refuse_full);
+                            const int32_t* cpred, const int32_t* creal, const double* cwait,
+                            const int64_t* crid, int32_t* placement, int refuse_full);
 
 int orc_place_round(const orc_params* p, orc_cluster* cl, int32_t C, const int32_t* cin,
                     const int32_t* cpred, const double* cwait, const int64_t* crid,
                     int32_t* placement)
 {
-    return place_round_impl(p, cl, C, cin, cpred, cwait, crid, placement, 0);
+    return place_round_impl(p, cl, C, cin, cpred, NULL, cwait, crid, placement, 0);
 }
 
-static void append_request(orc_cluster* cl, int w, int32_t a, int32_t r, double wait, int64_t rid)
+/* Append a request of the open round to worker w (gen 0, prefill pending). */
+static void append_request(orc_cluster* cl, int w, int32_t a, int32_t r, int32_t real,
+                           double wait, int64_t rid)
 {
     int64_t slot = (int64_t)w * cl->cap + cl->n[w];
     cl->in[slot] = a;
@@ -593,12 +603,29 @@ static void append_request(orc_cluster* cl, int w, int32_t a, int32_t r, double 
     cl->pend[slot] = 1;
     cl->wait[slot] = wait;
     if (cl->rid) cl->rid[slot] = rid;
+    if (cl->real) cl->real[slot] = real;
     cl->n[w] += 1;
 }
 
+/* Remove slot q of worker w: the worker's last slot moves into it. */
+static void remove_slot(orc_cluster* cl, int w, int q)
+{
+    int64_t slot = (int64_t)w * cl->cap + q;
+    int64_t last = (int64_t)w * cl->cap + cl->n[w] - 1;
+    cl->in[slot] = cl->in[last];
+    cl->gen[slot] = cl->gen[last];
+    cl->pred[slot] = cl->pred[last];
+    if (cl->tdec) cl->tdec[slot] = cl->tdec[last];
+    cl->pend[slot] = cl->pend[last];
+    cl->wait[slot] = cl->wait[last];
+    if (cl->rid) cl->rid[slot] = cl->rid[last];
+    if (cl->real) cl->real[slot] = cl->real[last];
+    cl->n[w] -= 1;
+}
+
 static int place_round_impl(const orc_params* p, orc_cluster* cl, int32_t C, const int32_t* cin,
-                            const int32_t* cpred, const double* cwait, const int64_t* crid,
-                            int32_t* placement, int refuse_full)
+                            const int32_t* cpred, const int32_t* creal, const double* cwait,
+                            const int64_t* crid, int32_t* placement, int refuse_full)
 {
     const int W = cl->W;
     if (p->policy != 0) {
@@ -613,7 +640,8 @@ static int place_round_impl(const orc_params* p, orc_cluster* cl, int32_t C, con
                 placement[c] = -3;
                 continue;
             }
-            append_request(cl, w, cin[c], cpred[c], cwait ? cwait[c] : 0.0, rid);
+            append_request(cl, w, cin[c], cpred[c], creal ? creal[c] : cpred[c],
+                           cwait ? cwait[c] : 0.0, rid);
             placement[c] = w;
         }
         return ORC_OK;
@@ -639,7 +667,8 @@ static int place_round_impl(const orc_params* p, orc_cluster* cl, int32_t C, con
             eval_pair(p, cl, w, &fut[w], T0, T1, cin[c], cpred[c], cwait ? cwait[c] : 0.0, &r);
             if (r.flags != 15) continue;
             if (cl->n[w] >= cl->cap) { rc = ORC_ERR_CAPACITY; break; }
-            append_request(cl, w, cin[c], cpred[c], cwait ? cwait[c] : 0.0, crid ? crid[c] : c);
+            append_request(cl, w, cin[c], cpred[c], creal ? creal[c] : cpred[c],
+                           cwait ? cwait[c] : 0.0, crid ? crid[c] : c);
             future_free(&fut[w]);
             have[w] = 0;
             placement[c] = w;
@@ -668,11 +697,16 @@ static int place_round_impl(const orc_params* p, orc_cluster* cl, int32_t C, con
  * record no TTFT. viol (nullable, 3 counters) accumulates the realized
  * violations: [0] TTFT above T_pre, [1] ATGT above T_dec (each beyond the
  * relative ORC_SLO_TOL), [2] decode iterations whose KV usage
- * h * context + j * batch exceeds M. Afterwards off[w] is the time from
- * t_now + dt to the worker's next iteration start. */
+ * h * context + j * batch exceeds M. With real lengths (cl->real) a request
+ * finishes when it has generated its real length; a request that reaches its
+ * prediction first is re-predicted (cl->repred) and counted in ev[0] (nullable),
+ * an early finish in ev[1]; both update Algorithm 2's per-worker errors
+ * (cl->le, cl->be). The realized ATGT divides by the tokens generated.
+ * Afterwards off[w] is the time from t_now + dt to the worker's next iteration
+ * start. */
 int orc_advance(const orc_params* p, orc_cluster* cl, double t_now, double dt,
                 int64_t* rec_rid, double* rec_val, uint8_t* rec_kind, int64_t* nrec,
-                int64_t rec_cap, int64_t* viol)
+                int64_t rec_cap, int64_t* viol, int64_t* ev)
 {
     const double t_end = t_now + dt;
     const int decode = p->phase == 1;
@@ -724,11 +758,37 @@ int orc_advance(const orc_params* p, orc_cluster* cl, double t_now, double dt,
                 cl->tdec[base + q] += t;
             }
             start += t;
+            /* Prediction errors (Sec. 4.3, Algorithm 2's indicators): a request
+             * that reaches its predicted length without finishing is
+             * re-predicted (l^e grows by the added length, b^e by one); one
+             * that finishes before its prediction lowers l^e by the unused
+             * length and b^e by one. */
+            for (int q = 0; q < cl->n[w]; ++q) {
+                int64_t slot = base + q;
+                int32_t real = cl->real ? cl->real[slot] : cl->pred[slot];
+                int32_t g = cl->gen[slot];
+                if (g >= real) {
+                    if (real < cl->pred[slot]) {
+                        if (cl->le) cl->le[w] += (int64_t)real - cl->pred[slot];
+                        if (cl->be) cl->be[w] -= 1;
+                        if (ev) ev[1] += 1;
+                    }
+                } else if (g >= cl->pred[slot]) {
+                    int32_t np = cl->repred ? cl->repred[g] : g + 1;
+                    if (np < g + 1) np = g + 1;
+                    if ((int64_t)cl->in[slot] + np > p->K) np = (int32_t)(p->K - cl->in[slot]);
+                    if (cl->le) cl->le[w] += (int64_t)np - cl->pred[slot];
+                    if (cl->be) cl->be[w] += 1;
+                    if (ev) ev[0] += 1;
+                    cl->pred[slot] = np;
+                }
+            }
             /* Retire finished requests; the last slot moves into the hole. */
             for (int q = 0; q < cl->n[w];) {
                 int64_t slot = base + q;
-                if (cl->gen[slot] >= cl->pred[slot]) {
-                    double atgt = cl->tdec[slot] / (double)cl->pred[slot];
+                int32_t real = cl->real ? cl->real[slot] : cl->pred[slot];
+                if (cl->gen[slot] >= real) {
+                    double atgt = cl->tdec[slot] / (double)cl->gen[slot];
                     if (rec_rid && *nrec < rec_cap) {
                         rec_rid[*nrec] = cl->rid ? cl->rid[slot] : slot;
                         rec_val[*nrec] = atgt;
@@ -736,15 +796,7 @@ int orc_advance(const orc_params* p, orc_cluster* cl, double t_now, double dt,
                     }
                     *nrec += 1;
                     if (viol && atgt > p->T_dec * (1.0 + ORC_SLO_TOL)) viol[1] += 1;
-                    int64_t last = base + cl->n[w] - 1;
-                    cl->in[slot] = cl->in[last];
-                    cl->gen[slot] = cl->gen[last];
-                    cl->pred[slot] = cl->pred[last];
-                    cl->tdec[slot] = cl->tdec[last];
-                    cl->pend[slot] = cl->pend[last];
-                    cl->wait[slot] = cl->wait[last];
-                    if (cl->rid) cl->rid[slot] = cl->rid[last];
-                    cl->n[w] -= 1;
+                    remove_slot(cl, w, q);
                 } else {
                     ++q;
                 }
@@ -753,6 +805,98 @@ int orc_advance(const orc_params* p, orc_cluster* cl, double t_now, double dt,
         cl->clock[w] = start;
         cl->off[w] = start > t_end ? start - t_end : 0.0;
     }
+    return ORC_OK;
+}
+
+/* ---------------------------------------------------------------------- */
+/* Algorithm 2 (Sec. 4.3, re-balancing with prediction error), run after a
+ * placement round and before the round's requests execute. Worker i's errors
+ * (l^e_i, b^e_i) define, through Eq. input limit (k2 l + c2 b = T_dec - c3),
+ * the line k2 l + c2 b - (k2 l^e_i + c2 b^e_i) = 0 through its error point,
+ * parallel to the SLO boundary; its distance to the origin is
+ * |e_i| / sqrt(k2^2 + c2^2) with e_i = k2 l^e_i + c2 b^e_i. Moving a new
+ * request j (predicted output l_j) from worker x to worker y moves l_j and one
+ * request of error from x to y: e_x -= d_j, e_y += d_j with d_j = k2 l_j + c2.
+ * The sum of distances is reduced greedily: the round's placements in index
+ * order; one on an over-utilized worker (e_x > 0) moves to the under-utilized
+ * worker (e_y < 0) that is feasible for it in the current state (all four
+ * flags, a free slot) and lowers the sum the most, gain
+ * (e_x - e_y) - |e_x - d_j| - |e_y + d_j| > 0; equal gains go to the larger
+ * capacity_norm, then the lower index. A moved request leaves its pending
+ * slot on x and becomes a pending request of y. placement[] is updated;
+ * *moves (nullable) counts the moves, obj (nullable, 2 doubles) receives the
+ * sum of distances before and after. */
+int orc_rebalance(const orc_params* p, orc_cluster* cl, int32_t C, const int32_t* cin,
+                  const int32_t* cpred, const double* cwait, int32_t* placement,
+                  const int64_t* le, const int32_t* be, int32_t* moves, double* obj)
+{
+    const int W = cl->W;
+    double* e = (double*)malloc(sizeof(double) * (size_t)W);
+    int32_t S = (int32_t)p->K + 2;
+    double* T0 = (double*)malloc(sizeof(double) * ((size_t)S + 2));
+    double* T1 = (double*)malloc(sizeof(double) * ((size_t)S + 2));
+    if (!e || !T0 || !T1) return ORC_ERR_MEM;
+    const double norm = sqrt(p->k2 * p->k2 + p->c2 * p->c2);
+    double before = 0.0;
+    for (int i = 0; i < W; ++i) {
+        e[i] = p->k2 * (double)le[i] + p->c2 * (double)be[i];
+        before += fabs(e[i]) / norm;
+    }
+    int32_t nmov = 0;
+    for (int32_t c = 0; c < C; ++c) {
+        int x = placement[c];
+        if (x < 0 || !(e[x] > 0.0)) continue;
+        double d = p->k2 * (double)cpred[c] + p->c2;
+        double wc = cwait ? cwait[c] : 0.0;
+        int best = -1;
+        double bgain = 0.0, bnorm = 0.0;
+        for (int y = 0; y < W; ++y) {
+            if (y == x || !(e[y] < 0.0) || cl->n[y] >= cl->cap) continue;
+            double gain = ((e[x] - e[y]) - fabs(e[x] - d)) - fabs(e[y] + d);
+            if (!(gain > 0.0)) continue;
+            orc_future f;
+            if (future_build(cl, y, &f) != ORC_OK) return ORC_ERR_MEM;
+            orc_pair r;
+            eval_pair(p, cl, y, &f, T0, T1, cin[c], cpred[c], wc, &r);
+            future_free(&f);
+            if (r.flags != 15) continue;
+            double ny = orc_capacity_norm(p, cl, y);
+            if (best < 0 || gain > bgain || (gain == bgain && ny > bnorm)) {
+                best = y;
+                bgain = gain;
+                bnorm = ny;
+            }
+        }
+        if (best < 0) continue;
+        /* the request's pending slot on x: the last one with its values */
+        int q = -1;
+        for (int k = cl->n[x] - 1; k >= 0 && q < 0; --k) {
+            int64_t slot = (int64_t)x * cl->cap + k;
+            if (cl->pend[slot] && cl->in[slot] == cin[c] && cl->pred[slot] == cpred[c] &&
+                cl->wait[slot] == wc)
+                q = k;
+        }
+        if (q < 0) continue;
+        int64_t slot = (int64_t)x * cl->cap + q;
+        int32_t real = cl->real ? cl->real[slot] : cpred[c];
+        int64_t rid = cl->rid ? cl->rid[slot] : c;
+        remove_slot(cl, x, q);
+        append_request(cl, best, cin[c], cpred[c], real, wc, rid);
+        e[x] -= d;
+        e[best] += d;
+        placement[c] = best;
+        nmov += 1;
+    }
+    double after = 0.0;
+    for (int i = 0; i < W; ++i) after += fabs(e[i]) / norm;
+    if (moves) *moves = nmov;
+    if (obj) {
+        obj[0] = before;
+        obj[1] = after;
+    }
+    free(e);
+    free(T0);
+    free(T1);
     return ORC_OK;
 }
 
@@ -769,13 +913,20 @@ int orc_advance(const orc_params* p, orc_cluster* cl, double t_now, double dt,
  * worker has no free slot fails. Every realized violation (see orc_advance)
  * also counts as a failure. If drain is set the simulation continues without
  * arrivals until every worker is empty, so that every admitted request's
- * realized TTFT and ATGT are recorded.
+ * realized TTFT and ATGT are recorded. With real output lengths (rreal,
+ * nullable: exact predictions) requests run to their real length and are
+ * re-predicted with repred (nullable) when they outgrow a prediction; with
+ * p->rebalance, Algorithm 2 (orc_rebalance) runs after every placement round
+ * on the errors the execution recorded since the previous heartbeat, which
+ * then restart from zero.
  * out[0] failed, out[1] placed, out[2] heartbeats, out[3] max realized TTFT,
  * out[4] max realized ATGT, out[5] realized records, out[6] realized
- * violations (included in out[0]). */
+ * violations (included in out[0]), out[7] re-predictions, out[8] early
+ * finishes, out[9] requests moved by Algorithm 2. */
 int orc_simulate(const orc_params* p, int32_t N, int32_t cap, int64_t M, double scale,
                  int64_t R, const double* t_arr, const int32_t* rin, const int32_t* rpred,
-                 double H, int32_t stop_at_fail, int32_t drain, double* out)
+                 const int32_t* rreal, const int32_t* repred, double H, int32_t stop_at_fail,
+                 int32_t drain, double* out)
 {
     orc_cluster cl;
     memset(&cl, 0, sizeof(cl));
@@ -794,6 +945,11 @@ int orc_simulate(const orc_params* p, int32_t N, int32_t cap, int64_t M, double 
     cl.pend = (uint8_t*)calloc(slots, 1);
     cl.wait = (double*)calloc(slots, sizeof(double));
     cl.rid = (int64_t*)calloc(slots, sizeof(int64_t));
+    cl.real = (int32_t*)calloc(slots, sizeof(int32_t));
+    cl.le = (int64_t*)calloc((size_t)N, sizeof(int64_t));
+    cl.be = (int32_t*)calloc((size_t)N, sizeof(int32_t));
+    cl.repred = repred;
+    int32_t* creal = (int32_t*)malloc(sizeof(int32_t) * (size_t)(R > 0 ? R : 1));
     int64_t* wl = (int64_t*)malloc(sizeof(int64_t) * (size_t)(R > 0 ? R : 1));
     int32_t* cin = (int32_t*)malloc(sizeof(int32_t) * (size_t)(R > 0 ? R : 1));
     int32_t* cpr = (int32_t*)malloc(sizeof(int32_t) * (size_t)(R > 0 ? R : 1));
@@ -804,13 +960,15 @@ int orc_simulate(const orc_params* p, int32_t N, int32_t cap, int64_t M, double 
     double* rv = (double*)malloc(sizeof(double) * (size_t)rec_cap);
     uint8_t* rk = (uint8_t*)malloc((size_t)rec_cap);
     if (!Mv || !sv || !cl.off || !cl.clock || !cl.n || !cl.in || !cl.gen || !cl.pred || !cl.tdec ||
-        !cl.pend || !cl.wait || !cl.rid || !wl || !cin || !cpr || !cw || !pl || !rr || !rv || !rk)
+        !cl.pend || !cl.wait || !cl.rid || !wl || !cin || !cpr || !cw || !pl || !rr || !rv || !rk ||
+        !cl.real || !cl.le || !cl.be || !creal)
         return ORC_ERR_MEM;
     for (int w = 0; w < N; ++w) { Mv[w] = M; sv[w] = scale; }
     cl.M = Mv;
     cl.scale = sv;
 
     int64_t next = 0, nwait = 0, failed = 0, placed = 0, hb = 0, nrec = 0, violations = 0;
+    int64_t events[2] = {0, 0}, moved = 0;
     double max_ttft = 0.0, max_atgt = 0.0;
     int rc = ORC_OK;
     for (;;) {
@@ -820,10 +978,18 @@ int orc_simulate(const orc_params* p, int32_t N, int32_t cap, int64_t M, double 
             for (int64_t i = 0; i < nwait; ++i) {
                 cin[i] = rin[wl[i]];
                 cpr[i] = rpred[wl[i]];
+                creal[i] = rreal ? rreal[wl[i]] : rpred[wl[i]];
                 cw[i] = t - t_arr[wl[i]];
             }
-            rc = place_round_impl(p, &cl, (int32_t)nwait, cin, cpr, cw, wl, pl, 1);
+            rc = place_round_impl(p, &cl, (int32_t)nwait, cin, cpr, creal, cw, wl, pl, 1);
             if (rc != ORC_OK) break;
+            if (p->rebalance && p->policy == 0) {
+                int32_t mv = 0;
+                rc = orc_rebalance(p, &cl, (int32_t)nwait, cin, cpr, cw, pl, cl.le, cl.be, &mv,
+                                   NULL);
+                if (rc != ORC_OK) break;
+                moved += mv;
+            }
             int64_t keep = 0;
             for (int64_t i = 0; i < nwait; ++i) {
                 if (pl[i] >= 0) { placed++; continue; }
@@ -836,7 +1002,11 @@ int orc_simulate(const orc_params* p, int32_t N, int32_t cap, int64_t M, double 
         if (failed > 0 && stop_at_fail) break;
         int64_t nr0 = nrec;
         int64_t vv[3] = {0, 0, 0};
-        orc_advance(p, &cl, t, H, rr, rv, rk, &nrec, rec_cap, vv);
+        for (int w = 0; w < N; ++w) {  /* Algorithm 2's errors restart every heartbeat */
+            cl.le[w] = 0;
+            cl.be[w] = 0;
+        }
+        orc_advance(p, &cl, t, H, rr, rv, rk, &nrec, rec_cap, vv, events);
         violations += vv[0] + vv[1] + vv[2];
         failed += vv[0] + vv[1] + vv[2];
         for (int64_t i = nr0; i < nrec && i < rec_cap; ++i) {
@@ -859,6 +1029,10 @@ int orc_simulate(const orc_params* p, int32_t N, int32_t cap, int64_t M, double 
     out[4] = max_atgt;
     out[5] = (double)nrec;
     out[6] = (double)violations;
+    out[7] = (double)events[0];
+    out[8] = (double)events[1];
+    out[9] = (double)moved;
+    free(cl.real); free(cl.le); free(cl.be); free(creal);
     free(Mv); free(sv); free(cl.off); free(cl.clock); free(cl.n); free(cl.in); free(cl.gen);
     free(cl.pred); free(cl.tdec); free(cl.pend); free(cl.wait); free(cl.rid);
     free(wl); free(cin); free(cpr); free(cw); free(pl); free(rr); free(rv); free(rk);
@@ -874,16 +1048,17 @@ int orc_simulate(const orc_params* p, int32_t N, int32_t cap, int64_t M, double 
  * construction. */
 int orc_min_workers(const orc_params* p, int32_t n_opt, const int32_t* gpus, const int64_t* M,
                     const double* scale, int32_t cap, int64_t R, const double* t_arr,
-                    const int32_t* rin, const int32_t* rpred, double H, int32_t n_max,
-                    int32_t* n_out)
+                    const int32_t* rin, const int32_t* rpred, const int32_t* rreal,
+                    const int32_t* repred, double H, int32_t n_max, int32_t* n_out)
 {
-    double out[7];
+    double out[10];
     const int32_t drain = p->policy != 0;
     for (int o = 0; o < n_opt; ++o) {
         int32_t lo = 0, hi = 1; /* lo fails (or is 0), hi to be tested */
         int found = 0;
         while (hi <= n_max) {
-            int rc = orc_simulate(p, hi, cap, M[o], scale[o], R, t_arr, rin, rpred, H, 1, drain, out);
+            int rc = orc_simulate(p, hi, cap, M[o], scale[o], R, t_arr, rin, rpred, rreal, repred,
+                                  H, 1, drain, out);
             if (rc != ORC_OK) return rc;
             if (out[0] == 0.0) { found = 1; break; }
             lo = hi;
@@ -892,8 +1067,8 @@ int orc_min_workers(const orc_params* p, int32_t n_opt, const int32_t* gpus, con
         if (!found) { n_out[o] = -1; continue; }
         while (hi - lo > 1) {
             int32_t mid = lo + (hi - lo) / 2;
-            int rc = orc_simulate(p, mid, cap, M[o], scale[o], R, t_arr, rin, rpred, H, 1, drain,
-                                  out);
+            int rc = orc_simulate(p, mid, cap, M[o], scale[o], R, t_arr, rin, rpred, rreal,
+                                  repred, H, 1, drain, out);
             if (rc != ORC_OK) return rc;
             if (out[0] == 0.0) hi = mid;
             else lo = mid;

@@ -40,7 +40,7 @@ class Params(C.Structure):
                 ("j", C.c_int64), ("T_pre", C.c_double), ("T_dec", C.c_double),
                 ("gamma", C.c_double), ("theta", C.c_double), ("K", C.c_int64),
                 ("mode", C.c_int64), ("phase", C.c_int64), ("policy", C.c_int64),
-                ("seed", C.c_uint64)]
+                ("seed", C.c_uint64), ("rebalance", C.c_int64)]
 
 
 class ClusterStruct(C.Structure):
@@ -48,7 +48,9 @@ class ClusterStruct(C.Structure):
                 ("M", C.c_void_p), ("scale", C.c_void_p), ("off", C.c_void_p),
                 ("clock", C.c_void_p), ("n", C.c_void_p), ("inp", C.c_void_p),
                 ("gen", C.c_void_p), ("pred", C.c_void_p), ("tdec", C.c_void_p),
-                ("pend", C.c_void_p), ("wait", C.c_void_p), ("rid", C.c_void_p)]
+                ("pend", C.c_void_p), ("wait", C.c_void_p), ("rid", C.c_void_p),
+                ("real", C.c_void_p), ("le", C.c_void_p), ("be", C.c_void_p),
+                ("repred", C.c_void_p)]
 
 
 _lib = None
@@ -64,15 +66,16 @@ def lib():
         _lib.orc_kv_curve.argtypes = [P, P, C.c_int, C.c_int32, C.c_int32, P]
         _lib.orc_kv_curve.restype = C.c_int32
         _lib.orc_place_round.argtypes = [P, P, C.c_int32, P, P, P, P, P]
-        _lib.orc_advance.argtypes = [P, P, C.c_double, C.c_double, P, P, P, P, C.c_int64, P]
+        _lib.orc_advance.argtypes = [P, P, C.c_double, C.c_double, P, P, P, P, C.c_int64, P, P]
+        _lib.orc_rebalance.argtypes = [P, P, C.c_int32, P, P, P, P, P, P, P, P]
         _lib.orc_splitmix64.argtypes = [C.c_uint64, C.c_uint64]
         _lib.orc_splitmix64.restype = C.c_uint64
         _lib.orc_po2_draw.argtypes = [C.c_uint64, C.c_int64, C.c_int, C.c_int32]
         _lib.orc_po2_draw.restype = C.c_int32
         _lib.orc_simulate.argtypes = [P, C.c_int32, C.c_int32, C.c_int64, C.c_double, C.c_int64,
-                                      P, P, P, C.c_double, C.c_int32, C.c_int32, P]
-        _lib.orc_min_workers.argtypes = [P, C.c_int32, P, P, P, C.c_int32, C.c_int64, P, P, P,
-                                         C.c_double, C.c_int32, P]
+                                      P, P, P, P, P, C.c_double, C.c_int32, C.c_int32, P]
+        _lib.orc_min_workers.argtypes = [P, C.c_int32, P, P, P, C.c_int32, C.c_int64, P, P, P, P,
+                                         P, C.c_double, C.c_int32, P]
         D = C.c_double
         _lib.orc_tp_config.argtypes = [D, D, D, D, D, C.c_int32, P, P]
         _lib.orc_trace_demand.argtypes = [P, C.c_int64, P, P, P, P]
@@ -95,7 +98,7 @@ def make_params(d):
                   float(d["c3"]), int(d["h"]), int(d["j"]), float(d["T_pre"]),
                   float(d["T_dec"]), float(d["gamma"]), float(d["theta"]), int(d["K"]),
                   int(d.get("mode", 0)), int(d.get("phase", 0)), int(d.get("policy", 0)),
-                  int(d.get("seed", 0)) & 0xFFFFFFFFFFFFFFFF)
+                  int(d.get("seed", 0)) & 0xFFFFFFFFFFFFFFFF, int(d.get("rebalance", 0)))
 
 
 def _ptr(a):
@@ -125,6 +128,10 @@ class Cluster:
         self.pend = np.zeros(S, np.uint8)
         self.wait = np.zeros(S, np.float64)
         self.rid = np.zeros(S, np.int64)
+        self.real = None          # real output lengths [W*cap], or None (exact)
+        self.le = np.zeros(W, np.int64)
+        self.be = np.zeros(W, np.int32)
+        self.repred = None        # re-prediction table [K+1], or None
         if roff is not None:
             for w in range(W):
                 a, b = int(roff[w]), int(roff[w + 1])
@@ -150,7 +157,8 @@ class Cluster:
         return ClusterStruct(self.W, self.cap, _ptr(self.M), _ptr(self.scale), _ptr(self.off),
                              _ptr(self.clock), _ptr(self.n), _ptr(self.inp), _ptr(self.gen),
                              _ptr(self.pred), _ptr(self.tdec) if use_tdec else None,
-                             _ptr(self.pend), _ptr(self.wait), _ptr(self.rid))
+                             _ptr(self.pend), _ptr(self.wait), _ptr(self.rid), _ptr(self.real),
+                             _ptr(self.le), _ptr(self.be), _ptr(self.repred))
 
     def score(self, cin, cpred, cwait=None, want=("flags", "margin", "mscale", "kvpeak",
                                                     "tcand", "near", "argbest")):
@@ -244,7 +252,31 @@ class Cluster:
         self.rid[slot] = rid
         self.n[w] += 1
 
-    def advance(self, t_now, dt, rec_cap=1 << 16, violations=None):
+    def set_real(self, real, repred=None):
+        """Real output lengths per slot (same layout as pred) and the
+        re-prediction table: execution then follows the real lengths."""
+        self.real = np.ascontiguousarray(real, np.int32).copy()
+        self.repred = None if repred is None else np.ascontiguousarray(repred, np.int32)
+
+    def rebalance(self, cin, cpred, cwait, placement, le, be):
+        """Algorithm 2 over a round's placements (updated in place); returns
+        (moves, objective before, objective after)."""
+        cin = np.ascontiguousarray(cin, np.int32)
+        cpred = np.ascontiguousarray(cpred, np.int32)
+        cw = None if cwait is None else np.ascontiguousarray(cwait, np.float64)
+        le = np.ascontiguousarray(le, np.int64)
+        be = np.ascontiguousarray(be, np.int32)
+        mv = C.c_int32(0)
+        obj = np.zeros(2)
+        st = self.struct()
+        rc = lib().orc_rebalance(C.byref(self._p), C.byref(st), len(cin), _ptr(cin), _ptr(cpred),
+                                 _ptr(cw), _ptr(placement), _ptr(le), _ptr(be), C.byref(mv),
+                                 _ptr(obj))
+        if rc != 0:
+            raise RuntimeError("orc_rebalance failed: %d" % rc)
+        return mv.value, obj[0], obj[1]
+
+    def advance(self, t_now, dt, rec_cap=1 << 16, violations=None, events=None):
         """Execute every worker for dt ms; returns the realized records (request
         id, value, kind 0 TTFT / 1 ATGT). ``violations`` (int64[3], optional)
         accumulates realized TTFT, ATGT and KV-overflow violations."""
@@ -256,7 +288,7 @@ class Cluster:
         self.has_tdec = True
         rc = lib().orc_advance(C.byref(self._p), C.byref(st), float(t_now), float(dt),
                                _ptr(rr), _ptr(rv), _ptr(rk), C.byref(nrec), rec_cap,
-                               _ptr(violations))
+                               _ptr(violations), _ptr(events))
         if rc != 0:
             raise RuntimeError("orc_advance failed")
         k = min(nrec.value, rec_cap)
@@ -279,21 +311,30 @@ def po2_draw(seed, rid, k, W):
     return int(lib().orc_po2_draw(int(seed) & 0xFFFFFFFFFFFFFFFF, int(rid), int(k), int(W)))
 
 
+def _trace_real(trace):
+    real = getattr(trace, "req_real", None)
+    rep = getattr(trace, "repred", None)
+    return (None if real is None else np.ascontiguousarray(real, np.int32),
+            None if rep is None else np.ascontiguousarray(rep, np.int32))
+
+
 def simulate(params, N, cap, M, scale, trace, H, stop_at_fail=True, drain=False):
-    out = np.zeros(7)
+    out = np.zeros(10)
     p = make_params(params)
     t = np.ascontiguousarray(trace.t_arr, np.float64)
     ri = np.ascontiguousarray(trace.req_in, np.int32)
     rp = np.ascontiguousarray(trace.req_pred, np.int32)
+    rr, rep = _trace_real(trace)
     rc = lib().orc_simulate(C.byref(p), int(N), int(cap), int(M), float(scale), len(t), _ptr(t),
-                            _ptr(ri), _ptr(rp), float(H), int(stop_at_fail), int(drain),
-                            _ptr(out))
+                            _ptr(ri), _ptr(rp), _ptr(rr), _ptr(rep), float(H), int(stop_at_fail),
+                            int(drain), _ptr(out))
     if rc == -2:
         raise OverflowError("worker request capacity exceeded")
     if rc != 0:
         raise RuntimeError("orc_simulate failed: %d" % rc)
     return dict(failed=int(out[0]), placed=int(out[1]), heartbeats=int(out[2]),
-                max_ttft=out[3], max_atgt=out[4], violations=int(out[6]))
+                max_ttft=out[3], max_atgt=out[4], violations=int(out[6]),
+                repredictions=int(out[7]), early_finishes=int(out[8]), moved=int(out[9]))
 
 
 def min_workers(params, gpus, M, scale, cap, trace, H, n_max):
@@ -305,8 +346,10 @@ def min_workers(params, gpus, M, scale, cap, trace, H, n_max):
     ri = np.ascontiguousarray(trace.req_in, np.int32)
     rp = np.ascontiguousarray(trace.req_pred, np.int32)
     n_out = np.zeros(len(g), np.int32)
+    rr, rep = _trace_real(trace)
     rc = lib().orc_min_workers(C.byref(p), len(g), _ptr(g), _ptr(Mv), _ptr(sv), int(cap), len(t),
-                               _ptr(t), _ptr(ri), _ptr(rp), float(H), int(n_max), _ptr(n_out))
+                               _ptr(t), _ptr(ri), _ptr(rp), _ptr(rr), _ptr(rep), float(H),
+                               int(n_max), _ptr(n_out))
     if rc != 0:
         raise RuntimeError("orc_min_workers failed: %d" % rc)
     return n_out

@@ -146,10 +146,44 @@ def config(name, **over):
 
 @dataclasses.dataclass
 class Trace:
-    """Request arrivals: times (ms, non-decreasing), input and predicted lengths."""
+    """Request arrivals: times (ms, non-decreasing), input and predicted lengths;
+    optionally the real output lengths (unknown to the scheduler) and the
+    re-prediction table a serving system would use when a request outgrows
+    its prediction."""
     t_arr: np.ndarray   # float64 [R]
     req_in: np.ndarray  # int32 [R]
     req_pred: np.ndarray  # int32 [R]
+    req_real: np.ndarray = None  # int32 [R] or None: predictions are exact
+    repred: np.ndarray = None    # int32 [K+1] or None
+
+
+def repredict_table(out_law, K, n=1_000_000, seed=99):
+    """Conditional mean output length given that it exceeds x, for x = 0..K
+    (rounded up; x + 1 where no draw exceeds x): what a predictor learned
+    from the output-length distribution predicts for a request that has
+    generated x tokens without finishing. Drawn from the same law."""
+    rng = np.random.default_rng(seed)
+    om, osg, olo, ohi = out_law
+    L = np.sort(lognormal_lengths(rng, om, osg, olo, ohi, n).astype(np.int64))
+    suffix = np.concatenate([np.cumsum(L[::-1])[::-1], [0]])
+    x = np.arange(K + 1)
+    first = np.searchsorted(L, x, side="right")    # draws > x start here
+    cnt = n - first
+    mean = np.where(cnt > 0, suffix[first] / np.maximum(cnt, 1), x + 1)
+    return np.maximum(np.ceil(mean), x + 1).astype(np.int32)
+
+
+def with_prediction_error(trace, sigma, seed, out_law=(256.0, 0.9, 8, 1024), K=8192):
+    """The same arrivals with the drawn output lengths as the real ones and
+    predictions off by a lognormal factor exp(N(0, sigma)), rounded and
+    clipped to the output law's range (and to K - input)."""
+    rng = np.random.default_rng(seed)
+    real = np.asarray(trace.req_pred, np.int32)
+    om, osg, olo, ohi = out_law
+    noisy = np.rint(real * np.exp(rng.normal(0.0, sigma, len(real))))
+    hi = np.minimum(ohi, K - np.asarray(trace.req_in, np.int64))
+    pred = np.clip(noisy, olo, hi).astype(np.int32)
+    return Trace(trace.t_arr, trace.req_in, pred, real, repredict_table(out_law, K))
 
 
 def diurnal_trace(seed, n_requests, peak_rate, trough_rate, in_law=(512.0, 0.8, 16, 2048),
