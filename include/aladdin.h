@@ -112,7 +112,7 @@ extern "C" {
  * Requirements: k1, k2 > 0; c1, c2, c3 >= 0; h >= 1; j >= 0; T_pre > 0;
  * T_dec > c3 (Eq. input limit); 0 < theta <= 1; gamma >= 0; 2 <= K <= 65536;
  * b_cap a power of two in [32, 1024]; mode, phase and policy one of the
- * values above. */
+ * values above; rebalance 0 or 1. */
 typedef struct aladdin_params {
     double k1, c1;       /* prefill: ms per input token, ms */
     double k2, c2, c3;   /* decode: ms per context token, ms per request, ms */
@@ -127,6 +127,8 @@ typedef struct aladdin_params {
     int32_t phase;       /* ALADDIN_PHASE_MIXED or ALADDIN_PHASE_DECODE */
     int32_t policy;      /* ALADDIN_POLICY_BESTFIT, _JSQ or _PO2 */
     uint64_t seed;       /* SplitMix64 seed of the power-of-two draws */
+    int32_t rebalance;   /* 1: Algorithm 2 after every best-fit round of a simulation
+                            (see aladdin_rebalance); 0: off */
 } aladdin_params;
 
 /* One worker configuration (Sec. 4.1): GPUs per worker, KV capacity in KV
@@ -240,7 +242,10 @@ int aladdin_place_round(aladdin_cluster* cl, int32_t n_cand, const int32_t* in,
  * [3] largest realized ATGT (ms per token), and the realized violations:
  * [4] TTFTs above T_pre, [5] ATGTs above T_dec (each beyond a relative 1e-5,
  * the rounding of the fp32 placement test), [6] decode iterations whose KV
- * usage h * context + j * batch exceeded the worker's capacity. */
+ * usage h * context + j * batch exceeded the worker's capacity. stats has 9
+ * doubles: [7] re-predictions and [8] early finishes (both zero here: a
+ * cluster built by this API holds exact predictions; the simulation follows
+ * a trace's real lengths). */
 int aladdin_cluster_advance(aladdin_cluster* cl, double dt_ms, double* stats);
 
 /* Copy the cluster state to host arrays (each nullable): n[W] requests per
@@ -248,6 +253,28 @@ int aladdin_cluster_advance(aladdin_cluster* cl, double dt_ms, double* stats);
  * round). Synchronous. */
 int aladdin_cluster_state(aladdin_cluster* cl, int32_t* n, int32_t* in, int32_t* gen,
                           int32_t* pred, uint8_t* pending);
+
+/* Algorithm 2 (Sec. 4.3, re-balancing with prediction error) over a round
+ * that aladdin_place_round placed (n_cand candidates in, pred, wait_ms, and
+ * their placement[], updated in place), before the round executes. le[w] and
+ * be[w] (W entries each) are worker w's output-length and batch-size errors
+ * (l^e, b^e): the tokens and requests its running requests deviate from
+ * their predictions (+ for a request that outgrew its prediction, by the
+ * added length; - for one that finished early, by the unused length). Its
+ * error e_w = k2 l^e + c2 b^e places it relative to Eq. input limit; the
+ * distance |e_w| / sqrt(k2^2 + c2^2) of that error line to the origin is
+ * what the moves reduce, summed over workers. In index order, a placement on
+ * a worker with e > 0 moves to the worker with e < 0 that is feasible for it
+ * in the current state (all four flags, a free slot) and lowers the sum the
+ * most: gain (e_x - e_y) - |e_x - d| - |e_y + d| > 0 with d = k2 pred + c2;
+ * equal gains go to the larger capacity_norm, then the lower index. Moved
+ * requests stay pending (prefill at the new worker's next boundary).
+ * *moves (nullable) receives the number of moves, obj (nullable, host, 2
+ * doubles) the summed distance before and after. Errors as
+ * aladdin_place_round. */
+int aladdin_rebalance(aladdin_cluster* cl, int32_t n_cand, const int32_t* in,
+                      const int32_t* pred, const float* wait_ms, int32_t* placement,
+                      const int64_t* le, const int32_t* be, int32_t* moves, double* obj);
 
 /* Kernel timing (tracing): while enabled, CUDA events on the cluster's stream
  * bracket every launch of the candidate x worker scoring kernel. Each call
@@ -265,12 +292,20 @@ int aladdin_cluster_timing(aladdin_cluster* cl, int32_t enable, double* kernel_m
 int aladdin_cluster_status(aladdin_cluster* cl);
 
 /* A request trace: arrival times (ms, non-decreasing), prompt and predicted
- * output lengths. */
+ * output lengths, and optionally prediction errors (Sec. 4.3): real[q] is the
+ * output length request q really generates (the scheduler sees only
+ * pred[q]); when a request has generated x tokens, reached its prediction
+ * and not finished, it is re-predicted to repred[x] (at least x + 1, at most
+ * K - in), the output length a predictor expects of a request known to
+ * exceed x (repred has K + 1 entries; NULL: x + 1). real NULL: predictions
+ * are exact. Host arrays. */
 typedef struct aladdin_trace {
     int64_t n;
     const double* t_arr_ms;
     const int32_t* in;
     const int32_t* pred;
+    const int32_t* real;     /* nullable, 1 <= real[q], in[q] + real[q] <= K */
+    const int32_t* repred;   /* nullable, K + 1 entries */
 } aladdin_trace;
 
 /* Minimum-worker search (Sec. 4.1, Sec. 6.4): for every worker configuration
@@ -298,11 +333,17 @@ int aladdin_min_workers(const aladdin_params* params, int32_t n_options,
  * within T_pre; on a decode instance it fails at its first heartbeat; JSQ and
  * PO2 place every request at once and one whose worker has no free slot
  * fails. Every realized violation (aladdin_cluster_advance stats [4]-[6])
- * counts as a failure too. out (host, 6 doubles): [0] failures, [1] placed
- * requests, [2] heartbeats run, [3] largest realized TTFT, [4] largest
- * realized ATGT, [5] realized violations (included in [0]). With
- * stop_at_fail the simulation ends at the heartbeat after the first failure;
- * with drain it continues after the last arrival until every worker is idle. */
+ * counts as a failure too. With prediction errors in the trace requests run
+ * to their real lengths (re-predicted as they outgrow predictions), and with
+ * params.rebalance (best-fit only) Algorithm 2 (aladdin_rebalance) runs after
+ * every round on the errors the workers recorded since the previous
+ * heartbeat, which then restart from zero. out (host, 9 doubles):
+ * [0] failures, [1] placed requests, [2] heartbeats run, [3] largest realized
+ * TTFT, [4] largest realized ATGT, [5] realized violations (included in
+ * [0]), [6] re-predictions, [7] early finishes, [8] requests moved by
+ * Algorithm 2. With stop_at_fail the simulation ends at the heartbeat after
+ * the first failure; with drain it continues after the last arrival until
+ * every worker is idle. */
 int aladdin_simulate(const aladdin_params* params, const aladdin_worker_cfg* cfg, int32_t n,
                      const aladdin_trace* trace, double heartbeat_ms, int32_t stop_at_fail,
                      int32_t drain, void* cuda_stream, double* out);

@@ -22,8 +22,8 @@ ERR_SCRATCH = -7
 MODE_EXACT, MODE_APPROX = 0, 1
 PHASE_MIXED, PHASE_DECODE = 0, 1
 POLICY_BESTFIT, POLICY_JSQ, POLICY_PO2 = 0, 1, 2
-ADVANCE_STATS = 7     # doubles written by aladdin_cluster_advance
-SIMULATE_OUT = 6      # doubles written by aladdin_simulate
+ADVANCE_STATS = 9     # doubles written by aladdin_cluster_advance
+SIMULATE_OUT = 9      # doubles written by aladdin_simulate
 NOALLOC_MAX_CAND = 32768
 FLAG_KV, FLAG_TTFT, FLAG_ONGOING, FLAG_NEW, FEASIBLE, FLAG_INVALID = 1, 2, 4, 8, 15, 128
 NONE, INVALID = -1, -2
@@ -51,7 +51,8 @@ class aladdin_params(C.Structure):
                 ("c3", C.c_double), ("h", C.c_int32), ("j", C.c_int32), ("T_pre", C.c_double),
                 ("T_dec", C.c_double), ("gamma", C.c_double), ("theta", C.c_double),
                 ("K", C.c_int32), ("b_cap", C.c_int32), ("mode", C.c_int32),
-                ("phase", C.c_int32), ("policy", C.c_int32), ("seed", C.c_uint64)]
+                ("phase", C.c_int32), ("policy", C.c_int32), ("seed", C.c_uint64),
+                ("rebalance", C.c_int32)]
 
 
 class aladdin_worker_cfg(C.Structure):
@@ -65,7 +66,7 @@ class aladdin_tp_model(C.Structure):
 
 class aladdin_trace(C.Structure):
     _fields_ = [("n", C.c_int64), ("t_arr_ms", C.c_void_p), ("in_", C.c_void_p),
-                ("pred", C.c_void_p)]
+                ("pred", C.c_void_p), ("real", C.c_void_p), ("repred", C.c_void_p)]
 
 
 _P = C.c_void_p
@@ -89,6 +90,7 @@ _sig = {
     "aladdin_fit_workers": [_P, _P, C.c_int32, _P, _P, C.c_double, C.c_double, C.c_int32, _P, _P,
                             _P, _P],
     "aladdin_predict_workers": [C.c_double, C.c_double, C.c_double, _P],
+    "aladdin_rebalance": [_P, C.c_int32, _P, _P, _P, _P, _P, _P, _P, _P],
 }
 for _n, _a in _sig.items():
     f = getattr(_lib, _n)
@@ -137,7 +139,7 @@ def make_params(d, b_cap):
                           float(d["T_dec"]), float(d["gamma"]), float(d["theta"]), int(d["K"]),
                           int(b_cap), int(d.get("mode", MODE_EXACT)),
                           int(d.get("phase", PHASE_MIXED)), int(d.get("policy", POLICY_BESTFIT)),
-                          int(d.get("seed", 0)) & 0xFFFFFFFFFFFFFFFF)
+                          int(d.get("seed", 0)) & 0xFFFFFFFFFFFFFFFF, int(d.get("rebalance", 0)))
 
 
 def make_cfgs(gpus, kv_capacity, lat_scale):
@@ -150,13 +152,24 @@ def make_cfgs(gpus, kv_capacity, lat_scale):
     return arr
 
 
-def make_trace(t_arr, req_in, req_pred):
+def make_trace(t_arr, req_in, req_pred, req_real=None, repred=None):
+    """An aladdin_trace over host arrays (kept alive by the returned object);
+    req_real / repred: prediction errors (see aladdin_trace)."""
     t = np.ascontiguousarray(t_arr, np.float64)
     i = np.ascontiguousarray(req_in, np.int32)
     p = np.ascontiguousarray(req_pred, np.int32)
-    tr = aladdin_trace(len(t), t.ctypes.data, i.ctypes.data, p.ctypes.data)
-    tr._keep = (t, i, p)
+    r = None if req_real is None else np.ascontiguousarray(req_real, np.int32)
+    q = None if repred is None else np.ascontiguousarray(repred, np.int32)
+    tr = aladdin_trace(len(t), t.ctypes.data, i.ctypes.data, p.ctypes.data,
+                       None if r is None else r.ctypes.data, None if q is None else q.ctypes.data)
+    tr._keep = (t, i, p, r, q)
     return tr
+
+
+def trace_of(tr):
+    """make_trace of a synth.Trace (with its prediction errors, if any)."""
+    return make_trace(tr.t_arr, tr.req_in, tr.req_pred, getattr(tr, "req_real", None),
+                      getattr(tr, "repred", None))
 
 
 # ---------------------------------------------------------------------------
@@ -203,6 +216,17 @@ def aladdin_score_detail(cl, n_cand, cand_in, cand_pred, wait_ms, flags, margin,
 def aladdin_place_round(cl, n_cand, cand_in, cand_pred, wait_ms, placement):
     _check(_lib.aladdin_place_round(cl, int(n_cand), _ptr(cand_in), _ptr(cand_pred),
                                     _ptr(wait_ms), _ptr(placement)), "aladdin_place_round")
+
+
+def aladdin_rebalance(cl, n_cand, cand_in, cand_pred, wait_ms, placement, le, be):
+    """Algorithm 2 over a placed round; placement is updated in place.
+    Returns (moves, summed distance before, after)."""
+    mv = C.c_int32(0)
+    obj = np.zeros(2)
+    _check(_lib.aladdin_rebalance(cl, int(n_cand), _ptr(cand_in), _ptr(cand_pred), _ptr(wait_ms),
+                                  _ptr(placement), _ptr(le), _ptr(be), C.byref(mv), _ptr(obj)),
+           "aladdin_rebalance")
+    return mv.value, obj[0], obj[1]
 
 
 def aladdin_cluster_advance(cl, dt_ms, stats=None):
@@ -357,6 +381,16 @@ class Cluster:
         pl = np.zeros(len(cin), np.int32)
         aladdin_place_round(self.handle, len(cin), cin, cpr, cw, pl)
         return pl
+
+    def rebalance(self, cand_in, cand_pred, wait_ms, placement, le, be):
+        """Host convenience for aladdin_rebalance (placement: int32 numpy array,
+        updated in place)."""
+        cin = np.ascontiguousarray(cand_in, np.int32)
+        cpr = np.ascontiguousarray(cand_pred, np.int32)
+        cw = None if wait_ms is None else np.ascontiguousarray(wait_ms, np.float32)
+        return aladdin_rebalance(self.handle, len(cin), cin, cpr, cw, placement,
+                                 np.ascontiguousarray(le, np.int64),
+                                 np.ascontiguousarray(be, np.int32))
 
     def advance(self, dt_ms):
         st = np.zeros(ADVANCE_STATS)

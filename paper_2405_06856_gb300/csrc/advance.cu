@@ -10,7 +10,12 @@
 // counted: TTFT above T_pre, ATGT above T_dec (each beyond SLO_TOL) and
 // decode iterations whose KV usage h * context + j * batch exceeds the
 // worker's capacity M (what a placement without a feasibility test, JSQ or
-// power of two, can cause).
+// power of two, can cause). With prediction errors (Sec. 4.3) a request runs
+// to its real length: one that reaches its prediction first is re-predicted
+// from the re-prediction table, one that finishes before its prediction
+// finishes early; both are Algorithm 2's error events (C.le, C.be). A lane
+// keeps each request's next event point min(real, pred) in registers and
+// reads the slot arrays only at events.
 // Times accumulate in fp64 with explicitly rounded operations, in the same
 // order as the CPU reference, so both sides produce the same schedule.
 #include "aladdin_host.h"
@@ -38,9 +43,11 @@ k_advance(DevParams P, ClusterDev C, double t_now, double dt, unsigned long long
     const double s = C.scaled[w];
     const double t_end = __dadd_rn(t_now, dt);
 
-    int in[E], gen[E], pred[E];
+    int in[E], gen[E], evt[E];  // evt: min(real, pred), the next event point
     double tdec[E];
-    bool alive[E];
+    unsigned alive = 0;  // bit e: element e holds a request
+    // events of one step: |le_acc| <= slots x iterations x K < 2^31
+    int le_acc = 0, be_acc = 0, nrep = 0, nearly = 0;
     long long Pint = 0;
     int npend = 0;
     double maxttft = 0.0, maxatgt = 0.0;
@@ -50,15 +57,15 @@ k_advance(DevParams P, ClusterDev C, double t_now, double dt, unsigned long long
 #pragma unroll
     for (int e = 0; e < E; ++e) {
         const int x = e * 32 + lane;
-        alive[e] = x < n;
+        if (x < n) alive |= 1u << e;
         in[e] = gen[e] = 0;
-        pred[e] = 1;
+        evt[e] = 1;
         tdec[e] = 0.0;
-        if (alive[e]) {
+        if (x < n) {
             const long long slot = base + x;
             in[e] = C.in[slot];
             gen[e] = C.gen[slot];
-            pred[e] = C.pred[slot];
+            evt[e] = min(C.pred[slot], C.real[slot]);
             tdec[e] = C.tdec[slot];
             if (C.pend[slot]) {
                 Pint += in[e];
@@ -72,7 +79,7 @@ k_advance(DevParams P, ClusterDev C, double t_now, double dt, unsigned long long
         // decode instance: the placements join the batch, nothing is stalled
 #pragma unroll
         for (int e = 0; e < E; ++e) {
-            if (!alive[e]) continue;
+            if (!((alive >> e) & 1u)) continue;
             if (C.pend[base + e * 32 + lane]) {
                 gen[e] = 0;
                 tdec[e] = 0.0;
@@ -83,7 +90,7 @@ k_advance(DevParams P, ClusterDev C, double t_now, double dt, unsigned long long
         const double lead = __dsub_rn(start, t_now);
 #pragma unroll
         for (int e = 0; e < E; ++e) {
-            if (!alive[e]) continue;
+            if (!((alive >> e) & 1u)) continue;
             const long long slot = base + e * 32 + lane;
             if (C.pend[slot]) {
                 const double ttft = __dadd_rn(__dadd_rn(C.wait[slot], lead), tau);
@@ -97,14 +104,14 @@ k_advance(DevParams P, ClusterDev C, double t_now, double dt, unsigned long long
         }
         start = __dadd_rn(start, tau);
     }
-    // Decode iterations (bounded: every iteration finishes at least one token
-    // of every active request, so at most max(pred) iterations run).
+    // Decode iterations (bounded: every iteration adds a token to every active
+    // request, so at most max(real) iterations run).
     for (;;) {
         int b = 0;
         long long K = 0;
 #pragma unroll
         for (int e = 0; e < E; ++e)
-            if (alive[e]) {
+            if ((alive >> e) & 1u) {
                 b += 1;
                 K += (long long)in[e] + gen[e] + 1;
             }
@@ -116,15 +123,33 @@ k_advance(DevParams P, ClusterDev C, double t_now, double dt, unsigned long long
             s, __dadd_rn(__dadd_rn(P.c3d, __dmul_rn(P.c2d, (double)b)), __dmul_rn(P.k2d, (double)K)));
 #pragma unroll
         for (int e = 0; e < E; ++e)
-            if (alive[e]) {
+            if ((alive >> e) & 1u) {
                 gen[e] += 1;
                 tdec[e] = __dadd_rn(tdec[e], t);
-                if (gen[e] >= pred[e]) {
-                    const double atgt = __ddiv_rn(tdec[e], (double)pred[e]);
-                    maxatgt = fmax(maxatgt, atgt);
-                    vatgt += atgt > P.T_dec_viol ? 1 : 0;
-                    nfin += 1;
-                    alive[e] = false;
+                if (gen[e] >= evt[e]) {
+                    const long long slot = base + e * 32 + lane;
+                    const int pr = C.pred[slot], rl = C.real[slot];
+                    if (gen[e] >= rl) {
+                        if (rl < pr) {  // finished before its prediction
+                            le_acc += rl - pr;
+                            be_acc -= 1;
+                            nearly += 1;
+                        }
+                        const double atgt = __ddiv_rn(tdec[e], (double)gen[e]);
+                        maxatgt = fmax(maxatgt, atgt);
+                        vatgt += atgt > P.T_dec_viol ? 1 : 0;
+                        nfin += 1;
+                        alive &= ~(1u << e);
+                    } else {  // reached its prediction unfinished: re-predict
+                        int np = C.repred ? C.repred[gen[e]] : gen[e] + 1;
+                        np = max(np, gen[e] + 1);
+                        if ((long long)in[e] + np > (long long)P.K) np = P.K - in[e];
+                        le_acc += np - pr;
+                        be_acc += 1;
+                        nrep += 1;
+                        C.pred[slot] = np;
+                        evt[e] = min(np, rl);
+                    }
                 }
             }
         start = __dadd_rn(start, t);
@@ -133,18 +158,24 @@ k_advance(DevParams P, ClusterDev C, double t_now, double dt, unsigned long long
     int pos = 0;
 #pragma unroll
     for (int e = 0; e < E; ++e) {
-        const unsigned bal = __ballot_sync(FULL, alive[e]);
+        const unsigned bal = __ballot_sync(FULL, (alive >> e) & 1u);
         const int before = __popc(bal & ((1u << lane) - 1u));
         const long long src = base + e * 32 + lane;
         // read the fields that are not kept in registers before any write
         double wt = 0.0;
-        if (alive[e]) wt = C.wait[src];
+        int pr = 1, rl = 1;
+        if ((alive >> e) & 1u) {
+            wt = C.wait[src];
+            pr = C.pred[src];
+            rl = C.real[src];
+        }
         __syncwarp();
-        if (alive[e]) {
+        if ((alive >> e) & 1u) {
             const long long dst = base + pos + before;
             C.in[dst] = in[e];
             C.gen[dst] = gen[e];
-            C.pred[dst] = pred[e];
+            C.pred[dst] = pr;
+            C.real[dst] = rl;
             C.tdec[dst] = tdec[e];
             C.pend[dst] = 0;
             C.wait[dst] = wt;
@@ -157,8 +188,16 @@ k_advance(DevParams P, ClusterDev C, double t_now, double dt, unsigned long long
     nfin = warp_reduce(nfin, OpAdd<unsigned long long>());
     vttft = warp_reduce(vttft, OpAdd<unsigned long long>());
     vatgt = warp_reduce(vatgt, OpAdd<unsigned long long>());
+    le_acc = warp_reduce(le_acc, OpAdd<int>());
+    be_acc = warp_reduce(be_acc, OpAdd<int>());
+    nrep = warp_reduce(nrep, OpAdd<int>());
+    nearly = warp_reduce(nearly, OpAdd<int>());
     if (lane == 0) {
         C.n[w] = pos;
+        if (le_acc || be_acc) {  // one warp per worker: no other writer
+            C.le[w] += (long long)le_acc;
+            C.be[w] += be_acc;
+        }
         C.clock[w] = start;
         C.off[w] = start > t_end ? (float)__dsub_rn(start, t_end) : 0.0f;
         if (stats) {
@@ -169,6 +208,8 @@ k_advance(DevParams P, ClusterDev C, double t_now, double dt, unsigned long long
             if (vttft) atomicAdd(&stats[4], vttft);
             if (vatgt) atomicAdd(&stats[5], vatgt);
             if (vkv) atomicAdd(&stats[6], vkv);
+            if (nrep) atomicAdd(&stats[7], (unsigned long long)nrep);
+            if (nearly) atomicAdd(&stats[8], (unsigned long long)nearly);
         }
         const unsigned long long v = vttft + vatgt + vkv;
         if (fail && v) atomicAdd(fail, v);

@@ -110,6 +110,12 @@ struct ClusterDev {
                                // written by every table build
     float2* wapx;              // [W] approximate mode: prompt bounds of (d) and of (b)
                                // before the candidate's gamma * l_pred
+    int32_t* real;             // [W*cap] real output length (= pred unless a trace
+                               // carries prediction errors)
+    long long* le;             // [W] Algorithm 2's output-length error l^e
+    int32_t* be;               // [W] Algorithm 2's batch-size error b^e
+    double* err_e;             // [W] Algorithm 2's scratch: k2 l^e + c2 b^e
+    const int32_t* repred;     // [K+1] re-prediction table, or nullptr (x + 1)
 };
 
 // Table row p of a worker (2 x float4, 32 bytes) and its side entry:

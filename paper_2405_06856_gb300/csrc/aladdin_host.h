@@ -56,6 +56,13 @@ struct RoundIO {
     void* xbuf;
     // power-of-two draws: request id of direct-mode candidate c is rid0 + c
     long long rid0;
+    // trace mode: real output lengths (nullable: exact predictions), and, when
+    // sim_pl is set, every candidate's placement (-1 none, -2 invalid), trace
+    // index and the candidate count, for Algorithm 2 after the round
+    const int32_t* treal;
+    int32_t* sim_pl;
+    long long* sim_tix;
+    int* sim_n;
 };
 constexpr int ROUND_XBUF_SMS = 1024;  // largest SM count the exchange buffer serves
 constexpr size_t ROUND_XBUF_BYTES = 32 * (size_t)ROUND_XBUF_SMS + 16;
@@ -65,10 +72,12 @@ cudaError_t launch_round(const DevParams& P, const ClusterDev& C, const RoundIO&
 // Execution of every worker for dt ms from t_now.
 // stats: device [0] prefills run, [1] finished, [2] max TTFT bits, [3] max
 // ATGT bits (non-negative doubles compare like their bit patterns), realized
-// violations [4] TTFT, [5] ATGT, [6] KV-overflow iterations. halt (device,
-// nullable): nothing runs when *halt != 0. fail (device, nullable): every
-// violation is also added to it (the simulation's failure counter).
-constexpr int STATS_N = 7;
+// violations [4] TTFT, [5] ATGT, [6] KV-overflow iterations, prediction-error
+// events [7] re-predictions, [8] early finishes. halt (device, nullable):
+// nothing runs when *halt != 0. fail (device, nullable): every violation is
+// also added to it (the simulation's failure counter). Each worker's error
+// events are added to C.le / C.be.
+constexpr int STATS_N = 9;
 cudaError_t launch_advance(const DevParams& P, const ClusterDev& C, double t_now, double dt,
                            unsigned long long* stats, const int* halt, cudaStream_t st,
                            unsigned long long* fail = nullptr);
@@ -78,6 +87,15 @@ cudaError_t launch_advance(const DevParams& P, const ClusterDev& C, double t_now
 // without a feasibility test. Tables are not rebuilt.
 cudaError_t launch_round_queue(const DevParams& P, const ClusterDev& C, const RoundIO& io,
                                cudaStream_t st);
+
+// Algorithm 2 over one round's placements. Direct mode (io.sim == 0): the
+// candidates io.in / io.pred / io.wait (io.n_cand) and io.placement (updated);
+// trace mode: io.sim_pl / io.sim_tix / *io.sim_n with the trace arrays and
+// io.t_now. Errors from C.le / C.be; moves (device, nullable) receives the
+// number of moves and obj (device, nullable, 2 doubles) the summed distance
+// before and after. Tables of the two workers of every move are rebuilt.
+cudaError_t launch_rebalance(const DevParams& P, const ClusterDev& C, const RoundIO& io,
+                             int* moves, double* obj, cudaStream_t st);
 
 // Exact integer sums over a trace for the worker-configuration model:
 // sums[0] = sum of predicted outputs (decode iterations), sums[1] = sum over

@@ -93,6 +93,7 @@ int check_params(const aladdin_params* p)
     if (p->policy != ALADDIN_POLICY_BESTFIT && p->policy != ALADDIN_POLICY_JSQ &&
         p->policy != ALADDIN_POLICY_PO2)
         return ALADDIN_ERR_ARG;
+    if (p->rebalance != 0 && p->rebalance != 1) return ALADDIN_ERR_ARG;
     return ALADDIN_OK;
 }
 
@@ -268,6 +269,11 @@ int cluster_alloc(aladdin_cluster* cl, const aladdin_params& p, int W,
     AL(novf, int, 1);
     AL(skey, uint32_t, slots);
     AL(wapx, float2, W);
+    AL(real, int32_t, slots);
+    AL(le, long long, W);
+    AL(be, int32_t, W);
+    AL(err_e, double, W);
+    d.repred = nullptr;
 #undef AL
     CK(cl->alloc(&p0, sizeof(unsigned long long) * STATS_N));
     cl->d_stats = (unsigned long long*)p0;
@@ -291,6 +297,8 @@ int cluster_alloc(aladdin_cluster* cl, const aladdin_params& p, int W,
     CK(cudaMemsetAsync(d.pend, 0, slots, st));
     CK(cudaMemsetAsync(d.wrec, 0, sizeof(float4) * W, st));
     CK(cudaMemsetAsync(d.err, 0, sizeof(unsigned int), st));
+    CK(cudaMemsetAsync(d.le, 0, sizeof(long long) * W, st));
+    CK(cudaMemsetAsync(d.be, 0, sizeof(int32_t) * W, st));
     CK(cudaMemsetAsync(cl->d_stats, 0, sizeof(unsigned long long) * STATS_N, st));
     CK(cudaMemsetAsync(cl->d_status, 0, sizeof(int) * 4, st));
     // host vectors above must outlive the async copies
@@ -365,6 +373,8 @@ int load_requests_host(aladdin_cluster* cl, const int32_t* req_off, const int32_
     CK(cudaMemcpyAsync(d.in, si.data(), sizeof(int32_t) * slots, cudaMemcpyHostToDevice, cl->st));
     CK(cudaMemcpyAsync(d.gen, sg.data(), sizeof(int32_t) * slots, cudaMemcpyHostToDevice, cl->st));
     CK(cudaMemcpyAsync(d.pred, sp.data(), sizeof(int32_t) * slots, cudaMemcpyHostToDevice, cl->st));
+    // a cluster built from requests holds exact predictions: real = pred
+    CK(cudaMemcpyAsync(d.real, sp.data(), sizeof(int32_t) * slots, cudaMemcpyHostToDevice, cl->st));
     CK(cudaMemcpyAsync(d.tdec, stdec.data(), sizeof(double) * slots, cudaMemcpyHostToDevice, cl->st));
     CK(cudaMemsetAsync(d.pend, 0, slots, cl->st));
     CK(cudaStreamSynchronize(cl->st));
@@ -390,9 +400,11 @@ __global__ void k_pack(DevParams P, ClusterDev C, const int32_t* __restrict__ of
     for (int q = lane; q < n; q += 32) {
         const long long dst = base + q;
         const int g = gen[a + q];
+        const int32_t pr = pred[a + q];
         C.in[dst] = in[a + q];
         C.gen[dst] = g;
-        C.pred[dst] = pred[a + q];
+        C.pred[dst] = pr;
+        C.real[dst] = pr;  // exact predictions
         C.tdec[dst] = tdec ? (double)tdec[a + q] : P.thetad * P.T_decd * (double)g;
         C.pend[dst] = 0;
     }
@@ -401,6 +413,7 @@ __global__ void k_pack(DevParams P, ClusterDev C, const int32_t* __restrict__ of
             C.in[base] = -1;
             C.gen[base] = 0;
             C.pred[base] = 1;
+            C.real[base] = 1;
             C.tdec[base] = 0.0;
             C.pend[base] = 0;
             atomicOr(C.err, 2u);
@@ -639,6 +652,66 @@ int aladdin_place_round(aladdin_cluster* cl, int32_t n_cand, const int32_t* in,
     return status == -2 ? ALADDIN_ERR_CAPACITY : ALADDIN_OK;
 }
 
+int aladdin_rebalance(aladdin_cluster* cl, int32_t n_cand, const int32_t* in,
+                      const int32_t* pred, const float* wait_ms, int32_t* placement,
+                      const int64_t* le, const int32_t* be, int32_t* moves, double* obj)
+{
+    if (!cl || n_cand < 0) return ALADDIN_ERR_ARG;
+    if (!le || !be) return ALADDIN_ERR_ARG;
+    if (n_cand > 0 && (!in || !pred || !placement)) return ALADDIN_ERR_ARG;
+    CK(cudaSetDevice(cl->device));
+    const size_t C = (size_t)(n_cand > 0 ? n_cand : 1);
+    const int32_t *din = nullptr, *dpred = nullptr;
+    const float* dwait = nullptr;
+    int rc;
+    if (n_cand > 0 &&
+        ((rc = stage_in(cl, cl->s_in, in, C, &din)) || (rc = stage_in(cl, cl->s_pred, pred, C, &dpred)) ||
+         (rc = stage_in(cl, cl->s_wait, wait_ms, C, &dwait))))
+        return rc;
+    // placement is read and written: device (or mapped) memory in place, else staged
+    int32_t* dpl = nullptr;
+    bool hpl = false;
+    if (n_cand > 0 && !device_view(placement, &dpl)) {
+        CK(cl->s_place.ensure(sizeof(int32_t) * C));
+        dpl = cl->s_place.as<int32_t>();
+        CK(cudaMemcpyAsync(dpl, placement, sizeof(int32_t) * C, cudaMemcpyHostToDevice, cl->st));
+        hpl = true;
+    }
+    const size_t W = (size_t)cl->W;
+    CK(cudaMemcpyAsync(cl->dev.le, le, sizeof(long long) * W, cudaMemcpyDefault, cl->st));
+    CK(cudaMemcpyAsync(cl->dev.be, be, sizeof(int32_t) * W, cudaMemcpyDefault, cl->st));
+    DevBuf res;
+    CK(res.ensure(sizeof(double) * 2 + sizeof(int)));
+    double* dobj = res.as<double>();
+    int* dmov = reinterpret_cast<int*>(dobj + 2);
+    CK(cudaMemsetAsync(dmov, 0, sizeof(int), cl->st));
+    RoundIO io;
+    std::memset(&io, 0, sizeof(io));
+    io.in = din;
+    io.pred = dpred;
+    io.wait = dwait;
+    io.n_cand = n_cand;
+    io.placement = dpl;
+    io.status = cl->d_status;
+    CK(launch_rebalance(cl->dp, cl->dev, io, dmov, dobj, cl->st));
+    CK(launch_rank(cl->dev, cl->st));
+    CK(cudaMemsetAsync(cl->dev.le, 0, sizeof(long long) * W, cl->st));
+    CK(cudaMemsetAsync(cl->dev.be, 0, sizeof(int32_t) * W, cl->st));
+    if (hpl) CK(cudaMemcpyAsync(placement, dpl, sizeof(int32_t) * C, cudaMemcpyDeviceToHost, cl->st));
+    double ho[2] = {0.0, 0.0};
+    int hm = 0;
+    CK(cudaMemcpyAsync(ho, dobj, sizeof(ho), cudaMemcpyDeviceToHost, cl->st));
+    CK(cudaMemcpyAsync(&hm, dmov, sizeof(int), cudaMemcpyDeviceToHost, cl->st));
+    CK(cudaStreamSynchronize(cl->st));
+    res.release();
+    if (moves) *moves = hm;
+    if (obj) {
+        obj[0] = ho[0];
+        obj[1] = ho[1];
+    }
+    return ALADDIN_OK;
+}
+
 int aladdin_cluster_advance(aladdin_cluster* cl, double dt_ms, double* stats)
 {
     if (!cl || !(std::isfinite(dt_ms) && dt_ms >= 0)) return ALADDIN_ERR_ARG;
@@ -738,12 +811,16 @@ struct DevTrace {
     double* t = nullptr;
     int32_t* in = nullptr;
     int32_t* pred = nullptr;
+    int32_t* real = nullptr;    // nullptr: exact predictions
+    int32_t* repred = nullptr;  // nullptr: re-predict x + 1
     std::vector<double> host_t;
     ~DevTrace()
     {
         if (t) cudaFree(t);
         if (in) cudaFree(in);
         if (pred) cudaFree(pred);
+        if (real) cudaFree(real);
+        if (repred) cudaFree(repred);
     }
 };
 
@@ -758,6 +835,8 @@ int upload_trace(const aladdin_params& p, const aladdin_trace* tr, DevTrace& d, 
             return ALADDIN_ERR_ARG;
         if (tr->in[i] < 0 || tr->pred[i] < 1 || (long long)tr->in[i] + tr->pred[i] > p.K)
             return ALADDIN_ERR_ARG;
+        if (tr->real && (tr->real[i] < 1 || (long long)tr->in[i] + tr->real[i] > p.K))
+            return ALADDIN_ERR_ARG;
     }
     const size_t n = (size_t)(tr->n > 0 ? tr->n : 1);
     CK(cudaMalloc(&d.t, sizeof(double) * n));
@@ -767,6 +846,16 @@ int upload_trace(const aladdin_params& p, const aladdin_trace* tr, DevTrace& d, 
         CK(cudaMemcpyAsync(d.t, tr->t_arr_ms, sizeof(double) * tr->n, cudaMemcpyHostToDevice, st));
         CK(cudaMemcpyAsync(d.in, tr->in, sizeof(int32_t) * tr->n, cudaMemcpyHostToDevice, st));
         CK(cudaMemcpyAsync(d.pred, tr->pred, sizeof(int32_t) * tr->n, cudaMemcpyHostToDevice, st));
+        if (tr->real) {
+            CK(cudaMalloc(&d.real, sizeof(int32_t) * n));
+            CK(cudaMemcpyAsync(d.real, tr->real, sizeof(int32_t) * tr->n, cudaMemcpyHostToDevice,
+                               st));
+        }
+    }
+    if (tr->repred) {
+        CK(cudaMalloc(&d.repred, sizeof(int32_t) * ((size_t)p.K + 1)));
+        CK(cudaMemcpyAsync(d.repred, tr->repred, sizeof(int32_t) * ((size_t)p.K + 1),
+                           cudaMemcpyHostToDevice, st));
     }
     CK(cudaStreamSynchronize(st));
     return ALADDIN_OK;
@@ -780,7 +869,7 @@ __global__ void k_busy(const int32_t* __restrict__ n, int W, int* out)
     if (threadIdx.x == 0) *out = any;
 }
 
-// One simulation; out[0..5] as aladdin_simulate.
+// One simulation; out[0..8] as aladdin_simulate.
 int simulate_impl(const aladdin_params& p, const aladdin_worker_cfg& cfg, int32_t N,
                   const DevTrace& tr, double H, bool stop_at_fail, bool drain, cudaStream_t st,
                   double* out)
@@ -791,13 +880,21 @@ int simulate_impl(const aladdin_params& p, const aladdin_worker_cfg& cfg, int32_
     if (rc) return rc;
     rc = refresh_tables(&cl);
     if (rc) return rc;
-    DevBuf wl, cnt;
+    cl.dev.repred = tr.repred;  // the kernels get the cluster view by value
+    const bool rebal = p.rebalance != 0 && p.policy == ALADDIN_POLICY_BESTFIT;
+    DevBuf wl, cnt, rpl, rtix;
     CK(wl.ensure(sizeof(long long) * (size_t)(tr.n > 0 ? tr.n : 1)));
     CK(cnt.ensure(sizeof(unsigned long long) * 4 + sizeof(int) * 4));
     unsigned long long* counters = cnt.as<unsigned long long>();
     int* nwait = reinterpret_cast<int*>(counters + 4);
     int* busy = nwait + 1;
+    int* rb_n = nwait + 2;      // candidates of the last round (Algorithm 2)
+    int* rb_moves = nwait + 3;  // requests moved by Algorithm 2
     CK(cudaMemsetAsync(cnt.p, 0, sizeof(unsigned long long) * 4 + sizeof(int) * 4, st));
+    if (rebal) {
+        CK(rpl.ensure(sizeof(int32_t) * (size_t)(tr.n > 0 ? tr.n : 1)));
+        CK(rtix.ensure(sizeof(long long) * (size_t)(tr.n > 0 ? tr.n : 1)));
+    }
 
     int64_t next = 0;
     long long hb = 0;
@@ -824,9 +921,22 @@ int simulate_impl(const aladdin_params& p, const aladdin_worker_cfg& cfg, int32_
         io.stop_at_fail = stop_at_fail ? 1 : 0;
         io.hb = hb;
         io.xbuf = cl.d_xround;
+        io.treal = tr.real;
+        if (rebal) {
+            io.sim_pl = rpl.as<int32_t>();
+            io.sim_tix = rtix.as<long long>();
+            io.sim_n = rb_n;
+        }
         const bool bestfit = p.policy == ALADDIN_POLICY_BESTFIT;
         if (bestfit) CK(launch_round(cl.dp, cl.dev, io, st));
         else CK(launch_round_queue(cl.dp, cl.dev, io, st));
+        if (rebal) {
+            // Algorithm 2 on the errors recorded since the previous heartbeat,
+            // which then restart from zero
+            CK(launch_rebalance(cl.dp, cl.dev, io, rb_moves, nullptr, st));
+            CK(cudaMemsetAsync(cl.dev.le, 0, sizeof(long long) * (size_t)cl.W, st));
+            CK(cudaMemsetAsync(cl.dev.be, 0, sizeof(int32_t) * (size_t)cl.W, st));
+        }
         next = end;
         // realized violations count as failures (counters[0])
         CK(launch_advance(cl.dp, cl.dev, t, H, cl.d_stats, cl.d_status, st, counters));
@@ -852,8 +962,10 @@ int simulate_impl(const aladdin_params& p, const aladdin_worker_cfg& cfg, int32_
         }
     }
     unsigned long long s[STATS_N];
+    int hm[2] = {0, 0};
     CK(cudaMemcpyAsync(s, cl.d_stats, sizeof(s), cudaMemcpyDeviceToHost, st));
     CK(cudaMemcpyAsync(hc, counters, sizeof(hc), cudaMemcpyDeviceToHost, st));
+    CK(cudaMemcpyAsync(hm, rb_n, sizeof(hm), cudaMemcpyDeviceToHost, st));
     CK(cudaStreamSynchronize(st));
     out[0] = (double)hc[0];
     out[1] = (double)hc[1];
@@ -861,6 +973,11 @@ int simulate_impl(const aladdin_params& p, const aladdin_worker_cfg& cfg, int32_
     std::memcpy(&out[3], &s[2], 8);
     std::memcpy(&out[4], &s[3], 8);
     out[5] = (double)(s[4] + s[5] + s[6]);
+    out[6] = (double)s[7];
+    out[7] = (double)s[8];
+    out[8] = (double)hm[1];
+    rpl.release();
+    rtix.release();
     wl.release();
     cnt.release();
     return ALADDIN_OK;
@@ -874,7 +991,7 @@ int search_min_workers(const aladdin_params& p, const aladdin_worker_cfg& cfg, c
     // JSQ and power of two admit without a test: drain to realize every
     // request's latencies
     const bool drain = p.policy != ALADDIN_POLICY_BESTFIT;
-    double out[6];
+    double out[9];
     int rc;
     int32_t lo = 0, hi = 1;
     bool found = false;

@@ -121,6 +121,7 @@ __global__ void __launch_bounds__(Q_THREADS) k_round_queue(DevParams P, ClusterD
                 C.in[slot] = a;
                 C.gen[slot] = 0;
                 C.pred[slot] = r;
+                C.real[slot] = io.sim && io.treal ? io.treal[tix] : r;
                 C.tdec[slot] = 0.0;
                 C.pend[slot] = 1;
                 C.wait[slot] = wd;

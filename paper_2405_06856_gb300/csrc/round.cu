@@ -49,16 +49,18 @@ __global__ void __launch_bounds__(ROUND_THREADS) k_round(DevParams P, ClusterDev
 
     for (int c = 0; c < n_cand; ++c) {
         long long tix = 0;
-        int32_t a, r;
+        int32_t a, r, rl;
         double wd;
         if (io.sim) {
             tix = c < n_wait0 ? io.wl[c] : io.arr_begin + (c - n_wait0);
             a = io.tin[tix];
             r = io.tpred[tix];
+            rl = io.treal ? io.treal[tix] : r;
             wd = io.t_now - io.t_arr[tix];
         } else {
             a = io.in[c];
             r = io.pred[c];
+            rl = r;
             wd = io.wait ? (double)io.wait[c] : 0.0;
         }
         const CandRec cr = make_cand(P, a, r, (float)wd, c);
@@ -110,6 +112,7 @@ __global__ void __launch_bounds__(ROUND_THREADS) k_round(DevParams P, ClusterDev
                     C.in[slot] = a;
                     C.gen[slot] = 0;
                     C.pred[slot] = r;
+                    C.real[slot] = rl;
                     C.tdec[slot] = 0.0;
                     C.pend[slot] = 1;
                     C.wait[slot] = wd;
@@ -125,6 +128,10 @@ __global__ void __launch_bounds__(ROUND_THREADS) k_round(DevParams P, ClusterDev
             }
         }
         if (tid == 0 && !sm.stop) {
+            if (io.sim && io.sim_pl) {
+                io.sim_pl[c] = winner;
+                io.sim_tix[c] = tix;
+            }
             if (!io.sim) {
                 io.placement[c] = winner;
             } else if (winner >= 0) {
@@ -145,6 +152,7 @@ __global__ void __launch_bounds__(ROUND_THREADS) k_round(DevParams P, ClusterDev
         }
     }
     if (tid == 0 && io.sim && !sm.stop) {
+        if (io.sim_n) *io.sim_n = n_cand;
         *io.n_wait = keep;
         if (io.stop_at_fail && io.counters[0] > 0) {
             *io.status = 1;
@@ -330,7 +338,7 @@ __global__ void __launch_bounds__(R2_THREADS, 1) k_round2(R2Args A)
     const int n_cand = io.sim ? n_wait0 + (int)(io.arr_end - io.arr_begin) : io.n_cand;
     int keep = 0;        // CTA 0 thread 0: new waiting-list length
     int pend_w = -1;     // this slice's winner of the previous step, not yet appended
-    int32_t pa = 0, pr = 0;
+    int32_t pa = 0, pr = 0, prl = 0;
     double pwd = 0.0;    // its request
 
     auto append = [&](int w) {  // rebuild group: commit the owed request to w
@@ -341,6 +349,7 @@ __global__ void __launch_bounds__(R2_THREADS, 1) k_round2(R2Args A)
             C.in[slot] = pa;
             C.gen[slot] = 0;
             C.pred[slot] = pr;
+            C.real[slot] = prl;
             C.tdec[slot] = 0.0;
             C.pend[slot] = 1;
             C.wait[slot] = pwd;
@@ -353,16 +362,18 @@ __global__ void __launch_bounds__(R2_THREADS, 1) k_round2(R2Args A)
     for (int c = 0; c < n_cand; ++c) {
         const int par = c & 1;
         long long tix = 0;
-        int32_t a, r;
+        int32_t a, r, rl;
         double wd;
         if (io.sim) {
             tix = c < n_wait0 ? io.wl[c] : io.arr_begin + (c - n_wait0);
             a = io.tin[tix];
             r = io.tpred[tix];
+            rl = io.treal ? io.treal[tix] : r;
             wd = io.t_now - io.t_arr[tix];
         } else {
             a = io.in[c];
             r = io.pred[c];
+            rl = r;
             wd = io.wait ? (double)io.wait[c] : 0.0;
         }
         const CandRec cr = make_cand(P, a, r, (float)wd, c);
@@ -473,8 +484,13 @@ __global__ void __launch_bounds__(R2_THREADS, 1) k_round2(R2Args A)
         pend_w = (winner >= w_lo && winner < w_lo + nloc) ? winner : -1;
         pa = a;
         pr = r;
+        prl = rl;
         pwd = wd;
         if (g == 0 && tid == 0) {
+            if (io.sim && io.sim_pl) {
+                io.sim_pl[c] = winner;
+                io.sim_tix[c] = tix;
+            }
             if (!io.sim) {
                 io.placement[c] = winner;
             } else if (winner >= 0) {
@@ -497,6 +513,7 @@ __global__ void __launch_bounds__(R2_THREADS, 1) k_round2(R2Args A)
                                 &sc, nullptr);
     }
     if (g == 0 && tid == 0 && io.sim && !sm.stop && *io.status == 0) {
+        if (io.sim_n) *io.sim_n = n_cand;
         *io.n_wait = keep;
         if (io.stop_at_fail && io.counters[0] > 0) {
             *io.status = 1;
