@@ -644,10 +644,39 @@ def worker_model(A, synth, stream, trace_n=100_000, fit_n=20_000,
     return out
 
 
+def prediction_errors(A, synth, stream, n_requests=100_000, n_workers=133,
+                      sigmas=(0.3, 0.6)):
+    """Algorithm 2 under prediction errors (Sec. 4.3): the diurnal trace with
+    predictions off by a lognormal factor exp(N(0, sigma)), served by best-fit
+    on a fixed fleet of 1-GPU workers (the count the exact-prediction search
+    needs) with and without re-balancing; realized violations (ATGT above
+    T_dec, KV above capacity, TTFT above T_pre) and requests moved."""
+    tr = synth.diurnal_trace(4, n_requests, 2000.0, 500.0)
+    out = {"workload": "diurnal trace of %d requests, %d 1-GPU workers (%d KV tokens), "
+                       "best-fit" % (n_requests, n_workers, MW_KV_PER_GPU)}
+    cfg = A.make_cfgs([1], [MW_KV_PER_GPU], [1.0])[0]
+    for sigma in sigmas:
+        te = synth.with_prediction_error(tr, sigma, 7)
+        row = {}
+        for rb in (0, 1):
+            p = dict(synth.BASE_PARAMS, rebalance=rb)
+            res = np.zeros(A.SIMULATE_OUT)
+            t0 = time.perf_counter()
+            A.aladdin_simulate(A.make_params(p, MW_B_CAP), cfg, n_workers, A.trace_of(te), 100.0,
+                               0, 1, res, stream=stream)
+            row["rebalance" if rb else "no_rebalance"] = {
+                "failed": int(res[0]), "violations": int(res[5]), "max_atgt_ms": round(res[4], 3),
+                "repredictions": int(res[6]), "early_finishes": int(res[7]),
+                "moved": int(res[8]), "sim_s": round(time.perf_counter() - t0, 2)}
+        out["sigma_%g" % sigma] = row
+    return out
+
+
 def run_policies(args):
     """Best-fit against JSQ and the power of two choices (Sec. 6.4): GPUs each
     needs, mixed setting and decode instances, on a 100,000-request trace; the
-    worker-configuration picker and the fitted worker-count model."""
+    worker-configuration picker and the fitted worker-count model; Algorithm 2
+    under prediction errors."""
     import torch
     from paper_2405_06856_gb300 import build as B
     B.build()
@@ -658,6 +687,7 @@ def run_policies(args):
     t0 = time.perf_counter()
     res = policy_compare(A, synth, stream, 100_000, [1, 2, 4, 8])
     res["worker_model"] = worker_model(A, synth, stream)
+    res["prediction_errors"] = prediction_errors(A, synth, stream)
     res["mode"] = "policies"
     res["wall_s"] = round(time.perf_counter() - t0, 1)
     print(json.dumps(res))
