@@ -372,30 +372,19 @@ __global__ void __launch_bounds__(SCORE_WARPS * 32, PEND ? 3 : ALADDIN_SCORE_MIN
                 for (int s = 1; s < SLOTS; ++s) nb = min(nb, ss[s].rnext);
                 have_rows = true;
             }
-            const float4* q = cs;
-            unsigned* kslot = &sm.kmin[warp][0];
-            for (int i = 0; i < nc; ++i, q += REC_F4, ++kslot) {
-                const float4 q4 = q[2];
-                const int ri = __float_as_int(q4.x);
-                const unsigned long long off =
-                    ((unsigned long long)__float_as_uint(q4.w) << 32) | __float_as_uint(q4.z);
-                if (ri == 0) {  // invalid candidate (warp-uniform)
-                    if (live) {
-#pragma unroll
-                        for (int s = 0; s < SLOTS; ++s) {
-                            if (SF) fbase[off + s] = 0x80;
-                            if (SMG) mbase[off + s] = __int_as_float(0x7fc00000);
-                        }
-                    }
-                    if (ARG) *kslot = 0xffffffffu;
-                    continue;
-                }
+            unsigned* const kbase = &sm.kmin[warp][0];
+            auto rec_off = [&](int i) {  // start of candidate i's output row
+                const float4 q4 = cs[i * REC_F4 + 2];
+                return ((unsigned long long)__float_as_uint(q4.w) << 32) | __float_as_uint(q4.z);
+            };
+            auto rec_ri = [&](int i) { return __float_as_int(cs[i * REC_F4 + 2].x); };
+            // Step every slot to the row whose segment holds ri (when some lane
+            // of the warp needs it); the next row is in L1 already, the one
+            // after is fetched now and needed only at the next crossing.
+            auto step_rows = [&](int ri) {
                 if (__any_sync(FULL, ri >= nb)) {
 #pragma unroll
                     for (int s = 0; s < SLOTS; ++s) {
-                        // step to the row whose segment holds ri; the next row
-                        // is already in registers, the one after is fetched
-                        // now and needed only at the next crossing
                         while (ri >= ss[s].rnext && p[s] < last_row) {
                             p[s] += 1;
                             const long long rb = (long long)wk[s] * A.C.rows;
@@ -415,11 +404,14 @@ __global__ void __launch_bounds__(SCORE_WARPS * 32, PEND ? 3 : ALADDIN_SCORE_MIN
 #pragma unroll
                     for (int s = 1; s < SLOTS; ++s) nb = min(nb, ss[s].rnext);
                 }
-                const float4 q0 = q[0], q1 = q[1];
+            };
+            // The group headrooms and margins of candidate i on this lane's
+            // workers (current rows), and its argbest key.
+            auto eval = [&](int i, float (&d)[4][SLOTS], float (&m)[SLOTS], unsigned& kmin) {
+                const float4 q0 = cs[i * REC_F4], q1 = cs[i * REC_F4 + 1];
                 const float a = q0.x, r = q0.y, ir = q0.z, Ua = q0.w;
                 const float id1 = q1.x, nX = q1.y, id2 = q1.z, Zc = q1.w;
-                float d[4][SLOTS], m[SLOTS];
-                unsigned kmin = 0xffffffffu;
+                kmin = 0xffffffffu;
 #pragma unroll
                 for (int s = 0; s < SLOTS; ++s) {
                     const Slot<PEND>& t = ss[s];
@@ -444,21 +436,69 @@ __global__ void __launch_bounds__(SCORE_WARPS * 32, PEND ? 3 : ALADDIN_SCORE_MIN
                     m[s] = fminf(fminf(d[0][s], d[1][s]), fminf(d[2][s], d[3][s]));
                     if (ARG) kmin = min(kmin, (__float_as_uint(m[s]) & 0x80000000u) | rank[s]);
                 }
+            };
+            auto store = [&](int i, const float (&d)[4][SLOTS], const float (&m)[SLOTS]) {
+                if (!live) return;
+                const unsigned long long off = rec_off(i);
+                if (SF) {
+                    const unsigned f = pack_flags<SLOTS>(d);
+                    if (SLOTS == 4) st_out(reinterpret_cast<unsigned int*>(fbase + off), f);
+                    else st_out(reinterpret_cast<unsigned short*>(fbase + off), (unsigned short)f);
+                }
+                if (SMG) {
+                    if (SLOTS == 4)
+                        st_out(reinterpret_cast<float4*>(mbase + off),
+                               make_float4(m[0], m[1], m[2 % SLOTS], m[3 % SLOTS]));
+                    else
+                        st_out(reinterpret_cast<float2*>(mbase + off), make_float2(m[0], m[1]));
+                }
+            };
+            auto score_one = [&](int i) {
+                float d[4][SLOTS], m[SLOTS];
+                unsigned kmin;
+                eval(i, d, m, kmin);
+                store(i, d, m);
+                if (ARG) kbase[i] = __reduce_min_sync(FULL, kmin);  // same value from every lane
+            };
+
+            // invalid candidates sort first (bucket 0): a prefix of the chunk
+            int i = 0;
+            for (; i < nc && rec_ri(i) == 0; ++i) {  // warp-uniform
                 if (live) {
-                    if (SF) {
-                        const unsigned f = pack_flags<SLOTS>(d);
-                        if (SLOTS == 4) st_out(reinterpret_cast<unsigned int*>(fbase + off), f);
-                        else st_out(reinterpret_cast<unsigned short*>(fbase + off), (unsigned short)f);
-                    }
-                    if (SMG) {
-                        if (SLOTS == 4)
-                            st_out(reinterpret_cast<float4*>(mbase + off),
-                                   make_float4(m[0], m[1], m[2 % SLOTS], m[3 % SLOTS]));
-                        else
-                            st_out(reinterpret_cast<float2*>(mbase + off), make_float2(m[0], m[1]));
+                    const unsigned long long off = rec_off(i);
+#pragma unroll
+                    for (int s = 0; s < SLOTS; ++s) {
+                        if (SF) fbase[off + s] = 0x80;
+                        if (SMG) mbase[off + s] = __int_as_float(0x7fc00000);
                     }
                 }
-                if (ARG) *kslot = __reduce_min_sync(FULL, kmin);  // same value from every lane
+                if (ARG) kbase[i] = 0xffffffffu;
+            }
+            // two candidates at a time on the same rows (independent chains the
+            // scheduler interleaves); one at a time where a breakpoint lies
+            // between them
+            for (; i + 1 < nc; i += 2) {
+                step_rows(rec_ri(i));
+                if (__any_sync(FULL, rec_ri(i + 1) >= nb)) {
+                    score_one(i);
+                    step_rows(rec_ri(i + 1));
+                    score_one(i + 1);
+                } else {
+                    float d0[4][SLOTS], m0[SLOTS], d1[4][SLOTS], m1[SLOTS];
+                    unsigned k0, k1;
+                    eval(i, d0, m0, k0);
+                    eval(i + 1, d1, m1, k1);
+                    store(i, d0, m0);
+                    store(i + 1, d1, m1);
+                    if (ARG) {
+                        kbase[i] = __reduce_min_sync(FULL, k0);
+                        kbase[i + 1] = __reduce_min_sync(FULL, k1);
+                    }
+                }
+            }
+            if (i < nc) {
+                step_rows(rec_ri(i));
+                score_one(i);
             }
         } else if (ARG) {
             for (int i = lane; i < nc; i += 32) sm.kmin[warp][i] = 0xffffffffu;
