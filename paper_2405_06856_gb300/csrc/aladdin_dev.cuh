@@ -61,6 +61,8 @@ struct DevParams {
     double k1d, c1d, k2d, c2d, c3d, T_pred, T_decd, gammad, thetad;
     // realized latencies above these count as SLO violations (execution)
     double T_pre_viol, T_dec_viol;
+    int32_t want_aux;        // 1: table builds also write the exact aggregates (AuxRow)
+                             // that only the verification outputs read
     int32_t decode;          // 1: decode instance of split-phase inference (no prefill)
     int32_t policy;          // ALADDIN_POLICY_* of placement rounds
     unsigned long long seed; // SplitMix64 seed of the power-of-two draws
@@ -503,13 +505,14 @@ __device__ __forceinline__ RowVals make_row(const DevParams& P, float inv_s, int
     return o;
 }
 
-__device__ __forceinline__ void store_row(const ClusterDev& C, long long rowid, const RowVals& o)
+__device__ __forceinline__ void store_row(const ClusterDev& C, long long rowid, const RowVals& o,
+                                          bool aux)
 {
     float4* t = C.tab + rowid * ROW_F4;
     t[0] = o.v0;
     t[1] = o.v1;
     C.tab2[rowid] = o.ext;
-    C.aux[rowid] = o.aux;
+    if (aux) C.aux[rowid] = o.aux;
 }
 
 // Shared-memory copies of one worker's breakpoints, record and key, kept by
@@ -1031,7 +1034,7 @@ __device__ unsigned build_table(const DevParams& P, const ClusterDev& C, int w,
                 const long long SM = SMx[e] == LL_NONE ? 0 : SMx[e];
                 const RowVals o = make_row(P, inv_s, M, sumP, r[e], nxt, np, A, pre_r[e], pre_ra[e],
                                            PMx[e], SM, pmA[e], pmAp[e], smS[e], smSp[e]);
-                store_row(C, rowbase + rowid[e], o);
+                store_row(C, rowbase + rowid[e], o, P.want_aux != 0);
                 if (cache && rowid[e] < R && rowid[e] < cache->rc)
                     cache->rho[rowid[e]] = (unsigned short)(nxt - 1);
                 if (want && r[e] <= rc && rc < nxt) {
@@ -1055,7 +1058,7 @@ __device__ unsigned build_table(const DevParams& P, const ClusterDev& C, int w,
             C.R[w] = 0;
             atomicOr(C.err, 1u);
         }
-        store_row(C, rowbase, o);
+        store_row(C, rowbase, o, P.want_aux != 0);
         if (want && (bad || n == 0 || rc < r0)) {
             float m;
             cf = eval_pair_mode(P.approx, o.v0, o.v1, o.ext, wr, wa, *cand, m);

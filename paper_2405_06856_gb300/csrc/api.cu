@@ -112,6 +112,7 @@ DevParams make_devparams(const aladdin_params& p)
     // is zero (the TTFT terms are switched off by d.decode).
     const bool dec = p.phase == ALADDIN_PHASE_DECODE;
     d.decode = dec ? 1 : 0;
+    d.want_aux = 0;  // set for the one build that aladdin_score_detail needs
     d.policy = p.policy;
     d.seed = (unsigned long long)p.seed;
     d.k1 = dec ? 0.0f : (float)p.k1;
@@ -159,6 +160,7 @@ struct aladdin_cluster {
     int W = 0, cap = 0, rows = 0;
     double t_now = 0.0;
     bool round_open = false;  // some worker holds requests placed in the open round
+    bool aux_valid = false;   // the exact row aggregates match the tables
     long long rid_next = 0;   // request id of the next power-of-two draw (place_round)
     std::vector<void*> owned;
     // scratch and staging (grow-only)
@@ -308,6 +310,7 @@ int cluster_alloc(aladdin_cluster* cl, const aladdin_params& p, int W,
 
 int refresh_tables(aladdin_cluster* cl)
 {
+    cl->aux_valid = false;
     CK(launch_build(cl->dp, cl->dev, nullptr, cl->W, cl->st));
     CK(launch_rank(cl->dev, cl->st));
     return ALADDIN_OK;
@@ -520,6 +523,14 @@ int score_impl(aladdin_cluster* cl, int32_t n, const int32_t* in, const int32_t*
             e0 = e1 = nullptr;
         }
     }
+    if ((dkv || dtc) && !cl->aux_valid) {
+        // the verification outputs read the exact row aggregates, which the
+        // builds of the scoring path leave out: one build that writes them
+        DevParams pa = cl->dp;
+        pa.want_aux = 1;
+        CK(launch_build(pa, cl->dev, nullptr, cl->W, cl->st));
+        cl->aux_valid = true;
+    }
     CK(launch_score(cl->dp, cl->dev, n, din, dpred, dwait, dflags, dmargin, darg, dkv, dtc, B,
                     cl->round_open, cl->st, e0, e1));
     if (hf) CK(cudaMemcpyAsync(flags, dflags, pairs, cudaMemcpyDeviceToHost, cl->st));
@@ -632,6 +643,7 @@ int aladdin_place_round(aladdin_cluster* cl, int32_t n_cand, const int32_t* in,
     io.status = cl->d_status;
     io.xbuf = cl->d_xround;
     io.rid0 = cl->rid_next;
+    cl->aux_valid = false;  // the round rebuilds tables without the aggregates
     if (cl->hp.policy == ALADDIN_POLICY_BESTFIT) {
         CK(launch_round(cl->dp, cl->dev, io, cl->st));
         CK(launch_rank(cl->dev, cl->st));
@@ -693,6 +705,7 @@ int aladdin_rebalance(aladdin_cluster* cl, int32_t n_cand, const int32_t* in,
     io.n_cand = n_cand;
     io.placement = dpl;
     io.status = cl->d_status;
+    cl->aux_valid = false;
     CK(launch_rebalance(cl->dp, cl->dev, io, dmov, dobj, cl->st));
     CK(launch_rank(cl->dev, cl->st));
     CK(cudaMemsetAsync(cl->dev.le, 0, sizeof(long long) * W, cl->st));
