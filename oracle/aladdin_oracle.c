@@ -76,6 +76,11 @@
  *   2 Po2       power of two choices: two workers drawn uniformly at random
  *               (SplitMix64, below), the one holding fewer requests, the
  *               first drawn on ties; no feasibility test.
+ * Grouped scheduling (Appendix A, distributed scheduling): with G > 1 groups
+ * the requests are dealt to groups round-robin (request id q to group
+ * q mod G) and each group's scheduler places only on its own workers
+ * (worker w belongs to group w mod G), under the same policy; Algorithm 2
+ * moves requests within their group.
  * In the simulation a placement that breaks an SLO shows up when the
  * workers execute: a realized TTFT above T_pre, a realized ATGT above T_dec
  * (each beyond a relative 1e-5) or an iteration whose KV exceeds M counts as
@@ -99,6 +104,7 @@ typedef struct {
     int64_t policy;       /* 0: best-fit; 1: JSQ; 2: power of two choices */
     uint64_t seed;        /* SplitMix64 seed of the power-of-two draws */
     int64_t rebalance;    /* 1: Algorithm 2 after every placement round (simulation) */
+    int64_t groups;       /* G > 1: distributed grouped scheduling (Appendix A) */
 } orc_params;
 
 /* Relative slack of a realized latency over its SLO before it counts as a
@@ -556,17 +562,28 @@ int32_t orc_po2_draw(uint64_t seed, int64_t rid, int k, int32_t W)
     return (int32_t)(((x >> 32) * (uint64_t)W) >> 32);
 }
 
-/* The worker a load-balancing policy picks (JSQ or power of two choices). */
+/* Grouped scheduling: may request rid be placed on worker w? */
+static int same_group(const orc_params* p, int w, int64_t rid)
+{
+    return p->groups <= 1 || (int64_t)w % p->groups == rid % p->groups;
+}
+
+/* The worker a load-balancing policy picks (JSQ or power of two choices)
+ * among the workers of the request's group; -1 if the group has none. */
 static int pick_by_queue(const orc_params* p, const orc_cluster* cl, int64_t rid)
 {
+    const int G = p->groups > 1 ? (int)p->groups : 1;
+    const int g = (int)(rid % G);
+    const int Wg = cl->W > g ? (cl->W - g + G - 1) / G : 0; /* workers g, g + G, ... */
+    if (Wg == 0) return -1;
     if (p->policy == 1) {
-        int best = 0;
-        for (int w = 1; w < cl->W; ++w)
+        int best = g;
+        for (int w = g + G; w < cl->W; w += G)
             if (cl->n[w] < cl->n[best]) best = w;
         return best;
     }
-    int w1 = orc_po2_draw(p->seed, rid, 0, cl->W);
-    int w2 = orc_po2_draw(p->seed, rid, 1, cl->W);
+    int w1 = g + G * orc_po2_draw(p->seed, rid, 0, Wg);
+    int w2 = g + G * orc_po2_draw(p->seed, rid, 1, Wg);
     return cl->n[w2] < cl->n[w1] ? w2 : w1;
 }
 
@@ -632,7 +649,7 @@ static int place_round_impl(const orc_params* p, orc_cluster* cl, int32_t C, con
         for (int32_t c = 0; c < C; ++c) {
             int64_t rid = crid ? crid[c] : c;
             int w = pick_by_queue(p, cl, rid);
-            if (cl->n[w] >= cl->cap) {
+            if (w < 0 || cl->n[w] >= cl->cap) {
                 if (!refuse_full) {
                     for (int32_t k = c; k < C; ++k) placement[k] = -1;
                     return ORC_ERR_CAPACITY;
@@ -659,6 +676,7 @@ static int place_round_impl(const orc_params* p, orc_cluster* cl, int32_t C, con
         if (capacity_order(p, cl, order) != ORC_OK) { rc = ORC_ERR_MEM; break; }
         for (int i = 0; i < W; ++i) {
             int w = order[i];
+            if (!same_group(p, w, crid ? crid[c] : c)) continue;
             if (!have[w]) {
                 if (future_build(cl, w, &fut[w]) != ORC_OK) { rc = ORC_ERR_MEM; break; }
                 have[w] = 1;
@@ -822,13 +840,16 @@ int orc_advance(const orc_params* p, orc_cluster* cl, double t_now, double dt,
  * worker (e_y < 0) that is feasible for it in the current state (all four
  * flags, a free slot) and lowers the sum the most, gain
  * (e_x - e_y) - |e_x - d_j| - |e_y + d_j| > 0; equal gains go to the larger
- * capacity_norm, then the lower index. A moved request leaves its pending
+ * capacity_norm, then the lower index (with grouped scheduling, among the
+ * workers of the request's group; its id is crid[c], c if NULL). A moved
+ * request leaves its pending
  * slot on x and becomes a pending request of y. placement[] is updated;
  * *moves (nullable) counts the moves, obj (nullable, 2 doubles) receives the
  * sum of distances before and after. */
 int orc_rebalance(const orc_params* p, orc_cluster* cl, int32_t C, const int32_t* cin,
-                  const int32_t* cpred, const double* cwait, int32_t* placement,
-                  const int64_t* le, const int32_t* be, int32_t* moves, double* obj)
+                  const int32_t* cpred, const double* cwait, const int64_t* crid,
+                  int32_t* placement, const int64_t* le, const int32_t* be, int32_t* moves,
+                  double* obj)
 {
     const int W = cl->W;
     double* e = (double*)malloc(sizeof(double) * (size_t)W);
@@ -852,6 +873,7 @@ int orc_rebalance(const orc_params* p, orc_cluster* cl, int32_t C, const int32_t
         double bgain = 0.0, bnorm = 0.0;
         for (int y = 0; y < W; ++y) {
             if (y == x || !(e[y] < 0.0) || cl->n[y] >= cl->cap) continue;
+            if (!same_group(p, y, crid ? crid[c] : c)) continue;
             double gain = ((e[x] - e[y]) - fabs(e[x] - d)) - fabs(e[y] + d);
             if (!(gain > 0.0)) continue;
             orc_future f;
@@ -985,8 +1007,8 @@ int orc_simulate(const orc_params* p, int32_t N, int32_t cap, int64_t M, double 
             if (rc != ORC_OK) break;
             if (p->rebalance && p->policy == 0) {
                 int32_t mv = 0;
-                rc = orc_rebalance(p, &cl, (int32_t)nwait, cin, cpr, cw, pl, cl.le, cl.be, &mv,
-                                   NULL);
+                rc = orc_rebalance(p, &cl, (int32_t)nwait, cin, cpr, cw, wl, pl, cl.le, cl.be,
+                                   &mv, NULL);
                 if (rc != ORC_OK) break;
                 moved += mv;
             }

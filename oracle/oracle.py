@@ -40,7 +40,7 @@ class Params(C.Structure):
                 ("j", C.c_int64), ("T_pre", C.c_double), ("T_dec", C.c_double),
                 ("gamma", C.c_double), ("theta", C.c_double), ("K", C.c_int64),
                 ("mode", C.c_int64), ("phase", C.c_int64), ("policy", C.c_int64),
-                ("seed", C.c_uint64), ("rebalance", C.c_int64)]
+                ("seed", C.c_uint64), ("rebalance", C.c_int64), ("groups", C.c_int64)]
 
 
 class ClusterStruct(C.Structure):
@@ -67,7 +67,7 @@ def lib():
         _lib.orc_kv_curve.restype = C.c_int32
         _lib.orc_place_round.argtypes = [P, P, C.c_int32, P, P, P, P, P]
         _lib.orc_advance.argtypes = [P, P, C.c_double, C.c_double, P, P, P, P, C.c_int64, P, P]
-        _lib.orc_rebalance.argtypes = [P, P, C.c_int32, P, P, P, P, P, P, P, P]
+        _lib.orc_rebalance.argtypes = [P, P, C.c_int32, P, P, P, P, P, P, P, P, P]
         _lib.orc_splitmix64.argtypes = [C.c_uint64, C.c_uint64]
         _lib.orc_splitmix64.restype = C.c_uint64
         _lib.orc_po2_draw.argtypes = [C.c_uint64, C.c_int64, C.c_int, C.c_int32]
@@ -98,7 +98,8 @@ def make_params(d):
                   float(d["c3"]), int(d["h"]), int(d["j"]), float(d["T_pre"]),
                   float(d["T_dec"]), float(d["gamma"]), float(d["theta"]), int(d["K"]),
                   int(d.get("mode", 0)), int(d.get("phase", 0)), int(d.get("policy", 0)),
-                  int(d.get("seed", 0)) & 0xFFFFFFFFFFFFFFFF, int(d.get("rebalance", 0)))
+                  int(d.get("seed", 0)) & 0xFFFFFFFFFFFFFFFF, int(d.get("rebalance", 0)),
+                  int(d.get("groups", 1)))
 
 
 def _ptr(a):
@@ -258,7 +259,7 @@ class Cluster:
         self.real = np.ascontiguousarray(real, np.int32).copy()
         self.repred = None if repred is None else np.ascontiguousarray(repred, np.int32)
 
-    def rebalance(self, cin, cpred, cwait, placement, le, be):
+    def rebalance(self, cin, cpred, cwait, placement, le, be, crid=None):
         """Algorithm 2 over a round's placements (updated in place); returns
         (moves, objective before, objective after)."""
         cin = np.ascontiguousarray(cin, np.int32)
@@ -269,9 +270,10 @@ class Cluster:
         mv = C.c_int32(0)
         obj = np.zeros(2)
         st = self.struct()
+        cr = None if crid is None else np.ascontiguousarray(crid, np.int64)
         rc = lib().orc_rebalance(C.byref(self._p), C.byref(st), len(cin), _ptr(cin), _ptr(cpred),
-                                 _ptr(cw), _ptr(placement), _ptr(le), _ptr(be), C.byref(mv),
-                                 _ptr(obj))
+                                 _ptr(cw), _ptr(cr), _ptr(placement), _ptr(le), _ptr(be),
+                                 C.byref(mv), _ptr(obj))
         if rc != 0:
             raise RuntimeError("orc_rebalance failed: %d" % rc)
         return mv.value, obj[0], obj[1]

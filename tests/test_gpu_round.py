@@ -332,3 +332,26 @@ def test_min_workers_four_options(A, orc, synth):
     assert np.array_equal(got, ref), (got, ref)
     tot = [g * n for g, n in zip(gpus, ref)]
     assert total == min(tot) and best == int(np.argmin(tot))
+
+
+def test_round_and_simulation_deterministic(A, synth):
+    """The same round on two fresh clusters (a cooperative grid of several
+    CTAs) gives the same placements and state bytes; the same simulation twice
+    gives the same outputs."""
+    wl = synth.config("w4096", n_cand=3000, b_cap=256)
+    res = []
+    for _ in range(2):
+        with A.Cluster.from_workload(wl) as cl:
+            pl = cl.place_round(wl.cand_in, wl.cand_pred, wl.cand_wait)
+            cl.advance(100.0)
+            res.append((pl.tobytes(),) + tuple(x.tobytes() for x in cl.state()))
+    assert res[0] == res[1]
+    tr = synth.with_prediction_error(synth.diurnal_trace(8, 3000, 80.0, 20.0), 0.4, 8)
+    p = dict(synth.BASE_PARAMS, T_dec=30.0, rebalance=1)
+    outs = []
+    for _ in range(2):
+        out = np.zeros(A.SIMULATE_OUT)
+        A.aladdin_simulate(A.make_params(p, 256), A.make_cfgs([1], [40000], [1.0])[0], 9,
+                           A.trace_of(tr), 100.0, 0, 1, out)
+        outs.append(out.tobytes())
+    assert outs[0] == outs[1]
