@@ -112,7 +112,10 @@ extern "C" {
  * Requirements: k1, k2 > 0; c1, c2, c3 >= 0; h >= 1; j >= 0; T_pre > 0;
  * T_dec > c3 (Eq. input limit); 0 < theta <= 1; gamma >= 0; 2 <= K <= 65536;
  * b_cap a power of two in [32, 1024]; mode, phase and policy one of the
- * values above; rebalance 0 or 1. */
+ * values above; rebalance 0 or 1; 0 <= groups <= 65536. Request ids (for the
+ * power-of-two draws and the groups) are trace indices in the simulation and
+ * the running candidate count in aladdin_place_round; aladdin_rebalance uses
+ * the ids of the latest aladdin_place_round. */
 typedef struct aladdin_params {
     double k1, c1;       /* prefill: ms per input token, ms */
     double k2, c2, c3;   /* decode: ms per context token, ms per request, ms */
@@ -129,6 +132,9 @@ typedef struct aladdin_params {
     uint64_t seed;       /* SplitMix64 seed of the power-of-two draws */
     int32_t rebalance;   /* 1: Algorithm 2 after every best-fit round of a simulation
                             (see aladdin_rebalance); 0: off */
+    int32_t groups;      /* distributed grouped scheduling (Appendix A): G > 1 groups,
+                            request id q in group q mod G placed only on workers
+                            w = g (mod G); 0 or 1: one central scheduler */
 } aladdin_params;
 
 /* One worker configuration (Sec. 4.1): GPUs per worker, KV capacity in KV

@@ -52,7 +52,7 @@ class aladdin_params(C.Structure):
                 ("T_dec", C.c_double), ("gamma", C.c_double), ("theta", C.c_double),
                 ("K", C.c_int32), ("b_cap", C.c_int32), ("mode", C.c_int32),
                 ("phase", C.c_int32), ("policy", C.c_int32), ("seed", C.c_uint64),
-                ("rebalance", C.c_int32)]
+                ("rebalance", C.c_int32), ("groups", C.c_int32)]
 
 
 class aladdin_worker_cfg(C.Structure):
@@ -139,7 +139,8 @@ def make_params(d, b_cap):
                           float(d["T_dec"]), float(d["gamma"]), float(d["theta"]), int(d["K"]),
                           int(b_cap), int(d.get("mode", MODE_EXACT)),
                           int(d.get("phase", PHASE_MIXED)), int(d.get("policy", POLICY_BESTFIT)),
-                          int(d.get("seed", 0)) & 0xFFFFFFFFFFFFFFFF, int(d.get("rebalance", 0)))
+                          int(d.get("seed", 0)) & 0xFFFFFFFFFFFFFFFF, int(d.get("rebalance", 0)),
+                          int(d.get("groups", 1)))
 
 
 def make_cfgs(gpus, kv_capacity, lat_scale):

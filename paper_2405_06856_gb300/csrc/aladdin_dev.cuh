@@ -65,6 +65,7 @@ struct DevParams {
                              // that only the verification outputs read
     int32_t decode;          // 1: decode instance of split-phase inference (no prefill)
     int32_t policy;          // ALADDIN_POLICY_* of placement rounds
+    int32_t groups;          // G > 1: request q is placed only on workers w = q (mod G)
     unsigned long long seed; // SplitMix64 seed of the power-of-two draws
 };
 

@@ -94,6 +94,7 @@ int check_params(const aladdin_params* p)
         p->policy != ALADDIN_POLICY_PO2)
         return ALADDIN_ERR_ARG;
     if (p->rebalance != 0 && p->rebalance != 1) return ALADDIN_ERR_ARG;
+    if (p->groups < 0 || p->groups > 65536) return ALADDIN_ERR_ARG;
     return ALADDIN_OK;
 }
 
@@ -114,6 +115,7 @@ DevParams make_devparams(const aladdin_params& p)
     d.decode = dec ? 1 : 0;
     d.want_aux = 0;  // set for the one build that aladdin_score_detail needs
     d.policy = p.policy;
+    d.groups = p.groups > 1 ? p.groups : 1;
     d.seed = (unsigned long long)p.seed;
     d.k1 = dec ? 0.0f : (float)p.k1;
     d.c1 = dec ? 0.0f : (float)p.c1;
@@ -161,7 +163,8 @@ struct aladdin_cluster {
     double t_now = 0.0;
     bool round_open = false;  // some worker holds requests placed in the open round
     bool aux_valid = false;   // the exact row aggregates match the tables
-    long long rid_next = 0;   // request id of the next power-of-two draw (place_round)
+    long long rid_next = 0;   // request id of the next place_round candidate (draws, groups)
+    long long rid_last = 0;   // the first id of the latest place_round (rebalance)
     std::vector<void*> owned;
     // scratch and staging (grow-only)
     DevBuf sorted, hist, best;
@@ -643,6 +646,7 @@ int aladdin_place_round(aladdin_cluster* cl, int32_t n_cand, const int32_t* in,
     io.status = cl->d_status;
     io.xbuf = cl->d_xround;
     io.rid0 = cl->rid_next;
+    cl->rid_last = cl->rid_next;
     cl->aux_valid = false;  // the round rebuilds tables without the aggregates
     if (cl->hp.policy == ALADDIN_POLICY_BESTFIT) {
         CK(launch_round(cl->dp, cl->dev, io, cl->st));
@@ -705,6 +709,7 @@ int aladdin_rebalance(aladdin_cluster* cl, int32_t n_cand, const int32_t* in,
     io.n_cand = n_cand;
     io.placement = dpl;
     io.status = cl->d_status;
+    io.rid0 = cl->rid_last;
     cl->aux_valid = false;
     CK(launch_rebalance(cl->dp, cl->dev, io, dmov, dobj, cl->st));
     CK(launch_rank(cl->dev, cl->st));

@@ -75,13 +75,18 @@ __global__ void __launch_bounds__(Q_THREADS) k_round_queue(DevParams P, ClusterD
             r = io.pred[c];
             wd = io.wait ? (double)io.wait[c] : 0.0;
         }
-        const bool valid = a >= 0 && r >= 1 && (long long)a + r <= (long long)P.K && wd >= 0.0 &&
-                           wd <= 3.0e38;
+        const bool valid0 = a >= 0 && r >= 1 && (long long)a + r <= (long long)P.K && wd >= 0.0 &&
+                            wd <= 3.0e38;
+        // grouped scheduling: group g = id mod G owns workers g, g + G, ...
+        const int G = P.groups;
+        const int grp = G > 1 ? (int)(tix % G) : 0;
+        const int Wg = W > grp ? (W - grp + G - 1) / G : 0;
+        const bool valid = valid0 && Wg > 0;
         int choice = -1;
         if (valid && jsq) {
             // smallest (count, index): counts < 2^31, indexes < 2^31
             unsigned long long best = ~0ull;
-            for (int w = tid; w < W; w += Q_THREADS) {
+            for (int w = grp + tid * G; w < W; w += Q_THREADS * G) {
                 const unsigned long long k =
                     ((unsigned long long)(unsigned)cnt[w] << 32) | (unsigned)w;
                 best = k < best ? k : best;
@@ -100,14 +105,14 @@ __global__ void __launch_bounds__(Q_THREADS) k_round_queue(DevParams P, ClusterD
         }
         if (tid == 0) {
             if (valid && !jsq) {
-                const int w1 = po2_draw(P.seed, tix, 0, W);
-                const int w2 = po2_draw(P.seed, tix, 1, W);
+                const int w1 = grp + G * po2_draw(P.seed, tix, 0, Wg);
+                const int w2 = grp + G * po2_draw(P.seed, tix, 1, Wg);
                 choice = cnt[w2] < cnt[w1] ? w2 : w1;
             }
-            if (!valid) {
+            if (!valid0) {
                 if (io.sim) io.counters[0] += 1;
                 else io.placement[c] = -2;  // ALADDIN_INVALID
-            } else if (cnt[choice] >= C.cap) {
+            } else if (!valid || cnt[choice] >= C.cap) {  // no worker in the group, or full
                 if (io.sim) {
                     io.counters[0] += 1;  // no free slot: the request fails
                 } else {

@@ -115,8 +115,10 @@ __global__ void __launch_bounds__(RB_THREADS) k_rebalance(DevParams P, ClusterDe
         if (!(ex > 0.0)) continue;
         int32_t a, r;
         double wd;
+        long long rid = io.rid0 + c;
         if (io.sim) {
             const long long tix = io.sim_tix[c];
+            rid = tix;
             a = io.tin[tix];
             r = io.tpred[tix];
             wd = io.t_now - io.t_arr[tix];
@@ -128,12 +130,14 @@ __global__ void __launch_bounds__(RB_THREADS) k_rebalance(DevParams P, ClusterDe
         const CandRec cr = make_cand(P, a, r, (float)wd, c);
         if (!cr.valid) continue;
         const double d = __dadd_rn(__dmul_rn(P.k2d, (double)r), P.c2d);
+        const int G = P.groups;
+        const int grp = G > 1 ? (int)(rid % G) : 0;  // moves stay in the request's group
         double bg = 0.0;
         unsigned long long bk = 0ull;
         int bw = -1;
         for (int y = tid; y < W; y += RB_THREADS) {
             const double ey = C.err_e[y];
-            if (y == x || !(ey < 0.0) || C.n[y] >= C.cap) continue;
+            if (y == x || !(ey < 0.0) || C.n[y] >= C.cap || (G > 1 && y % G != grp)) continue;
             const double g = __dsub_rn(__dsub_rn(__dsub_rn(ex, ey), fabs(__dsub_rn(ex, d))),
                                        fabs(__dadd_rn(ey, d)));
             if (!(g > 0.0)) continue;

@@ -64,11 +64,15 @@ __global__ void __launch_bounds__(ROUND_THREADS) k_round(DevParams P, ClusterDev
             wd = io.wait ? (double)io.wait[c] : 0.0;
         }
         const CandRec cr = make_cand(P, a, r, (float)wd, c);
+        // grouped scheduling: the request's group places on its own workers
+        const int G = P.groups;
+        const int grp = G > 1 ? (int)((io.sim ? tix : io.rid0 + c) % G) : 0;
         int winner = -2;
         if (cr.valid) {
             unsigned long long bk = 0ull;
             int bw = 0x7fffffff;
             for (int w = tid; w < C.W; w += ROUND_THREADS) {
+                if (G > 1 && w % G != grp) continue;
                 const long long rb = (long long)w * C.rows;
                 const int p = find_row<false>(C.tab, rb, C.R[w], cr.ri);
                 const float4* t = C.tab + (rb + p) * ROW_F4;
@@ -377,6 +381,9 @@ __global__ void __launch_bounds__(R2_THREADS, 1) k_round2(R2Args A)
             wd = io.wait ? (double)io.wait[c] : 0.0;
         }
         const CandRec cr = make_cand(P, a, r, (float)wd, c);
+        // grouped scheduling: the request's group places on its own workers
+        const int G = P.groups;
+        const int grp = G > 1 ? (int)((io.sim ? tix : io.rid0 + c) % G) : 0;
         unsigned long long bk = 0ull;
         int bw = NONE, bf = 0;
         const bool rebuilding = pend_w >= 0;
@@ -387,13 +394,14 @@ __global__ void __launch_bounds__(R2_THREADS, 1) k_round2(R2Args A)
             const unsigned f = build_table_fit<EW, NW, NW_INSERT>(P, C, pend_w, n_s[lw],
                                                        reinterpret_cast<unsigned char*>(&sm.build),
                                                        &sc, cr.valid ? &cr : nullptr);
-            if (tid == 0 && cr.valid && f == 15u) bk = key_s[lw], bw = pend_w, bf = n_s[lw] >= cap;
+            if (tid == 0 && cr.valid && f == 15u && (G <= 1 || pend_w % G == grp))
+                bk = key_s[lw], bw = pend_w, bf = n_s[lw] >= cap;
         } else if (cr.valid) {
             const int first = rebuilding ? tid - 32 * NW : tid;
             const int stride = rebuilding ? R2_THREADS - 32 * NW : R2_THREADS;
             for (int lw = first; lw < nloc; lw += stride) {
                 const int w = w_lo + lw;
-                if (w == pend_w) continue;
+                if (w == pend_w || (G > 1 && w % G != grp)) continue;
                 const long long rb = (long long)w * C.rows;
                 const int p = r2_find(rho + (long long)lw * rs, R_s[lw], rc, cr.ri, C.tab, rb);
                 const long long row = rb + p;

@@ -40,10 +40,11 @@ def test_library_exports_every_declared_symbol(lib):
 
 def test_struct_layout(lib):
     # 5 doubles, h and j, 4 doubles, K b_cap mode phase policy, pad, seed,
-    # rebalance, pad
+    # rebalance, groups
     assert ctypes.sizeof(lib.aladdin_params) == 5 * 8 + 2 * 4 + 4 * 8 + 5 * 4 + 4 + 8 + 4 + 4
     assert lib.aladdin_params.seed.offset == 104
     assert lib.aladdin_params.rebalance.offset == 112
+    assert lib.aladdin_params.groups.offset == 116
     assert ctypes.sizeof(lib.aladdin_worker_cfg) == 24
     assert ctypes.sizeof(lib.aladdin_trace) == 48
 
@@ -52,7 +53,7 @@ def test_struct_layout(lib):
                                  dict(theta=1.5), dict(K=1), dict(K=70000), dict(h=0),
                                  dict(j=-1), dict(c1=float("nan")), dict(T_pre=0.0),
                                  dict(phase=2), dict(policy=3), dict(policy=-1),
-                                 dict(rebalance=2)])
+                                 dict(rebalance=2), dict(groups=-1), dict(groups=70000)])
 def test_create_rejects_bad_params(lib, bad):
     from paper_2405_06856_gb300 import synth
     d = dict(synth.BASE_PARAMS)
