@@ -680,11 +680,36 @@ def prediction_errors(A, synth, stream, n_requests=100_000, n_workers=133,
     return out
 
 
+def grouped_scheduling(A, synth, stream, n_requests=100_000, groups=(1, 2, 4, 8)):
+    """Distributed grouped scheduling (Appendix A): requests dealt round-robin
+    to G groups, each placing on its own workers; the workers the search
+    needs for each G (1-GPU workers, best-fit) against the central
+    scheduler's."""
+    tr = synth.diurnal_trace(4, n_requests, 2000.0, 500.0)
+    trace = A.make_trace(tr.t_arr, tr.req_in, tr.req_pred)
+    out = {"workload": "diurnal trace of %d requests, 1-GPU workers (%d KV tokens), best-fit"
+                       % (n_requests, MW_KV_PER_GPU)}
+    base = None
+    for G in groups:
+        p = dict(synth.BASE_PARAMS, groups=G)
+        got = np.zeros(1, np.int32)
+        t0 = time.perf_counter()
+        A.aladdin_min_workers(A.make_params(p, MW_B_CAP),
+                              A.make_cfgs([1], [MW_KV_PER_GPU], [1.0]), trace, 100.0, 4096, got,
+                              stream=stream)
+        n = int(got[0])
+        base = n if G == 1 else base
+        out["G%d" % G] = {"min_workers": n, "workers_per_group": round(n / G, 1),
+                          "extra_vs_central": round(n / base - 1.0, 4) if base else None,
+                          "search_s": round(time.perf_counter() - t0, 2)}
+    return out
+
+
 def run_policies(args):
     """Best-fit against JSQ and the power of two choices (Sec. 6.4): GPUs each
     needs, mixed setting and decode instances, on a 100,000-request trace; the
     worker-configuration picker and the fitted worker-count model; Algorithm 2
-    under prediction errors."""
+    under prediction errors; grouped scheduling."""
     import torch
     from paper_2405_06856_gb300 import build as B
     B.build()
@@ -696,6 +721,7 @@ def run_policies(args):
     res = policy_compare(A, synth, stream, 100_000, [1, 2, 4, 8])
     res["worker_model"] = worker_model(A, synth, stream)
     res["prediction_errors"] = prediction_errors(A, synth, stream)
+    res["grouped_scheduling"] = grouped_scheduling(A, synth, stream)
     res["mode"] = "policies"
     res["wall_s"] = round(time.perf_counter() - t0, 1)
     print(json.dumps(res))
