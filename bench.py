@@ -449,6 +449,9 @@ def run_ours(args):
             rounds.append((time.perf_counter() - t0) * 1000.0)
     round_ms = min(rounds)
     r16k = rounds_w16384(A, synth, stream)
+    # group counts coprime with the workload's 1/2/4/8-GPU cycle of workers,
+    # so that every group holds all four worker sizes
+    r16k_grp = {"G%d" % G: rounds_w16384(A, synth, stream, groups=G) for G in (7, 63)}
     apx = approx_mode(A, synth, dev, stream, flush)
     pol = policy_compare(A, synth, stream, 20_000, [1, 2])
     wmod = worker_model(A, synth, stream, fit_n=0)
@@ -481,6 +484,7 @@ def run_ours(args):
             "round_latency_ms": {"workload": "256 workers x 64 requests, 2,048 candidates, one "
                                              "greedy round", "value": round_ms},
             "rounds_w16384": r16k,
+            "rounds_w16384_grouped": r16k_grp,
             "approx_mode": apx,
             "policies": pol,
             "worker_config": wmod,
@@ -494,13 +498,15 @@ def run_ours(args):
         dist.destroy_process_group()
 
 
-def rounds_w16384(A, synth, stream, n_rounds=10, dt_ms=100.0):
+def rounds_w16384(A, synth, stream, n_rounds=10, dt_ms=100.0, groups=1):
     """Ten consecutive greedy rounds on the 16,384-worker workload (1/2/4/8-GPU
     workers, 256 requests each): the 131,072 candidates arrive over ten
     heartbeats, each round placing its share, then every worker executes
     100 ms. Round time is the synchronous aladdin_place_round call with host
-    arrays (upload, the round, the capacity_norm ranking and the download)."""
-    wl = synth.config("w16384")
+    arrays (upload, the round, the capacity_norm ranking and the download).
+    groups > 1: grouped scheduling (Appendix A), the groups' rounds in
+    parallel."""
+    wl = synth.config("w16384", params=dict(groups=groups))
     bounds = np.linspace(0, wl.n_cand, n_rounds + 1).astype(int)
     rounds, advances, placed = [], [], 0
     with A.Cluster.from_workload(wl, stream=stream) as cl:
@@ -516,7 +522,8 @@ def rounds_w16384(A, synth, stream, n_rounds=10, dt_ms=100.0):
         assert cl.status() == A.OK
     return {"workload": "16,384 workers of 1/2/4/8 GPUs (KV 131,072 per GPU, latency x 1/sqrt(GPUs)), "
                         "256 requests each; 131,072 candidates over 10 greedy rounds of 13,107, "
-                        "100 ms of execution between rounds; seed 3",
+                        "100 ms of execution between rounds; seed 3"
+                        + ("; %d scheduling groups" % groups if groups > 1 else ""),
             "rounds": n_rounds, "candidates_per_round": int(bounds[1] - bounds[0]),
             "ms_per_round": statistics.mean(rounds), "ms_max_round": max(rounds),
             "ms_per_advance": statistics.mean(advances),

@@ -232,7 +232,11 @@ int aladdin_score_noalloc(aladdin_cluster* cl, int32_t n_cand, const int32_t* in
  * if no worker is feasible (best-fit; the cluster is fixed: no worker is
  * opened), ALADDIN_INVALID for an invalid candidate. Returns
  * ALADDIN_ERR_CAPACITY if a chosen worker has no free slot (placements up to
- * that candidate are kept, the later ones are ALADDIN_NONE). */
+ * that candidate are kept, the later ones are ALADDIN_NONE). With grouped
+ * scheduling (params.groups > 1) and best-fit the groups are independent
+ * schedulers and run in parallel, one CTA each: a group whose chosen worker
+ * is full stops there (its later candidates ALADDIN_NONE), the others go on,
+ * and the call returns ALADDIN_ERR_CAPACITY. */
 int aladdin_place_round(aladdin_cluster* cl, int32_t n_cand, const int32_t* in,
                         const int32_t* pred, const float* wait_ms, int32_t* placement);
 

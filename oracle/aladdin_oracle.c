@@ -671,12 +671,22 @@ static int place_round_impl(const orc_params* p, orc_cluster* cl, int32_t C, con
     uint8_t* have = (uint8_t*)calloc((size_t)W, 1);
     if (!T0 || !T1 || !order || !fut || !have) return ORC_ERR_MEM;
     int rc = ORC_OK;
+    /* With groups each group is its own scheduler: a group whose chosen worker
+     * has no free slot stops there (that candidate and its later ones stay
+     * unplaced) while the other groups go on; the round then reports
+     * ORC_ERR_CAPACITY. */
+    const int64_t G = p->groups > 1 ? p->groups : 1;
+    uint8_t* stopped = G > 1 ? (uint8_t*)calloc((size_t)G, 1) : NULL;
+    int cap_hit = 0;
+    if (G > 1 && !stopped) return ORC_ERR_MEM;
     for (int32_t c = 0; c < C && rc == ORC_OK; ++c) {
         placement[c] = -1;
+        const int64_t rid = crid ? crid[c] : c;
+        if (stopped && stopped[rid % G]) continue;
         if (capacity_order(p, cl, order) != ORC_OK) { rc = ORC_ERR_MEM; break; }
         for (int i = 0; i < W; ++i) {
             int w = order[i];
-            if (!same_group(p, w, crid ? crid[c] : c)) continue;
+            if (!same_group(p, w, rid)) continue;
             if (!have[w]) {
                 if (future_build(cl, w, &fut[w]) != ORC_OK) { rc = ORC_ERR_MEM; break; }
                 have[w] = 1;
@@ -684,7 +694,15 @@ static int place_round_impl(const orc_params* p, orc_cluster* cl, int32_t C, con
             orc_pair r;
             eval_pair(p, cl, w, &fut[w], T0, T1, cin[c], cpred[c], cwait ? cwait[c] : 0.0, &r);
             if (r.flags != 15) continue;
-            if (cl->n[w] >= cl->cap) { rc = ORC_ERR_CAPACITY; break; }
+            if (cl->n[w] >= cl->cap) {
+                if (stopped) {
+                    stopped[rid % G] = 1;
+                    cap_hit = 1;
+                } else {
+                    rc = ORC_ERR_CAPACITY;
+                }
+                break;
+            }
             append_request(cl, w, cin[c], cpred[c], creal ? creal[c] : cpred[c],
                            cwait ? cwait[c] : 0.0, crid ? crid[c] : c);
             future_free(&fut[w]);
@@ -700,6 +718,8 @@ static int place_round_impl(const orc_params* p, orc_cluster* cl, int32_t C, con
     free(order);
     free(fut);
     free(have);
+    free(stopped);
+    if (rc == ORC_OK && cap_hit) rc = ORC_ERR_CAPACITY;
     return rc;
 }
 

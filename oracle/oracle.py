@@ -221,7 +221,9 @@ class Cluster:
         lib().orc_order(C.byref(self._p), C.byref(st), _ptr(o))
         return o
 
-    def place_round(self, cin, cpred, cwait=None, crid=None):
+    def place_round(self, cin, cpred, cwait=None, crid=None, allow_capacity=False):
+        """One placement round; with allow_capacity a full worker does not
+        raise: returns (placements, True) instead."""
         cin = np.ascontiguousarray(cin, np.int32)
         cpred = np.ascontiguousarray(cpred, np.int32)
         cw = None if cwait is None else np.ascontiguousarray(cwait, np.float64)
@@ -231,10 +233,12 @@ class Cluster:
         rc = lib().orc_place_round(C.byref(self._p), C.byref(st), len(cin), _ptr(cin),
                                    _ptr(cpred), _ptr(cw), _ptr(cr), _ptr(pl))
         if rc == -2:
+            if allow_capacity:
+                return pl, True
             raise OverflowError("worker request capacity exceeded")
         if rc != 0:
             raise RuntimeError("orc_place_round failed: %d" % rc)
-        return pl
+        return (pl, False) if allow_capacity else pl
 
     def commit(self, w, a, r, wait=0.0, rid=0):
         """Append request (prompt a, predicted output r) to worker w as a

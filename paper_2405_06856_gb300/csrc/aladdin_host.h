@@ -82,6 +82,12 @@ cudaError_t launch_advance(const DevParams& P, const ClusterDev& C, double t_now
                            unsigned long long* stats, const int* halt, cudaStream_t st,
                            unsigned long long* fail = nullptr);
 
+// A best-fit round of a placement call under grouped scheduling (P.groups >
+// 1, direct mode): one CTA per group, the groups in parallel. A group whose
+// chosen worker is full stops (status -2); placements -1 / -2 as launch_round.
+cudaError_t launch_round_groups(const DevParams& P, const ClusterDev& C, const RoundIO& io,
+                                cudaStream_t st);
+
 // One round of a load-balancing policy (JSQ or power of two choices; the
 // RoundIO of launch_round): each candidate goes to the policy's worker
 // without a feasibility test. Tables are not rebuilt.

@@ -648,7 +648,11 @@ int aladdin_place_round(aladdin_cluster* cl, int32_t n_cand, const int32_t* in,
     io.rid0 = cl->rid_next;
     cl->rid_last = cl->rid_next;
     cl->aux_valid = false;  // the round rebuilds tables without the aggregates
-    if (cl->hp.policy == ALADDIN_POLICY_BESTFIT) {
+    if (cl->hp.policy == ALADDIN_POLICY_BESTFIT && cl->dp.groups > 1) {
+        // independent schedulers: one CTA per group, in parallel
+        CK(launch_round_groups(cl->dp, cl->dev, io, cl->st));
+        CK(launch_rank(cl->dev, cl->st));
+    } else if (cl->hp.policy == ALADDIN_POLICY_BESTFIT) {
         CK(launch_round(cl->dp, cl->dev, io, cl->st));
         CK(launch_rank(cl->dev, cl->st));
     } else {

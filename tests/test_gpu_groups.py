@@ -92,3 +92,24 @@ def test_grouped_search_and_rebalance(A, orc, synth):
     A.aladdin_simulate(A.make_params(p, 256), A.make_cfgs([1], [40000], [1.0])[0], 6,
                        A.trace_of(te), 100.0, 0, 1, out)
     assert int(out[0]) == ref["failed"] and int(out[8]) == ref["moved"] and ref["moved"] > 0
+
+
+def test_grouped_round_full_worker_stops_its_group(A, orc, synth):
+    """Two groups of one worker (32 slots): group 0's worker holds 31
+    requests, so its second candidate finds it full and group 0 stops; group 1
+    places all of its candidates. The call reports ALADDIN_ERR_CAPACITY."""
+    p = dict(synth.BASE_PARAMS, groups=2)
+    roff = np.array([0, 31, 31], np.int32)
+    args = (np.full(31, 100, np.int32), np.zeros(31, np.int32), np.full(31, 50, np.int32))
+    cin, cpr = np.full(40, 100, np.int32), np.full(40, 50, np.int32)
+    with A.Cluster(p, [1, 1], [10**6] * 2, [1.0] * 2, 32, roff, *args) as cl:
+        pl = np.zeros(40, np.int32)
+        with pytest.raises(A.AladdinError) as e:
+            A.aladdin_place_round(cl.handle, 40, cin, cpr, None, pl)
+        assert e.value.code == A.ERR_CAPACITY
+        n = cl.state()[0]
+    oc = orc.Cluster(p, [10**6] * 2, [1.0] * 2, 32, roff, *args)
+    ref, full = oc.place_round(cin, cpr, crid=np.arange(40), allow_capacity=True)
+    assert full and np.array_equal(pl, ref)
+    assert list(pl[:4]) == [0, 1, -1, 1] and (pl[1::2] == 1).all() and (pl[2::2] == -1).all()
+    assert list(n) == [32, 20] == list(oc.n)

@@ -83,3 +83,18 @@ def test_rebalance_stays_in_group(orc):
     mv, _, _ = cl.rebalance([200], [100], [0.0], pl, [10**4, -10**5, -10**4, 0], [0, 0, 0, 0],
                             crid=[0])
     assert mv == 1 and list(pl) == [2]
+
+
+def test_full_worker_stops_only_its_group(orc, synth):
+    """With groups, a best-fit group whose chosen worker has no free slot stops
+    (that candidate and its later ones stay unplaced); the other group goes on.
+    Two groups of one worker each, 4 slots: group 0's worker holds 3 requests,
+    so its second candidate finds it full; group 1 places all of its own."""
+    p = dict(synth.BASE_PARAMS, groups=2)
+    roff = np.array([0, 3, 3], np.int32)
+    cl = orc.Cluster(p, [10**6, 10**6], [1.0, 1.0], 4, roff, np.full(3, 100, np.int32),
+                     np.zeros(3, np.int32), np.full(3, 50, np.int32))
+    pl, full = cl.place_round([100] * 8, [50] * 8, crid=np.arange(8), allow_capacity=True)
+    assert full
+    assert list(pl) == [0, 1, -1, 1, -1, 1, -1, 1]
+    assert list(cl.n) == [4, 4]
