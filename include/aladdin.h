@@ -286,6 +286,21 @@ int aladdin_rebalance(aladdin_cluster* cl, int32_t n_cand, const int32_t* in,
                       const int32_t* pred, const float* wait_ms, int32_t* placement,
                       const int64_t* le, const int32_t* be, int32_t* moves, double* obj);
 
+/* Checkpoint and resume of a cluster's state (no counterpart in the paper):
+ * the requests of every slot (l_in, l_out, l_pred, real length, decode time
+ * so far, pending flag, wait), every worker's count, clock, offset and
+ * Algorithm 2 errors, and the cluster's clock, open-round flag and request
+ * ids. aladdin_cluster_save with buf NULL stores the size in *bytes;
+ * otherwise it writes that many bytes to buf (host memory, *bytes at least
+ * the size; synchronous). aladdin_cluster_restore loads such a buffer into
+ * a cluster of the same worker count and request slots (its own parameters
+ * and worker configurations stay) and rebuilds the tables and the
+ * capacity_norm ranking, so that the cluster continues exactly as the saved
+ * one would. ALADDIN_ERR_ARG for a buffer that is too short, not a
+ * checkpoint, or of another shape. */
+int aladdin_cluster_save(aladdin_cluster* cl, void* buf, int64_t* bytes);
+int aladdin_cluster_restore(aladdin_cluster* cl, const void* buf, int64_t bytes);
+
 /* Kernel timing (tracing): while enabled, CUDA events on the cluster's stream
  * bracket every launch of the candidate x worker scoring kernel. Each call
  * waits for the stream, returns in *kernel_ms (nullable) the summed event time

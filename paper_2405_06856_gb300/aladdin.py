@@ -91,6 +91,8 @@ _sig = {
                             _P, _P],
     "aladdin_predict_workers": [C.c_double, C.c_double, C.c_double, _P],
     "aladdin_rebalance": [_P, C.c_int32, _P, _P, _P, _P, _P, _P, _P, _P],
+    "aladdin_cluster_save": [_P, _P, _P],
+    "aladdin_cluster_restore": [_P, _P, C.c_int64],
 }
 for _n, _a in _sig.items():
     f = getattr(_lib, _n)
@@ -228,6 +230,20 @@ def aladdin_rebalance(cl, n_cand, cand_in, cand_pred, wait_ms, placement, le, be
                                   _ptr(placement), _ptr(le), _ptr(be), C.byref(mv), _ptr(obj)),
            "aladdin_rebalance")
     return mv.value, obj[0], obj[1]
+
+
+def aladdin_cluster_save(cl):
+    """The cluster's checkpoint as bytes."""
+    n = C.c_int64(0)
+    _check(_lib.aladdin_cluster_save(cl, None, C.byref(n)), "aladdin_cluster_save")
+    buf = np.zeros(n.value, np.uint8)
+    _check(_lib.aladdin_cluster_save(cl, buf.ctypes.data, C.byref(n)), "aladdin_cluster_save")
+    return buf.tobytes()
+
+
+def aladdin_cluster_restore(cl, blob):
+    buf = np.frombuffer(blob, np.uint8)
+    _check(_lib.aladdin_cluster_restore(cl, buf.ctypes.data, len(buf)), "aladdin_cluster_restore")
 
 
 def aladdin_cluster_advance(cl, dt_ms, stats=None):

@@ -759,6 +759,98 @@ int aladdin_cluster_advance(aladdin_cluster* cl, double dt_ms, double* stats)
     return ALADDIN_OK;
 }
 
+// Checkpoint layout: a header, then the device arrays in a fixed order.
+struct CheckpointHeader {
+    uint64_t magic;            // "ALADDIN1"
+    int32_t W, cap;
+    double t_now;
+    int64_t rid_next, rid_last;
+    int32_t round_open, pad;
+};
+constexpr uint64_t CKPT_MAGIC = 0x314e494444414c41ull;  // the bytes "ALADDIN1"
+
+// (device pointer, bytes) of every checkpointed array, in order.
+static void ckpt_arrays(aladdin_cluster* cl, void** ptr, size_t* len, int* count)
+{
+    const size_t W = (size_t)cl->W, S = W * (size_t)cl->cap;
+    ClusterDev& d = cl->dev;
+    void* p[] = {d.n, d.in, d.gen, d.pred, d.real, d.tdec, d.pend, d.wait, d.off, d.clock, d.le,
+                 d.be};
+    const size_t l[] = {4 * W, 4 * S, 4 * S, 4 * S, 4 * S, 8 * S, S, 8 * S, 4 * W, 8 * W,
+                        8 * W, 4 * W};
+    *count = (int)(sizeof(l) / sizeof(l[0]));
+    for (int i = 0; i < *count; ++i) {
+        ptr[i] = p[i];
+        len[i] = l[i];
+    }
+}
+
+int aladdin_cluster_save(aladdin_cluster* cl, void* buf, int64_t* bytes)
+{
+    if (!cl || !bytes) return ALADDIN_ERR_ARG;
+    void* ptr[16];
+    size_t len[16];
+    int k = 0;
+    ckpt_arrays(cl, ptr, len, &k);
+    size_t total = sizeof(CheckpointHeader);
+    for (int i = 0; i < k; ++i) total += len[i];
+    if (!buf) {
+        *bytes = (int64_t)total;
+        return ALADDIN_OK;
+    }
+    if (*bytes < (int64_t)total) return ALADDIN_ERR_ARG;
+    CK(cudaSetDevice(cl->device));
+    CheckpointHeader h;
+    std::memset(&h, 0, sizeof(h));
+    h.magic = CKPT_MAGIC;
+    h.W = cl->W;
+    h.cap = cl->cap;
+    h.t_now = cl->t_now;
+    h.rid_next = cl->rid_next;
+    h.rid_last = cl->rid_last;
+    h.round_open = cl->round_open ? 1 : 0;
+    unsigned char* out = static_cast<unsigned char*>(buf);
+    std::memcpy(out, &h, sizeof(h));
+    size_t at = sizeof(h);
+    for (int i = 0; i < k; ++i) {
+        CK(cudaMemcpyAsync(out + at, ptr[i], len[i], cudaMemcpyDeviceToHost, cl->st));
+        at += len[i];
+    }
+    CK(cudaStreamSynchronize(cl->st));
+    *bytes = (int64_t)total;
+    return ALADDIN_OK;
+}
+
+int aladdin_cluster_restore(aladdin_cluster* cl, const void* buf, int64_t bytes)
+{
+    if (!cl || !buf || bytes < (int64_t)sizeof(CheckpointHeader)) return ALADDIN_ERR_ARG;
+    CheckpointHeader h;
+    std::memcpy(&h, buf, sizeof(h));
+    if (h.magic != CKPT_MAGIC || h.W != cl->W || h.cap != cl->cap) return ALADDIN_ERR_ARG;
+    void* ptr[16];
+    size_t len[16];
+    int k = 0;
+    ckpt_arrays(cl, ptr, len, &k);
+    size_t total = sizeof(h);
+    for (int i = 0; i < k; ++i) total += len[i];
+    if (bytes < (int64_t)total) return ALADDIN_ERR_ARG;
+    CK(cudaSetDevice(cl->device));
+    const unsigned char* in = static_cast<const unsigned char*>(buf);
+    size_t at = sizeof(h);
+    for (int i = 0; i < k; ++i) {
+        CK(cudaMemcpyAsync(ptr[i], in + at, len[i], cudaMemcpyHostToDevice, cl->st));
+        at += len[i];
+    }
+    cl->t_now = h.t_now;
+    cl->rid_next = h.rid_next;
+    cl->rid_last = h.rid_last;
+    cl->round_open = h.round_open != 0;
+    int rc = refresh_tables(cl);
+    if (rc) return rc;
+    CK(cudaStreamSynchronize(cl->st));  // the host buffer may be released on return
+    return ALADDIN_OK;
+}
+
 int aladdin_cluster_state(aladdin_cluster* cl, int32_t* n, int32_t* in, int32_t* gen,
                           int32_t* pred, uint8_t* pending)
 {

@@ -355,3 +355,33 @@ def test_round_and_simulation_deterministic(A, synth):
                            A.trace_of(tr), 100.0, 0, 1, out)
         outs.append(out.tobytes())
     assert outs[0] == outs[1]
+
+
+def test_checkpoint_resume(A, synth):
+    """A cluster saved with an open round (pending placements, decode history,
+    clock) and restored into a fresh cluster of the same shape continues
+    exactly like the original: the same scores, placements and state."""
+    wl = synth.config("w256", n_cand=1500, b_cap=128, params=dict(T_dec=30.0))
+    h = (wl.req_gen * np.random.default_rng(3).uniform(8.0, 30.0, len(wl.req_gen))).astype(
+        np.float32)
+    with A.Cluster.from_workload(wl, tdec_ms=h) as a:
+        a.place_round(wl.cand_in[:400], wl.cand_pred[:400], wl.cand_wait[:400])
+        a.advance(100.0)
+        a.place_round(wl.cand_in[400:700], wl.cand_pred[400:700], wl.cand_wait[400:700])
+        blob = A.aladdin_cluster_save(a.handle)
+        with A.Cluster.from_workload(synth.config("w256", n_cand=4, b_cap=128,
+                                                  params=dict(T_dec=30.0))) as b:
+            A.aladdin_cluster_restore(b.handle, blob)
+            outs = []
+            for cl in (a, b):
+                s = cl.score(wl.cand_in[700:900], wl.cand_pred[700:900], wl.cand_wait[700:900])
+                pl = cl.place_round(wl.cand_in[700:], wl.cand_pred[700:], wl.cand_wait[700:])
+                st = cl.advance(100.0)
+                outs.append([s["flags"].tobytes(), s["margin"].tobytes(), s["argbest"].tobytes(),
+                             pl.tobytes()] + [x.tobytes() for x in cl.state()])
+            assert outs[0] == outs[1]
+    with A.Cluster.from_workload(synth.config("tiny")) as c:
+        with pytest.raises(A.AladdinError):
+            A.aladdin_cluster_restore(c.handle, blob)       # another shape
+        with pytest.raises(A.AladdinError):
+            A.aladdin_cluster_restore(c.handle, blob[:100])  # truncated
