@@ -2,10 +2,11 @@
 
 A step is one pass of the hot path over the 4,096-worker workload (128 ongoing
 requests per worker, 32,768 candidate queries, KV capacity 131,072, output
-lengths lognormal(256, 1.2) clipped at 4,096): the worker state, resident in
-HBM, is packed into the cluster and every worker's projection table is rebuilt
-(aladdin_cluster_load), then every candidate is scored against every worker
-with flags, margins and argbest written to HBM (aladdin_score).
+lengths lognormal(256, 1.2) clipped at 4,096), one aladdin_cluster_load_score
+call: the worker state, resident in HBM, is packed into the cluster and every
+worker's projection table is rebuilt (while the candidates are validated and
+sorted on a second stream), then every candidate is scored against every
+worker with flags, margins and argbest written to HBM.
 
 Prints one JSON line (rank 0). `value` is candidate x worker evaluations per
 second over all ranks with inputs resident in HBM; `e2e` is the same metric
@@ -380,9 +381,9 @@ def run_ours(args):
     flush = torch.empty(L2_FLUSH_BYTES // 4, dtype=torch.float32, device=dev)
     cl = A.Cluster.from_workload(wl, stream=stream)
 
-    def step():
-        A.aladdin_cluster_load(cl.handle, roff, rin, rgen, rpred)
-        A.aladdin_score(cl.handle, C, cin, cpr, cw, flags, margin, arg)
+    def step():  # the new state, then the candidates scored against it
+        A.aladdin_cluster_load_score(cl.handle, roff, rin, rgen, rpred, None, C, cin, cpr, cw,
+                                     flags, margin, arg)
 
     for _ in range(args.warmup):
         step()
@@ -418,8 +419,8 @@ def run_ours(args):
     h_arg = torch.empty(C, dtype=torch.int32).pin_memory()
 
     def step_host():
-        A.aladdin_cluster_load(cl.handle, h_roff, h_rin, h_rgen, h_rpred)
-        A.aladdin_score(cl.handle, C, h_cin, h_cpr, h_cw, h_flags, h_margin, h_arg)
+        A.aladdin_cluster_load_score(cl.handle, h_roff, h_rin, h_rgen, h_rpred, None, C, h_cin,
+                                     h_cpr, h_cw, h_flags, h_margin, h_arg)
 
     for _ in range(2):
         step_host()
@@ -780,8 +781,8 @@ def run_kernel_only(args):
     arg = torch.empty(C, dtype=torch.int32, device=dev)
     cl = A.Cluster.from_workload(wl, stream=torch.cuda.current_stream().cuda_stream)
     for _ in range(args.warmup + args.steps):
-        A.aladdin_cluster_load(cl.handle, roff, rin, rgen, rpred)
-        A.aladdin_score(cl.handle, C, cin, cpr, cw, flags, margin, arg)
+        A.aladdin_cluster_load_score(cl.handle, roff, rin, rgen, rpred, None, C, cin, cpr, cw,
+                                     flags, margin, arg)
     torch.cuda.synchronize()
     assert cl.status() == A.OK
     cl.close()

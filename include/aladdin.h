@@ -194,6 +194,20 @@ int aladdin_cluster_load(aladdin_cluster* cl, const int32_t* req_off, const int3
 int aladdin_score(aladdin_cluster* cl, int32_t n_cand, const int32_t* in, const int32_t* pred,
                   const float* wait_ms, uint8_t* flags, float* margin, int32_t* argbest);
 
+/* aladdin_cluster_load followed by aladdin_score in one call (a scheduling
+ * heartbeat: the workers' new state, then the waiting requests scored
+ * against it), with the same arguments and results. When every array is
+ * device memory (or mapped page-locked host memory) the candidates are
+ * validated and sorted on a second stream while the cluster's stream packs
+ * the state and builds the tables; the two join before the scoring kernel,
+ * and the call stays ordered on the cluster's stream like the two calls.
+ * Otherwise it runs the two calls in sequence. */
+int aladdin_cluster_load_score(aladdin_cluster* cl, const int32_t* req_off, const int32_t* in,
+                               const int32_t* gen, const int32_t* pred, const float* tdec_ms,
+                               int32_t n_cand, const int32_t* cand_in, const int32_t* cand_pred,
+                               const float* wait_ms, uint8_t* flags, float* margin,
+                               int32_t* argbest);
+
 /* As aladdin_score, plus two verification outputs per pair (each nullable):
  * kv_peak [n_cand*W]: the worker's peak KV usage over all future iterations
  * with the candidate added (exact integer), and t_cand_ms [n_cand*W]: the

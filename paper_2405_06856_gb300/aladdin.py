@@ -92,6 +92,7 @@ _sig = {
     "aladdin_predict_workers": [C.c_double, C.c_double, C.c_double, _P],
     "aladdin_rebalance": [_P, C.c_int32, _P, _P, _P, _P, _P, _P, _P, _P],
     "aladdin_cluster_save": [_P, _P, _P],
+    "aladdin_cluster_load_score": [_P, _P, _P, _P, _P, _P, C.c_int32, _P, _P, _P, _P, _P, _P],
     "aladdin_cluster_restore": [_P, _P, C.c_int64],
 }
 for _n, _a in _sig.items():
@@ -200,6 +201,17 @@ def aladdin_cluster_load(cl, req_off, req_in, req_gen, req_pred, tdec_ms=None):
 def aladdin_score(cl, n_cand, cand_in, cand_pred, wait_ms, flags, margin, argbest):
     _check(_lib.aladdin_score(cl, int(n_cand), _ptr(cand_in), _ptr(cand_pred), _ptr(wait_ms),
                               _ptr(flags), _ptr(margin), _ptr(argbest)), "aladdin_score")
+
+
+def aladdin_cluster_load_score(cl, req_off, req_in, req_gen, req_pred, tdec_ms, n_cand, cand_in,
+                               cand_pred, wait_ms, flags, margin, argbest):
+    """aladdin_cluster_load then aladdin_score in one call (overlapped on the
+    device when every array is device memory)."""
+    _check(_lib.aladdin_cluster_load_score(cl, _ptr(req_off), _ptr(req_in), _ptr(req_gen),
+                                           _ptr(req_pred), _ptr(tdec_ms), int(n_cand),
+                                           _ptr(cand_in), _ptr(cand_pred), _ptr(wait_ms),
+                                           _ptr(flags), _ptr(margin), _ptr(argbest)),
+           "aladdin_cluster_load_score")
 
 
 def aladdin_score_noalloc(cl, n_cand, cand_in, cand_pred, wait_ms, flags, margin, argbest):

@@ -23,12 +23,20 @@ struct ScoreBuffers {
 };
 
 // K3 pipeline: validate + derive + counting-sort candidates by predicted
-// output, score every pair, finalize argbest. Device pointers only.
+// output, score every pair, finalize argbest. Device pointers only. With
+// prepared, the candidates were sorted into B by launch_cand_prep already
+// (its stream ordered before st by the caller).
 cudaError_t launch_score(const DevParams& P, const ClusterDev& C, int n_cand, const int32_t* in,
                          const int32_t* pred, const float* wait, uint8_t* flags, float* margin,
                          int32_t* argbest, int64_t* kv_peak, float* t_cand, const ScoreBuffers& B,
                          bool pend, cudaStream_t st, cudaEvent_t ev0 = nullptr,
-                         cudaEvent_t ev1 = nullptr);
+                         cudaEvent_t ev1 = nullptr, bool prepared = false);
+// The candidate preparation of launch_score alone (it reads no table): the
+// validated per-candidate records sorted by predicted output, and the
+// argbest keys reset. W is the cluster's worker count (output row stride).
+cudaError_t launch_cand_prep(const DevParams& P, int W, int n_cand, const int32_t* in,
+                             const int32_t* pred, const float* wait, const ScoreBuffers& B,
+                             cudaStream_t st);
 
 // K4: one greedy round over candidates in index order.
 struct RoundIO {

@@ -173,6 +173,10 @@ struct aladdin_cluster {
     unsigned long long* d_stats = nullptr;
     int* d_status = nullptr;
     void* d_xround = nullptr;  // exchange buffer of the sliced placement round
+    // aladdin_cluster_load_score: a side stream for the candidate preparation
+    // and the events that fork it from and join it to the cluster's stream
+    cudaStream_t side = nullptr;
+    cudaEvent_t ev_fork = nullptr, ev_join = nullptr;
     // optional CUDA-event timing of the scoring kernel
     bool timing = false;
     std::vector<cudaEvent_t> ev;   // pairs (start, stop)
@@ -202,6 +206,9 @@ struct aladdin_cluster {
     }
     ~aladdin_cluster()
     {
+        if (ev_fork) cudaEventDestroy(ev_fork);
+        if (ev_join) cudaEventDestroy(ev_join);
+        if (side) cudaStreamDestroy(side);
         clear_events();
         for (cudaEvent_t e : ev_free) cudaEventDestroy(e);
         for (void* p : owned) cudaFree(p);
@@ -602,6 +609,83 @@ int aladdin_cluster_load(aladdin_cluster* cl, const int32_t* req_off, const int3
     if (rc) return rc;
     cl->round_open = false;
     return refresh_tables(cl);
+}
+
+int aladdin_cluster_load_score(aladdin_cluster* cl, const int32_t* req_off, const int32_t* in,
+                               const int32_t* gen, const int32_t* pred, const float* tdec_ms,
+                               int32_t n_cand, const int32_t* cand_in, const int32_t* cand_pred,
+                               const float* wait_ms, uint8_t* flags, float* margin,
+                               int32_t* argbest)
+{
+    if (!cl || n_cand < 0) return ALADDIN_ERR_ARG;
+    // every array on the device (or mapped): overlap; otherwise the two calls
+    auto dv = [](const void* p) {
+        void* d = nullptr;
+        return !p || device_view(p, &d);
+    };
+    const bool dev = req_off && dv(req_off) && dv(in) && dv(gen) && dv(pred) && dv(tdec_ms) &&
+                     dv(cand_in) && dv(cand_pred) && dv(wait_ms) && dv(flags) && dv(margin) &&
+                     dv(argbest) && (flags || margin || argbest);
+    int rc;
+    if (!dev || n_cand == 0) {
+        if ((rc = aladdin_cluster_load(cl, req_off, in, gen, pred, tdec_ms))) return rc;
+        return aladdin_score(cl, n_cand, cand_in, cand_pred, wait_ms, flags, margin, argbest);
+    }
+    if (!cand_in || !cand_pred) return ALADDIN_ERR_ARG;
+    CK(cudaSetDevice(cl->device));
+    if (!cl->side) {
+        CK(cudaStreamCreateWithFlags(&cl->side, cudaStreamNonBlocking));
+        CK(cudaEventCreateWithFlags(&cl->ev_fork, cudaEventDisableTiming));
+        CK(cudaEventCreateWithFlags(&cl->ev_join, cudaEventDisableTiming));
+    }
+    int32_t *cin = nullptr, *cpr = nullptr;
+    float* cw = nullptr;
+    uint8_t* df = nullptr;
+    float* dm = nullptr;
+    int32_t* da = nullptr;
+    device_view(cand_in, &cin);
+    device_view(cand_pred, &cpr);
+    if (wait_ms) device_view(wait_ms, &cw);
+    if (flags) device_view(flags, &df);
+    if (margin) device_view(margin, &dm);
+    if (argbest) device_view(argbest, &da);
+    const size_t C = (size_t)n_cand;
+    CK(cl->sorted.ensure(sizeof(float4) * 5 * C));
+    CK(cl->hist.ensure(sizeof(int32_t) * ((size_t)cl->hp.K + 2)));
+    CK(cl->best.ensure(sizeof(unsigned int) * C));
+    ScoreBuffers B{cl->sorted.as<float4>(), cl->hist.as<int32_t>(), cl->best.as<unsigned int>()};
+    // fork: the candidates are sorted on the side stream (they read no table)
+    // while the cluster's stream packs the state and builds the tables
+    CK(cudaEventRecord(cl->ev_fork, cl->st));
+    CK(cudaStreamWaitEvent(cl->side, cl->ev_fork, 0));
+    CK(launch_cand_prep(cl->dp, cl->W, n_cand, cin, cpr, cw, B, cl->side));
+    CK(cudaEventRecord(cl->ev_join, cl->side));
+    rc = load_requests(cl, req_off, in, gen, pred, tdec_ms);
+    if (!rc) {
+        cl->round_open = false;
+        rc = refresh_tables(cl);
+    }
+    CK(cudaStreamWaitEvent(cl->st, cl->ev_join, 0));  // join (also on error)
+    if (rc) return rc;
+    cudaEvent_t e0 = nullptr, e1 = nullptr;
+    if (cl->timing) {
+        e0 = cl->take_event();
+        e1 = cl->take_event();
+        if (e0 && e1) {
+            cl->ev.push_back(e0);
+            cl->ev.push_back(e1);
+        } else {
+            e0 = e1 = nullptr;
+        }
+    }
+    CK(launch_score(cl->dp, cl->dev, n_cand, cin, cpr, cw, df, dm, da, nullptr, nullptr, B, false,
+                    cl->st, e0, e1, true));
+    auto on_host = [](const void* p) { return p && ptr_kind(p) != PK_DEV; };
+    if (on_host(req_off) || on_host(in) || on_host(gen) || on_host(pred) || on_host(tdec_ms) ||
+        on_host(cand_in) || on_host(cand_pred) || on_host(wait_ms) || on_host(flags) ||
+        on_host(margin) || on_host(argbest))
+        CK(cudaStreamSynchronize(cl->st));
+    return ALADDIN_OK;
 }
 
 int aladdin_score(aladdin_cluster* cl, int32_t n_cand, const int32_t* in, const int32_t* pred,

@@ -703,23 +703,33 @@ __global__ void k_detail(DevParams P, ClusterDev C, int n, const int32_t* __rest
     }
 }
 
+cudaError_t launch_cand_prep(const DevParams& P, int W, int n, const int32_t* in,
+                             const int32_t* pred, const float* wait, const ScoreBuffers& B,
+                             cudaStream_t st)
+{
+    if (n <= 0) return cudaSuccess;
+    const int tb = 256, nb = (n + tb - 1) / tb;
+    cudaError_t e = cudaMemsetAsync(B.hist, 0, sizeof(int32_t) * (size_t)(P.K + 1), st);
+    if (e != cudaSuccess) return e;
+    k_cand_count<<<nb, tb, 0, st>>>(P, n, in, pred, wait, B.hist, B.best);
+    k_scan_hist<<<1, SCAN_THREADS, 0, st>>>(B.hist, P.K + 1);
+    k_cand_scatter<<<nb, tb, 0, st>>>(P, n, W, in, pred, wait, B.hist, B.sorted);
+    return cudaGetLastError();
+}
+
 cudaError_t launch_score(const DevParams& P, const ClusterDev& C, int n, const int32_t* in,
                          const int32_t* pred, const float* wait, uint8_t* flags, float* margin,
                          int32_t* argbest, int64_t* kv_peak, float* t_cand, const ScoreBuffers& B,
-                         bool pend, cudaStream_t st, cudaEvent_t ev0, cudaEvent_t ev1)
+                         bool pend, cudaStream_t st, cudaEvent_t ev0, cudaEvent_t ev1,
+                         bool prepared)
 {
     if (n <= 0) return cudaSuccess;
     cudaError_t e;
     const int tb = 256, nb = (n + tb - 1) / tb;
     const bool need_score = flags || margin || argbest;
     if (need_score) {
-        e = cudaMemsetAsync(B.hist, 0, sizeof(int32_t) * (size_t)(P.K + 1), st);
-        if (e != cudaSuccess) return e;
-        k_cand_count<<<nb, tb, 0, st>>>(P, n, in, pred, wait, B.hist, B.best);
-        k_scan_hist<<<1, SCAN_THREADS, 0, st>>>(B.hist, P.K + 1);
-        k_cand_scatter<<<nb, tb, 0, st>>>(P, n, C.W, in, pred, wait, B.hist, B.sorted);
-        e = cudaGetLastError();
-        if (e != cudaSuccess) return e;
+        if (!prepared && (e = launch_cand_prep(P, C.W, n, in, pred, wait, B, st)) != cudaSuccess)
+            return e;
 
         ScoreArgs A;
         A.C = C;

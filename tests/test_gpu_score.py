@@ -249,3 +249,42 @@ def test_page_locked_host_buffers(A, orc, synth):
         A.aladdin_place_round(cl.handle, C, pin(wl.cand_in), pin(wl.cand_pred), pin(wl.cand_wait), hp)
         rp = orc.Cluster.from_workload(wl).place_round(wl.cand_in, wl.cand_pred, wl.cand_wait)
         assert np.array_equal(hp.numpy(), rp)
+
+
+def test_load_score_equals_two_calls(A, synth):
+    """aladdin_cluster_load_score (candidates sorted on a second stream while
+    the tables are built) gives the bytes of aladdin_cluster_load followed by
+    aladdin_score, from device and from host arrays, and leaves the cluster in
+    the same state."""
+    import torch
+    wl = synth.config("w256", n_cand=1500)
+    wl2 = synth.config("w256", n_cand=1500, seed=77)   # the state loaded by the step
+    dev = torch.device("cuda")
+    t = lambda x: torch.from_numpy(np.ascontiguousarray(x)).to(dev)
+    C, W = wl.n_cand, wl.n_workers
+    outs = []
+    for mode in ("two", "one_dev", "one_host"):
+        with A.Cluster.from_workload(wl) as cl:
+            if mode == "one_host":
+                f = np.zeros((C, W), np.uint8)
+                m = np.zeros((C, W), np.float32)
+                a = np.zeros(C, np.int32)
+                A.aladdin_cluster_load_score(cl.handle, wl2.roff, wl2.req_in, wl2.req_gen,
+                                             wl2.req_pred, None, C, wl.cand_in, wl.cand_pred,
+                                             wl.cand_wait, f, m, a)
+            else:
+                f = torch.zeros((C, W), dtype=torch.uint8, device=dev)
+                m = torch.zeros((C, W), dtype=torch.float32, device=dev)
+                a = torch.zeros(C, dtype=torch.int32, device=dev)
+                args = (t(wl2.roff), t(wl2.req_in), t(wl2.req_gen), t(wl2.req_pred))
+                cand = (t(wl.cand_in), t(wl.cand_pred), t(wl.cand_wait))
+                if mode == "two":
+                    A.aladdin_cluster_load(cl.handle, *args)
+                    A.aladdin_score(cl.handle, C, *cand, f, m, a)
+                else:
+                    A.aladdin_cluster_load_score(cl.handle, *args, None, C, *cand, f, m, a)
+                torch.cuda.synchronize()
+                f, m, a = f.cpu().numpy(), m.cpu().numpy(), a.cpu().numpy()
+            outs.append((f.tobytes(), m.tobytes(), a.tobytes(),
+                         tuple(x.tobytes() for x in cl.state())))
+    assert outs[0] == outs[1] == outs[2]
