@@ -113,3 +113,28 @@ def test_grouped_round_full_worker_stops_its_group(A, orc, synth):
     assert full and np.array_equal(pl, ref)
     assert list(pl[:4]) == [0, 1, -1, 1] and (pl[1::2] == 1).all() and (pl[2::2] == -1).all()
     assert list(n) == [32, 20] == list(oc.n)
+
+
+@pytest.mark.parametrize("extra", [
+    dict(phase=1, mode=1, groups=2, rebalance=1, theta=0.9),     # decode, approximate, Alg. 2
+    dict(phase=1, policy=2, groups=3, seed=4),                  # decode, power of two
+    dict(phase=0, mode=1, groups=3, rebalance=1, theta=0.85),   # mixed, approximate, Alg. 2
+])
+def test_features_compose(A, orc, synth, extra):
+    """Decode instances, the approximate constraints, grouped scheduling,
+    Algorithm 2 and prediction errors together: the simulation matches the
+    oracle output for output."""
+    te = synth.with_prediction_error(synth.diurnal_trace(21, 1200, 60.0, 15.0), 0.4, 21)
+    p = dict(synth.BASE_PARAMS, T_dec=30.0, **extra)
+    for N in (5, 8):
+        ref = orc.simulate(p, N, 256, 40000, 1.0, te, 100.0, stop_at_fail=False, drain=True)
+        out = np.zeros(A.SIMULATE_OUT)
+        A.aladdin_simulate(A.make_params(p, 256), A.make_cfgs([1], [40000], [1.0])[0], N,
+                           A.trace_of(te), 100.0, 0, 1, out)
+        lab = (extra, N, out, ref)
+        assert int(out[0]) == ref["failed"] and int(out[1]) == ref["placed"], lab
+        assert int(out[2]) == ref["heartbeats"] and int(out[5]) == ref["violations"], lab
+        assert out[3] == pytest.approx(ref["max_ttft"], rel=1e-12), lab
+        assert out[4] == pytest.approx(ref["max_atgt"], rel=1e-12), lab
+        assert int(out[6]) == ref["repredictions"] and int(out[7]) == ref["early_finishes"], lab
+        assert int(out[8]) == ref["moved"], lab
