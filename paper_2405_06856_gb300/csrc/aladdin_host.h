@@ -16,8 +16,12 @@ cudaError_t launch_build(const DevParams& P, const ClusterDev& C, const int32_t*
 // capacity_norm ranks (descending key, lowest index on ties) and rank -> worker.
 cudaError_t launch_rank(const ClusterDev& C, cudaStream_t st);
 
+// float4 words of one sorted candidate record, the scoring kernels' input
+// (layout and writer: k_cand_scatter in score.cu)
+constexpr int CAND_REC_F4 = 3;
+
 struct ScoreBuffers {
-    float4* sorted;        // [n_cand * 5] sorted candidate records
+    float4* sorted;        // [n_cand * CAND_REC_F4] sorted candidate records
     int32_t* hist;         // [K + 2]
     unsigned int* best;    // [n_cand]
 };

@@ -518,7 +518,7 @@ int score_impl(aladdin_cluster* cl, int32_t n, const int32_t* in, const int32_t*
         (rc = stage_out(cl->s_kv, kv_peak, pairs, &dkv, &hk)) ||
         (rc = stage_out(cl->s_tc, t_cand, pairs, &dtc, &ht)))
         return rc;
-    CK(cl->sorted.ensure(sizeof(float4) * 5 * C));
+    CK(cl->sorted.ensure(sizeof(float4) * CAND_REC_F4 * C));
     CK(cl->hist.ensure(sizeof(int32_t) * ((size_t)cl->hp.K + 2)));
     CK(cl->best.ensure(sizeof(unsigned int) * C));
     ScoreBuffers B{cl->sorted.as<float4>(), cl->hist.as<int32_t>(), cl->best.as<unsigned int>()};
@@ -650,7 +650,7 @@ int aladdin_cluster_load_score(aladdin_cluster* cl, const int32_t* req_off, cons
     if (margin) device_view(margin, &dm);
     if (argbest) device_view(argbest, &da);
     const size_t C = (size_t)n_cand;
-    CK(cl->sorted.ensure(sizeof(float4) * 5 * C));
+    CK(cl->sorted.ensure(sizeof(float4) * CAND_REC_F4 * C));
     CK(cl->hist.ensure(sizeof(int32_t) * ((size_t)cl->hp.K + 2)));
     CK(cl->best.ensure(sizeof(unsigned int) * C));
     ScoreBuffers B{cl->sorted.as<float4>(), cl->hist.as<int32_t>(), cl->best.as<unsigned int>()};

@@ -25,7 +25,7 @@
 namespace {
 
 constexpr int NOALLOC_MAX_CAND = ALADDIN_NOALLOC_MAX_CAND;
-constexpr size_t REC_BYTES = (size_t)NOALLOC_MAX_CAND * 48;  // sorted records, 3 x float4 each
+constexpr size_t REC_BYTES = (size_t)NOALLOC_MAX_CAND * aladdin::CAND_REC_F4 * 16;  // sorted records
 constexpr size_t HIST_BYTES = ((size_t)(65536 + 2) * 4 + 255) / 256 * 256;  // K <= 65536
 constexpr size_t BEST_BYTES = (size_t)NOALLOC_MAX_CAND * 4;
 constexpr size_t SCRATCH_BYTES = REC_BYTES + HIST_BYTES + BEST_BYTES;
