@@ -357,7 +357,15 @@ typedef struct aladdin_trace {
  * meet them by construction. n_workers[o] = -1 if n_max workers fail.
  * best_option (nullable) receives the option with the fewest total GPUs
  * (gpus * n_workers; first on ties), total_gpus (nullable) that total. Trace
- * arrays are host memory. */
+ * arrays are host memory.
+ * Execution: cuda_stream carries the trace upload (synchronised before any
+ * simulation starts). The simulations run side by side on host threads of
+ * the library, each on a non-blocking stream of its own on the current
+ * device, with device memory from a private stream-ordered pool that is
+ * trimmed on return: the options' searches at once, and per search the next
+ * doubling steps or the next levels of bisection at once. The result equals
+ * that of the sequential doubling-and-bisection search. Returns when every
+ * simulation has finished. */
 int aladdin_min_workers(const aladdin_params* params, int32_t n_options,
                         const aladdin_worker_cfg* options, const aladdin_trace* trace,
                         double heartbeat_ms, int32_t n_max, void* cuda_stream,
@@ -441,7 +449,8 @@ int aladdin_pick_config(const aladdin_params* params, int32_t n_options,
  * squares over the traces whose rate exceeds R and whose search succeeded.
  * Returns ALADDIN_ERR_ARG (after filling n_workers, with k5 = c5 = 0) when
  * fewer than two such traces, or only one distinct rate, remain. Trace arrays
- * are host memory; every simulation runs on the GPU. */
+ * are host memory; every simulation runs on the GPU, the traces' searches
+ * side by side (as in aladdin_min_workers). */
 int aladdin_fit_workers(const aladdin_params* params, const aladdin_worker_cfg* cfg,
                         int32_t n_traces, const aladdin_trace* traces, const double* rates,
                         double R, double heartbeat_ms, int32_t n_max, void* cuda_stream,

@@ -75,11 +75,19 @@ struct RoundIO {
     int32_t* sim_pl;
     long long* sim_tix;
     int* sim_n;
+    // host routing only: never the multi-CTA (cooperative) sliced round, for
+    // simulations that run side by side with others
+    int single_cta;
 };
 constexpr int ROUND_XBUF_SMS = 1024;  // largest SM count the exchange buffer serves
 constexpr size_t ROUND_XBUF_BYTES = 32 * (size_t)ROUND_XBUF_SMS + 16;
 cudaError_t launch_round(const DevParams& P, const ClusterDev& C, const RoundIO& io,
                          cudaStream_t st);
+// CTAs of the best-fit round launch_round runs for W workers of cap slots
+// (K the length limit): > 1 cooperative, 1 the sliced round on one CTA, 0 the
+// plain single-CTA round, -1 none (a single-CTA request beyond what one CTA
+// holds at 1,024 slots, or a failed device query).
+int round_ctas(int W, int cap, int K, bool single_cta);
 
 // Execution of every worker for dt ms from t_now.
 // stats: device [0] prefills run, [1] finished, [2] max TTFT bits, [3] max

@@ -1,9 +1,15 @@
 // C ABI of the library (include/aladdin.h): cluster object, pointer
 // classification and staging, host-side validation, and the heartbeat loop of
 // the fleet simulation and minimum-worker search.
+#include <algorithm>
+#include <atomic>
+#include <chrono>
 #include <cmath>
 #include <cstring>
+#include <mutex>
 #include <new>
+#include <set>
+#include <thread>
 #include <vector>
 
 #include "../../include/aladdin.h"
@@ -182,9 +188,12 @@ struct aladdin_cluster {
     std::vector<cudaEvent_t> ev;   // pairs (start, stop)
     std::vector<cudaEvent_t> ev_free;
 
+    // stream-ordered pool of the device memory (nullptr: cudaMalloc): memory
+    // allocated and released in the order of the cluster's stream
+    cudaMemPool_t pool = nullptr;
     cudaError_t alloc(void** p, size_t bytes)
     {
-        cudaError_t e = cudaMalloc(p, bytes);
+        cudaError_t e = pool ? cudaMallocFromPoolAsync(p, bytes, pool, st) : cudaMalloc(p, bytes);
         if (e == cudaSuccess) owned.push_back(*p);
         return e;
     }
@@ -211,7 +220,10 @@ struct aladdin_cluster {
         if (side) cudaStreamDestroy(side);
         clear_events();
         for (cudaEvent_t e : ev_free) cudaEventDestroy(e);
-        for (void* p : owned) cudaFree(p);
+        for (void* p : owned) {
+            if (pool) cudaFreeAsync(p, st);
+            else cudaFree(p);
+        }
         DevBuf* bufs[] = {&sorted, &hist, &best, &s_in, &s_pred, &s_wait, &s_flags, &s_margin,
                           &s_arg, &s_kv, &s_tc, &s_place, &s_off, &s_rin, &s_rgen, &s_rpred,
                           &s_rtdec};
@@ -1012,6 +1024,9 @@ struct DevTrace {
     int32_t* real = nullptr;    // nullptr: exact predictions
     int32_t* repred = nullptr;  // nullptr: re-predict x + 1
     std::vector<double> host_t;
+    DevTrace() = default;
+    DevTrace(const DevTrace&) = delete;
+    DevTrace& operator=(const DevTrace&) = delete;
     ~DevTrace()
     {
         if (t) cudaFree(t);
@@ -1068,11 +1083,67 @@ __global__ void k_busy(const int32_t* __restrict__ n, int W, int* out)
 }
 
 // One simulation; out[0..8] as aladdin_simulate.
+// Stream-ordered memory pool of the current device for simulations that run
+// side by side: their clusters are allocated and released in stream order,
+// so no cudaFree synchronises the device under the others. Freed memory stays
+// in the pool for the next simulation until trim_sim_pool. nullptr on error.
+cudaMemPool_t sim_pool()
+{
+    static std::mutex mu;
+    static cudaMemPool_t pools[64] = {};
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) {
+        cudaGetLastError();
+        return nullptr;
+    }
+    std::lock_guard<std::mutex> lock(mu);
+    if (!pools[dev]) {
+        cudaMemPoolProps props;
+        std::memset(&props, 0, sizeof(props));
+        props.allocType = cudaMemAllocationTypePinned;
+        props.location.type = cudaMemLocationTypeDevice;
+        props.location.id = dev;
+        cudaMemPool_t pool = nullptr;
+        if (cudaMemPoolCreate(&pool, &props) != cudaSuccess) {
+            cudaGetLastError();
+            return nullptr;
+        }
+        unsigned long long keep = ~0ull;
+        cudaMemPoolSetAttribute(pool, cudaMemPoolAttrReleaseThreshold, &keep);
+        pools[dev] = pool;
+    }
+    return pools[dev];
+}
+
+// Returns the pool's free memory to the device (after a search, once every
+// simulation's stream has drained).
+void trim_sim_pool()
+{
+    cudaMemPool_t pool = sim_pool();
+    if (pool) cudaMemPoolTrimTo(pool, 0);
+}
+
+// Waits for the stream's work. Polite (polling with short sleeps instead of
+// the driver's spin) when many simulations share the host's cores.
+cudaError_t wait_stream(cudaStream_t st, bool polite)
+{
+    if (!polite) return cudaStreamSynchronize(st);
+    for (;;) {
+        const cudaError_t e = cudaStreamQuery(st);
+        if (e != cudaErrorNotReady) return e;
+        cudaGetLastError();  // "not ready" is recorded as the thread's last error
+        std::this_thread::sleep_for(std::chrono::microseconds(50));
+    }
+}
+
+// concurrent: other simulations may run at the same time (polite waits);
+// single_cta: no cooperative multi-CTA placement round.
 int simulate_impl(const aladdin_params& p, const aladdin_worker_cfg& cfg, int32_t N,
                   const DevTrace& tr, double H, bool stop_at_fail, bool drain, cudaStream_t st,
-                  double* out)
+                  double* out, bool concurrent = false, bool single_cta = false)
 {
     aladdin_cluster cl;
+    if (concurrent && (cl.pool = sim_pool()) == nullptr) return ALADDIN_ERR_CUDA;
     std::vector<aladdin_worker_cfg> cfgs((size_t)N, cfg);
     int rc = cluster_alloc(&cl, p, N, cfgs.data(), st);
     if (rc) return rc;
@@ -1080,18 +1151,20 @@ int simulate_impl(const aladdin_params& p, const aladdin_worker_cfg& cfg, int32_
     if (rc) return rc;
     cl.dev.repred = tr.repred;  // the kernels get the cluster view by value
     const bool rebal = p.rebalance != 0 && p.policy == ALADDIN_POLICY_BESTFIT;
-    DevBuf wl, cnt, rpl, rtix;
-    CK(wl.ensure(sizeof(long long) * (size_t)(tr.n > 0 ? tr.n : 1)));
-    CK(cnt.ensure(sizeof(unsigned long long) * 4 + sizeof(int) * 4));
-    unsigned long long* counters = cnt.as<unsigned long long>();
+    // the simulation's buffers, owned (and released) by its cluster
+    const size_t nt = (size_t)(tr.n > 0 ? tr.n : 1);
+    void *wl_p = nullptr, *cnt_p = nullptr, *rpl_p = nullptr, *rtix_p = nullptr;
+    CK(cl.alloc(&wl_p, sizeof(long long) * nt));
+    CK(cl.alloc(&cnt_p, sizeof(unsigned long long) * 4 + sizeof(int) * 4));
+    unsigned long long* counters = static_cast<unsigned long long*>(cnt_p);
     int* nwait = reinterpret_cast<int*>(counters + 4);
     int* busy = nwait + 1;
     int* rb_n = nwait + 2;      // candidates of the last round (Algorithm 2)
     int* rb_moves = nwait + 3;  // requests moved by Algorithm 2
-    CK(cudaMemsetAsync(cnt.p, 0, sizeof(unsigned long long) * 4 + sizeof(int) * 4, st));
+    CK(cudaMemsetAsync(cnt_p, 0, sizeof(unsigned long long) * 4 + sizeof(int) * 4, st));
     if (rebal) {
-        CK(rpl.ensure(sizeof(int32_t) * (size_t)(tr.n > 0 ? tr.n : 1)));
-        CK(rtix.ensure(sizeof(long long) * (size_t)(tr.n > 0 ? tr.n : 1)));
+        CK(cl.alloc(&rpl_p, sizeof(int32_t) * nt));
+        CK(cl.alloc(&rtix_p, sizeof(long long) * nt));
     }
 
     int64_t next = 0;
@@ -1108,7 +1181,7 @@ int simulate_impl(const aladdin_params& p, const aladdin_worker_cfg& cfg, int32_
         io.t_arr = tr.t;
         io.tin = tr.in;
         io.tpred = tr.pred;
-        io.wl = wl.as<long long>();
+        io.wl = static_cast<long long*>(wl_p);
         io.n_wait = nwait;
         io.arr_begin = next;
         io.arr_end = end;
@@ -1119,10 +1192,11 @@ int simulate_impl(const aladdin_params& p, const aladdin_worker_cfg& cfg, int32_
         io.stop_at_fail = stop_at_fail ? 1 : 0;
         io.hb = hb;
         io.xbuf = cl.d_xround;
+        io.single_cta = single_cta ? 1 : 0;
         io.treal = tr.real;
         if (rebal) {
-            io.sim_pl = rpl.as<int32_t>();
-            io.sim_tix = rtix.as<long long>();
+            io.sim_pl = static_cast<int32_t*>(rpl_p);
+            io.sim_tix = static_cast<long long*>(rtix_p);
             io.sim_n = rb_n;
         }
         const bool bestfit = p.policy == ALADDIN_POLICY_BESTFIT;
@@ -1149,7 +1223,7 @@ int simulate_impl(const aladdin_params& p, const aladdin_worker_cfg& cfg, int32_
             CK(cudaMemcpyAsync(hs, nwait, sizeof(hs), cudaMemcpyDeviceToHost, st));
             int status = 0;
             CK(cudaMemcpyAsync(&status, cl.d_status, sizeof(int), cudaMemcpyDeviceToHost, st));
-            CK(cudaStreamSynchronize(st));
+            CK(wait_stream(st, concurrent));
             if (status == -2) return ALADDIN_ERR_CAPACITY;
             if (status == -4) return ALADDIN_ERR_TIMEOUT;
             if (status == 1) {
@@ -1164,7 +1238,7 @@ int simulate_impl(const aladdin_params& p, const aladdin_worker_cfg& cfg, int32_
     CK(cudaMemcpyAsync(s, cl.d_stats, sizeof(s), cudaMemcpyDeviceToHost, st));
     CK(cudaMemcpyAsync(hc, counters, sizeof(hc), cudaMemcpyDeviceToHost, st));
     CK(cudaMemcpyAsync(hm, rb_n, sizeof(hm), cudaMemcpyDeviceToHost, st));
-    CK(cudaStreamSynchronize(st));
+    CK(wait_stream(st, concurrent));
     out[0] = (double)hc[0];
     out[1] = (double)hc[1];
     out[2] = halted ? (double)hc[2] : (double)hb;
@@ -1174,45 +1248,160 @@ int simulate_impl(const aladdin_params& p, const aladdin_worker_cfg& cfg, int32_
     out[6] = (double)s[7];
     out[7] = (double)s[8];
     out[8] = (double)hm[1];
-    rpl.release();
-    rtix.release();
-    wl.release();
-    cnt.release();
     return ALADDIN_OK;
 }
 
+// One simulation of the worker search: its worker count and, once it ran,
+// its status and whether the trace was served without a failure.
+struct SimProbe {
+    int32_t n = 0;
+    int rc = ALADDIN_OK;
+    bool pass = false;
+};
+
+// Held by the one simulation of the process that may run cooperative
+// (grid-synchronised, multi-CTA) placement rounds while others run beside
+// it: two such grids could each wait for SMs that the other holds.
+std::atomic<int> g_coop_token{0};
+
+// Runs the probes side by side, one host thread and one non-blocking stream
+// each. A simulation is a chain of small launches that keeps about one SM
+// busy, so several at once fill the GPU; they share only the read-only trace.
+// Rounds that would span several CTAs run on one CTA instead (the sliced
+// round with fewer rows per worker in shared memory; same placements), except
+// in probes that one CTA cannot serve, which wait for the cooperative token.
+// Falls back to one at a time if no thread can be started.
+void run_probes(const aladdin_params& p, const aladdin_worker_cfg& cfg, const DevTrace& tr,
+                double H, bool drain, int device, std::vector<SimProbe>& probes)
+{
+    const bool bestfit = p.policy == ALADDIN_POLICY_BESTFIT;
+    // probes that no single-CTA round serves must hold the cooperative token
+    std::vector<char> need(probes.size(), 0);
+    for (size_t k = 0; k < probes.size(); ++k)
+        need[k] = bestfit && round_ctas(probes[k].n, p.b_cap, p.K, true) < 0;
+    auto one = [&](size_t k) {
+        SimProbe* q = &probes[k];
+        cudaStream_t s = nullptr;
+        if (cudaSetDevice(device) != cudaSuccess ||
+            cudaStreamCreateWithFlags(&s, cudaStreamNonBlocking) != cudaSuccess) {
+            cudaGetLastError();
+            q->rc = ALADDIN_ERR_CUDA;
+            return;
+        }
+        const bool coop = need[k] != 0;
+        if (coop)
+            while (g_coop_token.exchange(1) != 0)
+                std::this_thread::sleep_for(std::chrono::milliseconds(1));
+        double out[9];
+        q->rc = simulate_impl(p, cfg, q->n, tr, H, true, drain, s, out, true, !coop);
+        q->pass = q->rc == ALADDIN_OK && out[0] == 0.0;
+        if (coop) g_coop_token.store(0);
+        cudaStreamDestroy(s);
+    };
+    std::vector<std::thread> th;
+    size_t started = 0;
+    try {
+        th.reserve(probes.size());
+        for (; probes.size() > 1 && started < probes.size(); ++started) th.emplace_back(one, started);
+    } catch (...) {
+    }
+    for (std::thread& t : th) t.join();
+    for (size_t k = started; k < probes.size(); ++k) one(k);
+}
+
+constexpr int SEARCH_DOUBLING_BATCH = 2;  // doubling steps simulated at once
+constexpr int SEARCH_TREE_DEPTH = 3;      // bisection levels simulated at once (7 probes)
+
+void tree_mids(int32_t lo, int32_t hi, int depth, std::set<int32_t>& mids)
+{
+    if (depth == 0 || hi - lo <= 1) return;
+    const int32_t mid = lo + (hi - lo) / 2;
+    mids.insert(mid);
+    tree_mids(lo, mid, depth - 1, mids);
+    tree_mids(mid, hi, depth - 1, mids);
+}
+
 // Smallest worker count in [1, n_max] of configuration cfg that serves the
-// trace with no failure (doubling then bisection), -1 if n_max fails.
+// trace with no failure, -1 if n_max fails: doubling (1, 2, 4, ..., n_max),
+// then bisection between the last failing and the first passing count. The
+// decisions are those of the plain sequential search; the simulations of the
+// next few decisions run at once (the doubling steps of a batch, the mids of
+// the next levels of the bisection tree) and their outcomes are then read
+// along the path the sequential search takes. Probes off that path change
+// nothing, their errors included.
 int search_min_workers(const aladdin_params& p, const aladdin_worker_cfg& cfg, const DevTrace& tr,
-                       double H, int32_t n_max, cudaStream_t st, int32_t* n_out)
+                       double H, int32_t n_max, int device, int32_t* n_out)
 {
     // JSQ and power of two admit without a test: drain to realize every
     // request's latencies
     const bool drain = p.policy != ALADDIN_POLICY_BESTFIT;
-    double out[9];
-    int rc;
-    int32_t lo = 0, hi = 1;
-    bool found = false;
-    while (hi <= n_max) {
-        if ((rc = simulate_impl(p, cfg, hi, tr, H, true, drain, st, out))) return rc;
-        if (out[0] == 0.0) {
-            found = true;
-            break;
-        }
-        lo = hi;
-        hi = (hi * 2 > n_max && hi < n_max) ? n_max : hi * 2;
+    std::vector<int32_t> seq;
+    for (int32_t hi = 1; hi <= n_max;) {
+        seq.push_back(hi);
+        if (hi == n_max) break;
+        hi = (hi > n_max / 2) ? n_max : hi * 2;
     }
-    if (!found) {
+    int32_t lo = 0, hi = -1;
+    for (size_t k = 0; k < seq.size() && hi < 0;) {
+        const size_t m = std::min(seq.size() - k, (size_t)SEARCH_DOUBLING_BATCH);
+        std::vector<SimProbe> probes(m);
+        for (size_t i = 0; i < m; ++i) probes[i].n = seq[k + i];
+        run_probes(p, cfg, tr, H, drain, device, probes);
+        for (size_t i = 0; i < m; ++i) {
+            if (probes[i].rc) return probes[i].rc;
+            if (probes[i].pass) {
+                hi = probes[i].n;
+                break;
+            }
+            lo = probes[i].n;
+        }
+        k += m;
+    }
+    if (hi < 0) {
         *n_out = -1;
         return ALADDIN_OK;
     }
     while (hi - lo > 1) {
-        const int32_t mid = lo + (hi - lo) / 2;
-        if ((rc = simulate_impl(p, cfg, mid, tr, H, true, drain, st, out))) return rc;
-        if (out[0] == 0.0) hi = mid;
-        else lo = mid;
+        std::set<int32_t> mids;
+        tree_mids(lo, hi, SEARCH_TREE_DEPTH, mids);
+        std::vector<SimProbe> probes;
+        for (int32_t n : mids) {
+            probes.emplace_back();
+            probes.back().n = n;
+        }
+        run_probes(p, cfg, tr, H, drain, device, probes);
+        for (int d = 0; d < SEARCH_TREE_DEPTH && hi - lo > 1; ++d) {
+            const int32_t mid = lo + (hi - lo) / 2;
+            const SimProbe* q = nullptr;
+            for (const SimProbe& x : probes)
+                if (x.n == mid) q = &x;
+            if (!q) return ALADDIN_ERR_ARG;  // unreachable: every mid on the path was probed
+            if (q->rc) return q->rc;
+            if (q->pass) hi = mid;
+            else lo = mid;
+        }
     }
     *n_out = hi;
+    return ALADDIN_OK;
+}
+
+// Runs jobs() for k in [0, n) side by side on host threads (one at a time if
+// no thread can be started); returns the first non-zero status in k order.
+template <typename F>
+int run_parallel(int n, F job)
+{
+    std::vector<int> rc((size_t)n, ALADDIN_OK);
+    std::vector<std::thread> th;
+    int started = 0;
+    try {
+        th.reserve((size_t)n);
+        for (; n > 1 && started < n; ++started) th.emplace_back([&, started] { rc[started] = job(started); });
+    } catch (...) {
+    }
+    for (std::thread& t : th) t.join();
+    for (int k = started; k < n; ++k) rc[k] = job(k);
+    for (int k = 0; k < n; ++k)
+        if (rc[k]) return rc[k];
     return ALADDIN_OK;
 }
 
@@ -1281,11 +1470,16 @@ int aladdin_min_workers(const aladdin_params* params, int32_t n_options,
         if ((rc = check_cfg(options[o]))) return rc;
     cudaStream_t st = (cudaStream_t)cuda_stream;
     DevTrace tr;
-    if ((rc = upload_trace(*params, trace, tr, st))) return rc;
-    for (int o = 0; o < n_options; ++o)
-        if ((rc = search_min_workers(*params, options[o], tr, heartbeat_ms, n_max, st,
-                                     &n_workers[o])))
-            return rc;
+    if ((rc = upload_trace(*params, trace, tr, st))) return rc;  // ends with a sync of st
+    int device = 0;
+    CK(cudaGetDevice(&device));
+    // the options' searches side by side (each on streams of its own)
+    rc = run_parallel(n_options, [&](int o) {
+        return search_min_workers(*params, options[o], tr, heartbeat_ms, n_max, device,
+                                  &n_workers[o]);
+    });
+    trim_sim_pool();
+    if (rc) return rc;
     int best = -1;
     int64_t bestg = 0;
     for (int o = 0; o < n_options; ++o) {
@@ -1375,12 +1569,18 @@ int aladdin_fit_workers(const aladdin_params* params, const aladdin_worker_cfg* 
     *k5 = 0.0;
     *c5 = 0.0;
     cudaStream_t st = (cudaStream_t)cuda_stream;
-    for (int k = 0; k < n_traces; ++k) {
-        DevTrace tr;
-        if ((rc = upload_trace(*params, &traces[k], tr, st))) return rc;
-        if ((rc = search_min_workers(*params, *cfg, tr, heartbeat_ms, n_max, st, &n_workers[k])))
-            return rc;
-    }
+    std::vector<DevTrace> trs((size_t)n_traces);
+    for (int k = 0; k < n_traces; ++k)
+        if ((rc = upload_trace(*params, &traces[k], trs[(size_t)k], st))) return rc;
+    int device = 0;
+    CK(cudaGetDevice(&device));
+    // the rates' searches side by side (each on streams of its own)
+    rc = run_parallel(n_traces, [&](int k) {
+        return search_min_workers(*params, *cfg, trs[(size_t)k], heartbeat_ms, n_max, device,
+                                  &n_workers[k]);
+    });
+    trim_sim_pool();
+    if (rc) return rc;
     // ordinary least squares over the usable points above R
     double m = 0.0, sx = 0.0, sy = 0.0, sxx = 0.0, sxy = 0.0;
     for (int k = 0; k < n_traces; ++k) {

@@ -539,12 +539,40 @@ static size_t r2_smem(int slice, int rc)
 }
 constexpr int R2_MIN_RC = 64;  // fewer rows per worker in shared memory: use the plain round
 
+// Grid of the sliced round for W workers of cap slots: G CTAs, each holding
+// the first rc rows of its slice of workers in shared memory. max_ctas = 1
+// asks for one CTA (then rc shrinks with W). false: no sliced round fits.
+template <int E>
+static bool r2_plan(int W, int cap, int K, int sms, int smem_max, int max_ctas, int* G_out,
+                    int* rc_out)
+{
+    if (K > 65536) return false;  // breakpoints held as 16-bit rho - 1
+    if (sms > ROUND_XBUF_SMS) return false;
+    const size_t budget = (size_t)smem_max - 1024;
+    const size_t base = r2_smem<E>(0, 0);
+    if (budget <= base + 32 + 2 * (R2_MIN_RC + R2_RHO_PAD)) return false;
+    // As few CTAs as hold every worker's rows; beyond the CTAs allowed, the
+    // slices hold only the first rc rows of each worker.
+    int rc = cap;
+    const long long slice_max = (long long)((budget - base) / (32 + 2 * (size_t)(rc + R2_RHO_PAD)));
+    int G = (int)((W + slice_max - 1) / slice_max);
+    const int gmax = max_ctas < sms ? max_ctas : sms;
+    if (G > gmax) {
+        G = gmax;
+        const long long sl = (W + G - 1) / G;
+        rc = ((int)((((budget - base) / (size_t)sl) - 32) / 2) - R2_RHO_PAD) & ~7;
+        if (rc < R2_MIN_RC) return false;
+    }
+    *G_out = G;
+    *rc_out = rc;
+    return true;
+}
+
 template <int E>
 static cudaError_t round2_e(const DevParams& P, const ClusterDev& C, const RoundIO& io,
                             cudaStream_t st, bool* used)
 {
     *used = false;
-    if (P.K > 65536) return cudaSuccess;  // breakpoints held as 16-bit rho - 1
     int dev = 0, sms = 0, smem_max = 0, coop = 0;
     cudaError_t e;
     if ((e = cudaGetDevice(&dev)) != cudaSuccess) return e;
@@ -553,27 +581,16 @@ static cudaError_t round2_e(const DevParams& P, const ClusterDev& C, const Round
             cudaSuccess ||
         (e = cudaDeviceGetAttribute(&coop, cudaDevAttrCooperativeLaunch, dev)) != cudaSuccess)
         return e;
-    if (sms > ROUND_XBUF_SMS) return cudaSuccess;
-    const size_t budget = (size_t)smem_max - 1024;
-    const size_t base = r2_smem<E>(0, 0);
-    if (budget <= base + 32 + 2 * (R2_MIN_RC + R2_RHO_PAD)) return cudaSuccess;
-    // As few CTAs as hold every worker's rows; beyond one CTA per SM, the
-    // slices hold only the first rc rows of each worker.
-    int rc = C.cap;
-    const long long slice_max =
-        (long long)((budget - base) / (32 + 2 * (size_t)(rc + R2_RHO_PAD)));
-    int G = (int)((C.W + slice_max - 1) / slice_max);
-    if (G > sms) {
-        G = sms;
-        const long long sl = (C.W + G - 1) / G;
-        rc = ((int)((((budget - base) / (size_t)sl) - 32) / 2) - R2_RHO_PAD) & ~7;
-        if (rc < R2_MIN_RC) return cudaSuccess;
-    }
-    if (G > 1 && !coop) return cudaSuccess;  // use the single-CTA round
+    int G = 0, rc = 0;
+    // several CTAs need a cooperative launch
+    const int max_ctas = (io.single_cta || !coop) ? 1 : sms;
+    if (!r2_plan<E>(C.W, C.cap, P.K, sms, smem_max, max_ctas, &G, &rc)) return cudaSuccess;
     const int slice = (C.W + G - 1) / G;
     const size_t smem = r2_smem<E>(slice, rc);
-    e = cudaFuncSetAttribute(k_round2<E>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                         (int)smem);
+    // the limit is a property of the kernel shared by every thread of the
+    // process: set it to the device maximum (the same value from every
+    // launch), never to this launch's size
+    e = cudaFuncSetAttribute(k_round2<E>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem_max);
     if (e != cudaSuccess) return e;
     R2Args A;
     A.P = P;
@@ -610,6 +627,33 @@ static cudaError_t round_e(const DevParams& P, const ClusterDev& C, const RoundI
     }
     k_round<E><<<1, ROUND_THREADS, smem, st>>>(P, C, io);
     return cudaGetLastError();
+}
+
+int round_ctas(int W, int cap, int K, bool single_cta)
+{
+    int dev = 0, sms = 0, smem_max = 0, coop = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess ||
+        cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess ||
+        cudaDeviceGetAttribute(&smem_max, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev) !=
+            cudaSuccess ||
+        cudaDeviceGetAttribute(&coop, cudaDevAttrCooperativeLaunch, dev) != cudaSuccess) {
+        cudaGetLastError();
+        return -1;
+    }
+    const int max_ctas = (single_cta || !coop) ? 1 : sms;
+    int G = 0, rc = 0;
+    bool ok = false;
+    switch (lanes_per_worker(cap)) {
+    case 1: ok = r2_plan<1>(W, cap, K, sms, smem_max, max_ctas, &G, &rc); break;
+    case 2: ok = r2_plan<2>(W, cap, K, sms, smem_max, max_ctas, &G, &rc); break;
+    case 4: ok = r2_plan<4>(W, cap, K, sms, smem_max, max_ctas, &G, &rc); break;
+    case 8: ok = r2_plan<8>(W, cap, K, sms, smem_max, max_ctas, &G, &rc); break;
+    case 16: ok = r2_plan<16>(W, cap, K, sms, smem_max, max_ctas, &G, &rc); break;
+    case 32: ok = r2_plan<32>(W, cap, K, sms, smem_max, max_ctas, &G, &rc); break;
+    default: return -1;
+    }
+    if (ok) return G;
+    return lanes_per_worker(cap) <= 16 ? 0 : -1;  // the plain round holds up to 512 slots
 }
 
 cudaError_t launch_round(const DevParams& P, const ClusterDev& C, const RoundIO& io,
