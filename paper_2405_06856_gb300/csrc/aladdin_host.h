@@ -3,6 +3,8 @@
 
 #include <cuda_runtime.h>
 
+#include <atomic>
+
 #include "aladdin_dev.cuh"
 
 namespace aladdin {
@@ -88,6 +90,32 @@ cudaError_t launch_round(const DevParams& P, const ClusterDev& C, const RoundIO&
 // plain single-CTA round, -1 none (a single-CTA request beyond what one CTA
 // holds at 1,024 slots, or a failed device query).
 int round_ctas(int W, int cap, int K, bool single_cta);
+
+// Attributes of the current device that launches size themselves by, read
+// once per device and cached (thread-safe).
+struct DevInfo {
+    int device, sms, smem_optin, coop;
+};
+cudaError_t device_info(DevInfo* out);
+
+// Raises Kern's dynamic shared-memory limit to the device maximum, once per
+// device. The limit is a process-wide property of the kernel; at the maximum,
+// launches of every size are allowed, so threads launching the kernel with
+// different sizes cannot undercut one another, and later launches skip the
+// driver call.
+template <auto Kern>
+cudaError_t allow_max_smem()
+{
+    static std::atomic<unsigned long long> done{0};  // one bit per device ordinal < 64
+    DevInfo d;
+    cudaError_t e = device_info(&d);
+    if (e != cudaSuccess) return e;
+    const unsigned long long bit = d.device < 64 ? 1ull << d.device : 0ull;
+    if (bit && (done.load(std::memory_order_acquire) & bit)) return cudaSuccess;
+    e = cudaFuncSetAttribute(Kern, cudaFuncAttributeMaxDynamicSharedMemorySize, d.smem_optin);
+    if (e == cudaSuccess && bit) done.fetch_or(bit, std::memory_order_acq_rel);
+    return e;
+}
 
 // Execution of every worker for dt ms from t_now.
 // stats: device [0] prefills run, [1] finished, [2] max TTFT bits, [3] max

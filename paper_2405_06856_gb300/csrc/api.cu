@@ -17,6 +17,37 @@
 
 using namespace aladdin;
 
+cudaError_t aladdin::device_info(DevInfo* out)
+{
+    static std::mutex mu;
+    static DevInfo cache[64];
+    static bool have[64] = {};
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return e;
+    if (dev >= 0 && dev < 64) {
+        std::lock_guard<std::mutex> lock(mu);
+        if (have[dev]) {
+            *out = cache[dev];
+            return cudaSuccess;
+        }
+    }
+    DevInfo d;
+    d.device = dev;
+    if ((e = cudaDeviceGetAttribute(&d.sms, cudaDevAttrMultiProcessorCount, dev)) != cudaSuccess ||
+        (e = cudaDeviceGetAttribute(&d.smem_optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev)) !=
+            cudaSuccess ||
+        (e = cudaDeviceGetAttribute(&d.coop, cudaDevAttrCooperativeLaunch, dev)) != cudaSuccess)
+        return e;
+    if (dev >= 0 && dev < 64) {
+        std::lock_guard<std::mutex> lock(mu);
+        cache[dev] = d;
+        have[dev] = true;
+    }
+    *out = d;
+    return cudaSuccess;
+}
+
 namespace {
 
 struct DevBuf {
@@ -1128,6 +1159,8 @@ void trim_sim_pool()
 cudaError_t wait_stream(cudaStream_t st, bool polite)
 {
     if (!polite) return cudaStreamSynchronize(st);
+    // short sleeps: the stream runs dry at the end of the window it waits for,
+    // so a late wake-up idles its SM (backing off to 1 ms measured slower)
     for (;;) {
         const cudaError_t e = cudaStreamQuery(st);
         if (e != cudaErrorNotReady) return e;
@@ -1309,8 +1342,12 @@ void run_probes(const aladdin_params& p, const aladdin_worker_cfg& cfg, const De
     for (size_t k = started; k < probes.size(); ++k) one(k);
 }
 
+#ifndef ALADDIN_SEARCH_TREE_DEPTH
+#define ALADDIN_SEARCH_TREE_DEPTH 3
+#endif
 constexpr int SEARCH_DOUBLING_BATCH = 2;  // doubling steps simulated at once
-constexpr int SEARCH_TREE_DEPTH = 3;      // bisection levels simulated at once (7 probes)
+// bisection levels simulated at once (2^depth - 1 probes)
+constexpr int SEARCH_TREE_DEPTH = ALADDIN_SEARCH_TREE_DEPTH;
 
 void tree_mids(int32_t lo, int32_t hi, int depth, std::set<int32_t>& mids)
 {

@@ -133,8 +133,7 @@ static cudaError_t round_grp_e(const DevParams& P, const ClusterDev& C, const Ro
 {
     const size_t smem = sizeof(GroupSmem<EW, NW>);
     if (smem > 48 * 1024) {
-        cudaError_t e = cudaFuncSetAttribute(k_round_grp<EW, NW>,
-                                             cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+        const cudaError_t e = allow_max_smem<k_round_grp<EW, NW>>();
         if (e != cudaSuccess) return e;
     }
     k_round_grp<EW, NW><<<P.groups, GR_THREADS, smem, st>>>(P, C, io);

@@ -155,15 +155,7 @@ cudaError_t launch_round_queue(const DevParams& P, const ClusterDev& C, const Ro
     const int shared = C.W <= Q_SMEM_MAX_W ? 1 : 0;
     const size_t smem = shared ? sizeof(int) * (size_t)C.W : 0;
     if (smem > 48 * 1024) {
-        // a process-wide property of the kernel: the device maximum, the same
-        // value from every thread, never this launch's size
-        int dev = 0, smem_max = 0;
-        cudaError_t e = cudaGetDevice(&dev);
-        if (e == cudaSuccess)
-            e = cudaDeviceGetAttribute(&smem_max, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev);
-        if (e == cudaSuccess)
-            e = cudaFuncSetAttribute(k_round_queue, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                     smem_max);
+        const cudaError_t e = allow_max_smem<k_round_queue>();
         if (e != cudaSuccess) return e;
     }
     k_round_queue<<<1, Q_THREADS, smem, st>>>(P, C, io, shared);

@@ -247,8 +247,7 @@ static cudaError_t rebalance_e(const DevParams& P, const ClusterDev& C, const Ro
 {
     const size_t smem = sizeof(RebalSmem<EW, NW>);
     if (smem > 48 * 1024) {
-        cudaError_t e = cudaFuncSetAttribute(k_rebalance<EW, NW>,
-                                             cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+        const cudaError_t e = allow_max_smem<k_rebalance<EW, NW>>();
         if (e != cudaSuccess) return e;
     }
     k_rebalance<EW, NW><<<1, RB_THREADS, smem, st>>>(P, C, io, moves, obj);

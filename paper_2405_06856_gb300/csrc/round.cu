@@ -573,25 +573,16 @@ static cudaError_t round2_e(const DevParams& P, const ClusterDev& C, const Round
                             cudaStream_t st, bool* used)
 {
     *used = false;
-    int dev = 0, sms = 0, smem_max = 0, coop = 0;
-    cudaError_t e;
-    if ((e = cudaGetDevice(&dev)) != cudaSuccess) return e;
-    if ((e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev)) != cudaSuccess ||
-        (e = cudaDeviceGetAttribute(&smem_max, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev)) !=
-            cudaSuccess ||
-        (e = cudaDeviceGetAttribute(&coop, cudaDevAttrCooperativeLaunch, dev)) != cudaSuccess)
-        return e;
+    DevInfo d;
+    cudaError_t e = device_info(&d);
+    if (e != cudaSuccess) return e;
     int G = 0, rc = 0;
     // several CTAs need a cooperative launch
-    const int max_ctas = (io.single_cta || !coop) ? 1 : sms;
-    if (!r2_plan<E>(C.W, C.cap, P.K, sms, smem_max, max_ctas, &G, &rc)) return cudaSuccess;
+    const int max_ctas = (io.single_cta || !d.coop) ? 1 : d.sms;
+    if (!r2_plan<E>(C.W, C.cap, P.K, d.sms, d.smem_optin, max_ctas, &G, &rc)) return cudaSuccess;
     const int slice = (C.W + G - 1) / G;
     const size_t smem = r2_smem<E>(slice, rc);
-    // the limit is a property of the kernel shared by every thread of the
-    // process: set it to the device maximum (the same value from every
-    // launch), never to this launch's size
-    e = cudaFuncSetAttribute(k_round2<E>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem_max);
-    if (e != cudaSuccess) return e;
+    if ((e = allow_max_smem<k_round2<E>>()) != cudaSuccess) return e;
     R2Args A;
     A.P = P;
     A.C = C;
@@ -621,8 +612,7 @@ static cudaError_t round_e(const DevParams& P, const ClusterDev& C, const RoundI
 {
     const size_t smem = sizeof(RoundSmem<E>);
     if (smem > 48 * 1024) {
-        cudaError_t e = cudaFuncSetAttribute(k_round<E>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                             (int)smem);
+        const cudaError_t e = allow_max_smem<k_round<E>>();
         if (e != cudaSuccess) return e;
     }
     k_round<E><<<1, ROUND_THREADS, smem, st>>>(P, C, io);
@@ -631,16 +621,13 @@ static cudaError_t round_e(const DevParams& P, const ClusterDev& C, const RoundI
 
 int round_ctas(int W, int cap, int K, bool single_cta)
 {
-    int dev = 0, sms = 0, smem_max = 0, coop = 0;
-    if (cudaGetDevice(&dev) != cudaSuccess ||
-        cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess ||
-        cudaDeviceGetAttribute(&smem_max, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev) !=
-            cudaSuccess ||
-        cudaDeviceGetAttribute(&coop, cudaDevAttrCooperativeLaunch, dev) != cudaSuccess) {
+    DevInfo d;
+    if (device_info(&d) != cudaSuccess) {
         cudaGetLastError();
         return -1;
     }
-    const int max_ctas = (single_cta || !coop) ? 1 : sms;
+    const int sms = d.sms, smem_max = d.smem_optin;
+    const int max_ctas = (single_cta || !d.coop) ? 1 : sms;
     int G = 0, rc = 0;
     bool ok = false;
     switch (lanes_per_worker(cap)) {

@@ -70,12 +70,10 @@ k_build_coop(DevParams P, ClusterDev C, const int32_t* __restrict__ list, int co
     build_table_fit<EW, NW>(P, C, w, C.n[w], reinterpret_cast<unsigned char*>(&sm));
 }
 
-template <typename K>
-static cudaError_t allow_smem(K kern, size_t smem)
+template <auto Kern>
+static cudaError_t allow_smem(size_t smem)
 {
-    if (smem > 48 * 1024)
-        return cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-    return cudaSuccess;
+    return smem > 48 * 1024 ? allow_max_smem<Kern>() : cudaSuccess;
 }
 
 constexpr int COOP_NW = 8;
@@ -90,13 +88,13 @@ static cudaError_t build_e(const DevParams& P, const ClusterDev& C, const int32_
     if constexpr (E > 16) {
         constexpr int EW = E / COOP_NW;
         const size_t sc = sizeof(BuildSmem<EW, COOP_NW>);
-        if ((e = allow_smem(k_build_coop<EW, COOP_NW>, sc)) != cudaSuccess) return e;
+        if ((e = allow_smem<k_build_coop<EW, COOP_NW>>(sc)) != cudaSuccess) return e;
         if (list) {
             k_build_coop<EW, COOP_NW><<<count, COOP_NW * 32, sc, st>>>(P, C, list, count, nullptr);
             return cudaGetLastError();
         }
         const size_t slo = sizeof(BuildSmem<E_LO>) * BUILD_WARPS;
-        if ((e = allow_smem(k_build_lo<E_LO>, slo)) != cudaSuccess) return e;
+        if ((e = allow_smem<k_build_lo<E_LO>>(slo)) != cudaSuccess) return e;
         if ((e = cudaMemsetAsync(C.novf, 0, sizeof(int), st)) != cudaSuccess) return e;
         k_build_lo<E_LO><<<blocks, BUILD_WARPS * 32, slo, st>>>(P, C, count, C.ovf, C.novf);
         k_build_coop<EW, COOP_NW><<<count, COOP_NW * 32, sc, st>>>(P, C, C.ovf, 0, C.novf);
@@ -106,15 +104,15 @@ static cudaError_t build_e(const DevParams& P, const ClusterDev& C, const int32_
             constexpr int EL = E > E_LO ? E_LO : E;
             const size_t slo = sizeof(BuildSmem<EL>) * BUILD_WARPS;
             const size_t shi = sizeof(BuildSmem<E>) * BUILD_WARPS;
-            if ((e = allow_smem(k_build_lo<EL>, slo)) != cudaSuccess) return e;
-            if ((e = allow_smem(k_build_ovf<E>, shi)) != cudaSuccess) return e;
+            if ((e = allow_smem<k_build_lo<EL>>(slo)) != cudaSuccess) return e;
+            if ((e = allow_smem<k_build_ovf<E>>(shi)) != cudaSuccess) return e;
             if ((e = cudaMemsetAsync(C.novf, 0, sizeof(int), st)) != cudaSuccess) return e;
             k_build_lo<EL><<<blocks, BUILD_WARPS * 32, slo, st>>>(P, C, count, C.ovf, C.novf);
             k_build_ovf<E><<<blocks, BUILD_WARPS * 32, shi, st>>>(P, C, C.ovf, C.novf);
             return cudaGetLastError();
         }
         const size_t smem = sizeof(BuildSmem<E>) * BUILD_WARPS;
-        if ((e = allow_smem(k_build<E>, smem)) != cudaSuccess) return e;
+        if ((e = allow_smem<k_build<E>>(smem)) != cudaSuccess) return e;
         k_build<E><<<blocks, BUILD_WARPS * 32, smem, st>>>(P, C, list, count);
         return cudaGetLastError();
     }
