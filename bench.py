@@ -836,6 +836,32 @@ def run_round_only(args):
     print("round mode ok: %d rounds, best %.2f ms" % (len(times), min(times)))
 
 
+def run_sim_only(args):
+    """One fleet simulation of the minimum-worker search's workload, alone:
+    147 one-GPU workers of 1,024 request slots over the first 12,500 requests
+    (about 10 s, 100 heartbeats) of the 1,000,000-request diurnal trace. The
+    command profiled for the simulation's launch list."""
+    import torch
+    from paper_2405_06856_gb300 import build as B
+    B.build()
+    from paper_2405_06856_gb300 import aladdin as A
+    from paper_2405_06856_gb300 import synth
+    torch.cuda.set_device(0)
+    tr, gpus, kv, scale = min_workers_config(synth)
+    k = 12_500
+    trace = A.make_trace(tr.t_arr[:k], tr.req_in[:k], tr.req_pred[:k])
+    cfg = A.make_cfgs(gpus[:1], kv[:1], scale[:1])[0]
+    out = np.zeros(A.SIMULATE_OUT)
+    torch.cuda.synchronize()
+    t0 = time.perf_counter()
+    A.aladdin_simulate(A.make_params(dict(synth.BASE_PARAMS), MW_B_CAP), cfg, 147, trace, 100.0,
+                       1, 0, out)
+    wall = time.perf_counter() - t0
+    print(json.dumps({"mode": "sim", "workers": 147, "requests": k, "failed": int(out[0]),
+                      "placed": int(out[1]), "heartbeats": int(out[2]), "wall_s": wall,
+                      "ms_per_heartbeat": 1000.0 * wall / max(out[2], 1.0)}))
+
+
 def profiled_traffic():
     """DRAM bytes per launch of the scoring kernel from the committed ncu
     summary, or None if the kernel source changed since it was taken."""
@@ -868,7 +894,7 @@ def main():
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--no-cpu-baseline", dest="cpu_baseline", action="store_false")
     ap.add_argument("--mode", default="full",
-                    choices=["full", "kernel", "round", "minworkers", "policies", "configs"],
+                    choices=["full", "kernel", "round", "sim", "minworkers", "policies", "configs"],
                     help="kernel: only warm-up + steps of the device-resident step (for profilers)")
     args = ap.parse_args()
     if args.warmup < 3:
@@ -879,6 +905,8 @@ def main():
         run_kernel_only(args)
     elif args.mode == "round":
         run_round_only(args)
+    elif args.mode == "sim":
+        run_sim_only(args)
     elif args.mode == "minworkers":
         run_min_workers(args)
     elif args.mode == "policies":

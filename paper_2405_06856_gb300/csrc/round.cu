@@ -342,6 +342,7 @@ __global__ void __launch_bounds__(R2_THREADS, 1) k_round2(R2Args A)
     const int n_cand = io.sim ? n_wait0 + (int)(io.arr_end - io.arr_begin) : io.n_cand;
     int keep = 0;        // CTA 0 thread 0: new waiting-list length
     int pend_w = -1;     // this slice's winner of the previous step, not yet appended
+    bool pend_small = false;  // its new count fits the 4-warp rebuild
     int32_t pa = 0, pr = 0, prl = 0;
     double pwd = 0.0;    // its request
 
@@ -360,7 +361,32 @@ __global__ void __launch_bounds__(R2_THREADS, 1) k_round2(R2Args A)
             C.n[w] = nw + 1;
             n_s[lw] = nw + 1;
         }
+    };
+    // Flags a worker of n requests carries with its evaluation through the
+    // reductions and the exchange: 1 no free slot, 2 its count after taking
+    // the candidate fits the 4-warp rebuild.
+    auto flag_bits = [&](int n) { return (n >= cap ? 1 : 0) | (n + 1 <= 128 ? 2 : 0); };
+    // Rebuild group of worker w's table after the append: NW warps, or (small)
+    // 4 warps with one element a lane when its new count fits 128: fewer
+    // cross-warp steps, and the other warps evaluate the next candidate
+    // meanwhile. small comes from the reduced winner flags, so every thread
+    // of the CTA takes the same branch (and the same barrier).
+    auto rebuild = [&](int w, bool small, const CandRec* cand) -> unsigned {
+        const int lw = w - w_lo;
+        SliceCache sc{rho + (long long)lw * rs, rc, &R_s[lw], &wrec_s[lw], &key_s[lw]};
+        append(w);
+        if constexpr (NW > 4) {
+            if (small) {
+                group_sync<4>();
+                return build_table_fit<1, 4, true>(P, C, w, n_s[lw],
+                                                   reinterpret_cast<unsigned char*>(&sm.build),
+                                                   &sc, cand);
+            }
+        }
         group_sync<NW>();
+        return build_table_fit<EW, NW, NW_INSERT>(P, C, w, n_s[lw],
+                                                  reinterpret_cast<unsigned char*>(&sm.build), &sc,
+                                                  cand);
     };
 
     for (int c = 0; c < n_cand; ++c) {
@@ -387,18 +413,15 @@ __global__ void __launch_bounds__(R2_THREADS, 1) k_round2(R2Args A)
         unsigned long long bk = 0ull;
         int bw = NONE, bf = 0;
         const bool rebuilding = pend_w >= 0;
-        if (rebuilding && warp < NW) {
-            append(pend_w);
+        const int nwr = rebuilding && NW > 4 && pend_small ? 4 : NW;  // rebuild warps
+        if (rebuilding && warp < nwr) {
+            const unsigned f = rebuild(pend_w, nwr == 4 && NW > 4, cr.valid ? &cr : nullptr);
             const int lw = pend_w - w_lo;
-            SliceCache sc{rho + (long long)lw * rs, rc, &R_s[lw], &wrec_s[lw], &key_s[lw]};
-            const unsigned f = build_table_fit<EW, NW, NW_INSERT>(P, C, pend_w, n_s[lw],
-                                                       reinterpret_cast<unsigned char*>(&sm.build),
-                                                       &sc, cr.valid ? &cr : nullptr);
             if (tid == 0 && cr.valid && f == 15u && (G <= 1 || pend_w % G == grp))
-                bk = key_s[lw], bw = pend_w, bf = n_s[lw] >= cap;
+                bk = key_s[lw], bw = pend_w, bf = flag_bits(n_s[lw]);
         } else if (cr.valid) {
-            const int first = rebuilding ? tid - 32 * NW : tid;
-            const int stride = rebuilding ? R2_THREADS - 32 * NW : R2_THREADS;
+            const int first = rebuilding ? tid - 32 * nwr : tid;
+            const int stride = rebuilding ? R2_THREADS - 32 * nwr : R2_THREADS;
             for (int lw = first; lw < nloc; lw += stride) {
                 const int w = w_lo + lw;
                 if (w == pend_w || (G > 1 && w % G != grp)) continue;
@@ -410,7 +433,7 @@ __global__ void __launch_bounds__(R2_THREADS, 1) k_round2(R2Args A)
                 const unsigned f =
                     eval_pair_mode(P.approx != 0, t[0], t[1], C.tab2[row], wrec_s[lw],
                                    P.approx ? C.wapx[w] : make_float2(0.0f, 0.0f), cr, m);
-                if (f == 15u) better_f(bk, bw, bf, key_s[lw], w, n_s[lw] >= cap);
+                if (f == 15u) better_f(bk, bw, bf, key_s[lw], w, flag_bits(n_s[lw]));
             }
         }
         reduce_f(bk, bw, bf);
@@ -428,7 +451,7 @@ __global__ void __launch_bounds__(R2_THREADS, 1) k_round2(R2Args A)
         if (A.G > 1) {
             if (warp == 0) {
                 if (lane == 0) {
-                    const int xi = bw == NONE ? NONE : (bw | (bf ? 0x40000000 : 0));
+                    const int xi = bw == NONE ? NONE : (bw | (bf << 29));
                     A.xrec[par * A.G + g] = make_ulonglong2(bk, (unsigned long long)(unsigned)xi);
                     red_release_add(A.arrive, 1u);  // orders the store before it
                 }
@@ -461,26 +484,26 @@ __global__ void __launch_bounds__(R2_THREADS, 1) k_round2(R2Args A)
                 for (int q = lane + 256; q < A.G; q += 32) {
                     const ulonglong2 v = __ldcg(&A.xrec[par * A.G + q]);
                     const int iq = (int)v.y;
-                    better_f(bk, bw, bf, v.x, iq == NONE ? NONE : (iq & 0x3fffffff),
-                             iq != NONE && (iq & 0x40000000));
+                    better_f(bk, bw, bf, v.x, iq == NONE ? NONE : (iq & 0x1fffffff),
+                             iq == NONE ? 0 : (iq >> 29) & 3);
                 }
 #pragma unroll
                 for (int k = 0; k < 8; ++k) {
                     const int iq = (int)xv[k].y;
-                    better_f(bk, bw, bf, xv[k].x, iq == NONE ? NONE : (iq & 0x3fffffff),
-                             iq != NONE && (iq & 0x40000000));
+                    better_f(bk, bw, bf, xv[k].x, iq == NONE ? NONE : (iq & 0x1fffffff),
+                             iq == NONE ? 0 : (iq >> 29) & 3);
                 }
                 reduce_f(bk, bw, bf);
-                if (lane == 0) sm.gwin[par] = bw == NONE ? NONE : (bw | (bf ? 0x40000000 : 0));
+                if (lane == 0) sm.gwin[par] = bw == NONE ? NONE : (bw | (bf << 29));
             }
             __syncthreads();
             if (sm.stop) break;
             const int gw = sm.gwin[par];
-            bw = gw == NONE ? NONE : (gw & 0x3fffffff);
-            bf = gw != NONE && (gw & 0x40000000);
+            bw = gw == NONE ? NONE : (gw & 0x1fffffff);
+            bf = gw == NONE ? 0 : (gw >> 29) & 3;
         }
         const int winner = !cr.valid ? -2 : (bw == NONE ? -1 : bw);
-        if (winner >= 0 && bf) {
+        if (winner >= 0 && (bf & 1)) {
             if (tid == 0 && g == 0) {
                 *io.status = -2;  // ALADDIN_ERR_CAPACITY
                 if (!io.sim)
@@ -490,6 +513,7 @@ __global__ void __launch_bounds__(R2_THREADS, 1) k_round2(R2Args A)
             break;
         }
         pend_w = (winner >= w_lo && winner < w_lo + nloc) ? winner : -1;
+        pend_small = (bf & 2) != 0;  // the reduced winner's flags: the same in every thread
         pa = a;
         pr = r;
         prl = rl;
@@ -512,13 +536,9 @@ __global__ void __launch_bounds__(R2_THREADS, 1) k_round2(R2Args A)
             }
         }
     }
-    if (pend_w >= 0 && warp < NW) {
-        append(pend_w);
-        const int lw = pend_w - w_lo;
-        SliceCache sc{rho + (long long)lw * rs, rc, &R_s[lw], &wrec_s[lw], &key_s[lw]};
-        build_table_fit<EW, NW, NW_INSERT>(P, C, pend_w, n_s[lw],
-                                           reinterpret_cast<unsigned char*>(&sm.build),
-                                &sc, nullptr);
+    if (pend_w >= 0) {
+        const bool small = NW > 4 && pend_small;
+        if (warp < (small ? 4 : NW)) rebuild(pend_w, small, nullptr);
     }
     if (g == 0 && tid == 0 && io.sim && !sm.stop && *io.status == 0) {
         if (io.sim_n) *io.sim_n = n_cand;
