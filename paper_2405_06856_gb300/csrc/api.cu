@@ -608,7 +608,7 @@ int aladdin_cluster_create(const aladdin_params* params, int32_t n_workers,
                            const aladdin_worker_cfg* cfg, const int32_t* req_off,
                            const int32_t* in, const int32_t* gen, const int32_t* pred,
                            const float* tdec_ms, void* cuda_stream, aladdin_cluster** out)
-{
+try {
     if (!out) return ALADDIN_ERR_ARG;
     *out = nullptr;
     int rc = check_params(params);
@@ -632,26 +632,32 @@ int aladdin_cluster_create(const aladdin_params* params, int32_t n_workers,
     }
     *out = cl;
     return ALADDIN_OK;
+} catch (...) {
+    return ALADDIN_ERR_NOMEM;  // a host allocation or thread start failed
 }
 
 int aladdin_cluster_destroy(aladdin_cluster* cl)
-{
+try {
     if (!cl) return ALADDIN_ERR_ARG;
     cudaSetDevice(cl->device);
     cudaStreamSynchronize(cl->st);
     delete cl;
     return ALADDIN_OK;
+} catch (...) {
+    return ALADDIN_ERR_NOMEM;  // a host allocation or thread start failed
 }
 
 int aladdin_cluster_load(aladdin_cluster* cl, const int32_t* req_off, const int32_t* in,
                          const int32_t* gen, const int32_t* pred, const float* tdec_ms)
-{
+try {
     if (!cl) return ALADDIN_ERR_ARG;
     CK(cudaSetDevice(cl->device));
     int rc = load_requests(cl, req_off, in, gen, pred, tdec_ms);
     if (rc) return rc;
     cl->round_open = false;
     return refresh_tables(cl);
+} catch (...) {
+    return ALADDIN_ERR_NOMEM;  // a host allocation or thread start failed
 }
 
 int aladdin_cluster_load_score(aladdin_cluster* cl, const int32_t* req_off, const int32_t* in,
@@ -659,7 +665,7 @@ int aladdin_cluster_load_score(aladdin_cluster* cl, const int32_t* req_off, cons
                                int32_t n_cand, const int32_t* cand_in, const int32_t* cand_pred,
                                const float* wait_ms, uint8_t* flags, float* margin,
                                int32_t* argbest)
-{
+try {
     if (!cl || n_cand < 0) return ALADDIN_ERR_ARG;
     // every array on the device (or mapped): overlap; otherwise the two calls
     auto dv = [](const void* p) {
@@ -729,24 +735,30 @@ int aladdin_cluster_load_score(aladdin_cluster* cl, const int32_t* req_off, cons
         on_host(margin) || on_host(argbest))
         CK(cudaStreamSynchronize(cl->st));
     return ALADDIN_OK;
+} catch (...) {
+    return ALADDIN_ERR_NOMEM;  // a host allocation or thread start failed
 }
 
 int aladdin_score(aladdin_cluster* cl, int32_t n_cand, const int32_t* in, const int32_t* pred,
                   const float* wait_ms, uint8_t* flags, float* margin, int32_t* argbest)
-{
+try {
     return score_impl(cl, n_cand, in, pred, wait_ms, flags, margin, argbest, nullptr, nullptr);
+} catch (...) {
+    return ALADDIN_ERR_NOMEM;  // a host allocation or thread start failed
 }
 
 int aladdin_score_detail(aladdin_cluster* cl, int32_t n_cand, const int32_t* in,
                          const int32_t* pred, const float* wait_ms, uint8_t* flags,
                          float* margin, int32_t* argbest, int64_t* kv_peak, float* t_cand_ms)
-{
+try {
     return score_impl(cl, n_cand, in, pred, wait_ms, flags, margin, argbest, kv_peak, t_cand_ms);
+} catch (...) {
+    return ALADDIN_ERR_NOMEM;  // a host allocation or thread start failed
 }
 
 int aladdin_place_round(aladdin_cluster* cl, int32_t n_cand, const int32_t* in,
                         const int32_t* pred, const float* wait_ms, int32_t* placement)
-{
+try {
     if (!cl || n_cand < 0) return ALADDIN_ERR_ARG;
     if (n_cand == 0) return ALADDIN_OK;
     if (!in || !pred || !placement) return ALADDIN_ERR_ARG;
@@ -797,12 +809,14 @@ int aladdin_place_round(aladdin_cluster* cl, int32_t n_cand, const int32_t* in,
     CK(cudaStreamSynchronize(cl->st));
     if (status == -4) return ALADDIN_ERR_TIMEOUT;
     return status == -2 ? ALADDIN_ERR_CAPACITY : ALADDIN_OK;
+} catch (...) {
+    return ALADDIN_ERR_NOMEM;  // a host allocation or thread start failed
 }
 
 int aladdin_rebalance(aladdin_cluster* cl, int32_t n_cand, const int32_t* in,
                       const int32_t* pred, const float* wait_ms, int32_t* placement,
                       const int64_t* le, const int32_t* be, int32_t* moves, double* obj)
-{
+try {
     if (!cl || n_cand < 0) return ALADDIN_ERR_ARG;
     if (!le || !be) return ALADDIN_ERR_ARG;
     if (n_cand > 0 && (!in || !pred || !placement)) return ALADDIN_ERR_ARG;
@@ -859,10 +873,12 @@ int aladdin_rebalance(aladdin_cluster* cl, int32_t n_cand, const int32_t* in,
         obj[1] = ho[1];
     }
     return ALADDIN_OK;
+} catch (...) {
+    return ALADDIN_ERR_NOMEM;  // a host allocation or thread start failed
 }
 
 int aladdin_cluster_advance(aladdin_cluster* cl, double dt_ms, double* stats)
-{
+try {
     if (!cl || !(std::isfinite(dt_ms) && dt_ms >= 0)) return ALADDIN_ERR_ARG;
     CK(cudaSetDevice(cl->device));
     CK(launch_advance(cl->dp, cl->dev, cl->t_now, dt_ms, cl->d_stats, nullptr, cl->st));
@@ -884,6 +900,8 @@ int aladdin_cluster_advance(aladdin_cluster* cl, double dt_ms, double* stats)
         for (int k = 4; k < STATS_N; ++k) stats[k] = (double)s[k];
     }
     return ALADDIN_OK;
+} catch (...) {
+    return ALADDIN_ERR_NOMEM;  // a host allocation or thread start failed
 }
 
 // Checkpoint layout: a header, then the device arrays in a fixed order.
@@ -913,7 +931,7 @@ static void ckpt_arrays(aladdin_cluster* cl, void** ptr, size_t* len, int* count
 }
 
 int aladdin_cluster_save(aladdin_cluster* cl, void* buf, int64_t* bytes)
-{
+try {
     if (!cl || !bytes) return ALADDIN_ERR_ARG;
     void* ptr[16];
     size_t len[16];
@@ -946,10 +964,12 @@ int aladdin_cluster_save(aladdin_cluster* cl, void* buf, int64_t* bytes)
     CK(cudaStreamSynchronize(cl->st));
     *bytes = (int64_t)total;
     return ALADDIN_OK;
+} catch (...) {
+    return ALADDIN_ERR_NOMEM;  // a host allocation or thread start failed
 }
 
 int aladdin_cluster_restore(aladdin_cluster* cl, const void* buf, int64_t bytes)
-{
+try {
     if (!cl || !buf || bytes < (int64_t)sizeof(CheckpointHeader)) return ALADDIN_ERR_ARG;
     CheckpointHeader h;
     std::memcpy(&h, buf, sizeof(h));
@@ -976,11 +996,13 @@ int aladdin_cluster_restore(aladdin_cluster* cl, const void* buf, int64_t bytes)
     if (rc) return rc;
     CK(cudaStreamSynchronize(cl->st));  // the host buffer may be released on return
     return ALADDIN_OK;
+} catch (...) {
+    return ALADDIN_ERR_NOMEM;  // a host allocation or thread start failed
 }
 
 int aladdin_cluster_state(aladdin_cluster* cl, int32_t* n, int32_t* in, int32_t* gen,
                           int32_t* pred, uint8_t* pending)
-{
+try {
     if (!cl) return ALADDIN_ERR_ARG;
     CK(cudaSetDevice(cl->device));
     const size_t slots = (size_t)cl->W * cl->cap;
@@ -992,11 +1014,13 @@ int aladdin_cluster_state(aladdin_cluster* cl, int32_t* n, int32_t* in, int32_t*
     if (pending) CK(cudaMemcpyAsync(pending, d.pend, slots, cudaMemcpyDeviceToHost, cl->st));
     CK(cudaStreamSynchronize(cl->st));
     return ALADDIN_OK;
+} catch (...) {
+    return ALADDIN_ERR_NOMEM;  // a host allocation or thread start failed
 }
 
 int aladdin_cluster_timing(aladdin_cluster* cl, int32_t enable, double* kernel_ms,
                            int64_t* launches)
-{
+try {
     if (!cl) return ALADDIN_ERR_ARG;
     CK(cudaSetDevice(cl->device));
     CK(cudaStreamSynchronize(cl->st));
@@ -1011,10 +1035,12 @@ int aladdin_cluster_timing(aladdin_cluster* cl, int32_t enable, double* kernel_m
     cl->clear_events();
     cl->timing = enable != 0;
     return ALADDIN_OK;
+} catch (...) {
+    return ALADDIN_ERR_NOMEM;  // a host allocation or thread start failed
 }
 
 int aladdin_cluster_status(aladdin_cluster* cl)
-{
+try {
     if (!cl) return ALADDIN_ERR_ARG;
     CK(cudaSetDevice(cl->device));
     unsigned int err = 0;
@@ -1022,6 +1048,8 @@ int aladdin_cluster_status(aladdin_cluster* cl)
     CK(cudaStreamSynchronize(cl->st));
     if (err & 4u) return ALADDIN_ERR_TIMEOUT;
     return err ? ALADDIN_ERR_STATE : ALADDIN_OK;
+} catch (...) {
+    return ALADDIN_ERR_NOMEM;  // a host allocation or thread start failed
 }
 
 }  // extern "C"
@@ -1481,7 +1509,7 @@ extern "C" {
 int aladdin_simulate(const aladdin_params* params, const aladdin_worker_cfg* cfg, int32_t n,
                      const aladdin_trace* trace, double heartbeat_ms, int32_t stop_at_fail,
                      int32_t drain, void* cuda_stream, double* out)
-{
+try {
     int rc = check_params(params);
     if (rc) return rc;
     if (!cfg || n < 1 || !out || !(std::isfinite(heartbeat_ms) && heartbeat_ms > 0))
@@ -1491,13 +1519,15 @@ int aladdin_simulate(const aladdin_params* params, const aladdin_worker_cfg* cfg
     DevTrace tr;
     if ((rc = upload_trace(*params, trace, tr, st))) return rc;
     return simulate_impl(*params, *cfg, n, tr, heartbeat_ms, stop_at_fail != 0, drain != 0, st, out);
+} catch (...) {
+    return ALADDIN_ERR_NOMEM;  // a host allocation or thread start failed
 }
 
 int aladdin_min_workers(const aladdin_params* params, int32_t n_options,
                         const aladdin_worker_cfg* options, const aladdin_trace* trace,
                         double heartbeat_ms, int32_t n_max, void* cuda_stream,
                         int32_t* n_workers, int32_t* best_option, int64_t* total_gpus)
-{
+try {
     int rc = check_params(params);
     if (rc) return rc;
     if (n_options < 1 || !options || !n_workers || n_max < 1 ||
@@ -1530,11 +1560,13 @@ int aladdin_min_workers(const aladdin_params* params, int32_t n_options,
     if (best_option) *best_option = best;
     if (total_gpus) *total_gpus = best < 0 ? -1 : bestg;
     return ALADDIN_OK;
+} catch (...) {
+    return ALADDIN_ERR_NOMEM;  // a host allocation or thread start failed
 }
 
 int aladdin_tp_configs(const aladdin_tp_model* tp, int32_t n, const int32_t* gpus,
                        aladdin_worker_cfg* out)
-{
+try {
     if (!tp || n < 1 || !gpus || !out) return ALADDIN_ERR_ARG;
     if (!(finite_nonneg(tp->k4) && finite_nonneg(tp->c4) && finite_nonneg(tp->kc) &&
           finite_nonneg(tp->m_gpu) && finite_nonneg(tp->m_model) && tp->k4 + tp->c4 > 0.0))
@@ -1549,23 +1581,27 @@ int aladdin_tp_configs(const aladdin_tp_model* tp, int32_t n, const int32_t* gpu
         out[o].lat_scale = (tp->k4 / ng + tp->c4 + tp->kc * (ng - 1.0) / ng) / (tp->k4 + tp->c4);
     }
     return ALADDIN_OK;
+} catch (...) {
+    return ALADDIN_ERR_NOMEM;  // a host allocation or thread start failed
 }
 
 int aladdin_trace_demand(const aladdin_params* params, const aladdin_trace* trace,
                          void* cuda_stream, double* m_r, double* l_ave)
-{
+try {
     int rc = check_params(params);
     if (rc) return rc;
     cudaStream_t st = (cudaStream_t)cuda_stream;
     DevTrace tr;
     if ((rc = upload_trace(*params, trace, tr, st))) return rc;
     return trace_demand_impl(*params, tr, st, m_r, l_ave);
+} catch (...) {
+    return ALADDIN_ERR_NOMEM;  // a host allocation or thread start failed
 }
 
 int aladdin_pick_config(const aladdin_params* params, int32_t n_options,
                         const aladdin_worker_cfg* options, const aladdin_trace* trace,
                         void* cuda_stream, double* t_max, int32_t* best_option)
-{
+try {
     int rc = check_params(params);
     if (rc) return rc;
     if (n_options < 1 || !options || !best_option) return ALADDIN_ERR_ARG;
@@ -1588,13 +1624,15 @@ int aladdin_pick_config(const aladdin_params* params, int32_t n_options,
     }
     *best_option = best;
     return ALADDIN_OK;
+} catch (...) {
+    return ALADDIN_ERR_NOMEM;  // a host allocation or thread start failed
 }
 
 int aladdin_fit_workers(const aladdin_params* params, const aladdin_worker_cfg* cfg,
                         int32_t n_traces, const aladdin_trace* traces, const double* rates,
                         double R, double heartbeat_ms, int32_t n_max, void* cuda_stream,
                         int32_t* n_workers, double* k5, double* c5)
-{
+try {
     int rc = check_params(params);
     if (rc) return rc;
     if (!cfg || n_traces < 1 || !traces || !rates || !n_workers || !k5 || !c5 || n_max < 1 ||
@@ -1634,15 +1672,19 @@ int aladdin_fit_workers(const aladdin_params* params, const aladdin_worker_cfg* 
     *k5 = (m * sxy - sx * sy) / den;
     *c5 = (sy - *k5 * sx) / m;
     return ALADDIN_OK;
+} catch (...) {
+    return ALADDIN_ERR_NOMEM;  // a host allocation or thread start failed
 }
 
 int aladdin_predict_workers(double k5, double c5, double rate, int64_t* n_workers)
-{
+try {
     if (!n_workers) return ALADDIN_ERR_ARG;
     const double v = std::ceil(k5 * rate + c5);
     if (!(std::isfinite(v) && v >= -9.2e18 && v <= 9.2e18)) return ALADDIN_ERR_ARG;
     *n_workers = (int64_t)v;
     return ALADDIN_OK;
+} catch (...) {
+    return ALADDIN_ERR_NOMEM;  // a host allocation or thread start failed
 }
 
 }  // extern "C"

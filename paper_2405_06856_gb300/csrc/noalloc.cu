@@ -70,7 +70,7 @@ bool on_device(const void* p)
 extern "C" int aladdin_score_noalloc(aladdin_cluster* cl, int32_t n_cand, const int32_t* in,
                                      const int32_t* pred, const float* wait_ms, uint8_t* flags,
                                      float* margin, int32_t* argbest)
-{
+try {
     aladdin::ClusterView v;
     if (!cl || n_cand < 0) return ALADDIN_ERR_ARG;
     int rc = aladdin::cluster_view(cl, &v);
@@ -99,4 +99,6 @@ extern "C" int aladdin_score_noalloc(aladdin_cluster* cl, int32_t n_cand, const 
         return ALADDIN_ERR_CUDA;
     }
     return ALADDIN_OK;
+} catch (...) {
+    return ALADDIN_ERR_NOMEM;  // a host allocation or thread start failed
 }
