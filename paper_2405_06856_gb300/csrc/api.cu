@@ -1397,6 +1397,11 @@ void tree_mids(int32_t lo, int32_t hi, int depth, std::set<int32_t>& mids)
 int search_min_workers(const aladdin_params& p, const aladdin_worker_cfg& cfg, const DevTrace& tr,
                        double H, int32_t n_max, int device, int32_t* n_out)
 {
+    // the caller's device (this may be a fresh host thread of run_parallel)
+    if (cudaSetDevice(device) != cudaSuccess) {
+        cudaGetLastError();
+        return ALADDIN_ERR_CUDA;
+    }
     // JSQ and power of two admit without a test: drain to realize every
     // request's latencies
     const bool drain = p.policy != ALADDIN_POLICY_BESTFIT;
