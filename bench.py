@@ -101,25 +101,37 @@ class ClockSampler:
         except Exception:
             self.proc.kill()
         self.f.close()
-        sm, mx, reasons = [], 0.0, set()
-        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
-        for line in open(self.path):
-            parts = [x.strip() for x in line.split(",")]
-            if len(parts) < 9:
-                continue
-            try:
-                sm.append(float(parts[1]))
-                mx = max(mx, float(parts[2]))
-            except ValueError:
-                continue
-            for k, v in zip(names, parts[5:9]):
-                if v.lower() == "active":
-                    reasons.add(k)
+        with open(self.path) as f:
+            lines = f.readlines()
         os.unlink(self.path)
-        if not sm:
-            return None
-        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": mx, "reasons": sorted(reasons),
-                "samples": len(sm)}
+        return clock_summary(lines)
+
+
+CLOCK_REASONS = ("hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap")
+
+
+def clock_summary(lines):
+    """Median SM clock, largest max clock and the throttle reasons seen in
+    nvidia-smi CSV lines (index, clocks.sm, clocks.max.sm, power.draw,
+    reasons.active, then the four reasons of CLOCK_REASONS as Active /
+    Not Active); None without a sample."""
+    sm, mx, reasons = [], 0.0, set()
+    for line in lines:
+        parts = [x.strip() for x in line.split(",")]
+        if len(parts) < 9:
+            continue
+        try:
+            sm.append(float(parts[1]))
+            mx = max(mx, float(parts[2]))
+        except ValueError:
+            continue
+        for k, v in zip(CLOCK_REASONS, parts[5:9]):
+            if v.lower() == "active":
+                reasons.add(k)
+    if not sm:
+        return None
+    return {"sm_mhz": statistics.median(sm), "sm_max_mhz": mx, "reasons": sorted(reasons),
+            "samples": len(sm)}
 
 
 def dist_setup(args):
