@@ -460,6 +460,26 @@ int aladdin_fit_workers(const aladdin_params* params, const aladdin_worker_cfg* 
  * the value is not finite or outside the int64 range. */
 int aladdin_predict_workers(double k5, double c5, double rate, int64_t* n_workers);
 
+/* Number of scheduling groups of distributed scheduling (Appendix A,
+ * Eq. group_arrival_limit). Requests arriving at rate_a (requests per second)
+ * are dealt round-robin to G groups (params.groups), so group i gets the rate
+ * r_i = rate_a / G and n_workers / G workers (n_workers e.g. from
+ * aladdin_predict_workers). G must satisfy
+ *   r_i <= rate_max      rate_max = r(T_s), the arrival rate one scheduler
+ *                        places within the scheduling latency limit T_s
+ *                        (measured by the caller);
+ *   n_workers / G >= 1 / (2 e)   if about half of the groups need one extra
+ *                        worker, the extra workers stay within a fraction e
+ *                        of the central scheduler's (the printed bound stands
+ *                        on r_i; it is read as the workers per group that the
+ *                        text derives, e = 10% giving five workers a group).
+ * *groups receives the fewest such G (the least extra workers): the smallest
+ * G >= 1 with G rate_max >= rate_a, if G <= 2 e n_workers and G <= n_workers.
+ * ALADDIN_ERR_ARG if no G meets both, or for rate_a < 0, rate_max <= 0,
+ * e <= 0 (or any of them not finite), n_workers < 1 or a null groups. */
+int aladdin_pick_groups(double rate_a, double rate_max, double e, int64_t n_workers,
+                        int64_t* groups);
+
 #ifdef __cplusplus
 }
 #endif

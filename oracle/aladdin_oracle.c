@@ -1222,3 +1222,23 @@ int64_t orc_predict_workers(double k5, double c5, double rate)
 {
     return (int64_t)ceil(k5 * rate + c5);
 }
+
+/* Appendix A, Eq. group_arrival_limit: the number G of scheduling groups of
+ * distributed scheduling. Round-robin dealing gives group i the rate
+ * r_i = rate_a / G and n_workers / G workers. Its scheduler must place
+ * r_i within the latency limit T_s (r_i <= r(T_s) = rate_max), and the
+ * group must keep at least 1 / (2e) workers, so that about half of the groups
+ * needing one extra worker costs at most a fraction e of extra workers (the
+ * printed lower bound stands on r_i; it is read as the workers per group the
+ * text derives). Both conditions multiplied out: rate_a <= G rate_max and
+ * 2 e n_workers >= G. The fewest such groups (the least extra workers), by
+ * enumeration over G = 1 .. n_workers; 0 if none. */
+int64_t orc_pick_groups(double rate_a, double rate_max, double e, int64_t n_workers)
+{
+    for (int64_t G = 1; G <= n_workers; ++G) {
+        const int fast_enough = rate_a <= (double)G * rate_max;
+        const int enough_workers = 2.0 * e * (double)n_workers >= (double)G;
+        if (fast_enough && enough_workers) return G;
+    }
+    return 0;
+}

@@ -87,6 +87,8 @@ def lib():
         _lib.orc_fit_workers.restype = C.c_int32
         _lib.orc_predict_workers.argtypes = [D, D, D]
         _lib.orc_predict_workers.restype = C.c_int64
+        _lib.orc_pick_groups.argtypes = [D, D, D, C.c_int64]
+        _lib.orc_pick_groups.restype = C.c_int64
         _lib.orc_capacity_norm.argtypes = [P, P, C.c_int]
         _lib.orc_capacity_norm.restype = C.c_double
         _lib.orc_order.argtypes = [P, P, P]
@@ -414,3 +416,10 @@ def fit_workers(rates, nw, R=0.0):
 
 def predict_workers(k5, c5, rate):
     return int(lib().orc_predict_workers(float(k5), float(c5), float(rate)))
+
+
+def pick_groups(rate_a, rate_max, e, n_workers):
+    """Appendix A, Eq. group_arrival_limit: the fewest scheduling groups whose
+    per-group arrival rate stays within rate_max and that keep at least
+    1 / (2e) workers each; 0 if none."""
+    return int(lib().orc_pick_groups(float(rate_a), float(rate_max), float(e), int(n_workers)))

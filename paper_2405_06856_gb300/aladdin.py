@@ -90,6 +90,7 @@ _sig = {
     "aladdin_fit_workers": [_P, _P, C.c_int32, _P, _P, C.c_double, C.c_double, C.c_int32, _P, _P,
                             _P, _P],
     "aladdin_predict_workers": [C.c_double, C.c_double, C.c_double, _P],
+    "aladdin_pick_groups": [C.c_double, C.c_double, C.c_double, C.c_int64, _P],
     "aladdin_rebalance": [_P, C.c_int32, _P, _P, _P, _P, _P, _P, _P, _P],
     "aladdin_cluster_save": [_P, _P, _P],
     "aladdin_cluster_load_score": [_P, _P, _P, _P, _P, _P, C.c_int32, _P, _P, _P, _P, _P, _P],
@@ -343,6 +344,13 @@ def aladdin_predict_workers(k5, c5, rate):
     _check(_lib.aladdin_predict_workers(float(k5), float(c5), float(rate), C.byref(n)),
            "aladdin_predict_workers")
     return n.value
+
+
+def aladdin_pick_groups(rate_a, rate_max, e, n_workers):
+    g = C.c_int64()
+    _check(_lib.aladdin_pick_groups(float(rate_a), float(rate_max), float(e), int(n_workers),
+                                    C.byref(g)), "aladdin_pick_groups")
+    return g.value
 
 
 # ---------------------------------------------------------------------------

@@ -1692,4 +1692,27 @@ try {
     return ALADDIN_ERR_NOMEM;  // a host allocation or thread start failed
 }
 
+int aladdin_pick_groups(double rate_a, double rate_max, double e, int64_t n_workers,
+                        int64_t* groups)
+try {
+    if (!groups || !(std::isfinite(rate_a) && rate_a >= 0.0) || !finite_pos(rate_max) ||
+        !finite_pos(e) || n_workers < 1)
+        return ALADDIN_ERR_ARG;
+    const double n = (double)n_workers;
+    // the most groups that keep 1 / (2e) workers each: G <= 2 e n_workers
+    const double g_workers = std::floor(2.0 * e * n);
+    // the fewest groups within one scheduler's rate: G rate_max >= rate_a
+    double g = std::ceil(rate_a / rate_max);
+    if (g < 1.0) g = 1.0;
+    if (!(g <= n + 1.0)) return ALADDIN_ERR_ARG;  // beyond one worker a group
+    // the division's rounding: settle on the products themselves
+    for (int k = 0; k < 4 && g > 1.0 && (g - 1.0) * rate_max >= rate_a; ++k) g -= 1.0;
+    for (int k = 0; k < 4 && g * rate_max < rate_a; ++k) g += 1.0;
+    if (g * rate_max < rate_a || g > g_workers || g > n) return ALADDIN_ERR_ARG;
+    *groups = (int64_t)g;
+    return ALADDIN_OK;
+} catch (...) {
+    return ALADDIN_ERR_NOMEM;  // a host allocation or thread start failed
+}
+
 }  // extern "C"

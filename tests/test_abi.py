@@ -120,3 +120,26 @@ def test_predict_workers_matches_oracle(lib, orc):
         assert lib.aladdin_predict_workers(k5, c5, r) == orc.predict_workers(k5, c5, r)
     with pytest.raises(lib.AladdinError):
         lib.aladdin_predict_workers(float("inf"), 0.0, 1.0)
+
+
+def test_pick_groups_matches_oracle(lib, orc):
+    """Appendix A's group count: the library's closed form against the
+    oracle's enumeration (0 there = no group count meets both conditions)."""
+    rng = np.random.default_rng(91)
+    cases = [(0.0, 1.0, 0.1, 5), (2500.0, 250.0, 0.1, 50), (2500.0, 250.0, 0.1, 49),
+             (2375.0, 250.0, 0.1, 50), (100.0, 1000.0, 0.05, 10), (2000.0, 100.0, 0.5, 20),
+             (2000.0, 100.0, 0.5, 15), (1e300, 1.0, 0.5, 10)]
+    for _ in range(300):
+        cases.append((float(rng.uniform(0.0, 30.0) * 400.0), float(rng.uniform(100.0, 900.0)),
+                      float(rng.uniform(0.02, 0.6)), int(rng.integers(1, 300))))
+    for ra, rmax, e, n in cases:
+        want = orc.pick_groups(ra, rmax, e, n)
+        if want == 0:
+            with pytest.raises(lib.AladdinError):
+                lib.aladdin_pick_groups(ra, rmax, e, n)
+        else:
+            assert lib.aladdin_pick_groups(ra, rmax, e, n) == want, (ra, rmax, e, n)
+    for bad in ((-1.0, 1.0, 0.1, 5), (1.0, 0.0, 0.1, 5), (1.0, 1.0, 0.0, 5),
+                (1.0, 1.0, 0.1, 0), (float("nan"), 1.0, 0.1, 5), (1.0, float("inf"), 0.1, 5)):
+        with pytest.raises(lib.AladdinError):
+            lib.aladdin_pick_groups(*bad)

@@ -98,3 +98,66 @@ def test_full_worker_stops_only_its_group(orc, synth):
     assert full
     assert list(pl) == [0, 1, -1, 1, -1, 1, -1, 1]
     assert list(cl.n) == [4, 4]
+
+
+# --- the number of groups (Appendix A, Eq. group_arrival_limit) -------------
+
+def _gold_groups():
+    import json
+    import os
+    with open(os.path.join(os.path.dirname(__file__), "golden", "group_count_example.json")) as f:
+        return json.load(f)
+
+
+def test_group_count_paper_example(orc):
+    """e = 10%: every group must keep at least five workers, so 50 workers
+    allow at most 10 groups and 49 at most 9."""
+    g = _gold_groups()
+    e, per = g["e"], g["min_workers_per_group"]
+    assert orc.pick_groups(0.0, 1.0, e, 1) == 0              # one worker cannot hold 5
+    assert orc.pick_groups(0.0, 1.0, e, per) == 1
+    # rate 10x one scheduler's limit needs 10 groups: 10 * 5 workers suffice,
+    # 10 * 5 - 1 do not
+    assert orc.pick_groups(10.0 * 250.0, 250.0, e, 10 * per) == 10
+    assert orc.pick_groups(10.0 * 250.0, 250.0, e, 10 * per - 1) == 0
+    # a rate just above 9 schedulers' limit also needs 10
+    assert orc.pick_groups(9.5 * 250.0, 250.0, e, 10 * per) == 10
+    assert orc.pick_groups(9.0 * 250.0, 250.0, e, 10 * per - 1) == 9
+
+
+def test_group_count_is_the_fewest_feasible(orc):
+    """Brute force in exact rational arithmetic: the fewest G with
+    rate_a / G <= rate_max and n / G >= 1 / (2e)."""
+    from fractions import Fraction as F
+    rng = np.random.default_rng(57)
+    checked = 0
+    for _ in range(400):
+        n = int(rng.integers(1, 400))
+        e = float(rng.uniform(0.01, 0.6))
+        rmax = float(rng.uniform(50.0, 5000.0))
+        ra = float(rng.uniform(0.0, 40.0) * rmax)
+        want = 0
+        for G in range(1, n + 1):
+            if F(ra) <= G * F(rmax) and F(n) * 2 * F(e) >= G:
+                want = G
+                break
+        # skip draws within rounding of a boundary of either condition
+        near = any(abs(F(ra) - G * F(rmax)) <= F(ra) * F(1, 10**9) or
+                   abs(F(n) * 2 * F(e) - G) <= F(1, 10**9) for G in range(1, n + 1))
+        if near:
+            continue
+        assert orc.pick_groups(ra, rmax, e, n) == want, (ra, rmax, e, n)
+        checked += 1
+    assert checked > 350
+
+
+def test_group_count_special_cases(orc):
+    # one scheduler keeps up: one group (the central scheduler)
+    assert orc.pick_groups(100.0, 1000.0, 0.05, 10) == 1
+    # the rate needs more groups than the workers allow
+    assert orc.pick_groups(2000.0, 100.0, 0.5, 15) == 0
+    # e = 1/2 lets every worker be its own group (one worker a group)
+    assert orc.pick_groups(2000.0, 100.0, 0.5, 20) == 20
+    # more tolerance allows more, smaller groups; never more groups than needed
+    for e in (0.05, 0.1, 0.2, 0.5):
+        assert orc.pick_groups(1000.0, 300.0, e, 400) == 4
