@@ -181,20 +181,31 @@ def test_load_device_state(A, orc, synth):
 
 
 def test_w4096_sampled(A, orc, synth):
-    """The 4,096-worker workload at full size: sampled pairs and sampled
-    argbest rows against the oracle."""
+    """The 4,096-worker workload at full size, scored by the call bench.py
+    times (aladdin_cluster_load_score from device arrays): sampled pairs and
+    sampled argbest rows against the oracle, and every byte equal to
+    aladdin_score on the loaded state."""
     import torch
     wl = synth.config("w4096")
     C, W = wl.n_cand, wl.n_workers
     dev = torch.device("cuda")
+    d = lambda x: torch.from_numpy(np.ascontiguousarray(x)).to(dev)
     with A.Cluster.from_workload(wl) as cl:
         f = torch.zeros((C, W), dtype=torch.uint8, device=dev)
         m = torch.zeros((C, W), dtype=torch.float32, device=dev)
         a = torch.zeros(C, dtype=torch.int32, device=dev)
-        A.aladdin_score(cl.handle, C, torch.from_numpy(wl.cand_in).to(dev),
-                        torch.from_numpy(wl.cand_pred).to(dev), torch.from_numpy(wl.cand_wait).to(dev),
-                        f, m, a)
+        cin, cpr, cw = d(wl.cand_in), d(wl.cand_pred), d(wl.cand_wait)
+        A.aladdin_cluster_load_score(cl.handle, d(wl.roff), d(wl.req_in), d(wl.req_gen),
+                                     d(wl.req_pred), None, C, cin, cpr, cw, f, m, a)
+        f2 = torch.zeros_like(f)
+        m2 = torch.zeros_like(m)
+        a2 = torch.zeros_like(a)
+        A.aladdin_score(cl.handle, C, cin, cpr, cw, f2, m2, a2)
         torch.cuda.synchronize()
+        assert cl.status() == A.OK
+        assert torch.equal(f, f2) and torch.equal(m.view(torch.int32), m2.view(torch.int32))
+        assert torch.equal(a, a2)
+        del f2, m2, a2
         rng = np.random.default_rng(9)
         pc = rng.integers(0, C, 3000).astype(np.int32)
         pw = rng.integers(0, W, 3000).astype(np.int32)
