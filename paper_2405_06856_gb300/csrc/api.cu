@@ -933,8 +933,8 @@ static void ckpt_arrays(aladdin_cluster* cl, void** ptr, size_t* len, int* count
 int aladdin_cluster_save(aladdin_cluster* cl, void* buf, int64_t* bytes)
 try {
     if (!cl || !bytes) return ALADDIN_ERR_ARG;
-    void* ptr[16];
-    size_t len[16];
+    void* ptr[16] = {};
+    size_t len[16] = {};
     int k = 0;
     ckpt_arrays(cl, ptr, len, &k);
     size_t total = sizeof(CheckpointHeader);
@@ -974,8 +974,8 @@ try {
     CheckpointHeader h;
     std::memcpy(&h, buf, sizeof(h));
     if (h.magic != CKPT_MAGIC || h.W != cl->W || h.cap != cl->cap) return ALADDIN_ERR_ARG;
-    void* ptr[16];
-    size_t len[16];
+    void* ptr[16] = {};
+    size_t len[16] = {};
     int k = 0;
     ckpt_arrays(cl, ptr, len, &k);
     size_t total = sizeof(h);
