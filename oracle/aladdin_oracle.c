@@ -9,7 +9,11 @@
  * code, header, table or constant with the CUDA library, and the product
  * path never reaches it.
  *
- * Models (Sec. 3), with the readings of the paper listed in the design doc:
+ * Models (Sec. 3). Where the paper is garbled or silent these readings are
+ * taken: Eq. kv cache's r is l_out, the tokens generated so far; Eq. iter
+ * time holds for every batch size b >= 1; ATGT is enforced over the
+ * remaining iterations plus the banked slack of Table 1's t^dec; the stall
+ * of a round's prefill hits only the requests decoding at round start.
  *   KV usage      Eq. kv cache: a request with c context tokens holds h*c + j
  *                 KV slots. In its s-th remaining decode iteration a request
  *                 with l_in input and l_out generated tokens holds

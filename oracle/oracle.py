@@ -14,6 +14,12 @@ import numpy as np
 HERE = os.path.dirname(os.path.abspath(__file__))
 SRC = os.path.join(HERE, "aladdin_oracle.c")
 LIB = os.path.join(HERE, "_build", "liboracle.so")
+# The oracle's own tests build deliberately broken copies of the source (one
+# planted mistake each) and check that a pin fails: ALADDIN_ORACLE_SRC names
+# such a copy, built beside it.
+if os.environ.get("ALADDIN_ORACLE_SRC"):
+    SRC = os.path.abspath(os.environ["ALADDIN_ORACLE_SRC"])
+    LIB = os.path.splitext(SRC)[0] + ".so"
 
 FLAG_KV, FLAG_TTFT, FLAG_ONGOING, FLAG_NEW = 1, 2, 4, 8
 FEASIBLE = 15

@@ -1,8 +1,11 @@
 """Comparison of CUDA outputs with the oracle, shared by the GPU tests.
 
-Tolerances (derivation in the design doc): the kernels compute every latency bound
-in fp32 from exact integer aggregates, a handful of roundings each, so a bound
-of magnitude B carries an error of order 1e-6 B; 1e-5 relative is the bar.
+Tolerances: the kernels compute every latency bound in fp32 from exact
+integer aggregates (int64 prefix sums of lengths and of r (r + 1) / 2 terms),
+with a handful of fp32 roundings per bound (about 5, each at most 2^-24
+relative of the term it rounds), so a bound of magnitude B carries an error
+of order 1e-6 B; 1e-5 relative of the bound's scale is the bar, a 10x margin.
+KV bounds are integers below 2^24 and exact in fp32.
 Feasibility flags are compared exactly except on pairs whose smallest latency
 slack is within 1e-5 of its scale in the oracle's fp64 arithmetic ("near"
 pairs), where fp32 may take the other side; those are counted and reported.
