@@ -176,31 +176,46 @@ def barrier(dist):
 # ---------------------------------------------------------------------------
 # CPU oracle baseline (bounded sample; spawn pool across host cores).
 
+_SLICE_CACHE = {}
+
+
 def _oracle_slice(args):
+    """Every pair of workers `wid` with the first `ncand` candidates, scored by
+    the oracle in this (spawned) process; the workload and the sub-cluster are
+    built once per process, outside the timed scoring."""
     wid, ncand = args
     from oracle import oracle as O
     from paper_2405_06856_gb300 import synth
-    wl = synth.config(WORKLOAD)
-    sub = O.Cluster(wl.params, wl.kv_capacity[wid], wl.lat_scale[wid], wl.b_cap,
-                    np.concatenate([[0], np.cumsum(np.diff(wl.roff)[wid])]).astype(np.int32),
-                    np.concatenate([wl.req_in[wl.roff[w]:wl.roff[w + 1]] for w in wid]),
-                    np.concatenate([wl.req_gen[wl.roff[w]:wl.roff[w + 1]] for w in wid]),
-                    np.concatenate([wl.req_pred[wl.roff[w]:wl.roff[w + 1]] for w in wid]))
+    key = (tuple(wid), ncand)
+    if key not in _SLICE_CACHE:
+        wl = synth.config(WORKLOAD)
+        sub = O.Cluster(wl.params, wl.kv_capacity[wid], wl.lat_scale[wid], wl.b_cap,
+                        np.concatenate([[0], np.cumsum(np.diff(wl.roff)[wid])]).astype(np.int32),
+                        np.concatenate([wl.req_in[wl.roff[w]:wl.roff[w + 1]] for w in wid]),
+                        np.concatenate([wl.req_gen[wl.roff[w]:wl.roff[w + 1]] for w in wid]),
+                        np.concatenate([wl.req_pred[wl.roff[w]:wl.roff[w + 1]] for w in wid]))
+        _SLICE_CACHE[key] = (sub, wl.cand_in[:ncand].copy(), wl.cand_pred[:ncand].copy(),
+                             wl.cand_wait[:ncand].copy())
+    sub, cin, cpr, cw = _SLICE_CACHE[key]
     t0 = time.perf_counter()
-    sub.score(wl.cand_in[:ncand], wl.cand_pred[:ncand], wl.cand_wait[:ncand],
-              want=("flags", "margin"))
+    sub.score(cin, cpr, cw, want=("flags", "margin"))
     return len(wid) * ncand, time.perf_counter() - t0
+
+
+def oracle_jobs(workers_per_core, ncand, cores):
+    return [(list(range(i * workers_per_core, (i + 1) * workers_per_core)), ncand)
+            for i in range(cores)]
 
 
 def oracle_baseline(workers_per_core=4, ncand=32768, cores=None):
     """Oracle evaluations/sec: each process scores all pairs of its own workers
-    against the first `ncand` candidates; throughput = pairs / wall time."""
+    against the first `ncand` candidates; throughput = pairs / wall time of
+    the parallel scoring (the slowest process)."""
     import multiprocessing as mp
     from oracle import oracle as O
     O.build()
     cores = cores or os.cpu_count() or 1
-    jobs = [(list(range(i * workers_per_core, (i + 1) * workers_per_core)), ncand)
-            for i in range(cores)]
+    jobs = oracle_jobs(workers_per_core, ncand, cores)
     ctx = mp.get_context("spawn")
     t0 = time.perf_counter()
     with ctx.Pool(cores) as pool:
@@ -209,7 +224,8 @@ def oracle_baseline(workers_per_core=4, ncand=32768, cores=None):
     pairs = sum(r[0] for r in res)
     busy = max(r[1] for r in res)
     return {"value": pairs / busy, "unit": UNIT, "cores": cores, "kind": "oracle",
-            "sample": "%d workers x %d candidates of %s (%d pairs, %.1f s per process, %.1f s wall)"
+            "sample": "%d workers x %d candidates of %s (%d pairs, %.1f s per process, %.1f s wall "
+                      "with process start-up)"
                       % (cores * workers_per_core, ncand, WORKLOAD, pairs, busy, wall)}
 
 
@@ -350,27 +366,46 @@ def run_configs(args):
 # ---------------------------------------------------------------------------
 
 def run_reference(args):
-    dist, rank, world, local = (None, 0, 1, 0)
+    """The reference arm: the CPU oracle on the host cores (the paper ships no
+    code to install). A step scores one bounded sample of the workload, the
+    same sample as the cpu_baseline leg (4 workers a core x 32,768
+    candidates); ms_per_step is the measured wall time of that sample, and
+    the time of a full 4,096 x 32,768 step is reported separately, labelled
+    as extrapolated."""
     if int(os.environ.get("WORLD_SIZE", "1")) > 1 and int(os.environ.get("RANK", "0")) != 0:
         return
-    steps, warm = args.steps, args.warmup
-    vals = []
-    base = None
-    for i in range(warm + steps):
-        b = oracle_baseline(workers_per_core=1, ncand=2048)
-        if i >= warm:
-            vals.append(b["value"])
-            base = b
-    v = float(statistics.median(vals)) if vals else 0.0
+    import multiprocessing as mp
+    from oracle import oracle as O
     from paper_2405_06856_gb300 import synth
+    O.build()
+    steps, warm = args.steps, args.warmup
+    cores = os.cpu_count() or 1
+    wpc, ncand = 4, 32768
+    jobs = oracle_jobs(wpc, ncand, cores)
+    walls, pairs = [], 0
+    with mp.get_context("spawn").Pool(cores) as pool:
+        pool.map(_oracle_slice, jobs)  # builds each process's sub-cluster, untimed
+        for i in range(warm + steps):
+            t0 = time.perf_counter()
+            res = pool.map(_oracle_slice, jobs)
+            wall = time.perf_counter() - t0
+            if i >= warm:
+                walls.append(wall)
+                pairs = sum(r[0] for r in res)
+    wall = float(statistics.median(walls))
+    v = pairs / wall
     wl = synth.config(WORKLOAD, n_cand=16)
-    ms = wl.n_workers * 32768 / v * 1000.0 if v > 0 else None
-    base["value"] = v
+    sample = ("%d workers x %d candidates of %s (%d pairs) on %d host processes, one step each; "
+              "median wall %.3f s over %d steps" % (cores * wpc, ncand, WORKLOAD, pairs, cores,
+                                                    wall, steps))
     line = {"impl": "reference", "metric": METRIC, "value": v, "unit": UNIT,
-            "n_gpus": args.gpus, "steps": steps, "warmup": warm, "ms_per_step": ms,
+            "n_gpus": args.gpus, "steps": steps, "warmup": warm, "ms_per_step": wall * 1000.0,
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
-            "data": "synthetic", "config": {"workload": WORKLOAD_DESC},
-            "cpu_baseline": base,
+            "data": "synthetic",
+            "config": {"workload": WORKLOAD_DESC, "sample": sample, "pairs_per_step": pairs,
+                       "extrapolated_full_step_ms": wl.n_workers * 32768 / v * 1000.0},
+            "cpu_baseline": {"value": v, "unit": UNIT, "cores": cores, "kind": "oracle",
+                             "sample": sample},
             "e2e": {"value": v, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
     print(json.dumps(line))
 
