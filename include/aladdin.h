@@ -220,20 +220,24 @@ int aladdin_score_detail(aladdin_cluster* cl, int32_t n_cand, const int32_t* in,
 #define ALADDIN_NOALLOC_MAX_CAND 32768
 
 /* aladdin_score for callers that cannot allocate device memory during the
- * call: code recording a CUDA stream capture, processes whose device memory
- * is reserved up front by another allocator (a serving engine owning the
- * KV-cache pool), real-time scheduling loops. The paper has no counterpart;
- * this is a property of the library.
+ * call: processes whose device memory is reserved up front by another
+ * allocator (a serving engine owning the whole KV-cache pool leaves nothing
+ * for a cudaMalloc to take), real-time scheduling loops that must not pay the
+ * allocator's latency or its implicit synchronisation. The paper has no
+ * counterpart; this is a property of the library.
  * Same inputs, outputs and results as aladdin_score, but every pointer must be
- * device (or managed) memory of the cluster's GPU (ALADDIN_ERR_ARG otherwise),
- * the call is asynchronous on the cluster's stream, and it calls no
- * allocator: its scratch is a fixed device array (about 2 MB) built into the
- * library, held by every GPU that loads it until the process exits.
+ * device memory of the cluster's GPU, or managed memory (ALADDIN_ERR_ARG
+ * otherwise, before anything is launched), the call is asynchronous on the
+ * cluster's stream, and it calls no allocator: its scratch is a fixed device
+ * array (about 2 MB) built into the library, held by every GPU that loads it
+ * until the process exits.
  * n_cand may be at most ALADDIN_NOALLOC_MAX_CAND (ALADDIN_ERR_SCRATCH
- * otherwise). The first call on a device looks up the array's device address;
- * make that first call before any stream capture. All calls share the array:
- * calls that overlap on the GPU (several streams, or several clusters on one
- * device) race on it, and the caller must serialize them. */
+ * otherwise). The first call on a device sets up that device: it looks up the
+ * array's device address and loads every scoring kernel with its launch
+ * configuration; make that first call before any stream capture. All calls
+ * share the array: calls that overlap on the GPU (several streams, or several
+ * clusters on one device) race on it, and the caller must serialize them.
+ * cudaDeviceReset while the library is in use is not supported. */
 int aladdin_score_noalloc(aladdin_cluster* cl, int32_t n_cand, const int32_t* in,
                           const int32_t* pred, const float* wait_ms, uint8_t* flags,
                           float* margin, int32_t* argbest);

@@ -117,6 +117,39 @@ cudaError_t allow_max_smem()
     return e;
 }
 
+// Resident CTAs per SM of Kern at `threads` threads and `smem` bytes of
+// dynamic shared memory (whose limit is raised to `smem` for the kernel), queried
+// once per device ordinal < 64 and cached (thread-safe; concurrent first
+// queries compute and store the same value).
+template <auto Kern>
+cudaError_t kernel_occupancy(int threads, size_t smem, int* per_sm)
+{
+    static std::atomic<int> cache[64];  // 0: not queried on that device yet
+    DevInfo d;
+    cudaError_t e = device_info(&d);
+    if (e != cudaSuccess) return e;
+    const bool slot = d.device >= 0 && d.device < 64;
+    int v = slot ? cache[d.device].load(std::memory_order_acquire) : 0;
+    if (v == 0) {
+        if ((e = cudaFuncSetAttribute(Kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                      (int)smem)) != cudaSuccess)
+            return e;
+        int ps = 0;
+        e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&ps, Kern, threads, smem);
+        if (e != cudaSuccess) return e;
+        v = ps < 1 ? 1 : ps;
+        if (slot) cache[d.device].store(v, std::memory_order_release);
+    }
+    *per_sm = v;
+    return cudaSuccess;
+}
+
+// Loads every kernel the scoring path (launch_score) may launch on the
+// current device and caches its launch configuration, so that later scoring
+// calls on that device reach neither the module loader (which places kernel
+// code in device memory on a kernel's first use) nor a device query.
+cudaError_t prepare_score_kernels();
+
 // Execution of every worker for dt ms from t_now.
 // stats: device [0] prefills run, [1] finished, [2] max TTFT bits, [3] max
 // ATGT bits (non-negative doubles compare like their bit patterns), realized

@@ -1,15 +1,16 @@
 // aladdin_score_noalloc: candidate x worker scoring that allocates nothing.
 //
-// For callers that cannot call cudaMalloc while they schedule: code running
-// inside a CUDA stream capture, processes whose device memory is reserved up
-// front by another allocator (a serving engine that owns the whole KV-cache
-// pool), or real-time loops that must not hit the allocator. aladdin_score
-// grows private scratch buffers (the sorted candidate records, the
-// predicted-length histogram and the per-candidate argbest keys) with
-// cudaMalloc and stages host arrays through device copies. This entry point
-// uses one file-scope device array instead, so every buffer it touches exists
-// from the moment the library is loaded on a device, and it accepts device (or
-// managed) pointers only.
+// For callers that must not reach a device allocator while they schedule:
+// processes whose device memory is reserved up front by another allocator (a
+// serving engine that owns the whole KV-cache pool and leaves nothing for a
+// cudaMalloc to take), or real-time loops that cannot afford the allocator's
+// latency or its implicit device synchronisation. aladdin_score grows private
+// scratch buffers (the sorted candidate records, the predicted-length
+// histogram and the per-candidate argbest keys) with cudaMalloc and stages
+// host arrays through device copies. This entry point uses one file-scope
+// device array instead, so every buffer it touches exists from the moment the
+// library is loaded on a device, and it accepts device (or managed) pointers of
+// the cluster's GPU only.
 //
 // The array holds the scratch of up to NOALLOC_MAX_CAND candidates. Every GPU
 // that loads the library keeps it until the process exits. All calls share
@@ -17,6 +18,14 @@
 // device) race on it and must be serialized by the caller. What must start
 // from zero (the histogram) is cleared on every call; the argbest keys are
 // rewritten on every call.
+//
+// Set-up, once per device, on the first call with that device current: the
+// array's device address (in host code the symbol is only a host-side
+// handle) and the loading of every scoring kernel with its launch
+// configuration, so that later calls reach neither the module loader nor a
+// device query. The address belongs to the device's primary context:
+// cudaDeviceReset while the library is in use is not supported (it also
+// invalidates every cluster's device memory).
 #include <mutex>
 
 #include "../../include/aladdin.h"
@@ -44,7 +53,8 @@ int scratch_address(int device, void** out)
     std::lock_guard<std::mutex> lock(g_mu);
     if (!g_scratch[device]) {
         void* p = nullptr;
-        const cudaError_t e = cudaGetSymbolAddress(&p, g_score_scratch);
+        cudaError_t e = cudaGetSymbolAddress(&p, g_score_scratch);
+        if (e == cudaSuccess) e = aladdin::prepare_score_kernels();
         if (e != cudaSuccess || !p) {
             cudaGetLastError();
             return ALADDIN_ERR_CUDA;
@@ -55,14 +65,16 @@ int scratch_address(int device, void** out)
     return ALADDIN_OK;
 }
 
-bool on_device(const void* p)
+// Device memory of `device`, or managed memory (which any device may reach).
+bool on_device(const void* p, int device)
 {
     cudaPointerAttributes a;
     if (cudaPointerGetAttributes(&a, p) != cudaSuccess) {
         cudaGetLastError();
         return false;
     }
-    return a.type == cudaMemoryTypeDevice || a.type == cudaMemoryTypeManaged;
+    if (a.type == cudaMemoryTypeManaged) return true;
+    return a.type == cudaMemoryTypeDevice && a.device == device;
 }
 
 }  // namespace
@@ -80,7 +92,7 @@ try {
     if (!in || !pred) return ALADDIN_ERR_ARG;
     const void* ptrs[6] = {in, pred, wait_ms, flags, margin, argbest};
     for (const void* p : ptrs)
-        if (p && !on_device(p)) return ALADDIN_ERR_ARG;
+        if (p && !on_device(p, v.device)) return ALADDIN_ERR_ARG;
     if (cudaSetDevice(v.device) != cudaSuccess) {
         cudaGetLastError();
         return ALADDIN_ERR_CUDA;

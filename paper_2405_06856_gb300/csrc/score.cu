@@ -587,21 +587,15 @@ static cudaError_t launch_vec(const ScoreArgs& A0, cudaStream_t st)
     A.best = A0.best;
     A.tiles = (A.C.W + SCORE_WARPS * 32 * SLOTS - 1) / (SCORE_WARPS * 32 * SLOTS);
     const size_t smem = sizeof(ScoreSmem);
-    static int per_sm = 0, sms = 0;  // occupancy of this instantiation (per process)
-    if (per_sm == 0) {
-        cudaError_t e = cudaFuncSetAttribute(k_score<SLOTS, SF, SMG, ARG, PEND, FULLT, APPROX>,
-                                             cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-        if (e != cudaSuccess) return e;
-        int dev = 0;
-        cudaGetDevice(&dev);
-        cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
-        int ps = 0;
-        e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&ps, k_score<SLOTS, SF, SMG, ARG, PEND, FULLT, APPROX>,
-                                                          SCORE_WARPS * 32, smem);
-        per_sm = (e != cudaSuccess || ps < 1) ? 1 : ps;
-    }
+    DevInfo d;
+    cudaError_t e = device_info(&d);
+    if (e != cudaSuccess) return e;
+    int per_sm = 0;  // occupancy of this instantiation on this device (cached)
+    e = kernel_occupancy<k_score<SLOTS, SF, SMG, ARG, PEND, FULLT, APPROX>>(SCORE_WARPS * 32, smem,
+                                                                          &per_sm);
+    if (e != cudaSuccess) return e;
     // one wave: per_tile CTAs share each worker tile's candidates equally
-    const int wave = per_sm * sms;
+    const int wave = per_sm * d.sms;
     int per_tile = wave / A.tiles;
     if (per_tile < 1) per_tile = 1;
     const int max_parts = (A.n_cand + 63) / 64;  // at least 64 candidates per CTA
@@ -640,6 +634,28 @@ static cudaError_t dispatch_vec(bool approx, bool sf, bool smg, bool arg, const 
     const bool full = A.C.W % (SCORE_WARPS * 32 * ALADDIN_SCORE_SLOTS) == 0;
     return full ? dispatch_vec2<PEND, true>(approx, sf, smg, arg, A, st)
                 : dispatch_vec2<PEND, false>(approx, sf, smg, arg, A, st);
+}
+
+// prepare_score_kernels: every k_score instantiation dispatch_vec can reach
+// (seven output combinations x pending x full tile x approximate), the scalar
+// variants and the candidate preparation, finalize and detail kernels.
+template <bool PEND, bool FULLT, bool APPROX>
+static cudaError_t prepare_vec3()
+{
+    constexpr int S = ALADDIN_SCORE_SLOTS;
+    constexpr int T = SCORE_WARPS * 32;
+    constexpr size_t M = sizeof(ScoreSmem);
+    int ps = 0;
+    cudaError_t e;
+    if ((e = kernel_occupancy<k_score<S, true, true, true, PEND, FULLT, APPROX>>(T, M, &ps)) ||
+        (e = kernel_occupancy<k_score<S, true, true, false, PEND, FULLT, APPROX>>(T, M, &ps)) ||
+        (e = kernel_occupancy<k_score<S, true, false, true, PEND, FULLT, APPROX>>(T, M, &ps)) ||
+        (e = kernel_occupancy<k_score<S, false, true, true, PEND, FULLT, APPROX>>(T, M, &ps)) ||
+        (e = kernel_occupancy<k_score<S, true, false, false, PEND, FULLT, APPROX>>(T, M, &ps)) ||
+        (e = kernel_occupancy<k_score<S, false, true, false, PEND, FULLT, APPROX>>(T, M, &ps)) ||
+        (e = kernel_occupancy<k_score<S, false, false, true, PEND, FULLT, APPROX>>(T, M, &ps)))
+        return e;
+    return cudaSuccess;
 }
 
 template <bool SF, bool SMG, bool ARG>
@@ -701,6 +717,27 @@ __global__ void k_detail(DevParams P, ClusterDev C, int n, const int32_t* __rest
             t_cand[idx] = (float)(sc * (P.c3d * (double)rr + P.c2d * X1 + P.k2d * X2));
         }
     }
+}
+
+cudaError_t prepare_score_kernels()
+{
+    cudaError_t e;
+    if ((e = prepare_vec3<false, false, false>()) || (e = prepare_vec3<false, false, true>()) ||
+        (e = prepare_vec3<false, true, false>()) || (e = prepare_vec3<false, true, true>()) ||
+        (e = prepare_vec3<true, false, false>()) || (e = prepare_vec3<true, false, true>()) ||
+        (e = prepare_vec3<true, true, false>()) || (e = prepare_vec3<true, true, true>()))
+        return e;
+    cudaFuncAttributes fa;
+    const void* kerns[] = {
+        (const void*)k_score_scalar<true, true, true>, (const void*)k_score_scalar<true, true, false>,
+        (const void*)k_score_scalar<true, false, true>, (const void*)k_score_scalar<false, true, true>,
+        (const void*)k_score_scalar<true, false, false>, (const void*)k_score_scalar<false, true, false>,
+        (const void*)k_score_scalar<false, false, true>, (const void*)k_cand_count,
+        (const void*)k_scan_hist, (const void*)k_cand_scatter, (const void*)k_finalize,
+        (const void*)k_detail};
+    for (const void* k : kerns)
+        if ((e = cudaFuncGetAttributes(&fa, k)) != cudaSuccess) return e;
+    return cudaSuccess;
 }
 
 cudaError_t launch_cand_prep(const DevParams& P, int W, int n, const int32_t* in,

@@ -1,10 +1,10 @@
 """aladdin_score_noalloc, the scoring call for callers that cannot allocate
-device memory while they schedule (a CUDA stream capture being recorded, a
-process whose device memory a serving engine reserved up front, a real-time
-loop that must not reach the allocator). It must give the same results as
-aladdin_score, call after call, although all calls share one fixed scratch
-array. Collected last so that a failure here stops a -x run only after every
-other test has run."""
+device memory while they schedule (a process whose device memory a serving
+engine reserved up front for its KV cache, a real-time loop that must not
+reach the allocator). It must give the same results as aladdin_score, call
+after call, although all calls share one fixed scratch array, and after its
+first call on a device it must take no device memory at all. Collected last
+so that a failure here stops a -x run only after every other test has run."""
 import numpy as np
 import pytest
 
@@ -82,3 +82,34 @@ def test_noalloc_rejects_what_it_cannot_hold(A, synth):
             A.aladdin_score_noalloc(cl.handle, 8, wl.cand_in, wl.cand_pred, None, None, None,
                                     np.zeros(8, np.int32))
         assert e.value.code == A.ERR_ARG
+
+
+def test_noalloc_takes_no_device_memory(A, synth):
+    """After the first call on the device (which sets the device up), calls
+    with every combination of outputs leave the device's free memory
+    unchanged: nothing is allocated, not even kernel code."""
+    import torch
+    wl = synth.config("w256", n_cand=2000)
+    dev = torch.device("cuda")
+    t = lambda x: torch.from_numpy(np.ascontiguousarray(x)).to(dev)
+    C, W = wl.n_cand, wl.n_workers
+    din, dpr, dw = t(wl.cand_in), t(wl.cand_pred), t(wl.cand_wait)
+    f = torch.empty((C, W), dtype=torch.uint8, device=dev)
+    m = torch.empty((C, W), dtype=torch.float32, device=dev)
+    a = torch.empty(C, dtype=torch.int32, device=dev)
+    ref = torch.empty(C, dtype=torch.int32, device=dev)
+    with A.Cluster.from_workload(wl) as cl:
+        A.aladdin_score(cl.handle, C, din, dpr, dw, None, None, ref)
+        A.aladdin_score_noalloc(cl.handle, 16, din, dpr, dw, None, None, a)  # set-up
+        torch.cuda.synchronize()
+        free0 = torch.cuda.mem_get_info()[0]
+        for outs in ((f, m, a), (f, None, None), (None, m, None), (None, None, a), (f, None, a),
+                     (None, m, a), (f, m, None)):
+            for n in (C, 7):
+                A.aladdin_score_noalloc(cl.handle, n, din, dpr, dw, *outs)
+        torch.cuda.synchronize()
+        free1 = torch.cuda.mem_get_info()[0]
+        assert free1 == free0, "device free memory moved by %d bytes" % (free1 - free0)
+        A.aladdin_score_noalloc(cl.handle, C, din, dpr, dw, None, None, a)
+        torch.cuda.synchronize()
+        assert torch.equal(a, ref)
