@@ -147,7 +147,8 @@ typedef struct {
     double mscale;        /* token scale of the binding latency bound; 0 if KV binds */
     int64_t kv_peak;      /* peak KV over all future iterations with the candidate */
     double t_cand;        /* candidate's projected decode time, all iterations (ms) */
-    double near;          /* smallest |slack| / scale over latency constraints at a_c */
+    double near;          /* over the latency groups, the smallest |min slack / scale|
+                             at a_c: how close the closest flag bit is to flipping */
 } orc_pair;
 
 enum { ORC_OK = 0, ORC_ERR_ARG = -1, ORC_ERR_CAPACITY = -2, ORC_ERR_MEM = -3 };
@@ -214,9 +215,11 @@ static int64_t floor_div(int64_t x, int64_t d) /* d > 0 */
     return q;
 }
 
-/* Running minimum of the constraint bounds. */
+/* Running minimum of the constraint bounds; gmin[g] is the smallest relative
+ * slack (slack / scale, signed) among group g's constraints at a_c. */
 typedef struct {
-    double bound, bscale, near;
+    double bound, bscale;
+    double gmin[4];
     int ok[4];
 } orc_acc;
 
@@ -234,8 +237,8 @@ static void lat_constraint(orc_acc* A, int group, double slack0, double slope,
         A->bound = b;
         A->bscale = slope > 0.0 ? scale_a / slope : 0.0;
     }
-    double rel = fabs(slack_a) / (scale_a > 0.0 ? scale_a : 1.0);
-    if (rel < A->near) A->near = rel;
+    double rel = slack_a / (scale_a > 0.0 ? scale_a : 1.0);
+    if (rel < A->gmin[group]) A->gmin[group] = rel;
 }
 
 /* Evaluate candidate (a_c, r_c, w_c) on worker w. T0, T1 are scratch arrays of
@@ -278,7 +281,7 @@ static void eval_pair(const orc_params* p, const orc_cluster* cl, int w, const o
     orc_acc A;
     A.bound = INFINITY;
     A.bscale = 0.0;
-    A.near = INFINITY;
+    for (int g = 0; g < 4; ++g) A.gmin[g] = INFINITY;
     for (int g = 0; g < 4; ++g) A.ok[g] = 1;
     const double a = (double)a_c;
 
@@ -374,7 +377,13 @@ static void eval_pair(const orc_params* p, const orc_cluster* cl, int w, const o
     out->margin = bound - a;
     out->mscale = bscale;
     out->kv_peak = kv_peak;
-    out->near = A.near;
+    /* A group's flag is the sign of its smallest slack; arithmetic with a
+     * relative error below e per constraint can flip it only when that
+     * smallest relative slack lies within e of zero. */
+    double near = INFINITY;
+    for (int g = 0; g < 4; ++g)
+        if (fabs(A.gmin[g]) < near) near = fabs(A.gmin[g]);
+    out->near = near;
 }
 
 /* ---------------------------------------------------------------------- */

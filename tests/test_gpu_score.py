@@ -299,3 +299,38 @@ def test_load_score_equals_two_calls(A, synth):
             outs.append((f.tobytes(), m.tobytes(), a.tobytes(),
                          tuple(x.tobytes() for x in cl.state())))
     assert outs[0] == outs[1] == outs[2]
+
+
+def test_history_hand_cases(A):
+    """The kernels reproduce the hand-worked decode-history, offset cases
+    (tests/golden/history_example.json): constraint (d) with banked slack
+    theta T_dec l_out - t^dec, and the TTFT bound after an execution step
+    whose last iteration straddles the heartbeat."""
+    import json
+    import os
+    from parity import REL
+    with open(os.path.join(os.path.dirname(__file__), "golden", "history_example.json")) as f:
+        g = json.load(f)
+    b = g["bank"]
+    w = b["worker"]
+    arr = lambda x, t=np.int32: np.ascontiguousarray(x, t)
+    cand = b["candidate"]
+    for c in b["cases"]:
+        with A.Cluster(b["params"], [1], [b["M"]], [1.0], 32, arr([0, 2]), arr(w["in"]),
+                       arr(w["gen"]), arr(w["pred"]), tdec_ms=arr(c["tdec"], np.float32)) as cl:
+            out = cl.score([cand["in"]], [cand["pred"]], [cand["wait"]])
+        assert int(out["flags"][0, 0]) == c["flags"], c
+        tol = REL * max(abs(c["margin"] + cand["in"]), 1.0)
+        assert abs(float(out["margin"][0, 0]) - c["margin"]) <= tol, (out["margin"], c)
+    o = g["offset"]
+    w = o["worker"]
+    with A.Cluster(o["params"], [1], [o["M"]], [1.0], 32, arr([0, 1]), arr(w["in"]), arr(w["gen"]),
+                   arr(w["pred"]), tdec_ms=arr([0.0], np.float32)) as cl:
+        cl.advance(o["heartbeat_ms"])
+        n, i, gen, p, pe = cl.state()
+        assert int(n[0]) == 1 and int(gen[0]) == o["after"]["gen"]
+        for c in o["cases"]:
+            out = cl.score([o["candidate"]["in"]], [o["candidate"]["pred"]], [c["wait"]])
+            assert int(out["flags"][0, 0]) == c["flags"], c
+            tol = REL * max(abs(c["margin"] + o["candidate"]["in"]), 1.0)
+            assert abs(float(out["margin"][0, 0]) - c["margin"]) <= tol, (out["margin"], c)
