@@ -183,7 +183,8 @@ def _oracle_slice(args):
     """Every pair of workers `wid` with the first `ncand` candidates, scored by
     the oracle in this (spawned) process; the workload and the sub-cluster are
     built once per process, outside the timed scoring."""
-    wid, ncand = args
+    wid, ncand = args[0], args[1]
+    keep = len(args) > 2 and args[2]
     from oracle import oracle as O
     from paper_2405_06856_gb300 import synth
     key = (tuple(wid), ncand)
@@ -198,24 +199,29 @@ def _oracle_slice(args):
                              wl.cand_wait[:ncand].copy())
     sub, cin, cpr, cw = _SLICE_CACHE[key]
     t0 = time.perf_counter()
-    sub.score(cin, cpr, cw, want=("flags", "margin"))
-    return len(wid) * ncand, time.perf_counter() - t0
+    out = sub.score(cin, cpr, cw, want=("flags", "margin", "near"))
+    dt = time.perf_counter() - t0
+    if keep:
+        return len(wid) * ncand, dt, wid, out["flags"], out["near"]
+    return len(wid) * ncand, dt
 
 
-def oracle_jobs(workers_per_core, ncand, cores):
-    return [(list(range(i * workers_per_core, (i + 1) * workers_per_core)), ncand)
+def oracle_jobs(workers_per_core, ncand, cores, keep=False):
+    return [(list(range(i * workers_per_core, (i + 1) * workers_per_core)), ncand, keep)
             for i in range(cores)]
 
 
-def oracle_baseline(workers_per_core=4, ncand=32768, cores=None):
+def oracle_baseline(workers_per_core=4, ncand=32768, cores=None, keep=False):
     """Oracle evaluations/sec: each process scores all pairs of its own workers
     against the first `ncand` candidates; throughput = pairs / wall time of
-    the parallel scoring (the slowest process)."""
+    the parallel scoring (the slowest process). keep: also return the
+    sample's oracle flags and near measures (worker ids, flags [ncand, nw],
+    near [ncand, nw]) for the parity report of the same pairs."""
     import multiprocessing as mp
     from oracle import oracle as O
     O.build()
     cores = cores or os.cpu_count() or 1
-    jobs = oracle_jobs(workers_per_core, ncand, cores)
+    jobs = oracle_jobs(workers_per_core, ncand, cores, keep)
     ctx = mp.get_context("spawn")
     t0 = time.perf_counter()
     with ctx.Pool(cores) as pool:
@@ -223,10 +229,32 @@ def oracle_baseline(workers_per_core=4, ncand=32768, cores=None):
     wall = time.perf_counter() - t0
     pairs = sum(r[0] for r in res)
     busy = max(r[1] for r in res)
-    return {"value": pairs / busy, "unit": UNIT, "cores": cores, "kind": "oracle",
+    line = {"value": pairs / busy, "unit": UNIT, "cores": cores, "kind": "oracle",
             "sample": "%d workers x %d candidates of %s (%d pairs, %.1f s per process, %.1f s wall "
                       "with process start-up)"
                       % (cores * workers_per_core, ncand, WORKLOAD, pairs, busy, wall)}
+    if not keep:
+        return line
+    wid = np.concatenate([r[2] for r in res])
+    return line, (wid, np.concatenate([r[3] for r in res], axis=1),
+                  np.concatenate([r[4] for r in res], axis=1))
+
+
+def parity_report(sample, flags_dev):
+    """The benchmarked call's flags on the oracle's sample pairs: mismatches
+    outside the near pairs (must be 0), near pairs and near flips by
+    direction (the tolerance rule of the parity tests: a pair is near when a
+    constraint group's smallest relative slack is within 1e-5 of zero)."""
+    import torch
+    wid, oflags, onear = sample
+    idx = torch.from_numpy(wid.astype(np.int64)).to(flags_dev.device)
+    g = flags_dev[: oflags.shape[0]].index_select(1, idx).cpu().numpy()
+    near = onear <= 1e-5
+    gf, of = g == 15, oflags == 15
+    return {"pairs": int(g.size), "far_mismatches": int((~near & (g != oflags)).sum()),
+            "near": int(near.sum()), "near_gpu_only": int((near & gf & ~of).sum()),
+            "near_oracle_only": int((near & ~gf & of).sum()),
+            "sample": "the cpu_baseline sample's pairs (oracle flags vs the benchmarked call's)"}
 
 
 def _oracle_config_job(job):
@@ -418,9 +446,9 @@ def run_ours(args):
     from paper_2405_06856_gb300 import synth
 
     # The oracle's process pool is started before the first CUDA call.
-    cpu = None
+    cpu = sample = None
     if args.cpu_baseline and int(os.environ.get("RANK", "0")) == 0 and args.gpus == 1:
-        cpu = oracle_baseline()
+        cpu, sample = oracle_baseline(keep=True)
 
     dist, rank, world, local = dist_setup(args)
     dev = torch.device("cuda", local)
@@ -477,6 +505,7 @@ def run_ours(args):
         clocks["window"] = "%.1f s of the same steps (untimed), then the timed steps" % CLOCK_WINDOW_S
     kern_ms, kern_n = A.aladdin_cluster_timing(cl.handle, 0)
     step_ms = sum(s.elapsed_time(e) for s, e in zip(starts, ends)) / args.steps
+    parity = parity_report(sample, flags) if sample is not None else None
     step_ms = barrier_max(dist, step_ms)
     value = whole_job_value(world, C * W, step_ms)
 
@@ -524,6 +553,7 @@ def run_ours(args):
     # so that every group holds all four worker sizes
     r16k_grp = {"G%d" % G: rounds_w16384(A, synth, stream, groups=G) for G in (7, 63)}
     apx = approx_mode(A, synth, dev, stream, flush)
+    mixed = mixed_mask(A, synth, dev, stream, flush)
     pol = policy_compare(A, synth, stream, 20_000, [1, 2])
     wmod = worker_model(A, synth, stream, fit_n=0)
 
@@ -557,11 +587,14 @@ def run_ours(args):
             "rounds_w16384": r16k,
             "rounds_w16384_grouped": r16k_grp,
             "approx_mode": apx,
+            "mixed_mask": mixed,
             "policies": pol,
             "worker_config": wmod,
             "clocks": clocks}
     if cpu is not None:
         line["cpu_baseline"] = cpu
+    if parity is not None:
+        line["parity_sample"] = parity
     if rank == 0:
         print(json.dumps(line))
     cl.close()
@@ -643,6 +676,53 @@ def approx_mode(A, synth, dev, stream, flush, launches=10):
             "w256_feasible_approx": round(float(ap.mean()), 4),
             "w256_approx_feasible_exact_infeasible": round(float((ap & ~ex).mean()), 4),
             "w256_exact_feasible_approx_infeasible": round(float((ex & ~ap).mean()), 4)}
+
+
+def mixed_mask(A, synth, dev, stream, flush, launches=10):
+    """The benchmarked step on the 4,096-worker workload with tighter limits
+    and a decode history (w4096_mixed: about half of the pairs feasible,
+    every constraint group binding): its scoring-kernel time and HBM fraction
+    against the all-feasible workload's."""
+    import torch
+    wl = synth.config("w4096_mixed")
+    tdec = synth.decode_history(wl, 18.0, 26.0, synth.MIXED_HISTORY_SEED)
+    W, C = wl.n_workers, wl.n_cand
+    d = lambda x: torch.from_numpy(np.ascontiguousarray(x)).to(dev)
+    roff, rin, rgen, rpred, rt = d(wl.roff), d(wl.req_in), d(wl.req_gen), d(wl.req_pred), d(tdec)
+    cin, cpr, cw = d(wl.cand_in), d(wl.cand_pred), d(wl.cand_wait)
+    f = torch.empty((C, W), dtype=torch.uint8, device=dev)
+    m = torch.empty((C, W), dtype=torch.float32, device=dev)
+    a = torch.empty(C, dtype=torch.int32, device=dev)
+    starts = [torch.cuda.Event(enable_timing=True) for _ in range(launches)]
+    ends = [torch.cuda.Event(enable_timing=True) for _ in range(launches)]
+    with A.Cluster.from_workload(wl, tdec_ms=tdec, stream=stream) as cl:
+        step = lambda: A.aladdin_cluster_load_score(cl.handle, roff, rin, rgen, rpred, rt, C, cin,
+                                                    cpr, cw, f, m, a)
+        for _ in range(3):
+            step()
+        torch.cuda.synchronize()
+        A.aladdin_cluster_timing(cl.handle, 1)
+        for i in range(launches):
+            flush.zero_()
+            starts[i].record()
+            step()
+            ends[i].record()
+        torch.cuda.synchronize()
+        kern_ms, kern_n = A.aladdin_cluster_timing(cl.handle, 0)
+        assert cl.status() == A.OK
+        feas = float((f == 15).float().mean().item())
+        cleared = [round(float(((f >> b) & 1 == 0).float().mean().item()), 4) for b in range(4)]
+    kern = kern_ms / max(kern_n, 1)
+    step_ms = sum(s.elapsed_time(e) for s, e in zip(starts, ends)) / launches
+    peak, _ = read_peaks()
+    achieved = algorithmic_bytes(W, int(np.diff(wl.roff).max()), C) / (kern / 1000.0) / 1e9
+    return {"workload": "w4096 sizes and draws with KV 90,000 tokens, TTFT 95 ms, ATGT 30 ms and "
+                        "decode histories of 18-26 ms a token (exact mode)",
+            "k_score_us": kern * 1000.0, "hbm_gbs": achieved, "hbm_frac": achieved / peak,
+            "ms_per_step": step_ms, "evals_per_s": C * W / (step_ms / 1000.0),
+            "feasible_fraction": round(feas, 4),
+            "cleared_fraction_by_group": dict(zip(("kv", "ttft", "ongoing_atgt", "new_atgt"),
+                                                  cleared))}
 
 
 def min_workers_config(synth):

@@ -126,6 +126,10 @@ def config(name, **over):
              coefficients x 1/sqrt(GPUs)), 256 requests each (1,024 request
              slots: an 8-GPU worker meets its SLOs with several hundred),
              131,072 candidates, output law as w4096, seed 3.
+    w4096_mixed  w4096's sizes and draws (seed 2) with tighter limits, so that
+             about half of the pairs are feasible and every constraint group
+             binds somewhere: KV 90,000 tokens, TTFT 95 ms, ATGT 30 ms; pair
+             it with decode_history(wl, 18.0, 26.0, MIXED_HISTORY_SEED).
     """
     if name == "tiny":
         kw = dict(seed=0, n_workers=16, per_worker=32, kv_per_gpu=16384, n_cand=64)
@@ -134,6 +138,9 @@ def config(name, **over):
     elif name == "w4096":
         kw = dict(seed=2, n_workers=4096, per_worker=128, kv_per_gpu=131072,
                   n_cand=32768, out_law=HEAVY_OUT)
+    elif name == "w4096_mixed":
+        kw = dict(seed=2, n_workers=4096, per_worker=128, kv_per_gpu=90000,
+                  n_cand=32768, out_law=HEAVY_OUT, params=dict(T_pre=95.0, T_dec=30.0))
     elif name == "w16384":
         kw = dict(seed=3, n_workers=16384, per_worker=256, kv_per_gpu=131072,
                   n_cand=131072, out_law=HEAVY_OUT, gpus_cycle=(1, 2, 4, 8),
@@ -142,6 +149,18 @@ def config(name, **over):
         raise KeyError(name)
     kw.update(over)
     return make_cluster(name, **kw)
+
+
+MIXED_HISTORY_SEED = 9
+
+
+def decode_history(wl, lo_ms, hi_ms, seed):
+    """Decode time so far (Table 1's t^dec, ms) of every ongoing request: its
+    generated tokens times a per-request rate drawn uniform in [lo_ms, hi_ms)
+    ms a token; float32, as the C ABI takes it."""
+    rng = np.random.default_rng(seed)
+    rate = rng.uniform(lo_ms, hi_ms, len(wl.req_gen))
+    return (wl.req_gen.astype(np.float64) * rate).astype(np.float32)
 
 
 @dataclasses.dataclass

@@ -226,6 +226,49 @@ def test_w4096_sampled(A, orc, synth):
         check_argbest(order, fr_rows, a.cpu().numpy()[rows], "w4096-rows")
 
 
+def test_w4096_mixed_sampled(A, orc, synth):
+    """The 4,096-worker workload with tighter limits and a decode history
+    (about half of the pairs feasible, every constraint group binding), at
+    full size through the benchmarked call: sampled pairs and argbest rows
+    against the oracle, near pairs bounded and reported."""
+    import torch
+    wl = synth.config("w4096_mixed")
+    tdec = synth.decode_history(wl, 18.0, 26.0, synth.MIXED_HISTORY_SEED)
+    C, W = wl.n_cand, wl.n_workers
+    dev = torch.device("cuda")
+    d = lambda x: torch.from_numpy(np.ascontiguousarray(x)).to(dev)
+    with A.Cluster.from_workload(wl, tdec_ms=tdec) as cl:
+        f = torch.zeros((C, W), dtype=torch.uint8, device=dev)
+        m = torch.zeros((C, W), dtype=torch.float32, device=dev)
+        a = torch.zeros(C, dtype=torch.int32, device=dev)
+        cin, cpr, cw = d(wl.cand_in), d(wl.cand_pred), d(wl.cand_wait)
+        A.aladdin_cluster_load_score(cl.handle, d(wl.roff), d(wl.req_in), d(wl.req_gen),
+                                     d(wl.req_pred), d(tdec), C, cin, cpr, cw, f, m, a)
+        torch.cuda.synchronize()
+        assert cl.status() == A.OK
+        fr = (f == 15).float().mean().item()
+        assert 0.3 < fr < 0.7, fr
+        for b in range(4):  # every group is cleared on some pair
+            assert ((f >> b) & 1 == 0).any().item(), b
+        rng = np.random.default_rng(19)
+        pc = rng.integers(0, C, 6000).astype(np.int32)
+        pw = rng.integers(0, W, 6000).astype(np.int32)
+        oc = orc.Cluster.from_workload(wl, tdec=tdec.astype(np.float64))
+        ref = oc.score_pairs(pc, pw, wl.cand_in, wl.cand_pred, wl.cand_wait)
+        ip, iw = torch.from_numpy(pc).long().to(dev), torch.from_numpy(pw).long().to(dev)
+        rep = {}
+        compare_pairs(ref, f[ip, iw].cpu().numpy(), m[ip, iw].cpu().numpy(), wl.cand_in[pc],
+                      label="w4096-mixed-sampled", report=rep)
+        print("w4096_mixed sampled pairs:", rep)
+        rows = rng.integers(0, C, 6)
+        sub = oc.score(wl.cand_in[rows], wl.cand_pred[rows], wl.cand_wait[rows],
+                       want=("flags", "margin", "mscale", "near", "argbest"))
+        fr_rows = f[torch.from_numpy(rows).long().to(dev)].cpu().numpy()
+        mr_rows = m[torch.from_numpy(rows).long().to(dev)].cpu().numpy()
+        compare_pairs(sub, fr_rows, mr_rows, wl.cand_in[rows], label="w4096-mixed-rows")
+        check_argbest(oc.order(), fr_rows, a.cpu().numpy()[rows], "w4096-mixed-rows")
+
+
 def test_page_locked_host_buffers(A, orc, synth):
     """Page-locked host arrays are read and written in place by the kernels
     (state packed on the device, outputs written over the CPU-GPU link): the
