@@ -334,6 +334,22 @@ int aladdin_cluster_timing(aladdin_cluster* cl, int32_t enable, double* kernel_m
  * ALADDIN_ERR_CUDA. Errors are sticky. Synchronous. */
 int aladdin_cluster_status(aladdin_cluster* cl);
 
+/* Test hook of the failure handling of bounded device waits; the paper has
+ * no counterpart. Every spin-wait of the library's kernels is bounded: the
+ * placement round's grid exchange polls an arrival counter at most
+ * grid_polls times (default 2^22, about a second) and the scoring kernel
+ * polls each candidate-copy mbarrier at most mbar_polls times (default
+ * 2^26); a wait that runs out sets the cluster's sticky timeout bit and its
+ * kernel returns (aladdin_place_round returns ALADDIN_ERR_TIMEOUT, scoring
+ * calls leave it to aladdin_cluster_status). 0 keeps a default. run_out = 1
+ * makes the next waits run out by design, without any fault: the round's
+ * exchange waits for one arrival more than its CTAs make, and the scoring
+ * kernel does not issue its first candidate copy. For tests only: a cluster
+ * whose wait ran out keeps an incomplete round or incomplete outputs.
+ * ALADDIN_ERR_ARG for negative limits or run_out outside {0, 1}. */
+int aladdin_cluster_test_waits(aladdin_cluster* cl, int64_t grid_polls, int64_t mbar_polls,
+                               int32_t run_out);
+
 /* A request trace: arrival times (ms, non-decreasing), prompt and predicted
  * output lengths, and optionally prediction errors (Sec. 4.3): real[q] is the
  * output length request q really generates (the scheduler sees only

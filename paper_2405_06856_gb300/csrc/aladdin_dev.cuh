@@ -67,6 +67,13 @@ struct DevParams {
     int32_t policy;          // ALADDIN_POLICY_* of placement rounds
     int32_t groups;          // G > 1: request q is placed only on workers w = q (mod G)
     unsigned long long seed; // SplitMix64 seed of the power-of-two draws
+    // Bounded device waits: polls before a wait gives up, sets the sticky
+    // timeout bit and leaves the kernel (ALADDIN_ERR_TIMEOUT).
+    long long grid_wait_limit;  // the placement round's grid exchange
+    long long mbar_wait_limit;  // the scoring kernel's candidate-copy barriers
+    int32_t wait_test;          // test hook, 1: the next waits run out by design (the
+                                // round's exchange waits for one arrival more than its
+                                // CTAs make; the scoring kernel withholds its first copy)
 };
 
 // Relative slack of a realized latency over its SLO before the execution step

@@ -9,6 +9,10 @@
 
 namespace aladdin {
 
+// Default poll limits of the bounded device waits (about a second each).
+constexpr long long GRID_WAIT_POLLS = 1ll << 22;  // the round's grid exchange
+constexpr long long MBAR_WAIT_POLLS = 1ll << 26;  // the scoring kernel's copy barriers
+
 // Elements per lane of the per-warp table builder for a slot capacity.
 inline int lanes_per_worker(int cap) { return cap / 32; }
 

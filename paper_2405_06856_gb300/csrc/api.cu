@@ -185,6 +185,9 @@ DevParams make_devparams(const aladdin_params& p)
     d.thetad = p.theta;
     d.T_pre_viol = p.T_pre * (1.0 + SLO_TOL);
     d.T_dec_viol = p.T_dec * (1.0 + SLO_TOL);
+    d.grid_wait_limit = GRID_WAIT_POLLS;
+    d.mbar_wait_limit = MBAR_WAIT_POLLS;
+    d.wait_test = 0;
     return d;
 }
 
@@ -1034,6 +1037,19 @@ try {
     if (launches) *launches = (int64_t)(cl->ev.size() / 2);
     cl->clear_events();
     cl->timing = enable != 0;
+    return ALADDIN_OK;
+} catch (...) {
+    return ALADDIN_ERR_NOMEM;  // a host allocation or thread start failed
+}
+
+int aladdin_cluster_test_waits(aladdin_cluster* cl, int64_t grid_polls, int64_t mbar_polls,
+                               int32_t run_out)
+try {
+    if (!cl || grid_polls < 0 || mbar_polls < 0 || (run_out != 0 && run_out != 1))
+        return ALADDIN_ERR_ARG;
+    cl->dp.grid_wait_limit = grid_polls ? grid_polls : GRID_WAIT_POLLS;
+    cl->dp.mbar_wait_limit = mbar_polls ? mbar_polls : MBAR_WAIT_POLLS;
+    cl->dp.wait_test = run_out;
     return ALADDIN_OK;
 } catch (...) {
     return ALADDIN_ERR_NOMEM;  // a host allocation or thread start failed

@@ -197,7 +197,6 @@ struct R2Split {
 // 8) plus this pad makes the per-worker stride an odd number of 32-bit words,
 // so that lanes searching neighbouring workers start on different banks.
 constexpr int R2_RHO_PAD = 2;
-constexpr long long GRID_WAIT_LIMIT = 1ll << 22;  // polls of the arrival counter (seconds)
 constexpr int NONE = 0x7fffffff;
 
 struct R2Args {
@@ -457,9 +456,9 @@ __global__ void __launch_bounds__(R2_THREADS, 1) k_round2(R2Args A)
                 }
                 // every lane acquires the counter, so its loads below see the
                 // other CTAs' entries
-                const unsigned target = (unsigned)(c + 1) * (unsigned)A.G;
+                const unsigned target = (unsigned)(c + 1) * (unsigned)A.G + (unsigned)P.wait_test;
                 bool ok = false;
-                for (long long it = 0; it < GRID_WAIT_LIMIT; ++it) {
+                for (long long it = 0; it < P.grid_wait_limit; ++it) {
                     if (ld_acquire(A.arrive) >= target) {
                         ok = true;
                         break;

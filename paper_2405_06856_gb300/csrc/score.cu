@@ -87,6 +87,8 @@ struct ScoreArgs {
     unsigned int* best;
     int tiles, chunks;
     int approx;  // approximate-mode constraints (b) and (d)
+    long long wait_limit;  // mbarrier polls before a wait gives up
+    int withhold;          // test hook: the first candidate copy is not issued
 };
 
 __global__ void k_cand_scatter(DevParams P, int n, int W, const int32_t* __restrict__ in,
@@ -157,7 +159,6 @@ __device__ __forceinline__ unsigned pack_flags(const float (&d)[4][SLOTS])
 #define ALADDIN_SCORE_MINB 5
 #endif
 constexpr int CHUNK = 256;                   // candidates per staged chunk
-constexpr long long WAIT_LIMIT = 1ll << 26;  // mbarrier polls before giving up
 constexpr unsigned ERR_TIMEOUT_BIT = 4u;
 
 __device__ __forceinline__ unsigned smem_addr(const void* p)
@@ -186,10 +187,11 @@ __device__ __forceinline__ void tma_load(void* dst, const void* src, unsigned by
         : "memory");
 }
 
-// Bounded wait for the phase with the given parity; false if the limit ran out.
-__device__ __forceinline__ bool mbar_wait(unsigned long long* bar, unsigned parity)
+// Bounded wait for the phase with the given parity; false if `limit` polls
+// ran out.
+__device__ __forceinline__ bool mbar_wait(unsigned long long* bar, unsigned parity, long long limit)
 {
-    for (long long it = 0; it < WAIT_LIMIT; ++it) {
+    for (long long it = 0; it < limit; ++it) {
         unsigned done;
         asm volatile(
             "{\n .reg .pred p;\n mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n selp.u32 %0, 1, 0, p;\n}"
@@ -210,6 +212,8 @@ struct VecArgs {
     unsigned int* best;
     int tiles;       // worker tiles of SCORE_WARPS * 32 * SLOTS
     int per_tile;    // CTAs per tile
+    long long wait_limit;  // mbarrier polls before a wait gives up
+    int withhold;    // test hook, 1: the first chunk's copy is not issued (its wait runs out)
 };
 
 struct __align__(16) ScoreSmem {
@@ -298,7 +302,7 @@ __global__ void __launch_bounds__(SCORE_WARPS * 32, PEND ? 3 : ALADDIN_SCORE_MIN
         sm.stop = 0;
     }
     __syncthreads();
-    if (tid == 0) {
+    if (tid == 0 && !A.withhold) {
         const int n0 = min(CHUNK, ce - cb);
         tma_load(sm.cs[0], A.cand + (size_t)cb * REC_F4, (unsigned)n0 * (REC_F4 * 16u), &sm.bar[0]);
     }
@@ -329,13 +333,16 @@ __global__ void __launch_bounds__(SCORE_WARPS * 32, PEND ? 3 : ALADDIN_SCORE_MIN
             tma_load(sm.cs[buf ^ 1], A.cand + (size_t)c1 * REC_F4, (unsigned)n1 * (REC_F4 * 16u),
                      &sm.bar[buf ^ 1]);
         }
-        if (!mbar_wait(&sm.bar[buf], (unsigned)((k >> 1) & 1))) {
+        if (!mbar_wait(&sm.bar[buf], (unsigned)((k >> 1) & 1), A.wait_limit)) {
             if (lane == 0) atomicOr(A.C.err, ERR_TIMEOUT_BIT);
             sm.stop = 1;
         }
         __syncthreads();
         if (sm.stop) {
-            if (tid == 0 && k + 1 < nchunks) mbar_wait(&sm.bar[buf ^ 1], (unsigned)(((k + 1) >> 1) & 1));
+            // the copy into the other buffer is in flight: let it land first
+            // (with the full limit whatever the cluster's test setting)
+            if (tid == 0 && k + 1 < nchunks)
+                mbar_wait(&sm.bar[buf ^ 1], (unsigned)(((k + 1) >> 1) & 1), MBAR_WAIT_POLLS);
             return;
         }
         const float4* cs = sm.cs[buf];
@@ -586,6 +593,8 @@ static cudaError_t launch_vec(const ScoreArgs& A0, cudaStream_t st)
     A.margin = A0.margin;
     A.best = A0.best;
     A.tiles = (A.C.W + SCORE_WARPS * 32 * SLOTS - 1) / (SCORE_WARPS * 32 * SLOTS);
+    A.wait_limit = A0.wait_limit;
+    A.withhold = A0.withhold;
     const size_t smem = sizeof(ScoreSmem);
     DevInfo d;
     cudaError_t e = device_info(&d);
@@ -778,6 +787,8 @@ cudaError_t launch_score(const DevParams& P, const ClusterDev& C, int n, const i
         A.chunks = (n + SCORE_CHUNK - 1) / SCORE_CHUNK;
         A.tiles = 0;
         A.approx = P.approx;
+        A.wait_limit = P.mbar_wait_limit;
+        A.withhold = P.wait_test;
         if (ev0) cudaEventRecord(ev0, st);
         const bool vec = (C.W % 4 == 0) && (((uintptr_t)flags & 3) == 0) &&
                          (((uintptr_t)margin & 15) == 0);
