@@ -35,12 +35,15 @@ struct ScoreBuffers {
 // K3 pipeline: validate + derive + counting-sort candidates by predicted
 // output, score every pair, finalize argbest. Device pointers only. With
 // prepared, the candidates were sorted into B by launch_cand_prep already
-// (its stream ordered before st by the caller).
+// (its stream ordered before st by the caller). With ranked (C.order), the
+// flags and margins are written in rank order: column k of a row is worker
+// ranked[k] (argbest unaffected).
 cudaError_t launch_score(const DevParams& P, const ClusterDev& C, int n_cand, const int32_t* in,
                          const int32_t* pred, const float* wait, uint8_t* flags, float* margin,
                          int32_t* argbest, int64_t* kv_peak, float* t_cand, const ScoreBuffers& B,
                          bool pend, cudaStream_t st, cudaEvent_t ev0 = nullptr,
-                         cudaEvent_t ev1 = nullptr, bool prepared = false);
+                         cudaEvent_t ev1 = nullptr, bool prepared = false,
+                         const int32_t* ranked = nullptr, int ld = 0);
 // The candidate preparation of launch_score alone (it reads no table): the
 // validated per-candidate records sorted by predicted output, and the
 // argbest keys reset. W is the cluster's worker count (output row stride).
@@ -84,6 +87,11 @@ struct RoundIO {
     // host routing only: never the multi-CTA (cooperative) sliced round, for
     // simulations that run side by side with others
     int single_cta;
+    // direct mode: device pointer to the first candidate still to place (the
+    // ones before it were placed by the incremental round), or nullptr (0)
+    const int* c_first;
+    // direct mode: some worker holds requests placed earlier in the open round
+    int round_open;
 };
 constexpr int ROUND_XBUF_SMS = 1024;  // largest SM count the exchange buffer serves
 constexpr size_t ROUND_XBUF_BYTES = 32 * (size_t)ROUND_XBUF_SMS + 16;
@@ -94,6 +102,25 @@ cudaError_t launch_round(const DevParams& P, const ClusterDev& C, const RoundIO&
 // plain single-CTA round, -1 none (a single-CTA request beyond what one CTA
 // holds at 1,024 slots, or a failed device query).
 int round_ctas(int W, int cap, int K, bool single_cta);
+
+// Scratch of the incremental round (grow-only, owned by the cluster).
+struct RoundIncBuffers {
+    uint8_t* flags;        // [chunk][(W + 31) & ~31] rank-order flags of the round-start state
+    void* rank;            // [W] 16-byte rank entries
+    int* c_stop;           // one int
+    ScoreBuffers score;    // candidate preparation of the pre-scoring (chunk candidates)
+};
+// Bytes of the incremental round's flag buffer for n_cand candidates (0: the
+// incremental round does not apply and needs nothing).
+size_t round_inc_flag_bytes(const DevParams& P, const ClusterDev& C, const RoundIO& io);
+// K4, incremental (direct-mode best-fit rounds of one scheduling group): every
+// candidate scored against the round-start state, then a single-CTA chain
+// that re-scores only the workers it modified; the sliced round finishes any
+// candidates left when the modified workers outgrow shared memory. *used =
+// false: not applicable (trace mode, several groups, the wait test hook),
+// nothing launched.
+cudaError_t launch_round_inc(const DevParams& P, const ClusterDev& C, const RoundIO& io,
+                             const RoundIncBuffers& B, cudaStream_t st, bool* used);
 
 // Attributes of the current device that launches size themselves by, read
 // once per device and cached (thread-safe).

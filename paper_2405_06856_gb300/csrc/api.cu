@@ -210,6 +210,7 @@ struct aladdin_cluster {
     DevBuf sorted, hist, best;
     DevBuf s_in, s_pred, s_wait, s_flags, s_margin, s_arg, s_kv, s_tc, s_place;
     DevBuf s_off, s_rin, s_rgen, s_rpred, s_rtdec;
+    DevBuf r_flags, r_rank, r_stop;  // incremental placement round
     unsigned long long* d_stats = nullptr;
     int* d_status = nullptr;
     void* d_xround = nullptr;  // exchange buffer of the sliced placement round
@@ -795,7 +796,27 @@ try {
         CK(launch_round_groups(cl->dp, cl->dev, io, cl->st));
         CK(launch_rank(cl->dev, cl->st));
     } else if (cl->hp.policy == ALADDIN_POLICY_BESTFIT) {
-        CK(launch_round(cl->dp, cl->dev, io, cl->st));
+        // incremental round where it applies, the sliced round otherwise
+        io.round_open = cl->round_open ? 1 : 0;
+        bool used = false;
+        const size_t fbytes = round_inc_flag_bytes(cl->dp, cl->dev, io);
+        if (fbytes > 0) {
+            const size_t chunk = fbytes / (size_t)((cl->W + 31) & ~31);
+            CK(cl->r_flags.ensure(fbytes));
+            CK(cl->r_rank.ensure(16 * (size_t)cl->W));
+            CK(cl->r_stop.ensure(sizeof(int)));
+            CK(cl->sorted.ensure(sizeof(float4) * CAND_REC_F4 * chunk));
+            CK(cl->hist.ensure(sizeof(int32_t) * ((size_t)cl->hp.K + 2)));
+            CK(cl->best.ensure(sizeof(unsigned int) * chunk));
+            RoundIncBuffers rb;
+            rb.flags = cl->r_flags.as<uint8_t>();
+            rb.rank = cl->r_rank.p;
+            rb.c_stop = cl->r_stop.as<int>();
+            rb.score = ScoreBuffers{cl->sorted.as<float4>(), cl->hist.as<int32_t>(),
+                                    cl->best.as<unsigned int>()};
+            CK(launch_round_inc(cl->dp, cl->dev, io, rb, cl->st, &used));
+        }
+        if (!used) CK(launch_round(cl->dp, cl->dev, io, cl->st));
         CK(launch_rank(cl->dev, cl->st));
     } else {
         // JSQ / power of two: no table is read while placing; every worker's

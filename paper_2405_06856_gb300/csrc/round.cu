@@ -10,7 +10,7 @@
 // requests followed by the heartbeat's arrivals; unplaced requests that can
 // still meet their TTFT stay in the waiting list, the others fail (on a
 // decode instance every unplaced request fails).
-#include "aladdin_host.h"
+#include "round_common.cuh"
 
 namespace aladdin {
 
@@ -42,12 +42,13 @@ __global__ void __launch_bounds__(ROUND_THREADS) k_round(DevParams P, ClusterDev
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
     const int n_wait0 = io.sim ? *io.n_wait : 0;
     const int n_cand = io.sim ? n_wait0 + (int)(io.arr_end - io.arr_begin) : io.n_cand;
+    const int c_begin = (!io.sim && io.c_first) ? *io.c_first : 0;
     int keep = 0;  // thread 0: new waiting-list length
-    if (tid == 0) sm.stop = (io.sim && *io.status != 0) ? 1 : 0;
+    if (tid == 0) sm.stop = ((io.sim && *io.status != 0) || c_begin >= n_cand) ? 1 : 0;
     __syncthreads();
     if (sm.stop) return;
 
-    for (int c = 0; c < n_cand; ++c) {
+    for (int c = c_begin; c < n_cand; ++c) {
         long long tix = 0;
         int32_t a, r, rl;
         double wd;
@@ -185,20 +186,6 @@ __global__ void __launch_bounds__(ROUND_THREADS) k_round(DevParams P, ClusterDev
 // registers within the 128 a thread of a 512-thread CTA has.
 constexpr int R2_THREADS = 512;
 constexpr int R2_WARPS = R2_THREADS / 32;
-template <int E>
-struct R2Split {
-    // up to 256 slots: NW warps cover the capacity with one element a lane;
-    // larger tables: 12 warps (4 left for evaluation) with up to E/8
-    // elements a lane, the build sized to the worker's count
-    static constexpr int NW = E <= 8 ? E : 12;
-    static constexpr int EW = E <= 8 ? 1 : E / 8;
-};
-// Breakpoint rows of a worker in shared memory are 16-bit; rc (a multiple of
-// 8) plus this pad makes the per-worker stride an odd number of 32-bit words,
-// so that lanes searching neighbouring workers start on different banks.
-constexpr int R2_RHO_PAD = 2;
-constexpr int NONE = 0x7fffffff;
-
 struct R2Args {
     DevParams P;
     ClusterDev C;
@@ -233,65 +220,6 @@ __device__ __forceinline__ unsigned ld_acquire(const unsigned* p)
     return v;
 }
 
-// Row of remaining length r: the first row q whose rho_{q+1} exceeds r (row R
-// is unbounded). Shared memory holds rho_{q+1} - 1 for the first rc rows; a
-// worker with more rows continues in the table's global rows.
-__device__ __forceinline__ int r2_find(const unsigned short* rho, int R, int rc, int r,
-                                       const float4* tab, long long rowbase)
-{
-    const int Rs = R < rc ? R : rc;
-    int lo = 0, hi = Rs;
-    while (lo < hi) {
-        const int mid = (lo + hi) >> 1;
-        if ((int)rho[mid] >= r) hi = mid;
-        else lo = mid + 1;
-    }
-    if (lo == Rs && R > Rs) {
-        hi = R;
-        while (lo < hi) {
-            const int mid = (lo + hi) >> 1;
-            if (__float_as_int(tab[(rowbase + mid) * ROW_F4].x) > r) hi = mid;
-            else lo = mid + 1;
-        }
-    }
-    return lo;
-}
-
-// better() carrying the winner's "worker full" flag along.
-__device__ __forceinline__ void better_f(unsigned long long& bk, int& bw, int& bf,
-                                         unsigned long long ok, int ow, int of)
-{
-    if (ow != NONE && (bw == NONE || ok > bk || (ok == bk && ow < bw))) {
-        bk = ok;
-        bw = ow;
-        bf = of;
-    }
-}
-
-// Warp-wide best_f: the largest key, then the lowest worker index among equal
-// keys (warp max/min reductions on the key's halves); every lane ends with it.
-__device__ __forceinline__ void reduce_f(unsigned long long& bk, int& bw, int& bf)
-{
-    const bool has = bw != NONE;
-    const unsigned hi = has ? (unsigned)(bk >> 32) : 0u;
-    const unsigned lo = has ? (unsigned)bk : 0u;
-    const unsigned mhi = __reduce_max_sync(FULL, hi);
-    const unsigned mlo = __reduce_max_sync(FULL, hi == mhi ? lo : 0u);
-    const bool top = has && hi == mhi && lo == mlo;
-    const unsigned widx = __reduce_min_sync(FULL, top ? (unsigned)bw : 0xffffffffu);
-    const unsigned who = __ballot_sync(FULL, top && (unsigned)bw == widx);
-    const int of = __shfl_sync(FULL, bf, who ? __ffs(who) - 1 : 0);
-    if (who) {
-        bk = ((unsigned long long)mhi << 32) | mlo;
-        bw = (int)widx;
-        bf = of;
-    } else {
-        bk = 0ull;
-        bw = NONE;
-        bf = 0;
-    }
-}
-
 template <int E>
 __global__ void __launch_bounds__(R2_THREADS, 1) k_round2(R2Args A)
 {
@@ -312,6 +240,10 @@ __global__ void __launch_bounds__(R2_THREADS, 1) k_round2(R2Args A)
     const ClusterDev& C = A.C;
     const RoundIO& io = A.io;
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    // direct mode after the incremental round: the candidates before c_begin
+    // are placed already (every CTA reads the same value)
+    const int c_begin = (!io.sim && io.c_first) ? *io.c_first : 0;
+    if (!io.sim && c_begin >= io.n_cand) return;
     const int g = blockIdx.x;
     const int w_lo = g * A.slice;
     const int nloc = max(0, min(C.W, w_lo + A.slice) - w_lo);
@@ -388,7 +320,7 @@ __global__ void __launch_bounds__(R2_THREADS, 1) k_round2(R2Args A)
                                                   cand);
     };
 
-    for (int c = 0; c < n_cand; ++c) {
+    for (int c = c_begin; c < n_cand; ++c) {
         const int par = c & 1;
         long long tix = 0;
         int32_t a, r, rl;
@@ -456,7 +388,8 @@ __global__ void __launch_bounds__(R2_THREADS, 1) k_round2(R2Args A)
                 }
                 // every lane acquires the counter, so its loads below see the
                 // other CTAs' entries
-                const unsigned target = (unsigned)(c + 1) * (unsigned)A.G + (unsigned)P.wait_test;
+                const unsigned target =
+                    (unsigned)(c - c_begin + 1) * (unsigned)A.G + (unsigned)P.wait_test;
                 bool ok = false;
                 for (long long it = 0; it < P.grid_wait_limit; ++it) {
                     if (ld_acquire(A.arrive) >= target) {

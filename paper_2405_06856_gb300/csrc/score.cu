@@ -89,6 +89,8 @@ struct ScoreArgs {
     int approx;  // approximate-mode constraints (b) and (d)
     long long wait_limit;  // mbarrier polls before a wait gives up
     int withhold;          // test hook: the first candidate copy is not issued
+    const int32_t* order;  // nullptr, or rank order: output column k is worker order[k]
+    int ld;                // output row stride (elements)
 };
 
 __global__ void k_cand_scatter(DevParams P, int n, int W, const int32_t* __restrict__ in,
@@ -214,6 +216,7 @@ struct VecArgs {
     int per_tile;    // CTAs per tile
     long long wait_limit;  // mbarrier polls before a wait gives up
     int withhold;    // test hook, 1: the first chunk's copy is not issued (its wait runs out)
+    const int32_t* order;  // nullptr, or rank order: output column k is worker order[k]
 };
 
 struct __align__(16) ScoreSmem {
@@ -351,7 +354,7 @@ __global__ void __launch_bounds__(SCORE_WARPS * 32, PEND ? 3 : ALADDIN_SCORE_MIN
                 const int r_first = __float_as_int(cs[2].x);
 #pragma unroll
                 for (int s = 0; s < SLOTS; ++s) {
-                    wk[s] = live ? w0 + s : W - 1;
+                    wk[s] = live ? (A.order ? __ldg(&A.order[w0 + s]) : w0 + s) : W - 1;
                     const long long rb = (long long)wk[s] * A.C.rows;
                     p[s] = find_row(A.C.tab, rb, __ldg(&A.C.R[wk[s]]), r_first);
                     const long long pn = rb + min(p[s] + 1, last_row);
@@ -533,9 +536,9 @@ __global__ void __launch_bounds__(SCORE_WARPS * 32) k_score_scalar(ScoreArgs A)
     if (unit >= A.tiles * A.chunks) return;
     const int tile = unit % A.tiles, chunk = unit / A.tiles;
     const int W = A.C.W;
-    const int w = tile * 32 + lane;
+    const int w = tile * 32 + lane;  // output column
     const bool live = w < W;
-    const int wc = live ? w : W - 1;
+    const int wc = live ? (A.order ? __ldg(&A.order[w]) : w) : W - 1;  // its worker
     const int c0 = chunk * SCORE_CHUNK;
     const int c1 = min(c0 + SCORE_CHUNK, A.n_cand);
     const long long rb = (long long)wc * A.C.rows;
@@ -555,7 +558,7 @@ __global__ void __launch_bounds__(SCORE_WARPS * 32) k_score_scalar(ScoreArgs A)
         cr.inv_d1 = q1.x; cr.nXd1 = q1.y; cr.inv_d2 = q1.z; cr.Zc = q1.w;
         cr.ri = __float_as_int(q2.x);
         cr.orig = __float_as_int(q2.y);
-        const size_t off = (size_t)cr.orig * (size_t)W + (size_t)w;
+        const size_t off = (size_t)cr.orig * (size_t)A.ld + (size_t)w;
         if (cr.ri == 0) {
             if (live) {
                 if (SF) A.flags[off] = 0x80;
@@ -595,6 +598,7 @@ static cudaError_t launch_vec(const ScoreArgs& A0, cudaStream_t st)
     A.tiles = (A.C.W + SCORE_WARPS * 32 * SLOTS - 1) / (SCORE_WARPS * 32 * SLOTS);
     A.wait_limit = A0.wait_limit;
     A.withhold = A0.withhold;
+    A.order = A0.order;
     const size_t smem = sizeof(ScoreSmem);
     DevInfo d;
     cudaError_t e = device_info(&d);
@@ -767,14 +771,15 @@ cudaError_t launch_score(const DevParams& P, const ClusterDev& C, int n, const i
                          const int32_t* pred, const float* wait, uint8_t* flags, float* margin,
                          int32_t* argbest, int64_t* kv_peak, float* t_cand, const ScoreBuffers& B,
                          bool pend, cudaStream_t st, cudaEvent_t ev0, cudaEvent_t ev1,
-                         bool prepared)
+                         bool prepared, const int32_t* ranked, int ld)
 {
     if (n <= 0) return cudaSuccess;
     cudaError_t e;
     const int tb = 256, nb = (n + tb - 1) / tb;
     const bool need_score = flags || margin || argbest;
+    const int row = ld > 0 ? ld : C.W;  // output row stride
     if (need_score) {
-        if (!prepared && (e = launch_cand_prep(P, C.W, n, in, pred, wait, B, st)) != cudaSuccess)
+        if (!prepared && (e = launch_cand_prep(P, row, n, in, pred, wait, B, st)) != cudaSuccess)
             return e;
 
         ScoreArgs A;
@@ -789,8 +794,10 @@ cudaError_t launch_score(const DevParams& P, const ClusterDev& C, int n, const i
         A.approx = P.approx;
         A.wait_limit = P.mbar_wait_limit;
         A.withhold = P.wait_test;
+        A.order = ranked;
+        A.ld = row;
         if (ev0) cudaEventRecord(ev0, st);
-        const bool vec = (C.W % 4 == 0) && (((uintptr_t)flags & 3) == 0) &&
+        const bool vec = (C.W % 4 == 0) && (row % 4 == 0) && (((uintptr_t)flags & 3) == 0) &&
                          (((uintptr_t)margin & 15) == 0);
         const bool sf = flags != nullptr, smg = margin != nullptr, arg = argbest != nullptr;
         if (vec) {
