@@ -417,7 +417,7 @@ struct BuildSmem {
     long long pll[6][NW];             // per-warp partials
     double pdm[NW];
     float pf[7][NW];
-    int pi[3][NW];
+    int pi[5][NW];
     unsigned cflag;
     uint8_t pend[N];
 };
@@ -434,20 +434,49 @@ __device__ __forceinline__ void group_sync()
     }
 }
 
+// Lanes of the smallest power of two >= NW.
+template <int NW>
+constexpr int lanes_p2()
+{
+    return NW <= 1 ? 1 : NW <= 2 ? 2 : NW <= 4 ? 4 : NW <= 8 ? 8 : NW <= 16 ? 16 : 32;
+}
+
 // Cross-warp combination of per-warp scan totals: the carry into warp q
 // (op over warps before q for a prefix, after q for a suffix) and the total.
+// Lane k < NW of every warp reads warp k's partial; a shuffle scan over those
+// lanes gives every lane the carries and the total (log2 NW steps, the same
+// exact min / max / integer results as a sequential fold).
 template <int NW, typename T, typename Op>
 __device__ __forceinline__ T carry_in(const T* part, int q, bool suffix, Op op, T ident, T& all)
 {
-    T c = ident;
-    all = ident;
+    const int lane = threadIdx.x & 31;
+    T incl = lane < NW ? part[lane] : ident;
 #pragma unroll
-    for (int k = 0; k < NW; ++k) {
-        const T t = part[k];
-        if (suffix ? k > q : k < q) c = op(c, t);
-        all = op(all, t);
+    for (int d = 1; d < lanes_p2<NW>(); d <<= 1) {
+        if (!suffix) {
+            const T u = __shfl_up_sync(FULL, incl, d);
+            if (lane >= d) incl = op(u, incl);
+        } else {
+            const T u = __shfl_down_sync(FULL, incl, d);
+            if (lane + d < 32) incl = op(incl, u);
+        }
     }
-    return c;
+    all = __shfl_sync(FULL, incl, suffix ? 0 : NW - 1);
+    const int src = suffix ? q + 1 : q - 1;  // inclusive value of the neighbour
+    const T c = __shfl_sync(FULL, incl, src >= 0 && src < NW ? src : 0);
+    return src >= 0 && src < NW ? c : ident;
+}
+
+// Combination over the NW warps of a value every warp holds (lane k reads
+// warp k's entry; xor reduction over the lanes).
+template <int NW, typename T, typename Op>
+__device__ __forceinline__ T combine_warps(const T* part, Op op, T ident)
+{
+    const int lane = threadIdx.x & 31;
+    T v = lane < NW ? part[lane] : ident;
+#pragma unroll
+    for (int d = lanes_p2<NW>() / 2; d > 0; d >>= 1) v = op(v, __shfl_xor_sync(FULL, v, d));
+    return __shfl_sync(FULL, v, 0);  // lanes past the reduced ones get it too
 }
 
 template <int NW, typename Set>
@@ -660,22 +689,12 @@ __device__ unsigned build_table(const DevParams& P, const ClusterDev& C, int w,
     }
     group_sync<NW>();
     if constexpr (NW > 1) {
-        sumP = 0;
-        sumIn = 0;
-        sumPred = 0;
-        wpmax = -f_inf();
-        npend = 0;
-        bad = 0;
-#pragma unroll
-        for (int k = 0; k < NW; ++k) {
-            sumP += sm.pll[0][k];
-            sumIn += sm.pll[1][k];
-            sumPred += sm.pll[2][k];
-            const float o3 = sm.pf[0][k];
-            wpmax = wpmax > o3 ? wpmax : o3;
-            npend += sm.pi[0][k];
-            bad |= sm.pi[1][k];
-        }
+        sumP = combine_warps<NW>(sm.pll[0], OpAdd<long long>(), 0LL);
+        sumIn = combine_warps<NW>(sm.pll[1], OpAdd<long long>(), 0LL);
+        sumPred = combine_warps<NW>(sm.pll[2], OpAdd<long long>(), 0LL);
+        wpmax = combine_warps<NW>(sm.pf[0], OpMax<float>(), -f_inf());
+        npend = combine_warps<NW>(sm.pi[0], OpAdd<int>(), 0);
+        bad = combine_warps<NW>(sm.pi[1], OpMax<int>(), 0);
     }
     // Approximate mode: prompt bounds of (d) (stall within the smallest
     // theta-scaled saved decode time) and of (b) (weighted context within
@@ -697,8 +716,7 @@ __device__ unsigned build_table(const DevParams& P, const ClusterDev& C, int w,
         if constexpr (NW > 1) {
             if (lane == 0) sm.pdm[q] = dmin;
             group_sync<NW>();
-#pragma unroll
-            for (int k = 0; k < NW; ++k) dmin = fmin(dmin, sm.pdm[k]);
+            dmin = combine_warps<NW>(sm.pdm, OpMin<double>(), dmin);
         }
         const double s_d = C.scaled[w];
         if (P.decode) {
@@ -715,8 +733,12 @@ __device__ unsigned build_table(const DevParams& P, const ClusterDev& C, int w,
     // invalid request): capacity_norm^2 is exact (integer and half-integer
     // terms below 2^53) and non-negative doubles order like their bit
     // patterns; with gamma = 1/2 the same order comes from integers.
+    // Row 0, the record and the key are written by the last lane of the last
+    // warp, which holds the highest elements (often padding) and so has the
+    // fewest rows of its own to write.
+    const bool row0_lane = q == NW - 1 && lane == 31;
     unsigned long long kq = 0ull;
-    if (q == 0 && lane == 0 && !bad) {
+    if (row0_lane && !bad) {
         if (P.gammad == 0.5) {
             // 4 capacity_norm^2 = (2B)^2 + (2 sum in + sum pred)^2 in integers
             // (the same order and ties as the exact double value)
@@ -746,11 +768,26 @@ __device__ unsigned build_table(const DevParams& P, const ClusterDev& C, int w,
         }
         group_sync<NW>();
         const unsigned knew = sm.cflag;
-        int lo = 0, hi = n - 1;  // old keys below knew (keys are distinct)
-        while (lo < hi) {
-            const int mid = (lo + hi) >> 1;
-            if (sm.runs[mid] < knew) lo = mid + 1;
-            else hi = mid;
+        int lo;  // old keys below knew (keys are distinct)
+        if constexpr (E == 1) {
+            // one key a thread: the count of old keys below knew is a
+            // barrier reduction over the group
+            const unsigned below = (x0 + lane < n - 1 && l_sk[0] < knew) ? 1u : 0u;
+            unsigned cnt;
+            asm volatile("{\n .reg .pred p;\n setp.ne.u32 p, %2, 0;\n"
+                         " bar.red.popc.u32 %0, 1, %1, p;\n}"
+                         : "=r"(cnt)
+                         : "r"(NW * 32), "r"(below)
+                         : "memory");
+            lo = (int)cnt;
+        } else {
+            int hi = n - 1;
+            lo = 0;
+            while (lo < hi) {
+                const int mid = (lo + hi) >> 1;
+                if (sm.runs[mid] < knew) lo = mid + 1;
+                else hi = mid;
+            }
         }
 #pragma unroll
         for (int e = 0; e < E; ++e) {
@@ -901,35 +938,38 @@ __device__ unsigned build_table(const DevParams& P, const ClusterDev& C, int w,
     if constexpr (NW > 1) r0 = n > 0 ? (int)(sm.sorted[0] >> 10) : 0x7fffffff;
     else r0 = __shfl_sync(FULL, r[0], 0);
     // Prefix sums over the sorted order.
+    // (r and a are at most K <= 65536 and a table holds at most 1,024
+    // requests, so their sums fit 32 bits; the r a sums need 64)
     int rowid[E];
-    long long pre_r[E], pre_ra[E], pre_a[E];
+    int pre_r[E], pre_a[E];
+    long long pre_ra[E];
 #pragma unroll
     for (int e = 0; e < E; ++e) {
         const bool valid = x0 + e * 32 + lane < n;
         rowid[e] = first[e];
         const long long rr = valid ? (long long)r[e] : 0;
         const long long aa = valid ? (long long)a[e] : 0;
-        pre_r[e] = rr;
+        pre_r[e] = (int)rr;
         pre_ra[e] = rr * aa + rr * (rr + 1) / 2;
-        pre_a[e] = aa;
+        pre_a[e] = (int)aa;
     }
     auto s_row = scan_set(rowid, OpAdd<int>(), 0);
-    auto s_r = scan_set(pre_r, OpAdd<long long>(), 0LL);
+    auto s_r = scan_set(pre_r, OpAdd<int>(), 0);
     auto s_ra = scan_set(pre_ra, OpAdd<long long>(), 0LL);
-    auto s_a = scan_set(pre_a, OpAdd<long long>(), 0LL);
+    auto s_a = scan_set(pre_a, OpAdd<int>(), 0);
     scan_prefix_fused(s_row, s_r, s_ra, s_a);
     if constexpr (NW > 1) {
         if (lane == 0) {
             sm.pi[2][q] = s_row.total;
-            sm.pll[3][q] = s_r.total;
+            sm.pi[3][q] = s_r.total;
             sm.pll[4][q] = s_ra.total;
-            sm.pll[5][q] = s_a.total;
+            sm.pi[4][q] = s_a.total;
         }
         group_sync<NW>();
         add_carry_prefix<NW>(s_row, sm.pi[2], q);
-        add_carry_prefix<NW>(s_r, sm.pll[3], q);
+        add_carry_prefix<NW>(s_r, sm.pi[3], q);
         add_carry_prefix<NW>(s_ra, sm.pll[4], q);
-        add_carry_prefix<NW>(s_a, sm.pll[5], q);
+        add_carry_prefix<NW>(s_a, sm.pi[4], q);
     }
     const int R = s_row.total;
     const long long tot_a = s_a.total;
@@ -1053,7 +1093,7 @@ __device__ unsigned build_table(const DevParams& P, const ClusterDev& C, int w,
             }
         }
     }
-    if (q == 0 && lane == 0) {
+    if (row0_lane) {
         RowVals o;
         if (!bad) {
             o = make_row(P, inv_s, M, sumP, 0, n > 0 ? r0 : 0x7fffffff, n, tot_a, 0, 0, LL_NONE,

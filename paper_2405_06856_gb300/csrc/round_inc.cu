@@ -36,6 +36,18 @@ constexpr int RI_MAX_SLOTS = 2048; // modified workers held in shared memory, at
 constexpr int RI_RC_MAX = 256;     // breakpoint rows a modified worker keeps in shared memory
 constexpr size_t RI_FLAGS_MAX = (size_t)512 << 20;  // bytes of rank-order flags a chunk holds
 
+// The rebuild group of the winner's table: tables of up to 256 slots, one
+// warp per 32 slots; larger tables, RI_NW_BIG warps with the build sized to
+// the worker's count (EW elements a lane cover the capacity).
+#ifndef ALADDIN_RI_NW_BIG
+#define ALADDIN_RI_NW_BIG 12
+#endif
+template <int E>
+struct RISplit {
+    static constexpr int NW = E <= 8 ? E : ALADDIN_RI_NW_BIG;
+    static constexpr int EW = E <= 8 ? 1 : (E + NW - 1) / NW <= 2 ? 2 : 4;
+};
+
 // Round-start entry of a rank position: the worker there, its key and count.
 struct __align__(16) RankEnt {
     unsigned long long key;
@@ -58,7 +70,7 @@ struct RIArgs {
 
 template <int E>
 struct RISmem {
-    BuildSmem<R2Split<E>::EW, R2Split<E>::NW> build;
+    BuildSmem<RISplit<E>::EW, RISplit<E>::NW> build;
     unsigned long long bk[2][RI_WARPS];
     int bw[2][RI_WARPS];
     int bf[2][RI_WARPS];
@@ -100,7 +112,8 @@ __device__ __forceinline__ unsigned feasible_bits(const uint8_t* row, int k)
 template <int E>
 __global__ void __launch_bounds__(RI_THREADS, 1) k_round_inc(RIArgs A)
 {
-    constexpr int NW = R2Split<E>::NW, EW = R2Split<E>::EW;
+    constexpr int NW = RISplit<E>::NW, EW = RISplit<E>::EW;
+    static_assert(NW * EW * 32 >= E * 32 && NW <= 12, "the rebuild group covers the capacity");
     constexpr bool NW_INSERT = NW > 1;
     extern __shared__ __align__(16) unsigned char smraw[];
     RISmem<E>& sm = *reinterpret_cast<RISmem<E>*>(smraw);
