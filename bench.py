@@ -556,6 +556,7 @@ def run_ours(args):
     mixed = mixed_mask(A, synth, dev, stream, flush)
     pol = policy_compare(A, synth, stream, 20_000, [1, 2])
     wmod = worker_model(A, synth, stream, fit_n=0)
+    search = min_workers_1m(A, synth, stream) if args.search else None
 
     peak, peak_kind = read_peaks()
     kern_avg = kern_ms / max(kern_n, 1)
@@ -590,6 +591,7 @@ def run_ours(args):
             "mixed_mask": mixed,
             "policies": pol,
             "worker_config": wmod,
+            "min_workers_1m": search,
             "clocks": clocks}
     if cpu is not None:
         line["cpu_baseline"] = cpu
@@ -911,6 +913,65 @@ def run_min_workers(args):
                       "total_gpus": int(total), "wall_s": wall}))
 
 
+def min_workers_1m(A, synth, stream):
+    """The minimum-worker search on the 1,000,000-request diurnal trace (Sec.
+    6.4's large-scale simulation): per worker option the fewest workers that
+    serve every request within its SLOs, the fewest GPUs over the options,
+    and the search's wall time."""
+    import torch
+    tr, gpus, kv, scale = min_workers_config(synth)
+    got = np.zeros(len(gpus), np.int32)
+    torch.cuda.synchronize()
+    t0 = time.perf_counter()
+    best, total = A.aladdin_min_workers(A.make_params(dict(synth.BASE_PARAMS), MW_B_CAP),
+                                        A.make_cfgs(gpus, kv, scale),
+                                        A.make_trace(tr.t_arr, tr.req_in, tr.req_pred), 100.0,
+                                        4096, got, stream=stream)
+    wall = time.perf_counter() - t0
+    return {"workload": "diurnal Poisson trace of %d requests over %.0f s (peak 2,000 req/s, "
+                        "peak:trough 4:1), %d KV tokens per GPU, latency x 1/sqrt(GPUs), %d request "
+                        "slots a worker, heartbeat 100 ms" % (len(tr.t_arr), tr.t_arr[-1] / 1000.0,
+                                                              MW_KV_PER_GPU, MW_B_CAP),
+            "gpus_per_worker": list(gpus), "min_workers": got.tolist(),
+            "gpus_per_option": [int(g * n) if n > 0 else None for g, n in zip(gpus, got.tolist())],
+            "best_gpus_per_worker": int(gpus[best]), "total_gpus": int(total), "wall_s": wall}
+
+
+def run_aux(args):
+    """Small runs of the auxiliary kernels, each warm-up + steps times on the
+    256-worker workload: a grouped best-fit round (k_round_grp, 7 groups), a
+    JSQ round (k_round_queue), the 100 ms execution step (k_advance) and
+    Algorithm 2's re-balancing of a round (k_rebalance). The command the
+    profiles of those kernels capture."""
+    import torch
+    from paper_2405_06856_gb300 import build as B
+    B.build()
+    from paper_2405_06856_gb300 import aladdin as A
+    from paper_2405_06856_gb300 import synth
+    torch.cuda.set_device(0)
+    stream = torch.cuda.current_stream().cuda_stream
+    rng = np.random.default_rng(5)
+    out = {}
+    for _ in range(args.warmup + args.steps):
+        for name, over in (("grouped", dict(groups=7)), ("jsq", dict(policy=A.POLICY_JSQ)),
+                           ("bestfit", {})):
+            w2 = synth.config("w256", b_cap=128, params=over)
+            with A.Cluster.from_workload(w2, stream=stream) as cl:
+                t0 = time.perf_counter()
+                pl = cl.place_round(w2.cand_in, w2.cand_pred, w2.cand_wait)
+                out.setdefault(name + "_round_ms", []).append((time.perf_counter() - t0) * 1e3)
+                if name == "bestfit":
+                    le = rng.integers(-4000, 4000, w2.n_workers)
+                    be = rng.integers(-8, 8, w2.n_workers)
+                    t0 = time.perf_counter()
+                    cl.rebalance(w2.cand_in, w2.cand_pred, w2.cand_wait, pl, le, be)
+                    out.setdefault("rebalance_ms", []).append((time.perf_counter() - t0) * 1e3)
+                t0 = time.perf_counter()
+                cl.advance(100.0)
+                out.setdefault(name + "_advance_ms", []).append((time.perf_counter() - t0) * 1e3)
+    print(json.dumps({"mode": "aux", **{k: round(min(v), 3) for k, v in out.items()}}))
+
+
 def run_kernel_only(args):
     """The device-resident step only (warm-up + steps), nothing else: the
     command profiled by ncu."""
@@ -1020,8 +1081,11 @@ def main():
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--no-cpu-baseline", dest="cpu_baseline", action="store_false")
+    ap.add_argument("--no-search", dest="search", action="store_false",
+                    help="leave the 1,000,000-request minimum-worker search (about 95 s) out")
     ap.add_argument("--mode", default="full",
-                    choices=["full", "kernel", "round", "sim", "minworkers", "policies", "configs"],
+                    choices=["full", "kernel", "round", "sim", "minworkers", "policies", "configs",
+                             "aux"],
                     help="kernel: only warm-up + steps of the device-resident step (for profilers)")
     args = ap.parse_args()
     if args.warmup < 3:
@@ -1040,6 +1104,8 @@ def main():
         run_policies(args)
     elif args.mode == "configs":
         run_configs(args)
+    elif args.mode == "aux":
+        run_aux(args)
     else:
         run_ours(args)
 

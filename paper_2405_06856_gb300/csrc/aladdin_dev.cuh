@@ -151,6 +151,15 @@ struct __align__(16) CandRec {
 
 __device__ __forceinline__ float f_inf() { return __int_as_float(0x7f800000); }
 
+// min(a, b, c): the three-operand form of min.f32 (sm_100 and later), the
+// same value as fminf(fminf(a, b), c) in one instruction.
+__device__ __forceinline__ float fmin3(float a, float b, float c)
+{
+    float d;
+    asm("min.f32 %0, %1, %2, %3;" : "=f"(d) : "f"(a), "f"(b), "f"(c));
+    return d;
+}
+
 __device__ __forceinline__ long long floor_div_ll(long long x, long long d)
 {
     if (d == 1) return x;
@@ -197,7 +206,7 @@ __device__ __forceinline__ void pair_headroom(const float4 v0, const float4 v1, 
     d[0] = fminf(v0.y, fmaf(c.r, np1n, v0.z)) - c.a;
     d[1] = fminf(fmaf(c.Zc, wr.x, -wr.y), wr.z) - c.a;
     d[2] = fminf(v1.z, fmaf(v1.w, c.inv_d1, c.nXd1)) - c.a;
-    d[3] = fminf(fminf(ext.x - c.a, fmaf(ext.y, c.inv_d2, c.Ua)),
+    d[3] = fmin3(ext.x - c.a, fmaf(ext.y, c.inv_d2, c.Ua),
                  fmaf(v0.w, c.inv_r, fmaf(v1.y, c.r, c.Ua - v1.x)));
 }
 
@@ -207,7 +216,7 @@ __device__ __forceinline__ unsigned eval_pair(const float4 v0, const float4 v1, 
 {
     float d[4];
     pair_headroom(v0, v1, ext, wr, c, d);
-    margin = fminf(fminf(d[0], d[1]), fminf(d[2], d[3]));
+    margin = fmin3(fminf(d[0], d[1]), d[2], d[3]);
     return (d[0] >= 0.0f ? 1u : 0u) | (d[1] >= 0.0f ? 2u : 0u) | (d[2] >= 0.0f ? 4u : 0u) |
            (d[3] >= 0.0f ? 8u : 0u);
 }
@@ -225,7 +234,7 @@ __device__ __forceinline__ unsigned eval_pair_mode(bool approx, const float4 v0,
     d[1] = fminf(fmaf(c.Zc, wr.x, -wr.y), wr.z) - c.a;
     d[2] = wa.x - c.a;
     d[3] = wa.y - c.Ua;
-    margin = fminf(fminf(d[0], d[1]), fminf(d[2], d[3]));
+    margin = fmin3(fminf(d[0], d[1]), d[2], d[3]);
     return (d[0] >= 0.0f ? 1u : 0u) | (d[1] >= 0.0f ? 2u : 0u) | (d[2] >= 0.0f ? 4u : 0u) |
            (d[3] >= 0.0f ? 8u : 0u);
 }

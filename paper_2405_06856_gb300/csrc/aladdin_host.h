@@ -16,9 +16,20 @@ constexpr long long MBAR_WAIT_POLLS = 1ll << 26;  // the scoring kernel's copy b
 // Elements per lane of the per-warp table builder for a slot capacity.
 inline int lanes_per_worker(int cap) { return cap / 32; }
 
+// Requests in CSR form on the device (worker w holds [off[w], off[w+1]) of
+// the arrays; tdec nullable), packed into the cluster's slots.
+struct PackSrc {
+    const int32_t* off;
+    const int32_t* in;
+    const int32_t* gen;
+    const int32_t* pred;
+    const float* tdec;
+};
 // K2: rebuild the tables of `count` workers (all workers when list == nullptr).
+// With src (list == nullptr), every worker's requests are first packed from
+// src into its slots by the warp that builds its table, in the same kernel.
 cudaError_t launch_build(const DevParams& P, const ClusterDev& C, const int32_t* list, int count,
-                         cudaStream_t st);
+                         cudaStream_t st, const PackSrc* src = nullptr);
 // capacity_norm ranks (descending key, lowest index on ties) and rank -> worker.
 cudaError_t launch_rank(const ClusterDev& C, cudaStream_t st);
 

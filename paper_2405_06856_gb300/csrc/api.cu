@@ -441,63 +441,30 @@ int load_requests_host(aladdin_cluster* cl, const int32_t* req_off, const int32_
     return ALADDIN_OK;
 }
 
-// Device path: pack CSR requests into slots on the GPU (one warp per worker);
-// a worker whose request count exceeds the slots or that holds an invalid
-// request is replaced by a single invalid request so that the table builder
-// marks it infeasible and records the error.
-__global__ void k_pack(DevParams P, ClusterDev C, const int32_t* __restrict__ off,
-                       const int32_t* __restrict__ in, const int32_t* __restrict__ gen,
-                       const int32_t* __restrict__ pred, const float* __restrict__ tdec)
-{
-    const int lane = threadIdx.x & 31;
-    const int w = blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
-    if (w >= C.W) return;
-    const int a = off[w], b = off[w + 1];
-    const long long base = (long long)w * C.cap;
-    int n = b - a;
-    const bool over = n < 0 || n > C.cap;
-    if (over) n = 0;
-    for (int q = lane; q < n; q += 32) {
-        const long long dst = base + q;
-        const int g = gen[a + q];
-        const int32_t pr = pred[a + q];
-        C.in[dst] = in[a + q];
-        C.gen[dst] = g;
-        C.pred[dst] = pr;
-        C.real[dst] = pr;  // exact predictions
-        C.tdec[dst] = tdec ? (double)tdec[a + q] : P.thetad * P.T_decd * (double)g;
-        C.pend[dst] = 0;
-    }
-    if (lane == 0) {
-        if (over) {
-            C.in[base] = -1;
-            C.gen[base] = 0;
-            C.pred[base] = 1;
-            C.real[base] = 1;
-            C.tdec[base] = 0.0;
-            C.pend[base] = 0;
-            atomicOr(C.err, 2u);
-        }
-        C.n[w] = over ? 1 : n;
-    }
-}
-
+// Load requests given in CSR form and rebuild every table. Device or
+// page-locked host arrays are packed on the device, by the warps that build
+// the tables, in the same kernel (read in place); pageable host arrays are
+// validated and packed on the host.
 int load_requests(aladdin_cluster* cl, const int32_t* req_off, const int32_t* in,
                   const int32_t* gen, const int32_t* pred, const float* tdec)
 {
     if (!req_off) return ALADDIN_ERR_ARG;
-    // device or page-locked host arrays: packed on the device, read in place
     int32_t *d_off = nullptr, *d_in = nullptr, *d_gen = nullptr, *d_pred = nullptr;
     float* d_tdec = nullptr;
     const bool dev = device_view(req_off, &d_off) && (!in || device_view(in, &d_in)) &&
                      (!gen || device_view(gen, &d_gen)) && (!pred || device_view(pred, &d_pred)) &&
                      (!tdec || device_view(tdec, &d_tdec));
-    if (!dev) return load_requests_host(cl, req_off, in, gen, pred, tdec);
+    cl->round_open = false;
+    if (!dev) {
+        int rc = load_requests_host(cl, req_off, in, gen, pred, tdec);
+        if (rc) return rc;
+        return refresh_tables(cl);
+    }
     if (!in || !gen || !pred) return ALADDIN_ERR_ARG;
-    const int wpb = 4;
-    k_pack<<<(cl->W + wpb - 1) / wpb, 32 * wpb, 0, cl->st>>>(cl->dp, cl->dev, d_off, d_in, d_gen,
-                                                             d_pred, d_tdec);
-    CK(cudaGetLastError());
+    cl->aux_valid = false;
+    const PackSrc S{d_off, d_in, d_gen, d_pred, d_tdec};
+    CK(launch_build(cl->dp, cl->dev, nullptr, cl->W, cl->st, &S));
+    CK(launch_rank(cl->dev, cl->st));
     return ALADDIN_OK;
 }
 
@@ -656,10 +623,7 @@ int aladdin_cluster_load(aladdin_cluster* cl, const int32_t* req_off, const int3
 try {
     if (!cl) return ALADDIN_ERR_ARG;
     CK(cudaSetDevice(cl->device));
-    int rc = load_requests(cl, req_off, in, gen, pred, tdec_ms);
-    if (rc) return rc;
-    cl->round_open = false;
-    return refresh_tables(cl);
+    return load_requests(cl, req_off, in, gen, pred, tdec_ms);
 } catch (...) {
     return ALADDIN_ERR_NOMEM;  // a host allocation or thread start failed
 }
@@ -714,10 +678,6 @@ try {
     CK(launch_cand_prep(cl->dp, cl->W, n_cand, cin, cpr, cw, B, cl->side));
     CK(cudaEventRecord(cl->ev_join, cl->side));
     rc = load_requests(cl, req_off, in, gen, pred, tdec_ms);
-    if (!rc) {
-        cl->round_open = false;
-        rc = refresh_tables(cl);
-    }
     CK(cudaStreamWaitEvent(cl->st, cl->ev_join, 0));  // join (also on error)
     if (rc) return rc;
     cudaEvent_t e0 = nullptr, e1 = nullptr;

@@ -437,13 +437,13 @@ __global__ void __launch_bounds__(SCORE_WARPS * 32, PEND ? 3 : ALADDIN_SCORE_MIN
                         const float ca = fmaf(t.b0n, ir, fmaf(t.nh, r, Ua - t.b1));
                         if (PEND) {
                             d[1][s] = fminf(tt, ZW[s]) - a;
-                            d[3][s] = fminf(fminf(t.pmAp - a, fmaf(t.Gpt, id2, Ua)), ca);
+                            d[3][s] = fmin3(t.pmAp - a, fmaf(t.Gpt, id2, Ua), ca);
                         } else {
                             d[1][s] = tt - a;
                             d[3][s] = ca;
                         }
                     }
-                    m[s] = fminf(fminf(d[0][s], d[1][s]), fminf(d[2][s], d[3][s]));
+                    m[s] = fmin3(fminf(d[0][s], d[1][s]), d[2][s], d[3][s]);
                     if (ARG) kmin = min(kmin, (__float_as_uint(m[s]) & 0x80000000u) | rank[s]);
                 }
             };

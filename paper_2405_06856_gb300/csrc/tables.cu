@@ -6,9 +6,49 @@ namespace aladdin {
 
 constexpr int BUILD_WARPS = 4;
 
+// One warp packs worker w's requests from CSR arrays into its slots: a worker
+// whose request count exceeds the slots is replaced by a single invalid
+// request, so that the table builder marks it infeasible and records the
+// error (bit 2). Returns the worker's request count (every lane).
+__device__ __forceinline__ int pack_worker(const DevParams& P, const ClusterDev& C,
+                                           const PackSrc& S, int w)
+{
+    const int lane = threadIdx.x & 31;
+    const int a = S.off[w], b = S.off[w + 1];
+    const long long base = (long long)w * C.cap;
+    int n = b - a;
+    const bool over = n < 0 || n > C.cap;
+    if (over) n = 0;
+    for (int q = lane; q < n; q += 32) {
+        const long long dst = base + q;
+        const int g = S.gen[a + q];
+        const int32_t pr = S.pred[a + q];
+        C.in[dst] = S.in[a + q];
+        C.gen[dst] = g;
+        C.pred[dst] = pr;
+        C.real[dst] = pr;  // exact predictions
+        C.tdec[dst] = S.tdec ? (double)S.tdec[a + q] : P.thetad * P.T_decd * (double)g;
+        C.pend[dst] = 0;
+    }
+    if (lane == 0) {
+        if (over) {
+            C.in[base] = -1;
+            C.gen[base] = 0;
+            C.pred[base] = 1;
+            C.real[base] = 1;
+            C.tdec[base] = 0.0;
+            C.pend[base] = 0;
+            atomicOr(C.err, 2u);
+        }
+        C.n[w] = over ? 1 : n;
+    }
+    __syncwarp();  // the slots are visible to the warp's build
+    return over ? 1 : n;
+}
+
 template <int E>
 __global__ void __launch_bounds__(BUILD_WARPS * 32)
-k_build(DevParams P, ClusterDev C, const int32_t* __restrict__ list, int count)
+k_build(DevParams P, ClusterDev C, const int32_t* __restrict__ list, int count, PackSrc S)
 {
     extern __shared__ __align__(16) unsigned char smraw[];
     BuildSmem<E>* sm = reinterpret_cast<BuildSmem<E>*>(smraw);
@@ -16,6 +56,7 @@ k_build(DevParams P, ClusterDev C, const int32_t* __restrict__ list, int count)
     const int idx = blockIdx.x * BUILD_WARPS + warp;
     if (idx >= count) return;  // whole warp leaves together
     const int w = list ? list[idx] : idx;
+    if (S.off) pack_worker(P, C, S, w);
     build_table<E>(P, C, w, sm[warp]);
 }
 
@@ -28,14 +69,16 @@ constexpr int E_LO = 4;
 
 template <int E>
 __global__ void __launch_bounds__(BUILD_WARPS * 32)
-k_build_lo(DevParams P, ClusterDev C, int count, int32_t* __restrict__ ovf, int* __restrict__ novf)
+k_build_lo(DevParams P, ClusterDev C, int count, int32_t* __restrict__ ovf, int* __restrict__ novf,
+           PackSrc S)
 {
     extern __shared__ __align__(16) unsigned char smraw[];
     BuildSmem<E>* sm = reinterpret_cast<BuildSmem<E>*>(smraw);
     const int warp = threadIdx.x >> 5;
     const int w = blockIdx.x * BUILD_WARPS + warp;
     if (w >= count) return;
-    if (C.n[w] > 32 * E) {  // warp-uniform
+    const int n = S.off ? pack_worker(P, C, S, w) : C.n[w];
+    if (n > 32 * E) {  // warp-uniform
         if ((threadIdx.x & 31) == 0) ovf[atomicAdd(novf, 1)] = w;
         return;
     }
@@ -80,7 +123,7 @@ constexpr int COOP_NW = 8;
 
 template <int E>
 static cudaError_t build_e(const DevParams& P, const ClusterDev& C, const int32_t* list, int count,
-                           cudaStream_t st)
+                           cudaStream_t st, const PackSrc& S)
 {
     if (count <= 0) return cudaSuccess;
     const int blocks = (count + BUILD_WARPS - 1) / BUILD_WARPS;
@@ -96,7 +139,7 @@ static cudaError_t build_e(const DevParams& P, const ClusterDev& C, const int32_
         const size_t slo = sizeof(BuildSmem<E_LO>) * BUILD_WARPS;
         if ((e = allow_smem<k_build_lo<E_LO>>(slo)) != cudaSuccess) return e;
         if ((e = cudaMemsetAsync(C.novf, 0, sizeof(int), st)) != cudaSuccess) return e;
-        k_build_lo<E_LO><<<blocks, BUILD_WARPS * 32, slo, st>>>(P, C, count, C.ovf, C.novf);
+        k_build_lo<E_LO><<<blocks, BUILD_WARPS * 32, slo, st>>>(P, C, count, C.ovf, C.novf, S);
         k_build_coop<EW, COOP_NW><<<count, COOP_NW * 32, sc, st>>>(P, C, C.ovf, 0, C.novf);
         return cudaGetLastError();
     } else {
@@ -107,27 +150,32 @@ static cudaError_t build_e(const DevParams& P, const ClusterDev& C, const int32_
             if ((e = allow_smem<k_build_lo<EL>>(slo)) != cudaSuccess) return e;
             if ((e = allow_smem<k_build_ovf<E>>(shi)) != cudaSuccess) return e;
             if ((e = cudaMemsetAsync(C.novf, 0, sizeof(int), st)) != cudaSuccess) return e;
-            k_build_lo<EL><<<blocks, BUILD_WARPS * 32, slo, st>>>(P, C, count, C.ovf, C.novf);
+            k_build_lo<EL><<<blocks, BUILD_WARPS * 32, slo, st>>>(P, C, count, C.ovf, C.novf, S);
             k_build_ovf<E><<<blocks, BUILD_WARPS * 32, shi, st>>>(P, C, C.ovf, C.novf);
             return cudaGetLastError();
         }
         const size_t smem = sizeof(BuildSmem<E>) * BUILD_WARPS;
         if ((e = allow_smem<k_build<E>>(smem)) != cudaSuccess) return e;
-        k_build<E><<<blocks, BUILD_WARPS * 32, smem, st>>>(P, C, list, count);
+        k_build<E><<<blocks, BUILD_WARPS * 32, smem, st>>>(P, C, list, count, S);
         return cudaGetLastError();
     }
 }
 
 cudaError_t launch_build(const DevParams& P, const ClusterDev& C, const int32_t* list, int count,
-                         cudaStream_t st)
+                         cudaStream_t st, const PackSrc* src)
 {
+    PackSrc S{};
+    if (src) {
+        if (list) return cudaErrorInvalidValue;  // packing covers every worker
+        S = *src;
+    }
     switch (lanes_per_worker(C.cap)) {
-    case 1: return build_e<1>(P, C, list, count, st);
-    case 2: return build_e<2>(P, C, list, count, st);
-    case 4: return build_e<4>(P, C, list, count, st);
-    case 8: return build_e<8>(P, C, list, count, st);
-    case 16: return build_e<16>(P, C, list, count, st);
-    case 32: return build_e<32>(P, C, list, count, st);
+    case 1: return build_e<1>(P, C, list, count, st, S);
+    case 2: return build_e<2>(P, C, list, count, st, S);
+    case 4: return build_e<4>(P, C, list, count, st, S);
+    case 8: return build_e<8>(P, C, list, count, st, S);
+    case 16: return build_e<16>(P, C, list, count, st, S);
+    case 32: return build_e<32>(P, C, list, count, st, S);
     default: return cudaErrorInvalidValue;
     }
 }
