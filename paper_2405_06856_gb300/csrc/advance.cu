@@ -177,6 +177,7 @@ k_advance(DevParams P, ClusterDev C, double t_now, double dt, unsigned long long
             C.pred[dst] = pr;
             C.real[dst] = rl;
             C.tdec[dst] = tdec[e];
+            C.bank[dst] = banked_slack(P, gen[e], tdec[e]);
             C.pend[dst] = 0;
             C.wait[dst] = wt;
         }

@@ -103,6 +103,9 @@ struct ClusterDev {
     int32_t* gen;              // [W*cap]
     int32_t* pred;             // [W*cap]
     double* tdec;              // [W*cap] decode time so far (ms)
+    float* bank;               // [W*cap] banked decode slack of an ongoing request,
+                               // (float)(theta T_dec l_out - t^dec) in double, written
+                               // wherever l_out or t^dec change (unused while pending)
     uint8_t* pend;             // [W*cap] 1: placed this round, prefill pending
     double* wait;              // [W*cap] pending: wait since arrival at placement
     float4* tab;               // [W*rows*ROW_F4] scoring rows
@@ -150,6 +153,13 @@ struct __align__(16) CandRec {
 };
 
 __device__ __forceinline__ float f_inf() { return __int_as_float(0x7f800000); }
+
+// Banked decode slack of a request that has generated g tokens in td ms
+// (Table 1's t^dec): theta T_dec g - td in double, rounded once to float.
+__device__ __forceinline__ float banked_slack(const DevParams& P, int g, double td)
+{
+    return (float)(P.thetad * P.T_decd * (double)g - td);
+}
 
 // min(a, b, c): the three-operand form of min.f32 (sm_100 and later), the
 // same value as fminf(fminf(a, b), c) in one instruction.
@@ -604,7 +614,8 @@ __device__ unsigned build_table(const DevParams& P, const ClusterDev& C, int w,
     constexpr bool PRELOAD = E <= FUSE_MAX_E;  // registers allow it
     constexpr int EL = PRELOAD ? E : 1;
     int l_pd[EL], l_g[EL], l_pr[EL], l_in[EL];
-    double l_td[EL], l_wt[EL];
+    float l_bk[EL];
+    double l_wt[EL];
     unsigned l_sk[INSERT ? E : 1];
     if constexpr (INSERT) {
         // The previous build's sorted keys (all requests but the last, which
@@ -622,13 +633,14 @@ __device__ unsigned build_table(const DevParams& P, const ClusterDev& C, int w,
             const long long slot = base + x;
             l_pd[e] = 0;
             l_g[e] = l_pr[e] = l_in[e] = 0;
-            l_td[e] = l_wt[e] = 0.0;
+            l_bk[e] = 0.0f;
+            l_wt[e] = 0.0;
             if (x < C.cap) {
                 l_pd[e] = C.pend[slot];
                 l_g[e] = C.gen[slot];
                 l_pr[e] = C.pred[slot];
                 l_in[e] = C.in[slot];
-                l_td[e] = C.tdec[slot];
+                l_bk[e] = C.bank[slot];
                 l_wt[e] = C.wait[slot];
             }
         }
@@ -657,8 +669,7 @@ __device__ unsigned build_table(const DevParams& P, const ClusterDev& C, int w,
             key[e] = ((unsigned)r << 10) | (unsigned)i;
             sm.a[i] = a;
             sm.pend[i] = (uint8_t)pd;
-            const double td = PRELOAD ? l_td[e % EL] : C.tdec[slot];
-            sm.bank[i] = pd ? 0.0f : (float)(P.thetad * P.T_decd * (double)g - td);
+            sm.bank[i] = pd ? 0.0f : (PRELOAD ? l_bk[e % EL] : C.bank[slot]);
             sumIn += in;
             sumPred += pr;
             if (pd) {

@@ -30,6 +30,9 @@ struct PackSrc {
 // src into its slots by the warp that builds its table, in the same kernel.
 cudaError_t launch_build(const DevParams& P, const ClusterDev& C, const int32_t* list, int count,
                          cudaStream_t st, const PackSrc* src = nullptr);
+// The banked decode slack (ClusterDev::bank) of every slot from its l_out and
+// t^dec, after the host wrote the slot arrays.
+cudaError_t launch_bank(const DevParams& P, const ClusterDev& C, cudaStream_t st);
 // capacity_norm ranks (descending key, lowest index on ties) and rank -> worker.
 cudaError_t launch_rank(const ClusterDev& C, cudaStream_t st);
 

@@ -313,6 +313,7 @@ int cluster_alloc(aladdin_cluster* cl, const aladdin_params& p, int W,
     AL(gen, int32_t, slots);
     AL(pred, int32_t, slots);
     AL(tdec, double, slots);
+    AL(bank, float, slots);
     AL(pend, uint8_t, slots);
     AL(wait, double, slots);
     AL(tab, float4, rows * ROW_F4);
@@ -368,6 +369,7 @@ int cluster_alloc(aladdin_cluster* cl, const aladdin_params& p, int W,
 int refresh_tables(aladdin_cluster* cl)
 {
     cl->aux_valid = false;
+    CK(launch_bank(cl->dp, cl->dev, cl->st));
     CK(launch_build(cl->dp, cl->dev, nullptr, cl->W, cl->st));
     CK(launch_rank(cl->dev, cl->st));
     return ALADDIN_OK;

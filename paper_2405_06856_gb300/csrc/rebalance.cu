@@ -197,6 +197,7 @@ __global__ void __launch_bounds__(RB_THREADS) k_rebalance(DevParams P, ClusterDe
                     C.pred[sl] = C.pred[last];
                     C.real[sl] = C.real[last];
                     C.tdec[sl] = C.tdec[last];
+                    C.bank[sl] = C.bank[last];
                     C.pend[sl] = C.pend[last];
                     C.wait[sl] = C.wait[last];
                     C.n[x] -= 1;

@@ -27,7 +27,10 @@ __device__ __forceinline__ int pack_worker(const DevParams& P, const ClusterDev&
         C.gen[dst] = g;
         C.pred[dst] = pr;
         C.real[dst] = pr;  // exact predictions
-        C.tdec[dst] = S.tdec ? (double)S.tdec[a + q] : P.thetad * P.T_decd * (double)g;
+        // without a history every request has used exactly its budget: no slack
+        const double td = S.tdec ? (double)S.tdec[a + q] : P.thetad * P.T_decd * (double)g;
+        C.tdec[dst] = td;
+        C.bank[dst] = S.tdec ? banked_slack(P, g, td) : 0.0f;
         C.pend[dst] = 0;
     }
     if (lane == 0) {
@@ -37,6 +40,7 @@ __device__ __forceinline__ int pack_worker(const DevParams& P, const ClusterDev&
             C.pred[base] = 1;
             C.real[base] = 1;
             C.tdec[base] = 0.0;
+            C.bank[base] = 0.0f;
             C.pend[base] = 0;
             atomicOr(C.err, 2u);
         }
@@ -44,6 +48,24 @@ __device__ __forceinline__ int pack_worker(const DevParams& P, const ClusterDev&
     }
     __syncwarp();  // the slots are visible to the warp's build
     return over ? 1 : n;
+}
+
+// The banked decode slack of every slot from its l_out and t^dec (after the
+// host wrote the slots: creation, host loads, restore).
+__global__ void k_bank(DevParams P, ClusterDev C)
+{
+    const long long slots = (long long)C.W * C.cap;
+    for (long long s = (long long)blockIdx.x * blockDim.x + threadIdx.x; s < slots;
+         s += (long long)gridDim.x * blockDim.x)
+        C.bank[s] = banked_slack(P, C.gen[s], C.tdec[s]);
+}
+
+cudaError_t launch_bank(const DevParams& P, const ClusterDev& C, cudaStream_t st)
+{
+    const long long slots = (long long)C.W * C.cap;
+    const long long nb = (slots + 255) / 256;
+    k_bank<<<(int)(nb < 4096 ? nb : 4096), 256, 0, st>>>(P, C);
+    return cudaGetLastError();
 }
 
 template <int E>
