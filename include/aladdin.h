@@ -350,6 +350,17 @@ int aladdin_cluster_status(aladdin_cluster* cl);
 int aladdin_cluster_test_waits(aladdin_cluster* cl, int64_t grid_polls, int64_t mbar_polls,
                                int32_t run_out);
 
+/* Test hook of the incremental placement round; the paper has no
+ * counterpart. A best-fit round first scores every candidate against the
+ * round-start state, then re-evaluates only the workers it modifies, holding
+ * them in a bounded number of shared-memory slots; when they run out, the
+ * round continues with the sliced round from the current state, and very
+ * large rounds are split into chunks of candidates, each a fresh incremental
+ * round. max_slots > 0 caps the slots and chunk > 0 the candidates per chunk,
+ * so that tests reach both paths on small clusters (0: the defaults). The
+ * placements do not depend on either. ALADDIN_ERR_ARG for negative values. */
+int aladdin_cluster_test_round(aladdin_cluster* cl, int32_t max_slots, int32_t chunk);
+
 /* A request trace: arrival times (ms, non-decreasing), prompt and predicted
  * output lengths, and optionally prediction errors (Sec. 4.3): real[q] is the
  * output length request q really generates (the scheduler sees only

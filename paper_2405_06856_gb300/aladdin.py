@@ -82,6 +82,7 @@ _sig = {
     "aladdin_cluster_state": [_P, _P, _P, _P, _P, _P],
     "aladdin_cluster_status": [_P],
     "aladdin_cluster_test_waits": [_P, C.c_int64, C.c_int64, C.c_int32],
+    "aladdin_cluster_test_round": [_P, C.c_int32, C.c_int32],
     "aladdin_cluster_timing": [_P, C.c_int32, _P, _P],
     "aladdin_min_workers": [_P, C.c_int32, _P, _P, C.c_double, C.c_int32, _P, _P, _P, _P],
     "aladdin_simulate": [_P, _P, C.c_int32, _P, C.c_double, C.c_int32, C.c_int32, _P, _P],
@@ -276,6 +277,11 @@ def aladdin_cluster_status(cl):
 def aladdin_cluster_test_waits(cl, grid_polls, mbar_polls, run_out):
     _check(_lib.aladdin_cluster_test_waits(cl, int(grid_polls), int(mbar_polls), int(run_out)),
            "aladdin_cluster_test_waits")
+
+
+def aladdin_cluster_test_round(cl, max_slots, chunk):
+    _check(_lib.aladdin_cluster_test_round(cl, int(max_slots), int(chunk)),
+           "aladdin_cluster_test_round")
 
 
 def aladdin_cluster_timing(cl, enable):

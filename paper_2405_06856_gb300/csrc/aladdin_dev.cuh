@@ -74,6 +74,10 @@ struct DevParams {
     int32_t wait_test;          // test hook, 1: the next waits run out by design (the
                                 // round's exchange waits for one arrival more than its
                                 // CTAs make; the scoring kernel withholds its first copy)
+    int32_t round_slots_max;    // test hook (0: off): at most this many modified-worker
+                                // slots in the incremental round
+    int32_t round_chunk;        // test hook (0: off): at most this many candidates per
+                                // chunk of the incremental round
 };
 
 // Relative slack of a realized latency over its SLO before the execution step

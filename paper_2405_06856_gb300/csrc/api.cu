@@ -188,6 +188,8 @@ DevParams make_devparams(const aladdin_params& p)
     d.grid_wait_limit = GRID_WAIT_POLLS;
     d.mbar_wait_limit = MBAR_WAIT_POLLS;
     d.wait_test = 0;
+    d.round_slots_max = 0;
+    d.round_chunk = 0;
     return d;
 }
 
@@ -1033,6 +1035,16 @@ try {
     cl->dp.grid_wait_limit = grid_polls ? grid_polls : GRID_WAIT_POLLS;
     cl->dp.mbar_wait_limit = mbar_polls ? mbar_polls : MBAR_WAIT_POLLS;
     cl->dp.wait_test = run_out;
+    return ALADDIN_OK;
+} catch (...) {
+    return ALADDIN_ERR_NOMEM;  // a host allocation or thread start failed
+}
+
+int aladdin_cluster_test_round(aladdin_cluster* cl, int32_t max_slots, int32_t chunk)
+try {
+    if (!cl || max_slots < 0 || chunk < 0) return ALADDIN_ERR_ARG;
+    cl->dp.round_slots_max = max_slots;
+    cl->dp.round_chunk = chunk;
     return ALADDIN_OK;
 } catch (...) {
     return ALADDIN_ERR_NOMEM;  // a host allocation or thread start failed

@@ -345,11 +345,13 @@ static cudaError_t round_inc_e(const DevParams& P, const ClusterDev& C, const Ro
     if (e != cudaSuccess) return e;
     int nwin = 0, mmax = 0, rc = 0;
     if (!ri_plan<E>(C.W, C.cap, P.K, d.smem_optin, &nwin, &mmax, &rc)) return cudaSuccess;
+    if (P.round_slots_max > 0 && mmax > P.round_slots_max) mmax = P.round_slots_max;
     const size_t smem = ri_smem<E>(C.W, nwin, mmax, rc);
     if ((e = allow_max_smem<k_round_inc<E>>()) != cudaSuccess) return e;
     const int ldf = (C.W + 31) & ~31;
     const size_t per_row = (size_t)ldf;
-    const int chunk = (int)std::min<size_t>((size_t)io.n_cand, std::max<size_t>(1, RI_FLAGS_MAX / per_row));
+    int chunk = (int)std::min<size_t>((size_t)io.n_cand, std::max<size_t>(1, RI_FLAGS_MAX / per_row));
+    if (P.round_chunk > 0 && chunk > P.round_chunk) chunk = P.round_chunk;
     for (int c0 = 0; c0 < io.n_cand; c0 += chunk) {
         const int n = std::min(chunk, io.n_cand - c0);
         if (c0 > 0 && (e = launch_rank(C, st)) != cudaSuccess) return e;  // the chunk's start state

@@ -67,6 +67,29 @@ def test_round_w256(A, orc, synth):
         assert (pl >= 0).any()
 
 
+@pytest.mark.parametrize("max_slots,chunk", [(3, 0), (0, 97), (5, 131)])
+def test_round_incremental_hand_offs(A, orc, synth, max_slots, chunk):
+    """The incremental round's two hand-offs on a small cluster: with few
+    modified-worker slots the sliced round continues from the candidate that
+    needs one more, and with small chunks every chunk of candidates is a
+    fresh incremental round from the current state. Both place like the
+    oracle, over two calls (the second within the open round)."""
+    wl = synth.config("w256", n_cand=900, b_cap=128)
+    oc = orc.Cluster.from_workload(wl)
+    with A.Cluster.from_workload(wl) as cl:
+        A.aladdin_cluster_test_round(cl.handle, max_slots, chunk)
+        for lo, hi in ((0, 520), (520, 900)):
+            pl = cl.place_round(wl.cand_in[lo:hi], wl.cand_pred[lo:hi], wl.cand_wait[lo:hi])
+            ref = oc.place_round(wl.cand_in[lo:hi], wl.cand_pred[lo:hi], wl.cand_wait[lo:hi])
+            assert np.array_equal(pl, ref), np.argwhere(pl != ref)[:5]
+        assert_same_state(cl, oc, "hand-offs-%d-%d" % (max_slots, chunk))
+        assert cl.status() == A.OK
+    with A.Cluster.from_workload(wl) as cl:
+        with pytest.raises(A.AladdinError) as e:
+            A.aladdin_cluster_test_round(cl.handle, -1, 0)
+        assert e.value.code == A.ERR_ARG
+
+
 def test_round_capacity_error(A, synth):
     wl = synth.make_cluster("cap", 210, 2, 30, 10**6, 40, params=dict(T_pre=1e6, T_dec=1e6),
                             b_cap=32)
