@@ -220,6 +220,15 @@ struct aladdin_cluster {
     // and the events that fork it from and join it to the cluster's stream
     cudaStream_t side = nullptr;
     cudaEvent_t ev_fork = nullptr, ev_join = nullptr;
+    // aladdin_cluster_load_score: the state-load half of a call (packing and
+    // table build, ranking, candidate sort on the side stream) as a CUDA graph,
+    // kept for the next call with the same arguments and scratch; the scoring
+    // kernel stays a separate launch (its timing events are recorded live)
+    cudaGraphExec_t load_graph = nullptr;
+    cudaStream_t cap_st = nullptr;  // the stream the graph is captured on
+    uintptr_t load_key[16] = {};  // the arguments and scratch the graph was captured with
+    int load_hits = 0;            // consecutive calls with that key (capture on the second)
+    unsigned dp_version = 0;      // bumped whenever dp changes (test hooks)
     // optional CUDA-event timing of the scoring kernel
     bool timing = false;
     std::vector<cudaEvent_t> ev;   // pairs (start, stop)
@@ -252,9 +261,11 @@ struct aladdin_cluster {
     }
     ~aladdin_cluster()
     {
+        if (load_graph) cudaGraphExecDestroy(load_graph);
         if (ev_fork) cudaEventDestroy(ev_fork);
         if (ev_join) cudaEventDestroy(ev_join);
         if (side) cudaStreamDestroy(side);
+        if (cap_st) cudaStreamDestroy(cap_st);
         clear_events();
         for (cudaEvent_t e : ev_free) cudaEventDestroy(e);
         for (void* p : owned) {
@@ -449,6 +460,19 @@ int load_requests_host(aladdin_cluster* cl, const int32_t* req_off, const int32_
 // page-locked host arrays are packed on the device, by the warps that build
 // the tables, in the same kernel (read in place); pageable host arrays are
 // validated and packed on the host.
+// The device path of load_requests with the arrays' device addresses known.
+int load_requests_dev(aladdin_cluster* cl, const int32_t* d_off, const int32_t* d_in,
+                      const int32_t* d_gen, const int32_t* d_pred, const float* d_tdec)
+{
+    if (!d_in || !d_gen || !d_pred) return ALADDIN_ERR_ARG;
+    cl->round_open = false;
+    cl->aux_valid = false;
+    const PackSrc S{d_off, d_in, d_gen, d_pred, d_tdec};
+    CK(launch_build(cl->dp, cl->dev, nullptr, cl->W, cl->st, &S));
+    CK(launch_rank(cl->dev, cl->st));
+    return ALADDIN_OK;
+}
+
 int load_requests(aladdin_cluster* cl, const int32_t* req_off, const int32_t* in,
                   const int32_t* gen, const int32_t* pred, const float* tdec)
 {
@@ -465,11 +489,7 @@ int load_requests(aladdin_cluster* cl, const int32_t* req_off, const int32_t* in
         return refresh_tables(cl);
     }
     if (!in || !gen || !pred) return ALADDIN_ERR_ARG;
-    cl->aux_valid = false;
-    const PackSrc S{d_off, d_in, d_gen, d_pred, d_tdec};
-    CK(launch_build(cl->dp, cl->dev, nullptr, cl->W, cl->st, &S));
-    CK(launch_rank(cl->dev, cl->st));
-    return ALADDIN_OK;
+    return load_requests_dev(cl, d_off, d_in, d_gen, d_pred, d_tdec);
 }
 
 // Stage an input array on the device: returns a device pointer.
@@ -639,14 +659,17 @@ int aladdin_cluster_load_score(aladdin_cluster* cl, const int32_t* req_off, cons
                                int32_t* argbest)
 try {
     if (!cl || n_cand < 0) return ALADDIN_ERR_ARG;
-    // every array on the device (or mapped): overlap; otherwise the two calls
-    auto dv = [](const void* p) {
-        void* d = nullptr;
-        return !p || device_view(p, &d);
-    };
-    const bool dev = req_off && dv(req_off) && dv(in) && dv(gen) && dv(pred) && dv(tdec_ms) &&
-                     dv(cand_in) && dv(cand_pred) && dv(wait_ms) && dv(flags) && dv(margin) &&
-                     dv(argbest) && (flags || margin || argbest);
+    // every array on the device (or mapped): overlap; otherwise the two calls.
+    // Each pointer is classified once (a driver query each).
+    const void* ptrs[11] = {req_off, in, gen, pred, tdec_ms, cand_in, cand_pred,
+                            wait_ms, flags, margin, argbest};
+    void* view[11];
+    bool dev = req_off && (flags || margin || argbest), any_host = false;
+    for (int i = 0; i < 11 && dev; ++i) {
+        const PtrKind k = ptr_kind(ptrs[i], &view[i]);
+        if (ptrs[i] && k != PK_DEV && k != PK_MAPPED) dev = false;
+        if (ptrs[i] && k != PK_DEV) any_host = true;
+    }
     int rc;
     if (!dev || n_cand == 0) {
         if ((rc = aladdin_cluster_load(cl, req_off, in, gen, pred, tdec_ms))) return rc;
@@ -659,31 +682,94 @@ try {
         CK(cudaEventCreateWithFlags(&cl->ev_fork, cudaEventDisableTiming));
         CK(cudaEventCreateWithFlags(&cl->ev_join, cudaEventDisableTiming));
     }
-    int32_t *cin = nullptr, *cpr = nullptr;
-    float* cw = nullptr;
-    uint8_t* df = nullptr;
-    float* dm = nullptr;
-    int32_t* da = nullptr;
-    device_view(cand_in, &cin);
-    device_view(cand_pred, &cpr);
-    if (wait_ms) device_view(wait_ms, &cw);
-    if (flags) device_view(flags, &df);
-    if (margin) device_view(margin, &dm);
-    if (argbest) device_view(argbest, &da);
+    const int32_t* cin = static_cast<const int32_t*>(view[5]);
+    const int32_t* cpr = static_cast<const int32_t*>(view[6]);
+    const float* cw = static_cast<const float*>(view[7]);
+    uint8_t* df = static_cast<uint8_t*>(view[8]);
+    float* dm = static_cast<float*>(view[9]);
+    int32_t* da = static_cast<int32_t*>(view[10]);
     const size_t C = (size_t)n_cand;
     CK(cl->sorted.ensure(sizeof(float4) * CAND_REC_F4 * C));
     CK(cl->hist.ensure(sizeof(int32_t) * ((size_t)cl->hp.K + 2)));
     CK(cl->best.ensure(sizeof(unsigned int) * C));
     ScoreBuffers B{cl->sorted.as<float4>(), cl->hist.as<int32_t>(), cl->best.as<unsigned int>()};
     // fork: the candidates are sorted on the side stream (they read no table)
-    // while the cluster's stream packs the state and builds the tables
-    CK(cudaEventRecord(cl->ev_fork, cl->st));
-    CK(cudaStreamWaitEvent(cl->side, cl->ev_fork, 0));
-    CK(launch_cand_prep(cl->dp, cl->W, n_cand, cin, cpr, cw, B, cl->side));
-    CK(cudaEventRecord(cl->ev_join, cl->side));
-    rc = load_requests(cl, req_off, in, gen, pred, tdec_ms);
-    CK(cudaStreamWaitEvent(cl->st, cl->ev_join, 0));  // join (also on error)
-    if (rc) return rc;
+    // while the cluster's stream packs the state and builds the tables. The
+    // table build, on the critical path, is enqueued first; the side stream
+    // starts from the fork point recorded before it.
+    auto enqueue_load = [&]() -> int {
+        CK(cudaEventRecord(cl->ev_fork, cl->st));
+        const int r = load_requests_dev(
+            cl, static_cast<const int32_t*>(view[0]), static_cast<const int32_t*>(view[1]),
+            static_cast<const int32_t*>(view[2]), static_cast<const int32_t*>(view[3]),
+            static_cast<const float*>(view[4]));
+        CK(cudaStreamWaitEvent(cl->side, cl->ev_fork, 0));
+        CK(launch_cand_prep(cl->dp, cl->W, n_cand, cin, cpr, cw, B, cl->side));
+        CK(cudaEventRecord(cl->ev_join, cl->side));
+        CK(cudaStreamWaitEvent(cl->st, cl->ev_join, 0));  // join (also on error)
+        return r;
+    };
+    // A repeated call (same arrays, sizes, scratch and parameters) replays the
+    // load half captured as a graph: one launch instead of about a dozen
+    // commands the GPU would process one by one. The first call with a key
+    // runs eagerly (and sets every kernel attribute up), the second captures.
+    uintptr_t key[16] = {};
+    for (int i = 0; i < 11; ++i) key[i] = reinterpret_cast<uintptr_t>(view[i]);
+    key[11] = (uintptr_t)n_cand;
+    key[12] = reinterpret_cast<uintptr_t>(cl->sorted.p);
+    key[13] = reinterpret_cast<uintptr_t>(cl->hist.p);
+    key[14] = reinterpret_cast<uintptr_t>(cl->best.p);
+    key[15] = (uintptr_t)cl->dp_version;
+    // a stream the caller is capturing itself takes the eager path, leaving
+    // the cached graph alone
+    cudaStreamCaptureStatus cap = cudaStreamCaptureStatusNone;
+    CK(cudaStreamIsCapturing(cl->st, &cap));
+    if (cap != cudaStreamCaptureStatusNone) {
+        rc = enqueue_load();
+        if (rc) return rc;
+    } else {
+    const bool same = std::memcmp(key, cl->load_key, sizeof(key)) == 0;
+    if (!same) {
+        if (cl->load_graph) CK(cudaGraphExecDestroy(cl->load_graph));
+        cl->load_graph = nullptr;
+        std::memcpy(cl->load_key, key, sizeof(key));
+        cl->load_hits = 0;
+    }
+    cl->load_hits += 1;
+    if (!cl->load_graph && cl->load_hits >= 2) {
+        // captured on a private stream (the legacy default stream cannot be
+        // captured); the graph is then launched on the cluster's stream
+        if (!cl->cap_st) CK(cudaStreamCreateWithFlags(&cl->cap_st, cudaStreamNonBlocking));
+        cudaGraph_t g = nullptr;
+        const cudaStream_t user = cl->st;
+        cl->st = cl->cap_st;
+        cudaError_t ce = cudaStreamBeginCapture(cl->st, cudaStreamCaptureModeThreadLocal);
+        int r = ce == cudaSuccess ? enqueue_load() : ALADDIN_ERR_CUDA;
+        if (ce == cudaSuccess) ce = cudaStreamEndCapture(cl->st, &g);
+        cl->st = user;
+        if (r || ce != cudaSuccess || !g) {
+            if (g) cudaGraphDestroy(g);
+            cudaGetLastError();
+            cl->load_hits = -1000000;  // not capturable: stay eager for this key
+        } else {
+            const cudaError_t ie = cudaGraphInstantiate(&cl->load_graph, g, 0);
+            cudaGraphDestroy(g);
+            if (ie != cudaSuccess) {
+                cudaGetLastError();
+                cl->load_graph = nullptr;
+                cl->load_hits = -1000000;
+            }
+        }
+    }
+    if (cl->load_graph) {
+        CK(cudaGraphLaunch(cl->load_graph, cl->st));
+        cl->round_open = false;
+        cl->aux_valid = false;
+    } else {
+        rc = enqueue_load();
+        if (rc) return rc;
+    }
+    }
     cudaEvent_t e0 = nullptr, e1 = nullptr;
     if (cl->timing) {
         e0 = cl->take_event();
@@ -697,11 +783,7 @@ try {
     }
     CK(launch_score(cl->dp, cl->dev, n_cand, cin, cpr, cw, df, dm, da, nullptr, nullptr, B, false,
                     cl->st, e0, e1, true));
-    auto on_host = [](const void* p) { return p && ptr_kind(p) != PK_DEV; };
-    if (on_host(req_off) || on_host(in) || on_host(gen) || on_host(pred) || on_host(tdec_ms) ||
-        on_host(cand_in) || on_host(cand_pred) || on_host(wait_ms) || on_host(flags) ||
-        on_host(margin) || on_host(argbest))
-        CK(cudaStreamSynchronize(cl->st));
+    if (any_host) CK(cudaStreamSynchronize(cl->st));  // page-locked host arrays in use
     return ALADDIN_OK;
 } catch (...) {
     return ALADDIN_ERR_NOMEM;  // a host allocation or thread start failed
@@ -1035,6 +1117,7 @@ try {
     cl->dp.grid_wait_limit = grid_polls ? grid_polls : GRID_WAIT_POLLS;
     cl->dp.mbar_wait_limit = mbar_polls ? mbar_polls : MBAR_WAIT_POLLS;
     cl->dp.wait_test = run_out;
+    cl->dp_version += 1;
     return ALADDIN_OK;
 } catch (...) {
     return ALADDIN_ERR_NOMEM;  // a host allocation or thread start failed
@@ -1045,6 +1128,7 @@ try {
     if (!cl || max_slots < 0 || chunk < 0) return ALADDIN_ERR_ARG;
     cl->dp.round_slots_max = max_slots;
     cl->dp.round_chunk = chunk;
+    cl->dp_version += 1;
     return ALADDIN_OK;
 } catch (...) {
     return ALADDIN_ERR_NOMEM;  // a host allocation or thread start failed

@@ -269,6 +269,42 @@ def test_w4096_mixed_sampled(A, orc, synth):
         check_argbest(oc.order(), fr_rows, a.cpu().numpy()[rows], "w4096-mixed-rows")
 
 
+def test_load_score_repeated_calls(A, synth):
+    """Repeated aladdin_cluster_load_score calls with the same arrays (the
+    library replays its state-load half as a CUDA graph from the second
+    call) read the arrays' current contents: each of five calls, with a new
+    state and new candidates written into the same device arrays, gives the
+    bytes of a separate load and score."""
+    import torch
+    dev = torch.device("cuda")
+    base = synth.config("w256", n_cand=700)
+    C, W = base.n_cand, base.n_workers
+    N = len(base.req_in)
+    roff = torch.from_numpy(base.roff).to(dev)
+    rin, rgen, rpred = (torch.empty(N, dtype=torch.int32, device=dev) for _ in range(3))
+    cin, cpr = (torch.empty(C, dtype=torch.int32, device=dev) for _ in range(2))
+    cw = torch.empty(C, dtype=torch.float32, device=dev)
+    f = torch.empty((C, W), dtype=torch.uint8, device=dev)
+    m = torch.empty((C, W), dtype=torch.float32, device=dev)
+    a = torch.empty(C, dtype=torch.int32, device=dev)
+    with A.Cluster.from_workload(base) as cl, A.Cluster.from_workload(base) as ref:
+        for seed in range(5):
+            wl = synth.config("w256", n_cand=700, seed=40 + seed)
+            assert np.array_equal(wl.roff, base.roff)
+            for t, x in ((rin, wl.req_in), (rgen, wl.req_gen), (rpred, wl.req_pred),
+                         (cin, wl.cand_in), (cpr, wl.cand_pred), (cw, wl.cand_wait)):
+                t.copy_(torch.from_numpy(x))
+            A.aladdin_cluster_load_score(cl.handle, roff, rin, rgen, rpred, None, C, cin, cpr, cw,
+                                         f, m, a)
+            ref.load(wl.roff, wl.req_in, wl.req_gen, wl.req_pred)
+            g = ref.score(wl.cand_in, wl.cand_pred, wl.cand_wait)
+            torch.cuda.synchronize()
+            assert cl.status() == A.OK
+            assert np.array_equal(f.cpu().numpy(), g["flags"]), seed
+            assert np.array_equal(m.cpu().numpy().view(np.int32), g["margin"].view(np.int32)), seed
+            assert np.array_equal(a.cpu().numpy(), g["argbest"]), seed
+
+
 def test_page_locked_host_buffers(A, orc, synth):
     """Page-locked host arrays are read and written in place by the kernels
     (state packed on the device, outputs written over the CPU-GPU link): the
