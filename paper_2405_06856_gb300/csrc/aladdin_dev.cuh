@@ -118,7 +118,6 @@ struct ClusterDev {
     int32_t* R;                // [W] breakpoints
     float4* wrec;              // [W] {1/s, ZO, ZW, rank bits}
     unsigned long long* key;   // [W] order-preserving code of capacity_norm^2 (0: unusable)
-    int32_t* rank;             // [W]
     int32_t* order;            // [W] worker at rank
     unsigned int* err;         // sticky error bits (1: invalid request)
     int32_t* ovf;              // [W] workers left to the full-capacity table build

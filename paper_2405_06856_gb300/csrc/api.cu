@@ -335,7 +335,6 @@ int cluster_alloc(aladdin_cluster* cl, const aladdin_params& p, int W,
     AL(R, int32_t, W);
     AL(wrec, float4, W);
     AL(key, unsigned long long, W);
-    AL(rank, int32_t, W);
     AL(order, int32_t, W);
     AL(err, unsigned int, 1);
     AL(ovf, int32_t, W);

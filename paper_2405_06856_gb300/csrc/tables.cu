@@ -202,48 +202,58 @@ cudaError_t launch_build(const DevParams& P, const ClusterDev& C, const int32_t*
     }
 }
 
-// rank[w] = number of workers ordered before w: larger key, or equal key and
-// smaller index (a stable descending sort by capacity_norm). A 2-D grid of
-// CTAs counts, for a tile of 256 workers, the workers of one 256-key chunk
-// that precede each of them (integer compares on keys staged in shared
-// memory) and adds the count to rank[w]; k_order then inverts the ranks.
-constexpr int RANK_TILE = 256;
-constexpr int RANK_CHUNK = 256;
+// rank(w) = number of workers ordered before w: larger key, or equal key and
+// smaller index (a stable descending sort by capacity_norm). One CTA ranks a
+// block of 32 workers (a lane each) against every key: its 8 warps split the
+// keys, staged in shared memory a chunk at a time and read as broadcasts, and
+// the 8 partial counts are summed in shared memory. The CTA then writes the
+// inverse permutation (order[rank] = w) and the rank into w's record itself,
+// so the ranking is one launch. Keys left of the block (smaller index) count
+// when they are >= the worker's key, keys right of it when they are >, and
+// only the block's own 32 keys take the full test.
+constexpr int RANK_WARPS = 8;
+constexpr int RANK_CHUNK = 4096;  // keys staged at a time (32 KB)
 
-__global__ void __launch_bounds__(RANK_TILE) k_rank_count(ClusterDev C)
+__global__ void __launch_bounds__(RANK_WARPS * 32) k_rank(ClusterDev C)
 {
     __shared__ unsigned long long ks[RANK_CHUNK];
-    const int w = blockIdx.x * RANK_TILE + threadIdx.x;
-    const int v0 = blockIdx.y * RANK_CHUNK;
-    const int lim = min(RANK_CHUNK, C.W - v0);
-    for (int i = threadIdx.x; i < lim; i += RANK_TILE) ks[i] = C.key[v0 + i];
-    __syncthreads();
-    if (w >= C.W) return;
-    const unsigned long long kw = C.key[w];
+    __shared__ int part[RANK_WARPS][32];
+    const int lane = threadIdx.x & 31, q = threadIdx.x >> 5;
+    const int b0 = blockIdx.x * 32, w = b0 + lane;
+    const int W = C.W;
+    const unsigned long long kw = w < W ? C.key[w] : 0ull;
     int cnt = 0;
-    for (int i = 0; i < lim; ++i) {
-        const unsigned long long kv = ks[i];
-        cnt += (kv > kw) || (kv == kw && v0 + i < w);
+    for (int v0 = 0; v0 < W; v0 += RANK_CHUNK) {
+        const int lim = min(RANK_CHUNK, W - v0);
+        __syncthreads();
+        for (int i = threadIdx.x; i < lim; i += RANK_WARPS * 32) ks[i] = __ldg(&C.key[v0 + i]);
+        __syncthreads();
+        // this warp's share of the chunk: [j0, j1) in worker indexes
+        const int per = (lim + RANK_WARPS - 1) / RANK_WARPS;
+        const int j0 = v0 + min(lim, q * per), j1 = v0 + min(lim, (q + 1) * per);
+        const int l0 = min(j1, max(j0, b0)), l1 = max(j0, min(j1, b0 + 32));
+        for (int j = j0; j < l0; ++j) cnt += ks[j - v0] >= kw;
+        for (int j = l0; j < l1; ++j) {
+            const unsigned long long kv = ks[j - v0];
+            cnt += (kv > kw) || (kv == kw && j < w);
+        }
+        for (int j = l1; j < j1; ++j) cnt += ks[j - v0] > kw;
     }
-    if (cnt) atomicAdd(&C.rank[w], cnt);
-}
-
-__global__ void k_order(ClusterDev C)
-{
-    const int w = blockIdx.x * blockDim.x + threadIdx.x;
-    if (w >= C.W) return;
-    const int r = C.rank[w];
-    C.order[r] = w;
-    C.wrec[w].w = __int_as_float(r);
+    part[q][lane] = cnt;
+    __syncthreads();
+    if (q == 0 && w < W) {
+        int r = 0;
+#pragma unroll
+        for (int k = 0; k < RANK_WARPS; ++k) r += part[k][lane];
+        C.order[r] = w;
+        C.wrec[w].w = __int_as_float(r);
+    }
 }
 
 cudaError_t launch_rank(const ClusterDev& C, cudaStream_t st)
 {
-    cudaError_t e = cudaMemsetAsync(C.rank, 0, sizeof(int32_t) * (size_t)C.W, st);
-    if (e != cudaSuccess) return e;
-    dim3 grid((C.W + RANK_TILE - 1) / RANK_TILE, (C.W + RANK_CHUNK - 1) / RANK_CHUNK);
-    k_rank_count<<<grid, RANK_TILE, 0, st>>>(C);
-    k_order<<<(C.W + 255) / 256, 256, 0, st>>>(C);
+    if (C.W <= 0) return cudaSuccess;
+    k_rank<<<(C.W + 31) / 32, RANK_WARPS * 32, 0, st>>>(C);
     return cudaGetLastError();
 }
 
