@@ -204,20 +204,20 @@ cudaError_t launch_build(const DevParams& P, const ClusterDev& C, const int32_t*
 
 // rank(w) = number of workers ordered before w: larger key, or equal key and
 // smaller index (a stable descending sort by capacity_norm). One CTA ranks a
-// block of 32 workers (a lane each) against every key: its 8 warps split the
-// keys, staged in shared memory a chunk at a time and read as broadcasts, and
-// the 8 partial counts are summed in shared memory. The CTA then writes the
-// inverse permutation (order[rank] = w) and the rank into w's record itself,
-// so the ranking is one launch. Keys left of the block (smaller index) count
-// when they are >= the worker's key, keys right of it when they are >, and
-// only the block's own 32 keys take the full test.
-constexpr int RANK_WARPS = 8;
+// block of 32 workers (a lane each) against every key: its 32 warps split the
+// keys, staged in shared memory a chunk at a time and read two at a time as
+// broadcasts, and the 32 partial counts are summed through shared memory. The
+// CTA then writes the inverse permutation (order[rank] = w) and the rank into
+// w's record itself, so the ranking is one launch. Keys left of the block
+// (smaller index) count when they are >= the worker's key, keys right of it
+// when they are >, and only the block's own 32 keys take the full test.
+constexpr int RANK_WARPS = 32;
 constexpr int RANK_CHUNK = 4096;  // keys staged at a time (32 KB)
 
 __global__ void __launch_bounds__(RANK_WARPS * 32) k_rank(ClusterDev C)
 {
-    __shared__ unsigned long long ks[RANK_CHUNK];
-    __shared__ int part[RANK_WARPS][32];
+    __shared__ __align__(16) unsigned long long ks[RANK_CHUNK];
+    __shared__ int part[RANK_WARPS][33];
     const int lane = threadIdx.x & 31, q = threadIdx.x >> 5;
     const int b0 = blockIdx.x * 32, w = b0 + lane;
     const int W = C.W;
@@ -228,25 +228,44 @@ __global__ void __launch_bounds__(RANK_WARPS * 32) k_rank(ClusterDev C)
         __syncthreads();
         for (int i = threadIdx.x; i < lim; i += RANK_WARPS * 32) ks[i] = __ldg(&C.key[v0 + i]);
         __syncthreads();
-        // this warp's share of the chunk: [j0, j1) in worker indexes
-        const int per = (lim + RANK_WARPS - 1) / RANK_WARPS;
+        // this warp's share of the chunk, [j0, j1) in worker indexes, an even
+        // number of keys except at the chunk's end
+        const int per = ((lim + RANK_WARPS - 1) / RANK_WARPS + 1) & ~1;
         const int j0 = v0 + min(lim, q * per), j1 = v0 + min(lim, (q + 1) * per);
         const int l0 = min(j1, max(j0, b0)), l1 = max(j0, min(j1, b0 + 32));
-        for (int j = j0; j < l0; ++j) cnt += ks[j - v0] >= kw;
-        for (int j = l0; j < l1; ++j) {
-            const unsigned long long kv = ks[j - v0];
-            cnt += (kv > kw) || (kv == kw && j < w);
+        if (l0 == j1 && ((j1 - j0) & 1) == 0) {  // all left of the block: pairs
+            const ulonglong2* k2 = reinterpret_cast<const ulonglong2*>(ks + (j0 - v0));
+#pragma unroll 8
+            for (int t = 0; t < (j1 - j0) / 2; ++t) {
+                const ulonglong2 kv = k2[t];
+                cnt += (kv.x >= kw) + (kv.y >= kw);
+            }
+        } else if (l0 == j0 && l1 == j0 && ((j1 - j0) & 1) == 0) {  // all right: pairs
+            const ulonglong2* k2 = reinterpret_cast<const ulonglong2*>(ks + (j0 - v0));
+#pragma unroll 8
+            for (int t = 0; t < (j1 - j0) / 2; ++t) {
+                const ulonglong2 kv = k2[t];
+                cnt += (kv.x > kw) + (kv.y > kw);
+            }
+        } else {
+            for (int j = j0; j < l0; ++j) cnt += ks[j - v0] >= kw;
+            for (int j = l0; j < l1; ++j) {
+                const unsigned long long kv = ks[j - v0];
+                cnt += (kv > kw) || (kv == kw && j < w);
+            }
+            for (int j = l1; j < j1; ++j) cnt += ks[j - v0] > kw;
         }
-        for (int j = l1; j < j1; ++j) cnt += ks[j - v0] > kw;
     }
     part[q][lane] = cnt;
     __syncthreads();
-    if (q == 0 && w < W) {
+    if (q == 0) {
         int r = 0;
-#pragma unroll
+#pragma unroll 8
         for (int k = 0; k < RANK_WARPS; ++k) r += part[k][lane];
-        C.order[r] = w;
-        C.wrec[w].w = __int_as_float(r);
+        if (w < W) {
+            C.order[r] = w;
+            C.wrec[w].w = __int_as_float(r);
+        }
     }
 }
 

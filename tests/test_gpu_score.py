@@ -180,6 +180,44 @@ def test_load_device_state(A, orc, synth):
                   wl2.req_in, gen, wl2.req_pred)
 
 
+@pytest.mark.parametrize("theta,T_dec", [(1.0, 32.0 * (1.0 + 2.0 ** -52)),
+                                         (0.8, 50.0), (0.6180339887498949, 47.123456789)])
+def test_device_pack_decode_budget(A, synth, theta, T_dec):
+    """Requests packed from device arrays without a decode history get the
+    decode time of a request that used exactly its budget, theta T_dec l_out,
+    as the fp64 product (theta T_dec) * l_out: equal to numpy's for output
+    lengths up to 2^16 - 1, ties included (with theta T_dec = 32 (1 + 2^-52)
+    the exact product for l_out = 3 * 2^k lies halfway between two doubles),
+    and the whole packed state equals the state created from the same host
+    arrays."""
+    import torch
+    wl = synth.make_cluster("pack", 77, 96, 40, 1 << 22, 4, per_worker_random=True,
+                            out_law=(3000.0, 1.5, 2, 65000), in_law=(64.0, 0.5, 1, 500),
+                            params=dict(theta=theta, T_dec=T_dec, K=65536))
+    special = np.array([0, 1, 3, 5, 6, 12, 24576, 32769, 49152, 65534], np.int32)
+    k = len(special)
+    wl.req_gen[:k] = special
+    wl.req_pred[:k] = np.maximum(wl.req_pred[:k], special + 1)
+    wl.req_in[:k] = np.minimum(wl.req_in[:k], 65536 - wl.req_pred[:k])
+    dev = torch.device("cuda")
+    t = lambda x: torch.from_numpy(np.ascontiguousarray(x)).to(dev)
+    with A.Cluster.from_workload(wl) as host, A.Cluster.from_workload(wl) as packed:
+        packed.load(t(wl.roff), t(wl.req_in), t(wl.req_gen), t(wl.req_pred))
+        torch.cuda.synchronize()
+        assert packed.status() == A.OK
+        ch, cp = A.aladdin_cluster_save(host.handle), A.aladdin_cluster_save(packed.handle)
+    assert ch == cp
+    # the decode-time section of the checkpoint, against numpy's products
+    W, S = wl.n_workers, wl.n_workers * wl.b_cap
+    tail = 8 * S + S + 8 * S + 4 * W + 8 * W + 8 * W + 4 * W  # tdec .. be
+    td = np.frombuffer(cp[len(cp) - tail:len(cp) - tail + 8 * S], np.float64).reshape(W, wl.b_cap)
+    thT = np.float64(theta) * np.float64(T_dec)
+    for w in range(W):
+        lo, hi = wl.roff[w], wl.roff[w + 1]
+        want = thT * wl.req_gen[lo:hi].astype(np.float64)
+        assert td[w, :hi - lo].tobytes() == want.tobytes(), w
+
+
 def test_w4096_sampled(A, orc, synth):
     """The 4,096-worker workload at full size, scored by the call bench.py
     times (aladdin_cluster_load_score from device arrays): sampled pairs and
