@@ -237,10 +237,16 @@ struct aladdin_cluster {
     // stream-ordered pool of the device memory (nullptr: cudaMalloc): memory
     // allocated and released in the order of the cluster's stream
     cudaMemPool_t pool = nullptr;
+    // Zero-filled, so that state a load does not write (the waits of slots
+    // that are not pending, for instance) reads the same in every cluster
+    // and every checkpoint.
     cudaError_t alloc(void** p, size_t bytes)
     {
         cudaError_t e = pool ? cudaMallocFromPoolAsync(p, bytes, pool, st) : cudaMalloc(p, bytes);
-        if (e == cudaSuccess) owned.push_back(*p);
+        if (e == cudaSuccess) {
+            owned.push_back(*p);
+            e = cudaMemsetAsync(*p, 0, bytes, st);
+        }
         return e;
     }
     void clear_events()

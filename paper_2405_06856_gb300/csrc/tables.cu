@@ -214,6 +214,14 @@ cudaError_t launch_build(const DevParams& P, const ClusterDev& C, const int32_t*
 constexpr int RANK_WARPS = 32;
 constexpr int RANK_CHUNK = 4096;  // keys staged at a time (32 KB)
 
+// -1 if x < y, else 0: the sign of x - y. The capacity_norm keys stay below
+// 2^63 (a non-negative double's bits plus one, or an integer sum of squares
+// below 2^57), so the difference does not overflow.
+__device__ __forceinline__ int neg_if_lt(unsigned long long x, unsigned long long y)
+{
+    return (int)((long long)(x - y) >> 63);
+}
+
 __global__ void __launch_bounds__(RANK_WARPS * 32) k_rank(ClusterDev C)
 {
     __shared__ __align__(16) unsigned long long ks[RANK_CHUNK];
@@ -235,17 +243,19 @@ __global__ void __launch_bounds__(RANK_WARPS * 32) k_rank(ClusterDev C)
         const int l0 = min(j1, max(j0, b0)), l1 = max(j0, min(j1, b0 + 32));
         if (l0 == j1 && ((j1 - j0) & 1) == 0) {  // all left of the block: pairs
             const ulonglong2* k2 = reinterpret_cast<const ulonglong2*>(ks + (j0 - v0));
+            int lt = 0;  // minus the keys below the worker's
 #pragma unroll 8
             for (int t = 0; t < (j1 - j0) / 2; ++t) {
                 const ulonglong2 kv = k2[t];
-                cnt += (kv.x >= kw) + (kv.y >= kw);
+                lt += neg_if_lt(kv.x, kw) + neg_if_lt(kv.y, kw);
             }
+            cnt += (j1 - j0) + lt;
         } else if (l0 == j0 && l1 == j0 && ((j1 - j0) & 1) == 0) {  // all right: pairs
             const ulonglong2* k2 = reinterpret_cast<const ulonglong2*>(ks + (j0 - v0));
 #pragma unroll 8
             for (int t = 0; t < (j1 - j0) / 2; ++t) {
                 const ulonglong2 kv = k2[t];
-                cnt += (kv.x > kw) + (kv.y > kw);
+                cnt -= neg_if_lt(kw, kv.x) + neg_if_lt(kw, kv.y);
             }
         } else {
             for (int j = j0; j < l0; ++j) cnt += ks[j - v0] >= kw;
