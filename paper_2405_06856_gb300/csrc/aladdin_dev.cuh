@@ -119,6 +119,8 @@ struct ClusterDev {
     float4* wrec;              // [W] {1/s, ZO, ZW, rank bits}
     unsigned long long* key;   // [W] order-preserving code of capacity_norm^2 (0: unusable)
     int32_t* order;            // [W] worker at rank
+    unsigned long long* rk;    // [ceil(W / 1024) * 1024] ranking scratch: keys sorted per chunk
+    int32_t* ri;               // [same] their workers
     unsigned int* err;         // sticky error bits (1: invalid request)
     int32_t* ovf;              // [W] workers left to the full-capacity table build
     int* novf;                 // their count

@@ -342,6 +342,8 @@ int cluster_alloc(aladdin_cluster* cl, const aladdin_params& p, int W,
     AL(wrec, float4, W);
     AL(key, unsigned long long, W);
     AL(order, int32_t, W);
+    AL(rk, unsigned long long, (W + 1023) / 1024 * 1024);
+    AL(ri, int32_t, (W + 1023) / 1024 * 1024);
     AL(err, unsigned int, 1);
     AL(ovf, int32_t, W);
     AL(novf, int, 1);

@@ -203,26 +203,145 @@ cudaError_t launch_build(const DevParams& P, const ClusterDev& C, const int32_t*
 }
 
 // rank(w) = number of workers ordered before w: larger key, or equal key and
-// smaller index (a stable descending sort by capacity_norm). One CTA ranks a
-// block of 32 workers (a lane each) against every key: its 32 warps split the
-// keys, staged in shared memory a chunk at a time and read two at a time as
-// broadcasts, and the 32 partial counts are summed through shared memory. The
-// CTA then writes the inverse permutation (order[rank] = w) and the rank into
-// w's record itself, so the ranking is one launch. Keys left of the block
-// (smaller index) count when they are >= the worker's key, keys right of it
-// when they are >, and only the block's own 32 keys take the full test.
+// smaller index (a stable descending sort by capacity_norm). The capacity_norm
+// keys stay below 2^63 (a non-negative double's bits plus one, or an integer
+// sum of squares below 2^57).
+//
+// From 8,192 to 24,576 workers: a sort in two launches. k_rank_sort sorts
+// each chunk of 1,024 consecutive workers in a CTA (a bitonic network over
+// (key, index), one element a thread: the exchanges across warps through
+// shared memory, the ones within a warp by shuffles). k_rank_merge then places
+// every element, a thread each: its position in its own chunk plus, for every
+// other chunk, the number of that chunk's keys ahead of it, found by a binary
+// search over the chunk's sorted keys (all W keys are copied into each merge
+// CTA's shared memory). Workers of a chunk to the left have smaller indices,
+// so their equal keys count as ahead; those of a chunk to the right do not.
+// Below 8,192 workers (where the all-pairs count is faster: 6.8 against 13.4
+// us at 4,096 workers under ncu; 17.7 against 16.8 at 8,192, 60 against 24 at
+// 16,384) and above 24,576 (where the keys no longer fit one CTA's shared
+// memory), k_rank_count counts for each worker the keys ahead of it directly
+// (all pairs).
+constexpr int RANK_S = 1024;                    // workers a chunk (threads a CTA)
+constexpr int RANK_MERGE_MAX = 24 * RANK_S;     // keys the merge holds in shared memory
+#ifndef ALADDIN_RANK_SORT_MIN
+#define ALADDIN_RANK_SORT_MIN 8192
+#endif
+constexpr int RANK_SORT_MIN = ALADDIN_RANK_SORT_MIN;  // fewer workers: the all-pairs count
+
+// a comes before b
+__device__ __forceinline__ bool rank_before(unsigned long long ka, int ia, unsigned long long kb,
+                                            int ib)
+{
+    return ka > kb || (ka == kb && ia < ib);
+}
+
+__global__ void __launch_bounds__(RANK_S) k_rank_sort(ClusterDev C)
+{
+    __shared__ unsigned long long xk[RANK_S];
+    __shared__ int xi[RANK_S];
+    const int t = threadIdx.x, W = C.W;
+    const int w = blockIdx.x * RANK_S + t;
+    // padding sorts after every worker (key 0, indices above W - 1)
+    unsigned long long k = w < W ? C.key[w] : 0ull;
+    int i = w;
+    for (int size = 2; size <= RANK_S; size <<= 1) {
+        const bool up = (t & size) == 0;  // this block of the network sorts "before" first
+        for (int stride = size >> 1; stride > 0; stride >>= 1) {
+            unsigned long long pk;
+            int pi;
+            if (stride >= 32) {
+                xk[t] = k;
+                xi[t] = i;
+                __syncthreads();
+                pk = xk[t ^ stride];
+                pi = xi[t ^ stride];
+                __syncthreads();
+            } else {
+                pk = __shfl_xor_sync(FULL, k, stride);
+                pi = __shfl_xor_sync(FULL, i, stride);
+            }
+            // the lower position of the pair keeps the element that comes
+            // first (in an "up" block), the upper one the other
+            const bool lower = (t & stride) == 0;
+            const bool mine_first = rank_before(k, i, pk, pi);
+            if (mine_first != (lower == up)) {
+                k = pk;
+                i = pi;
+            }
+        }
+    }
+    C.rk[w] = k;
+    C.ri[w] = i;
+}
+
+// Number of keys of the descending run ks[0, n) that are >= key (ge) or > key.
+__device__ __forceinline__ int rank_count_ahead(const unsigned long long* ks, int n,
+                                                unsigned long long key, bool ge)
+{
+    int lo = 0, hi = n;
+    while (lo < hi) {
+        const int mid = (lo + hi) >> 1;
+        const unsigned long long v = ks[mid];
+        if (ge ? v >= key : v > key) lo = mid + 1;
+        else hi = mid;
+    }
+    return lo;
+}
+
+constexpr int RANK_MT = 256;  // threads of a merge CTA (a quarter of a chunk's elements)
+
+__global__ void __launch_bounds__(RANK_MT) k_rank_merge(ClusterDev C)
+{
+    extern __shared__ __align__(16) unsigned char smraw[];
+    unsigned long long* ks = reinterpret_cast<unsigned long long*>(smraw);
+    const int W = C.W;
+    const int nchunks = (W + RANK_S - 1) / RANK_S;
+    const ulonglong2* src = reinterpret_cast<const ulonglong2*>(C.rk);
+    ulonglong2* dst = reinterpret_cast<ulonglong2*>(ks);
+    // eight loads in flight a thread (the copy is latency-bound otherwise)
+    const int n2 = nchunks * RANK_S / 2;  // key pairs
+    for (int p0 = threadIdx.x; p0 < n2; p0 += 8 * RANK_MT) {
+        ulonglong2 v[8];
+#pragma unroll
+        for (int u = 0; u < 8; ++u)
+            if (p0 + u * RANK_MT < n2) v[u] = __ldg(&src[p0 + u * RANK_MT]);
+#pragma unroll
+        for (int u = 0; u < 8; ++u)
+            if (p0 + u * RANK_MT < n2) dst[p0 + u * RANK_MT] = v[u];
+    }
+    __syncthreads();
+    const int e = blockIdx.x * RANK_MT + threadIdx.x;  // sorted position overall
+    const int c = e / RANK_S, t = e % RANK_S;
+    const int n_c = min(RANK_S, W - c * RANK_S);  // workers of this chunk (a prefix of it)
+    if (t >= n_c) return;
+    const unsigned long long key = ks[c * RANK_S + t];
+    int r = t;
+    for (int c2 = 0; c2 < nchunks; ++c2) {
+        if (c2 == c) continue;
+        const int n2 = min(RANK_S, W - c2 * RANK_S);
+        r += rank_count_ahead(ks + c2 * RANK_S, n2, key, c2 < c);
+    }
+    const int w = C.ri[c * RANK_S + t];
+    C.order[r] = w;
+    C.wrec[w].w = __int_as_float(r);
+}
+
+// All pairs, for clusters beyond RANK_MERGE_MAX workers: a CTA of 32 warps
+// ranks 32 workers (a lane each); its warps split the keys, staged in shared
+// memory a chunk at a time and read two at a time as broadcasts. Keys left of
+// the worker's block count when >= its key, keys right of it when >, only the
+// block's own 32 keys take the full test; the comparison is the sign of the
+// 64-bit difference.
 constexpr int RANK_WARPS = 32;
 constexpr int RANK_CHUNK = 4096;  // keys staged at a time (32 KB)
 
-// -1 if x < y, else 0: the sign of x - y. The capacity_norm keys stay below
-// 2^63 (a non-negative double's bits plus one, or an integer sum of squares
-// below 2^57), so the difference does not overflow.
+// -1 if x < y, else 0 (keys below 2^63: the difference does not overflow)
 __device__ __forceinline__ int neg_if_lt(unsigned long long x, unsigned long long y)
 {
     return (int)((long long)(x - y) >> 63);
 }
 
-__global__ void __launch_bounds__(RANK_WARPS * 32) k_rank(ClusterDev C)
+__global__ void __launch_bounds__(RANK_WARPS * 32) k_rank_count(ClusterDev C)
 {
     __shared__ __align__(16) unsigned long long ks[RANK_CHUNK];
     __shared__ int part[RANK_WARPS][33];
@@ -245,16 +364,16 @@ __global__ void __launch_bounds__(RANK_WARPS * 32) k_rank(ClusterDev C)
             const ulonglong2* k2 = reinterpret_cast<const ulonglong2*>(ks + (j0 - v0));
             int lt = 0;  // minus the keys below the worker's
 #pragma unroll 8
-            for (int t = 0; t < (j1 - j0) / 2; ++t) {
-                const ulonglong2 kv = k2[t];
+            for (int s = 0; s < (j1 - j0) / 2; ++s) {
+                const ulonglong2 kv = k2[s];
                 lt += neg_if_lt(kv.x, kw) + neg_if_lt(kv.y, kw);
             }
             cnt += (j1 - j0) + lt;
         } else if (l0 == j0 && l1 == j0 && ((j1 - j0) & 1) == 0) {  // all right: pairs
             const ulonglong2* k2 = reinterpret_cast<const ulonglong2*>(ks + (j0 - v0));
 #pragma unroll 8
-            for (int t = 0; t < (j1 - j0) / 2; ++t) {
-                const ulonglong2 kv = k2[t];
+            for (int s = 0; s < (j1 - j0) / 2; ++s) {
+                const ulonglong2 kv = k2[s];
                 cnt -= neg_if_lt(kw, kv.x) + neg_if_lt(kw, kv.y);
             }
         } else {
@@ -282,7 +401,16 @@ __global__ void __launch_bounds__(RANK_WARPS * 32) k_rank(ClusterDev C)
 cudaError_t launch_rank(const ClusterDev& C, cudaStream_t st)
 {
     if (C.W <= 0) return cudaSuccess;
-    k_rank<<<(C.W + 31) / 32, RANK_WARPS * 32, 0, st>>>(C);
+    const int nchunks = (C.W + RANK_S - 1) / RANK_S;
+    if (C.W > RANK_MERGE_MAX || C.W < RANK_SORT_MIN) {
+        k_rank_count<<<(C.W + 31) / 32, RANK_WARPS * 32, 0, st>>>(C);
+        return cudaGetLastError();
+    }
+    k_rank_sort<<<nchunks, RANK_S, 0, st>>>(C);
+    const size_t smem = sizeof(unsigned long long) * (size_t)nchunks * RANK_S;
+    cudaError_t e = allow_smem<k_rank_merge>(smem);
+    if (e != cudaSuccess) return e;
+    k_rank_merge<<<nchunks * (RANK_S / RANK_MT), RANK_MT, smem, st>>>(C);
     return cudaGetLastError();
 }
 

@@ -218,6 +218,41 @@ def test_device_pack_decode_budget(A, synth, theta, T_dec):
         assert td[w, :hi - lo].tobytes() == want.tobytes(), w
 
 
+@pytest.mark.parametrize("W", [700, 5000, 9000, 20000, 30000])
+def test_rank_order_with_ties(A, orc, synth, W):
+    """The capacity_norm order behind argbest (larger key first, lower index
+    first among equal keys) on clusters ranked by the all-pairs count (700,
+    5,000 and 30,000 workers) and by the chunk sort and merge (9,000 and
+    20,000 workers, 9 and 20 chunks of 1,024): workers share one of
+    five request sets, so keys tie across chunks, and their KV capacities
+    differ, so the feasible workers of a candidate are scattered through each
+    tie group. Every argbest must be the first feasible worker in the oracle's
+    order."""
+    rng = np.random.default_rng(W)
+    sets = [rng.integers(16, 400, size=(k, 2)).astype(np.int32) for k in (1, 2, 3, 5, 8)]
+    pick = rng.integers(0, len(sets), W)
+    counts = np.array([len(sets[s]) for s in pick], np.int32)
+    roff = np.zeros(W + 1, np.int32)
+    np.cumsum(counts, out=roff[1:])
+    req = np.concatenate([sets[s] for s in pick])
+    req_in = req[:, 0].copy()
+    req_pred = (req[:, 1] + 8).astype(np.int32)
+    req_gen = np.minimum(req[:, 1] // 2, req_pred - 1).astype(np.int32)
+    kv = rng.choice(np.array([4000, 6000, 9000, 60000], np.int64), W)
+    C = 24
+    cand_in = rng.integers(16, 3000, C).astype(np.int32)
+    cand_pred = rng.integers(8, 300, C).astype(np.int32)
+    wl = synth.Workload("ties", dict(synth.BASE_PARAMS), np.ones(W, np.int32), kv,
+                        np.ones(W, np.float32), roff, req_in, req_gen, req_pred, cand_in,
+                        cand_pred, np.zeros(C, np.float32), 32)
+    with A.Cluster.from_workload(wl) as cl:
+        g = cl.score(wl.cand_in, wl.cand_pred, wl.cand_wait)
+    order = orc.Cluster.from_workload(wl).order()
+    f = g["flags"] == 15
+    assert 0 < f.mean() < 1
+    check_argbest(order, g["flags"], g["argbest"], "ties-W%d" % W)
+
+
 def test_w4096_sampled(A, orc, synth):
     """The 4,096-worker workload at full size, scored by the call bench.py
     times (aladdin_cluster_load_score from device arrays): sampled pairs and
