@@ -443,18 +443,20 @@ struct BuildSmem {
     float pf[7][NW];
     int pi[5][NW];
     unsigned cflag;
+    unsigned newk[8];                 // insertion: the appended keys
     uint8_t pend[N];
 };
 
-// Barrier of the NW warps building one table (warps 0..NW-1 of the CTA when
-// NW > 1; named barrier 1, so that the other warps may run on).
-template <int NW>
+// Barrier of the NW warps building one table (NW consecutive warps of the
+// CTA when NW > 1; a named barrier, 1 unless the caller runs two builds side
+// by side, so that the other warps may run on).
+template <int NW, int BAR = 1>
 __device__ __forceinline__ void group_sync()
 {
     if constexpr (NW == 1) {
         __syncwarp();
     } else {
-        asm volatile("bar.sync 1, %0;" ::"r"(NW * 32) : "memory");
+        asm volatile("bar.sync %0, %1;" ::"n"(BAR), "r"(NW * 32) : "memory");
     }
 }
 
@@ -587,31 +589,43 @@ struct SliceCache {
 };
 
 // Build worker w's table (rows 0..R), its record and its capacity_norm key.
-// Called by all lanes of NW warps (warps 0..NW-1 of the CTA when NW > 1);
-// element x = (q EW + e) 32 + lane of warp q, so 32 EW NW slots are covered.
-// Requests are loaded from the slot arrays; an invalid request (in < 0, gen
-// outside [0, pred), in + pred > K) makes the worker infeasible for every
-// candidate and sets err bit 1. With `cache`, the worker's shared-memory
-// copies are refreshed as well. With a valid `cand`, the candidate is
-// evaluated against the new table by the lane that holds its row, and every
-// lane returns its flags (else 0).
-template <int EW, int NW = 1, bool INSERT = false>
+// Called by all lanes of NW warps (warps W0..W0+NW-1 of the CTA when NW > 1,
+// synchronised by named barrier BAR); element x = (q EW + e) 32 + lane of
+// the group's warp q, so 32 EW NW slots are covered. Requests are loaded from
+// the slot arrays, the first n_in of them (the worker's count when n_in < 0);
+// an invalid request (in < 0, gen outside [0, pred), in + pred > K) makes the
+// worker infeasible for every candidate and sets err bit 1. With `cache`, the
+// worker's shared-memory copies are refreshed as well. With a valid `cand`,
+// the candidate is evaluated against the new table by the lane that holds
+// its row, and every lane returns its flags (else 0). EVAL: the evaluation
+// only (a state that is not committed): nothing is written outside `sm`
+// except the state's capacity_norm key into *key_out. INSERT: the last `ins`
+// slots (1 to 3) were appended since the build that left its sorted keys in
+// skey, and are inserted into that order instead of sorting afresh (ins up
+// to INS_MAX). !SKEY:
+// the sorted keys are left in sm.sorted for the caller to store (a caller
+// that runs an evaluation of the same worker beside this build).
+constexpr int INS_MAX = 5;  // appended keys an insertion build takes
+
+template <int EW, int NW = 1, bool INSERT = false, int BAR = 1, int W0 = 0, bool EVAL = false,
+          bool SKEY = true>
 __device__ unsigned build_table(const DevParams& P, const ClusterDev& C, int w,
                                 BuildSmem<EW, NW>& sm, const SliceCache* cache = nullptr,
-                                const CandRec* cand = nullptr)
+                                const CandRec* cand = nullptr, int n_in = -1,
+                                unsigned long long* key_out = nullptr, int ins = 1)
 {
     static_assert(!INSERT || NW > 1, "the insertion path is for cooperative builds");
     constexpr int E = EW;
     constexpr int RUN = 32 * EW;  // elements per warp
     const int lane = threadIdx.x & 31;
-    const int q = NW > 1 ? (int)(threadIdx.x >> 5) : 0;
+    const int q = NW > 1 ? (int)(threadIdx.x >> 5) - W0 : 0;
     const int x0 = q * RUN;
     const long long base = (long long)w * C.cap;
     const long long rowbase = (long long)w * C.rows;
     // Independent loads first: the slot loads do not wait for n (slots below
     // the capacity lie inside the worker's slot range; those past n are
     // masked). A build may cover more elements than the capacity (padding).
-    const int n = C.n[w];
+    const int n = n_in >= 0 ? n_in : C.n[w];
     const float s = C.scale[w];
     const int M = C.M[w];
     const float off = C.off[w];
@@ -623,8 +637,8 @@ __device__ unsigned build_table(const DevParams& P, const ClusterDev& C, int w,
     double l_wt[EL];
     unsigned l_sk[INSERT ? E : 1];
     if constexpr (INSERT) {
-        // The previous build's sorted keys (all requests but the last, which
-        // was just appended).
+        // The previous build's sorted keys (all requests but the last `ins`,
+        // which were appended since).
 #pragma unroll
         for (int e = 0; e < E; ++e) {
             const int x = x0 + e * 32 + lane;
@@ -712,7 +726,7 @@ __device__ unsigned build_table(const DevParams& P, const ClusterDev& C, int w,
             sm.pi[1][q] = bad;
         }
     }
-    group_sync<NW>();
+    group_sync<NW, BAR>();
     if constexpr (NW > 1) {
         sumP = combine_warps<NW>(sm.pll[0], OpAdd<long long>(), 0LL);
         sumIn = combine_warps<NW>(sm.pll[1], OpAdd<long long>(), 0LL);
@@ -740,7 +754,7 @@ __device__ unsigned build_table(const DevParams& P, const ClusterDev& C, int w,
         for (int d = 16; d > 0; d >>= 1) dmin = fmin(dmin, __shfl_xor_sync(FULL, dmin, d));
         if constexpr (NW > 1) {
             if (lane == 0) sm.pdm[q] = dmin;
-            group_sync<NW>();
+            group_sync<NW, BAR>();
             dmin = combine_warps<NW>(sm.pdm, OpMin<double>(), dmin);
         }
         const double s_d = C.scaled[w];
@@ -784,48 +798,78 @@ __device__ unsigned build_table(const DevParams& P, const ClusterDev& C, int w,
     // each warp's run and merge the runs.
     constexpr bool COUNT_RANK = NW > 1 && N <= 256 && !INSERT;
     if constexpr (INSERT) {
-        // Insert the appended request's key into the previous sorted order.
+        // Insert the appended requests' keys into the previous sorted order
+        // (keys are distinct): a new key lands after the old and new keys
+        // below it, an old key moves up by the new keys below it.
+        const int n0 = n - ins;  // keys of the previous order
 #pragma unroll
         for (int e = 0; e < E; ++e) {
             const int x = x0 + e * 32 + lane;
-            if (x < n - 1) sm.runs[x] = l_sk[e];
-            if (x == n - 1) sm.cflag = key[e];
+            if (x < n0) sm.runs[x] = l_sk[e];
+            if (x >= n0 && x < n) sm.newk[x - n0] = key[e];
         }
-        group_sync<NW>();
-        const unsigned knew = sm.cflag;
-        int lo;  // old keys below knew (keys are distinct)
-        if constexpr (E == 1) {
-            // one key a thread: the count of old keys below knew is a
-            // barrier reduction over the group
-            const unsigned below = (x0 + lane < n - 1 && l_sk[0] < knew) ? 1u : 0u;
-            unsigned cnt;
-            asm volatile("{\n .reg .pred p;\n setp.ne.u32 p, %2, 0;\n"
-                         " bar.red.popc.u32 %0, 1, %1, p;\n}"
-                         : "=r"(cnt)
-                         : "r"(NW * 32), "r"(below)
-                         : "memory");
-            lo = (int)cnt;
-        } else {
-            int hi = n - 1;
-            lo = 0;
-            while (lo < hi) {
-                const int mid = (lo + hi) >> 1;
-                if (sm.runs[mid] < knew) lo = mid + 1;
-                else hi = mid;
+        group_sync<NW, BAR>();
+        unsigned nk[INS_MAX];
+        int pos[INS_MAX];
+#pragma unroll
+        for (int j = 0; j < INS_MAX; ++j) {
+            nk[j] = j < ins ? sm.newk[j] : 0xffffffffu;
+            pos[j] = 0;
+        }
+#pragma unroll
+        for (int j = 0; j < INS_MAX; ++j) {
+            if (j >= ins) break;  // uniform
+            int lo;  // old keys below nk[j]
+            if constexpr (E == 1) {
+                // one key a thread: a barrier reduction over the group
+                const unsigned below = (x0 + lane < n0 && l_sk[0] < nk[j]) ? 1u : 0u;
+                unsigned cnt;
+                asm volatile("{\n .reg .pred p;\n setp.ne.u32 p, %2, 0;\n"
+                             " bar.red.popc.u32 %0, %3, %1, p;\n}"
+                             : "=r"(cnt)
+                             : "r"(NW * 32), "r"(below), "n"(BAR)
+                             : "memory");
+                lo = (int)cnt;
+            } else {
+                int hi = n0;
+                lo = 0;
+                while (lo < hi) {
+                    const int mid = (lo + hi) >> 1;
+                    if (sm.runs[mid] < nk[j]) lo = mid + 1;
+                    else hi = mid;
+                }
+            }
+            pos[j] = lo;
+#pragma unroll
+            for (int j2 = 0; j2 < INS_MAX; ++j2) pos[j] += (j2 < ins && nk[j2] < nk[j]) ? 1 : 0;
+        }
+#pragma unroll
+        for (int e = 0; e < E; ++e) {
+            const int x = x0 + e * 32 + lane;
+            if (x < n0) {
+                const unsigned k = l_sk[e];
+                int sh = 0;
+#pragma unroll
+                for (int j = 0; j < INS_MAX; ++j) sh += (j < ins && nk[j] < k) ? 1 : 0;
+                sm.sorted[x + sh] = k;
             }
         }
+        if (q == 0 && lane < ins) {
+#pragma unroll
+            for (int j = 0; j < INS_MAX; ++j)
+                if (j == lane) sm.sorted[pos[j]] = nk[j];
+        }
+        group_sync<NW, BAR>();
 #pragma unroll
         for (int e = 0; e < E; ++e) {
             const int x = x0 + e * 32 + lane;
-            key[e] = x < n ? (x < lo ? sm.runs[x] : (x == lo ? knew : sm.runs[x - 1])) : 0xffffffffu;
-            if (x < n) sm.sorted[x] = key[e];
+            key[e] = x < n ? sm.sorted[x] : 0xffffffffu;
         }
-        group_sync<NW>();
     }
     if constexpr (COUNT_RANK) {
 #pragma unroll
         for (int e = 0; e < E; ++e) sm.runs[x0 + e * 32 + lane] = key[e];
-        group_sync<NW>();
+        group_sync<NW, BAR>();
         int rank[E];
 #pragma unroll
         for (int e = 0; e < E; ++e) rank[e] = 0;
@@ -840,7 +884,7 @@ __device__ unsigned build_table(const DevParams& P, const ClusterDev& C, int w,
 #pragma unroll
         for (int e = 0; e < E; ++e)
             if (x0 + e * 32 + lane < n) sm.sorted[rank[e]] = key[e];
-        group_sync<NW>();
+        group_sync<NW, BAR>();
 #pragma unroll
         for (int e = 0; e < E; ++e) {
             const int x = x0 + e * 32 + lane;
@@ -882,7 +926,7 @@ __device__ unsigned build_table(const DevParams& P, const ClusterDev& C, int w,
         // earlier runs first).
 #pragma unroll
         for (int e = 0; e < E; ++e) sm.runs[x0 + e * 32 + lane] = key[e];
-        group_sync<NW>();
+        group_sync<NW, BAR>();
 #pragma unroll
         for (int e = 0; e < E; ++e) {
             // In every other run, the count of keys before this one: a
@@ -907,7 +951,7 @@ __device__ unsigned build_table(const DevParams& P, const ClusterDev& C, int w,
                 if (q2 != q) rank += cnt[q2];
             sm.sorted[rank] = key[e];
         }
-        group_sync<NW>();
+        group_sync<NW, BAR>();
 #pragma unroll
         for (int e = 0; e < E; ++e) key[e] = sm.sorted[x0 + e * 32 + lane];
     }
@@ -934,7 +978,7 @@ __device__ unsigned build_table(const DevParams& P, const ClusterDev& C, int w,
 #pragma unroll
     for (int e = 0; e < E; ++e) {
         const int x = x0 + e * 32 + lane;
-        if (x < n) C.skey[base + x] = key[e];
+        if (!EVAL && SKEY && x < n) C.skey[base + x] = key[e];
     }
     // Neighbours in sorted order.
     int rnext[E], first[E], last[E];
@@ -990,7 +1034,7 @@ __device__ unsigned build_table(const DevParams& P, const ClusterDev& C, int w,
             sm.pll[4][q] = s_ra.total;
             sm.pi[4][q] = s_a.total;
         }
-        group_sync<NW>();
+        group_sync<NW, BAR>();
         add_carry_prefix<NW>(s_row, sm.pi[2], q);
         add_carry_prefix<NW>(s_r, sm.pi[3], q);
         add_carry_prefix<NW>(s_ra, sm.pll[4], q);
@@ -1017,7 +1061,7 @@ __device__ unsigned build_table(const DevParams& P, const ClusterDev& C, int w,
             sm.Tp[rowid[e]] = s * (P.c3 * (float)rr + P.c2 * (float)Sb + P.k2 * (float)SK);
         }
     }
-    group_sync<NW>();
+    group_sync<NW, BAR>();
 
     // Per-request bounds and slacks.
     const float stall0 = s * (P.k1 * (float)sumP + P.c1);
@@ -1069,7 +1113,7 @@ __device__ unsigned build_table(const DevParams& P, const ClusterDev& C, int w,
             sm.pf[4][q] = s_smSp.total;
             sm.pll[1][q] = s_SM.total;
         }
-        group_sync<NW>();
+        group_sync<NW, BAR>();
         add_carry_prefix<NW>(s_pmA, sm.pf[1], q);
         add_carry_prefix<NW>(s_pmAp, sm.pf[2], q);
         add_carry_prefix<NW>(s_PM, sm.pll[0], q);
@@ -1099,15 +1143,18 @@ __device__ unsigned build_table(const DevParams& P, const ClusterDev& C, int w,
     if (!bad) {
 #pragma unroll
         for (int e = 0; e < E; ++e) {
-            if (last[e]) {
-                const int x = x0 + e * 32 + lane;
+            const int xe = x0 + e * 32 + lane;
+            const int nxe = (xe == n - 1) ? 0x7fffffff : rnext[e];
+            // an evaluation build forms only the candidate's row
+            if (last[e] && (!EVAL || (want && r[e] <= rc && rc < nxe))) {
+                const int x = xe;
                 const int np = n - (x + 1);
                 const long long A = tot_a - pre_a[e];
-                const int nxt = (x == n - 1) ? 0x7fffffff : rnext[e];
+                const int nxt = nxe;
                 const long long SM = SMx[e] == LL_NONE ? 0 : SMx[e];
                 const RowVals o = make_row(P, inv_s, M, sumP, r[e], nxt, np, A, pre_r[e], pre_ra[e],
                                            PMx[e], SM, pmA[e], pmAp[e], smS[e], smSp[e]);
-                store_row(C, rowbase + rowid[e], o, P.want_aux != 0);
+                if constexpr (!EVAL) store_row(C, rowbase + rowid[e], o, P.want_aux != 0);
                 if (cache && rowid[e] < R && rowid[e] < cache->rc)
                     cache->rho[rowid[e]] = (unsigned short)(nxt - 1);
                 if (want && r[e] <= rc && rc < nxt) {
@@ -1118,28 +1165,32 @@ __device__ unsigned build_table(const DevParams& P, const ClusterDev& C, int w,
             }
         }
     }
-    if (row0_lane) {
+    if (row0_lane && (!EVAL || (want && (bad || n == 0 || rc < r0)))) {
         RowVals o;
         if (!bad) {
             o = make_row(P, inv_s, M, sumP, 0, n > 0 ? r0 : 0x7fffffff, n, tot_a, 0, 0, LL_NONE,
                          SM0 == LL_NONE ? 0 : SM0, f_inf(), f_inf(), smS0, smSp0);
-            C.R[w] = R;
+            if constexpr (!EVAL) C.R[w] = R;
         } else {
             // An invalid request: no candidate fits this worker.
             o = make_row(P, inv_s, M, 0, 0, 0x7fffffff, 0, 0, 0, 0, LL_NONE, (long long)M + 1,
                          f_inf(), f_inf(), f_inf(), f_inf());
-            C.R[w] = 0;
-            atomicOr(C.err, 1u);
+            if constexpr (!EVAL) {
+                C.R[w] = 0;
+                atomicOr(C.err, 1u);
+            }
         }
-        store_row(C, rowbase, o, P.want_aux != 0);
+        if constexpr (!EVAL) store_row(C, rowbase, o, P.want_aux != 0);
         if (want && (bad || n == 0 || rc < r0)) {
             float m;
             cf = eval_pair_mode(P.approx, o.v0, o.v1, o.ext, wr, wa, *cand, m);
             mine = true;
         }
-        C.wrec[w] = wr;
-        if (P.approx) C.wapx[w] = wa;
-        C.key[w] = kq;
+        if constexpr (!EVAL) {
+            C.wrec[w] = wr;
+            if (P.approx) C.wapx[w] = wa;
+            C.key[w] = kq;
+        }
         if (cache) {
             if (!bad && n > 0 && R > 0) cache->rho[0] = (unsigned short)(r0 - 1);
             *cache->R = bad ? 0 : R;
@@ -1147,9 +1198,12 @@ __device__ unsigned build_table(const DevParams& P, const ClusterDev& C, int w,
             *cache->key = kq;
         }
     }
+    if constexpr (EVAL) {
+        if (row0_lane && key_out) *key_out = kq;
+    }
     if constexpr (NW > 1) {
         if (mine) sm.cflag = cf;  // exactly one lane of the group holds the row
-        group_sync<NW>();
+        group_sync<NW, BAR>();
         return want ? sm.cflag : 0u;
     } else {
         __syncwarp();
@@ -1164,24 +1218,31 @@ __device__ unsigned build_table(const DevParams& P, const ClusterDev& C, int w,
 // elements, not 1,024). smem holds a BuildSmem<EWMAX, NW>; the smaller
 // variants use a prefix of it. n is the worker's current count (uniform over
 // the NW warps).
-template <int EWMAX, int NW, bool INSERT = false>
+template <int EWMAX, int NW, bool INSERT = false, int BAR = 1, int W0 = 0, bool EVAL = false,
+          bool SKEY = true>
 __device__ __forceinline__ unsigned build_table_fit(const DevParams& P, const ClusterDev& C, int w,
                                                     int n, unsigned char* smem,
                                                     const SliceCache* cache = nullptr,
-                                                    const CandRec* cand = nullptr)
+                                                    const CandRec* cand = nullptr,
+                                                    unsigned long long* key_out = nullptr,
+                                                    int ins = 1)
 {
+    // an evaluation build is given its count (beyond the worker's own)
+    const int n_in = EVAL ? n : -1;
     if constexpr (EWMAX >= 4) {
         if (n > 64 * NW)  // more than the EW = 2 variant covers
-            return build_table<4, NW, INSERT>(P, C, w, *reinterpret_cast<BuildSmem<4, NW>*>(smem),
-                                              cache, cand);
+            return build_table<4, NW, INSERT, BAR, W0, EVAL, SKEY>(
+                P, C, w, *reinterpret_cast<BuildSmem<4, NW>*>(smem), cache, cand, n_in, key_out,
+                ins);
     }
     if constexpr (EWMAX >= 2) {
         if (n > 32 * NW)
-            return build_table<2, NW, INSERT>(P, C, w, *reinterpret_cast<BuildSmem<2, NW>*>(smem),
-                                              cache, cand);
+            return build_table<2, NW, INSERT, BAR, W0, EVAL, SKEY>(
+                P, C, w, *reinterpret_cast<BuildSmem<2, NW>*>(smem), cache, cand, n_in, key_out,
+                ins);
     }
-    return build_table<1, NW, INSERT>(P, C, w, *reinterpret_cast<BuildSmem<1, NW>*>(smem), cache,
-                                      cand);
+    return build_table<1, NW, INSERT, BAR, W0, EVAL, SKEY>(
+        P, C, w, *reinterpret_cast<BuildSmem<1, NW>*>(smem), cache, cand, n_in, key_out, ins);
 }
 
 }  // namespace aladdin

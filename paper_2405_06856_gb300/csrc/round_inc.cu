@@ -68,15 +68,37 @@ struct RIArgs {
     int nwin;                  // rank positions held in shared memory
 };
 
+// Look-ahead (tables of up to 128 slots, rebuilt by at most 4 warps): while
+// one group rebuilds the pending worker's table and evaluates candidate c on
+// it, RI_LA - 1 more groups build that worker's state with c (and c + 1)
+// appended as well (evaluation only, nothing committed) and evaluate c + 1
+// (and c + 2) on it, and the remaining warps scan and evaluate for every one
+// of those candidates. When c goes to the pending worker, c + 1 is decided in
+// the same step, and so on: a step places up to RI_LA candidates. Most
+// candidates of a best-fit round go to the worker that took the previous one.
+#ifndef ALADDIN_RI_LA
+#define ALADDIN_RI_LA 2
+#endif
+constexpr int RI_LA = ALADDIN_RI_LA;  // candidates a look-ahead step may place
+
+template <int E>
+constexpr bool ri_lookahead()
+{
+    return RISplit<E>::NW <= 4;
+}
+
 template <int E>
 struct RISmem {
     BuildSmem<RISplit<E>::EW, RISplit<E>::NW> build;
-    unsigned long long bk[2][RI_WARPS];
-    int bw[2][RI_WARPS];
-    int bf[2][RI_WARPS];
-    CandRec cand[2];           // candidate records (parity of the step)
-    int craw[2][4];            // prompt, predicted, real output length
-    double cwd[2];             // wait (ms)
+    // the look-ahead groups' scratch
+    BuildSmem<1, ri_lookahead<E>() ? RISplit<E>::NW : 1> bla[ri_lookahead<E>() ? RI_LA - 1 : 1];
+    unsigned long long bk[2][RI_LA][RI_WARPS];  // [step parity][candidate c + j][warp]
+    int bw[2][RI_LA][RI_WARPS];
+    int bf[2][RI_LA][RI_WARPS];
+    CandRec cand[8];           // candidate records, by candidate index mod 8
+    int craw[8][4];            // prompt, predicted, real output length
+    double cwd[8];             // wait (ms)
+    unsigned long long la_key[RI_LA]; // the look-ahead states' capacity_norm keys
 };
 
 // Winner flags carried through the reductions: bit 29 the worker is full,
@@ -149,119 +171,193 @@ __global__ void __launch_bounds__(RI_THREADS, 1) k_round_inc(RIArgs A)
     for (int k = tid; k < nwords; k += RI_THREADS) modbits[k] = 0u;
     // the prefetching thread (in the last warp, never part of a rebuild)
     const bool pf = tid == RI_THREADS - 1;
-    auto fetch = [&](int c, int par) {
-        const int32_t a = io.in[c], r = io.pred[c];
-        const float wf = io.wait ? io.wait[c] : 0.0f;
-        sm.cand[par] = make_cand(P, a, r, wf, c);
-        sm.craw[par][0] = a;
-        sm.craw[par][1] = r;
-        sm.craw[par][2] = r;
-        sm.cwd[par] = (double)wf;
+    auto fetch = [&](int k) {
+        const int b = k & 7;
+        const int32_t a = io.in[k], r = io.pred[k];
+        const float wf = io.wait ? io.wait[k] : 0.0f;
+        sm.cand[b] = make_cand(P, a, r, wf, k);
+        sm.craw[b][0] = a;
+        sm.craw[b][1] = r;
+        sm.craw[b][2] = r;
+        sm.cwd[b] = (double)wf;
     };
-    if (pf && n_cand > 0) fetch(0, 0);
-    __syncthreads();
+    int fetched = 0;  // candidates fetched (meaningful in the prefetching thread)
+    if (pf)
+        while (fetched < n_cand && fetched < 2) fetch(fetched++);
 
+    constexpr bool LA = ri_lookahead<E>();
     int mcount = 0;           // slots in use (every thread tracks the same value)
     int last_pos = -1;        // rank position marked modified at the previous step
-    int pend_w = -1, pend_s = -1;  // the previous step's winner, not yet appended
-    bool pend_small = false;  // its new count fits the 4-warp rebuild
-    int32_t pa = 0, pr = 0, prl = 0;
-    double pwd = 0.0;
+    int pend_w = -1, pend_s = -1;  // the worker whose table is owed a rebuild
+    int pend_cnt = 0;         // requests appended to it since its table was built
+    bool pend_small = false;  // its count fits the 4-warp rebuild
     int stop_at = n_cand;     // first candidate left to the sliced round
+    int c_step = 0;           // the step's first candidate
 
-    auto append = [&](int w, int s) {  // the rebuild group commits the owed request
-        if (tid == 0) {
-            const int nw = mn[s] >= 0 ? mn[s] : C.n[w];
-            const long long slot = (long long)w * C.cap + nw;
-            C.in[slot] = pa;
-            C.gen[slot] = 0;
-            C.pred[slot] = pr;
-            C.real[slot] = prl;
-            C.tdec[slot] = 0.0;
-            C.pend[slot] = 1;
-            C.wait[slot] = pwd;
-            C.n[w] = nw + 1;
-            mn[s] = nw + 1;
+    // tid 0: candidate k's request into worker w's next slot (slot s)
+    auto append = [&](int w, int s, int k) {
+        const int b = k & 7;
+        const int nw = mn[s] >= 0 ? mn[s] : C.n[w];
+        const long long slot = (long long)w * C.cap + nw;
+        C.in[slot] = sm.craw[b][0];
+        C.gen[slot] = 0;
+        C.pred[slot] = sm.craw[b][1];
+        C.real[slot] = sm.craw[b][2];
+        C.tdec[slot] = 0.0;
+        C.pend[slot] = 1;
+        C.wait[slot] = sm.cwd[b];
+        C.n[w] = nw + 1;
+        mn[s] = nw + 1;
+    };
+    // the rebuild group commits the worker's table, inserting the `ins`
+    // requests appended since its last build into that build's sorted keys.
+    // With the look-ahead, the sorted keys are stored after the step's
+    // barrier (skey_store): the look-ahead group reads the previous ones.
+    auto rebuild = [&](int w, int s, bool small, int ins, const CandRec* cand) -> unsigned {
+        SliceCache sc{rho + (long long)s * rs, rc, &mR[s], &mwrec[s], &mkey[s]};
+        unsigned char* bs = reinterpret_cast<unsigned char*>(&sm.build);
+        if constexpr (NW > 4) {
+            if (small) return build_table_fit<1, 4, true>(P, C, w, mn[s], bs, &sc, cand);
+        }
+        return build_table_fit<EW, NW, NW_INSERT, 1, 0, false, !LA>(P, C, w, mn[s], bs, &sc, cand,
+                                                                    nullptr, ins);
+    };
+    auto skey_store = [&](int w, int s) {  // the rebuild group, after its build
+        if constexpr (LA && NW > 1) {
+            const int n = mn[s];
+            for (int x = tid; x < n; x += 32 * NW) C.skey[(long long)w * C.cap + x] = sm.build.sorted[x];
         }
     };
-    auto rebuild = [&](int w, int s, bool small, const CandRec* cand) -> unsigned {
-        SliceCache sc{rho + (long long)s * rs, rc, &mR[s], &mwrec[s], &mkey[s]};
-        append(w, s);
-        if constexpr (NW > 4) {
-            if (small) {
-                group_sync<4>();
-                return build_table_fit<1, 4, true>(P, C, w, mn[s],
-                                                   reinterpret_cast<unsigned char*>(&sm.build),
-                                                   &sc, cand);
+    // candidate cq (index k): the modified workers other than the pending
+    // one, against their current tables, and the first unmodified feasible
+    // position of every word of its round-start flag row
+    auto scan_eval = [&](const CandRec& cq, int k, int first, int stride, unsigned long long& bk,
+                         int& bw, int& bf) {
+        if (!cq.valid) return;
+        for (int i = first; i < mcount; i += stride) {
+            if (i == pend_s) continue;
+            const int w = mw[i];
+            const long long rb = (long long)w * C.rows;
+            const int p = r2_find(rho + (long long)i * rs, mR[i], rc, cq.ri, C.tab, rb);
+            const long long row = rb + p;
+            const float4* t = C.tab + row * ROW_F4;
+            float m;
+            const unsigned f =
+                eval_pair_mode(P.approx != 0, t[0], t[1], C.tab2[row], mwrec[i],
+                               P.approx ? C.wapx[w] : make_float2(0.0f, 0.0f), cq, m);
+            if (f == 15u) better_f(bk, bw, bf, mkey[i], w, ri_flags(i, mn[i], cap));
+        }
+        const uint8_t* frow = A.F + (size_t)k * A.ldf;
+        for (int kw = first; kw < nwords; kw += stride) {
+            unsigned bits = feasible_bits(frow, kw) & ~modbits[kw];
+            if (kw == (last_pos >> 5) && last_pos >= 0) bits &= ~(1u << (last_pos & 31));
+            const int left = W - 32 * kw;
+            if (left < 32) bits &= (1u << left) - 1u;
+            if (bits) {
+                const int pos = 32 * kw + __ffs(bits) - 1;
+                const RankEnt e = pos < nwin ? win[pos] : A.rank_ent[pos];
+                better_f(bk, bw, bf, e.key, e.w, ri_flags(pos, e.n, cap) | RI_UNMOD);
             }
         }
-        group_sync<NW>();
-        return build_table_fit<EW, NW, NW_INSERT>(P, C, w, mn[s],
-                                                  reinterpret_cast<unsigned char*>(&sm.build), &sc,
-                                                  cand);
+    };
+
+    // look-ahead group g (1 .. RI_LA - 1, warps g NW .. g NW + NW - 1): the
+    // pending worker with candidates c .. c + g - 1 appended as well (their
+    // slots written by the group's first thread), evaluated for c + g
+    auto la_eval = [&](int g, int nw, int ins, const CandRec* cq) -> unsigned {
+        if (tid == 32 * NW * g) {
+            for (int j = 0; j < g; ++j) {
+                const int b = (c_step + j) & 7;
+                const long long slot = (long long)pend_w * C.cap + nw + j;
+                C.in[slot] = sm.craw[b][0];
+                C.gen[slot] = 0;
+                C.pred[slot] = sm.craw[b][1];
+                C.real[slot] = sm.craw[b][2];
+                C.tdec[slot] = 0.0;
+                C.pend[slot] = 1;
+                C.wait[slot] = sm.cwd[b];
+            }
+        }
+        unsigned char* bs = reinterpret_cast<unsigned char*>(&sm.bla[g - 1]);
+        if (g == 1) {
+            group_sync<NW, 2>();
+            return build_table_fit<1, NW, NW_INSERT, 2, NW, true>(P, C, pend_w, nw + 1, bs, nullptr,
+                                                                  cq, &sm.la_key[1], ins);
+        }
+        group_sync<NW, 3>();
+        return build_table_fit<1, NW, NW_INSERT, 3, 2 * NW, true>(P, C, pend_w, nw + 2, bs, nullptr,
+                                                                  cq, &sm.la_key[2], ins);
     };
 
     int c = 0;
-    for (; c < n_cand; ++c) {
-        const int par = c & 1;
-        const CandRec cr = sm.cand[par];
-        const int32_t a = sm.craw[par][0], r = sm.craw[par][1], rl = sm.craw[par][2];
-        const double wd = sm.cwd[par];
-        unsigned long long bk = 0ull;
-        int bw = NONE, bf = 0;
+    for (int stp = 0; c < n_cand; ++stp) {
+        __syncthreads();  // the last step's appends, slots and fetched records are visible
+        c_step = c;
+        const int par = stp & 1;
+        const CandRec cr = sm.cand[c & 7];
         const bool rebuilding = pend_w >= 0;
+        // candidates looked at this step: c, and while valid and room is left
+        // on the pending worker, c + 1 .. c + RI_LA - 1
+        int la = 1;
+        if constexpr (LA) {
+            if (rebuilding && cr.valid) {
+                while (la < RI_LA && c + la < n_cand && sm.cand[(c + la) & 7].valid &&
+                       mn[pend_s] + la + 1 <= cap)
+                    ++la;
+            }
+        }
         const int nwr = !rebuilding ? 0 : (NW > 4 && pend_small ? 4 : NW);  // rebuild warps
+        const int scan0 = la > 1 ? la * NW : nwr;  // first scanning warp
+        unsigned long long bk[RI_LA];
+        int bw[RI_LA], bf[RI_LA];
+#pragma unroll
+        for (int j = 0; j < RI_LA; ++j) bk[j] = 0ull, bw[j] = NONE, bf[j] = 0;
         if (warp < nwr) {
-            const unsigned f = rebuild(pend_w, pend_s, nwr == 4 && NW > 4, cr.valid ? &cr : nullptr);
+            const unsigned f = rebuild(pend_w, pend_s, nwr == 4 && NW > 4, pend_cnt,
+                                       cr.valid ? &cr : nullptr);
             if (tid == 0 && cr.valid && f == 15u)
-                bk = mkey[pend_s], bw = pend_w, bf = ri_flags(pend_s, mn[pend_s], cap);
-        } else {
-            if (cr.valid) {
-                const int first = tid - 32 * nwr, stride = RI_THREADS - 32 * nwr;
-                // the modified workers, against their current tables
-                for (int i = first; i < mcount; i += stride) {
-                    if (i == pend_s) continue;
-                    const int w = mw[i];
-                    const long long rb = (long long)w * C.rows;
-                    const int p = r2_find(rho + (long long)i * rs, mR[i], rc, cr.ri, C.tab, rb);
-                    const long long row = rb + p;
-                    const float4* t = C.tab + row * ROW_F4;
-                    float m;
-                    const unsigned f =
-                        eval_pair_mode(P.approx != 0, t[0], t[1], C.tab2[row], mwrec[i],
-                                       P.approx ? C.wapx[w] : make_float2(0.0f, 0.0f), cr, m);
-                    if (f == 15u) better_f(bk, bw, bf, mkey[i], w, ri_flags(i, mn[i], cap));
-                }
-                // the first unmodified feasible position of every word of the
-                // candidate's round-start flag row
-                const uint8_t* frow = A.F + (size_t)c * A.ldf;
-                for (int k = first; k < nwords; k += stride) {
-                    unsigned bits = feasible_bits(frow, k) & ~modbits[k];
-                    if (k == (last_pos >> 5) && last_pos >= 0) bits &= ~(1u << (last_pos & 31));
-                    const int left = W - 32 * k;
-                    if (left < 32) bits &= (1u << left) - 1u;
-                    if (bits) {
-                        const int pos = 32 * k + __ffs(bits) - 1;
-                        const RankEnt e = pos < nwin ? win[pos] : A.rank_ent[pos];
-                        better_f(bk, bw, bf, e.key, e.w, ri_flags(pos, e.n, cap) | RI_UNMOD);
-                    }
+                bk[0] = mkey[pend_s], bw[0] = pend_w, bf[0] = ri_flags(pend_s, mn[pend_s], cap);
+        } else if (warp < scan0) {
+            if constexpr (LA) {
+                const int g = warp / NW;  // 1 .. la - 1
+                const int nw = mn[pend_s];
+                const CandRec cq = sm.cand[(c + g) & 7];
+                const unsigned f = la_eval(g, nw, pend_cnt + g, &cq);
+                if (tid == 32 * NW * g && f == 15u) {
+#pragma unroll
+                    for (int j = 1; j < RI_LA; ++j)
+                        if (j == g)
+                            bk[j] = sm.la_key[j], bw[j] = pend_w,
+                            bf[j] = ri_flags(pend_s, nw + j, cap);
                 }
             }
-            if (pf && c + 1 < n_cand) fetch(c + 1, par ^ 1);
+        } else {
+            const int first = tid - 32 * scan0, stride = RI_THREADS - 32 * scan0;
+#pragma unroll
+            for (int j = 0; j < RI_LA; ++j)
+                if (j < la) scan_eval(sm.cand[(c + j) & 7], c + j, first, stride, bk[j], bw[j], bf[j]);
+            if (pf)
+                while (fetched < n_cand && fetched < c + 2 * RI_LA) fetch(fetched++);
         }
-        reduce_f(bk, bw, bf);
+#pragma unroll
+        for (int j = 0; j < RI_LA; ++j)
+            if (j < la) reduce_f(bk[j], bw[j], bf[j]);
         if (lane == 0) {
-            sm.bk[par][warp] = bk;
-            sm.bw[par][warp] = bw;
-            sm.bf[par][warp] = bf;
+#pragma unroll
+            for (int j = 0; j < RI_LA; ++j) {
+                sm.bk[par][j][warp] = bk[j];
+                sm.bw[par][j][warp] = bw[j];
+                sm.bf[par][j][warp] = bf[j];
+            }
         }
         __syncthreads();
-        bk = lane < RI_WARPS ? sm.bk[par][lane] : 0ull;
-        bw = lane < RI_WARPS ? sm.bw[par][lane] : NONE;
-        bf = lane < RI_WARPS ? sm.bf[par][lane] : 0;
-        reduce_f(bk, bw, bf);  // every thread ends with the winner
-        const int winner = !cr.valid ? -2 : (bw == NONE ? -1 : bw);
-        if (winner >= 0 && (bf & RI_FULL)) {
+        if (warp < nwr) skey_store(pend_w, pend_s);
+        unsigned long long kk = lane < RI_WARPS ? sm.bk[par][0][lane] : 0ull;
+        int ww = lane < RI_WARPS ? sm.bw[par][0][lane] : NONE;
+        int ff = lane < RI_WARPS ? sm.bf[par][0][lane] : 0;
+        reduce_f(kk, ww, ff);  // every thread ends with the winner
+        const int winner = !cr.valid ? -2 : (ww == NONE ? -1 : ww);
+        if (winner >= 0 && (ff & RI_FULL)) {
             if (tid == 0) {
                 *io.status = -2;  // ALADDIN_ERR_CAPACITY
                 for (int k = c; k < n_cand; ++k) io.placement[k] = -1;
@@ -269,38 +365,61 @@ __global__ void __launch_bounds__(RI_THREADS, 1) k_round_inc(RIArgs A)
             pend_w = -1;
             break;
         }
+        // c + 1, c + 2 are decided now while their predecessors went to the
+        // pending worker: every other worker's state is the one their
+        // evaluations saw
+        int placed = 1;
+        if (la > 1 && winner == pend_w) {
+            for (int j = 1; j < la; ++j) {
+                unsigned long long k2 = lane < RI_WARPS ? sm.bk[par][j][lane] : 0ull;
+                int w2 = lane < RI_WARPS ? sm.bw[par][j][lane] : NONE;
+                int f2 = lane < RI_WARPS ? sm.bf[par][j][lane] : 0;
+                reduce_f(k2, w2, f2);
+                if (w2 != pend_w) break;
+                ++placed;
+            }
+        }
         int s = -1;
         last_pos = -1;
         if (winner >= 0) {
-            if (bf & RI_UNMOD) {
+            if (ff & RI_UNMOD) {
                 if (mcount == mmax) {  // no slot left: the sliced round takes over here
                     stop_at = c;
-                    pend_w = -1;  // the previous winner was appended at this step's start
+                    pend_w = -1;  // the pending worker's table was rebuilt at this step
                     break;
                 }
                 s = mcount++;
-                last_pos = bf & RI_IDX;
+                last_pos = ff & RI_IDX;
                 if (tid == 0) {
                     mw[s] = winner;
                     mn[s] = -1;  // the append reads the round-start count
                     modbits[last_pos >> 5] |= 1u << (last_pos & 31);
                 }
             } else {
-                s = bf & RI_IDX;
+                s = ff & RI_IDX;
+            }
+        }
+        if (tid == 0) {
+            io.placement[c] = winner;
+            if (winner >= 0) append(winner, s, c);
+            for (int j = 1; j < placed; ++j) {
+                io.placement[c + j] = winner;
+                append(winner, s, c + j);
             }
         }
         pend_w = winner >= 0 ? winner : -1;
         pend_s = s;
-        pend_small = winner >= 0 && (bf & RI_SMALL) != 0;  // the same in every thread
-        pa = a;
-        pr = r;
-        prl = rl;
-        pwd = wd;
-        if (tid == 0) io.placement[c] = winner;
+        pend_cnt = placed;
+        pend_small = winner >= 0 && (ff & RI_SMALL) != 0;  // the same in every thread
+        c += placed;
     }
+    __syncthreads();  // the last appends are visible to the rebuild group
     if (pend_w >= 0) {
         const int nwr = NW > 4 && pend_small ? 4 : NW;
-        if (warp < nwr) rebuild(pend_w, pend_s, nwr == 4 && NW > 4, nullptr);
+        if (warp < nwr) {
+            rebuild(pend_w, pend_s, nwr == 4 && NW > 4, pend_cnt, nullptr);
+            skey_store(pend_w, pend_s);
+        }
     }
     if (tid == 0) *A.c_stop = stop_at;
 }
