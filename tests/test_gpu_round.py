@@ -56,6 +56,25 @@ def test_round_tiny(A, orc, synth, seed, tdec):
                       "after-round")
 
 
+@pytest.mark.parametrize("b_cap,seed", [(32, 205), (64, 206)])
+def test_round_small_tables(A, orc, synth, b_cap, seed):
+    """Rounds on tables of 32 and 64 slots (one and two rebuild warps, each
+    with its look-ahead group): placements and the final state equal the
+    oracle's, with runs of candidates on the same worker."""
+    wl = synth.make_cluster("small", seed, 300, 6, 30000, 700, per_worker_random=True,
+                            b_cap=b_cap, params=dict(T_pre=400.0, T_dec=10.2))
+    with A.Cluster.from_workload(wl) as cl:
+        pl = cl.place_round(wl.cand_in, wl.cand_pred, wl.cand_wait)
+        assert cl.status() == A.OK
+        oc = orc.Cluster.from_workload(wl)
+        ref = oc.place_round(wl.cand_in, wl.cand_pred, wl.cand_wait)
+        assert np.array_equal(pl, ref), np.argwhere(pl != ref)[:5]
+        assert_same_state(cl, oc, "small-%d" % b_cap)
+    placed = pl[pl >= 0]
+    assert len(placed) > 0
+    assert (placed[1:] == placed[:-1]).mean() > 0.3  # runs on one worker
+
+
 def test_round_w256(A, orc, synth):
     wl = synth.config("w256", n_cand=512, b_cap=128)
     with A.Cluster.from_workload(wl) as cl:
