@@ -325,6 +325,12 @@ __global__ void __launch_bounds__(SCORE_WARPS * 32, PEND ? 3 : ALADDIN_SCORE_MIN
     unsigned rank[SLOTS];
     int nb = 0;  // smallest next breakpoint over this lane's workers
     bool have_rows = false;
+    // The KV and decode-time bounds of a pair depend on the worker's row and
+    // the candidate's predicted length only (not on its prompt or wait):
+    // computed once for a run of candidates of equal length on unchanged rows
+    // (the candidates are sorted by length), minus each candidate's a after.
+    float xkv[SLOTS], xdt[SLOTS];
+    int x_ri = -1;  // the length they hold (warp-uniform); -1: none
 
     for (int k = 0; k < nchunks; ++k) {
         const int buf = k & 1;
@@ -393,6 +399,7 @@ __global__ void __launch_bounds__(SCORE_WARPS * 32, PEND ? 3 : ALADDIN_SCORE_MIN
             // after is fetched now and needed only at the next crossing.
             auto step_rows = [&](int ri) {
                 if (__any_sync(FULL, ri >= nb)) {
+                    x_ri = -1;
 #pragma unroll
                     for (int s = 0; s < SLOTS; ++s) {
                         while (ri >= ss[s].rnext && p[s] < last_row) {
@@ -422,10 +429,21 @@ __global__ void __launch_bounds__(SCORE_WARPS * 32, PEND ? 3 : ALADDIN_SCORE_MIN
                 const float a = q0.x, r = q0.y, ir = q0.z, Ua = q0.w;
                 const float id1 = q1.x, nX = q1.y, id2 = q1.z, Zc = q1.w;
                 kmin = 0xffffffffu;
+                if constexpr (!APPROX) {
+                    const int ri = rec_ri(i);
+                    if (ri != x_ri) {  // warp-uniform
+#pragma unroll
+                        for (int s = 0; s < SLOTS; ++s) {
+                            xkv[s] = fminf(ss[s].kvB1, fmaf(r, ss[s].np1n, ss[s].kvE));
+                            xdt[s] = fminf(ss[s].pmA, fmaf(ss[s].Gt, id1, nX));
+                        }
+                        x_ri = ri;
+                    }
+                }
 #pragma unroll
                 for (int s = 0; s < SLOTS; ++s) {
                     const Slot<PEND>& t = ss[s];
-                    d[0][s] = fminf(t.kvB1, fmaf(r, t.np1n, t.kvE)) - a;
+                    d[0][s] = (APPROX ? fminf(t.kvB1, fmaf(r, t.np1n, t.kvE)) : xkv[s]) - a;
                     const float tt = fmaf(Zc, inv_s[s], nZO[s]);
                     if constexpr (APPROX) {
                         // (d) and (b) of the placement MIP; Ua holds a + gamma r
@@ -433,7 +451,7 @@ __global__ void __launch_bounds__(SCORE_WARPS * 32, PEND ? 3 : ALADDIN_SCORE_MIN
                         d[3][s] = bq[s % (APPROX ? SLOTS : 1)] - Ua;
                         d[1][s] = (PEND ? fminf(tt, ZW[s]) : tt) - a;
                     } else {
-                        d[2][s] = fminf(t.pmA, fmaf(t.Gt, id1, nX)) - a;
+                        d[2][s] = xdt[s] - a;
                         const float ca = fmaf(t.b0n, ir, fmaf(t.nh, r, Ua - t.b1));
                         if (PEND) {
                             d[1][s] = fminf(tt, ZW[s]) - a;
