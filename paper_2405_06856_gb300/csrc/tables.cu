@@ -107,6 +107,10 @@ k_build_lo(DevParams P, ClusterDev C, int count, int32_t* __restrict__ ovf, int*
     build_table<E>(P, C, w, sm[warp]);
 }
 
+// A grid of at most OVF_BLOCKS CTAs whose warps take the listed workers in
+// turn: usually the list is empty, and a small grid costs less to launch.
+constexpr int OVF_BLOCKS = 256;
+
 template <int E>
 __global__ void __launch_bounds__(BUILD_WARPS * 32)
 k_build_ovf(DevParams P, ClusterDev C, const int32_t* __restrict__ ovf, const int* __restrict__ novf)
@@ -114,9 +118,9 @@ k_build_ovf(DevParams P, ClusterDev C, const int32_t* __restrict__ ovf, const in
     extern __shared__ __align__(16) unsigned char smraw[];
     BuildSmem<E>* sm = reinterpret_cast<BuildSmem<E>*>(smraw);
     const int warp = threadIdx.x >> 5;
-    const int idx = blockIdx.x * BUILD_WARPS + warp;
-    if (idx >= *novf) return;
-    build_table<E>(P, C, ovf[idx], sm[warp]);
+    const int n = *novf;
+    for (int idx = blockIdx.x * BUILD_WARPS + warp; idx < n; idx += gridDim.x * BUILD_WARPS)
+        build_table<E>(P, C, ovf[idx], sm[warp]);
 }
 
 // Tables of 1,024 slots: one CTA of NW cooperating warps per worker (a
@@ -173,7 +177,8 @@ static cudaError_t build_e(const DevParams& P, const ClusterDev& C, const int32_
             if ((e = allow_smem<k_build_ovf<E>>(shi)) != cudaSuccess) return e;
             if ((e = cudaMemsetAsync(C.novf, 0, sizeof(int), st)) != cudaSuccess) return e;
             k_build_lo<EL><<<blocks, BUILD_WARPS * 32, slo, st>>>(P, C, count, C.ovf, C.novf, S);
-            k_build_ovf<E><<<blocks, BUILD_WARPS * 32, shi, st>>>(P, C, C.ovf, C.novf);
+            k_build_ovf<E><<<blocks < OVF_BLOCKS ? blocks : OVF_BLOCKS, BUILD_WARPS * 32, shi, st>>>(
+                P, C, C.ovf, C.novf);
             return cudaGetLastError();
         }
         const size_t smem = sizeof(BuildSmem<E>) * BUILD_WARPS;

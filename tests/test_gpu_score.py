@@ -253,6 +253,30 @@ def test_rank_order_with_ties(A, orc, synth, W):
     check_argbest(order, g["flags"], g["argbest"], "ties-W%d" % W)
 
 
+def test_build_overflow_workers(A, orc, synth):
+    """Tables of 256 slots where many workers hold more than the 128 requests
+    the first-level warp build takes (the rest are listed and built by the
+    second level): created from host arrays and loaded from device arrays,
+    the pairs score like the oracle."""
+    import torch
+    wl = synth.make_cluster("ovf", 160, 300, 220, 400000, 256, per_worker_random=True,
+                            b_cap=256, params=dict(T_pre=900.0, T_dec=60.0))
+    counts = np.diff(wl.roff)
+    assert (counts > 128).sum() > 50 and (counts <= 128).sum() > 50
+    ref = orc.Cluster.from_workload(wl).score(wl.cand_in, wl.cand_pred, wl.cand_wait)
+    t = lambda x: torch.from_numpy(np.ascontiguousarray(x)).to(torch.device("cuda"))
+    with A.Cluster.from_workload(wl) as cl:
+        g = cl.score(wl.cand_in, wl.cand_pred, wl.cand_wait)
+        compare_pairs(ref, g["flags"], g["margin"], wl.cand_in, label="ovf-host")
+        cl.load(t(wl.roff), t(wl.req_in), t(wl.req_gen), t(wl.req_pred))
+        torch.cuda.synchronize()
+        g2 = cl.score(wl.cand_in, wl.cand_pred, wl.cand_wait)
+        assert cl.status() == A.OK
+        for k in ("flags", "margin", "argbest"):
+            assert g2[k].tobytes() == g[k].tobytes(), k
+    assert 0 < (g["flags"] == 15).mean() < 1
+
+
 def test_w4096_sampled(A, orc, synth):
     """The 4,096-worker workload at full size, scored by the call bench.py
     times (aladdin_cluster_load_score from device arrays): sampled pairs and
