@@ -16,11 +16,13 @@
 // counts, records and keys in shared memory, and a bit set marks their rank
 // positions. Per candidate the threads scan its flag row for the first
 // unmodified feasible position (32 positions per word) and evaluate the
-// modified workers; one block reduction picks the winner. The winner is
-// committed lazily: at the next step a group of warps appends the request
-// and rebuilds the winner's table, evaluating the next candidate against it
-// in the same pass, while the other warps do the scan and the evaluations.
-// No grid-wide exchange is needed. When the modified workers outgrow the
+// modified workers; one block reduction picks the winner. The winner's
+// request is appended at the decision; at the next step a group of warps
+// rebuilds its table (inserting the appended keys into its sorted order),
+// evaluating the next candidate against it in the same pass, while the other
+// warps do the scan and the evaluations (and, on tables of up to 128 slots,
+// a second group looks one candidate ahead: see below). No grid-wide exchange
+// is needed. When the modified workers outgrow the
 // shared-memory slots the kernel stops at that candidate and the sliced
 // round (k_round2) finishes the rest from the current state.
 #include <algorithm>
