@@ -264,8 +264,11 @@ __global__ void __launch_bounds__(RI_THREADS, 1) k_round_inc(RIArgs A)
     };
 
     // look-ahead group g (1 .. RI_LA - 1, warps g NW .. g NW + NW - 1): the
-    // pending worker with candidates c .. c + g - 1 appended as well (their
-    // slots written by the group's first thread), evaluated for c + g
+    // pending worker with candidates c .. c + g - 1 appended as well,
+    // evaluated for c + g. The group's first thread writes their requests
+    // into the slots past the worker's count: the append writes the same
+    // values there when a candidate is placed on the worker, and otherwise
+    // they lie past the count, where no build or evaluation reads.
     auto la_eval = [&](int g, int nw, int ins, const CandRec* cq) -> unsigned {
         if (tid == 32 * NW * g) {
             for (int j = 0; j < g; ++j) {
